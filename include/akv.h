@@ -1,0 +1,270 @@
+/*
+ * akv.h — C ABI of the AnchorKV decode-attention hot path on GB300 (sm_103a).
+ *
+ * AnchorKV (arXiv 2608.02901) stores, per layer and KV head, a few anchor
+ * vectors exactly and every other key/value as an anchor index plus one
+ * projection coefficient, with a 2-bit rotated residual for budgeted
+ * positions (Section 3.1, Eq. 1-3; Appendix A.1, Eq. 12-14).  This library
+ * provides the two calls of the paper's problem statement (Section 3, the
+ * opening of "Method"; Algorithm 1):
+ *
+ *   akv_encode      : dense bf16 K, V            -> packed compressed cache
+ *   akv_decode_attn : one query per head + cache -> attention output
+ *
+ * plus a host packer for caches whose logical arrays are given directly.
+ * Neither call ever writes a decompressed K or V row to device memory: the
+ * reconstruction of Eq. 3 is folded into the attention arithmetic.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - All pointers are plain addresses.  "device" pointers are CUDA global
+ *    memory of the current device; "host" pointers are CPU memory.  The
+ *    caller owns every buffer; the library allocates no device memory and
+ *    never synchronises the stream it is given (all work is stream-ordered).
+ *  - Every call validates its arguments on the host before any launch and
+ *    reports problems as an akv_status; it never throws and never aborts.
+ *    akv_last_error() returns a thread-local text for the last failure.
+ *  - bf16 / fp16 values are passed as their 16-bit IEEE encodings.
+ *  - head_dim is 128.  The query-group size G = n_q_heads / n_kv_heads must be
+ *    1, 2, 4 or 8; query head j reads KV head floor(j / G).
+ *
+ * The byte layout of the arena is normative and documented with the
+ * akv_arena_header and akv_unit_desc structures below.
+ */
+#ifndef AKV_H_
+#define AKV_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* akv_stream_t; /* a cudaStream_t; NULL = legacy default stream */
+
+typedef enum akv_status {
+  AKV_OK = 0,
+  AKV_ERR_INVALID = 1,     /* malformed argument: null pointer, bad size, short buffer, bad alignment */
+  AKV_ERR_UNSUPPORTED = 2, /* well-formed but outside what this build implements (head_dim, G, k*G) */
+  AKV_ERR_TOO_SMALL = 3,   /* a caller buffer (arena, workspace) is smaller than required */
+  AKV_ERR_CUDA = 4         /* a CUDA runtime call or kernel launch failed */
+} akv_status;
+
+#define AKV_HEAD_DIM 128
+#define AKV_FLAG_ROTATE 1u /* residuals carry the randomized Hadamard rotation (Appendix A.1, Eq. 12) */
+#define AKV_ARENA_MAGIC 0x31564B41u /* "AKV1" */
+#define AKV_ARENA_VERSION 1u
+#define AKV_MAX_ANCHORS 65535 /* anchor indices are uint16 (Table 1, b_a = 2) */
+
+/*
+ * Compression parameters of one layer (Section 3.2 "Anchor selection",
+ * Section 3.4 "Byte-Budgeted Residual Allocation").
+ *
+ *  k   = min(S, max(min(W, S), ceil(anchor_frac * S)))   anchors per (request, KV head),
+ *        the last min(W, S) positions always among them (Section 3.2);
+ *  N_K = min(floor(res_frac_k * S), S - k)               key residual slots;
+ *  N_V = min(floor(res_frac_v * S), S - k)               value residual slots.
+ *  Products are evaluated in double precision from the float fractions.
+ *
+ *  seed      picks the uniformly sampled anchors (the "random rest" of Algorithm 1);
+ *  rot_seed  picks the Hadamard sign pattern s, shared by every layer and head
+ *            (Appendix A.1, "Rotation");
+ *  flags     AKV_FLAG_ROTATE on: residuals are rotated before quantization.
+ */
+typedef struct akv_params {
+  int32_t batch;      /* B >= 1 */
+  int32_t n_kv_heads; /* H >= 1 */
+  int32_t n_q_heads;  /* H_q = G * H, G in {1,2,4,8} */
+  int32_t head_dim;   /* must be 128 */
+  float anchor_frac;  /* in [0, 1] */
+  float res_frac_k;   /* in [0, 1] */
+  float res_frac_v;   /* in [0, 1] */
+  int32_t window;     /* W >= 0 (32 in the paper, Section 4.1) */
+  uint64_t seed;
+  uint64_t rot_seed;
+  uint32_t flags;
+  uint32_t reserved; /* must be 0 */
+} akv_params;
+
+/*
+ * Arena header, at byte 0 of every arena (256 bytes).  The arena is
+ * self-describing: header, then n_units descriptors of 256 bytes each, then
+ * one 256-byte-aligned segment per (request b, KV head h), unit u = b*H + h.
+ */
+typedef struct akv_arena_header {
+  uint32_t magic;   /* AKV_ARENA_MAGIC */
+  uint32_t version; /* AKV_ARENA_VERSION */
+  uint64_t total_bytes;
+  akv_params params;
+  int32_t n_units; /* B * H */
+  int32_t max_len; /* max_b S_b */
+  uint64_t desc_offset; /* = 256 */
+  uint64_t sign_bits[2]; /* bit j of the 128-bit word: s_j = -1 when set (rotation signs) */
+  uint8_t pad[256 - 8 - 8 - sizeof(akv_params) - 8 - 8 - 16];
+} akv_arena_header;
+
+/*
+ * Per-unit descriptor (256 bytes).  Offsets are bytes from the arena base;
+ * every section starts on a 128-byte boundary.  Sections, in order:
+ *
+ *   anchor_k   [k][128] bf16   anchor keys, slots in ascending position   (Table 1: anchor keys)
+ *   anchor_v   [k][128] bf16   anchor values                              (Table 1: anchor values)
+ *   anchor_pos [k] int32       anchor positions (not read by decode)
+ *   stream_k   [S] uint32      per position: anchor slot a(i) in bits 0-15,
+ *                              fp16 gamma_i in bits 16-31 (Eq. 1, Eq. 2);
+ *                              an anchor stores (own slot, 1.0)
+ *   stream_v   [S] uint32      same for values
+ *   bitmap_k   [ceil(S/64)] uint64   bit i%64 of word i/64 set <=> i in R_K
+ *   prefix_k   [ceil(S/64)] uint32   exclusive popcount of bitmap_k words
+ *   bitmap_v, prefix_v                same for values
+ *   codes_k    [N_K][32] uint8  2-bit codes of the rotated residual, code j in
+ *                              byte j/4 bits 2(j%4)..2(j%4)+1; slots in position order
+ *   scales_k   [N_K] uint32     fp16 scale in bits 0-15, fp16 min in bits 16-31
+ *   codes_v, scales_v           same for values
+ *
+ * The slot of a residual position i is prefix[i/64] + popcount(bitmap[i/64] &
+ * ((1 << (i%64)) - 1)) (the O(1) position-to-slot lookup of Appendix A.1,
+ * "Layout").  Dequantized rotated residual: c^_j = min + code_j * scale; the
+ * residual is r~ = s o (H_128 c^) / 128 with H_128 the unnormalised Sylvester
+ * Hadamard matrix (or r~ = c^ when AKV_FLAG_ROTATE is off).
+ */
+typedef struct akv_unit_desc {
+  int32_t len;       /* S */
+  int32_t n_anchors; /* k */
+  int32_t n_res_k;   /* N_K */
+  int32_t n_res_v;   /* N_V */
+  int32_t n_words;   /* ceil(S / 64) */
+  int32_t b, h;
+  int32_t reserved0;
+  uint64_t off_anchor_k, off_anchor_v, off_anchor_pos;
+  uint64_t off_stream_k, off_stream_v;
+  uint64_t off_bitmap_k, off_prefix_k, off_bitmap_v, off_prefix_v;
+  uint64_t off_codes_k, off_scales_k, off_codes_v, off_scales_v;
+  uint64_t data_bytes; /* bytes of the sections (no padding): what one decode reads for this unit */
+  uint8_t pad[256 - 32 - 14 * 8];
+} akv_unit_desc;
+
+/* ---- Introspection ------------------------------------------------------ */
+
+/* Human-readable name of a status code.  Never NULL. */
+const char* akv_status_string(akv_status s);
+
+/* Thread-local detail text of the last failing call on this thread ("" if none). */
+const char* akv_last_error(void);
+
+/* ---- Layout ------------------------------------------------------------- */
+
+/*
+ * Per-unit shape implied by the parameters (the k, N_K, N_V formulas above).
+ *   ctx_lens_host : host [B] int32, 1 <= S_b <= 2^30
+ *   out_shapes    : host [B*H][4] int32, filled with (S, k, N_K, N_V) per unit
+ * Errors: AKV_ERR_INVALID for null pointers or out-of-range parameters,
+ * AKV_ERR_UNSUPPORTED for head_dim != 128, G not in {1,2,4,8}, k > 65535.
+ */
+akv_status akv_unit_shapes(const akv_params* p, const int32_t* ctx_lens_host, int32_t* out_shapes);
+
+/*
+ * Bytes of the arena for these parameters and context lengths, and bytes of
+ * the device workspace akv_encode needs for the same inputs.  Either output
+ * pointer may be NULL.  The arena size includes header, descriptors and
+ * 128/256-byte section padding.
+ */
+akv_status akv_cache_size(const akv_params* p, const int32_t* ctx_lens_host, size_t* arena_bytes,
+                          size_t* encode_ws_bytes);
+
+/*
+ * Writes the arena header and descriptor table (the first 256 * (1 + B*H)
+ * bytes) into a HOST buffer, so that a caller can read offsets without
+ * touching the device.  header_bytes must be >= 256 * (1 + B*H).
+ */
+akv_status akv_cache_header_host(const akv_params* p, const int32_t* ctx_lens_host, void* header_host,
+                                 size_t header_bytes);
+
+/* ---- Encode ------------------------------------------------------------- */
+
+/*
+ * Compresses dense keys and values into the arena (Algorithm 1, with anchor
+ * selection "last W + uniform rest" and residual slots ranked by residual
+ * norm, the paper's ablation variant (ii) of Section 4.3).
+ *
+ *   K, V  : device bf16 [B][H][s_max][128] (row-major; positions >= S_b unused)
+ *   arena : device, arena_bytes >= akv_cache_size(...).arena_bytes, 256-byte aligned
+ *   ws    : device scratch, ws_bytes >= encode_ws_bytes, 256-byte aligned;
+ *           contents on entry are ignored and on exit are unspecified
+ * Decisions (assignment, gamma, slot ranking, codes) are taken in IEEE fp64
+ * with a fixed operation order, so the packed bytes are reproducible bit for
+ * bit.  Errors: AKV_ERR_INVALID (null, misaligned, s_max < max S_b),
+ * AKV_ERR_TOO_SMALL (arena or ws short), AKV_ERR_CUDA (launch failure).
+ */
+akv_status akv_encode(const akv_params* p, const int32_t* ctx_lens_host, const void* K, const void* V,
+                      int32_t s_max, void* arena, size_t arena_bytes, void* ws, size_t ws_bytes,
+                      akv_stream_t stream);
+
+/* ---- Host packer -------------------------------------------------------- */
+
+/*
+ * Logical arrays of one unit, all HOST memory, sizes from akv_unit_shapes.
+ * res_pos_* hold the residual positions in strictly ascending order; every
+ * other array is indexed by position (stream arrays) or by slot.
+ */
+typedef struct akv_unit_host {
+  const uint16_t* anchor_k;   /* [k][128] bf16 */
+  const uint16_t* anchor_v;   /* [k][128] bf16 */
+  const int32_t* anchor_pos;  /* [k] ascending */
+  const uint16_t* idx_k;      /* [S] anchor slot per position */
+  const uint16_t* gamma_k;    /* [S] fp16 */
+  const uint16_t* idx_v;      /* [S] */
+  const uint16_t* gamma_v;    /* [S] */
+  const int32_t* res_pos_k;   /* [N_K] */
+  const uint8_t* codes_k;     /* [N_K][32] */
+  const uint16_t* scale_k;    /* [N_K] fp16 */
+  const uint16_t* min_k;      /* [N_K] fp16 */
+  const int32_t* res_pos_v;   /* [N_V] */
+  const uint8_t* codes_v;     /* [N_V][32] */
+  const uint16_t* scale_v;    /* [N_V] fp16 */
+  const uint16_t* min_v;      /* [N_V] fp16 */
+} akv_unit_host;
+
+/*
+ * Builds a complete arena image in HOST memory from per-unit logical arrays
+ * (units[B*H]); the caller copies it to the device.  Validates anchor slot
+ * indices (< k), ascending residual positions (< S) and buffer size.
+ */
+akv_status akv_cache_pack_host(const akv_params* p, const int32_t* ctx_lens_host, const akv_unit_host* units,
+                               void* arena_host, size_t arena_bytes);
+
+/* ---- Decode ------------------------------------------------------------- */
+
+/*
+ * Bytes of device workspace akv_decode_attn needs (0 for the cluster kernel
+ * of this build; callers should still query it).
+ */
+akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_lens_host, size_t* ws_bytes);
+
+/*
+ * Single-query decode attention read directly from the compressed cache
+ * (Eq. 3 inside Eq. 4): for each request b and query head j with KV head
+ * h = j / G,
+ *     l_i = sm_scale * q . x^K_i,   out = sum_i softmax(l)_i x^V_i,
+ * over all S_b positions (no mask), with x^ reconstructed per Eq. 3.
+ *
+ *   arena     : device, as written by akv_encode or copied from akv_cache_pack_host
+ *               for the same (p, ctx_lens_host)
+ *   q         : device bf16 [B][H_q][128]
+ *   out       : device bf16 [B][H_q][128], round-to-nearest-even of the fp32 result
+ *   out_f32   : device fp32 [B][H_q][128] or NULL
+ *   ws        : device workspace of >= akv_decode_workspace_size bytes (may be NULL if 0)
+ * Errors: AKV_ERR_INVALID (null/misaligned pointers, bad sizes),
+ * AKV_ERR_UNSUPPORTED (k * G beyond the shared-memory tables of this build),
+ * AKV_ERR_CUDA (launch failure).
+ */
+akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,
+                           size_t arena_bytes, const void* q, void* out, float* out_f32, float sm_scale,
+                           void* ws, size_t ws_bytes, akv_stream_t stream);
+
+#ifdef __cplusplus
+} /* extern "C" */
+#endif
+
+#endif /* AKV_H_ */

@@ -1,0 +1,671 @@
+/*
+ * akv_oracle.c -- plain, slow, fp64 CPU oracle of AnchorKV (arXiv 2608.02901).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing in the product path links, loads or
+ * calls this file; only the tests, the smoke check and the CPU-baseline leg
+ * of the benchmark do.  It shares no code, header, table or constant
+ * generator with the CUDA library: every formula below is written from the
+ * paper (and from the readings recorded where the paper is silent).
+ *
+ * What it computes
+ *   encode  : Section 3.1 Eq. 1 (absolute-cosine nearest anchor), Eq. 2
+ *             (projection coefficient, residual), Section 3.2 (last W
+ *             positions are anchors, the rest sampled uniformly), Appendix
+ *             A.1 Eq. 12 (randomized Hadamard rotation) and a 4-level
+ *             2-bit quantizer with per-token fp16 scale and min; residual
+ *             slots ranked by residual norm (Section 4.3, variant (ii)).
+ *   attend  : Eq. 3 reconstruction of every key and value, then Eq. 4
+ *             softmax attention, all in fp64, one token at a time.
+ *   attend_factorized : the same attention regrouped by anchor (anchor
+ *             scores computed once, value weights summed per anchor, inverse
+ *             rotation applied once after accumulation -- Section 4.4 and
+ *             Appendix E.1 rely on this linearity); used only to pin that
+ *             regrouping against the definition.
+ *   unpack  : an independent reader of the packed arena layout.
+ *
+ * Compiled with -ffp-contract=off so that every product and sum is the
+ * separately rounded IEEE operation written here.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define OR_D 128
+
+/* ------------------------------------------------------------------------ */
+/* Scalar helpers                                                            */
+/* ------------------------------------------------------------------------ */
+
+/* SplitMix64 output function (Steele, Lea and Flood, OOPSLA 2014): the state
+ * advanced by the golden-ratio increment, then the 64-bit finaliser. */
+uint64_t or_splitmix64(uint64_t x) {
+  uint64_t z = x + 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+/* bf16 bits -> exact double. */
+double or_bf16_to_double(uint16_t b) {
+  uint32_t u = ((uint32_t)b) << 16;
+  float f;
+  memcpy(&f, &u, 4);
+  return (double)f;
+}
+
+/* fp16 bits -> exact double. */
+double or_fp16_to_double(uint16_t h) {
+  int sign = (h >> 15) & 1;
+  int e = (h >> 10) & 0x1F;
+  int m = h & 0x3FF;
+  double v;
+  if (e == 0) {
+    v = ldexp((double)m, -24);
+  } else if (e == 31) {
+    v = m ? NAN : INFINITY;
+  } else {
+    v = ldexp((double)(1024 + m), e - 25);
+  }
+  return sign ? -v : v;
+}
+
+/* double -> fp16 bits, round to nearest even, saturating at +-65504.
+ * Direct from the double value (no float intermediate). */
+uint16_t or_fp16_from_double(double x) {
+  if (isnan(x)) return 0x7E00;
+  uint16_t sign = signbit(x) ? 0x8000 : 0;
+  double a = fabs(x);
+  if (a >= 65504.0) return (uint16_t)(sign | 0x7BFF);
+  if (a < ldexp(1.0, -14)) {
+    /* subnormal range: integer multiples of 2^-24 */
+    double r = rint(a * 16777216.0);
+    return (uint16_t)(sign | (uint16_t)r);
+  }
+  int e;
+  double m = frexp(a, &e); /* a = m 2^e, m in [0.5, 1) */
+  double frac = (2.0 * m - 1.0) * 1024.0;
+  double r = rint(frac);
+  uint32_t bits = ((uint32_t)(e + 14) << 10) + (uint32_t)r;
+  if (bits >= 0x7C00) bits = 0x7BFF;
+  return (uint16_t)(sign | bits);
+}
+
+/* Rotation signs s_j (Appendix A.1, Eq. 12): bit (j mod 64) of
+ * splitmix64(rot_seed + floor(j / 64)); a set bit means -1. */
+void or_signs(uint64_t rot_seed, double* s) {
+  for (int j = 0; j < OR_D; ++j) {
+    uint64_t w = or_splitmix64(rot_seed + (uint64_t)(j / 64));
+    s[j] = ((w >> (j % 64)) & 1ull) ? -1.0 : 1.0;
+  }
+}
+
+/* In-place unnormalised Walsh-Hadamard transform of length 128 in Sylvester
+ * (natural) order: stages h = 1, 2, ..., 64, pairs (a, b) -> (a + b, a - b). */
+void or_wht128(double* v) {
+  for (int h = 1; h < OR_D; h <<= 1) {
+    for (int i = 0; i < OR_D; i += 2 * h) {
+      for (int j = i; j < i + h; ++j) {
+        double a = v[j], b = v[j + h];
+        v[j] = a + b;
+        v[j + h] = a - b;
+      }
+    }
+  }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Shapes (Section 3.2 anchor budget incl. the window; residual budgets)     */
+/* ------------------------------------------------------------------------ */
+
+void or_unit_shape(int32_t S, float f_a, float f_rk, float f_rv, int32_t W, int32_t* k, int32_t* nk,
+                   int32_t* nv) {
+  int32_t w = W < S ? W : S;
+  double ka = ceil((double)f_a * (double)S);
+  int32_t kk = (int32_t)ka;
+  if (kk < w) kk = w;
+  if (kk > S) kk = S;
+  int32_t rk = (int32_t)floor((double)f_rk * (double)S);
+  int32_t rv = (int32_t)floor((double)f_rv * (double)S);
+  if (rk > S - kk) rk = S - kk;
+  if (rv > S - kk) rv = S - kk;
+  *k = kk;
+  *nk = rk;
+  *nv = rv;
+}
+
+/* ------------------------------------------------------------------------ */
+/* One unit's logical compressed cache                                       */
+/* ------------------------------------------------------------------------ */
+
+typedef struct or_unit {
+  int32_t S, k, nk, nv;
+  uint16_t* anchor_k;  /* [k][128] bf16 */
+  uint16_t* anchor_v;  /* [k][128] bf16 */
+  int32_t* anchor_pos; /* [k] */
+  uint16_t* idx_k;     /* [S] */
+  uint16_t* gam_k;     /* [S] fp16 */
+  uint16_t* idx_v;
+  uint16_t* gam_v;
+  int32_t* res_k; /* [nk] ascending positions */
+  uint8_t* codes_k; /* [nk][32] */
+  uint16_t* scale_k; /* [nk] fp16 */
+  uint16_t* min_k;   /* [nk] fp16 */
+  int32_t* res_v;
+  uint8_t* codes_v;
+  uint16_t* scale_v;
+  uint16_t* min_v;
+} or_unit;
+
+typedef struct {
+  uint64_t key;
+  int32_t pos;
+} or_keypos;
+
+static int cmp_key_asc(const void* a, const void* b) {
+  const or_keypos* x = (const or_keypos*)a;
+  const or_keypos* y = (const or_keypos*)b;
+  if (x->key < y->key) return -1;
+  if (x->key > y->key) return 1;
+  return (x->pos < y->pos) ? -1 : (x->pos > y->pos);
+}
+
+typedef struct {
+  double e;
+  int32_t pos;
+} or_errpos;
+
+/* larger residual energy first; equal energies: lower position first */
+static int cmp_err_desc(const void* a, const void* b) {
+  const or_errpos* x = (const or_errpos*)a;
+  const or_errpos* y = (const or_errpos*)b;
+  if (x->e > y->e) return -1;
+  if (x->e < y->e) return 1;
+  return (x->pos < y->pos) ? -1 : (x->pos > y->pos);
+}
+
+static int cmp_i32(const void* a, const void* b) {
+  int32_t x = *(const int32_t*)a, y = *(const int32_t*)b;
+  return (x > y) - (x < y);
+}
+
+/* Quantize one residual (Appendix A.1 rotation, then 4-level uniform codes
+ * on [min, max] with fp16 scale and min) and pack 4 codes per byte. */
+static void or_quantize(const double* r, const double* s, int rotate, uint8_t* codes, uint16_t* sc_out,
+                        uint16_t* mn_out) {
+  double v[OR_D];
+  for (int j = 0; j < OR_D; ++j) v[j] = rotate ? s[j] * r[j] : r[j];
+  if (rotate) or_wht128(v);
+  double vmin = v[0], vmax = v[0];
+  for (int j = 1; j < OR_D; ++j) {
+    if (v[j] < vmin) vmin = v[j];
+    if (v[j] > vmax) vmax = v[j];
+  }
+  uint16_t mn_h = or_fp16_from_double(vmin);
+  double mn = or_fp16_to_double(mn_h);
+  double t = (vmax - mn) / 3.0;
+  if (!(t > 0.0)) t = 0.0;
+  uint16_t sc_h = or_fp16_from_double(t);
+  double sc = or_fp16_to_double(sc_h);
+  memset(codes, 0, 32);
+  for (int j = 0; j < OR_D; ++j) {
+    int c = 0;
+    if (sc != 0.0) {
+      double q = rint((v[j] - mn) / sc);
+      if (q < 0.0) q = 0.0;
+      if (q > 3.0) q = 3.0;
+      c = (int)q;
+    }
+    codes[j / 4] |= (uint8_t)(c << (2 * (j % 4)));
+  }
+  *sc_out = sc_h;
+  *mn_out = mn_h;
+}
+
+/* Exported for the quantizer pins: rotate (if set) and quantize one residual r[128]. */
+void or_quantize_residual(const double* r, uint64_t rot_seed, int rotate, uint8_t* codes, uint16_t* sc,
+                          uint16_t* mn) {
+  double s[OR_D];
+  or_signs(rot_seed, s);
+  or_quantize(r, s, rotate, codes, sc, mn);
+}
+
+/* Encode one side (keys or values) of one unit given the anchor set. */
+static void or_encode_side(int32_t S, int32_t k, int32_t nres, const uint16_t* X /*[S][128]*/,
+                           const int32_t* anchor_pos, const int32_t* slot_of, const double* s, int rotate,
+                           uint16_t* idx, uint16_t* gam, int32_t* res, uint8_t* codes, uint16_t* scale,
+                           uint16_t* mins) {
+  /* squared anchor norms */
+  double* n = (double*)malloc(sizeof(double) * (size_t)(k > 0 ? k : 1));
+  for (int32_t a = 0; a < k; ++a) {
+    const uint16_t* xa = X + (size_t)anchor_pos[a] * OR_D;
+    double acc = 0.0;
+    for (int j = 0; j < OR_D; ++j) {
+      double t = or_bf16_to_double(xa[j]);
+      acc = acc + t * t;
+    }
+    n[a] = acc;
+  }
+  or_errpos* cand = (or_errpos*)malloc(sizeof(or_errpos) * (size_t)(S > 0 ? S : 1));
+  int32_t ncand = 0;
+  double xi[OR_D], r[OR_D];
+  for (int32_t i = 0; i < S; ++i) {
+    if (slot_of[i] >= 0) { /* anchors are exact: own slot, gamma = 1 */
+      idx[i] = (uint16_t)slot_of[i];
+      gam[i] = 0x3C00;
+      continue;
+    }
+    const uint16_t* x = X + (size_t)i * OR_D;
+    for (int j = 0; j < OR_D; ++j) xi[j] = or_bf16_to_double(x[j]);
+    /* Eq. 1: largest |<x_i, x_a>| / ||x_a|| (||x_i|| is common to all a). */
+    int32_t best = -1;
+    double bestc = -1.0, bestd = 0.0;
+    for (int32_t a = 0; a < k; ++a) {
+      if (n[a] == 0.0) continue;
+      const uint16_t* xa = X + (size_t)anchor_pos[a] * OR_D;
+      double d = 0.0;
+      for (int j = 0; j < OR_D; ++j) d = d + xi[j] * or_bf16_to_double(xa[j]);
+      double c = fabs(d) / sqrt(n[a]);
+      if (c > bestc) {
+        bestc = c;
+        best = a;
+        bestd = d;
+      }
+    }
+    uint16_t g_h = 0;
+    if (best >= 0) g_h = or_fp16_from_double(bestd / n[best]); /* Eq. 2 */
+    idx[i] = (uint16_t)(best >= 0 ? best : 0);
+    gam[i] = g_h;
+    /* Eq. 2 residual with the stored coefficient, and its energy */
+    double g = or_fp16_to_double(g_h);
+    const uint16_t* xa = X + (size_t)anchor_pos[best >= 0 ? best : 0] * OR_D;
+    double e = 0.0;
+    for (int j = 0; j < OR_D; ++j) {
+      double p = (best >= 0) ? g * or_bf16_to_double(xa[j]) : 0.0;
+      double rj = xi[j] - p;
+      e = e + rj * rj;
+    }
+    cand[ncand].e = e;
+    cand[ncand].pos = i;
+    ++ncand;
+  }
+  /* residual slots: the nres largest energies among non-anchors */
+  qsort(cand, (size_t)ncand, sizeof(or_errpos), cmp_err_desc);
+  for (int32_t t = 0; t < nres; ++t) res[t] = cand[t].pos;
+  qsort(res, (size_t)nres, sizeof(int32_t), cmp_i32);
+  for (int32_t t = 0; t < nres; ++t) {
+    int32_t i = res[t];
+    const uint16_t* x = X + (size_t)i * OR_D;
+    const uint16_t* xa = X + (size_t)anchor_pos[idx[i]] * OR_D;
+    double g = or_fp16_to_double(gam[i]);
+    int valid = 0;
+    for (int32_t a = 0; a < k; ++a)
+      if (n[a] != 0.0) valid = 1;
+    for (int j = 0; j < OR_D; ++j) {
+      double p = valid ? g * or_bf16_to_double(xa[j]) : 0.0;
+      r[j] = or_bf16_to_double(x[j]) - p;
+    }
+    or_quantize(r, s, rotate, codes + (size_t)t * 32, &scale[t], &mins[t]);
+  }
+  free(cand);
+  free(n);
+}
+
+/*
+ * Encode one (request b, KV head h) unit.  K and V are bf16 bits [S][128].
+ * The caller allocates every array of `u` with the sizes of or_unit_shape
+ * and sets u->S, k, nk, nv.
+ */
+int or_encode_unit(const uint16_t* K, const uint16_t* V, int32_t b, int32_t h, int32_t W, uint64_t seed,
+                   uint64_t rot_seed, int rotate, or_unit* u) {
+  int32_t S = u->S, k = u->k;
+  int32_t w = W < S ? W : S;
+  /* Section 3.2: the last w positions are anchors; the k - w others are a
+   * uniform sample of [0, S - w): the positions with the smallest hash. */
+  int32_t* slot_of = (int32_t*)malloc(sizeof(int32_t) * (size_t)S);
+  char* is_anchor = (char*)calloc((size_t)S, 1);
+  int32_t rest = k - w;
+  if (rest > 0) {
+    int32_t pool = S - w;
+    or_keypos* kp = (or_keypos*)malloc(sizeof(or_keypos) * (size_t)pool);
+    uint64_t base = seed ^ ((uint64_t)b << 40) ^ ((uint64_t)h << 32);
+    for (int32_t p = 0; p < pool; ++p) {
+      kp[p].key = or_splitmix64(base ^ (uint64_t)p);
+      kp[p].pos = p;
+    }
+    qsort(kp, (size_t)pool, sizeof(or_keypos), cmp_key_asc);
+    for (int32_t t = 0; t < rest; ++t) is_anchor[kp[t].pos] = 1;
+    free(kp);
+  }
+  for (int32_t p = S - w; p < S; ++p) is_anchor[p] = 1;
+  int32_t t = 0;
+  for (int32_t p = 0; p < S; ++p) {
+    if (is_anchor[p]) {
+      u->anchor_pos[t] = p;
+      slot_of[p] = t;
+      ++t;
+    } else {
+      slot_of[p] = -1;
+    }
+  }
+  if (t != k) {
+    free(slot_of);
+    free(is_anchor);
+    return -1;
+  }
+  for (int32_t a = 0; a < k; ++a) {
+    memcpy(u->anchor_k + (size_t)a * OR_D, K + (size_t)u->anchor_pos[a] * OR_D, OR_D * 2);
+    memcpy(u->anchor_v + (size_t)a * OR_D, V + (size_t)u->anchor_pos[a] * OR_D, OR_D * 2);
+  }
+  double s[OR_D];
+  or_signs(rot_seed, s);
+  or_encode_side(S, k, u->nk, K, u->anchor_pos, slot_of, s, rotate, u->idx_k, u->gam_k, u->res_k, u->codes_k,
+                 u->scale_k, u->min_k);
+  or_encode_side(S, k, u->nv, V, u->anchor_pos, slot_of, s, rotate, u->idx_v, u->gam_v, u->res_v, u->codes_v,
+                 u->scale_v, u->min_v);
+  free(slot_of);
+  free(is_anchor);
+  return 0;
+}
+
+/* Batched encode: K, V are [n_units][s_max][128]; units[u] describe b = u / H, h = u % H. */
+int or_encode_batch(const uint16_t* K, const uint16_t* V, int32_t s_max, int32_t n_units, int32_t H, int32_t W,
+                    uint64_t seed, uint64_t rot_seed, int rotate, or_unit* units) {
+  int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(| : bad)
+  for (int32_t u = 0; u < n_units; ++u) {
+    size_t off = (size_t)u * (size_t)s_max * OR_D;
+    if (or_encode_unit(K + off, V + off, u / H, u % H, W, seed, rot_seed, rotate, &units[u]) != 0) bad |= 1;
+  }
+  return bad ? -1 : 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Reconstruction (Eq. 3) and attention (Eq. 4)                              */
+/* ------------------------------------------------------------------------ */
+
+/* r~ = U^T C^{-1}(q) of Eq. 14 with U = H diag(s) / sqrt(D): here the stored
+ * codes dequantize to c^ = min + code * scale in the sqrt(D)-scaled rotated
+ * domain, so r~ = s o (H c^) / D. */
+static void or_dequant_residual(const uint8_t* codes, uint16_t sc_h, uint16_t mn_h, const double* s, int rotate,
+                                double* out) {
+  double sc = or_fp16_to_double(sc_h), mn = or_fp16_to_double(mn_h);
+  for (int j = 0; j < OR_D; ++j) {
+    int c = (codes[j / 4] >> (2 * (j % 4))) & 3;
+    out[j] = mn + (double)c * sc;
+  }
+  if (rotate) {
+    or_wht128(out);
+    for (int j = 0; j < OR_D; ++j) out[j] = s[j] * out[j] / (double)OR_D;
+  }
+}
+
+/* x^_i of Eq. 3 for one side, for every position; out [S][128]. */
+void or_reconstruct_side(int32_t S, const uint16_t* anchors, const uint16_t* idx, const uint16_t* gam, int32_t nres,
+                         const int32_t* res, const uint8_t* codes, const uint16_t* scale, const uint16_t* mins,
+                         uint64_t rot_seed, int rotate, double* out) {
+  double s[OR_D], rt[OR_D];
+  or_signs(rot_seed, s);
+  for (int32_t i = 0; i < S; ++i) {
+    double g = or_fp16_to_double(gam[i]);
+    const uint16_t* xa = anchors + (size_t)idx[i] * OR_D;
+    for (int j = 0; j < OR_D; ++j) out[(size_t)i * OR_D + j] = g * or_bf16_to_double(xa[j]);
+  }
+  for (int32_t t = 0; t < nres; ++t) {
+    or_dequant_residual(codes + (size_t)t * 32, scale[t], mins[t], s, rotate, rt);
+    for (int j = 0; j < OR_D; ++j) out[(size_t)res[t] * OR_D + j] += rt[j];
+  }
+}
+
+/* Definitional attention for one unit: G query rows (bf16 bits [G][128]),
+ * out [G][128] fp64.  Each key and value is rebuilt per Eq. 3 and the
+ * softmax of Eq. 4 is taken over all S positions. */
+void or_attend_unit(const or_unit* u, const uint16_t* q, int32_t G, double sm_scale, uint64_t rot_seed, int rotate,
+                    double* out) {
+  int32_t S = u->S;
+  double s[OR_D];
+  or_signs(rot_seed, s);
+  int32_t* slot_k = (int32_t*)malloc(sizeof(int32_t) * (size_t)S);
+  int32_t* slot_v = (int32_t*)malloc(sizeof(int32_t) * (size_t)S);
+  for (int32_t i = 0; i < S; ++i) slot_k[i] = slot_v[i] = -1;
+  for (int32_t t = 0; t < u->nk; ++t) slot_k[u->res_k[t]] = t;
+  for (int32_t t = 0; t < u->nv; ++t) slot_v[u->res_v[t]] = t;
+  double* logit = (double*)malloc(sizeof(double) * (size_t)S * (size_t)G);
+  double x[OR_D], rt[OR_D], qd[8][OR_D];
+  for (int32_t g = 0; g < G; ++g)
+    for (int j = 0; j < OR_D; ++j) qd[g][j] = or_bf16_to_double(q[(size_t)g * OR_D + j]);
+  for (int32_t i = 0; i < S; ++i) {
+    double gk = or_fp16_to_double(u->gam_k[i]);
+    const uint16_t* xa = u->anchor_k + (size_t)u->idx_k[i] * OR_D;
+    for (int j = 0; j < OR_D; ++j) x[j] = gk * or_bf16_to_double(xa[j]);
+    if (slot_k[i] >= 0) {
+      int32_t t = slot_k[i];
+      or_dequant_residual(u->codes_k + (size_t)t * 32, u->scale_k[t], u->min_k[t], s, rotate, rt);
+      for (int j = 0; j < OR_D; ++j) x[j] += rt[j];
+    }
+    for (int32_t g = 0; g < G; ++g) {
+      double d = 0.0;
+      for (int j = 0; j < OR_D; ++j) d += qd[g][j] * x[j];
+      logit[(size_t)i * G + g] = sm_scale * d;
+    }
+  }
+  for (int32_t g = 0; g < G; ++g) {
+    double m = -INFINITY;
+    for (int32_t i = 0; i < S; ++i)
+      if (logit[(size_t)i * G + g] > m) m = logit[(size_t)i * G + g];
+    double den = 0.0;
+    for (int32_t i = 0; i < S; ++i) {
+      double e = exp(logit[(size_t)i * G + g] - m);
+      logit[(size_t)i * G + g] = e;
+      den += e;
+    }
+    for (int32_t i = 0; i < S; ++i) logit[(size_t)i * G + g] /= den;
+  }
+  for (int32_t g = 0; g < G; ++g)
+    for (int j = 0; j < OR_D; ++j) out[(size_t)g * OR_D + j] = 0.0;
+  for (int32_t i = 0; i < S; ++i) {
+    double gv = or_fp16_to_double(u->gam_v[i]);
+    const uint16_t* xa = u->anchor_v + (size_t)u->idx_v[i] * OR_D;
+    for (int j = 0; j < OR_D; ++j) x[j] = gv * or_bf16_to_double(xa[j]);
+    if (slot_v[i] >= 0) {
+      int32_t t = slot_v[i];
+      or_dequant_residual(u->codes_v + (size_t)t * 32, u->scale_v[t], u->min_v[t], s, rotate, rt);
+      for (int j = 0; j < OR_D; ++j) x[j] += rt[j];
+    }
+    for (int32_t g = 0; g < G; ++g) {
+      double a = logit[(size_t)i * G + g];
+      for (int j = 0; j < OR_D; ++j) out[(size_t)g * OR_D + j] += a * x[j];
+    }
+  }
+  free(logit);
+  free(slot_k);
+  free(slot_v);
+}
+
+/* Batched definitional attention: q bf16 [n_units][G][128] (unit u = b*H + h
+ * owns query heads h*G .. h*G+G-1 of request b), out fp64 same shape.
+ * Units with sel[u] == 0 are skipped (sel may be NULL). */
+void or_attend_batch(const or_unit* units, int32_t n_units, const uint16_t* q, int32_t G, double sm_scale,
+                     uint64_t rot_seed, int rotate, const uint8_t* sel, double* out) {
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int32_t u = 0; u < n_units; ++u) {
+    if (sel && !sel[u]) continue;
+    or_attend_unit(&units[u], q + (size_t)u * G * OR_D, G, sm_scale, rot_seed, rotate, out + (size_t)u * G * OR_D);
+  }
+}
+
+/* The same attention regrouped by anchor: anchor scores once per anchor,
+ * value weights summed per anchor before one product with the anchor values,
+ * and the inverse rotation applied once to the accumulated residual codes. */
+void or_attend_factorized(const or_unit* u, const uint16_t* q, int32_t G, double sm_scale, uint64_t rot_seed,
+                          int rotate, double* out) {
+  int32_t S = u->S, k = u->k;
+  double s[OR_D];
+  or_signs(rot_seed, s);
+  double qd[8][OR_D], qr[8][OR_D], qsum[8];
+  for (int32_t g = 0; g < G; ++g) {
+    for (int j = 0; j < OR_D; ++j) qd[g][j] = or_bf16_to_double(q[(size_t)g * OR_D + j]);
+    for (int j = 0; j < OR_D; ++j) qr[g][j] = rotate ? s[j] * qd[g][j] : qd[g][j];
+    if (rotate) {
+      or_wht128(qr[g]);
+      for (int j = 0; j < OR_D; ++j) qr[g][j] /= (double)OR_D;
+    }
+    qsum[g] = 0.0;
+    for (int j = 0; j < OR_D; ++j) qsum[g] += qr[g][j];
+  }
+  double* sa = (double*)malloc(sizeof(double) * (size_t)(k ? k : 1) * G);
+  for (int32_t a = 0; a < k; ++a)
+    for (int32_t g = 0; g < G; ++g) {
+      double d = 0.0;
+      for (int j = 0; j < OR_D; ++j) d += qd[g][j] * or_bf16_to_double(u->anchor_k[(size_t)a * OR_D + j]);
+      sa[(size_t)a * G + g] = d;
+    }
+  double* lg = (double*)malloc(sizeof(double) * (size_t)S * G);
+  for (int32_t i = 0; i < S; ++i)
+    for (int32_t g = 0; g < G; ++g)
+      lg[(size_t)i * G + g] = or_fp16_to_double(u->gam_k[i]) * sa[(size_t)u->idx_k[i] * G + g];
+  for (int32_t t = 0; t < u->nk; ++t) {
+    int32_t i = u->res_k[t];
+    double sc = or_fp16_to_double(u->scale_k[t]), mn = or_fp16_to_double(u->min_k[t]);
+    for (int32_t g = 0; g < G; ++g) {
+      double d = 0.0;
+      for (int j = 0; j < OR_D; ++j) d += qr[g][j] * (double)((u->codes_k[(size_t)t * 32 + j / 4] >> (2 * (j % 4))) & 3);
+      lg[(size_t)i * G + g] += mn * qsum[g] + sc * d;
+    }
+  }
+  for (int32_t g = 0; g < G; ++g) {
+    double m = -INFINITY, den = 0.0;
+    for (int32_t i = 0; i < S; ++i) {
+      lg[(size_t)i * G + g] *= sm_scale;
+      if (lg[(size_t)i * G + g] > m) m = lg[(size_t)i * G + g];
+    }
+    for (int32_t i = 0; i < S; ++i) {
+      lg[(size_t)i * G + g] = exp(lg[(size_t)i * G + g] - m);
+      den += lg[(size_t)i * G + g];
+    }
+    for (int32_t i = 0; i < S; ++i) lg[(size_t)i * G + g] /= den;
+  }
+  double* w = (double*)calloc((size_t)(k ? k : 1) * G, sizeof(double));
+  for (int32_t i = 0; i < S; ++i)
+    for (int32_t g = 0; g < G; ++g)
+      w[(size_t)u->idx_v[i] * G + g] += lg[(size_t)i * G + g] * or_fp16_to_double(u->gam_v[i]);
+  double acc[8][OR_D];
+  for (int32_t g = 0; g < G; ++g)
+    for (int j = 0; j < OR_D; ++j) acc[g][j] = 0.0;
+  for (int32_t t = 0; t < u->nv; ++t) {
+    int32_t i = u->res_v[t];
+    double sc = or_fp16_to_double(u->scale_v[t]), mn = or_fp16_to_double(u->min_v[t]);
+    for (int32_t g = 0; g < G; ++g) {
+      double p = lg[(size_t)i * G + g];
+      for (int j = 0; j < OR_D; ++j)
+        acc[g][j] += p * (mn + sc * (double)((u->codes_v[(size_t)t * 32 + j / 4] >> (2 * (j % 4))) & 3));
+    }
+  }
+  for (int32_t g = 0; g < G; ++g) {
+    if (rotate) {
+      or_wht128(acc[g]);
+      for (int j = 0; j < OR_D; ++j) acc[g][j] = s[j] * acc[g][j] / (double)OR_D;
+    }
+    for (int j = 0; j < OR_D; ++j) {
+      double o = acc[g][j];
+      for (int32_t a = 0; a < k; ++a) o += w[(size_t)a * G + g] * or_bf16_to_double(u->anchor_v[(size_t)a * OR_D + j]);
+      out[(size_t)g * OR_D + j] = o;
+    }
+  }
+  free(w);
+  free(lg);
+  free(sa);
+}
+
+/* ------------------------------------------------------------------------ */
+/* Independent reader of the packed arena                                    */
+/* ------------------------------------------------------------------------ */
+
+/* Header: magic u32 @0, version u32 @4, total_bytes u64 @8, params (56 B) @16,
+ * n_units i32 @72, max_len i32 @76, desc_offset u64 @80, sign bits 2 x u64 @88.
+ * Descriptor (256 B each at desc_offset + 256 u): len, k, n_res_k, n_res_v,
+ * n_words, b, h, reserved (i32 each), then u64 offsets: anchor_k, anchor_v,
+ * anchor_pos, stream_k, stream_v, bitmap_k, prefix_k, bitmap_v, prefix_v,
+ * codes_k, scales_k, codes_v, scales_v, then data_bytes. */
+static uint32_t rd32(const uint8_t* p) {
+  uint32_t v;
+  memcpy(&v, p, 4);
+  return v;
+}
+static uint64_t rd64(const uint8_t* p) {
+  uint64_t v;
+  memcpy(&v, p, 8);
+  return v;
+}
+
+/* Returns 0 and the shape of unit u, or -1 on a malformed arena. */
+int or_arena_shape(const uint8_t* arena, uint64_t bytes, int32_t u, int32_t* shape4) {
+  if (bytes < 256 || rd32(arena) != 0x31564B41u || rd32(arena + 4) != 1u) return -1;
+  int32_t n_units = (int32_t)rd32(arena + 72);
+  uint64_t doff = rd64(arena + 80);
+  if (u < 0 || u >= n_units || doff + 256ull * (uint64_t)(u + 1) > bytes) return -1;
+  const uint8_t* d = arena + doff + 256ull * (uint64_t)u;
+  for (int t = 0; t < 4; ++t) shape4[t] = (int32_t)rd32(d + 4 * t);
+  return 0;
+}
+
+/* Copies unit u's logical arrays out of the arena into the caller's buffers
+ * (shape first from or_arena_shape).  Returns 0, or -1 on any inconsistency
+ * (bitmap popcount vs slot counts, prefix table, anchor slot range). */
+int or_arena_unpack(const uint8_t* arena, uint64_t bytes, int32_t u, or_unit* out) {
+  int32_t sh[4];
+  if (or_arena_shape(arena, bytes, u, sh) != 0) return -1;
+  const uint8_t* d = arena + rd64(arena + 80) + 256ull * (uint64_t)u;
+  int32_t S = sh[0], k = sh[1], nk = sh[2], nv = sh[3];
+  int32_t nw = (int32_t)rd32(d + 16);
+  if (nw != (S + 63) / 64) return -1;
+  uint64_t off[13];
+  for (int t = 0; t < 13; ++t) off[t] = rd64(d + 32 + 8 * t);
+  uint64_t end[13] = {off[0] + (uint64_t)k * 256, off[1] + (uint64_t)k * 256, off[2] + 4ull * k,
+                      off[3] + 4ull * S,          off[4] + 4ull * S,          off[5] + 8ull * nw,
+                      off[6] + 4ull * nw,         off[7] + 8ull * nw,         off[8] + 4ull * nw,
+                      off[9] + 32ull * nk,        off[10] + 4ull * nk,        off[11] + 32ull * nv,
+                      off[12] + 4ull * nv};
+  for (int t = 0; t < 13; ++t)
+    if (end[t] > bytes || (off[t] % 16) != 0) return -1;
+  memcpy(out->anchor_k, arena + off[0], (size_t)k * 256);
+  memcpy(out->anchor_v, arena + off[1], (size_t)k * 256);
+  memcpy(out->anchor_pos, arena + off[2], (size_t)k * 4);
+  for (int side = 0; side < 2; ++side) {
+    const uint8_t* st = arena + off[3 + side];
+    uint16_t* idx = side ? out->idx_v : out->idx_k;
+    uint16_t* gam = side ? out->gam_v : out->gam_k;
+    for (int32_t i = 0; i < S; ++i) {
+      uint32_t e = rd32(st + 4ull * i);
+      idx[i] = (uint16_t)(e & 0xFFFFu);
+      gam[i] = (uint16_t)(e >> 16);
+      if (idx[i] >= k) return -1;
+    }
+    const uint8_t* bm = arena + off[5 + 2 * side];
+    const uint8_t* pf = arena + off[6 + 2 * side];
+    int32_t n = side ? nv : nk;
+    int32_t* res = side ? out->res_v : out->res_k;
+    int32_t cnt = 0;
+    for (int32_t w = 0; w < nw; ++w) {
+      if ((int32_t)rd32(pf + 4ull * w) != cnt) return -1;
+      uint64_t word = rd64(bm + 8ull * w);
+      for (int bit = 0; bit < 64; ++bit) {
+        if ((word >> bit) & 1ull) {
+          int32_t pos = w * 64 + bit;
+          if (pos >= S || cnt >= n) return -1;
+          res[cnt++] = pos;
+        }
+      }
+    }
+    if (cnt != n) return -1;
+    const uint8_t* cd = arena + off[9 + 2 * side];
+    const uint8_t* sc = arena + off[10 + 2 * side];
+    memcpy(side ? out->codes_v : out->codes_k, cd, (size_t)n * 32);
+    for (int32_t t = 0; t < n; ++t) {
+      uint32_t e = rd32(sc + 4ull * t);
+      (side ? out->scale_v : out->scale_k)[t] = (uint16_t)(e & 0xFFFFu);
+      (side ? out->min_v : out->min_k)[t] = (uint16_t)(e >> 16);
+    }
+  }
+  return 0;
+}
