@@ -1,0 +1,435 @@
+#!/usr/bin/env python
+"""Benchmark of AnchorKV decode attention on GB300.
+
+Workload (default "8b-32k"): Llama-3.1-8B layer shape, 32 query / 8 KV heads,
+head_dim 128, context 32768, batch 1, 2 % anchors and 10 % residual slots
+(about 20x smaller than the bf16 cache), encoded on the GPU from the clustered
+synthetic K/V recipe.  A step is one decode-attention call for one layer with
+a fresh query; the timed region cycles through 32 distinct layer caches
+(217 MB, larger than the 129 MB L2) and 64 fresh query sets, replayed from a
+CUDA graph.  The metric is compressed bytes read per second (GB/s) and
+microseconds per step.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl akv|reference] [--workload NAME]
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode-attn µs/step and HBM GB/s (% of ~8 TB/s) over 20× AnchorKV cache, 1 GB300"
+WORKLOADS = {
+    # name: (batch, n_kv_heads, n_q_heads, context, source)
+    "8b-32k": (1, 8, 32, 32768, "encoded"),
+    "8b-128k": (4, 8, 32, 131072, "seeded"),
+    "70b-128k": (8, 8, 64, 131072, "seeded"),
+}
+N_LAYERS = 32
+N_TOKENS = 64
+DEC_KERNEL_SRC = os.path.join(ROOT, "paper_2608_02901_gb300", "csrc", "akv_decode.cu")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=N_LAYERS * N_TOKENS * 100)
+    ap.add_argument("--warmup", type=int, default=N_LAYERS * N_TOKENS)
+    ap.add_argument("--impl", default="akv", choices=["akv", "reference"])
+    ap.add_argument("--workload", default="8b-32k", choices=sorted(WORKLOADS))
+    ap.add_argument("--layers", type=int, default=N_LAYERS)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def unit_bytes(S, k, nk, nv, G):
+    """Compressed bytes one decode step reads for one (request, KV head), plus its q and out rows."""
+    words = (S + 63) // 64
+    return 512 * k + 8 * S + 24 * words + 36 * (nk + nv) + 2 * (2 * G * 128)
+
+
+def dist_setup(args):
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend=backend)
+    if torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    return rank, world, local
+
+
+def dist_max(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def dist_barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        finally:
+            os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def kernel_traffic():
+    """DRAM bytes per decode launch from the committed ncu summary, if it matches the current kernel source."""
+    src_hash = hashlib.sha256(open(DEC_KERNEL_SRC, "rb").read()).hexdigest()[:16]
+    path = os.path.join(ROOT, "profiles", "akv_decode_8b32k_ncu.md")
+    if not os.path.exists(path):
+        return None
+    vals = {}
+    for line in open(path):
+        if ":" in line and line.startswith("- "):
+            key, val = line[2:].split(":", 1)
+            vals[key.strip()] = val.strip().strip("`")
+    if vals.get("kernel_source_sha256_16") != src_hash:
+        return None
+    try:
+        return int(vals["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+def build_layers(torch, akv, gen, p, lens, layers, source, dev):
+    """Device arenas of `layers` distinct layer caches and the bytes one decode reads."""
+    arena_bytes, ws_bytes = akv.akv_cache_size(p, lens)
+    shapes = akv.akv_unit_shapes(p, lens)
+    step_bytes = sum(unit_bytes(int(S), int(k), int(nk), int(nv), p.G) for S, k, nk, nv in shapes)
+    arenas = []
+    if source == "encoded":
+        ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+        S = lens[0]
+        for layer in range(layers):
+            K, V = gen.clustered_batch_torch(p.batch, p.n_kv_heads, S, seed=1000 + layer, device=dev)
+            arena = torch.empty(arena_bytes, dtype=torch.uint8, device=dev)
+            akv.akv_encode(p, lens, K, V, arena, ws)
+            arenas.append(arena)
+            del K, V
+        torch.cuda.synchronize()
+        del ws
+    else:
+        base = None
+        for layer in range(layers):
+            if layer < 2:
+                units = [akv.unit_host_from_logical(gen.seeded_cache(int(S), int(k), int(nk), int(nv), p.window,
+                                                                       2000 + layer, u))
+                         for u, (S, k, nk, nv) in enumerate(shapes)]
+                img = akv.akv_cache_pack_host(p, lens, units)
+                arena = torch.from_numpy(img).to(dev)
+                base = arena if layer == 0 else base
+            else:  # further layers: device copies of the first two (distinct memory, same statistics)
+                arena = arenas[layer % 2].clone()
+            arenas.append(arena)
+    return arenas, arena_bytes, step_bytes
+
+
+def run_akv(args, rank, world, local):
+    import torch
+
+    import gen
+    import paper_2608_02901_gb300 as akv
+
+    dev = torch.device("cuda", local)
+    B, H, Hq, S, source = WORKLOADS[args.workload]
+    lens = [S] * B
+    p = akv.Params(batch=B, n_kv_heads=H, n_q_heads=Hq, seed=11 + rank, rot_seed=0x5EED)
+    layers = args.layers
+    arenas, arena_bytes, step_bytes = build_layers(torch, akv, gen, p, lens, layers, source, dev)
+    n_tok = N_TOKENS
+    qs = gen.queries_torch(n_tok * layers * B * Hq, seed=77 + rank, device=dev).view(n_tok, layers, B, Hq, 128)
+    out = torch.empty((n_tok, layers, B, Hq, 128), dtype=torch.bfloat16, device=dev)
+    chunk = n_tok * layers
+
+    def step(i, stream=None):
+        t, layer = divmod(i % chunk, layers)
+        akv.akv_decode_attn(p, lens, arenas[layer], qs[t, layer], out[t, layer], None, 1.0, None, stream)
+
+    # warm-up (also sets kernel attributes before capture)
+    for i in range(min(args.warmup, chunk)):
+        step(i)
+    torch.cuda.synchronize()
+    stream = torch.cuda.Stream(device=dev)
+    graphs = {}
+
+    def graph_for(n):
+        if n not in graphs:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for i in range(n):
+                    step(i, torch.cuda.current_stream())
+            graphs[n] = g
+        return graphs[n]
+
+    full, rem = divmod(args.steps, chunk)
+    g_full = graph_for(chunk) if full else None
+    g_rem = graph_for(rem) if rem else None
+    # graph warm-up: W steps total, at least 3
+    w_left = max(3, args.warmup)
+    with torch.cuda.stream(stream):
+        while w_left > 0:
+            graph_for(chunk).replay()
+            w_left -= chunk
+    torch.cuda.synchronize()
+
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    dist_barrier(world)
+    torch.cuda.synchronize()
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    smi_index = vis.split(",")[local] if vis else str(local)
+    with ClockSampler(smi_index) as clk:
+        with torch.cuda.stream(stream):
+            ev0.record(stream)
+            for _ in range(full):
+                g_full.replay()
+            if g_rem is not None:
+                g_rem.replay()
+            ev1.record(stream)
+        ev1.synchronize()
+    torch.cuda.synchronize()
+    dist_barrier(world)
+    ms = ev0.elapsed_time(ev1)
+    ms = dist_max(ms, world)
+    clocks = clk.summary()
+    sec = ms / 1e3
+    value = world * step_bytes * args.steps / sec / 1e9
+    us_step = ms * 1e3 / args.steps
+
+    # end to end through the C ABI with host buffers: pinned q in, pinned out back, every step
+    e2e_steps = min(args.steps, 2 * chunk)
+    q_host = torch.empty((n_tok, layers, B, Hq, 128), dtype=torch.bfloat16, pin_memory=True)
+    q_host.copy_(qs.cpu())
+    o_host = torch.empty((B, Hq, 128), dtype=torch.bfloat16, pin_memory=True)
+    q_dev = torch.empty((B, Hq, 128), dtype=torch.bfloat16, device=dev)
+    o_dev = torch.empty((B, Hq, 128), dtype=torch.bfloat16, device=dev)
+    torch.cuda.synchronize()
+    dist_barrier(world)
+    with torch.cuda.stream(stream):
+        t0 = time.perf_counter()
+        for i in range(e2e_steps):
+            t, layer = divmod(i % chunk, layers)
+            q_dev.copy_(q_host[t, layer], non_blocking=True)
+            akv.akv_decode_attn(p, lens, arenas[layer], q_dev, o_dev, None, 1.0, None, stream)
+            o_host.copy_(o_dev, non_blocking=True)
+            stream.synchronize()
+        e2e_sec = time.perf_counter() - t0
+    e2e_sec = dist_max(e2e_sec, world)
+    h2d = B * Hq * 128 * 2
+    e2e = {"value": round(world * step_bytes * e2e_steps / e2e_sec / 1e9, 3), "unit": "GB/s",
+           "us_per_step": round(e2e_sec * 1e6 / e2e_steps, 3), "steps": e2e_steps,
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": h2d}
+
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except (OSError, ValueError):
+        pass
+    peak = float(peaks.get("hbm_gbs", 6800.0))
+    achieved = step_bytes / (sec / args.steps) / 1e9  # per launch: one decode kernel per step
+    roofline = {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": kernel_traffic(),
+                "peak_source": "measured" if "hbm_gbs" in peaks else "fallback",
+                "bytes_per_launch": step_bytes, "frac_of_8tbs": round(achieved / 8000.0, 4)}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(torch, akv, p, lens, arenas)
+
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": "GB/s", "us_per_step": round(us_step, 4),
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 6),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded clustered K/V, encoded on GPU)" if source == "encoded" else "synthetic (seeded cache)",
+        "config": {"workload": args.workload, "batch": B, "n_kv_heads": H, "n_q_heads": Hq, "context": S,
+                   "anchor_frac": p.anchor_frac, "res_frac": p.res_frac_k, "layers_cycled": layers,
+                   "fresh_queries": N_TOKENS, "arena_bytes_per_layer": arena_bytes,
+                   "l2": f"inputs larger than L2: {layers} distinct layer caches, {layers * arena_bytes / 1e6:.0f} MB cycled",
+                   "timing": "CUDA graph replay, CUDA events on the launching stream", "parallelism": f"dp{world}"},
+        "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": args.steps, "clocks": clocks,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def _oracle_units_from_arena(torch, arena):
+    import oracle
+    return oracle.unpack_arena(arena.cpu().numpy())
+
+
+def cpu_baseline(torch, akv, p, lens, arenas, budget_s=12.0):
+    """The fp64 oracle, as it stands, on the host cores: whole layers of the same workload."""
+    import gen
+    import oracle
+    units = _oracle_units_from_arena(torch, arenas[0])
+    G = p.G
+    q = gen.queries(p.batch * p.n_q_heads, seed=5)
+    shapes = akv.akv_unit_shapes(p, lens)
+    layer_bytes = sum(unit_bytes(int(S), int(k), int(nk), int(nv), G) for S, k, nk, nv in shapes)
+    done, t0 = 0, time.perf_counter()
+    while True:
+        oracle.attend(units, q.reshape(p.n_units, G, 128), G, 1.0, p.rot_seed)
+        done += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    sec = time.perf_counter() - t0
+    cores = min(os.cpu_count() or 1, p.n_units)
+    return {"value": round(layer_bytes * done / sec / 1e9, 5), "unit": "GB/s", "cores": cores, "kind": "oracle",
+            "sample": f"{done} full layer steps ({p.n_units} units, OpenMP over units) of the {lens[0]}-token layer",
+            "seconds": round(sec, 2), "us_per_step": round(sec * 1e6 / done, 1)}
+
+
+def run_reference(args, rank, world, local):
+    """The oracle (fp64 CPU) timed as the reference arm on a bounded sample of the same workload."""
+    if rank != 0:
+        return
+    import gen
+    import oracle
+    import paper_2608_02901_gb300 as akv_params_only  # Params/shape helpers are pure host code
+    B, H, Hq, S, source = WORKLOADS[args.workload]
+    G = Hq // H
+    p = akv_params_only.Params(batch=1, n_kv_heads=1, n_q_heads=G, seed=11, rot_seed=0x5EED)
+    # one (request, KV head) unit of the workload; each step attends one query group over a prefix of it
+    k, nk, nv = oracle.unit_shape(S, p.anchor_frac, p.res_frac_k, p.res_frac_v, p.window)
+    if source == "encoded":
+        K, V = gen.clustered_batch(1, 1, [S], seed=1000)
+        unit = oracle.encode(K, V, [S], 1, p.anchor_frac, p.res_frac_k, p.res_frac_v, p.window, p.seed,
+                             p.rot_seed)[0]
+    else:
+        d = gen.seeded_cache(S, k, nk, nv, p.window, 2000, 0)
+        unit = oracle.alloc_unit(S, k, nk, nv)
+        for f in ("anchor_k", "anchor_v", "anchor_pos", "idx_k", "gam_k", "idx_v", "gam_v", "res_k", "codes_k",
+                  "scale_k", "min_k", "res_v", "codes_v", "scale_v", "min_v"):
+            getattr(unit, f)[...] = d[f]
+    total_budget = 150.0
+    per_step = total_budget / max(1, args.steps + args.warmup)
+    # estimate the oracle's time per position on this host
+    q = gen.queries(G, seed=3)
+    t0 = time.perf_counter()
+    oracle.attend([unit], q.reshape(1, G, 128), G, 1.0, p.rot_seed)
+    per_pos = (time.perf_counter() - t0) / S
+    P = int(max(64, min(S, per_step / max(per_pos, 1e-12))))
+    sub = _prefix_unit(oracle, unit, P)
+    sub_bytes = unit_bytes(sub.S, sub.k, sub.nk, sub.nv, G)
+    for _ in range(args.warmup):
+        oracle.attend([sub], q.reshape(1, G, 128), G, 1.0, p.rot_seed)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.attend([sub], q.reshape(1, G, 128), G, 1.0, p.rot_seed)
+    sec = time.perf_counter() - t0
+    val = sub_bytes * args.steps / sec / 1e9
+    line = {"impl": "reference", "metric": METRIC, "value": round(val, 6), "unit": "GB/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(sec * 1e3 / args.steps, 6),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": args.workload, "context": S, "sample_positions": P},
+            "cpu_baseline": {"value": round(val, 6), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                             "sample": f"one query group over the first {P} of {S} positions of one unit per step"},
+            "e2e": {"value": round(val, 6), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def _prefix_unit(oracle, u, P):
+    """The first P positions of a unit's logical cache (all anchors kept, residual slots restricted)."""
+    if P >= u.S:
+        return u
+    mk, mv = u.res_k < P, u.res_v < P
+    sub = oracle.alloc_unit(P, u.k, int(mk.sum()), int(mv.sum()))
+    sub.anchor_k[...] = u.anchor_k
+    sub.anchor_v[...] = u.anchor_v
+    sub.anchor_pos[...] = u.anchor_pos
+    for f in ("idx_k", "gam_k", "idx_v", "gam_v"):
+        getattr(sub, f)[...] = getattr(u, f)[:P]
+    sub.res_k[...] = u.res_k[mk]
+    sub.codes_k[...] = u.codes_k[mk]
+    sub.scale_k[...] = u.scale_k[mk]
+    sub.min_k[...] = u.min_k[mk]
+    sub.res_v[...] = u.res_v[mv]
+    sub.codes_v[...] = u.codes_v[mv]
+    sub.scale_v[...] = u.scale_v[mv]
+    sub.min_v[...] = u.min_v[mv]
+    return sub
+
+
+def main():
+    args = parse()
+    rank, world, local = dist_setup(args)
+    try:
+        if args.impl == "reference":
+            run_reference(args, rank, world, local)
+        else:
+            run_akv(args, rank, world, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

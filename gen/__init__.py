@@ -134,3 +134,37 @@ def seeded_cache(S: int, k: int, nk: int, nv: int, W: int, seed: int, unit: int)
                 idx_k=idx_k, gam_k=gam_k, idx_v=idx_v, gam_v=gam_v,
                 res_k=res_k, codes_k=codes_k, scale_k=scale_k, min_k=min_k,
                 res_v=res_v, codes_v=codes_v, scale_v=scale_v, min_v=min_v)
+
+
+# ---- device-side variants of the same recipes (benchmark inputs only) --------
+
+def clustered_batch_torch(B: int, H: int, S: int, seed: int, device, n_centres: int = 64, n_outliers: int = 4,
+                          outlier_scale: float = 8.0):
+    """clustered_kv drawn with torch's generator on the device: bf16 [B][H][S][128] K and V."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(int(seed) & 0x7FFFFFFFFFFFFFFF)
+    K = torch.empty((B, H, S, D), dtype=torch.bfloat16, device=device)
+    V = torch.empty((B, H, S, D), dtype=torch.bfloat16, device=device)
+    ch = torch.as_tensor(outlier_channels(seed, n_outliers), device=device)
+    for b in range(B):
+        for h in range(H):
+            ck = torch.randn((n_centres, D), generator=g, device=device)
+            cv = torch.randn((n_centres, D), generator=g, device=device)
+            cid = torch.randint(0, n_centres, (S,), generator=g, device=device)
+            nk = torch.randn((S, 1), generator=g, device=device)
+            nv = torch.randn((S, 1), generator=g, device=device)
+            k = (1.0 + 0.2 * nk) * (ck[cid] + 0.3 * torch.randn((S, D), generator=g, device=device))
+            v = (1.0 + 0.2 * nv) * (cv[cid] + 0.3 * torch.randn((S, D), generator=g, device=device))
+            k[:, ch] *= outlier_scale
+            K[b, h] = k.to(torch.bfloat16)
+            V[b, h] = v.to(torch.bfloat16)
+    return K, V
+
+
+def queries_torch(n_rows: int, seed: int, device):
+    """queries drawn with torch's generator on the device: bf16 [n_rows][128]."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(int(seed) & 0x7FFFFFFFFFFFFFFF)
+    return (torch.randn((n_rows, D), generator=g, device=device) / np.sqrt(D)).to(torch.bfloat16)

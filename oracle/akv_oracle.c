@@ -235,13 +235,15 @@ static void or_encode_side(int32_t S, int32_t k, int32_t nres, const uint16_t* X
                            const int32_t* anchor_pos, const int32_t* slot_of, const double* s, int rotate,
                            uint16_t* idx, uint16_t* gam, int32_t* res, uint8_t* codes, uint16_t* scale,
                            uint16_t* mins) {
-  /* squared anchor norms */
+  /* anchor rows as doubles (exact) and their squared norms */
   double* n = (double*)malloc(sizeof(double) * (size_t)(k > 0 ? k : 1));
+  double* xad = (double*)malloc(sizeof(double) * (size_t)(k > 0 ? k : 1) * OR_D);
   for (int32_t a = 0; a < k; ++a) {
     const uint16_t* xa = X + (size_t)anchor_pos[a] * OR_D;
     double acc = 0.0;
     for (int j = 0; j < OR_D; ++j) {
       double t = or_bf16_to_double(xa[j]);
+      xad[(size_t)a * OR_D + j] = t;
       acc = acc + t * t;
     }
     n[a] = acc;
@@ -262,9 +264,9 @@ static void or_encode_side(int32_t S, int32_t k, int32_t nres, const uint16_t* X
     double bestc = -1.0, bestd = 0.0;
     for (int32_t a = 0; a < k; ++a) {
       if (n[a] == 0.0) continue;
-      const uint16_t* xa = X + (size_t)anchor_pos[a] * OR_D;
+      const double* xa = xad + (size_t)a * OR_D;
       double d = 0.0;
-      for (int j = 0; j < OR_D; ++j) d = d + xi[j] * or_bf16_to_double(xa[j]);
+      for (int j = 0; j < OR_D; ++j) d = d + xi[j] * xa[j];
       double c = fabs(d) / sqrt(n[a]);
       if (c > bestc) {
         bestc = c;
@@ -308,6 +310,7 @@ static void or_encode_side(int32_t S, int32_t k, int32_t nres, const uint16_t* X
     or_quantize(r, s, rotate, codes + (size_t)t * 32, &scale[t], &mins[t]);
   }
   free(cand);
+  free(xad);
   free(n);
 }
 

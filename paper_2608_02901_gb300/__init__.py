@@ -1,0 +1,239 @@
+"""Python binding of the AnchorKV decode-attention library (``libakv.so``).
+
+Argument marshalling only: every function below converts its arguments to
+plain pointers and sizes and calls the C entry point of the same name
+declared in ``include/akv.h``.  Device buffers are torch CUDA tensors; host
+buffers are numpy arrays.  If ``libakv.so`` has not been built, importing the
+library fails loudly -- there is no fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libakv.so")
+
+AKV_OK, AKV_ERR_INVALID, AKV_ERR_UNSUPPORTED, AKV_ERR_TOO_SMALL, AKV_ERR_CUDA = range(5)
+AKV_FLAG_ROTATE = 1
+HEAD_DIM = 128
+
+EXPORTED = (
+    "akv_status_string", "akv_last_error", "akv_unit_shapes", "akv_cache_size", "akv_cache_header_host",
+    "akv_encode", "akv_cache_pack_host", "akv_decode_workspace_size", "akv_decode_attn",
+)
+
+
+class AkvError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str):
+        super().__init__(f"{where}: status {status} ({_status_name(status)}): {detail}")
+        self.status = status
+
+
+class _Params(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32), ("n_q_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("anchor_frac", ctypes.c_float), ("res_frac_k", ctypes.c_float),
+                ("res_frac_v", ctypes.c_float), ("window", ctypes.c_int32), ("seed", ctypes.c_uint64),
+                ("rot_seed", ctypes.c_uint64), ("flags", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+
+
+class _UnitHost(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in (
+        "anchor_k", "anchor_v", "anchor_pos", "idx_k", "gamma_k", "idx_v", "gamma_v", "res_pos_k", "codes_k",
+        "scale_k", "min_k", "res_pos_v", "codes_v", "scale_v", "min_v")]
+
+
+@dataclass
+class Params:
+    """Compression parameters of one layer (see akv_params in include/akv.h)."""
+    batch: int
+    n_kv_heads: int
+    n_q_heads: int
+    anchor_frac: float = 0.02
+    res_frac_k: float = 0.10
+    res_frac_v: float = 0.10
+    window: int = 32
+    seed: int = 0
+    rot_seed: int = 0x5EED
+    rotate: bool = True
+    head_dim: int = HEAD_DIM
+
+    @property
+    def G(self) -> int:
+        return self.n_q_heads // self.n_kv_heads
+
+    @property
+    def n_units(self) -> int:
+        return self.batch * self.n_kv_heads
+
+    def c(self) -> _Params:
+        return _Params(self.batch, self.n_kv_heads, self.n_q_heads, self.head_dim, self.anchor_frac,
+                       self.res_frac_k, self.res_frac_v, self.window, self.seed & (2**64 - 1),
+                       self.rot_seed & (2**64 - 1), AKV_FLAG_ROTATE if self.rotate else 0, 0)
+
+
+_lib = None
+
+
+def lib():
+    """Load libakv.so; raises if it has not been built (no fallback path exists)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(f"libakv.so not built at {LIB_PATH}: run `python -c 'import __graft_entry__ as g; g.build()'`")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, i32p, st = ctypes.c_void_p, ctypes.POINTER(ctypes.c_int32), ctypes.c_int
+        P = ctypes.POINTER(_Params)
+        sz = ctypes.POINTER(ctypes.c_size_t)
+        L.akv_status_string.restype = ctypes.c_char_p
+        L.akv_status_string.argtypes = [st]
+        L.akv_last_error.restype = ctypes.c_char_p
+        L.akv_last_error.argtypes = []
+        L.akv_unit_shapes.restype = st
+        L.akv_unit_shapes.argtypes = [P, i32p, i32p]
+        L.akv_cache_size.restype = st
+        L.akv_cache_size.argtypes = [P, i32p, sz, sz]
+        L.akv_cache_header_host.restype = st
+        L.akv_cache_header_host.argtypes = [P, i32p, vp, ctypes.c_size_t]
+        L.akv_encode.restype = st
+        L.akv_encode.argtypes = [P, i32p, vp, vp, ctypes.c_int32, vp, ctypes.c_size_t, vp, ctypes.c_size_t, vp]
+        L.akv_cache_pack_host.restype = st
+        L.akv_cache_pack_host.argtypes = [P, i32p, ctypes.POINTER(_UnitHost), vp, ctypes.c_size_t]
+        L.akv_decode_workspace_size.restype = st
+        L.akv_decode_workspace_size.argtypes = [P, i32p, sz]
+        L.akv_decode_attn.restype = st
+        L.akv_decode_attn.argtypes = [P, i32p, vp, ctypes.c_size_t, vp, vp, vp, ctypes.c_float, vp,
+                                      ctypes.c_size_t, vp]
+        _lib = L
+    return _lib
+
+
+def _status_name(s: int) -> str:
+    try:
+        return lib().akv_status_string(s).decode()
+    except Exception:  # noqa: BLE001 - only used to format an error text
+        return str(s)
+
+
+def _check(status: int, where: str):
+    if status != AKV_OK:
+        raise AkvError(status, where, lib().akv_last_error().decode())
+
+
+def _lens(ctx_lens) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(ctx_lens, dtype=np.int32))
+
+
+def _i32p(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
+
+
+def _dev_ptr(t) -> int | None:
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    return t.data_ptr()
+
+
+def _stream_ptr(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return getattr(stream, "cuda_stream", stream)
+
+
+# ---- entry points (same names as the C ABI) --------------------------------------
+
+def akv_status_string(s: int) -> str:
+    return lib().akv_status_string(s).decode()
+
+
+def akv_last_error() -> str:
+    return lib().akv_last_error().decode()
+
+
+def akv_unit_shapes(p: Params, ctx_lens) -> np.ndarray:
+    lens = _lens(ctx_lens)
+    out = np.zeros((p.n_units, 4), np.int32)
+    _check(lib().akv_unit_shapes(ctypes.byref(p.c()), _i32p(lens), _i32p(out)), "akv_unit_shapes")
+    return out
+
+
+def akv_cache_size(p: Params, ctx_lens):
+    lens = _lens(ctx_lens)
+    a, w = ctypes.c_size_t(), ctypes.c_size_t()
+    _check(lib().akv_cache_size(ctypes.byref(p.c()), _i32p(lens), ctypes.byref(a), ctypes.byref(w)),
+           "akv_cache_size")
+    return a.value, w.value
+
+
+def akv_cache_header_host(p: Params, ctx_lens) -> np.ndarray:
+    lens = _lens(ctx_lens)
+    buf = np.zeros(256 * (1 + p.n_units), np.uint8)
+    _check(lib().akv_cache_header_host(ctypes.byref(p.c()), _i32p(lens), buf.ctypes.data, buf.size),
+           "akv_cache_header_host")
+    return buf
+
+
+def akv_encode(p: Params, ctx_lens, K, V, arena, ws, stream=None):
+    """K, V: CUDA bf16 [B][H][s_max][128]; arena, ws: CUDA uint8 buffers."""
+    lens = _lens(ctx_lens)
+    s_max = int(K.shape[2])
+    _check(lib().akv_encode(ctypes.byref(p.c()), _i32p(lens), _dev_ptr(K), _dev_ptr(V), s_max, _dev_ptr(arena),
+                            arena.numel() * arena.element_size(), _dev_ptr(ws), ws.numel() * ws.element_size(),
+                            _stream_ptr(stream)), "akv_encode")
+
+
+_UNIT_FIELDS = (("anchor_k", np.uint16), ("anchor_v", np.uint16), ("anchor_pos", np.int32), ("idx_k", np.uint16),
+                ("gamma_k", np.uint16), ("idx_v", np.uint16), ("gamma_v", np.uint16), ("res_pos_k", np.int32),
+                ("codes_k", np.uint8), ("scale_k", np.uint16), ("min_k", np.uint16), ("res_pos_v", np.int32),
+                ("codes_v", np.uint8), ("scale_v", np.uint16), ("min_v", np.uint16))
+
+
+def akv_cache_pack_host(p: Params, ctx_lens, units) -> np.ndarray:
+    """units: sequence of B*H mappings with the akv_unit_host array names; returns the arena image."""
+    lens = _lens(ctx_lens)
+    arena_bytes, _ = akv_cache_size(p, lens)
+    keep = []
+    arr = (_UnitHost * len(units))()
+    for i, u in enumerate(units):
+        for name, dt in _UNIT_FIELDS:
+            a = np.ascontiguousarray(u[name], dtype=dt)
+            keep.append(a)
+            setattr(arr[i], name, a.ctypes.data if a.size else None)
+    out = np.zeros(arena_bytes, np.uint8)
+    _check(lib().akv_cache_pack_host(ctypes.byref(p.c()), _i32p(lens), arr, out.ctypes.data, out.size),
+           "akv_cache_pack_host")
+    return out
+
+
+def akv_decode_workspace_size(p: Params, ctx_lens) -> int:
+    lens = _lens(ctx_lens)
+    w = ctypes.c_size_t()
+    _check(lib().akv_decode_workspace_size(ctypes.byref(p.c()), _i32p(lens), ctypes.byref(w)),
+           "akv_decode_workspace_size")
+    return w.value
+
+
+def akv_decode_attn(p: Params, ctx_lens, arena, q, out, out_f32=None, sm_scale: float = 1.0, ws=None, stream=None):
+    """q, out: CUDA bf16 [B][H_q][128]; out_f32 optional fp32 of the same shape."""
+    lens = _lens(ctx_lens)
+    ws_bytes = 0 if ws is None else ws.numel() * ws.element_size()
+    _check(lib().akv_decode_attn(ctypes.byref(p.c()), _i32p(lens), _dev_ptr(arena),
+                                 arena.numel() * arena.element_size(), _dev_ptr(q), _dev_ptr(out),
+                                 _dev_ptr(out_f32), float(sm_scale), _dev_ptr(ws), ws_bytes, _stream_ptr(stream)),
+           "akv_decode_attn")
+
+
+def unit_host_from_logical(u: dict) -> dict:
+    """Map a logical-array dict (gen.seeded_cache naming) to akv_unit_host names."""
+    return dict(anchor_k=u["anchor_k"], anchor_v=u["anchor_v"], anchor_pos=u["anchor_pos"], idx_k=u["idx_k"],
+                gamma_k=u["gam_k"], idx_v=u["idx_v"], gamma_v=u["gam_v"], res_pos_k=u["res_k"],
+                codes_k=u["codes_k"], scale_k=u["scale_k"], min_k=u["min_k"], res_pos_v=u["res_v"],
+                codes_v=u["codes_v"], scale_v=u["scale_v"], min_v=u["min_v"])

@@ -1,0 +1,316 @@
+// Host side of the C ABI: parameter validation, arena layout, the host packer
+// and the thin wrappers that hand validated work to the kernel launchers.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+
+#include "akv_internal.h"
+
+namespace akv {
+
+namespace {
+thread_local std::string g_last_error;
+
+uint64_t align_up(uint64_t x, uint64_t a) { return (x + a - 1) / a * a; }
+}  // namespace
+
+akv_status fail(akv_status s, const std::string& msg) {
+  g_last_error = msg;
+  return s;
+}
+
+uint64_t splitmix64(uint64_t x) {
+  // SplitMix64 finaliser applied to x advanced by the golden-ratio increment.
+  uint64_t z = x + 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+void rotation_signs(uint64_t rot_seed, uint64_t bits[2]) {
+  bits[0] = splitmix64(rot_seed);
+  bits[1] = splitmix64(rot_seed + 1);
+}
+
+akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out) {
+  if (!p || !ctx_lens || !out) return fail(AKV_ERR_INVALID, "null params, ctx_lens or output");
+  if (p->head_dim != kD) return fail(AKV_ERR_UNSUPPORTED, "head_dim must be 128");
+  if (p->batch < 1 || p->n_kv_heads < 1 || p->n_q_heads < 1)
+    return fail(AKV_ERR_INVALID, "batch, n_kv_heads and n_q_heads must be >= 1");
+  if (p->n_q_heads % p->n_kv_heads != 0) return fail(AKV_ERR_INVALID, "n_q_heads must be a multiple of n_kv_heads");
+  int G = p->n_q_heads / p->n_kv_heads;
+  if (G != 1 && G != 2 && G != 4 && G != 8) return fail(AKV_ERR_UNSUPPORTED, "query group size must be 1, 2, 4 or 8");
+  if (p->n_kv_heads > 256 || p->batch > (1 << 24)) return fail(AKV_ERR_UNSUPPORTED, "too many heads or requests");
+  auto frac_ok = [](float f) { return std::isfinite(f) && f >= 0.0f && f <= 1.0f; };
+  if (!frac_ok(p->anchor_frac) || !frac_ok(p->res_frac_k) || !frac_ok(p->res_frac_v))
+    return fail(AKV_ERR_INVALID, "fractions must be finite and in [0, 1]");
+  if (p->window < 0) return fail(AKV_ERR_INVALID, "window must be >= 0");
+  if (p->reserved != 0 || (p->flags & ~AKV_FLAG_ROTATE) != 0) return fail(AKV_ERR_INVALID, "unknown flags");
+
+  Layout& L = *out;
+  L = Layout();
+  L.G = G;
+  const int32_t n_units = p->batch * p->n_kv_heads;
+  L.shape.resize(n_units);
+  L.desc.resize(n_units);
+  uint64_t off = kHeaderBytes + kDescBytes * (uint64_t)n_units;
+  for (int32_t b = 0; b < p->batch; ++b) {
+    const int32_t S = ctx_lens[b];
+    if (S < 1 || S > (1 << 30)) return fail(AKV_ERR_INVALID, "context lengths must be in [1, 2^30]");
+    // Anchor budget including the window; residual budgets capped by the non-anchors.
+    const int32_t w = p->window < S ? p->window : S;
+    int64_t k = (int64_t)std::ceil((double)p->anchor_frac * (double)S);
+    if (k < w) k = w;
+    if (k > S) k = S;
+    int64_t nk = (int64_t)std::floor((double)p->res_frac_k * (double)S);
+    int64_t nv = (int64_t)std::floor((double)p->res_frac_v * (double)S);
+    if (nk > S - k) nk = S - k;
+    if (nv > S - k) nv = S - k;
+    if (k < 1) return fail(AKV_ERR_INVALID, "anchor budget is zero (window 0 and anchor_frac * S < 1)");
+    if (k > AKV_MAX_ANCHORS) return fail(AKV_ERR_UNSUPPORTED, "more than 65535 anchors in one unit");
+    for (int32_t h = 0; h < p->n_kv_heads; ++h) {
+      const int32_t u = b * p->n_kv_heads + h;
+      UnitShape& sh = L.shape[u];
+      sh.S = S;
+      sh.k = (int32_t)k;
+      sh.nk = (int32_t)nk;
+      sh.nv = (int32_t)nv;
+      const uint64_t nw = (uint64_t)(S + 63) / 64;
+      const uint64_t sizes[kNumSections] = {
+          (uint64_t)k * 256, (uint64_t)k * 256, (uint64_t)k * 4, (uint64_t)S * 4, (uint64_t)S * 4,
+          nw * 8,            nw * 4,            nw * 8,          nw * 4,          (uint64_t)nk * 32,
+          (uint64_t)nk * 4,  (uint64_t)nv * 32, (uint64_t)nv * 4};
+      akv_unit_desc& d = L.desc[u];
+      std::memset(&d, 0, sizeof(d));
+      d.len = S;
+      d.n_anchors = (int32_t)k;
+      d.n_res_k = (int32_t)nk;
+      d.n_res_v = (int32_t)nv;
+      d.n_words = (int32_t)nw;
+      d.b = b;
+      d.h = h;
+      off = align_up(off, kSegmentAlign);
+      uint64_t* offs = &d.off_anchor_k;
+      uint64_t data = 0;
+      for (int s = 0; s < kNumSections; ++s) {
+        off = align_up(off, kSectionAlign);
+        offs[s] = off;
+        off += sizes[s];
+        if (s != kAnchorPos) data += sizes[s];
+      }
+      d.data_bytes = data;
+      if (S > L.max_len) L.max_len = S;
+      if (k > L.max_k) L.max_k = (int32_t)k;
+      if (nk > L.max_nk) L.max_nk = (int32_t)nk;
+      if (nv > L.max_nv) L.max_nv = (int32_t)nv;
+    }
+  }
+  L.total_bytes = align_up(off, kSegmentAlign) + kTailPad;
+  akv_arena_header& H = L.header;
+  std::memset(&H, 0, sizeof(H));
+  H.magic = AKV_ARENA_MAGIC;
+  H.version = AKV_ARENA_VERSION;
+  H.total_bytes = L.total_bytes;
+  H.params = *p;
+  H.n_units = n_units;
+  H.max_len = L.max_len;
+  H.desc_offset = kHeaderBytes;
+  rotation_signs(p->rot_seed, H.sign_bits);
+  return AKV_OK;
+}
+
+void encode_ws_layout(const Layout& L, EncodeWs* ws) {
+  // Per unit: two u64 key arrays [S] (anchor hashes, then residual energies
+  // per side), slot map i32 [S], residual positions i32 [N_K + N_V],
+  // anchor norms (squared, and square roots) f64 [k] per side, 256 B control.
+  // A table of per-unit byte offsets (u64 each) leads the workspace.
+  ws->unit_off.resize(L.shape.size());
+  uint64_t off = align_up((uint64_t)L.shape.size() * 8, 256);
+  for (size_t u = 0; u < L.shape.size(); ++u) {
+    const UnitShape& s = L.shape[u];
+    ws->unit_off[u] = off;
+    uint64_t b = 0;
+    b += align_up((uint64_t)s.S * 8, 256) * 2;
+    b += align_up((uint64_t)s.S * 4, 256);
+    b += align_up((uint64_t)(s.nk + s.nv) * 4 + 16, 256);
+    b += align_up((uint64_t)s.k * 8, 256) * 4;
+    b += 256;
+    off += b;
+  }
+  ws->total = off + 256;
+}
+
+}  // namespace akv
+
+using namespace akv;
+
+extern "C" {
+
+const char* akv_status_string(akv_status s) {
+  switch (s) {
+    case AKV_OK: return "AKV_OK";
+    case AKV_ERR_INVALID: return "AKV_ERR_INVALID";
+    case AKV_ERR_UNSUPPORTED: return "AKV_ERR_UNSUPPORTED";
+    case AKV_ERR_TOO_SMALL: return "AKV_ERR_TOO_SMALL";
+    case AKV_ERR_CUDA: return "AKV_ERR_CUDA";
+  }
+  return "AKV_ERR_UNKNOWN";
+}
+
+const char* akv_last_error(void) { return g_last_error.c_str(); }
+
+akv_status akv_unit_shapes(const akv_params* p, const int32_t* ctx_lens_host, int32_t* out_shapes) {
+  g_last_error.clear();
+  if (!out_shapes) return fail(AKV_ERR_INVALID, "null out_shapes");
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L);
+  if (st != AKV_OK) return st;
+  for (size_t u = 0; u < L.shape.size(); ++u) {
+    out_shapes[4 * u + 0] = L.shape[u].S;
+    out_shapes[4 * u + 1] = L.shape[u].k;
+    out_shapes[4 * u + 2] = L.shape[u].nk;
+    out_shapes[4 * u + 3] = L.shape[u].nv;
+  }
+  return AKV_OK;
+}
+
+akv_status akv_cache_size(const akv_params* p, const int32_t* ctx_lens_host, size_t* arena_bytes,
+                          size_t* encode_ws_bytes) {
+  g_last_error.clear();
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L);
+  if (st != AKV_OK) return st;
+  if (arena_bytes) *arena_bytes = (size_t)L.total_bytes;
+  if (encode_ws_bytes) {
+    EncodeWs W;
+    encode_ws_layout(L, &W);
+    *encode_ws_bytes = (size_t)W.total;
+  }
+  return AKV_OK;
+}
+
+akv_status akv_cache_header_host(const akv_params* p, const int32_t* ctx_lens_host, void* header_host,
+                                 size_t header_bytes) {
+  g_last_error.clear();
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L);
+  if (st != AKV_OK) return st;
+  if (!header_host) return fail(AKV_ERR_INVALID, "null header buffer");
+  const size_t need = kHeaderBytes + kDescBytes * L.desc.size();
+  if (header_bytes < need) return fail(AKV_ERR_TOO_SMALL, "header buffer shorter than 256 * (1 + B*H)");
+  std::memcpy(header_host, &L.header, sizeof(L.header));
+  std::memcpy((char*)header_host + kHeaderBytes, L.desc.data(), kDescBytes * L.desc.size());
+  return AKV_OK;
+}
+
+akv_status akv_cache_pack_host(const akv_params* p, const int32_t* ctx_lens_host, const akv_unit_host* units,
+                               void* arena_host, size_t arena_bytes) {
+  g_last_error.clear();
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L);
+  if (st != AKV_OK) return st;
+  if (!units || !arena_host) return fail(AKV_ERR_INVALID, "null units or arena");
+  if (arena_bytes < L.total_bytes) return fail(AKV_ERR_TOO_SMALL, "arena shorter than akv_cache_size");
+  uint8_t* A = (uint8_t*)arena_host;
+  std::memset(A, 0, (size_t)L.total_bytes);
+  std::memcpy(A, &L.header, sizeof(L.header));
+  std::memcpy(A + kHeaderBytes, L.desc.data(), kDescBytes * L.desc.size());
+  for (size_t u = 0; u < L.shape.size(); ++u) {
+    const UnitShape& sh = L.shape[u];
+    const akv_unit_desc& d = L.desc[u];
+    const akv_unit_host& in = units[u];
+    const int32_t S = sh.S, k = sh.k;
+    if (!in.anchor_k || !in.anchor_v || !in.anchor_pos || !in.idx_k || !in.gamma_k || !in.idx_v || !in.gamma_v ||
+        (sh.nk && (!in.res_pos_k || !in.codes_k || !in.scale_k || !in.min_k)) ||
+        (sh.nv && (!in.res_pos_v || !in.codes_v || !in.scale_v || !in.min_v)))
+      return fail(AKV_ERR_INVALID, "null array in unit " + std::to_string(u));
+    std::memcpy(A + d.off_anchor_k, in.anchor_k, (size_t)k * 256);
+    std::memcpy(A + d.off_anchor_v, in.anchor_v, (size_t)k * 256);
+    std::memcpy(A + d.off_anchor_pos, in.anchor_pos, (size_t)k * 4);
+    for (int side = 0; side < 2; ++side) {
+      const uint16_t* idx = side ? in.idx_v : in.idx_k;
+      const uint16_t* gam = side ? in.gamma_v : in.gamma_k;
+      uint32_t* stream = (uint32_t*)(A + (side ? d.off_stream_v : d.off_stream_k));
+      for (int32_t i = 0; i < S; ++i) {
+        if (idx[i] >= k) return fail(AKV_ERR_INVALID, "anchor index out of range in unit " + std::to_string(u));
+        stream[i] = (uint32_t)idx[i] | ((uint32_t)gam[i] << 16);
+      }
+      const int32_t n = side ? sh.nv : sh.nk;
+      const int32_t* pos = side ? in.res_pos_v : in.res_pos_k;
+      uint64_t* bm = (uint64_t*)(A + (side ? d.off_bitmap_v : d.off_bitmap_k));
+      uint32_t* pf = (uint32_t*)(A + (side ? d.off_prefix_v : d.off_prefix_k));
+      for (int32_t t = 0; t < n; ++t) {
+        if (pos[t] < 0 || pos[t] >= S || (t > 0 && pos[t] <= pos[t - 1]))
+          return fail(AKV_ERR_INVALID, "residual positions must be ascending and < S in unit " + std::to_string(u));
+        bm[pos[t] >> 6] |= 1ull << (pos[t] & 63);
+      }
+      uint32_t run = 0;
+      for (int32_t w = 0; w < d.n_words; ++w) {
+        pf[w] = run;
+        run += (uint32_t)__builtin_popcountll(bm[w]);
+      }
+      const uint8_t* codes = side ? in.codes_v : in.codes_k;
+      const uint16_t* sc = side ? in.scale_v : in.scale_k;
+      const uint16_t* mn = side ? in.min_v : in.min_k;
+      if (n) std::memcpy(A + (side ? d.off_codes_v : d.off_codes_k), codes, (size_t)n * 32);
+      uint32_t* scales = (uint32_t*)(A + (side ? d.off_scales_v : d.off_scales_k));
+      for (int32_t t = 0; t < n; ++t) scales[t] = (uint32_t)sc[t] | ((uint32_t)mn[t] << 16);
+    }
+  }
+  return AKV_OK;
+}
+
+akv_status akv_encode(const akv_params* p, const int32_t* ctx_lens_host, const void* K, const void* V,
+                      int32_t s_max, void* arena, size_t arena_bytes, void* ws, size_t ws_bytes,
+                      akv_stream_t stream) {
+  g_last_error.clear();
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L);
+  if (st != AKV_OK) return st;
+  if (!K || !V || !arena || !ws) return fail(AKV_ERR_INVALID, "null K, V, arena or workspace");
+  if (((uintptr_t)arena % 256) || ((uintptr_t)ws % 256) || ((uintptr_t)K % 16) || ((uintptr_t)V % 16))
+    return fail(AKV_ERR_INVALID, "arena and workspace must be 256-byte aligned, K and V 16-byte aligned");
+  if (s_max < L.max_len) return fail(AKV_ERR_INVALID, "s_max is smaller than the longest context");
+  if (L.shape.size() > 65535) return fail(AKV_ERR_UNSUPPORTED, "encode handles at most 65535 (request, head) units");
+  if (arena_bytes < L.total_bytes) return fail(AKV_ERR_TOO_SMALL, "arena shorter than akv_cache_size");
+  EncodeWs W;
+  encode_ws_layout(L, &W);
+  if (ws_bytes < W.total) return fail(AKV_ERR_TOO_SMALL, "encode workspace shorter than akv_cache_size");
+  int err = launch_encode(L, W, *p, K, V, s_max, arena, ws, (void*)stream);
+  if (err) return fail(AKV_ERR_CUDA, std::string("encode launch failed: ") + cuda_error_string(err));
+  return AKV_OK;
+}
+
+akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_lens_host, size_t* ws_bytes) {
+  g_last_error.clear();
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L);
+  if (st != AKV_OK) return st;
+  if (!ws_bytes) return fail(AKV_ERR_INVALID, "null ws_bytes");
+  *ws_bytes = 0;
+  return AKV_OK;
+}
+
+akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,
+                           size_t arena_bytes, const void* q, void* out, float* out_f32, float sm_scale,
+                           void* ws, size_t ws_bytes, akv_stream_t stream) {
+  (void)ws;
+  (void)ws_bytes;
+  g_last_error.clear();
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L);
+  if (st != AKV_OK) return st;
+  if (!arena || !q || !out) return fail(AKV_ERR_INVALID, "null arena, q or out");
+  if (((uintptr_t)arena % 256) || ((uintptr_t)q % 16) || ((uintptr_t)out % 16) || ((uintptr_t)out_f32 % 16))
+    return fail(AKV_ERR_INVALID, "arena must be 256-byte aligned; q, out, out_f32 16-byte aligned");
+  if (arena_bytes < L.total_bytes) return fail(AKV_ERR_TOO_SMALL, "arena shorter than akv_cache_size");
+  if (!std::isfinite(sm_scale)) return fail(AKV_ERR_INVALID, "sm_scale must be finite");
+  std::string why;
+  int err = launch_decode(L, *p, arena, q, out, out_f32, sm_scale, (void*)stream, &why);
+  if (err == -1) return fail(AKV_ERR_UNSUPPORTED, why);
+  if (err) return fail(AKV_ERR_CUDA, std::string("decode launch failed: ") + cuda_error_string(err) + " " + why);
+  return AKV_OK;
+}
+
+}  // extern "C"

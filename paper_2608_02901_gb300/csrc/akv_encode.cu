@@ -1,0 +1,533 @@
+// Plain GPU encoder of the AnchorKV compressed cache (Algorithm 1 with the
+// anchor and slot rules of this build).  Correct, not tuned: every decision
+// (assignment, gamma, residual energy ranking, rotation, codes) is taken in
+// IEEE fp64 with a fixed operation order, so the packed bytes are
+// reproducible bit for bit.  Compiled with --fmad=false; where a fused
+// multiply-add is used explicitly its product is exact, so rounding once or
+// twice gives the same result.
+//
+// Kernels, in launch order, each over all units of the batch:
+//   enc_hash      anchor-selection hashes of the non-window positions
+//   enc_anchors   select the k - W smallest hashes, number anchor slots by position
+//   enc_rows      copy anchor rows into the arena, squared norms per side
+//   enc_assign    Eq. 1 nearest anchor, Eq. 2 gamma, residual energies
+//   enc_slots     top-N residual energies per side -> bitmap, prefix, slot list
+//   enc_quant     Eq. 12 rotation and 2-bit quantization of every slot
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include <cstring>
+#include <vector>
+
+#include "akv_internal.h"
+
+namespace akv {
+namespace {
+
+// Per-unit scratch pointers, derived from the workspace table the host writes.
+struct EncUnitWs {
+  uint64_t* key0;     // [S] anchor hashes, then key residual energies
+  uint64_t* key1;     // [S] value residual energies
+  int32_t* slot_of;   // [S] anchor slot or -1
+  int32_t* res_pos;   // [N_K + N_V] residual positions (keys, then values)
+  double* n2[2];      // [k] squared anchor norms per side
+  double* rn[2];      // [k] their square roots
+  uint32_t* ctrl;     // [0]: side 0 has a nonzero anchor, [1]: side 1
+};
+
+struct EncArgs {
+  const uint8_t* arena_c;
+  uint8_t* arena;
+  const uint8_t* ws_base;
+  const uint64_t* ws_off;  // [units] byte offsets of each unit's scratch
+  const __nv_bfloat16* K;
+  const __nv_bfloat16* V;
+  int32_t s_max;
+  int32_t n_kv_heads;
+  int32_t window;
+  int32_t rotate;
+  uint64_t seed;
+  unsigned long long sign_lo, sign_hi;
+};
+
+__device__ __forceinline__ const akv_unit_desc* unit_desc(const EncArgs& A, int u) {
+  return reinterpret_cast<const akv_unit_desc*>(A.arena_c + 256) + u;
+}
+
+__device__ __forceinline__ uint64_t au(uint64_t x, uint64_t a) { return (x + a - 1) / a * a; }
+
+__device__ EncUnitWs unit_ws(const EncArgs& A, int u, const akv_unit_desc* d) {
+  uint8_t* p = const_cast<uint8_t*>(A.ws_base) + A.ws_off[u];
+  EncUnitWs w;
+  const uint64_t S = (uint64_t)d->len, k = (uint64_t)d->n_anchors, n = (uint64_t)(d->n_res_k + d->n_res_v);
+  w.key0 = (uint64_t*)p;
+  p += au(S * 8, 256);
+  w.key1 = (uint64_t*)p;
+  p += au(S * 8, 256);
+  w.slot_of = (int32_t*)p;
+  p += au(S * 4, 256);
+  w.res_pos = (int32_t*)p;
+  p += au(n * 4 + 16, 256);
+  for (int s = 0; s < 2; ++s) {
+    w.n2[s] = (double*)p;
+    p += au(k * 8, 256);
+    w.rn[s] = (double*)p;
+    p += au(k * 8, 256);
+  }
+  w.ctrl = (uint32_t*)p;
+  return w;
+}
+
+__device__ __forceinline__ uint64_t splitmix64_dev(uint64_t x) {
+  uint64_t z = x + 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ double bf16_to_f64(__nv_bfloat16 v) { return (double)__bfloat162float(v); }
+__device__ __forceinline__ double fp16_bits_to_f64(uint32_t h) {
+  return (double)__half2float(__ushort_as_half((unsigned short)(h & 0xFFFFu)));
+}
+
+// fp64 -> fp16 bits, round to nearest even on the integer significand,
+// saturating at +-65504 (values are finite here; NaN maps to 0x7E00).
+__device__ uint32_t f64_to_fp16_bits(double x) {
+  const unsigned long long bits = (unsigned long long)__double_as_longlong(x);
+  const uint32_t sign = (uint32_t)(bits >> 63) << 15;
+  const int ex = (int)((bits >> 52) & 0x7FF);
+  const unsigned long long frac = bits & 0xFFFFFFFFFFFFFull;
+  if (ex == 0x7FF) return frac ? 0x7E00u : (sign | 0x7BFFu);
+  if (fabs(x) >= 65504.0) return sign | 0x7BFFu;
+  if (ex == 0) return sign;  // fp64 subnormals are far below half an fp16 ulp
+  const int e = ex - 1023;
+  if (e < -25) return sign;
+  const unsigned long long m = frac | (1ull << 52);  // 53-bit significand
+  const int sh = (e >= -14) ? 42 : 42 + (-14 - e);   // bits dropped
+  unsigned long long r = m >> sh;
+  const unsigned long long rem = m & ((1ull << sh) - 1ull);
+  const unsigned long long half = 1ull << (sh - 1);
+  if (rem > half || (rem == half && (r & 1ull))) ++r;
+  uint32_t out;
+  if (e >= -14) out = (uint32_t)(((e + 14) << 10) + (int)r);  // r carries the implicit 1024
+  else out = (uint32_t)r;                                      // subnormal (1024 -> smallest normal)
+  if (out >= 0x7C00u) out = 0x7BFFu;
+  return sign | out;
+}
+
+// r-th smallest (1-based) of n 64-bit keys (optionally of their complements),
+// MSB-first radix select by 8-bit digits; returns the key and the rank of the
+// answer among keys equal to it (*rank_in_eq, 1-based).  Block-wide.
+__device__ uint64_t block_select(const uint64_t* keys, int n, uint32_t r, bool complement, uint32_t* hist,
+                                 uint32_t* bcast, uint32_t* rank_in_eq) {
+  uint64_t prefix = 0, mask = 0;
+  for (int shift = 56; shift >= 0; shift -= 8) {
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+      uint64_t key = keys[i];
+      if (complement) key = ~key;
+      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      uint32_t cum = 0, sel = 255;
+      for (uint32_t bkt = 0; bkt < 256; ++bkt) {
+        if (cum + hist[bkt] >= r) {
+          sel = bkt;
+          break;
+        }
+        cum += hist[bkt];
+      }
+      bcast[0] = sel;
+      bcast[1] = r - cum;
+    }
+    __syncthreads();
+    prefix |= (uint64_t)bcast[0] << shift;
+    mask |= 0xFFull << shift;
+    r = bcast[1];
+    __syncthreads();
+  }
+  *rank_in_eq = r;
+  return complement ? ~prefix : prefix;
+}
+
+// Exclusive block scan of 0/1 flags for a block of 1024 threads; returns the
+// prefix and writes the block total to *total.
+__device__ int block_scan_flag(int flag, int* warp_tot, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const unsigned bal = __ballot_sync(0xffffffffu, flag);
+  const int pre_lane = __popc(bal & ((1u << lane) - 1u));
+  if (lane == 0) warp_tot[warp] = __popc(bal);
+  __syncthreads();
+  if (warp == 0) {
+    const int nw = blockDim.x >> 5;
+    int v = lane < nw ? warp_tot[lane] : 0;
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (lane < nw) warp_tot[lane] = incl - v;
+    if (lane == 31) warp_tot[32] = incl;
+  }
+  __syncthreads();
+  const int pre = warp_tot[warp] + pre_lane;
+  *total = warp_tot[32];
+  __syncthreads();
+  return pre;
+}
+
+// ---- kernels -----------------------------------------------------------------
+
+__global__ void enc_hash(const EncArgs A) {
+  const int u = blockIdx.y;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len;
+  const int p = blockIdx.x * blockDim.x + threadIdx.x;
+  if (p >= S) return;
+  EncUnitWs w = unit_ws(A, u, d);
+  const int win = min(A.window, S);
+  const uint64_t base = A.seed ^ ((uint64_t)d->b << 40) ^ ((uint64_t)d->h << 32);
+  w.key0[p] = (p < S - win) ? splitmix64_dev(base ^ (uint64_t)p) : ~0ull;
+}
+
+__global__ void __launch_bounds__(1024) enc_anchors(const EncArgs A) {
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t bc[2];
+  __shared__ int wt[33];
+  const int u = blockIdx.x;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len, k = d->n_anchors;
+  EncUnitWs w = unit_ws(A, u, d);
+  const int win = min(A.window, S);
+  const int pool = S - win, rest = k - win;
+  uint64_t thr = 0;
+  bool any = rest > 0;
+  if (any) {
+    uint32_t req;
+    thr = block_select(w.key0, pool, (uint32_t)rest, false, hist, bc, &req);
+  }
+  int32_t* apos = reinterpret_cast<int32_t*>(A.arena + d->off_anchor_pos);
+  int base = 0;
+  for (int c0 = 0; c0 < S; c0 += 1024) {
+    const int p = c0 + threadIdx.x;
+    int flag = 0;
+    if (p < S) flag = (p >= pool) || (any && w.key0[p] <= thr);
+    int tot;
+    const int pre = block_scan_flag(flag, wt, &tot);
+    if (p < S) {
+      w.slot_of[p] = flag ? base + pre : -1;
+      if (flag) apos[base + pre] = p;
+    }
+    base += tot;
+  }
+  if (threadIdx.x < 2) w.ctrl[threadIdx.x] = 0;
+}
+
+// One warp per anchor: copy rows, squared norms (sequential in j) per side.
+__global__ void enc_rows(const EncArgs A) {
+  const int u = blockIdx.y;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int k = d->n_anchors;
+  const int a = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (a >= k) return;
+  EncUnitWs w = unit_ws(A, u, d);
+  const int pos = reinterpret_cast<const int32_t*>(A.arena_c + d->off_anchor_pos)[a];
+  for (int side = 0; side < 2; ++side) {
+    const __nv_bfloat16* X = (side ? A.V : A.K) + ((size_t)u * A.s_max + pos) * 128;
+    __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(A.arena + (side ? d->off_anchor_v : d->off_anchor_k)) +
+                         (size_t)a * 128;
+    for (int j = lane; j < 128; j += 32) dst[j] = X[j];
+    if (lane == 0) {
+      double n = 0.0;
+      for (int j = 0; j < 128; ++j) {
+        const double t = bf16_to_f64(X[j]);
+        n = __dadd_rn(n, __dmul_rn(t, t));
+      }
+      w.n2[side][a] = n;
+      w.rn[side][a] = __dsqrt_rn(n);
+      if (n != 0.0) atomicOr(&w.ctrl[side], 1u);
+    }
+  }
+}
+
+constexpr int AS_POS = 64;  // positions per assignment block
+constexpr int AS_ANC = 32;  // anchors per smem chunk
+constexpr int AS_THREADS = 256;
+constexpr size_t AS_SMEM = (size_t)128 * AS_POS * 8 + (size_t)AS_ANC * 128 * 8 + 4 * AS_POS * (8 + 8 + 4) + 64;
+
+__global__ void __launch_bounds__(AS_THREADS) enc_assign(const EncArgs A) {
+  extern __shared__ __align__(16) unsigned char sm_raw[];
+  double* xs = reinterpret_cast<double*>(sm_raw);                 // [128][64] positions, transposed
+  double* xa = xs + 128 * AS_POS;                                 // [32][128] anchor chunk
+  double* bcv = xa + AS_ANC * 128;                                // [4][64]
+  double* bdv = bcv + 4 * AS_POS;                                 // [4][64]
+  int* bav = reinterpret_cast<int*>(bdv + 4 * AS_POS);            // [4][64]
+
+  const int u = blockIdx.y, side = blockIdx.z;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len, k = d->n_anchors;
+  const int p0 = blockIdx.x * AS_POS;
+  if (p0 >= S) return;
+  EncUnitWs w = unit_ws(A, u, d);
+  const __nv_bfloat16* X = (side ? A.V : A.K) + (size_t)u * A.s_max * 128;
+  const __nv_bfloat16* AT = reinterpret_cast<const __nv_bfloat16*>(A.arena_c + (side ? d->off_anchor_v : d->off_anchor_k));
+  const double* n2 = w.n2[side];
+  const double* rn = w.rn[side];
+  const int tid = threadIdx.x;
+
+  for (int e = tid; e < AS_POS * 128; e += AS_THREADS) {
+    const int pi = e >> 7, j = e & 127;
+    const int p = p0 + pi;
+    xs[j * AS_POS + pi] = (p < S) ? bf16_to_f64(X[(size_t)p * 128 + j]) : 0.0;
+  }
+  const int pi = tid % AS_POS, ag = tid / AS_POS;
+  double bestc = -1.0, bestd = 0.0;
+  int besta = -1;
+  for (int ac = 0; ac < k; ac += AS_ANC) {
+    __syncthreads();
+    for (int e = tid; e < AS_ANC * 128; e += AS_THREADS) {
+      const int t = e >> 7, j = e & 127;
+      xa[e] = (ac + t < k) ? bf16_to_f64(AT[(size_t)(ac + t) * 128 + j]) : 0.0;
+    }
+    __syncthreads();
+    double dd[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) dd[t] = 0.0;
+    const double* xr = xa + (ag * 8) * 128;
+    for (int j = 0; j < 128; ++j) {
+      const double x = xs[j * AS_POS + pi];
+#pragma unroll
+      for (int t = 0; t < 8; ++t) dd[t] = __fma_rn(x, xr[t * 128 + j], dd[t]);  // product of two bf16: exact
+    }
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+      const int a = ac + ag * 8 + t;
+      if (a < k && n2[a] != 0.0) {
+        const double c = __ddiv_rn(fabs(dd[t]), rn[a]);
+        if (c > bestc) {
+          bestc = c;
+          besta = a;
+          bestd = dd[t];
+        }
+      }
+    }
+  }
+  bcv[ag * AS_POS + pi] = bestc;
+  bdv[ag * AS_POS + pi] = bestd;
+  bav[ag * AS_POS + pi] = besta;
+  __syncthreads();
+  if (tid >= AS_POS) return;
+  const int p = p0 + tid;
+  if (p >= S) return;
+  double c = -1.0, dbest = 0.0;
+  int a = -1;
+  for (int g = 0; g < 4; ++g) {
+    const int ga = bav[g * AS_POS + tid];
+    if (ga < 0) continue;
+    const double gc = bcv[g * AS_POS + tid];
+    if (a < 0 || gc > c || (gc == c && ga < a)) {
+      c = gc;
+      a = ga;
+      dbest = bdv[g * AS_POS + tid];
+    }
+  }
+  uint32_t* stream = reinterpret_cast<uint32_t*>(A.arena + (side ? d->off_stream_v : d->off_stream_k));
+  uint64_t* key = side ? w.key1 : w.key0;
+  const int sl = w.slot_of[p];
+  if (sl >= 0) {
+    stream[p] = (uint32_t)sl | (0x3C00u << 16);
+    key[p] = 0;
+    return;
+  }
+  const uint32_t gh = (a >= 0) ? f64_to_fp16_bits(__ddiv_rn(dbest, n2[a])) : 0u;
+  stream[p] = (uint32_t)(a >= 0 ? a : 0) | (gh << 16);
+  const double g = fp16_bits_to_f64(gh);
+  const __nv_bfloat16* xar = AT + (size_t)(a >= 0 ? a : 0) * 128;
+  double e = 0.0;
+  for (int j = 0; j < 128; ++j) {
+    const double pj = (a >= 0) ? __dmul_rn(g, bf16_to_f64(xar[j])) : 0.0;
+    const double r = __dsub_rn(xs[j * AS_POS + tid], pj);
+    e = __dadd_rn(e, __dmul_rn(r, r));
+  }
+  key[p] = (uint64_t)__double_as_longlong(e) + 1ull;
+}
+
+// Per (unit, side): the N largest keys (ties: lower position), bitmap, prefix, slot list.
+__global__ void __launch_bounds__(1024) enc_slots(const EncArgs A) {
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t bc[2];
+  __shared__ int wt[33];
+  __shared__ uint32_t halves[32];
+  const int u = blockIdx.x, side = blockIdx.y;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len, N = side ? d->n_res_v : d->n_res_k;
+  EncUnitWs w = unit_ws(A, u, d);
+  const uint64_t* key = side ? w.key1 : w.key0;
+  uint64_t* bm = reinterpret_cast<uint64_t*>(A.arena + (side ? d->off_bitmap_v : d->off_bitmap_k));
+  uint32_t* pf = reinterpret_cast<uint32_t*>(A.arena + (side ? d->off_prefix_v : d->off_prefix_k));
+  int32_t* rp = w.res_pos + (side ? d->n_res_k : 0);
+  uint64_t thr = ~0ull;
+  uint32_t need = 0;
+  if (N > 0) thr = block_select(key, S, (uint32_t)N, true, hist, bc, &need);
+  int base = 0, eq_seen = 0;
+  for (int c0 = 0; c0 < S; c0 += 1024) {
+    const int p = c0 + threadIdx.x;
+    const uint64_t kv = (p < S) ? key[p] : 0ull;
+    const int is_eq = (N > 0 && p < S && kv == thr) ? 1 : 0;
+    int eq_tot;
+    const int eq_pre = block_scan_flag(is_eq, wt, &eq_tot);
+    const int sel = (N > 0 && p < S) && (kv > thr || (is_eq && (uint32_t)(eq_seen + eq_pre) < need));
+    eq_seen += eq_tot;
+    const unsigned bal = __ballot_sync(0xffffffffu, sel);
+    if ((threadIdx.x & 31) == 0) halves[threadIdx.x >> 5] = bal;
+    int tot;
+    const int pre = block_scan_flag(sel, wt, &tot);
+    if (sel) rp[base + pre] = p;
+    // 16 words of 64 positions per chunk; threads 0..15 write them
+    if (threadIdx.x < 16) {
+      const int wi = (c0 >> 6) + threadIdx.x;
+      if (wi < d->n_words) {
+        const uint64_t word = (uint64_t)halves[2 * threadIdx.x] | ((uint64_t)halves[2 * threadIdx.x + 1] << 32);
+        bm[wi] = word;
+        int before = 0;
+        for (int t = 0; t < (int)threadIdx.x; ++t)
+          before += __popcll((uint64_t)halves[2 * t] | ((uint64_t)halves[2 * t + 1] << 32));
+        pf[wi] = (uint32_t)(base + before);
+      }
+    }
+    base += tot;
+    __syncthreads();
+  }
+}
+
+// One warp per residual slot: r = x - gamma x_a (fp64), v = H(s o r), quantize.
+__global__ void enc_quant(const EncArgs A) {
+  __shared__ double vbuf[8][128];
+  const int u = blockIdx.y, side = blockIdx.z;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int N = side ? d->n_res_v : d->n_res_k;
+  const int wi = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int s = blockIdx.x * 8 + wi;
+  if (s >= N) return;
+  EncUnitWs w = unit_ws(A, u, d);
+  const int p = w.res_pos[(side ? d->n_res_k : 0) + s];
+  const uint32_t st = reinterpret_cast<const uint32_t*>(A.arena_c + (side ? d->off_stream_v : d->off_stream_k))[p];
+  const int a = (int)(st & 0xFFFFu);
+  const double g = fp16_bits_to_f64(st >> 16);
+  const bool valid = w.ctrl[side] != 0u;
+  const __nv_bfloat16* X = (side ? A.V : A.K) + ((size_t)u * A.s_max + p) * 128;
+  const __nv_bfloat16* XA =
+      reinterpret_cast<const __nv_bfloat16*>(A.arena_c + (side ? d->off_anchor_v : d->off_anchor_k)) + (size_t)a * 128;
+  double* v = vbuf[wi];
+  for (int j = lane; j < 128; j += 32) {
+    const double pj = valid ? __dmul_rn(g, bf16_to_f64(XA[j])) : 0.0;
+    double r = __dsub_rn(bf16_to_f64(X[j]), pj);
+    if (A.rotate) {
+      const unsigned long long sb = j < 64 ? A.sign_lo : A.sign_hi;
+      if ((sb >> (j & 63)) & 1ull) r = -r;
+    }
+    v[j] = r;
+  }
+  __syncwarp();
+  if (A.rotate) {
+    for (int hh = 1; hh < 128; hh <<= 1) {
+      for (int pr = lane; pr < 64; pr += 32) {
+        const int j = (pr / hh) * 2 * hh + (pr % hh);
+        const double x = v[j], y = v[j + hh];
+        v[j] = __dadd_rn(x, y);
+        v[j + hh] = __dsub_rn(x, y);
+      }
+      __syncwarp();
+    }
+  }
+  // min / max with the first index winning ties (as a sequential scan does)
+  double mnv = v[4 * lane], mxv = mnv;
+  int mni = 4 * lane, mxi = mni;
+  for (int c = 1; c < 4; ++c) {
+    const double x = v[4 * lane + c];
+    if (x < mnv) { mnv = x; mni = 4 * lane + c; }
+    if (x > mxv) { mxv = x; mxi = 4 * lane + c; }
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    const double omn = __shfl_xor_sync(0xffffffffu, mnv, o);
+    const int omi = __shfl_xor_sync(0xffffffffu, mni, o);
+    const double omx = __shfl_xor_sync(0xffffffffu, mxv, o);
+    const int oxi = __shfl_xor_sync(0xffffffffu, mxi, o);
+    if (omn < mnv || (omn == mnv && omi < mni)) { mnv = omn; mni = omi; }
+    if (omx > mxv || (omx == mxv && oxi < mxi)) { mxv = omx; mxi = oxi; }
+  }
+  const uint32_t mnh = f64_to_fp16_bits(mnv);
+  const double mn = fp16_bits_to_f64(mnh);
+  double t = __ddiv_rn(__dsub_rn(mxv, mn), 3.0);
+  if (!(t > 0.0)) t = 0.0;
+  const uint32_t sch = f64_to_fp16_bits(t);
+  const double sc = fp16_bits_to_f64(sch);
+  uint32_t byte = 0;
+  for (int c = 0; c < 4; ++c) {
+    int code = 0;
+    if (sc != 0.0) {
+      double qv = rint(__ddiv_rn(__dsub_rn(v[4 * lane + c], mn), sc));
+      qv = fmin(fmax(qv, 0.0), 3.0);
+      code = (int)qv;
+    }
+    byte |= (uint32_t)code << (2 * c);
+  }
+  uint8_t* codes = A.arena + (side ? d->off_codes_v : d->off_codes_k) + (size_t)s * 32;
+  codes[lane] = (uint8_t)byte;
+  if (lane == 0) {
+    uint32_t* sca = reinterpret_cast<uint32_t*>(A.arena + (side ? d->off_scales_v : d->off_scales_k));
+    sca[s] = sch | (mnh << 16);
+  }
+}
+
+}  // namespace
+
+int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const void* K, const void* V, int32_t s_max,
+                  void* arena, void* ws, void* stream) {
+  cudaStream_t st = (cudaStream_t)stream;
+  const int units = (int)L.shape.size();
+  cudaError_t e;
+  // header + descriptors, then the per-unit workspace table at the start of ws
+  std::vector<uint8_t> head(kHeaderBytes + kDescBytes * (size_t)units);
+  std::memcpy(head.data(), &L.header, sizeof(L.header));
+  std::memcpy(head.data() + kHeaderBytes, L.desc.data(), kDescBytes * (size_t)units);
+  if ((e = cudaMemsetAsync(arena, 0, (size_t)L.total_bytes, st)) != cudaSuccess) return (int)e;
+  if ((e = cudaMemcpyAsync(arena, head.data(), head.size(), cudaMemcpyHostToDevice, st)) != cudaSuccess) return (int)e;
+  std::vector<uint64_t> table(W.unit_off.begin(), W.unit_off.end());
+  if ((e = cudaMemcpyAsync(ws, table.data(), (size_t)units * 8, cudaMemcpyHostToDevice, st)) != cudaSuccess)
+    return (int)e;
+
+  EncArgs A;
+  A.arena_c = (const uint8_t*)arena;
+  A.arena = (uint8_t*)arena;
+  A.ws_base = (const uint8_t*)ws;
+  A.ws_off = (const uint64_t*)ws;
+  A.K = (const __nv_bfloat16*)K;
+  A.V = (const __nv_bfloat16*)V;
+  A.s_max = s_max;
+  A.n_kv_heads = p.n_kv_heads;
+  A.window = p.window;
+  A.rotate = (p.flags & AKV_FLAG_ROTATE) ? 1 : 0;
+  A.seed = p.seed;
+  A.sign_lo = L.header.sign_bits[0];
+  A.sign_hi = L.header.sign_bits[1];
+
+  const unsigned maxS = (unsigned)L.max_len;
+  enc_hash<<<dim3((maxS + 255) / 256, units), 256, 0, st>>>(A);
+  enc_anchors<<<units, 1024, 0, st>>>(A);
+  enc_rows<<<dim3((unsigned)(L.max_k + 7) / 8, units), 256, 0, st>>>(A);
+  if ((e = cudaFuncSetAttribute(enc_assign, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AS_SMEM)) != cudaSuccess)
+    return (int)e;
+  enc_assign<<<dim3((maxS + AS_POS - 1) / AS_POS, units, 2), AS_THREADS, AS_SMEM, st>>>(A);
+  enc_slots<<<dim3(units, 2), 1024, 0, st>>>(A);
+  const int maxN = std::max(L.max_nk, L.max_nv);
+  if (maxN > 0) enc_quant<<<dim3((unsigned)(maxN + 7) / 8, units, 2), 256, 0, st>>>(A);
+  return (int)cudaGetLastError();
+}
+
+}  // namespace akv

@@ -1,0 +1,77 @@
+"""Shared helpers of the GPU parity tests (inputs, device copies, tolerances)."""
+from __future__ import annotations
+
+import numpy as np
+
+import gen
+import oracle
+import paper_2608_02901_gb300 as akv
+
+# Tolerances (written out in DESIGN.md, "Parity bar"):
+#  fp32 output vs the fp64 oracle: fp32 accumulation over <= 2^17 terms of
+#  magnitude <= 1 with exp2 approximations; 1e-4 absolute is ~100x the expected error.
+F32_MAX_ABS = 1e-4
+#  bf16 output: max-abs 5e-3 and mean-abs 5e-4, except that an element with
+#  |y| >= 2 may differ by its bf16 half-ulp (7.8e-3 in [2, 4)) plus the fp32 bound.
+BF16_MAX_ABS = 5e-3
+BF16_MEAN_ABS = 5e-4
+
+
+def bf16_half_ulp(y: np.ndarray) -> np.ndarray:
+    a = np.maximum(np.abs(y), 2.0**-126)
+    e = np.floor(np.log2(a))
+    return 0.5 * 2.0 ** (e - 7)
+
+
+def check_outputs(out_bf16: np.ndarray, out_f32: np.ndarray, ref: np.ndarray, where: str = ""):
+    assert np.all(np.isfinite(out_f32)), where
+    e32 = np.abs(out_f32.astype(np.float64) - ref)
+    tol32 = F32_MAX_ABS * np.maximum(1.0, np.abs(ref))
+    assert np.all(e32 <= tol32), f"{where}: fp32 max err {e32.max():.3e}"
+    e16 = np.abs(out_bf16.astype(np.float64) - ref)
+    bound = np.maximum(BF16_MAX_ABS, bf16_half_ulp(ref) + tol32)
+    assert np.all(e16 <= bound), f"{where}: bf16 max err {e16.max():.3e}"
+    if np.abs(ref).max() < 64:
+        assert e16.mean() <= BF16_MEAN_ABS, f"{where}: bf16 mean err {e16.mean():.3e}"
+    return e16.max(), e16.mean(), e32.max()
+
+
+def to_dev_u16(a: np.ndarray, torch, dev, dtype=None):
+    t = torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev)
+    return t.view(dtype or torch.bfloat16)
+
+
+def seeded_units(p: akv.Params, lens, seed=5, mutate=None):
+    shapes = akv.akv_unit_shapes(p, lens)
+    units = []
+    for u, (S, k, nk, nv) in enumerate(shapes):
+        d = gen.seeded_cache(int(S), int(k), int(nk), int(nv), p.window, seed, u)
+        if mutate:
+            mutate(u, d)
+        units.append(d)
+    return units
+
+
+def oracle_unit(d: dict) -> oracle.Unit:
+    u = oracle.alloc_unit(d["S"], d["k"], d["nk"], d["nv"])
+    for name in ("anchor_k", "anchor_v", "anchor_pos", "idx_k", "gam_k", "idx_v", "gam_v", "res_k", "codes_k",
+                 "scale_k", "min_k", "res_v", "codes_v", "scale_v", "min_v"):
+        getattr(u, name)[...] = d[name]
+    return u
+
+
+def decode_on_gpu(torch, p: akv.Params, lens, arena_dev, q: np.ndarray, sm_scale: float):
+    dev = arena_dev.device
+    B, Hq = p.batch, p.n_q_heads
+    qt = to_dev_u16(q.reshape(B, Hq, 128), torch, dev)
+    out = torch.empty((B, Hq, 128), dtype=torch.bfloat16, device=dev)
+    out32 = torch.empty((B, Hq, 128), dtype=torch.float32, device=dev)
+    akv.akv_decode_attn(p, lens, arena_dev, qt, out, out32, sm_scale=sm_scale)
+    torch.cuda.synchronize()
+    return out.float().cpu().numpy(), out32.cpu().numpy()
+
+
+def oracle_decode(p: akv.Params, units, q: np.ndarray, sm_scale: float, sel=None):
+    G = p.G
+    ref = oracle.attend(units, q.reshape(p.n_units, G, 128), G, sm_scale, p.rot_seed, p.rotate, sel=sel)
+    return ref.reshape(p.batch, p.n_q_heads, 128)

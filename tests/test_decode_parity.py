@@ -1,0 +1,122 @@
+"""Decode parity: the CUDA path through the C ABI against the fp64 oracle (GPU)."""
+import math
+
+import numpy as np
+import pytest
+
+import gen
+import oracle
+import paper_2608_02901_gb300 as akv
+from helpers import check_outputs, decode_on_gpu, oracle_decode, oracle_unit, seeded_units, to_dev_u16
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dev():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    akv.lib()
+    return torch.device("cuda:0")
+
+
+def _run_seeded(dev, p, lens, sm_scale=1.0, seed=5, mutate=None, qseed=17):
+    units = seeded_units(p, lens, seed=seed, mutate=mutate)
+    arena = akv.akv_cache_pack_host(p, lens, [akv.unit_host_from_logical(u) for u in units])
+    arena_dev = torch.from_numpy(arena).to(dev)
+    q = gen.queries(p.batch * p.n_q_heads, seed=qseed)
+    out, out32 = decode_on_gpu(torch, p, lens, arena_dev, q, sm_scale)
+    ref = oracle_decode(p, [oracle_unit(u) for u in units], q, sm_scale)
+    return check_outputs(out, out32, ref, where=f"lens={lens} G={p.G}")
+
+
+@pytest.mark.parametrize("G", [1, 2, 4, 8])
+@pytest.mark.parametrize("lens", [[1], [5, 31], [32, 33, 64], [511, 512, 513], [1000, 4173]])
+def test_seeded_small_and_ragged(dev, G, lens):
+    p = akv.Params(batch=len(lens), n_kv_heads=2, n_q_heads=2 * G, seed=3, rot_seed=77)
+    _run_seeded(dev, p, lens)
+
+
+@pytest.mark.parametrize("fr", [(0.02, 0.0, 0.0), (0.02, 1.0, 1.0), (0.5, 0.3, 0.0), (0.01, 0.2, 0.05)])
+@pytest.mark.parametrize("sm_scale", [1.0, 1.0 / math.sqrt(128)])
+def test_budgets_and_scales(dev, fr, sm_scale):
+    p = akv.Params(batch=2, n_kv_heads=2, n_q_heads=8, anchor_frac=fr[0], res_frac_k=fr[1], res_frac_v=fr[2],
+                   seed=9, rot_seed=5)
+    _run_seeded(dev, p, [3000, 2047], sm_scale=sm_scale)
+
+
+def test_rotation_off(dev):
+    p = akv.Params(batch=1, n_kv_heads=2, n_q_heads=4, rotate=False, res_frac_k=0.3, res_frac_v=0.3)
+    _run_seeded(dev, p, [2500])
+
+
+def test_negative_and_saturated_gamma_and_zero_anchor(dev):
+    def mutate(u, d):
+        d["gam_k"] = d["gam_k"].copy()
+        d["gam_v"] = d["gam_v"].copy()
+        non = np.setdiff1d(np.arange(d["S"]), d["anchor_pos"])
+        d["gam_k"][non[::3]] ^= 0x8000  # negative gamma
+        d["gam_v"][non[1::5]] ^= 0x8000
+        if u == 0:
+            d["gam_v"][non[7]] = 0x7BFF  # fp16 maximum on a value coefficient
+        d["anchor_k"] = d["anchor_k"].copy()
+        d["anchor_k"][1] = 0  # an all-zero anchor key
+    p = akv.Params(batch=2, n_kv_heads=1, n_q_heads=4)
+    _run_seeded(dev, p, [1500, 900], mutate=mutate)
+
+
+def test_many_units_cluster_sizes(dev, monkeypatch):
+    p = akv.Params(batch=4, n_kv_heads=4, n_q_heads=16)
+    for c in ("1", "2", "3", "8", "16"):
+        monkeypatch.setenv("AKV_CLUSTER", c)
+        _run_seeded(dev, p, [8192, 3000, 6001, 700], qseed=int(c))
+
+
+def test_tiny_encoded_config(dev):
+    """configs[0]-shaped case: S=4096, one KV head, G=1, encoded on the GPU."""
+    S = 4096
+    p = akv.Params(batch=1, n_kv_heads=1, n_q_heads=1, seed=7, rot_seed=11)
+    K, V = gen.clustered_batch(1, 1, [S], seed=42)
+    a_bytes, w_bytes = akv.akv_cache_size(p, [S])
+    arena = torch.empty(a_bytes, dtype=torch.uint8, device=dev)
+    ws = torch.empty(w_bytes, dtype=torch.uint8, device=dev)
+    akv.akv_encode(p, [S], to_dev_u16(K, torch, dev), to_dev_u16(V, torch, dev), arena, ws)
+    units = oracle.unpack_arena(arena.cpu().numpy())
+    for t in range(4):
+        for sm in (1.0, 1 / math.sqrt(128)):
+            q = gen.queries(1, seed=100 + t)
+            out, out32 = decode_on_gpu(torch, p, [S], arena, q, sm)
+            ref = oracle_decode(p, units, q, sm)
+            check_outputs(out, out32, ref, "tiny")
+
+
+def test_8b_32k_encoded(dev):
+    """Llama-3.1-8B layer shape, 32K context, GPU encode, several fresh queries."""
+    S, H, Hq = 32768, 8, 32
+    p = akv.Params(batch=1, n_kv_heads=H, n_q_heads=Hq, seed=1, rot_seed=2)
+    K, V = gen.clustered_batch(1, H, [S], seed=42)
+    a_bytes, w_bytes = akv.akv_cache_size(p, [S])
+    arena = torch.empty(a_bytes, dtype=torch.uint8, device=dev)
+    ws = torch.empty(w_bytes, dtype=torch.uint8, device=dev)
+    akv.akv_encode(p, [S], to_dev_u16(K, torch, dev), to_dev_u16(V, torch, dev), arena, ws)
+    units = oracle.unpack_arena(arena.cpu().numpy())
+    for t in range(3):
+        q = gen.queries(Hq, seed=200 + t)
+        out, out32 = decode_on_gpu(torch, p, [S], arena, q, 1.0)
+        check_outputs(out, out32, oracle_decode(p, units, q, 1.0), "8b-32k")
+
+
+@pytest.mark.parametrize("shape", [("8b-128k", 4, 8, 32), ("70b-128k", 8, 8, 64)])
+def test_128k_seeded(dev, shape):
+    name, B, H, Hq = shape
+    S = 131072
+    p = akv.Params(batch=B, n_kv_heads=H, n_q_heads=Hq, seed=4, rot_seed=8)
+    _run_seeded(dev, p, [S] * B, seed=11)
+
+
+def test_ragged_sweep_points(dev):
+    lens = gen.ragged_lens(16, 8192, 131072, seed=3)
+    for fa, fr in ((0.01, 0.0), (0.04, 0.2), (0.02, 0.1)):
+        p = akv.Params(batch=16, n_kv_heads=8, n_q_heads=32, anchor_frac=fa, res_frac_k=fr, res_frac_v=fr)
+        _run_seeded(dev, p, lens, seed=int(fa * 1000 + fr * 100))
