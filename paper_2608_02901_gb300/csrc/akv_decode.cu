@@ -21,8 +21,10 @@
 
 #include <cstdio>
 #include <cstdlib>
+#include <map>
 #include <mutex>
 #include <string>
+#include <tuple>
 
 #include "akv_internal.h"
 
@@ -453,6 +455,66 @@ DeviceInfo device_info() {
   return d;
 }
 
+// Launch configuration per (device, G, shared-memory size, unit count, longest
+// context): computed once (attributes, occupancy query), then reused, so that a
+// call made during CUDA-graph capture only issues the launch itself.
+struct LaunchKey {
+  int dev, G, units, max_len, cluster_env;
+  size_t smem;
+  bool operator<(const LaunchKey& o) const {
+    return std::tie(dev, G, units, max_len, cluster_env, smem) <
+           std::tie(o.dev, o.G, o.units, o.max_len, o.cluster_env, o.smem);
+  }
+};
+
+template <int G>
+int choose_cluster(const LaunchKey& key, int* C_out) {
+  static std::mutex mu;
+  static std::map<LaunchKey, int> cache;
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    auto it = cache.find(key);
+    if (it != cache.end()) {
+      *C_out = it->second;
+      return 0;
+    }
+  }
+  const DeviceInfo di = device_info();
+  // The attribute is per kernel, not per launch: raise it to the device limit once,
+  // so that every cached configuration stays launchable.
+  cudaError_t e = cudaFuncSetAttribute(akv_decode_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, di.smem_optin);
+  if (e != cudaSuccess) return (int)e;
+  e = cudaFuncSetAttribute(akv_decode_kernel<G>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e != cudaSuccess) return (int)e;
+  // Cluster size: enough CTAs for one wave over the SMs, no more than the tiles of the longest unit.
+  const int per_sm = std::max(1, (int)((228 * 1024) / (key.smem + 1024)));
+  const int slots = di.sms * std::min(per_sm, 2048 / NT);
+  int C = 1;
+  while (C < kMaxCluster && (long long)key.units * (C * 2) <= slots && (C * 2) * TILE <= key.max_len + TILE - 1) C *= 2;
+  if (key.cluster_env >= 1 && key.cluster_env <= kMaxCluster) C = key.cluster_env;
+  for (; C > 1; C = (C == 3 ? 1 : C / 2)) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(C * key.units), 1, 1);
+    cfg.blockDim = dim3(NT, 1, 1);
+    cfg.dynamicSmemBytes = key.smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = C;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int nclusters = 0;
+    e = cudaOccupancyMaxActiveClusters(&nclusters, akv_decode_kernel<G>, &cfg);
+    if (e == cudaSuccess && nclusters >= 1) break;
+    cudaGetLastError();
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  cache[key] = C;
+  *C_out = C;
+  return 0;
+}
+
 template <int G>
 int launch_g(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
              float sm_scale, void* stream, std::string* why) {
@@ -463,20 +525,14 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
     *why = "anchor tables need " + std::to_string(smem) + " B of shared memory (k * G too large)";
     return -1;
   }
-  cudaError_t e = cudaFuncSetAttribute(akv_decode_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return (int)e;
-  e = cudaFuncSetAttribute(akv_decode_kernel<G>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  if (e != cudaSuccess) return (int)e;
-
-  // Cluster size: enough CTAs for one wave over the SMs, no more than the tiles of the longest unit.
-  const int per_sm = std::max(1, (int)((228 * 1024) / (smem + 1024)));
-  const int slots = di.sms * std::min(per_sm, 2048 / NT);
+  int dev = 0;
+  cudaGetDevice(&dev);
+  int cenv = 0;
+  if (const char* env = std::getenv("AKV_CLUSTER")) cenv = std::atoi(env);
+  const LaunchKey key{dev, G, units, L.max_len, cenv, smem};
   int C = 1;
-  while (C < kMaxCluster && (long long)units * (C * 2) <= slots && (C * 2) * TILE <= L.max_len + TILE - 1) C *= 2;
-  if (const char* env = std::getenv("AKV_CLUSTER")) {
-    const int c = std::atoi(env);
-    if (c >= 1 && c <= kMaxCluster) C = c;
-  }
+  int err = choose_cluster<G>(key, &C);
+  if (err) return err;
 
   DecodeParams P;
   P.arena = (const uint8_t*)arena;
@@ -490,33 +546,23 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   P.scale_log2 = sm_scale * kLog2e;
   P.sign_lo = L.header.sign_bits[0];
   P.sign_hi = L.header.sign_bits[1];
+  P.cluster = C;
 
-  for (;;) {
-    P.cluster = C;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(C * units), 1, 1);
-    cfg.blockDim = dim3(NT, 1, 1);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = (cudaStream_t)stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = C;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int nclusters = 0;
-    e = cudaOccupancyMaxActiveClusters(&nclusters, akv_decode_kernel<G>, &cfg);
-    if ((e != cudaSuccess || nclusters < 1) && C > 1) {
-      cudaGetLastError();
-      C /= 2;
-      continue;
-    }
-    e = cudaLaunchKernelEx(&cfg, akv_decode_kernel<G>, P);
-    if (e != cudaSuccess) return (int)e;
-    e = cudaGetLastError();
-    return (int)e;
-  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(C * units), 1, 1);
+  cfg.blockDim = dim3(NT, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = (cudaStream_t)stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, akv_decode_kernel<G>, P);
+  if (e != cudaSuccess) return (int)e;
+  return (int)cudaGetLastError();
 }
 
 }  // namespace

@@ -7,12 +7,16 @@ import gen
 import oracle
 import paper_2608_02901_gb300 as akv
 
-# Tolerances (written out in DESIGN.md, "Parity bar"):
-#  fp32 output vs the fp64 oracle: fp32 accumulation over <= 2^17 terms of
-#  magnitude <= 1 with exp2 approximations; 1e-4 absolute is ~100x the expected error.
+# Parity bar (written out in DESIGN.md, "Parity bar"):
+#  * fp32 output vs the fp64 oracle: max-abs <= 1e-4 * max(1, |y|).  The kernel
+#    accumulates in fp32 over <= 2^17 terms of magnitude <= 1 with hardware exp2;
+#    1e-4 is ~100x the expected error and 50x tighter than the 5e-3 target.
+#  * bf16 output: exactly the round-to-nearest-even of the kernel's fp32 result,
+#    and within one bf16 ulp of the oracle rounded to bf16 the same way.
+#  * the target bar (max-abs 5e-3, mean-abs 5e-4) on the bf16 output, widened only
+#    where bf16 rounding alone exceeds it: an element may differ by its half-ulp
+#    (7.8e-3 for |y| in [2, 4)), and the mean may reach the mean half-ulp.
 F32_MAX_ABS = 1e-4
-#  bf16 output: max-abs 5e-3 and mean-abs 5e-4, except that an element with
-#  |y| >= 2 may differ by its bf16 half-ulp (7.8e-3 in [2, 4)) plus the fp32 bound.
 BF16_MAX_ABS = 5e-3
 BF16_MEAN_ABS = 5e-4
 
@@ -23,16 +27,26 @@ def bf16_half_ulp(y: np.ndarray) -> np.ndarray:
     return 0.5 * 2.0 ** (e - 7)
 
 
+def f32_to_bf16_rne(x: np.ndarray) -> np.ndarray:
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    r = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint32) << 16
+    return r.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
 def check_outputs(out_bf16: np.ndarray, out_f32: np.ndarray, ref: np.ndarray, where: str = ""):
     assert np.all(np.isfinite(out_f32)), where
     e32 = np.abs(out_f32.astype(np.float64) - ref)
     tol32 = F32_MAX_ABS * np.maximum(1.0, np.abs(ref))
     assert np.all(e32 <= tol32), f"{where}: fp32 max err {e32.max():.3e}"
+    assert np.array_equal(out_bf16.astype(np.float64), f32_to_bf16_rne(out_f32)), f"{where}: bf16 != RNE(fp32)"
+    # both sides rounded to bf16 the same way differ by at most their fp32 gap plus two half-ulps
+    ref16 = gen.bf16_to_f64(gen.bf16_bits(ref))
+    gap = np.abs(out_bf16 - ref16)
+    assert np.all(gap <= (e32 + bf16_half_ulp(out_f32) + bf16_half_ulp(ref)) * (1 + 1e-9)), f"{where}: bf16 rounding"
     e16 = np.abs(out_bf16.astype(np.float64) - ref)
-    bound = np.maximum(BF16_MAX_ABS, bf16_half_ulp(ref) + tol32)
-    assert np.all(e16 <= bound), f"{where}: bf16 max err {e16.max():.3e}"
-    if np.abs(ref).max() < 64:
-        assert e16.mean() <= BF16_MEAN_ABS, f"{where}: bf16 mean err {e16.mean():.3e}"
+    hu = bf16_half_ulp(ref)
+    assert np.all(e16 <= np.maximum(BF16_MAX_ABS, hu + tol32)), f"{where}: bf16 max err {e16.max():.3e}"
+    assert e16.mean() <= max(BF16_MEAN_ABS, hu.mean()), f"{where}: bf16 mean err {e16.mean():.3e}"
     return e16.max(), e16.mean(), e32.max()
 
 
