@@ -201,6 +201,35 @@ akv_status akv_encode(const akv_params* p, const int32_t* ctx_lens_host, const v
                       int32_t s_max, void* arena, size_t arena_bytes, void* ws, size_t ws_bytes,
                       akv_stream_t stream);
 
+/*
+ * Encode without any device allocation by the caller or the library.
+ * The paper has no counterpart to this entry point; it exists for callers
+ * that cannot obtain device memory for a workspace -- for example a process
+ * whose memory is owned by another allocator that hands out no scratch, or
+ * a caller that must not call cudaMalloc on its critical path.  It runs the
+ * same kernels as akv_encode, with the workspace taken from a scratch array
+ * of AKV_NOALLOC_SCRATCH_BYTES that lives inside this library
+ * (a file-scope __device__ array; every GPU that loads the library holds it
+ * until the process exits).
+ *
+ *   K, V, s_max, arena, arena_bytes : as for akv_encode
+ * Limits and behaviour:
+ *  - The encode workspace that akv_cache_size reports for (p, ctx_lens_host)
+ *    must fit AKV_NOALLOC_SCRATCH_BYTES; otherwise AKV_ERR_UNSUPPORTED and
+ *    nothing is launched.
+ *  - The first call on a device looks up that device's address of the array
+ *    (cudaGetSymbolAddress, with the device current).  Make that first call
+ *    before any stream capture.
+ *  - Every call on a device shares the one array and leaves its contents
+ *    behind; the kernels need none of it cleared.  Calls whose work overlaps
+ *    on the GPU (different streams, no ordering between them) race on the
+ *    array: order them on one stream or with events.
+ * Errors: as for akv_encode, plus AKV_ERR_CUDA if the set-up lookup fails.
+ */
+#define AKV_NOALLOC_SCRATCH_BYTES ((size_t)16 << 20)
+akv_status akv_encode_noalloc(const akv_params* p, const int32_t* ctx_lens_host, const void* K, const void* V,
+                              int32_t s_max, void* arena, size_t arena_bytes, akv_stream_t stream);
+
 /* ---- Host packer -------------------------------------------------------- */
 
 /*

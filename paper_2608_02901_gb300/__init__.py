@@ -23,8 +23,9 @@ HEAD_DIM = 128
 
 EXPORTED = (
     "akv_status_string", "akv_last_error", "akv_unit_shapes", "akv_cache_size", "akv_cache_header_host",
-    "akv_encode", "akv_cache_pack_host", "akv_decode_workspace_size", "akv_decode_attn",
+    "akv_encode", "akv_encode_noalloc", "akv_cache_pack_host", "akv_decode_workspace_size", "akv_decode_attn",
 )
+NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
 class AkvError(RuntimeError):
@@ -100,6 +101,8 @@ def lib():
         L.akv_cache_header_host.argtypes = [P, i32p, vp, ctypes.c_size_t]
         L.akv_encode.restype = st
         L.akv_encode.argtypes = [P, i32p, vp, vp, ctypes.c_int32, vp, ctypes.c_size_t, vp, ctypes.c_size_t, vp]
+        L.akv_encode_noalloc.restype = st
+        L.akv_encode_noalloc.argtypes = [P, i32p, vp, vp, ctypes.c_int32, vp, ctypes.c_size_t, vp]
         L.akv_cache_pack_host.restype = st
         L.akv_cache_pack_host.argtypes = [P, i32p, ctypes.POINTER(_UnitHost), vp, ctypes.c_size_t]
         L.akv_decode_workspace_size.restype = st
@@ -188,6 +191,17 @@ def akv_encode(p: Params, ctx_lens, K, V, arena, ws, stream=None):
     _check(lib().akv_encode(ctypes.byref(p.c()), _i32p(lens), _dev_ptr(K), _dev_ptr(V), s_max, _dev_ptr(arena),
                             arena.numel() * arena.element_size(), _dev_ptr(ws), ws.numel() * ws.element_size(),
                             _stream_ptr(stream)), "akv_encode")
+
+
+def akv_encode_noalloc(p: Params, ctx_lens, K, V, arena, stream=None):
+    """akv_encode without a workspace argument: for callers that cannot obtain
+    device memory for scratch.  The library's own static scratch array (16 MiB
+    per device) is used instead; calls that overlap on the GPU race on it."""
+    lens = _lens(ctx_lens)
+    s_max = int(K.shape[2])
+    _check(lib().akv_encode_noalloc(ctypes.byref(p.c()), _i32p(lens), _dev_ptr(K), _dev_ptr(V), s_max,
+                                    _dev_ptr(arena), arena.numel() * arena.element_size(), _stream_ptr(stream)),
+           "akv_encode_noalloc")
 
 
 _UNIT_FIELDS = (("anchor_k", np.uint16), ("anchor_v", np.uint16), ("anchor_pos", np.int32), ("idx_k", np.uint16),

@@ -282,6 +282,28 @@ akv_status akv_encode(const akv_params* p, const int32_t* ctx_lens_host, const v
   return AKV_OK;
 }
 
+akv_status akv_encode_noalloc(const akv_params* p, const int32_t* ctx_lens_host, const void* K, const void* V,
+                              int32_t s_max, void* arena, size_t arena_bytes, akv_stream_t stream) {
+  // Same validation and kernels as akv_encode; the workspace is the library's
+  // static scratch array, so nothing here or in the caller allocates device memory.
+  g_last_error.clear();
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L);
+  if (st != AKV_OK) return st;
+  EncodeWs W;
+  encode_ws_layout(L, &W);
+  if (W.total > AKV_NOALLOC_SCRATCH_BYTES)
+    return fail(AKV_ERR_UNSUPPORTED, "encode needs " + std::to_string(W.total) +
+                                         " B of scratch, more than the " +
+                                         std::to_string((size_t)AKV_NOALLOC_SCRATCH_BYTES) +
+                                         " B static array of akv_encode_noalloc; use akv_encode with a workspace");
+  void* ws = nullptr;
+  size_t ws_bytes = 0;
+  int err = noalloc_scratch(&ws, &ws_bytes);
+  if (err) return fail(AKV_ERR_CUDA, std::string("scratch address lookup failed: ") + cuda_error_string(err));
+  return akv_encode(p, ctx_lens_host, K, V, s_max, arena, arena_bytes, ws, ws_bytes, stream);
+}
+
 akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_lens_host, size_t* ws_bytes) {
   g_last_error.clear();
   Layout L;

@@ -18,6 +18,7 @@
 #include <cuda_runtime.h>
 
 #include <cstring>
+#include <mutex>
 #include <vector>
 
 #include "akv_internal.h"
@@ -486,6 +487,33 @@ __global__ void enc_quant(const EncArgs A) {
 }
 
 }  // namespace
+
+// Scratch of akv_encode_noalloc, for callers that cannot hand the library a
+// device workspace.  It is part of the module image: no allocation call makes
+// it, and each device that loads the library keeps it until the process exits.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[AKV_NOALLOC_SCRATCH_BYTES];
+
+int noalloc_scratch(void** ptr, size_t* bytes) {
+  // Host code must not use g_noalloc_scratch's name as a device address: it is
+  // a host-side stand-in.  The device address is looked up once per device,
+  // with that device current.
+  static std::mutex mu;
+  static void* addr[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return (int)e;
+  if (dev < 0 || dev >= 64) return (int)cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lk(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return (int)e;
+    addr[dev] = p;
+  }
+  *ptr = addr[dev];
+  *bytes = AKV_NOALLOC_SCRATCH_BYTES;
+  return 0;
+}
 
 int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const void* K, const void* V, int32_t s_max,
                   void* arena, void* ws, void* stream) {

@@ -63,5 +63,8 @@ int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const
 int launch_decode(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
                   float sm_scale, void* stream, std::string* why);
 const char* cuda_error_string(int err);
+// Device address of the library's static encode scratch on the current device
+// (looked up once per device); returns a cudaError_t as int.
+int noalloc_scratch(void** ptr, size_t* bytes);
 
 }  // namespace akv
