@@ -59,6 +59,11 @@ def unit_bytes(S, k, nk, nv, G):
     return 512 * k + 8 * S + 24 * words + 36 * (nk + nv) + 2 * (2 * G * 128)
 
 
+def rank_seed(base: int, rank: int) -> int:
+    """Seed of a rank's shard: every rank encodes and decodes its own batch (weak scaling)."""
+    return base + 1000003 * rank
+
+
 def dist_setup(args):
     import torch
     rank = int(os.environ.get("RANK", "0"))
@@ -159,7 +164,7 @@ def kernel_traffic():
         return None
 
 
-def build_layers(torch, akv, gen, p, lens, layers, source, dev):
+def build_layers(torch, akv, gen, p, lens, layers, source, dev, rank=0):
     """Device arenas of `layers` distinct layer caches and the bytes one decode reads."""
     arena_bytes, ws_bytes = akv.akv_cache_size(p, lens)
     shapes = akv.akv_unit_shapes(p, lens)
@@ -169,7 +174,7 @@ def build_layers(torch, akv, gen, p, lens, layers, source, dev):
         ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
         S = lens[0]
         for layer in range(layers):
-            K, V = gen.clustered_batch_torch(p.batch, p.n_kv_heads, S, seed=1000 + layer, device=dev)
+            K, V = gen.clustered_batch_torch(p.batch, p.n_kv_heads, S, seed=rank_seed(1000 + layer, rank), device=dev)
             arena = torch.empty(arena_bytes, dtype=torch.uint8, device=dev)
             akv.akv_encode(p, lens, K, V, arena, ws)
             arenas.append(arena)
@@ -181,7 +186,7 @@ def build_layers(torch, akv, gen, p, lens, layers, source, dev):
         for layer in range(layers):
             if layer < 2:
                 units = [akv.unit_host_from_logical(gen.seeded_cache(int(S), int(k), int(nk), int(nv), p.window,
-                                                                       2000 + layer, u))
+                                                                       rank_seed(2000 + layer, rank), u))
                          for u, (S, k, nk, nv) in enumerate(shapes)]
                 img = akv.akv_cache_pack_host(p, lens, units)
                 arena = torch.from_numpy(img).to(dev)
@@ -201,9 +206,9 @@ def run_akv(args, rank, world, local):
     dev = torch.device("cuda", local)
     B, H, Hq, S, source = WORKLOADS[args.workload]
     lens = [S] * B
-    p = akv.Params(batch=B, n_kv_heads=H, n_q_heads=Hq, seed=11 + rank, rot_seed=0x5EED)
+    p = akv.Params(batch=B, n_kv_heads=H, n_q_heads=Hq, seed=rank_seed(11, rank), rot_seed=0x5EED)
     layers = args.layers
-    arenas, arena_bytes, step_bytes = build_layers(torch, akv, gen, p, lens, layers, source, dev)
+    arenas, arena_bytes, step_bytes = build_layers(torch, akv, gen, p, lens, layers, source, dev, rank)
     n_tok = N_TOKENS
     qs = gen.queries_torch(n_tok * layers * B * Hq, seed=77 + rank, device=dev).view(n_tok, layers, B, Hq, 128)
     out = torch.empty((n_tok, layers, B, Hq, 128), dtype=torch.bfloat16, device=dev)
