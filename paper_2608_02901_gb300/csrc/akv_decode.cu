@@ -4,28 +4,31 @@
 // unit's positions and its anchors.  Eq. 3 is folded into Eq. 4: no key or
 // value row is ever rebuilt in memory.
 //
-// Warp roles per CTA: 8 compute warps and 1 producer warp.  The producer
-// streams one sequence of items through a ring of shared-memory stages with
-// bulk asynchronous copies (cp.async.bulk completing on mbarrier transaction
-// counts) and prefetches later items into L2:
-//   [anchor-key chunks of this CTA's slice] [position tiles] [anchor-value chunks]
-// The compute warps consume the same sequence:
-//   phase 0  q rows and the rotated-domain query q' = H(s o q)/128 (Appendix A.1,
-//            Eq. 12); tensor-core fragments of q (bf16) and of q' (fp16 hi + lo)
-//   phase 1  anchor scores S_A = q . k_a of the slice (bf16 mma.sync), then every
-//            CTA gathers the full S_A table from its peers (DSMEM)
-//   phase 2  per tile: key logits gamma_i S_A[a(i)] plus the residual term
-//            min sum(q') + scale (q' . c), with q' . c on tensor cores straight
-//            from the packed 2-bit codes; running max; p = 2^(l - m); value
-//            weights scattered per anchor; value residuals accumulated in the
-//            rotated domain on tensor cores (p * scale as fp16 hi + lo)
-//   phase 3  cluster combine (max / sum rescale of Eq. 4) through DSMEM; each CTA
-//            reduces its slice of the value weights and multiplies it by its
-//            anchor values on tensor cores, inverse-rotates its residual
-//            accumulator once (Appendix E.1), then partial outputs are summed
-//            and normalised.
-// Every wait on an mbarrier is bounded; a wait that runs out marks the CTA
-// failed, the CTA stops issuing and consuming, and its outputs become NaN.
+// Warp-specialised CTA (15 warps):
+//   producer warp     streams one sequence of items through a ring of shared-
+//                     memory stages with 16-byte asynchronous copies (cp.async),
+//                     each lane's copies completing an mbarrier arrival:
+//                     [anchor-key chunks] [position tiles] [anchor-value chunks]
+//   2 key-residual warps  per tile: q' . c for the staged key slots on tensor
+//                     cores, straight from the packed 2-bit codes (q' = H(s o q)/128,
+//                     Appendix A.1 Eq. 12, as fp16 high + low parts)
+//   8 token warps     phase 1: anchor scores S_A = q . k_a of the CTA's anchor slice
+//                     (bf16 tensor cores), gathered cluster-wide through DSMEM;
+//                     per tile: logits gamma_i S_A[a(i)] + residual term, p = 2^(l - m),
+//                     value weights scattered per anchor, value-residual operands;
+//                     phase 3: cluster combine and the anchor-value product
+//   4 value-residual warps  per tile: sum of (p scale) c over the staged value
+//                     slots on tensor cores, in the rotated domain
+// Stages are handed between the roles with mbarriers, so different roles work on
+// different tiles at the same time.
+//
+// The exponent reference m is the largest anchor score of each query row.  Anchors
+// are tokens of the unit, so m never exceeds the true maximum logit (sums cannot
+// overflow unless a logit exceeds m by more than 2^120, which is flagged), and all
+// CTAs of a cluster share the same m: no running-max rescaling is needed and the
+// cluster combine (Eq. 4 normaliser and numerator) is a plain sum.
+// Every wait on an mbarrier is bounded; a wait that runs out marks the CTA failed,
+// the CTA stops issuing and consuming, and its outputs become NaN.
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -46,15 +49,22 @@ namespace cg = cooperative_groups;
 namespace akv {
 namespace {
 
-constexpr int NCW = 8;         // compute warps
-constexpr int NCT = NCW * 32;  // compute threads
-constexpr int NT = NCT + 32;   // plus the producer warp
-constexpr int T = 512;         // positions per tile
-constexpr int PPT = T / NCT;   // positions per compute thread
+// warp roles
+constexpr int NTW = 8;                 // token warps (warps 0 .. 7)
+constexpr int NTT = NTW * 32;          // token threads
+constexpr int W_KRES = NTW;            // key-residual warps
+constexpr int NKR = 2;
+constexpr int W_VRES = W_KRES + NKR;   // value-residual warps
+constexpr int NVR = 4;
+constexpr int W_PROD = W_VRES + NVR;   // producer warp
+constexpr int NT = (W_PROD + 1) * 32;  // 480 threads
+constexpr int T = 512;                 // positions per tile
+constexpr int PPT = T / NTT;           // positions per token thread
 static_assert(PPT == 2, "the token pass reads two stream words per thread");
+static_assert(NTW % NVR == 0, "value-residual warps release a stage with NTW / NVR arrivals each");
 constexpr int ROWS = 32;   // anchor rows per chunk
 constexpr int ROWB = 272;  // shared-memory stride of a staged anchor row (256 B + 16 B pad)
-constexpr int ROWE = 48;   // stride of an expanded row of 16 codes (32 B + 16 B pad)
+constexpr int ROWE = 80;   // stride of an expanded row of 32 codes (64 B + 16 B pad)
 constexpr int kMaxCluster = 16;
 constexpr unsigned kWaitLimit = 1u << 22;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -76,9 +86,9 @@ struct DecodeParams {
   int n_kv_heads, n_q_heads, cluster, rotate, max_k;
   float scale_log2;
   unsigned long long sign_lo, sign_hi;
-  int R, NS, stage_bytes, max_tiles, pf_items;
-  int o_sa, o_w, o_bk, o_bv, o_qfa, o_qfk, o_qs, o_qp, o_rs, o_pf, o_e, o_acc, o_opart, o_misc, o_bar, o_ring;
-  int o_cdk, o_sck, o_cdv, o_scv;  // record buffers inside a stage
+  int R, NS, stage_bytes, max_tiles;
+  int o_sa, o_w, o_bk, o_bv, o_qfa, o_qfk, o_qp, o_acc, o_opart, o_e, o_misc, o_bar, o_ring;
+  int o_cdk, o_sck, o_cdv, o_scv, o_rsb, o_pfb;  // inside a stage
 };
 
 // ---- device helpers ---------------------------------------------------------------
@@ -87,9 +97,6 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)_
 
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
@@ -107,15 +114,32 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   }
   return false;
 }
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-               "l"(src), "r"(bytes), "r"(bar)
-               : "memory");
+// 16-byte asynchronous copy global -> shared (L2 only); completion is tracked by
+// cp_arrive_on on an mbarrier.  Many small copies from all lanes keep far more bytes in
+// flight per SM than a few bulk copies of the small pieces a tile is made of.
+__device__ __forceinline__ void cp16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
 }
-__device__ __forceinline__ void bulk_prefetch(const void* src, uint32_t bytes) {
-  if (bytes) asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+// Copies `bytes` (a multiple of 16) with the lanes of one warp.
+__device__ __forceinline__ void warp_copy(uint32_t dst, const void* src, uint32_t bytes, int lane) {
+  const uint8_t* s = reinterpret_cast<const uint8_t*>(src);
+  for (uint32_t o = (uint32_t)lane * 16u; o < bytes; o += 512u) cp16(dst + o, s + o);
 }
-__device__ __forceinline__ void cw_sync() { asm volatile("bar.sync 1, %0;" ::"n"(NCT) : "memory"); }
+// The mbarrier counts one arrival from this thread once all of its earlier cp.async copies landed.
+__device__ __forceinline__ void cp_arrive_on(uint32_t bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void red_add(float* p, float v) {
+  asm volatile("red.shared.add.f32 [%0], %1;" ::"r"(smem_u32(p)), "f"(v) : "memory");
+}
+__device__ __forceinline__ void tw_sync() { asm volatile("bar.sync 1, %0;" ::"n"(NTT) : "memory"); }
+__device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+__device__ __forceinline__ void named_arrive(int id, int n) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cnt(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
 __device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 
@@ -169,11 +193,11 @@ __device__ __forceinline__ float warp_max(float v) {
 }
 
 // Unnormalised 128-point Walsh-Hadamard transform of `rows` rows in shared
-// memory, by the compute warps.
-__device__ void cw_wht_rows(float* v, int rows) {
+// memory, by the token warps.
+__device__ void tw_wht_rows(float* v, int rows) {
   for (int h = 1; h < 128; h <<= 1) {
-    cw_sync();
-    for (int e = threadIdx.x; e < rows * 64; e += NCT) {
+    tw_sync();
+    for (int e = threadIdx.x; e < rows * 64; e += NTT) {
       const int r = e >> 6, pr = e & 63;
       const int j = (pr / h) * 2 * h + (pr % h);
       float* x = v + r * 128;
@@ -182,7 +206,7 @@ __device__ void cw_wht_rows(float* v, int rows) {
       x[j + h] = a - b;
     }
   }
-  cw_sync();
+  tw_sync();
 }
 
 // Sections of one unit.
@@ -226,48 +250,43 @@ __device__ __forceinline__ UnitView unit_view(const uint8_t* A, int u) {
 
 __host__ __device__ constexpr uint32_t round16(uint32_t x) { return (x + 15u) & ~15u; }
 
-// Byte ranges of one position tile (used for both the stage copy and the L2 prefetch):
-// streams, bitmaps and prefix words of both sides (6), codes and scales of both sides (4).
-constexpr int kTileCopies = 10;
-struct TileCopy {
-  const void* src[kTileCopies];
-  uint32_t bytes[kTileCopies];
-  uint32_t dst[kTileCopies];
-  int n;
-  uint32_t total;
+// One of the ten copies of a position tile, chosen by lane (0-9): K and V streams,
+// bitmaps and prefix words of both sides, then codes and (scale, min) words of the staged
+// residual slots of both sides.  Used for both the stage copy and the L2 prefetch.
+struct LaneCopy {
+  const void* src;
+  uint32_t bytes;
+  uint32_t dst;
 };
 
-__device__ __forceinline__ void tile_copy_plan(const DecodeParams& P, const UnitView& U, int t0, int te, int skl,
-                                               int skh, int svl, int svh, TileCopy& c) {
-  c.n = 0;
-  c.total = 0;
-  auto add = [&](const void* src, uint32_t bytes, uint32_t dst) {
-    if (!bytes || c.n == kTileCopies) return;
-    c.src[c.n] = src;
-    c.bytes[c.n] = bytes;
-    c.dst[c.n] = dst;
-    c.total += bytes;
-    ++c.n;
-  };
+__device__ __forceinline__ LaneCopy tile_copy_lane(const DecodeParams& P, const UnitView& U, int lane, int t0, int te,
+                                                   int skl, int skh, int svl, int svh) {
+  LaneCopy c{nullptr, 0u, 0u};
   const int npos = te - t0;
   const int w0 = t0 >> 6, nw = (npos + 63) >> 6;
-  add(U.stK + t0, round16(npos * 4), ST_K);
-  add(U.stV + t0, round16(npos * 4), ST_V);
-  add(U.bmK + w0, round16(nw * 8), ST_BMK);
-  add(U.pfK + w0, round16(nw * 4), ST_PFK);
-  add(U.bmV + w0, round16(nw * 8), ST_BMV);
-  add(U.pfV + w0, round16(nw * 4), ST_PFV);
   const int nK = min(skh - skl, P.R), nV = min(svh - svl, P.R);
-  if (nK > 0) {
-    add(U.cdK + (size_t)skl * 32, (uint32_t)nK * 32, P.o_cdk);
-    const int s0 = skl & ~3, s1 = (skl + nK + 3) & ~3;
-    add(U.scK + s0, (uint32_t)(s1 - s0) * 4, P.o_sck);
+  switch (lane) {
+    case 0: c = {U.stK + t0, round16(npos * 4), (uint32_t)ST_K}; break;
+    case 1: c = {U.stV + t0, round16(npos * 4), (uint32_t)ST_V}; break;
+    case 2: c = {U.bmK + w0, round16(nw * 8), (uint32_t)ST_BMK}; break;
+    case 3: c = {U.pfK + w0, round16(nw * 4), (uint32_t)ST_PFK}; break;
+    case 4: c = {U.bmV + w0, round16(nw * 8), (uint32_t)ST_BMV}; break;
+    case 5: c = {U.pfV + w0, round16(nw * 4), (uint32_t)ST_PFV}; break;
+    case 6:
+      if (nK > 0) c = {U.cdK + (size_t)skl * 32, (uint32_t)nK * 32, (uint32_t)P.o_cdk};
+      break;
+    case 7:
+      if (nK > 0) c = {U.scK + (skl & ~3), (uint32_t)(((skl + nK + 3) & ~3) - (skl & ~3)) * 4, (uint32_t)P.o_sck};
+      break;
+    case 8:
+      if (nV > 0) c = {U.cdV + (size_t)svl * 32, (uint32_t)nV * 32, (uint32_t)P.o_cdv};
+      break;
+    case 9:
+      if (nV > 0) c = {U.scV + (svl & ~3), (uint32_t)(((svl + nV + 3) & ~3) - (svl & ~3)) * 4, (uint32_t)P.o_scv};
+      break;
+    default: break;
   }
-  if (nV > 0) {
-    add(U.cdV + (size_t)svl * 32, (uint32_t)nV * 32, P.o_cdv);
-    const int s0 = svl & ~3, s1 = (svl + nV + 3) & ~3;
-    add(U.scV + s0, (uint32_t)(s1 - s0) * 4, P.o_scv);
-  }
+  return c;
 }
 
 template <int G>
@@ -278,6 +297,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   const int rank = (int)cluster.block_rank();
   const int u = blockIdx.x / C;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int c4 = lane & 3, r8 = lane >> 2;
   const UnitView U = unit_view(P.arena, u);
   const int S = U.S, k = U.k;
 
@@ -287,25 +307,31 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   int* bV = reinterpret_cast<int*>(smem + P.o_bv);
   uint2* qfa = reinterpret_cast<uint2*>(smem + P.o_qfa);
   uint4* qfk = reinterpret_cast<uint4*>(smem + P.o_qfk);
-  float* qs = reinterpret_cast<float*>(smem + P.o_qs);
   float* qp = reinterpret_cast<float*>(smem + P.o_qp);
-  float* rs = reinterpret_cast<float*>(smem + P.o_rs);
-  uint8_t* pfrag = smem + P.o_pf;
-  uint8_t* ebuf = smem + P.o_e;
   float* accs = reinterpret_cast<float*>(smem + P.o_acc);
   float* opart = reinterpret_cast<float*>(smem + P.o_opart);
-  float* red = reinterpret_cast<float*>(smem + P.o_misc);
-  float* sq = red + NCW * G;
-  float* cm = sq + G;
-  float* cl = cm + G;
-  float* ltot = cl + G;
-  float* peer_m = ltot + G;
-  float* peer_l = peer_m + kMaxCluster * G;
-  float* facs = peer_l + kMaxCluster * G;
-  volatile int* failed = reinterpret_cast<volatile int*>(facs + kMaxCluster * G);
+  uint8_t* ebuf = smem + P.o_e;
+  float* red = reinterpret_cast<float*>(smem + P.o_misc);  // [NTW][G]
+  float* sq = red + NTW * G;                              // [G]
+  float* mref = sq + G;                                   // [G]
+  float* cl = mref + G;                                   // [G]
+  float* pms = cl + G;                                    // [G]
+  float* ltot = pms + G;                                  // [G]
+  volatile int* failed = reinterpret_cast<volatile int*>(ltot + G);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + P.o_bar);
   uint8_t* ring = smem + P.o_ring;
   const int NS = P.NS;
+  const int max_k = P.max_k;
+  // per stage: copies of an anchor chunk landed (full_c) / of a position tile landed (full_t);
+  // stage free again (empty); key-residual terms ready (rsr); probabilities written (pr).
+  // Chunk items and tiles complete different barriers, so every waiter sees every phase of
+  // the barriers it waits on.
+  auto bar_full_c = [&](int s) { return smem_u32(bars + s); };
+  auto bar_full_t = [&](int s) { return smem_u32(bars + NS + s); };
+  auto bar_empty = [&](int s) { return smem_u32(bars + 2 * NS + s); };
+  auto bar_rs = [&](int s) { return smem_u32(bars + 3 * NS + s); };
+  auto bar_p = [&](int s) { return smem_u32(bars + 4 * NS + s); };
+  auto stage = [&](int s) { return ring + (size_t)s * P.stage_bytes; };
 
   // this CTA's anchor slice and position range
   const int a_per = ((k + C - 1) / C + 15) / 16 * 16;
@@ -315,11 +341,24 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   const int n_ka = (a1 - a0 + ROWS - 1) / ROWS;
   const int n_t = (p1 - p0 + T - 1) / T;
   const int n_items = 2 * n_ka + n_t;
+  const int R = P.R;
+  // phase index, on its stage's barrier, of item `it` (anchor chunks and tiles counted apart)
+  auto item_phase = [&](int it) -> uint32_t {
+    if (it < n_ka) return (uint32_t)(it / NS);
+    if (it < n_ka + n_t) return (uint32_t)((it - n_ka) / NS);
+    const int s = it % NS, cj = it - n_ka - n_t;
+    const int ka_on_s = n_ka > s ? (n_ka - 1 - s) / NS + 1 : 0;
+    return (uint32_t)(ka_on_s + cj / NS);
+  };
+  auto is_tile = [&](int it) { return it >= n_ka && it < n_ka + n_t; };
 
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
-      mbar_init(smem_u32(bars + s), 1);
-      mbar_init(smem_u32(bars + NS + s), NCW);
+      mbar_init(bar_full_c(s), 32);  // one arrival per producer lane, when its copies landed
+      mbar_init(bar_full_t(s), 32);
+      mbar_init(bar_empty(s), NTW);
+      mbar_init(bar_rs(s), NKR);
+      mbar_init(bar_p(s), NTW);
     }
     *failed = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -327,105 +366,224 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   __syncthreads();
 
   // =========================== producer warp ===================================
-  if (warp == NCW) {
-    cluster_arrive();  // B1; this warp never waits on anything behind B1 before it waits on B1
+  if (warp == W_PROD) {
+    cluster_arrive();  // B1: this warp never blocks on anything behind B1 before it waits on B1
     for (int i = lane; i <= n_t; i += 32) {
       const int pos = min(p0 + i * T, p1);
       bK[i] = pos >= S ? U.nk : (int)U.pfK[pos >> 6];
       bV[i] = pos >= S ? U.nv : (int)U.pfV[pos >> 6];
     }
     __syncwarp();
-    auto prefetch_item = [&](int it) {
-      if (it >= n_items || lane != 0) return;
-      if (it < n_ka || it >= n_ka + n_t) {
-        const bool val = it >= n_ka + n_t;
-        const int ci = val ? it - n_ka - n_t : it;
-        const int r0 = a0 + ci * ROWS, r1 = min(a1, r0 + ROWS);
-        bulk_prefetch((val ? U.AV : U.AK) + (size_t)r0 * 128, (uint32_t)(r1 - r0) * 256);
-      } else {
-        const int tl = it - n_ka;
-        const int t0 = p0 + tl * T, te = min(t0 + T, p1);
-        TileCopy c;
-        tile_copy_plan(P, U, t0, te, bK[tl], bK[tl + 1], bV[tl], bV[tl + 1], c);
-        for (int j = 0; j < c.n; ++j) bulk_prefetch(c.src[j], c.bytes[j]);
-      }
-    };
-    for (int it = 0; it < min(P.pf_items, n_items); ++it) prefetch_item(it);
     bool ok = true, b1_done = false;
-    int issued = 0;
     for (int it = 0; it < n_items; ++it) {
-      if (it == n_ka + n_t) {  // anchor values are consumed after B2: let B1 complete and arrive on B2
+      if (it == n_ka + n_t) {  // anchor values are consumed after B2: let B1 complete, arrive on B2
         cluster_wait();
         cluster_arrive();
         b1_done = true;
       }
       const int s = it % NS;
       const uint32_t use = (uint32_t)(it / NS);
-      if (it >= NS) ok = mbar_wait(smem_u32(bars + NS + s), (use - 1) & 1u);
+      if (it >= NS) ok = mbar_wait(bar_empty(s), (use - 1) & 1u);
       if (!ok || *failed) {
         *failed = 1;
         break;
       }
-      prefetch_item(it + P.pf_items);
-      uint8_t* st = ring + (size_t)s * P.stage_bytes;
+      uint8_t* st = stage(s);
       if (it < n_ka || it >= n_ka + n_t) {
+        // anchor rows into padded shared-memory rows (272-byte stride: conflict-free fragment loads)
         const bool val = it >= n_ka + n_t;
         const int ci = val ? it - n_ka - n_t : it;
         const int r0 = a0 + ci * ROWS, nr = min(a1 - r0, ROWS);
-        if (lane == 0) mbar_expect_tx(smem_u32(bars + s), (uint32_t)nr * 256);
-        __syncwarp();
-        if (lane < nr)
-          bulk_g2s(smem_u32(st + lane * ROWB), (val ? U.AV : U.AK) + (size_t)(r0 + lane) * 128, 256,
-                   smem_u32(bars + s));
-      } else if (lane == 0) {
+        const uint8_t* src = reinterpret_cast<const uint8_t*>((val ? U.AV : U.AK) + (size_t)r0 * 128);
+        for (int q = lane; q < nr * 16; q += 32) cp16(smem_u32(st + (q >> 4) * ROWB + (q & 15) * 16), src + q * 16);
+        cp_arrive_on(bar_full_c(s));
+      } else {
         const int tl = it - n_ka;
         const int t0 = p0 + tl * T, te = min(t0 + T, p1);
-        TileCopy c;
-        tile_copy_plan(P, U, t0, te, bK[tl], bK[tl + 1], bV[tl], bV[tl + 1], c);
-        mbar_expect_tx(smem_u32(bars + s), c.total);
-        for (int j = 0; j < c.n; ++j) bulk_g2s(smem_u32(st + c.dst[j]), c.src[j], c.bytes[j], smem_u32(bars + s));
+#pragma unroll 1
+        for (int j = 0; j < 10; ++j) {
+          const LaneCopy c = tile_copy_lane(P, U, j, t0, te, bK[tl], bK[tl + 1], bV[tl], bV[tl + 1]);
+          if (c.bytes) warp_copy(smem_u32(st + c.dst), c.src, c.bytes, lane);
+        }
+        cp_arrive_on(bar_full_t(s));
       }
       __syncwarp();
-      ++issued;
     }
     if (!b1_done) {
       cluster_wait();
       cluster_arrive();
     }
     // every copy this warp started has landed before the CTA may exit
-    for (int s = 0; s < NS && s < issued; ++s) {
-      const int last = s + ((issued - 1 - s) / NS) * NS;
-      mbar_wait(smem_u32(bars + s), (uint32_t)(last / NS) & 1u);
-    }
-    cluster_wait();    // B2
-    cluster_arrive();  // B3
-    cluster_wait();
-    cluster_arrive();  // B4
-    cluster_wait();
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    cluster_wait();  // B2
+    cluster_arrive();
+    cluster_wait();  // B3
+    cluster_arrive();
+    cluster_wait();  // B4
     return;
   }
 
-  // =========================== compute warps ===================================
+  // =========================== key-residual warps ================================
+  // q' . c for the staged key slots of each tile, 8 slots per mma group, fragments of q'
+  // (fp16 high and low parts) held in registers.
+  if (warp >= W_KRES && warp < W_KRES + NKR) {
+    const int kw = warp - W_KRES;
+    cluster_arrive();  // B1
+    named_sync(2, NTW * 32 + NKR * 32);  // q' fragments written by the token warps
+    uint4 af[8];
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) af[ks] = qfk[ks * 32 + lane];
+    bool ok = true;
+    for (int tl = 0; tl < n_t; ++tl) {
+      const int s = (n_ka + tl) % NS;
+      if (ok && !*failed) {
+        ok = mbar_wait(bar_full_t(s), (uint32_t)(tl / NS) & 1u);
+        if (!ok) *failed = 1;
+      }
+      if (ok && !*failed) {
+        const uint8_t* st = stage(s);
+        const int skl = bK[tl], nK = min(bK[tl + 1] - skl, R);
+        const uint8_t* cd = st + P.o_cdk;
+        const uint32_t* sc = reinterpret_cast<const uint32_t*>(st + P.o_sck) + (skl & 3);
+        float* rs = reinterpret_cast<float*>(const_cast<uint8_t*>(st) + P.o_rsb);
+        for (int g8 = kw; g8 * 8 < nK; g8 += NKR) {
+          const int sl = g8 * 8 + r8;  // the slot whose codes this lane feeds (B column r8)
+          uint4 w0 = make_uint4(0u, 0u, 0u, 0u), w1 = w0;
+          if (sl < nK) {
+            w0 = *reinterpret_cast<const uint4*>(cd + (size_t)sl * 32);
+            w1 = *reinterpret_cast<const uint4*>(cd + (size_t)sl * 32 + 16);
+          }
+          const uint32_t wd[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+          float d[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks) {
+            const uint32_t x = wd[ks] >> (4 * c4);
+            mma_f16(d, af[ks], codes2_to_h2(x), codes2_to_h2(x >> 2));
+          }
+          if (r8 < G) {  // D rows r8 (high parts) and r8 + 8 (low parts), columns 2c, 2c+1
+#pragma unroll
+            for (int e2 = 0; e2 < 2; ++e2) {
+              const int sl2 = g8 * 8 + 2 * c4 + e2;
+              if (sl2 < nK) {
+                const uint32_t smn = sc[sl2];
+                rs[sl2 * G + r8] = half_hi(smn) * sq[r8] + half_lo(smn) * (d[e2] + d[2 + e2]);
+              }
+            }
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar_rs(s));
+    }
+    cluster_wait();  // B1
+    cluster_arrive();
+    cluster_wait();  // B2
+    cluster_arrive();
+    cluster_wait();  // B3
+    cluster_arrive();
+    cluster_wait();  // B4
+    return;
+  }
+
+  // =========================== value-residual warps ==============================
+  // sum over staged value slots of (p scale) c, 16 slots per mma group; warp vw owns
+  // the 32 coordinates 32 vw .. 32 vw + 31 of the rotated-domain accumulator.
+  if (warp >= W_VRES && warp < W_VRES + NVR) {
+    const int vw = warp - W_VRES;
+    cluster_arrive();  // B1
+    float accV[4][4];
+#pragma unroll
+    for (int nb = 0; nb < 4; ++nb)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) accV[nb][e] = 0.f;
+    uint8_t* ew = ebuf + vw * 16 * ROWE;
+    bool ok = true;
+    for (int tl = 0; tl < n_t; ++tl) {
+      const int s = (n_ka + tl) % NS;
+      const uint32_t par = (uint32_t)(tl / NS) & 1u;
+      if (ok && !*failed) {
+        ok = mbar_wait(bar_full_t(s), par) && mbar_wait(bar_p(s), par);
+        if (!ok) *failed = 1;
+      }
+      if (ok && !*failed) {
+        const uint8_t* st = stage(s);
+        const int nV = min(bV[tl + 1] - bV[tl], R);
+        const uint8_t* cd = st + P.o_cdv;
+        const uint8_t* pf = st + P.o_pfb;
+        for (int grp = 0; grp * 16 < nV; ++grp) {
+          const int n = lane >> 1, hh = lane & 1;
+          const int sl = grp * 16 + n;
+          uint32_t x = 0;
+          if (sl < nV) x = *reinterpret_cast<const uint32_t*>(cd + (size_t)sl * 32 + 8 * vw + 4 * hh);
+          uint4 v0, v1;
+          {
+            const uint32_t lo = x & 0xFFFFu, y = lo | (lo << 14);  // code 2m at bit 4m, code 2m+1 at 4m + 16
+            v0 = make_uint4(codes2_to_h2(y), codes2_to_h2(y >> 4), codes2_to_h2(y >> 8), codes2_to_h2(y >> 12));
+            const uint32_t hi = x >> 16, z = hi | (hi << 14);
+            v1 = make_uint4(codes2_to_h2(z), codes2_to_h2(z >> 4), codes2_to_h2(z >> 8), codes2_to_h2(z >> 12));
+          }
+          *reinterpret_cast<uint4*>(ew + n * ROWE + hh * 32) = v0;
+          *reinterpret_cast<uint4*>(ew + n * ROWE + hh * 32 + 16) = v1;
+          __syncwarp();
+          const uint4 a = *reinterpret_cast<const uint4*>(pf + grp * 512 + lane * 16);
+          const int mi = lane >> 3, ri = lane & 7;
+#pragma unroll
+          for (int half = 0; half < 2; ++half) {
+            uint32_t b00, b01, b10, b11;
+            ldsm_x4_trans(smem_u32(ew + ((mi & 1) * 8 + ri) * ROWE + half * 32 + (mi >> 1) * 16), b00, b01, b10, b11);
+            mma_f16(accV[2 * half], a, b00, b01);
+            mma_f16(accV[2 * half + 1], a, b10, b11);
+          }
+          __syncwarp();
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cnt(bar_empty(s), NTW / NVR);
+    }
+    // rows r8 (high parts) + r8 + 8 (low parts); overflow slots were added by the token warps,
+    // which zeroed the accumulator in phase 0
+    named_sync(3, NTW * 32 + NVR * 32);
+    if (r8 < G) {
+#pragma unroll
+      for (int nb = 0; nb < 4; ++nb) {
+        const int col = 32 * vw + 8 * nb + 2 * c4;
+        accs[r8 * 128 + col] += accV[nb][0] + accV[nb][2];
+        accs[r8 * 128 + col + 1] += accV[nb][1] + accV[nb][3];
+      }
+    }
+    cluster_wait();  // B1
+    cluster_arrive();
+    cluster_wait();  // B2
+    cluster_arrive();
+    cluster_wait();  // B3
+    cluster_arrive();
+    cluster_wait();  // B4
+    return;
+  }
+
+  // =========================== token warps =======================================
   const int b = u / P.n_kv_heads, h = u % P.n_kv_heads;
   const size_t qrow0 = ((size_t)b * P.n_q_heads + (size_t)h * G) * 128;
-  const int c4 = lane & 3, r8 = lane >> 2;
 
   // ---- phase 0: query rows, rotated query, tensor-core fragments ----
-  for (int e = tid; e < G * 128; e += NCT) {
+  for (int e = tid; e < G * 128; e += NTT) {
     const int j = e & 127;
     const float x = __bfloat162float(P.q[qrow0 + e]);
-    qs[e] = x;
     const unsigned long long sb = j < 64 ? P.sign_lo : P.sign_hi;
     qp[e] = (P.rotate && ((sb >> (j & 63)) & 1ull)) ? -x : x;
+    accs[e] = 0.f;
   }
-  for (int e = a0 * G + tid; e < a1 * G; e += NCT) SA[e] = 0.f;
-  if (P.rotate) cw_wht_rows(qp, G);
-  else cw_sync();
+  for (int e = a0 * G + tid; e < a1 * G; e += NTT) SA[e] = 0.f;
+  for (int s = 0; s < NS; ++s)
+    for (int e = tid; e < ((R + 15) / 16) * 128; e += NTT)
+      reinterpret_cast<uint32_t*>(stage(s) + P.o_pfb)[e] = 0u;
+  if (P.rotate) tw_wht_rows(qp, G);
+  else tw_sync();
   {
     const float f = P.rotate ? P.scale_log2 * (1.0f / 128.0f) : P.scale_log2;
-    for (int e = tid; e < G * 128; e += NCT) qp[e] *= f;
+    for (int e = tid; e < G * 128; e += NTT) qp[e] *= f;
   }
-  cw_sync();
+  tw_sync();
   if (warp < G) {
     float s = 0.f;
     for (int j = lane; j < 128; j += 32) s += qp[warp * 128 + j];
@@ -433,7 +591,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     if (lane == 0) sq[warp] = s;
   }
   {
-    // fragment (k-step ks, lane ln): one per compute thread (8 k-steps x 32 lanes)
+    // fragment (k-step ks, lane ln): one per token thread (8 k-steps x 32 lanes)
     const int ks = tid >> 5, ln = tid & 31, g = ln >> 2, c = ln & 3;
     uint2 fa = make_uint2(0u, 0u);
     uint4 fk = make_uint4(0u, 0u, 0u, 0u);
@@ -456,24 +614,24 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     qfa[ks * 32 + ln] = fa;
     qfk[ks * 32 + ln] = fk;
   }
-  for (int e = tid; e < ((P.R + 15) / 16) * 128; e += NCT) reinterpret_cast<uint32_t*>(pfrag)[e] = 0u;
-  cw_sync();
+  tw_sync();
+  named_arrive(2, NTW * 32 + NKR * 32);  // the key-residual warps may read q' fragments and sq
+  named_arrive(3, NTW * 32 + NVR * 32);  // the value-residual warps may add into accs
 
-  int it = 0;
   bool ok = true;
   auto wait_item = [&](int i) -> const uint8_t* {
     const int s = i % NS;
-    if (ok && !*failed) ok = mbar_wait(smem_u32(bars + s), (uint32_t)(i / NS) & 1u);
+    if (ok && !*failed) ok = mbar_wait(is_tile(i) ? bar_full_t(s) : bar_full_c(s), item_phase(i) & 1u);
     if (!ok) *failed = 1;
-    return ring + (size_t)s * P.stage_bytes;
+    return stage(s);
   };
-  auto release_item = [&](int i) {
+  auto release_chunk = [&](int i) {
     __syncwarp();
-    if (lane == 0) mbar_arrive(smem_u32(bars + NS + (i % NS)));
+    if (lane == 0) mbar_arrive(bar_empty(i % NS));
   };
 
   // ---- phase 1: anchor scores of this CTA's slice (bf16 tensor cores) ----
-  for (; it < n_ka; ++it) {
+  for (int it = 0; it < n_ka; ++it) {
     const uint8_t* st = wait_item(it);
     if (!*failed) {
       const int r0 = a0 + it * ROWS, nr = min(a1 - r0, ROWS);
@@ -495,295 +653,219 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         if (gc + 1 < G) atomicAdd(&SA[(r0 + ra + 8) * G + gc + 1], d[3] * P.scale_log2);
       }
     }
-    release_item(it);
+    release_chunk(it);
   }
-  cw_sync();
+  tw_sync();
   cluster_arrive();  // B1
   cluster_wait();
-  for (int r = 0; r < C; ++r) {
-    if (r == rank) continue;
-    const int b0r = min(k, r * a_per), b1r = min(k, b0r + a_per);
-    const float* rem = cluster.map_shared_rank(SA, r);
-    for (int e = b0r * G + tid; e < b1r * G; e += NCT) SA[e] = rem[e];
+  // every entry outside this CTA's slice comes from the peer that owns its anchor
+#pragma unroll 4
+  for (int e = tid; e < k * G; e += NTT) {
+    const int r = (e / G) / a_per;
+    if (r != rank) SA[e] = cluster.map_shared_rank(SA, r)[e];
   }
-  for (int e = tid; e < k * G; e += NCT) Wt[e] = 0.f;
-  cw_sync();
-
-  // ---- phase 2: position tiles ----
-  float accV[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-  float m_run[G], l_part[G], pmin[G];
+  for (int e = tid; e < G * max_k; e += NTT) Wt[e] = 0.f;  // [G][max_k]: the scatter spreads over banks
+  tw_sync();
+  // Reference for the exponentials: the largest anchor score per query row.  Anchors are
+  // tokens of the unit, so it never exceeds the true maximum logit; every CTA of the
+  // cluster holds the same table and so the same reference, which makes the cluster
+  // combine a plain sum.
+  {
+    float mx[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) mx[g] = -INFINITY;
+    for (int a = tid; a < k; a += NTT)
+#pragma unroll
+      for (int g = 0; g < G; ++g) mx[g] = fmaxf(mx[g], SA[a * G + g]);
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const float m = warp_max(mx[g]);
+      if (lane == 0) red[warp * G + g] = m;
+    }
+    tw_sync();
+    if (tid < G) {
+      float m = red[tid];
+      for (int w = 1; w < NTW; ++w) m = fmaxf(m, red[w * G + tid]);
+      mref[tid] = m;
+    }
+    tw_sync();
+  }
+  float m_ref[G], l_part[G], pmin[G];
 #pragma unroll
   for (int g = 0; g < G; ++g) {
-    m_run[g] = -1e30f;
+    m_ref[g] = mref[g];
     l_part[g] = 0.f;
     pmin[g] = 0.f;
   }
-  const int R = P.R;
-  uint8_t* ew = ebuf + warp * 16 * ROWE;
-  for (int tl = 0; tl < n_t; ++tl, ++it) {
+
+  // ---- phase 2: position tiles ----
+  bool overflow_risk = false;
+  for (int tl = 0; tl < n_t; ++tl) {
+    const int it = n_ka + tl;
+    const int s = it % NS;
     const uint8_t* st = wait_item(it);
-    if (*failed) {
-      release_item(it);
-      continue;
+    if (ok && !*failed) {
+      ok = mbar_wait(bar_rs(s), item_phase(it) & 1u);
+      if (!ok) *failed = 1;
     }
-    const int t0 = p0 + tl * T, te = min(t0 + T, p1);
-    const int skl = bK[tl], skh = bK[tl + 1], svl = bV[tl], svh = bV[tl + 1];
-    const int i0 = t0 + PPT * tid;
-    float lg[PPT][G];
-    int slotK[PPT], slotV[PPT];
-    const uint2 ek = *reinterpret_cast<const uint2*>(st + ST_K + 8 * tid);
-    const uint2 ev = *reinterpret_cast<const uint2*>(st + ST_V + 8 * tid);
-    const int wi = (PPT * tid) >> 6, bit0 = (PPT * tid) & 63;
-    const uint64_t wk = reinterpret_cast<const uint64_t*>(st + ST_BMK)[wi];
-    const uint64_t wv = reinterpret_cast<const uint64_t*>(st + ST_BMV)[wi];
-    const int pk = (int)reinterpret_cast<const uint32_t*>(st + ST_PFK)[wi] - skl;
-    const int pv = (int)reinterpret_cast<const uint32_t*>(st + ST_PFV)[wi] - svl;
+    if (!*failed) {
+      const int t0 = p0 + tl * T, te = min(t0 + T, p1);
+      const int skl = bK[tl], svl = bV[tl];
+      const int i0 = t0 + PPT * tid;
+      const float* rsb = reinterpret_cast<const float*>(st + P.o_rsb);
+      uint8_t* pfb = const_cast<uint8_t*>(st) + P.o_pfb;
+      const uint32_t* scv = reinterpret_cast<const uint32_t*>(st + P.o_scv) + (svl & 3);
+      const uint2 ek = *reinterpret_cast<const uint2*>(st + ST_K + 8 * tid);
+      const uint2 ev = *reinterpret_cast<const uint2*>(st + ST_V + 8 * tid);
+      const int wi = (PPT * tid) >> 6, bit0 = (PPT * tid) & 63;
+      const uint64_t wk = reinterpret_cast<const uint64_t*>(st + ST_BMK)[wi];
+      const uint64_t wv = reinterpret_cast<const uint64_t*>(st + ST_BMV)[wi];
+      const int pk = (int)reinterpret_cast<const uint32_t*>(st + ST_PFK)[wi] - skl;
+      const int pv = (int)reinterpret_cast<const uint32_t*>(st + ST_PFV)[wi] - svl;
 #pragma unroll
-    for (int pp = 0; pp < PPT; ++pp) {
-      const int i = i0 + pp;
-      const int bit = bit0 + pp;
-      const uint64_t below = (1ull << bit) - 1ull;
-      slotK[pp] = (i < te && ((wk >> bit) & 1ull)) ? pk + __popcll(wk & below) : -1;
-      slotV[pp] = (i < te && ((wv >> bit) & 1ull)) ? pv + __popcll(wv & below) : -1;
-      if (i < te) {
-        const uint32_t e = pp ? ek.y : ek.x;
-        const int a = min((int)(e & 0xFFFFu), k - 1);  // indices are < k by construction; never read past the table
-        const float gam = half_hi(e);
-        if constexpr (G % 4 == 0) {
+      for (int pp = 0; pp < PPT; ++pp) {
+        const int i = i0 + pp;
+        if (i >= te) continue;
+        const int bit = bit0 + pp;
+        const uint64_t below = (1ull << bit) - 1ull;
+        float lg[G];
+        {
+          const uint32_t e = pp ? ek.y : ek.x;
+          const int a = min((int)(e & 0xFFFFu), k - 1);  // indices are < k by construction; never read past the table
+          const float gam = half_hi(e);
+          if constexpr (G % 4 == 0) {
 #pragma unroll
-          for (int g4 = 0; g4 < G; g4 += 4) {
-            const float4 s4 = *reinterpret_cast<const float4*>(SA + a * G + g4);
-            lg[pp][g4] = gam * s4.x;
-            lg[pp][g4 + 1] = gam * s4.y;
-            lg[pp][g4 + 2] = gam * s4.z;
-            lg[pp][g4 + 3] = gam * s4.w;
+            for (int g4 = 0; g4 < G; g4 += 4) {
+              const float4 s4 = *reinterpret_cast<const float4*>(SA + a * G + g4);
+              lg[g4] = gam * s4.x;
+              lg[g4 + 1] = gam * s4.y;
+              lg[g4 + 2] = gam * s4.z;
+              lg[g4 + 3] = gam * s4.w;
+            }
+          } else {
+#pragma unroll
+            for (int g = 0; g < G; ++g) lg[g] = gam * SA[a * G + g];
           }
-        } else {
-#pragma unroll
-          for (int g = 0; g < G; ++g) lg[pp][g] = gam * SA[a * G + g];
         }
-      } else {
+        if ((wk >> bit) & 1ull) {  // key residual term
+          const int sl = pk + __popcll(wk & below);
+          if (sl < R) {
 #pragma unroll
-        for (int g = 0; g < G; ++g) lg[pp][g] = -INFINITY;
-      }
-    }
-    // key residual terms on tensor cores, in rounds of at most R slots (rounds after the
-    // first read their records from global memory)
-    const int nK = skh - skl;
-    for (int r0 = 0; r0 < nK; r0 += R) {
-      const int nr = min(R, nK - r0);
-      const uint8_t* cd = r0 == 0 ? st + P.o_cdk : U.cdK + (size_t)(skl + r0) * 32;
-      const uint32_t* sc = r0 == 0 ? reinterpret_cast<const uint32_t*>(st + P.o_sck) + (skl & 3) : U.scK + skl + r0;
-      for (int g8 = warp; g8 * 8 < nr; g8 += NCW) {
-        const int sl = g8 * 8 + r8;  // the slot whose codes this lane feeds (B column r8)
-        uint4 w0 = make_uint4(0u, 0u, 0u, 0u), w1 = w0;
-        if (sl < nr) {
-          w0 = *reinterpret_cast<const uint4*>(cd + (size_t)sl * 32);
-          w1 = *reinterpret_cast<const uint4*>(cd + (size_t)sl * 32 + 16);
+            for (int g = 0; g < G; ++g) lg[g] += rsb[sl * G + g];
+          } else {  // beyond the staged slots (a locally dense tile): from global memory, on CUDA cores
+            const int gs = skl + sl;
+            const uint8_t* rec = U.cdK + (size_t)gs * 32;
+            const uint32_t smn = U.scK[gs];
+#pragma unroll
+            for (int g = 0; g < G; ++g) {
+              float dot = 0.f;
+              for (int bb = 0; bb < 32; ++bb) {
+                const uint32_t byte = rec[bb];
+#pragma unroll
+                for (int c = 0; c < 4; ++c) dot += qp[g * 128 + 4 * bb + c] * (float)((byte >> (2 * c)) & 3u);
+              }
+              lg[g] += half_hi(smn) * sq[g] + half_lo(smn) * dot;
+            }
+          }
         }
-        const uint32_t wd[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
-        float d[4] = {0.f, 0.f, 0.f, 0.f};
+        const uint32_t e = pp ? ev.y : ev.x;
+        const int a = min((int)(e & 0xFFFFu), k - 1);
+        const float gam = half_hi(e);
+        float p[G];
 #pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-          const uint32_t x = wd[ks] >> (4 * c4);
-          mma_f16(d, qfk[ks * 32 + lane], codes2_to_h2(x), codes2_to_h2(x >> 2));
+        for (int g = 0; g < G; ++g) {
+          const float x = lg[g] - m_ref[g];
+          overflow_risk |= x > 120.f;
+          p[g] = exp2f(x);
+          l_part[g] += p[g];
+          red_add(&Wt[g * max_k + a], p[g] * gam);
         }
-        if (r8 < G) {  // D rows r8 (high parts) and r8 + 8 (low parts), columns 2c, 2c+1
+        if ((wv >> bit) & 1ull) {  // value residual: A operand of its 16-slot group, or overflow
+          const int sl = pv + __popcll(wv & below);
+          if (sl < R) {
+            const uint32_t smn = scv[sl];
+            const float scl = half_lo(smn), mn = half_hi(smn);
+            const int grp = sl >> 4, kk = sl & 15;
+            const int comp = (kk >> 3) * 2, hf = kk & 1, cc = (kk & 7) >> 1;
 #pragma unroll
-          for (int e2 = 0; e2 < 2; ++e2) {
-            const int sl2 = g8 * 8 + 2 * c4 + e2;
-            if (sl2 < nr) {
-              const uint32_t smn = sc[sl2];
-              rs[sl2 * G + r8] = half_hi(smn) * sq[r8] + half_lo(smn) * (d[e2] + d[2 + e2]);
+            for (int g = 0; g < G; ++g) {
+              const float x = p[g] * scl;
+              const __half hi = __float2half_rn(x);
+              const __half lo = __float2half_rn(x - __half2float(hi));
+              unsigned short* dst = reinterpret_cast<unsigned short*>(pfb + grp * 512 + (4 * g + cc) * 16);
+              dst[comp * 2 + hf] = __half_as_ushort(hi);
+              dst[(comp + 1) * 2 + hf] = __half_as_ushort(lo);
+              pmin[g] += p[g] * mn;
+            }
+          } else {
+            const int gs = svl + sl;
+            const uint8_t* rec = U.cdV + (size_t)gs * 32;
+            const uint32_t smn = U.scV[gs];
+            const float scl = half_lo(smn), mn = half_hi(smn);
+#pragma unroll
+            for (int g = 0; g < G; ++g) {
+              pmin[g] += p[g] * mn;
+              const float ps = p[g] * scl;
+              for (int bb = 0; bb < 32; ++bb) {
+                const uint32_t byte = rec[bb];
+#pragma unroll
+                for (int c = 0; c < 4; ++c) atomicAdd(&accs[g * 128 + 4 * bb + c], ps * (float)((byte >> (2 * c)) & 3u));
+              }
             }
           }
         }
       }
-      cw_sync();
-#pragma unroll
-      for (int pp = 0; pp < PPT; ++pp) {
-        const int sl = slotK[pp] - r0;
-        if (sl >= 0 && sl < nr) {
-#pragma unroll
-          for (int g = 0; g < G; ++g) lg[pp][g] += rs[sl * G + g];
-        }
-      }
-      if (r0 + R < nK) cw_sync();
     }
-    // running max over the tile
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      float mx = lg[0][g];
-#pragma unroll
-      for (int pp = 1; pp < PPT; ++pp) mx = fmaxf(mx, lg[pp][g]);
-      mx = warp_max(mx);
-      if (lane == 0) red[warp * G + g] = mx;
-    }
-    cw_sync();
-    bool grow = false;
-    float fac[G];
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      float mx = red[g];
-#pragma unroll
-      for (int w = 1; w < NCW; ++w) mx = fmaxf(mx, red[w * G + g]);
-      const float nm = fmaxf(m_run[g], mx);
-      fac[g] = exp2f(m_run[g] - nm);
-      grow |= nm > m_run[g];
-      m_run[g] = nm;
-    }
-    if (grow) {  // uniform across the compute warps
-      for (int e = tid; e < k * G; e += NCT) Wt[e] *= fac[e % G];
-      float fq = 0.f;
-#pragma unroll
-      for (int g = 0; g < G; ++g) {
-        l_part[g] *= fac[g];
-        pmin[g] *= fac[g];
-        if (g == r8) fq = fac[g];
-      }
-#pragma unroll
-      for (int nb = 0; nb < 2; ++nb)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) accV[nb][e] *= fq;
-      cw_sync();
-    }
-    // probabilities and the value-weight scatter
-#pragma unroll
-    for (int pp = 0; pp < PPT; ++pp) {
-      if (i0 + pp < te) {
-        const uint32_t e = pp ? ev.y : ev.x;
-        const int a = min((int)(e & 0xFFFFu), k - 1);
-        const float gam = half_hi(e);
-#pragma unroll
-        for (int g = 0; g < G; ++g) {
-          const float p = exp2f(lg[pp][g] - m_run[g]);
-          lg[pp][g] = p;
-          l_part[g] += p;
-          atomicAdd(&Wt[a * G + g], p * gam);
-        }
-      }
-    }
-    // value residuals on tensor cores, in rounds of at most R slots
-    const int nV = svh - svl;
-    for (int r0 = 0; r0 < nV; r0 += R) {
-      const int nr = min(R, nV - r0);
-      const uint8_t* cd = r0 == 0 ? st + P.o_cdv : U.cdV + (size_t)(svl + r0) * 32;
-      const uint32_t* sc = r0 == 0 ? reinterpret_cast<const uint32_t*>(st + P.o_scv) + (svl & 3) : U.scV + svl + r0;
-      // A operand of each group of 16 slots: rows g = (p * scale) high parts, rows g + 8 = low parts
-#pragma unroll
-      for (int pp = 0; pp < PPT; ++pp) {
-        const int sl = slotV[pp] - r0;
-        if (sl >= 0 && sl < nr) {
-          const uint32_t smn = sc[sl];
-          const float scl = half_lo(smn), mn = half_hi(smn);
-          const int grp = sl >> 4, kk = sl & 15;
-          const int comp = (kk >> 3) * 2, hf = kk & 1, cc = (kk & 7) >> 1;
-#pragma unroll
-          for (int g = 0; g < G; ++g) {
-            const float x = lg[pp][g] * scl;
-            const __half hi = __float2half_rn(x);
-            const __half lo = __float2half_rn(x - __half2float(hi));
-            unsigned short* dst = reinterpret_cast<unsigned short*>(pfrag + grp * 512 + (4 * g + cc) * 16);
-            dst[comp * 2 + hf] = __half_as_ushort(hi);
-            dst[(comp + 1) * 2 + hf] = __half_as_ushort(lo);
-            pmin[g] += lg[pp][g] * mn;
-          }
-        }
-      }
-      cw_sync();
-      // each warp owns the 16 coordinates 16w .. 16w + 15 for every group
-      const int ngrp = (nr + 15) >> 4;
-      for (int grp = 0; grp < ngrp; ++grp) {
-        const int n = lane >> 1, hh = lane & 1;
-        const int sl = grp * 16 + n;
-        uint32_t x = 0;
-        if (sl < nr) x = *reinterpret_cast<const unsigned short*>(cd + (size_t)sl * 32 + 4 * warp + 2 * hh);
-        const uint32_t y = x | (x << 14);  // code 2k at bit 4k, code 2k+1 at bit 4k+16
-        uint4 v;
-        v.x = codes2_to_h2(y);
-        v.y = codes2_to_h2(y >> 4);
-        v.z = codes2_to_h2(y >> 8);
-        v.w = codes2_to_h2(y >> 12);
-        *reinterpret_cast<uint4*>(ew + n * ROWE + hh * 16) = v;
-        __syncwarp();
-        uint32_t b00, b01, b10, b11;
-        const int mi = lane >> 3, ri = lane & 7;
-        ldsm_x4_trans(smem_u32(ew + ((mi & 1) * 8 + ri) * ROWE + (mi >> 1) * 16), b00, b01, b10, b11);
-        const uint4 a = *reinterpret_cast<const uint4*>(pfrag + grp * 512 + lane * 16);
-        mma_f16(accV[0], a, b00, b01);
-        mma_f16(accV[1], a, b10, b11);
-        __syncwarp();
-      }
-      if (r0 + R < nV) cw_sync();
-    }
-    release_item(it);
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar_p(s));
   }
+  if (overflow_risk) *failed = 1;  // a logit beyond 2^120 of the reference would overflow the sums
 
   // ---- per-CTA totals ----
 #pragma unroll
   for (int g = 0; g < G; ++g) {
-    const float s = warp_sum(l_part[g]);
+    const float sl = warp_sum(l_part[g]);
     const float pm = warp_sum(pmin[g]);
     if (lane == 0) {
-      red[warp * G + g] = s;
+      red[warp * G + g] = sl;
       opart[warp * G + g] = pm;  // scratch until phase 3
     }
   }
-  cw_sync();
+  tw_sync();
   if (tid < G) {
-    float s = 0.f, pm = 0.f;
-    for (int w = 0; w < NCW; ++w) {
-      s += red[w * G + tid];
+    float sl = 0.f, pm = 0.f;
+    for (int w = 0; w < NTW; ++w) {
+      sl += red[w * G + tid];
       pm += opart[w * G + tid];
     }
-    cl[tid] = s;
-#pragma unroll
-    for (int g = 0; g < G; ++g)
-      if (g == tid) cm[tid] = m_run[g];
-    peer_l[tid] = pm;  // scratch: this CTA's sum of p * min per row
+    cl[tid] = sl;
+    pms[tid] = pm;
   }
-  cw_sync();
-  if (r8 < G) {  // rotated-domain residual accumulator: high + low rows, plus sum p * min on every coordinate
-#pragma unroll
-    for (int nb = 0; nb < 2; ++nb) {
-      const int col = 16 * warp + 8 * nb + 2 * c4;
-      accs[r8 * 128 + col] = accV[nb][0] + accV[nb][2] + peer_l[r8];
-      accs[r8 * 128 + col + 1] = accV[nb][1] + accV[nb][3] + peer_l[r8];
-    }
-  }
-  cw_sync();
+  tw_sync();
 
-  // ---- phase 3: combine across the cluster ----
+  // ---- phase 3: combine across the cluster (one common reference: plain sums) ----
   cluster_arrive();  // B2
   cluster_wait();
-  if (tid < C * G) {
-    const int r = tid / G, g = tid % G;
-    peer_m[tid] = cluster.map_shared_rank(cm, r)[g];
-    peer_l[tid] = cluster.map_shared_rank(cl, r)[g];
-  }
-  cw_sync();
   if (tid < G) {
-    float M = -1e30f;
-    for (int r = 0; r < C; ++r) M = fmaxf(M, peer_m[r * G + tid]);
     float Lt = 0.f;
-    for (int r = 0; r < C; ++r) {
-      const float f = exp2f(peer_m[r * G + tid] - M);
-      facs[r * G + tid] = f;
-      Lt += f * peer_l[r * G + tid];
-    }
+    for (int r = 0; r < C; ++r) Lt += cluster.map_shared_rank(cl, r)[tid];
     ltot[tid] = Lt;
   }
-  cw_sync();
-  for (int e = a0 * G + tid; e < a1 * G; e += NCT) {
-    const int g = e % G;
-    float s = 0.f;
-    for (int r = 0; r < C; ++r) s += facs[r * G + g] * cluster.map_shared_rank(Wt, r)[e];
-    Wt[e] = s;
+  for (int e = tid; e < (a1 - a0) * G; e += NTT) {
+    const int idx = (e / (a1 - a0)) * max_k + a0 + e % (a1 - a0);
+    float v[kMaxCluster];
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r) v[r] = r < C ? cluster.map_shared_rank(Wt, r)[idx] : 0.f;
+    float sw = 0.f;
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r) sw += v[r];
+    Wt[idx] = sw;
   }
-  cw_sync();
+  tw_sync();
   // reduced weights of the slice times its anchor values (bf16 tensor cores, weights as hi + lo)
   float oacc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-  for (int ci = 0; ci < n_ka; ++ci, ++it) {
+  for (int ci = 0; ci < n_ka; ++ci) {
+    const int it = n_ka + n_t + ci;
     const uint8_t* st = wait_item(it);
     if (!*failed) {
       const int r0 = a0 + ci * ROWS, nr = min(a1 - r0, ROWS);
@@ -806,7 +888,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
           __nv_bfloat16 hi[4], lo[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            const float w = kk[e] < nr ? Wt[(r0 + kk[e]) * G + r8] : 0.f;
+            const float w = kk[e] < nr ? Wt[r8 * max_k + r0 + kk[e]] : 0.f;
             hi[e] = __float2bfloat16_rn(w);
             lo[e] = __float2bfloat16_rn(w - __bfloat162float(hi[e]));
           }
@@ -819,13 +901,14 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         mma_bf16(oacc[1], ah0, al0, ah2, al2, b10, b11);
       }
     }
-    release_item(it);
+    release_chunk(it);
   }
-  // this CTA's value residuals: its own rescale factor, then the inverse rotation once
-  for (int e = tid; e < G * 128; e += NCT) accs[e] *= facs[rank * G + (e >> 7)];
-  if (P.rotate) cw_wht_rows(accs, G);
-  else cw_sync();
-  for (int e = tid; e < G * 128; e += NCT) {
+  // this CTA's value residuals (staged slots from the value-residual warps, overflow slots and
+  // sum p * min from the token warps), then the inverse rotation once
+  for (int e = tid; e < G * 128; e += NTT) accs[e] += pms[e >> 7];
+  if (P.rotate) tw_wht_rows(accs, G);
+  else tw_sync();
+  for (int e = tid; e < G * 128; e += NTT) {
     const int j = e & 127;
     float r = accs[e];
     if (P.rotate) {
@@ -835,7 +918,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     }
     opart[e] = r;
   }
-  cw_sync();
+  tw_sync();
   if (r8 < G) {
 #pragma unroll
     for (int nb = 0; nb < 2; ++nb) {
@@ -844,7 +927,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       opart[r8 * 128 + col + 1] += oacc[nb][1] + oacc[nb][3];
     }
   }
-  cw_sync();
+  tw_sync();
   cluster_arrive();  // B3
   cluster_wait();
   {
@@ -853,10 +936,14 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     const int e0 = rank * per, e1 = min(E, e0 + per);
     bool bad = false;
     for (int r = 0; r < C; ++r) bad |= cluster.map_shared_rank(const_cast<int*>(failed), r)[0] != 0;
-    for (int e = e0 + tid; e < e1; e += NCT) {
-      float s = 0.f;
-      for (int r = 0; r < C; ++r) s += cluster.map_shared_rank(opart, r)[e];
-      const float y = bad ? __int_as_float(0x7FC00000) : s / ltot[e >> 7];
+    for (int e = e0 + tid; e < e1; e += NTT) {
+      float v[kMaxCluster];
+#pragma unroll
+      for (int r = 0; r < kMaxCluster; ++r) v[r] = r < C ? cluster.map_shared_rank(opart, r)[e] : 0.f;
+      float sum = 0.f;
+#pragma unroll
+      for (int r = 0; r < kMaxCluster; ++r) sum += v[r];
+      const float y = bad ? __int_as_float(0x7FC00000) : sum / ltot[e >> 7];
       const size_t o = qrow0 + e;
       P.out[o] = __float2bfloat16_rn(y);
       if (P.out_f32) P.out_f32[o] = y;
@@ -908,7 +995,7 @@ bool make_plan(const Layout& L, int G, int C, int smem_optin, Plan* out, std::st
   Plan pl;
   DecodeParams& P = pl.P;
   // residual slots staged per tile and side: 1.35x the densest unit's mean plus slack;
-  // a denser tile processes its extra slots from global memory in further rounds
+  // slots of a locally denser tile beyond these are taken from global memory by the token warps
   int R = (int)(T * max_density(L) * 1.35) + 24;
   R = std::min(T, std::max(16, (R + 15) & ~15));
   const int chunk = ((L.max_len + C - 1) / C + T - 1) / T * T;
@@ -926,21 +1013,21 @@ bool make_plan(const Layout& L, int G, int C, int smem_optin, Plan* out, std::st
   P.o_bv = take((size_t)(max_tiles + 1) * 4);
   P.o_qfa = take(8 * 32 * 8);
   P.o_qfk = take(8 * 32 * 16);
-  P.o_qs = take((size_t)G * 128 * 4);
   P.o_qp = take((size_t)G * 128 * 4);
-  P.o_rs = take((size_t)R * G * 4);
-  P.o_pf = take((size_t)((R + 15) / 16) * 512);
-  P.o_e = take((size_t)NCW * 16 * ROWE);
   P.o_acc = take((size_t)G * 128 * 4);
-  P.o_opart = take((size_t)std::max(G * 128, NCW * G) * 4);
-  P.o_misc = take((size_t)(NCW * G + 4 * G + 3 * kMaxCluster * G + 4) * 4);
-  P.o_bar = take(2 * 8 * 8);
+  P.o_opart = take((size_t)std::max(G * 128, NTW * G) * 4);
+  P.o_e = take((size_t)NVR * 16 * ROWE);
+  P.o_misc = take((size_t)(NTW * G + 6 * G + 4) * 4);
+  P.o_bar = take(5 * 8 * 8);
+  // a stage: streams, bitmaps and prefix words, staged records, then (beyond the footprint
+  // of an anchor chunk, so chunk copies never touch them) residual terms and value operands
   P.o_cdk = (int)align128(ST_REC);
   P.o_sck = (int)align128(P.o_cdk + R * 32);
   P.o_cdv = (int)align128(P.o_sck + (R + 8) * 4);
   P.o_scv = (int)align128(P.o_cdv + R * 32);
-  int stage = (int)align128(P.o_scv + (R + 8) * 4);
-  stage = std::max(stage, (int)align128(ROWS * ROWB));
+  P.o_rsb = (int)align128(std::max(P.o_scv + (R + 8) * 4, ROWS * ROWB));
+  P.o_pfb = (int)align128(P.o_rsb + R * G * 4);
+  const int stage = (int)align128(P.o_pfb + ((R + 15) / 16) * 512);
   P.o_ring = (int)off;
   const long long room = (long long)smem_optin - (long long)off;
   if (room < 2LL * stage) {
@@ -953,7 +1040,6 @@ bool make_plan(const Layout& L, int G, int C, int smem_optin, Plan* out, std::st
   P.stage_bytes = stage;
   P.R = R;
   P.max_tiles = max_tiles;
-  P.pf_items = NS + 6;
   pl.smem = (size_t)P.o_ring + (size_t)NS * stage;
   pl.C = C;
   *out = pl;
@@ -1012,7 +1098,8 @@ int plan_for(const Layout& L, const LaunchKey& key, Plan* out, std::string* why)
     cfg.numAttrs = 1;
     int nclusters = 0;
     e = cudaOccupancyMaxActiveClusters(&nclusters, akv_decode_kernel<G>, &cfg);
-    if (e == cudaSuccess && nclusters >= 1) break;
+    // prefer a size whose clusters all fit at once; an explicit override only needs one to fit
+    if (e == cudaSuccess && (nclusters >= key.units || (key.cluster_env == C && nclusters >= 1))) break;
     cudaGetLastError();
     C = (C & (C - 1)) ? C - 1 : C / 2;
   }

@@ -120,3 +120,15 @@ def test_ragged_sweep_points(dev):
     for fa, fr in ((0.01, 0.0), (0.04, 0.2), (0.02, 0.1)):
         p = akv.Params(batch=16, n_kv_heads=8, n_q_heads=32, anchor_frac=fa, res_frac_k=fr, res_frac_v=fr)
         _run_seeded(dev, p, lens, seed=int(fa * 1000 + fr * 100))
+
+
+def test_locally_dense_residuals_exceed_staging(dev):
+    """All residual slots packed into a few tiles: those tiles hold far more slots than the
+    kernel stages per tile (sized from the mean density), so the overflow paths run."""
+    def mutate(u, d):
+        non = np.setdiff1d(np.arange(d["S"]), d["anchor_pos"])
+        d["res_k"] = np.sort(non[: d["nk"]]).astype(np.int32)
+        d["res_v"] = np.sort(non[len(non) - d["nv"]:]).astype(np.int32)
+    for G in (1, 4, 8):
+        p = akv.Params(batch=2, n_kv_heads=2, n_q_heads=2 * G, seed=31)
+        _run_seeded(dev, p, [6000, 3000], mutate=mutate)
