@@ -53,9 +53,10 @@ typedef enum akv_status {
 
 #define AKV_HEAD_DIM 128
 #define AKV_FLAG_ROTATE 1u /* residuals carry the randomized Hadamard rotation (Appendix A.1, Eq. 12) */
-#define AKV_ARENA_MAGIC 0x31564B41u /* "AKV1" */
-#define AKV_ARENA_VERSION 1u
+#define AKV_ARENA_MAGIC 0x32564B41u /* "AKV2" */
+#define AKV_ARENA_VERSION 2u
 #define AKV_MAX_ANCHORS 65535 /* anchor indices are uint16 (Table 1, b_a = 2) */
+#define AKV_TILE_TOKENS 1024  /* tokens per tile block of the packed token stream */
 
 /*
  * Compression parameters of one layer (Section 3.2 "Anchor selection",
@@ -101,48 +102,68 @@ typedef struct akv_arena_header {
   int32_t max_len; /* max_b S_b */
   uint64_t desc_offset; /* = 256 */
   uint64_t sign_bits[2]; /* bit j of the 128-bit word: s_j = -1 when set (rotation signs) */
-  uint8_t pad[256 - 8 - 8 - sizeof(akv_params) - 8 - 8 - 16];
+  int32_t tile_tokens;   /* AKV_TILE_TOKENS */
+  int32_t reserved1;
+  uint8_t pad[256 - 8 - 8 - sizeof(akv_params) - 8 - 8 - 16 - 8];
 } akv_arena_header;
 
 /*
- * Per-unit descriptor (256 bytes).  Offsets are bytes from the arena base;
- * every section starts on a 128-byte boundary.  Sections, in order:
+ * Per-unit descriptor (256 bytes).  Offsets are bytes from the arena base.
  *
- *   anchor_k   [k][128] bf16   anchor keys, slots in ascending position   (Table 1: anchor keys)
- *   anchor_v   [k][128] bf16   anchor values                              (Table 1: anchor values)
- *   anchor_pos [k] int32       anchor positions (not read by decode)
- *   stream_k   [S] uint32      per position: anchor slot a(i) in bits 0-15,
- *                              fp16 gamma_i in bits 16-31 (Eq. 1, Eq. 2);
- *                              an anchor stores (own slot, 1.0)
- *   stream_v   [S] uint32      same for values
- *   bitmap_k   [ceil(S/64)] uint64   bit i%64 of word i/64 set <=> i in R_K
- *   prefix_k   [ceil(S/64)] uint32   exclusive popcount of bitmap_k words
- *   bitmap_v, prefix_v                same for values
- *   codes_k    [N_K][32] uint8  2-bit codes of the rotated residual, code j in
- *                              byte j/4 bits 2(j%4)..2(j%4)+1; slots in position order
- *   scales_k   [N_K] uint32     fp16 scale in bits 0-15, fp16 min in bits 16-31
- *   codes_v, scales_v           same for values
+ * Token order.  The S tokens of a unit (anchors included) are stored sorted
+ * by their VALUE anchor slot, ties by position: the stored order is the
+ * stable sort of positions by a_V(i).  Attention over all S positions with
+ * no mask (Eq. 4) does not depend on the order of its terms, and in this
+ * order every anchor's value weight w[a] = sum p_i gamma_i (Eq. 3) is a sum
+ * over one contiguous run.  Positions themselves are not stored (decode never
+ * needs them); anchor_pos keeps the anchors' positions.
  *
- * The slot of a residual position i is prefix[i/64] + popcount(bitmap[i/64] &
- * ((1 << (i%64)) - 1)) (the O(1) position-to-slot lookup of Appendix A.1,
- * "Layout").  Dequantized rotated residual: c^_j = min + code_j * scale; the
- * residual is r~ = s o (H_128 c^) / 128 with H_128 the unnormalised Sylvester
- * Hadamard matrix (or r~ = c^ when AKV_FLAG_ROTATE is off).
+ * Sections, in order (each 128-byte aligned):
+ *   anchor_k   [k][128] bf16  anchor keys, slots in ascending position (Table 1: anchor keys).
+ *                             Row a is stored as 16 chunks of 16 bytes; chunk c (dims
+ *                             8c .. 8c+7) sits at chunk place c XOR (a mod 8), so that a
+ *                             linear copy to shared memory reads back without bank conflicts.
+ *   anchor_v   [k][128] bf16  anchor values, same swizzle
+ *   anchor_pos [k] int32      anchor positions (not read by decode)
+ *   tile_table [n_tiles + 1] uint32  byte offset of tile block j from off_tiles
+ *                             (multiples of 16); entry n_tiles = bytes used
+ *   tiles                     n_tiles = ceil(S / AKV_TILE_TOKENS) tile blocks
+ *
+ * Tile block j holds the stored tokens [j T, min(S, (j+1) T)), T = AKV_TILE_TOKENS:
+ * n tokens, n64 = n rounded up to 64, nw = n64 / 64, nk / nv residual records.
+ *   +0              kst [n64] uint32  key anchor slot a_K in bits 0-15, fp16 gamma^K in
+ *                                     bits 16-31 (Eq. 1, Eq. 2); an anchor stores (own slot,
+ *                                     1.0); entries n .. n64-1 are 0
+ *   +4 n64          vst [n64] uint32  the same for values (a_V non-decreasing over the tile)
+ *   +8 n64          bmk [nw] uint64   bit t%64 of word t/64 set <=> token t has a key residual
+ *   +8 n64 + 8 nw   bmv [nw] uint64   value residuals
+ *   +8 n64 + 16 nw  rkk [nw] uint16   exclusive popcount prefix of bmk words (zero-padded to 16 B)
+ *   then            rkv [nw] uint16   of bmv words (zero-padded to 16 B)
+ *   F = 8 n64 + 16 nw + 2 * round16(2 nw) bytes so far
+ *   +F              smk [nk] uint32   fp16 scale in bits 0-15, fp16 min in bits 16-31 (padded to 16 B)
+ *   then            smv [nv] uint32   (padded to 16 B)
+ *   then            cdk [nk][32] uint8  2-bit codes of the rotated key residual, code j in
+ *                                     byte j/4, bits 2(j%4)..2(j%4)+1
+ *   then            cdv [nv][32] uint8
+ * Record r of a side belongs to the r-th token (in stored order) whose bit is set;
+ * token t's record is rk[t/64] + popcount(bm[t/64] & ((1 << (t%64)) - 1)) (the O(1)
+ * position-to-slot lookup of Appendix A.1, "Layout", local to the tile).
+ * Dequantized rotated residual: c^_j = min + code_j * scale; the residual is
+ * r~ = s o (H_128 c^) / 128 with H_128 the unnormalised Sylvester Hadamard matrix
+ * (or r~ = c^ when AKV_FLAG_ROTATE is off).
  */
 typedef struct akv_unit_desc {
   int32_t len;       /* S */
   int32_t n_anchors; /* k */
   int32_t n_res_k;   /* N_K */
   int32_t n_res_v;   /* N_V */
-  int32_t n_words;   /* ceil(S / 64) */
+  int32_t n_tiles;   /* ceil(S / AKV_TILE_TOKENS) */
   int32_t b, h;
   int32_t reserved0;
-  uint64_t off_anchor_k, off_anchor_v, off_anchor_pos;
-  uint64_t off_stream_k, off_stream_v;
-  uint64_t off_bitmap_k, off_prefix_k, off_bitmap_v, off_prefix_v;
-  uint64_t off_codes_k, off_scales_k, off_codes_v, off_scales_v;
-  uint64_t data_bytes; /* bytes of the sections (no padding): what one decode reads for this unit */
-  uint8_t pad[256 - 32 - 14 * 8];
+  uint64_t off_anchor_k, off_anchor_v, off_anchor_pos, off_tile_table, off_tiles;
+  uint64_t tiles_capacity; /* bytes reserved for the tile blocks (an upper bound of their use) */
+  uint64_t data_bytes;     /* anchors + tile table + tiles_capacity: the most one decode reads */
+  uint8_t pad[256 - 32 - 7 * 8];
 } akv_unit_desc;
 
 /* ---- Introspection ------------------------------------------------------ */
@@ -160,7 +181,8 @@ const char* akv_last_error(void);
  *   ctx_lens_host : host [B] int32, 1 <= S_b <= 2^30
  *   out_shapes    : host [B*H][4] int32, filled with (S, k, N_K, N_V) per unit
  * Errors: AKV_ERR_INVALID for null pointers or out-of-range parameters,
- * AKV_ERR_UNSUPPORTED for head_dim != 128, G not in {1,2,4,8}, k > 65535.
+ * AKV_ERR_UNSUPPORTED for head_dim != 128, G not in {1,2,4,8}, k > 65535, or a
+ * unit whose tile blocks could exceed 2^32 bytes.
  */
 akv_status akv_unit_shapes(const akv_params* p, const int32_t* ctx_lens_host, int32_t* out_shapes);
 
@@ -257,8 +279,10 @@ typedef struct akv_unit_host {
 
 /*
  * Builds a complete arena image in HOST memory from per-unit logical arrays
- * (units[B*H]); the caller copies it to the device.  Validates anchor slot
- * indices (< k), ascending residual positions (< S) and buffer size.
+ * (units[B*H]), indexed by position; the packer puts the tokens into stored
+ * order (stable sort by value anchor slot) and builds the tile blocks.  The
+ * caller copies the image to the device.  Validates anchor slot indices (< k),
+ * ascending residual positions (< S) and buffer size.
  */
 akv_status akv_cache_pack_host(const akv_params* p, const int32_t* ctx_lens_host, const akv_unit_host* units,
                                void* arena_host, size_t arena_bytes);

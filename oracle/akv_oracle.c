@@ -21,7 +21,8 @@
  *             rotation applied once after accumulation -- Section 4.4 and
  *             Appendix E.1 rely on this linearity); used only to pin that
  *             regrouping against the definition.
- *   unpack  : an independent reader of the packed arena layout.
+ *   unpack  : an independent reader of the packed arena layout (tile blocks,
+ *             tokens in the arena's stored order).
  *
  * Compiled with -ffp-contract=off so that every product and sum is the
  * separately rounded IEEE operation written here.
@@ -603,7 +604,7 @@ static uint64_t rd64(const uint8_t* p) {
 
 /* Returns 0 and the shape of unit u, or -1 on a malformed arena. */
 int or_arena_shape(const uint8_t* arena, uint64_t bytes, int32_t u, int32_t* shape4) {
-  if (bytes < 256 || rd32(arena) != 0x31564B41u || rd32(arena + 4) != 1u) return -1;
+  if (bytes < 256 || rd32(arena) != 0x32564B41u || rd32(arena + 4) != 2u || rd32(arena + 104) != 1024u) return -1;
   int32_t n_units = (int32_t)rd32(arena + 72);
   uint64_t doff = rd64(arena + 80);
   if (u < 0 || u >= n_units || doff + 256ull * (uint64_t)(u + 1) > bytes) return -1;
@@ -612,63 +613,86 @@ int or_arena_shape(const uint8_t* arena, uint64_t bytes, int32_t u, int32_t* sha
   return 0;
 }
 
-/* Copies unit u's logical arrays out of the arena into the caller's buffers
- * (shape first from or_arena_shape).  Returns 0, or -1 on any inconsistency
- * (bitmap popcount vs slot counts, prefix table, anchor slot range). */
+/* Copies unit u's logical arrays out of the arena (shape first from
+ * or_arena_shape).  The arena keeps tokens in its stored order (sorted by value
+ * anchor slot); the arrays come back in that order, and res_k / res_v hold the
+ * stored indices of the tokens with a residual.  Returns 0, or -1 on any
+ * inconsistency (tile table, rank words, record counts, anchor slot range,
+ * value slots out of order). */
 int or_arena_unpack(const uint8_t* arena, uint64_t bytes, int32_t u, or_unit* out) {
   int32_t sh[4];
   if (or_arena_shape(arena, bytes, u, sh) != 0) return -1;
   const uint8_t* d = arena + rd64(arena + 80) + 256ull * (uint64_t)u;
   int32_t S = sh[0], k = sh[1], nk = sh[2], nv = sh[3];
-  int32_t nw = (int32_t)rd32(d + 16);
-  if (nw != (S + 63) / 64) return -1;
-  uint64_t off[13];
-  for (int t = 0; t < 13; ++t) off[t] = rd64(d + 32 + 8 * t);
-  uint64_t end[13] = {off[0] + (uint64_t)k * 256, off[1] + (uint64_t)k * 256, off[2] + 4ull * k,
-                      off[3] + 4ull * S,          off[4] + 4ull * S,          off[5] + 8ull * nw,
-                      off[6] + 4ull * nw,         off[7] + 8ull * nw,         off[8] + 4ull * nw,
-                      off[9] + 32ull * nk,        off[10] + 4ull * nk,        off[11] + 32ull * nv,
-                      off[12] + 4ull * nv};
-  for (int t = 0; t < 13; ++t)
-    if (end[t] > bytes || (off[t] % 16) != 0) return -1;
-  memcpy(out->anchor_k, arena + off[0], (size_t)k * 256);
-  memcpy(out->anchor_v, arena + off[1], (size_t)k * 256);
-  memcpy(out->anchor_pos, arena + off[2], (size_t)k * 4);
-  for (int side = 0; side < 2; ++side) {
-    const uint8_t* st = arena + off[3 + side];
-    uint16_t* idx = side ? out->idx_v : out->idx_k;
-    uint16_t* gam = side ? out->gam_v : out->gam_k;
-    for (int32_t i = 0; i < S; ++i) {
-      uint32_t e = rd32(st + 4ull * i);
-      idx[i] = (uint16_t)(e & 0xFFFFu);
-      gam[i] = (uint16_t)(e >> 16);
-      if (idx[i] >= k) return -1;
+  const int32_t T = 1024;
+  int32_t nt = (int32_t)rd32(d + 16);
+  if (nt != (S + T - 1) / T) return -1;
+  uint64_t o_ak = rd64(d + 32), o_av = rd64(d + 40), o_ap = rd64(d + 48), o_tt = rd64(d + 56), o_ti = rd64(d + 64);
+  uint64_t cap = rd64(d + 72);
+  if (o_ak + 256ull * k > bytes || o_av + 256ull * k > bytes || o_ap + 4ull * k > bytes ||
+      o_tt + 4ull * (nt + 1) > bytes || o_ti + cap > bytes || (o_ak % 16) || (o_av % 16) || (o_ti % 16))
+    return -1;
+  for (int32_t a = 0; a < k; ++a)
+    for (int c = 0; c < 16; ++c) {
+      memcpy(out->anchor_k + (size_t)a * 128 + 8 * c, arena + o_ak + (size_t)a * 256 + 16 * (c ^ (a & 7)), 16);
+      memcpy(out->anchor_v + (size_t)a * 128 + 8 * c, arena + o_av + (size_t)a * 256 + 16 * (c ^ (a & 7)), 16);
     }
-    const uint8_t* bm = arena + off[5 + 2 * side];
-    const uint8_t* pf = arena + off[6 + 2 * side];
-    int32_t n = side ? nv : nk;
-    int32_t* res = side ? out->res_v : out->res_k;
-    int32_t cnt = 0;
-    for (int32_t w = 0; w < nw; ++w) {
-      if ((int32_t)rd32(pf + 4ull * w) != cnt) return -1;
-      uint64_t word = rd64(bm + 8ull * w);
-      for (int bit = 0; bit < 64; ++bit) {
-        if ((word >> bit) & 1ull) {
-          int32_t pos = w * 64 + bit;
-          if (pos >= S || cnt >= n) return -1;
-          res[cnt++] = pos;
-        }
+  memcpy(out->anchor_pos, arena + o_ap, (size_t)k * 4);
+  int32_t cnt[2] = {0, 0};
+  uint32_t prev_av = 0;
+  for (int32_t j = 0; j < nt; ++j) {
+    uint32_t b0 = rd32(arena + o_tt + 4ull * j), b1 = rd32(arena + o_tt + 4ull * (j + 1));
+    if ((b0 % 16) || b1 < b0 || b1 > cap) return -1;
+    const uint8_t* blk = arena + o_ti + b0;
+    int32_t n = S - j * T < T ? S - j * T : T;
+    int32_t nw = (n + 63) / 64, n64 = 64 * nw;
+    const uint8_t* kst = blk;
+    const uint8_t* vst = blk + 4ull * n64;
+    const uint8_t* bm[2] = {blk + 8ull * n64, blk + 8ull * n64 + 8ull * nw};
+    int32_t rk_pad = ((2 * nw + 15) / 16) * 16;
+    const uint8_t* rk[2] = {blk + 8ull * n64 + 16ull * nw, blk + 8ull * n64 + 16ull * nw + rk_pad};
+    uint32_t F = 8u * n64 + 16u * nw + 2u * rk_pad;
+    /* records of this tile, per side */
+    int32_t m[2] = {0, 0};
+    for (int side = 0; side < 2; ++side)
+      for (int32_t w = 0; w < nw; ++w) {
+        uint64_t word = rd64(bm[side] + 8ull * w);
+        if ((uint32_t)(rd32(rk[side] + 2ull * w) & 0xFFFFu) != (uint32_t)m[side]) return -1;
+        if (w == nw - 1 && n % 64 && (word >> (n % 64))) return -1; /* bits past the last token */
+        for (int bit = 0; bit < 64; ++bit) m[side] += (int32_t)((word >> bit) & 1ull);
+      }
+    uint32_t sm_off[2] = {F, F + (uint32_t)(((4 * m[0] + 15) / 16) * 16)};
+    uint32_t cd_off[2];
+    cd_off[0] = sm_off[1] + (uint32_t)(((4 * m[1] + 15) / 16) * 16);
+    cd_off[1] = cd_off[0] + 32u * (uint32_t)m[0];
+    if (b0 + cd_off[1] + 32u * (uint32_t)m[1] != b1) return -1;
+    if (cnt[0] + m[0] > nk || cnt[1] + m[1] > nv) return -1;
+    int32_t r[2] = {0, 0};
+    for (int32_t t = 0; t < n; ++t) {
+      int32_t i = j * T + t;
+      uint32_t ek = rd32(kst + 4ull * t), ev = rd32(vst + 4ull * t);
+      out->idx_k[i] = (uint16_t)(ek & 0xFFFFu);
+      out->gam_k[i] = (uint16_t)(ek >> 16);
+      out->idx_v[i] = (uint16_t)(ev & 0xFFFFu);
+      out->gam_v[i] = (uint16_t)(ev >> 16);
+      if (out->idx_k[i] >= k || out->idx_v[i] >= k || (ev & 0xFFFFu) < prev_av) return -1;
+      prev_av = ev & 0xFFFFu;
+      for (int side = 0; side < 2; ++side) {
+        if (!((rd64(bm[side] + 8ull * (t >> 6)) >> (t & 63)) & 1ull)) continue;
+        int32_t g = cnt[side] + r[side];
+        (side ? out->res_v : out->res_k)[g] = i;
+        uint32_t e = rd32(blk + sm_off[side] + 4ull * r[side]);
+        (side ? out->scale_v : out->scale_k)[g] = (uint16_t)(e & 0xFFFFu);
+        (side ? out->min_v : out->min_k)[g] = (uint16_t)(e >> 16);
+        memcpy((side ? out->codes_v : out->codes_k) + 32ull * g, blk + cd_off[side] + 32ull * r[side], 32);
+        ++r[side];
       }
     }
-    if (cnt != n) return -1;
-    const uint8_t* cd = arena + off[9 + 2 * side];
-    const uint8_t* sc = arena + off[10 + 2 * side];
-    memcpy(side ? out->codes_v : out->codes_k, cd, (size_t)n * 32);
-    for (int32_t t = 0; t < n; ++t) {
-      uint32_t e = rd32(sc + 4ull * t);
-      (side ? out->scale_v : out->scale_k)[t] = (uint16_t)(e & 0xFFFFu);
-      (side ? out->min_v : out->min_k)[t] = (uint16_t)(e >> 16);
-    }
+    for (int32_t t = n; t < n64; ++t)
+      if (rd32(kst + 4ull * t) || rd32(vst + 4ull * t)) return -1;
+    cnt[0] += m[0];
+    cnt[1] += m[1];
   }
+  if (cnt[0] != nk || cnt[1] != nv) return -1;
   return 0;
 }

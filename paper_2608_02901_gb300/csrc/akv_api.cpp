@@ -1,9 +1,11 @@
 // Host side of the C ABI: parameter validation, arena layout, the host packer
 // and the thin wrappers that hand validated work to the kernel launchers.
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
 #include <string>
+#include <vector>
 
 #include "akv_internal.h"
 
@@ -76,30 +78,34 @@ akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out
       sh.k = (int32_t)k;
       sh.nk = (int32_t)nk;
       sh.nv = (int32_t)nv;
-      const uint64_t nw = (uint64_t)(S + 63) / 64;
-      const uint64_t sizes[kNumSections] = {
-          (uint64_t)k * 256, (uint64_t)k * 256, (uint64_t)k * 4, (uint64_t)S * 4, (uint64_t)S * 4,
-          nw * 8,            nw * 4,            nw * 8,          nw * 4,          (uint64_t)nk * 32,
-          (uint64_t)nk * 4,  (uint64_t)nv * 32, (uint64_t)nv * 4};
+      const int32_t nt = (S + kTile - 1) / kTile;
+      sh.nt = nt;
+      // tile blocks: fixed parts exactly, records and at most 24 bytes of padding per tile
+      uint64_t cap = 0;
+      for (int32_t j = 0; j < nt; ++j) cap += tile_fixed_bytes(std::min(kTile, S - j * kTile));
+      cap += 36ull * (uint64_t)(nk + nv) + 24ull * (uint64_t)nt;
+      if (cap >= (1ull << 32)) return fail(AKV_ERR_UNSUPPORTED, "a unit's tile blocks could exceed 2^32 bytes");
+      const uint64_t sizes[kNumSections] = {(uint64_t)k * 256, (uint64_t)k * 256, (uint64_t)k * 4,
+                                            4ull * (uint64_t)(nt + 1), cap};
       akv_unit_desc& d = L.desc[u];
       std::memset(&d, 0, sizeof(d));
       d.len = S;
       d.n_anchors = (int32_t)k;
       d.n_res_k = (int32_t)nk;
       d.n_res_v = (int32_t)nv;
-      d.n_words = (int32_t)nw;
+      d.n_tiles = nt;
       d.b = b;
       d.h = h;
       off = align_up(off, kSegmentAlign);
       uint64_t* offs = &d.off_anchor_k;
-      uint64_t data = 0;
       for (int s = 0; s < kNumSections; ++s) {
         off = align_up(off, kSectionAlign);
         offs[s] = off;
         off += sizes[s];
-        if (s != kAnchorPos) data += sizes[s];
       }
-      d.data_bytes = data;
+      d.tiles_capacity = cap;
+      d.data_bytes = sizes[kAnchorK] + sizes[kAnchorV] + sizes[kTileTable] + cap;
+      if (nt > L.max_tiles) L.max_tiles = nt;
       if (S > L.max_len) L.max_len = S;
       if (k > L.max_k) L.max_k = (int32_t)k;
       if (nk > L.max_nk) L.max_nk = (int32_t)nk;
@@ -116,6 +122,7 @@ akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out
   H.n_units = n_units;
   H.max_len = L.max_len;
   H.desc_offset = kHeaderBytes;
+  H.tile_tokens = kTile;
   rotation_signs(p->rot_seed, H.sign_bits);
   return AKV_OK;
 }
@@ -123,7 +130,9 @@ akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out
 void encode_ws_layout(const Layout& L, EncodeWs* ws) {
   // Per unit: two u64 key arrays [S] (anchor hashes, then residual energies
   // per side), slot map i32 [S], residual positions i32 [N_K + N_V],
-  // anchor norms (squared, and square roots) f64 [k] per side, 256 B control.
+  // anchor norms (squared, and square roots) f64 [k] per side, 256 B control,
+  // stream words u32 [S] per side, flags u8 [S], stored order and inverse
+  // i32 [S], run starts u32 [k + 1], record counts u32 [2 n_tiles].
   // A table of per-unit byte offsets (u64 each) leads the workspace.
   ws->unit_off.resize(L.shape.size());
   uint64_t off = align_up((uint64_t)L.shape.size() * 8, 256);
@@ -136,6 +145,11 @@ void encode_ws_layout(const Layout& L, EncodeWs* ws) {
     b += align_up((uint64_t)(s.nk + s.nv) * 4 + 16, 256);
     b += align_up((uint64_t)s.k * 8, 256) * 4;
     b += 256;
+    b += align_up((uint64_t)s.S * 4, 256) * 2;        // stream words per side
+    b += align_up((uint64_t)s.S, 256);                // residual flags
+    b += align_up((uint64_t)s.S * 4, 256) * 2;        // stored order and its inverse
+    b += align_up((uint64_t)(s.k + 1) * 4, 256);      // value-anchor run starts
+    b += align_up((uint64_t)s.nt * 8, 256);           // records per tile and side
     off += b;
   }
   ws->total = off + 256;
@@ -225,38 +239,79 @@ akv_status akv_cache_pack_host(const akv_params* p, const int32_t* ctx_lens_host
         (sh.nk && (!in.res_pos_k || !in.codes_k || !in.scale_k || !in.min_k)) ||
         (sh.nv && (!in.res_pos_v || !in.codes_v || !in.scale_v || !in.min_v)))
       return fail(AKV_ERR_INVALID, "null array in unit " + std::to_string(u));
-    std::memcpy(A + d.off_anchor_k, in.anchor_k, (size_t)k * 256);
-    std::memcpy(A + d.off_anchor_v, in.anchor_v, (size_t)k * 256);
+    // anchor rows, 16-byte chunks swizzled by the slot (chunk c at place c ^ (a % 8))
+    for (int side = 0; side < 2; ++side) {
+      const uint16_t* src = side ? in.anchor_v : in.anchor_k;
+      uint8_t* dst = A + (side ? d.off_anchor_v : d.off_anchor_k);
+      for (int32_t a = 0; a < k; ++a)
+        for (int c = 0; c < 16; ++c)
+          std::memcpy(dst + (size_t)a * 256 + 16 * (c ^ (a & 7)), src + (size_t)a * 128 + 8 * c, 16);
+    }
     std::memcpy(A + d.off_anchor_pos, in.anchor_pos, (size_t)k * 4);
+    // residual slot of each position per side (-1: none)
+    std::vector<int32_t> slot[2];
     for (int side = 0; side < 2; ++side) {
       const uint16_t* idx = side ? in.idx_v : in.idx_k;
-      const uint16_t* gam = side ? in.gamma_v : in.gamma_k;
-      uint32_t* stream = (uint32_t*)(A + (side ? d.off_stream_v : d.off_stream_k));
-      for (int32_t i = 0; i < S; ++i) {
+      for (int32_t i = 0; i < S; ++i)
         if (idx[i] >= k) return fail(AKV_ERR_INVALID, "anchor index out of range in unit " + std::to_string(u));
-        stream[i] = (uint32_t)idx[i] | ((uint32_t)gam[i] << 16);
-      }
       const int32_t n = side ? sh.nv : sh.nk;
       const int32_t* pos = side ? in.res_pos_v : in.res_pos_k;
-      uint64_t* bm = (uint64_t*)(A + (side ? d.off_bitmap_v : d.off_bitmap_k));
-      uint32_t* pf = (uint32_t*)(A + (side ? d.off_prefix_v : d.off_prefix_k));
+      slot[side].assign((size_t)S, -1);
       for (int32_t t = 0; t < n; ++t) {
         if (pos[t] < 0 || pos[t] >= S || (t > 0 && pos[t] <= pos[t - 1]))
           return fail(AKV_ERR_INVALID, "residual positions must be ascending and < S in unit " + std::to_string(u));
-        bm[pos[t] >> 6] |= 1ull << (pos[t] & 63);
+        slot[side][(size_t)pos[t]] = t;
       }
-      uint32_t run = 0;
-      for (int32_t w = 0; w < d.n_words; ++w) {
-        pf[w] = run;
-        run += (uint32_t)__builtin_popcountll(bm[w]);
-      }
-      const uint8_t* codes = side ? in.codes_v : in.codes_k;
-      const uint16_t* sc = side ? in.scale_v : in.scale_k;
-      const uint16_t* mn = side ? in.min_v : in.min_k;
-      if (n) std::memcpy(A + (side ? d.off_codes_v : d.off_codes_k), codes, (size_t)n * 32);
-      uint32_t* scales = (uint32_t*)(A + (side ? d.off_scales_v : d.off_scales_k));
-      for (int32_t t = 0; t < n; ++t) scales[t] = (uint32_t)sc[t] | ((uint32_t)mn[t] << 16);
     }
+    // stored order: stable counting sort of positions by value anchor slot
+    std::vector<int32_t> start((size_t)k + 1, 0), perm((size_t)S);
+    for (int32_t i = 0; i < S; ++i) ++start[(size_t)in.idx_v[i] + 1];
+    for (int32_t a = 0; a < k; ++a) start[(size_t)a + 1] += start[(size_t)a];
+    for (int32_t i = 0; i < S; ++i) perm[(size_t)start[in.idx_v[i]]++] = i;
+    // tile blocks
+    uint32_t* table = (uint32_t*)(A + d.off_tile_table);
+    uint8_t* tiles = A + d.off_tiles;
+    uint32_t off = 0;
+    for (int32_t j = 0; j < sh.nt; ++j) {
+      const int32_t t0 = j * kTile, n = std::min(kTile, S - t0);
+      const uint32_t nw = tile_words(n), n64 = 64 * nw;
+      int32_t cnt[2] = {0, 0};
+      for (int32_t t = 0; t < n; ++t)
+        for (int side = 0; side < 2; ++side) cnt[side] += slot[side][(size_t)perm[(size_t)(t0 + t)]] >= 0;
+      table[j] = off;
+      if ((uint64_t)off + tile_block_bytes(n, cnt[0], cnt[1]) > d.tiles_capacity)
+        return fail(AKV_ERR_INVALID, "tile blocks exceed their reserved capacity");  // cannot happen: bound
+      uint8_t* blk = tiles + off;
+      uint32_t* kst = (uint32_t*)blk;
+      uint32_t* vst = kst + n64;
+      uint64_t* bm[2] = {(uint64_t*)(vst + n64), (uint64_t*)(vst + n64) + nw};
+      uint16_t* rk[2] = {(uint16_t*)(bm[1] + nw), (uint16_t*)(bm[1] + nw) + round16(2 * nw) / 2};
+      const uint32_t F = tile_fixed_bytes(n);
+      uint32_t* sm[2] = {(uint32_t*)(blk + F), (uint32_t*)(blk + F + round16(4 * (uint32_t)cnt[0]))};
+      uint8_t* cd[2];
+      cd[0] = blk + F + round16(4 * (uint32_t)cnt[0]) + round16(4 * (uint32_t)cnt[1]);
+      cd[1] = cd[0] + 32 * (size_t)cnt[0];
+      int32_t r[2] = {0, 0};
+      for (int32_t t = 0; t < n; ++t) {
+        const int32_t i = perm[(size_t)(t0 + t)];
+        kst[t] = (uint32_t)in.idx_k[i] | ((uint32_t)in.gamma_k[i] << 16);
+        vst[t] = (uint32_t)in.idx_v[i] | ((uint32_t)in.gamma_v[i] << 16);
+        if ((t & 63) == 0)
+          for (int side = 0; side < 2; ++side) rk[side][t >> 6] = (uint16_t)r[side];
+        for (int side = 0; side < 2; ++side) {
+          const int32_t sl = slot[side][(size_t)i];
+          if (sl < 0) continue;
+          bm[side][t >> 6] |= 1ull << (t & 63);
+          const uint16_t sc = side ? in.scale_v[sl] : in.scale_k[sl];
+          const uint16_t mn = side ? in.min_v[sl] : in.min_k[sl];
+          sm[side][r[side]] = (uint32_t)sc | ((uint32_t)mn << 16);
+          std::memcpy(cd[side] + 32 * (size_t)r[side], (side ? in.codes_v : in.codes_k) + 32 * (size_t)sl, 32);
+          ++r[side];
+        }
+      }
+      off += tile_block_bytes(n, cnt[0], cnt[1]);
+    }
+    table[sh.nt] = off;
   }
   return AKV_OK;
 }

@@ -7,12 +7,16 @@
 // twice gives the same result.
 //
 // Kernels, in launch order, each over all units of the batch:
-//   enc_hash      anchor-selection hashes of the non-window positions
-//   enc_anchors   select the k - W smallest hashes, number anchor slots by position
-//   enc_rows      copy anchor rows into the arena, squared norms per side
-//   enc_assign    Eq. 1 nearest anchor, Eq. 2 gamma, residual energies
-//   enc_slots     top-N residual energies per side -> bitmap, prefix, slot list
-//   enc_quant     Eq. 12 rotation and 2-bit quantization of every slot
+//   enc_hash       anchor-selection hashes of the non-window positions
+//   enc_anchors    select the k - W smallest hashes, number anchor slots by position
+//   enc_rows       copy anchor rows into the arena (16-byte chunks swizzled), squared norms
+//   enc_assign     Eq. 1 nearest anchor, Eq. 2 gamma, residual energies (per position)
+//   enc_slots      top-N residual energies per side -> residual flags and slot list
+//   enc_order      stored order: stable counting sort of positions by value anchor slot
+//   enc_tile_count residual records per tile and side
+//   enc_tile_table tile block offsets
+//   enc_tile_fill  streams, bitmaps and rank words of every tile block
+//   enc_quant      Eq. 12 rotation and 2-bit quantization of every slot, into its tile
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
@@ -35,6 +39,12 @@ struct EncUnitWs {
   double* n2[2];      // [k] squared anchor norms per side
   double* rn[2];      // [k] their square roots
   uint32_t* ctrl;     // [0]: side 0 has a nonzero anchor, [1]: side 1
+  uint32_t* st[2];    // [S] stream word (slot | fp16 gamma << 16) per position and side
+  uint8_t* flag;      // [S] bit 0: key residual, bit 1: value residual
+  int32_t* perm;      // [S] position of stored token t
+  int32_t* inv;       // [S] stored index of position i
+  uint32_t* cursor;   // [k + 1] value-anchor counts, then start of each run
+  uint32_t* tcnt;     // [2 * n_tiles] residual records per tile (keys, values)
 };
 
 struct EncArgs {
@@ -77,7 +87,26 @@ __device__ EncUnitWs unit_ws(const EncArgs& A, int u, const akv_unit_desc* d) {
     p += au(k * 8, 256);
   }
   w.ctrl = (uint32_t*)p;
+  p += 256;
+  for (int s = 0; s < 2; ++s) {
+    w.st[s] = (uint32_t*)p;
+    p += au(S * 4, 256);
+  }
+  w.flag = p;
+  p += au(S, 256);
+  w.perm = (int32_t*)p;
+  p += au(S * 4, 256);
+  w.inv = (int32_t*)p;
+  p += au(S * 4, 256);
+  w.cursor = (uint32_t*)p;
+  p += au((k + 1) * 4, 256);
+  w.tcnt = (uint32_t*)p;
   return w;
+}
+
+// Anchor row a of a side in the source K or V (the arena holds it swizzled).
+__device__ __forceinline__ const __nv_bfloat16* anchor_src(const EncArgs& A, int u, int side, const int32_t* apos, int a) {
+  return (side ? A.V : A.K) + ((size_t)u * A.s_max + (size_t)apos[a]) * 128;
 }
 
 __device__ __forceinline__ uint64_t splitmix64_dev(uint64_t x) {
@@ -242,7 +271,8 @@ __global__ void enc_rows(const EncArgs A) {
     const __nv_bfloat16* X = (side ? A.V : A.K) + ((size_t)u * A.s_max + pos) * 128;
     __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(A.arena + (side ? d->off_anchor_v : d->off_anchor_k)) +
                          (size_t)a * 128;
-    for (int j = lane; j < 128; j += 32) dst[j] = X[j];
+    // dim j is in chunk j / 8, stored at chunk place (j / 8) ^ (a % 8)
+    for (int j = lane; j < 128; j += 32) dst[8 * ((j >> 3) ^ (a & 7)) + (j & 7)] = X[j];
     if (lane == 0) {
       double n = 0.0;
       for (int j = 0; j < 128; ++j) {
@@ -276,7 +306,7 @@ __global__ void __launch_bounds__(AS_THREADS) enc_assign(const EncArgs A) {
   if (p0 >= S) return;
   EncUnitWs w = unit_ws(A, u, d);
   const __nv_bfloat16* X = (side ? A.V : A.K) + (size_t)u * A.s_max * 128;
-  const __nv_bfloat16* AT = reinterpret_cast<const __nv_bfloat16*>(A.arena_c + (side ? d->off_anchor_v : d->off_anchor_k));
+  const int32_t* apos = reinterpret_cast<const int32_t*>(A.arena_c + d->off_anchor_pos);
   const double* n2 = w.n2[side];
   const double* rn = w.rn[side];
   const int tid = threadIdx.x;
@@ -293,7 +323,7 @@ __global__ void __launch_bounds__(AS_THREADS) enc_assign(const EncArgs A) {
     __syncthreads();
     for (int e = tid; e < AS_ANC * 128; e += AS_THREADS) {
       const int t = e >> 7, j = e & 127;
-      xa[e] = (ac + t < k) ? bf16_to_f64(AT[(size_t)(ac + t) * 128 + j]) : 0.0;
+      xa[e] = (ac + t < k) ? bf16_to_f64(anchor_src(A, u, side, apos, ac + t)[j]) : 0.0;
     }
     __syncthreads();
     double dd[8];
@@ -337,7 +367,7 @@ __global__ void __launch_bounds__(AS_THREADS) enc_assign(const EncArgs A) {
       dbest = bdv[g * AS_POS + tid];
     }
   }
-  uint32_t* stream = reinterpret_cast<uint32_t*>(A.arena + (side ? d->off_stream_v : d->off_stream_k));
+  uint32_t* stream = w.st[side];
   uint64_t* key = side ? w.key1 : w.key0;
   const int sl = w.slot_of[p];
   if (sl >= 0) {
@@ -348,7 +378,7 @@ __global__ void __launch_bounds__(AS_THREADS) enc_assign(const EncArgs A) {
   const uint32_t gh = (a >= 0) ? f64_to_fp16_bits(__ddiv_rn(dbest, n2[a])) : 0u;
   stream[p] = (uint32_t)(a >= 0 ? a : 0) | (gh << 16);
   const double g = fp16_bits_to_f64(gh);
-  const __nv_bfloat16* xar = AT + (size_t)(a >= 0 ? a : 0) * 128;
+  const __nv_bfloat16* xar = anchor_src(A, u, side, apos, a >= 0 ? a : 0);
   double e = 0.0;
   for (int j = 0; j < 128; ++j) {
     const double pj = (a >= 0) ? __dmul_rn(g, bf16_to_f64(xar[j])) : 0.0;
@@ -358,19 +388,17 @@ __global__ void __launch_bounds__(AS_THREADS) enc_assign(const EncArgs A) {
   key[p] = (uint64_t)__double_as_longlong(e) + 1ull;
 }
 
-// Per (unit, side): the N largest keys (ties: lower position), bitmap, prefix, slot list.
-__global__ void __launch_bounds__(1024) enc_slots(const EncArgs A) {
+// Per (unit, side): the N largest keys (ties: lower position) -> flags and the
+// ascending slot list.
+__global__ void __launch_bounds__(1024) enc_slots(const EncArgs A, int side) {
   __shared__ uint32_t hist[256];
   __shared__ uint32_t bc[2];
   __shared__ int wt[33];
-  __shared__ uint32_t halves[32];
-  const int u = blockIdx.x, side = blockIdx.y;
+  const int u = blockIdx.x;
   const akv_unit_desc* d = unit_desc(A, u);
   const int S = d->len, N = side ? d->n_res_v : d->n_res_k;
   EncUnitWs w = unit_ws(A, u, d);
   const uint64_t* key = side ? w.key1 : w.key0;
-  uint64_t* bm = reinterpret_cast<uint64_t*>(A.arena + (side ? d->off_bitmap_v : d->off_bitmap_k));
-  uint32_t* pf = reinterpret_cast<uint32_t*>(A.arena + (side ? d->off_prefix_v : d->off_prefix_k));
   int32_t* rp = w.res_pos + (side ? d->n_res_k : 0);
   uint64_t thr = ~0ull;
   uint32_t need = 0;
@@ -384,25 +412,157 @@ __global__ void __launch_bounds__(1024) enc_slots(const EncArgs A) {
     const int eq_pre = block_scan_flag(is_eq, wt, &eq_tot);
     const int sel = (N > 0 && p < S) && (kv > thr || (is_eq && (uint32_t)(eq_seen + eq_pre) < need));
     eq_seen += eq_tot;
-    const unsigned bal = __ballot_sync(0xffffffffu, sel);
-    if ((threadIdx.x & 31) == 0) halves[threadIdx.x >> 5] = bal;
     int tot;
     const int pre = block_scan_flag(sel, wt, &tot);
     if (sel) rp[base + pre] = p;
-    // 16 words of 64 positions per chunk; threads 0..15 write them
-    if (threadIdx.x < 16) {
-      const int wi = (c0 >> 6) + threadIdx.x;
-      if (wi < d->n_words) {
-        const uint64_t word = (uint64_t)halves[2 * threadIdx.x] | ((uint64_t)halves[2 * threadIdx.x + 1] << 32);
-        bm[wi] = word;
-        int before = 0;
-        for (int t = 0; t < (int)threadIdx.x; ++t)
-          before += __popcll((uint64_t)halves[2 * t] | ((uint64_t)halves[2 * t + 1] << 32));
-        pf[wi] = (uint32_t)(base + before);
-      }
+    // flags of both sides share bytes: the side-0 launch writes them, the side-1 launch
+    // (ordered after it on the stream) ORs its bit in
+    if (p < S) {
+      if (side == 0) w.flag[p] = (uint8_t)sel;
+      else if (sel) w.flag[p] |= 2u;
     }
     base += tot;
     __syncthreads();
+  }
+}
+
+// Exclusive block scan of non-negative counts (1024 threads); returns the prefix and
+// writes the block total to *total.
+__device__ uint32_t block_scan_u32(uint32_t v, uint32_t* warp_tot, uint32_t* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  if (lane == 31) warp_tot[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    uint32_t x = warp_tot[lane], xi = x;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t t = __shfl_up_sync(0xffffffffu, xi, o);
+      if (lane >= o) xi += t;
+    }
+    warp_tot[lane] = xi - x;
+    if (lane == 31) warp_tot[32] = xi;
+  }
+  __syncthreads();
+  const uint32_t pre = warp_tot[warp] + incl - v;
+  *total = warp_tot[32];
+  __syncthreads();
+  return pre;
+}
+
+// Stored order of one unit: positions sorted by value anchor slot, ties by position
+// (a stable counting sort).  One block per unit; the scatter is done by one warp in
+// position order, 32 positions at a time, so equal slots keep their position order.
+__global__ void __launch_bounds__(1024) enc_order(const EncArgs A) {
+  __shared__ uint32_t wt[33];
+  const int u = blockIdx.x;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len, k = d->n_anchors;
+  EncUnitWs w = unit_ws(A, u, d);
+  for (int a = threadIdx.x; a <= k; a += blockDim.x) w.cursor[a] = 0u;
+  __syncthreads();
+  for (int p = threadIdx.x; p < S; p += blockDim.x) atomicAdd(&w.cursor[w.st[1][p] & 0xFFFFu], 1u);
+  __syncthreads();
+  uint32_t run = 0;
+  for (int c0 = 0; c0 < k; c0 += 1024) {
+    const int a = c0 + threadIdx.x;
+    const uint32_t v = a < k ? w.cursor[a] : 0u;
+    uint32_t tot;
+    const uint32_t pre = block_scan_u32(v, wt, &tot);
+    if (a < k) w.cursor[a] = run + pre;
+    run += tot;
+  }
+  __syncthreads();
+  if (threadIdx.x >= 32) return;
+  const int lane = threadIdx.x;
+  for (int c0 = 0; c0 < S; c0 += 32) {
+    const int p = c0 + lane;
+    const uint32_t a = p < S ? (w.st[1][p] & 0xFFFFu) : 0xFFFFFFFFu;
+    const unsigned peers = __match_any_sync(0xffffffffu, a);
+    const uint32_t base = p < S ? w.cursor[a] : 0u;
+    __syncwarp();
+    const int rank = __popc(peers & ((1u << lane) - 1u));
+    if (p < S) {
+      w.perm[base + rank] = p;
+      w.inv[p] = (int32_t)(base + rank);
+      if (rank == 0) w.cursor[a] = base + (uint32_t)__popc(peers);
+    }
+    __syncwarp();
+  }
+}
+
+__device__ __forceinline__ int tile_len(int S, int j) { return min(kTile, S - j * kTile); }
+
+// Residual records of each tile and side (one thread per stored token).
+__global__ void __launch_bounds__(kTile) enc_tile_count(const EncArgs A) {
+  const int u = blockIdx.y, j = blockIdx.x;
+  const akv_unit_desc* d = unit_desc(A, u);
+  if (j >= d->n_tiles) return;
+  EncUnitWs w = unit_ws(A, u, d);
+  const int t = j * kTile + threadIdx.x;
+  const uint32_t f = t < d->len ? w.flag[w.perm[t]] : 0u;
+  const int nk = __syncthreads_count(f & 1u), nv = __syncthreads_count(f & 2u);
+  if (threadIdx.x == 0) {
+    w.tcnt[2 * j] = (uint32_t)nk;
+    w.tcnt[2 * j + 1] = (uint32_t)nv;
+  }
+}
+
+// Tile block offsets of every unit (one thread per unit).
+__global__ void enc_tile_table(const EncArgs A, int units) {
+  const int u = blockIdx.x * blockDim.x + threadIdx.x;
+  if (u >= units) return;
+  const akv_unit_desc* d = unit_desc(A, u);
+  EncUnitWs w = unit_ws(A, u, d);
+  uint32_t* table = reinterpret_cast<uint32_t*>(A.arena + d->off_tile_table);
+  uint32_t off = 0;
+  for (int j = 0; j < d->n_tiles; ++j) {
+    table[j] = off;
+    off += tile_block_bytes(tile_len(d->len, j), (int)w.tcnt[2 * j], (int)w.tcnt[2 * j + 1]);
+  }
+  table[d->n_tiles] = off;
+}
+
+// Streams, bitmaps and rank words of one tile block (one thread per stored token).
+__global__ void __launch_bounds__(kTile) enc_tile_fill(const EncArgs A) {
+  __shared__ uint32_t halves[2][kTile / 32];
+  const int u = blockIdx.y, j = blockIdx.x;
+  const akv_unit_desc* d = unit_desc(A, u);
+  if (j >= d->n_tiles) return;
+  EncUnitWs w = unit_ws(A, u, d);
+  const int n = tile_len(d->len, j), nw = (int)tile_words(n), n64 = 64 * nw;
+  const uint32_t off = reinterpret_cast<const uint32_t*>(A.arena_c + d->off_tile_table)[j];
+  uint8_t* blk = A.arena + d->off_tiles + off;
+  uint32_t* kst = reinterpret_cast<uint32_t*>(blk);
+  uint32_t* vst = kst + n64;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  uint32_t f = 0;
+  if (t < n) {
+    const int i = w.perm[j * kTile + t];
+    kst[t] = w.st[0][i];
+    vst[t] = w.st[1][i];
+    f = w.flag[i];
+  }
+  const unsigned bk = __ballot_sync(0xffffffffu, f & 1u), bv = __ballot_sync(0xffffffffu, f & 2u);
+  if (lane == 0) {
+    halves[0][warp] = bk;
+    halves[1][warp] = bv;
+  }
+  __syncthreads();
+  if (t < 2 * nw) {
+    const int side = t / nw, wi = t % nw;
+    uint64_t* bm = reinterpret_cast<uint64_t*>(blk + 8u * n64) + side * nw;
+    uint16_t* rk = reinterpret_cast<uint16_t*>(blk + 8u * n64 + 16u * nw + side * round16(2u * nw));
+    const uint64_t word = (uint64_t)halves[side][2 * wi] | ((uint64_t)halves[side][2 * wi + 1] << 32);
+    bm[wi] = word;
+    int before = 0;
+    for (int x = 0; x < 2 * wi; ++x) before += __popc(halves[side][x]);
+    rk[wi] = (uint16_t)before;
   }
 }
 
@@ -417,13 +577,12 @@ __global__ void enc_quant(const EncArgs A) {
   if (s >= N) return;
   EncUnitWs w = unit_ws(A, u, d);
   const int p = w.res_pos[(side ? d->n_res_k : 0) + s];
-  const uint32_t st = reinterpret_cast<const uint32_t*>(A.arena_c + (side ? d->off_stream_v : d->off_stream_k))[p];
+  const uint32_t st = w.st[side][p];
   const int a = (int)(st & 0xFFFFu);
   const double g = fp16_bits_to_f64(st >> 16);
   const bool valid = w.ctrl[side] != 0u;
   const __nv_bfloat16* X = (side ? A.V : A.K) + ((size_t)u * A.s_max + p) * 128;
-  const __nv_bfloat16* XA =
-      reinterpret_cast<const __nv_bfloat16*>(A.arena_c + (side ? d->off_anchor_v : d->off_anchor_k)) + (size_t)a * 128;
+  const __nv_bfloat16* XA = anchor_src(A, u, side, reinterpret_cast<const int32_t*>(A.arena_c + d->off_anchor_pos), a);
   double* v = vbuf[wi];
   for (int j = lane; j < 128; j += 32) {
     const double pj = valid ? __dmul_rn(g, bf16_to_f64(XA[j])) : 0.0;
@@ -478,12 +637,21 @@ __global__ void enc_quant(const EncArgs A) {
     }
     byte |= (uint32_t)code << (2 * c);
   }
-  uint8_t* codes = A.arena + (side ? d->off_codes_v : d->off_codes_k) + (size_t)s * 32;
-  codes[lane] = (uint8_t)byte;
-  if (lane == 0) {
-    uint32_t* sca = reinterpret_cast<uint32_t*>(A.arena + (side ? d->off_scales_v : d->off_scales_k));
-    sca[s] = sch | (mnh << 16);
-  }
+  // record r of its tile: the rank of the token among the tile's tokens with this side's bit
+  const int ts = w.inv[p], j = ts / kTile, tl = ts % kTile;
+  const int n = tile_len(d->len, j), nw = (int)tile_words(n), n64 = 64 * nw;
+  const int nkj = (int)w.tcnt[2 * j], nvj = (int)w.tcnt[2 * j + 1];
+  const uint8_t* blkc = A.arena_c + d->off_tiles + reinterpret_cast<const uint32_t*>(A.arena_c + d->off_tile_table)[j];
+  const uint64_t word = reinterpret_cast<const uint64_t*>(blkc + 8u * n64)[side * nw + (tl >> 6)];
+  const uint16_t* rk = reinterpret_cast<const uint16_t*>(blkc + 8u * n64 + 16u * nw + side * round16(2u * nw));
+  const int r = (int)rk[tl >> 6] + __popcll(word & ((1ull << (tl & 63)) - 1ull));
+  const uint32_t F = tile_fixed_bytes(n);
+  const uint32_t sm_off = F + (side ? round16(4u * (uint32_t)nkj) : 0u) + 4u * (uint32_t)r;
+  const uint32_t cd_off = F + round16(4u * (uint32_t)nkj) + round16(4u * (uint32_t)nvj) +
+                          (side ? 32u * (uint32_t)nkj : 0u) + 32u * (uint32_t)r;
+  uint8_t* blk = const_cast<uint8_t*>(blkc);
+  blk[cd_off + lane] = (uint8_t)byte;
+  if (lane == 0) *reinterpret_cast<uint32_t*>(blk + sm_off) = sch | (mnh << 16);
 }
 
 }  // namespace
@@ -552,7 +720,12 @@ int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const
   if ((e = cudaFuncSetAttribute(enc_assign, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AS_SMEM)) != cudaSuccess)
     return (int)e;
   enc_assign<<<dim3((maxS + AS_POS - 1) / AS_POS, units, 2), AS_THREADS, AS_SMEM, st>>>(A);
-  enc_slots<<<dim3(units, 2), 1024, 0, st>>>(A);
+  enc_slots<<<units, 1024, 0, st>>>(A, 0);  // writes the flag bytes
+  enc_slots<<<units, 1024, 0, st>>>(A, 1);  // ORs the value bit in
+  enc_order<<<units, 1024, 0, st>>>(A);
+  enc_tile_count<<<dim3((unsigned)L.max_tiles, units), kTile, 0, st>>>(A);
+  enc_tile_table<<<(units + 127) / 128, 128, 0, st>>>(A, units);
+  enc_tile_fill<<<dim3((unsigned)L.max_tiles, units), kTile, 0, st>>>(A);
   const int maxN = std::max(L.max_nk, L.max_nv);
   if (maxN > 0) enc_quant<<<dim3((unsigned)(maxN + 7) / 8, units, 2), 256, 0, st>>>(A);
   return (int)cudaGetLastError();

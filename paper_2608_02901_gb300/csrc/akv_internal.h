@@ -20,14 +20,30 @@ constexpr uint64_t kTailPad = 256;  // bytes after the last section, so 16-byte 
 static_assert(sizeof(akv_arena_header) == 256, "header must be 256 bytes");
 static_assert(sizeof(akv_unit_desc) == 256, "descriptor must be 256 bytes");
 
+#ifdef __CUDACC__
+#define AKV_HD __host__ __device__
+#else
+#define AKV_HD
+#endif
+
+constexpr int kTile = AKV_TILE_TOKENS;
+
+// Geometry of one tile block (the layout documented with akv_unit_desc).
+AKV_HD constexpr uint32_t round16(uint32_t x) { return (x + 15u) & ~15u; }
+AKV_HD constexpr uint32_t tile_words(int n) { return (uint32_t)(n + 63) / 64u; }
+// streams, bitmaps and rank words of a tile of n tokens
+AKV_HD constexpr uint32_t tile_fixed_bytes(int n) {
+  return 8u * 64u * tile_words(n) + 16u * tile_words(n) + 2u * round16(2u * tile_words(n));
+}
+AKV_HD constexpr uint32_t tile_block_bytes(int n, int nk, int nv) {
+  return tile_fixed_bytes(n) + round16(4u * (uint32_t)nk) + round16(4u * (uint32_t)nv) + 32u * (uint32_t)(nk + nv);
+}
+
 // Section indices inside one unit segment, in storage order.
-enum Section {
-  kAnchorK = 0, kAnchorV, kAnchorPos, kStreamK, kStreamV, kBitmapK, kPrefixK, kBitmapV, kPrefixV,
-  kCodesK, kScalesK, kCodesV, kScalesV, kNumSections
-};
+enum Section { kAnchorK = 0, kAnchorV, kAnchorPos, kTileTable, kTiles, kNumSections };
 
 struct UnitShape {
-  int32_t S = 0, k = 0, nk = 0, nv = 0;
+  int32_t S = 0, k = 0, nk = 0, nv = 0, nt = 0;
 };
 
 struct Layout {
@@ -35,7 +51,7 @@ struct Layout {
   std::vector<akv_unit_desc> desc;     // per unit, offsets from the arena base
   akv_arena_header header{};
   uint64_t total_bytes = 0;
-  int32_t max_len = 0, max_k = 0, max_nk = 0, max_nv = 0;
+  int32_t max_len = 0, max_k = 0, max_nk = 0, max_nv = 0, max_tiles = 0;
   int G = 0;
 };
 

@@ -50,6 +50,40 @@ def check_outputs(out_bf16: np.ndarray, out_f32: np.ndarray, ref: np.ndarray, wh
     return e16.max(), e16.mean(), e32.max()
 
 
+UNIT_FIELDS = ("anchor_k", "anchor_v", "anchor_pos", "idx_k", "gam_k", "idx_v", "gam_v", "res_k", "codes_k",
+               "scale_k", "min_k", "res_v", "codes_v", "scale_v", "min_v")
+
+
+def stored_order(u) -> dict:
+    """A unit's logical arrays (a dict or an oracle.Unit, indexed by position) rearranged
+    into the arena's stored order: tokens sorted by value anchor slot, ties by position.
+    Residual lists become the sorted stored indices, their records moved along."""
+    get = (lambda n: np.asarray(u[n])) if isinstance(u, dict) else (lambda n: np.asarray(getattr(u, n)))
+    idx_v = get("idx_v")
+    perm = np.argsort(idx_v, kind="stable")
+    inv = np.empty_like(perm)
+    inv[perm] = np.arange(perm.size)
+    out = {n: get(n) for n in ("anchor_k", "anchor_v", "anchor_pos")}
+    for n in ("idx_k", "gam_k", "idx_v", "gam_v"):
+        out[n] = get(n)[perm]
+    for side in ("k", "v"):
+        st = inv[get("res_" + side)]
+        order = np.argsort(st, kind="stable")
+        out["res_" + side] = st[order].astype(np.int32)
+        for n in ("codes_", "scale_", "min_"):
+            out[n + side] = get(n + side)[order]
+    return out
+
+
+def assert_same_unit(got, want: dict, where: str = ""):
+    for f in UNIT_FIELDS:
+        a, b = np.asarray(getattr(got, f)), np.asarray(want[f])
+        if not np.array_equal(a, b):
+            bad = np.flatnonzero((a != b).reshape(a.shape[0], -1).any(axis=1)) if a.ndim and a.shape == b.shape else []
+            raise AssertionError(f"{where} field {f}: shapes {a.shape}/{b.shape}, {len(bad)} mismatching rows, "
+                                 f"first {bad[:5]}")
+
+
 def to_dev_u16(a: np.ndarray, torch, dev, dtype=None):
     t = torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev)
     return t.view(dtype or torch.bfloat16)

@@ -10,6 +10,7 @@ import gen
 import oracle
 from oracle import accounting as acc
 import paper_2608_02901_gb300 as akv
+from helpers import assert_same_unit, stored_order
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
@@ -51,30 +52,37 @@ def test_unit_shapes_match_oracle(S, fr):
 
 
 def test_layout_header_and_sections():
-    lens = [4096, 1000, 33]
-    p = akv.Params(batch=3, n_kv_heads=2, n_q_heads=8, seed=3, rot_seed=9)
+    lens = [4096, 1000, 33, 5000]
+    p = akv.Params(batch=4, n_kv_heads=2, n_q_heads=8, seed=3, rot_seed=9)
     arena_bytes, ws_bytes = akv.akv_cache_size(p, lens)
     hdr = akv.akv_cache_header_host(p, lens)
-    assert hdr[:4].view(np.uint32)[0] == 0x31564B41 and hdr[4:8].view(np.uint32)[0] == 1
+    assert hdr[:4].view(np.uint32)[0] == 0x32564B41 and hdr[4:8].view(np.uint32)[0] == 2
     assert hdr[8:16].view(np.uint64)[0] == arena_bytes
-    assert hdr[72:76].view(np.int32)[0] == 6 and hdr[76:80].view(np.int32)[0] == 4096
+    assert hdr[72:76].view(np.int32)[0] == 8 and hdr[76:80].view(np.int32)[0] == 5000
+    assert hdr[104:108].view(np.int32)[0] == 1024
     # sign bits: s_j = -1 iff bit j set, the same pattern the oracle derives from rot_seed
     bits = hdr[88:104].view(np.uint64)
     s = np.array([-1.0 if (int(bits[j // 64]) >> (j % 64)) & 1 else 1.0 for j in range(128)])
     assert np.array_equal(s, oracle.signs(9))
-    prev_end = 256 * 7
-    for u in range(6):
+    prev_end = 256 * 9
+    for u in range(8):
         d = hdr[256 * (u + 1): 256 * (u + 2)]
-        S, k, nk, nv, nw, b, h = d[:28].view(np.int32)
-        assert (b, h) == (u // 2, u % 2) and S == lens[b] and nw == (S + 63) // 64
-        offs = d[32:136].view(np.uint64)
-        sizes = [k * 256, k * 256, 4 * k, 4 * S, 4 * S, 8 * nw, 4 * nw, 8 * nw, 4 * nw, 32 * nk, 4 * nk, 32 * nv, 4 * nv]
+        S, k, nk, nv, nt, b, h = d[:28].view(np.int32)
+        assert (b, h) == (u // 2, u % 2) and S == lens[b] and nt == (S + 1023) // 1024
+        offs = d[32:72].view(np.uint64)
+        cap, data = (int(x) for x in d[72:88].view(np.uint64))
+        # fixed part of every tile (streams, bitmaps, rank words), records, <= 24 B padding per tile
+        fixed = 0
+        for j in range(nt):
+            nw = (min(1024, S - 1024 * j) + 63) // 64
+            fixed += 512 * nw + 16 * nw + 2 * ((2 * nw + 15) // 16 * 16)
+        assert cap == fixed + 36 * (nk + nv) + 24 * nt
+        sizes = [k * 256, k * 256, 4 * k, 4 * (nt + 1), cap]
         assert offs[0] % 256 == 0
         for o, sz in zip(offs, sizes):
             assert o % 128 == 0 and o >= prev_end
             prev_end = o + sz
-        data = int(d[136:144].view(np.uint64)[0])
-        assert data == acc.decode_read_bytes(S, k, nk, nv, G=0)
+        assert data == 512 * k + 4 * (nt + 1) + cap
     assert prev_end <= arena_bytes
     assert ws_bytes > 0
 
@@ -92,10 +100,39 @@ def test_pack_roundtrip_through_independent_unpacker():
     arena = akv.akv_cache_pack_host(p, lens, [akv.unit_host_from_logical(u) for u in units])
     back = oracle.unpack_arena(arena)
     assert len(back) == len(units)
-    for u, b in zip(units, back):
+    for i, (u, b) in enumerate(zip(units, back)):
+        assert_same_unit(b, stored_order(u), f"unit {i}")
+    # attention does not depend on the token order: the unpacked (stored-order) units
+    # attend exactly like the position-ordered ones
+    q = gen.queries(p.n_units * p.G, seed=3).reshape(p.n_units, p.G, 128)
+    pos_units = [oracle.alloc_unit(d["S"], d["k"], d["nk"], d["nv"]) for d in units]
+    for pu, d in zip(pos_units, units):
         for name in ("anchor_k", "anchor_v", "anchor_pos", "idx_k", "gam_k", "idx_v", "gam_v", "res_k", "codes_k",
                      "scale_k", "min_k", "res_v", "codes_v", "scale_v", "min_v"):
-            assert np.array_equal(np.asarray(u[name]), getattr(b, name)), name
+            getattr(pu, name)[...] = d[name]
+    a = oracle.attend(pos_units, q, p.G, 1.0, p.rot_seed, p.rotate)
+    b = oracle.attend(back, q, p.G, 1.0, p.rot_seed, p.rotate)
+    assert np.max(np.abs(a - b)) <= 1e-12 * max(1.0, np.max(np.abs(a)))
+
+
+def test_stored_order_is_sorted_by_value_anchor_and_tiles_are_consistent():
+    lens = [3000]
+    p = akv.Params(batch=1, n_kv_heads=1, n_q_heads=1, anchor_frac=0.01, res_frac_k=0.2, res_frac_v=0.1)
+    units = _seeded_units(p, lens, seed=9)
+    arena = akv.akv_cache_pack_host(p, lens, [akv.unit_host_from_logical(u) for u in units])
+    back = oracle.unpack_arena(arena)[0]
+    assert np.all(np.diff(back.idx_v.astype(np.int64)) >= 0)
+    hdr = akv.akv_cache_header_host(p, lens)
+    d = hdr[256:512]
+    o_tt = int(d[56:64].view(np.uint64)[0])
+    nt = int(d[16:20].view(np.int32)[0])
+    table = arena[o_tt:o_tt + 4 * (nt + 1)].view(np.uint32)
+    assert table[0] == 0 and np.all(np.diff(table.astype(np.int64)) > 0) and np.all(table % 16 == 0)
+    # a damaged table is refused by the independent reader
+    bad = arena.copy()
+    bad[o_tt + 4:o_tt + 8] = np.frombuffer(np.uint32(table[1] + 16).tobytes(), np.uint8)
+    with pytest.raises(ValueError):
+        oracle.unpack_arena(bad)
 
 
 def _err(fn, *a):
