@@ -64,7 +64,7 @@ constexpr int W_PROD = W_VRES + NVR;   // producer warp
 constexpr int NT = (W_PROD + 1) * 32;  // 480 threads
 constexpr int T = kTile;               // tokens per tile block
 constexpr int REG = T / NTW;           // tokens of a tile per token warp
-static_assert(REG % 128 == 0, "a token warp's region holds whole iterations of 8 slices");
+static_assert(REG == 128, "a token lane's chunk (REG * GS / 32 tokens) lies in one bitmap word");
 static_assert(NTW % NVR == 0, "value-residual warps release a stage with NTW / NVR arrivals each");
 constexpr int CH = 64;                 // anchor rows per chunk item
 constexpr int ROWE = 80;               // stride of an expanded row of 32 codes (64 B + 16 B pad)
@@ -264,8 +264,6 @@ struct TileView {
   int n, nw, n64, nk, nv;
   uint32_t sm_k, sm_v, cd_k, cd_v;  // byte offsets of scales and codes in the block
   __device__ __forceinline__ const uint8_t* at(uint32_t off) const { return off < staged ? st + off : gb + off; }
-  __device__ __forceinline__ uint32_t kst(int t) const { return reinterpret_cast<const uint32_t*>(st)[t]; }
-  __device__ __forceinline__ uint32_t vst(int t) const { return reinterpret_cast<const uint32_t*>(st)[n64 + t]; }
   __device__ __forceinline__ uint64_t bm(int side, int w) const {
     return reinterpret_cast<const uint64_t*>(st + 8 * n64)[side * nw + w];
   }
@@ -293,22 +291,30 @@ __device__ __forceinline__ TileView tile_view(const uint8_t* st, const uint2 met
   return v;
 }
 
-// q'_g . c of one key record on CUDA cores (records beyond the staged count).
-__device__ float key_record_dot(const TileView& tv, int r, const float* qpg) {
-  const uint8_t* rec = tv.at(tv.cd_k + 32u * (uint32_t)r);
-  const uint8_t* rec2 = tv.at(tv.cd_k + 32u * (uint32_t)r + 16u);
+// Records beyond the staged count (a locally dense tile) take these rare paths on CUDA
+// cores, kept out of line so that the token loop stays small.
+// Key residual term scale (q'_g . c) + min sum(q'_g) of key record r.
+__device__ __noinline__ float key_record_term(const TileView& tv, int r, const float* qpg, float sqg) {
+  const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_k + 4u * (uint32_t)r));
   float dot = 0.f;
   for (int bb = 0; bb < 32; ++bb) {
-    const uint32_t byte = bb < 16 ? rec[bb] : rec2[bb - 16];
+    const uint32_t byte = *tv.at(tv.cd_k + 32u * (uint32_t)r + (uint32_t)bb);
 #pragma unroll
     for (int c = 0; c < 4; ++c) dot += qpg[4 * bb + c] * (float)((byte >> (2 * c)) & 3u);
   }
-  return dot;
+  return half_hi(smn) * sqg + half_lo(smn) * dot;
+}
+// accg += ps * c of value record r (rotated domain).
+__device__ __noinline__ void value_record_add(const TileView& tv, int r, float ps, float* accg) {
+  for (int bb = 0; bb < 32; ++bb) {
+    const uint32_t byte = *tv.at(tv.cd_v + 32u * (uint32_t)r + (uint32_t)bb);
+#pragma unroll
+    for (int c = 0; c < 4; ++c) atomicAdd(&accg[4 * bb + c], ps * (float)((byte >> (2 * c)) & 3u));
+  }
 }
 
 template <int GS>
 __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P) {
-  constexpr int SPI = 8 / GS;  // 16-token slices per iteration: every lane computes one (slice, head)
   extern __shared__ __align__(128) uint8_t smem[];
   cg::cluster_group cluster = cg::this_cluster();
   const int C = P.cluster;
@@ -457,29 +463,41 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         const TileView tv = tile_view(stage(s), meta[s], U, j0 + tl, P.cap);
         const int nK = min(tv.nk, R);
         float* rs = reinterpret_cast<float*>(stage(s) + P.o_rs);
-        for (int g8 = kw; g8 * 8 < nK; g8 += NKR) {
-          const int sl = g8 * 8 + r8;  // the record whose codes this lane feeds (B column r8)
-          uint4 w0 = make_uint4(0u, 0u, 0u, 0u), w1 = w0;
-          if (sl < nK) {
-            w0 = *reinterpret_cast<const uint4*>(tv.at(tv.cd_k + 32u * (uint32_t)sl));
-            w1 = *reinterpret_cast<const uint4*>(tv.at(tv.cd_k + 32u * (uint32_t)sl + 16u));
-          }
-          const uint32_t wd[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
-          float d[4] = {0.f, 0.f, 0.f, 0.f};
+        // two groups of 8 records at a time, each as two independent mma chains
+        for (int g8 = kw; g8 * 8 < nK; g8 += 2 * NKR) {
+          const int gsel[2] = {g8, g8 + NKR};
+          uint32_t wd[2][8];
 #pragma unroll
-          for (int ks = 0; ks < 8; ++ks) {
-            const uint32_t x = wd[ks] >> (4 * c4);
-            mma_f16(d, af[ks], codes2_to_h2(x), codes2_to_h2(x >> 2));
+          for (int q = 0; q < 2; ++q) {
+            const int sl = gsel[q] * 8 + r8;  // the record whose codes this lane feeds (B column r8)
+            uint4 w0 = make_uint4(0u, 0u, 0u, 0u), w1 = w0;
+            if (sl < nK) {
+              w0 = *reinterpret_cast<const uint4*>(tv.at(tv.cd_k + 32u * (uint32_t)sl));
+              w1 = *reinterpret_cast<const uint4*>(tv.at(tv.cd_k + 32u * (uint32_t)sl + 16u));
+            }
+            wd[q][0] = w0.x; wd[q][1] = w0.y; wd[q][2] = w0.z; wd[q][3] = w0.w;
+            wd[q][4] = w1.x; wd[q][5] = w1.y; wd[q][6] = w1.z; wd[q][7] = w1.w;
           }
+          float d[2][2][4] = {};
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks)
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const uint32_t x = wd[q][ks] >> (4 * c4);
+              mma_f16(d[q][ks & 1], af[ks], codes2_to_h2(x), codes2_to_h2(x >> 2));
+            }
           if (r8 < GS) {  // D rows r8 (high parts) and r8 + 8 (low parts), columns 2c, 2c+1
 #pragma unroll
-            for (int e2 = 0; e2 < 2; ++e2) {
-              const int sl2 = g8 * 8 + 2 * c4 + e2;
-              if (sl2 < nK) {
-                const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_k + 4u * (uint32_t)sl2));
-                rs[sl2 * GS + r8] = half_hi(smn) * sq[r8] + half_lo(smn) * (d[e2] + d[2 + e2]);
+            for (int q = 0; q < 2; ++q)
+#pragma unroll
+              for (int e2 = 0; e2 < 2; ++e2) {
+                const int sl2 = gsel[q] * 8 + 2 * c4 + e2;
+                if (sl2 < nK) {
+                  const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_k + 4u * (uint32_t)sl2));
+                  const float dot = (d[q][0][e2] + d[q][1][e2]) + (d[q][0][2 + e2] + d[q][1][2 + e2]);
+                  rs[sl2 * GS + r8] = half_hi(smn) * sq[r8] + half_lo(smn) * dot;
+                }
               }
-            }
           }
         }
       }
@@ -503,12 +521,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   if (warp >= W_VRES && warp < W_VRES + NVR) {
     const int vw = warp - W_VRES;
     cluster_arrive();  // B1
-    float accV[4][4];
-#pragma unroll
-    for (int nb = 0; nb < 4; ++nb)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) accV[nb][e] = 0.f;
-    uint8_t* ew = ebuf + vw * 16 * ROWE;
+    float accV[2][4][4] = {};  // two independent sets (alternate groups), summed at the end
+    uint8_t* ew = ebuf + vw * 2 * 16 * ROWE;
     bool ok = true;
     for (int tl = 0; tl < n_t; ++tl) {
       const int s = (n_ka + tl) % NS;
@@ -521,29 +535,35 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         const TileView tv = tile_view(stage(s), meta[s], U, j0 + tl, P.cap);
         const int nV = min(tv.nv, R);
         const uint8_t* pf = stage(s) + P.o_pf;
-        for (int grp = 0; grp * 16 < nV; ++grp) {
+        for (int grp = 0; grp * 16 < nV; grp += 2) {
           const int n = lane >> 1, hh = lane & 1;
-          const int sl = grp * 16 + n;
-          uint32_t x = 0;
-          if (sl < nV) x = *reinterpret_cast<const uint32_t*>(tv.at(tv.cd_v + 32u * (uint32_t)sl + 8u * vw + 4u * hh));
-          uint4 v0, v1;
-          {
+#pragma unroll
+          for (int q = 0; q < 2; ++q) {
+            const int sl = (grp + q) * 16 + n;
+            uint32_t x = 0;
+            if (sl < nV) x = *reinterpret_cast<const uint32_t*>(tv.at(tv.cd_v + 32u * (uint32_t)sl + 8u * vw + 4u * hh));
             const uint32_t lo = x & 0xFFFFu, y = lo | (lo << 14);  // code 2m at bit 4m, code 2m+1 at 4m + 16
-            v0 = make_uint4(codes2_to_b2(y), codes2_to_b2(y >> 4), codes2_to_b2(y >> 8), codes2_to_b2(y >> 12));
             const uint32_t hi = x >> 16, z = hi | (hi << 14);
-            v1 = make_uint4(codes2_to_b2(z), codes2_to_b2(z >> 4), codes2_to_b2(z >> 8), codes2_to_b2(z >> 12));
+            uint8_t* e = ew + q * 16 * ROWE;
+            *reinterpret_cast<uint4*>(e + n * ROWE + hh * 32) =
+                make_uint4(codes2_to_b2(y), codes2_to_b2(y >> 4), codes2_to_b2(y >> 8), codes2_to_b2(y >> 12));
+            *reinterpret_cast<uint4*>(e + n * ROWE + hh * 32 + 16) =
+                make_uint4(codes2_to_b2(z), codes2_to_b2(z >> 4), codes2_to_b2(z >> 8), codes2_to_b2(z >> 12));
           }
-          *reinterpret_cast<uint4*>(ew + n * ROWE + hh * 32) = v0;
-          *reinterpret_cast<uint4*>(ew + n * ROWE + hh * 32 + 16) = v1;
           __syncwarp();
-          const uint4 a = *reinterpret_cast<const uint4*>(pf + grp * 512 + lane * 16);
           const int mi = lane >> 3, ri = lane & 7;
 #pragma unroll
-          for (int half = 0; half < 2; ++half) {
-            uint32_t b00, b01, b10, b11;
-            ldsm_x4_trans(smem_u32(ew + ((mi & 1) * 8 + ri) * ROWE + half * 32 + (mi >> 1) * 16), b00, b01, b10, b11);
-            mma_bf16(accV[2 * half], a.x, a.y, a.z, a.w, b00, b01);
-            mma_bf16(accV[2 * half + 1], a.x, a.y, a.z, a.w, b10, b11);
+          for (int q = 0; q < 2; ++q) {
+            if ((grp + q) * 16 >= nV) break;  // warp-uniform
+            const uint4 a = *reinterpret_cast<const uint4*>(pf + (grp + q) * 512 + lane * 16);
+            const uint8_t* e = ew + q * 16 * ROWE;
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+              uint32_t b00, b01, b10, b11;
+              ldsm_x4_trans(smem_u32(e + ((mi & 1) * 8 + ri) * ROWE + half * 32 + (mi >> 1) * 16), b00, b01, b10, b11);
+              mma_bf16(accV[q][2 * half], a.x, a.y, a.z, a.w, b00, b01);
+              mma_bf16(accV[q][2 * half + 1], a.x, a.y, a.z, a.w, b10, b11);
+            }
           }
           __syncwarp();
         }
@@ -558,8 +578,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
       for (int nb = 0; nb < 4; ++nb) {
         const int col = 32 * vw + 8 * nb + 2 * c4;
-        atomicAdd(&accs[r8 * 128 + col], accV[nb][0] + accV[nb][2]);
-        atomicAdd(&accs[r8 * 128 + col + 1], accV[nb][1] + accV[nb][3]);
+        atomicAdd(&accs[r8 * 128 + col], (accV[0][nb][0] + accV[0][nb][2]) + (accV[1][nb][0] + accV[1][nb][2]));
+        atomicAdd(&accs[r8 * 128 + col + 1], (accV[0][nb][1] + accV[0][nb][3]) + (accV[1][nb][1] + accV[1][nb][3]));
       }
     }
     cluster_wait();  // B1
@@ -587,7 +607,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   for (int e = a0 * GS + tid; e < a1 * GS; e += NTT) SA[e] = 0.f;
   for (int e = tid; e < kc * GS; e += NTT) Wt[e] = 0.f;  // before B1: peers add into it only after B1
   for (int s = 0; s < NS; ++s)
-    for (int e = tid; e < ((R + 15) / 16) * 128; e += NTT)
+    for (int e = tid; e < ((R + 15) / 16 + 1) * 128; e += NTT)
       reinterpret_cast<uint32_t*>(stage(s) + P.o_pf)[e] = 0u;
   if (P.rotate) tw_wht_rows(qp, GS);
   else tw_sync();
@@ -709,11 +729,14 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     }
     tw_sync();
   }
-  // lane roles of the token pass: head g_own of slice js (of SPI slices per iteration)
-  const int g_own = r8 % GS, js = r8 / GS;
+  // lane roles of the token pass: head g_own (adjacent lanes), and a chunk of LT consecutive
+  // stored tokens of the warp's 128-token region of each tile
+  constexpr int LT = REG * GS / 32;  // 16, 8 or 4 tokens
+  const int g_own = lane % GS, chunk = lane / GS;
   const float m_own = mref[g_own];
   float l_part = 0.f, pmin = 0.f;
   const float* qp_own = qp + g_own * 128;
+  const int spare_grp = (R + 15) / 16;  // value operands of tokens without a value residual go here
 
   // ---- phase 2: tile blocks ----
   bool overflow_risk = false;
@@ -729,191 +752,136 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       const TileView tv = tile_view(st, meta[s], U, j0 + tl, P.cap);
       const float* rsb = reinterpret_cast<const float*>(st + P.o_rs);
       uint8_t* pfb = const_cast<uint8_t*>(st) + P.o_pf;
-      // value-weight accumulator of a window of 16 anchors [abase, abase + 16): rows are
-      // anchors, columns c < GS the high part of head c, GS <= c < 2 GS the low part of
-      // head c - GS
-      float D[4] = {0.f, 0.f, 0.f, 0.f};
-      int abase = 0;
-      bool live = false;
-      auto flush = [&]() {
-        float v[4] = {D[0], D[1], D[2], D[3]};
-        if constexpr (GS == 4) {
-#pragma unroll
-          for (int e = 0; e < 4; ++e) v[e] += __shfl_xor_sync(0xffffffffu, v[e], 2);
-        } else if constexpr (GS == 2) {
-#pragma unroll
-          for (int e = 0; e < 4; ++e) v[e] += __shfl_xor_sync(0xffffffffu, v[e], 1);
-        } else {
-          v[0] += v[1];
-          v[2] += v[3];
-        }
-        if (2 * c4 < GS || (GS == 1 && c4 == 0)) {
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            if (GS == 1 && (e & 1)) continue;
-            const int row = r8 + 8 * (e >> 1);
-            const int g = GS == 1 ? 0 : 2 * c4 + (e & 1);
-            const int a = abase + row;
-            if (v[e] != 0.f && a < k) {
-              const int owner = a / kc;
-              red_cluster(&Wt[(a - owner * kc) * GS + g], owner, v[e]);
+      const int t0 = warp * REG + chunk * LT;  // a multiple of LT: the chunk sits in one bitmap word
+      const int te = min(t0 + LT, tv.n);
+      if (t0 < te) {
+        const int wi = t0 >> 6, sh = t0 & 63;
+        const uint64_t wk = tv.bm(0, wi), wv = tv.bm(1, wi);
+        const uint64_t below = (1ull << sh) - 1ull;
+        int rkn = tv.rk(0, wi) + __popcll(wk & below);  // record of the next key-residual token
+        int rvn = tv.rk(1, wi) + __popcll(wv & below);
+        const uint32_t bk = (uint32_t)(wk >> sh), bv = (uint32_t)(wv >> sh);
+        // value weights: the sum over the current run of equal value anchors, in a register
+        int cur = (int)(*reinterpret_cast<const uint32_t*>(tv.st + 4 * (tv.n64 + t0)) & 0xFFFFu);
+        float acc = 0.f;
+        auto flush = [&]() {
+          if (acc != 0.f && cur < k) {
+            if (cur >= a0 && cur < a1) {  // this CTA owns the anchor
+              atomicAdd(&Wt[(cur - a0) * GS + g_own], acc);
+            } else {
+              const int owner = cur / kc;
+              red_cluster(&Wt[(cur - owner * kc) * GS + g_own], owner, acc);
             }
           }
-        }
+        };
+        const uint32_t lmask = LT == 32 ? 0xFFFFFFFFu : ((1u << LT) - 1u);
+        const bool staged_all = rkn + __popc(bk & lmask) <= R && rvn + __popc(bv & lmask) <= R;
+        if (staged_all) {
+          // every record of the chunk is staged: no branch but the run change; tokens without a
+          // residual read record 0 and write their (zero) value operand to the spare group
+#pragma unroll 1
+          for (int q4 = t0; q4 < te; q4 += 4) {  // 16-byte loads; entries past n (< n64) read as 0
+            const uint4 ka = *reinterpret_cast<const uint4*>(tv.st + 4 * q4);
+            const uint4 va = *reinterpret_cast<const uint4*>(tv.st + 4 * (tv.n64 + q4));
+            const uint32_t ek[4] = {ka.x, ka.y, ka.z, ka.w}, ev[4] = {va.x, va.y, va.z, va.w};
 #pragma unroll
-        for (int e = 0; e < 4; ++e) D[e] = 0.f;
-      };
-      const int rbeg = warp * REG;
-      for (int sb = rbeg; sb < rbeg + REG && sb < tv.n; sb += 16 * SPI) {
-        // ---- this lane's slice js: four tokens, head g_own ----
-        const int tb = sb + 16 * js;
-        const int tt[4] = {tb + 2 * c4, tb + 2 * c4 + 1, tb + 2 * c4 + 8, tb + 2 * c4 + 9};
-        float cval[4] = {0.f, 0.f, 0.f, 0.f};
-        uint32_t av_own[4] = {0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu};
-        if (tb < tv.n) {  // then tb + 15 < n64: every read below stays inside the tile's arrays
-          const int wi = tb >> 6;
-          const uint64_t wk = tv.bm(0, wi), wv = tv.bm(1, wi);
-          const int rk0 = tv.rk(0, wi), rv0 = tv.rk(1, wi);
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int t = tt[e];
-            if (t >= tv.n) continue;  // past the tile's last token: p = 0, no anchor
-            const uint32_t ek = tv.kst(t), ev = tv.vst(t);
-            av_own[e] = ev & 0xFFFFu;
-            const int a = min((int)(ek & 0xFFFFu), k - 1);  // indices are < k by construction; never read past
-            float x = half_hi(ek) * SA[a * GS + g_own];
-            const uint64_t below = (1ull << (t & 63)) - 1ull;
-            if ((wk >> (t & 63)) & 1ull) {  // key residual term
-              const int r = rk0 + __popcll(wk & below);
-              if (r < R) {
-                x += rsb[r * GS + g_own];
-              } else {  // beyond the staged records (a locally dense tile): CUDA cores
-                const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_k + 4u * (uint32_t)r));
-                x += half_hi(smn) * sq[g_own] + half_lo(smn) * key_record_dot(tv, r, qp_own);
+            for (int e = 0; e < 4; ++e) {
+              if (q4 + e >= te) break;
+              const int bit = q4 + e - t0;
+              const int a = min((int)(ek[e] & 0xFFFFu), k - 1);  // indices are < k by construction
+              const uint32_t kb = (bk >> bit) & 1u, vb = (bv >> bit) & 1u;
+              const float rt = rsb[(kb ? rkn : 0) * GS + g_own];
+              rkn += (int)kb;
+              float x = fmaf(half_hi(ek[e]), SA[a * GS + g_own], kb ? rt : 0.f) - m_own;
+              overflow_risk |= x > 120.f;
+              const float p = exp2f(x);
+              l_part += p;
+              const int av = (int)(ev[e] & 0xFFFFu);
+              if (av != cur) {  // stored order: a new run of value anchor av
+                flush();
+                cur = av;
+                acc = 0.f;
               }
+              acc = fmaf(p, half_hi(ev[e]), acc);
+              const int r = vb ? rvn : 0;
+              rvn += (int)vb;
+              uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.st + tv.sm_v + 4u * (uint32_t)r);
+              smn = vb ? smn : 0u;
+              pmin = fmaf(p, half_hi(smn), pmin);
+              __nv_bfloat16 hi, lo;
+              split_b(p * half_lo(smn), hi, lo);
+              const int grp = vb ? (r >> 4) : spare_grp, kk = r & 15;
+              const int comp = (kk >> 3) * 2, hf = kk & 1, cc = (kk & 7) >> 1;
+              unsigned short* dst = reinterpret_cast<unsigned short*>(pfb + grp * 512 + (4 * g_own + cc) * 16);
+              dst[comp * 2 + hf] = __bfloat16_as_ushort(hi);
+              dst[(comp + 1) * 2 + hf] = __bfloat16_as_ushort(lo);
             }
-            x -= m_own;
-            overflow_risk |= x > 120.f;
-            const float p = exp2f(x);
-            l_part += p;
-            cval[e] = p * half_hi(ev);
-            if ((wv >> (t & 63)) & 1ull) {  // value residual: A operand of its group, or overflow
-              const int r = rv0 + __popcll(wv & below);
-              const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_v + 4u * (uint32_t)r));
-              const float scl = half_lo(smn), mn = half_hi(smn);
-              pmin += p * mn;
-              if (r < R) {
-                const int grp = r >> 4, kk = r & 15;
-                const int comp = (kk >> 3) * 2, hf = kk & 1, cc = (kk & 7) >> 1;
-                __nv_bfloat16 hi, lo;
-                split_b(p * scl, hi, lo);
-                unsigned short* dst = reinterpret_cast<unsigned short*>(pfb + grp * 512 + (4 * g_own + cc) * 16);
-                dst[comp * 2 + hf] = __bfloat16_as_ushort(hi);
-                dst[(comp + 1) * 2 + hf] = __bfloat16_as_ushort(lo);
-              } else {
-                const float ps = p * scl;
-                for (int bb = 0; bb < 32; ++bb) {
-                  const uint32_t byte = *tv.at(tv.cd_v + 32u * (uint32_t)r + (uint32_t)bb);
+          }
+        } else {
+#pragma unroll 1
+          for (int q4 = t0; q4 < te; q4 += 4) {
+            const uint4 ka = *reinterpret_cast<const uint4*>(tv.st + 4 * q4);
+            const uint4 va = *reinterpret_cast<const uint4*>(tv.st + 4 * (tv.n64 + q4));
+            const uint32_t ek[4] = {ka.x, ka.y, ka.z, ka.w}, ev[4] = {va.x, va.y, va.z, va.w};
 #pragma unroll
-                  for (int c = 0; c < 4; ++c)
-                    atomicAdd(&accs[g_own * 128 + 4 * bb + c], ps * (float)((byte >> (2 * c)) & 3u));
+            for (int e = 0; e < 4; ++e) {
+              if (q4 + e >= te) break;
+              const int a = min((int)(ek[e] & 0xFFFFu), k - 1);
+              float x = half_hi(ek[e]) * SA[a * GS + g_own];
+              const int bit = q4 + e - t0;
+              if ((bk >> bit) & 1u) {  // key residual term
+                const int r = rkn++;
+                x += r < R ? rsb[r * GS + g_own] : key_record_term(tv, r, qp_own, sq[g_own]);
+              }
+              x -= m_own;
+              overflow_risk |= x > 120.f;
+              const float p = exp2f(x);
+              l_part += p;
+              const int av = (int)(ev[e] & 0xFFFFu);
+              if (av != cur) {
+                flush();
+                cur = av;
+                acc = 0.f;
+              }
+              acc += p * half_hi(ev[e]);
+              if ((bv >> bit) & 1u) {  // value residual: A operand of its group, or beyond the staged ones
+                const int r = rvn++;
+                const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_v + 4u * (uint32_t)r));
+                const float scl = half_lo(smn), mn = half_hi(smn);
+                pmin += p * mn;
+                if (r < R) {
+                  const int grp = r >> 4, kk = r & 15;
+                  const int comp = (kk >> 3) * 2, hf = kk & 1, cc = (kk & 7) >> 1;
+                  __nv_bfloat16 hi, lo;
+                  split_b(p * scl, hi, lo);
+                  unsigned short* dst = reinterpret_cast<unsigned short*>(pfb + grp * 512 + (4 * g_own + cc) * 16);
+                  dst[comp * 2 + hf] = __bfloat16_as_ushort(hi);
+                  dst[(comp + 1) * 2 + hf] = __bfloat16_as_ushort(lo);
+                } else {
+                  value_record_add(tv, r, p * scl, accs + g_own * 128);
                 }
               }
             }
           }
         }
-        // ---- value weights: one-hot(anchor window) x (p gamma^V) on the tensor cores ----
-#pragma unroll
-        for (int jp = 0; jp < SPI; ++jp) {
-          const int tbp = sb + 16 * jp;
-          if (tbp >= tv.n) break;
-          // B operand (tokens x columns), column r8: high or low part of head r8 % GS,
-          // computed by the lane of slice jp that holds that head
-          const int src = ((jp * GS + (r8 % GS)) << 2) | c4;
-          float bv[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) bv[e] = __shfl_sync(0xffffffffu, cval[e], src);
-          uint32_t b0, b1;
-          {
-            __nv_bfloat16 hi[4], lo[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) split_b(bv[e], hi[e], lo[e]);
-            if (r8 < GS) {
-              b0 = pack_b2(hi[0], hi[1]);
-              b1 = pack_b2(hi[2], hi[3]);
-            } else if (r8 < 2 * GS) {
-              b0 = pack_b2(lo[0], lo[1]);
-              b1 = pack_b2(lo[2], lo[3]);
-            } else {
-              b0 = b1 = 0u;
-            }
-          }
-          // anchors of this slice's tokens at the A-fragment positions (rows r8, r8 + 8)
-          uint32_t av[4];
-          if (jp == js) {
-#pragma unroll
-            for (int e = 0; e < 4; ++e) av[e] = av_own[e];
-          } else {
-            const uint2 p01 = *reinterpret_cast<const uint2*>(tv.st + 4 * (tv.n64 + tbp + 2 * c4));
-            const uint2 p89 = *reinterpret_cast<const uint2*>(tv.st + 4 * (tv.n64 + tbp + 2 * c4 + 8));
-            av[0] = p01.x & 0xFFFFu;
-            av[1] = p01.y & 0xFFFFu;
-            av[2] = p89.x & 0xFFFFu;
-            av[3] = p89.y & 0xFFFFu;
-          }
-          // stored order makes a slice's anchors non-decreasing: first and last bound them
-          const int alo = (int)(tv.vst(tbp) & 0xFFFFu);
-          const int ahi = (int)(tv.vst(min(tbp + 15, tv.n - 1)) & 0xFFFFu);
-          if (live && ahi >= abase + 16) {
-            flush();
-            live = false;
-          }
-          if (!live) {
-            abase = alo;
-            live = true;
-          }
-          for (;;) {
-            uint32_t am[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const uint32_t rel = av[e] - (uint32_t)abase;
-              const uint32_t m0 = rel == (uint32_t)r8 ? 0x3F80u : 0u, m1 = rel == (uint32_t)(r8 + 8) ? 0x3F80u : 0u;
-              am[e] = m0 | (m1 << 16);
-            }
-            // a0: row r8, tokens 2c, 2c+1; a1: row r8+8; a2, a3: tokens 2c+8, 2c+9
-            const uint32_t A0 = (am[0] & 0xFFFFu) | (am[1] << 16);
-            const uint32_t A1 = (am[0] >> 16) | (am[1] & 0xFFFF0000u);
-            const uint32_t A2 = (am[2] & 0xFFFFu) | (am[3] << 16);
-            const uint32_t A3 = (am[2] >> 16) | (am[3] & 0xFFFF0000u);
-            mma_bf16(D, A0, A1, A2, A3, b0, b1);
-            if (ahi < abase + 16) break;
-            flush();
-            abase += 16;
-          }
-        }
+        flush();
       }
-      if (live) flush();
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(bar_p(s));
   }
   if (overflow_risk) *failed = 1;  // a logit beyond 2^120 of the reference would overflow the sums
 
-  // ---- per-CTA totals: lanes with r8 % GS == g hold head g ----
+  // ---- per-CTA totals: lanes with lane % GS == g hold head g ----
   {
 #pragma unroll
-    for (int o = 1; o < 4; o <<= 1) {
+    for (int o = GS; o < 32; o <<= 1) {
       l_part += __shfl_xor_sync(0xffffffffu, l_part, o);
       pmin += __shfl_xor_sync(0xffffffffu, pmin, o);
     }
-#pragma unroll
-    for (int o = 4 * GS; o < 32; o <<= 1) {
-      l_part += __shfl_xor_sync(0xffffffffu, l_part, o);
-      pmin += __shfl_xor_sync(0xffffffffu, pmin, o);
-    }
-    if (lane < 4 * GS && c4 == 0) {
-      red[warp * GS + r8] = l_part;
-      opart[warp * GS + r8] = pmin;  // scratch until phase 3
+    if (lane < GS) {
+      red[warp * GS + lane] = l_part;
+      opart[warp * GS + lane] = pmin;  // scratch until phase 3
     }
   }
   tw_sync();
@@ -1085,7 +1053,7 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_qp = take((size_t)GS * 128 * 4);
   P.o_acc = take((size_t)GS * 128 * 4);
   P.o_opart = take((size_t)std::max(GS * 128, NTW * GS) * 4);
-  P.o_e = take((size_t)NVR * 16 * ROWE);
+  P.o_e = take((size_t)NVR * 2 * 16 * ROWE);
   P.o_misc = take((size_t)(NTW * GS + 6 * GS + 4) * 4);
   P.o_meta = take(8 * 8);
   P.o_bar = take(5 * 8 * 8);
@@ -1094,7 +1062,7 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   const int sb = (int)align128((size_t)std::max(cap, CH * 256));
   P.o_rs = sb;
   P.o_pf = (int)align128((size_t)sb + (size_t)R * GS * 4);
-  const int stage = (int)align128((size_t)P.o_pf + (size_t)((R + 15) / 16) * 512);
+  const int stage = (int)align128((size_t)P.o_pf + (size_t)((R + 15) / 16 + 1) * 512);
   P.o_ring = (int)off;
   const long long room = (long long)smem_optin - (long long)off;
   if (room < 2LL * stage) return false;
