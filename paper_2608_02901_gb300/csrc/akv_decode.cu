@@ -83,7 +83,8 @@ struct DecodeParams {
   unsigned long long sign_lo, sign_hi;
   int R, NS, stage_bytes, cap;
   int o_sa, o_w, o_qfa, o_qfk, o_qp, o_acc, o_opart, o_e, o_misc, o_meta, o_bar, o_ring;
-  int o_rs, o_pf;  // inside a stage
+  int o_pfb;       // value-residual operands, two buffers (tiles alternate)
+  int o_rs;        // inside a stage
 };
 
 // ---- device helpers ---------------------------------------------------------------
@@ -313,6 +314,35 @@ __device__ __noinline__ void value_record_add(const TileView& tv, int r, float p
   }
 }
 
+// A row of GS consecutive floats (16-, 8- or 4-byte aligned) into registers.
+template <int GS>
+__device__ __forceinline__ void load_row(const float* p, float (&out)[GS]) {
+  if constexpr (GS == 4) {
+    const float4 v = *reinterpret_cast<const float4*>(p);
+    out[0] = v.x; out[1] = v.y; out[2] = v.z; out[3] = v.w;
+  } else if constexpr (GS == 2) {
+    const float2 v = *reinterpret_cast<const float2*>(p);
+    out[0] = v.x; out[1] = v.y;
+  } else {
+    out[0] = p[0];
+  }
+}
+
+// Token t of the tile (index in stored order) holding value record r: the r-th set bit
+// of the value bitmap, found from the rank words.
+__device__ __forceinline__ int value_record_token(const TileView& tv, int r) {
+  int w = 0;
+#pragma unroll
+  for (int step = 8; step; step >>= 1)
+    if (w + step < tv.nw && tv.rk(1, w + step) <= r) w += step;
+  const int rem = r - tv.rk(1, w);
+  const uint64_t word = tv.bm(1, w);
+  const uint32_t lo = (uint32_t)word, hi = (uint32_t)(word >> 32);
+  const int plo = __popc(lo);
+  const int bit = rem < plo ? (int)__fns(lo, 0, rem + 1) : 32 + (int)__fns(hi, 0, rem - plo + 1);
+  return 64 * w + bit;
+}
+
 template <int GS>
 __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P) {
   extern __shared__ __align__(128) uint8_t smem[];
@@ -346,13 +376,13 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   uint8_t* ring = smem + P.o_ring;
   const int NS = P.NS;
   // per stage: an anchor chunk landed (full_c) / a tile block landed (full_t); stage free
-  // again (empty); key-residual terms ready (rs); probabilities written (p).  Chunk items
-  // and tiles complete different barriers, so every waiter sees every phase it waits on.
+  // again (empty: all token and value-residual warps are done with it); key-residual
+  // terms ready (rs).  Chunk items and tiles complete different barriers, so every waiter
+  // sees every phase it waits on.
   auto bar_full_c = [&](int s) { return smem_u32(bars + s); };
   auto bar_full_t = [&](int s) { return smem_u32(bars + NS + s); };
   auto bar_empty = [&](int s) { return smem_u32(bars + 2 * NS + s); };
   auto bar_rs = [&](int s) { return smem_u32(bars + 3 * NS + s); };
-  auto bar_p = [&](int s) { return smem_u32(bars + 4 * NS + s); };
   auto stage = [&](int s) { return ring + (size_t)s * P.stage_bytes; };
 
   // this CTA's anchors (it owns their value weights) and tile blocks
@@ -377,9 +407,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     for (int s = 0; s < NS; ++s) {
       mbar_init(bar_full_c(s), 1);  // the producer's expect_tx arrival; bytes complete the phase
       mbar_init(bar_full_t(s), 1);
-      mbar_init(bar_empty(s), NTW);
+      mbar_init(bar_empty(s), NTW + NVR);
       mbar_init(bar_rs(s), NKR);
-      mbar_init(bar_p(s), NTW);
     }
     *failed = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -515,26 +544,87 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   }
 
   // =========================== value-residual warps ==============================
-  // sum over staged value records of (p scale) c, 16 records per mma group (bf16 operands:
-  // p scale as high + low parts, codes exact); warp vw owns the 32 coordinates
-  // 32 vw .. 32 vw + 31 of the rotated-domain accumulator.
+  // Per tile, for the value records only: the token's probability p (recomputed from the
+  // anchor scores and the key-residual terms), then sum over records of (p scale) c on
+  // tensor cores (bf16 operands: p scale as high + low parts, codes exact), in the rotated
+  // domain.  Step 1: each warp builds the A operands of every NVR-th group of 16 records
+  // into a shared buffer (two buffers, tiles alternate); step 2: each warp multiplies all
+  // groups into the 32 coordinates 32 vw .. 32 vw + 31 it owns.  Records beyond the staged
+  // count are added on CUDA cores in step 1.
   if (warp >= W_VRES && warp < W_VRES + NVR) {
     const int vw = warp - W_VRES;
     cluster_arrive();  // B1
+    named_sync(3, NTW * 32 + NVR * 32);  // anchor-score table, references and accs are ready
     float accV[2][4][4] = {};  // two independent sets (alternate groups), summed at the end
     uint8_t* ew = ebuf + vw * 2 * 16 * ROWE;
+    // step-1 roles: record slot (lane % 16) of a group, heads hb, hb + 2, ... (hb = lane / 16)
+    constexpr int HPL = GS >= 2 ? GS / 2 : 1;
+    const int sl16 = lane & 15, hb = lane >> 4;
+    const bool head_lane = hb < GS;
+    float mv[HPL], pminv[HPL];
+#pragma unroll
+    for (int i = 0; i < HPL; ++i) {
+      mv[i] = head_lane ? mref[hb + 2 * i] : 0.f;
+      pminv[i] = 0.f;
+    }
+    const int ngrp_st = (R + 15) / 16;
     bool ok = true;
     for (int tl = 0; tl < n_t; ++tl) {
       const int s = (n_ka + tl) % NS;
       const uint32_t par = (uint32_t)(tl / NS) & 1u;
       if (ok && !warp_failed(failed)) {
-        ok = mbar_wait_w(bar_full_t(s), par) && mbar_wait_w(bar_p(s), par);
+        ok = mbar_wait_w(bar_full_t(s), par) && mbar_wait_w(bar_rs(s), par);
         if (!ok) *failed = 1;
       }
-      if (ok && !warp_failed(failed)) {
-        const TileView tv = tile_view(stage(s), meta[s], U, j0 + tl, P.cap);
-        const int nV = min(tv.nv, R);
-        const uint8_t* pf = stage(s) + P.o_pf;
+      const bool go = ok && !warp_failed(failed);
+      TileView tv;
+      uint8_t* pf = smem + P.o_pfb + (tl & 1) * ngrp_st * 512;
+      int nV = 0;
+      if (go) {
+        tv = tile_view(stage(s), meta[s], U, j0 + tl, P.cap);
+        nV = min(tv.nv, R);
+        const float* rsb = reinterpret_cast<const float*>(stage(s) + P.o_rs);
+        for (int grp = vw; grp * 16 < tv.nv; grp += NVR) {
+          const int r = grp * 16 + sl16;
+          if (r < tv.nv && head_lane) {
+            const int t = value_record_token(tv, r);
+            const uint32_t ek = reinterpret_cast<const uint32_t*>(tv.st)[t];
+            const int a = min((int)(ek & 0xFFFFu), k - 1);
+            const float gk = half_hi(ek);
+            const int wi = t >> 6;
+            const uint64_t wk = tv.bm(0, wi);
+            const bool kb = (wk >> (t & 63)) & 1ull;
+            const int rk = tv.rk(0, wi) + __popcll(wk & ((1ull << (t & 63)) - 1ull));
+            const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_v + 4u * (uint32_t)r));
+            const float scl = half_lo(smn), mn = half_hi(smn);
+#pragma unroll
+            for (int i = 0; i < HPL; ++i) {
+              const int g = hb + 2 * i;
+              float rt = 0.f;
+              if (kb) rt = rk < R ? rsb[rk * GS + g] : key_record_term(tv, rk, qp + g * 128, sq[g]);
+              const float p = exp2f(fmaf(gk, SA[a * GS + g], rt) - mv[i]);  // as the token warps form it
+              pminv[i] = fmaf(p, mn, pminv[i]);
+              const float ps = p * scl;
+              if (r < R) {
+                // A-operand place of (record r, head g): group r / 16, lane 4 g + (r % 8) / 2,
+                // register 2 ((r / 8) % 2) (high part) or + 1 (low part), half r % 2
+                __nv_bfloat16 phi, plo;
+                split_b(ps, phi, plo);
+                unsigned short* dst = reinterpret_cast<unsigned short*>(
+                    pf + grp * 512 + (4 * g + ((r & 7) >> 1)) * 16 + ((r >> 3) & 1) * 8 + (r & 1) * 2);
+                dst[0] = __bfloat16_as_ushort(phi);
+                dst[2] = __bfloat16_as_ushort(plo);
+              } else {
+                value_record_add(tv, r, ps, accs + g * 128);
+              }
+            }
+          }
+        }
+      }
+      // every warp's operands of this tile are written, and every warp is done with the
+      // other buffer (its previous tile)
+      named_sync(4, NVR * 32);
+      if (go) {
         for (int grp = 0; grp * 16 < nV; grp += 2) {
           const int n = lane >> 1, hh = lane & 1;
 #pragma unroll
@@ -569,11 +659,10 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         }
       }
       __syncwarp();
-      if (lane == 0) mbar_arrive_cnt(bar_empty(s), NTW / NVR);
+      if (lane == 0) mbar_arrive(bar_empty(s));
     }
-    // rows r8 (high parts) + r8 + 8 (low parts); overflow records were added by the token
-    // warps, which zeroed the accumulator in phase 0
-    named_sync(3, NTW * 32 + NVR * 32);
+    // rows r8 (high parts) + r8 + 8 (low parts); records beyond the staged count were added
+    // in step 1; sum p min per head
     if (r8 < GS) {
 #pragma unroll
       for (int nb = 0; nb < 4; ++nb) {
@@ -581,6 +670,12 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         atomicAdd(&accs[r8 * 128 + col], (accV[0][nb][0] + accV[0][nb][2]) + (accV[1][nb][0] + accV[1][nb][2]));
         atomicAdd(&accs[r8 * 128 + col + 1], (accV[0][nb][1] + accV[0][nb][3]) + (accV[1][nb][1] + accV[1][nb][3]));
       }
+    }
+#pragma unroll
+    for (int i = 0; i < HPL; ++i) {
+#pragma unroll
+      for (int o = 1; o < 16; o <<= 1) pminv[i] += __shfl_xor_sync(0xffffffffu, pminv[i], o);
+      if (sl16 == 0 && head_lane) atomicAdd(&pms[hb + 2 * i], pminv[i]);
     }
     cluster_wait();  // B1
     cluster_arrive();
@@ -606,9 +701,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   }
   for (int e = a0 * GS + tid; e < a1 * GS; e += NTT) SA[e] = 0.f;
   for (int e = tid; e < kc * GS; e += NTT) Wt[e] = 0.f;  // before B1: peers add into it only after B1
-  for (int s = 0; s < NS; ++s)
-    for (int e = tid; e < ((R + 15) / 16 + 1) * 128; e += NTT)
-      reinterpret_cast<uint32_t*>(stage(s) + P.o_pf)[e] = 0u;
+  for (int e = tid; e < ((R + 15) / 16) * 256; e += NTT) reinterpret_cast<uint32_t*>(smem + P.o_pfb)[e] = 0u;
+  if (tid < GS) pms[tid] = 0.f;
   if (P.rotate) tw_wht_rows(qp, GS);
   else tw_sync();
   {
@@ -648,7 +742,6 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   }
   tw_sync();
   named_arrive(2, NTW * 32 + NKR * 32);  // the key-residual warps may read q' fragments and sq
-  named_arrive(3, NTW * 32 + NVR * 32);  // the value-residual warps may add into accs
 
   bool ok = true;
   auto wait_item = [&](int i) -> const uint8_t* {
@@ -657,9 +750,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     if (!ok) *failed = 1;
     return stage(s);
   };
-  auto release_chunk = [&](int i) {
+  auto release_chunk = [&](int i) {  // the value-residual warps' share of a chunk's release: warp 0
     __syncwarp();
-    if (lane == 0) mbar_arrive(bar_empty(i % NS));
+    if (lane == 0) mbar_arrive_cnt(bar_empty(i % NS), warp == 0 ? 1 + NVR : 1);
   };
 
   // ---- phase 1: anchor scores of this CTA's slice (bf16 tensor cores) ----
@@ -729,16 +822,30 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     }
     tw_sync();
   }
-  // lane roles of the token pass: head g_own (adjacent lanes), and a chunk of LT consecutive
-  // stored tokens of the warp's 128-token region of each tile
-  constexpr int LT = REG * GS / 32;  // 16, 8 or 4 tokens
-  const int g_own = lane % GS, chunk = lane / GS;
-  const float m_own = mref[g_own];
-  float l_part = 0.f, pmin = 0.f;
-  const float* qp_own = qp + g_own * 128;
-  const int spare_grp = (R + 15) / 16;  // value operands of tokens without a value residual go here
+  named_arrive(3, NTW * 32 + NVR * 32);  // the value-residual warps may use SA, mref and accs
+  float m_ref[GS], l_part[GS];
+#pragma unroll
+  for (int g = 0; g < GS; ++g) {
+    m_ref[g] = mref[g];
+    l_part[g] = 0.f;
+  }
+  // Value weights of a run: one reduction per head into the anchor's owner CTA.
+  auto flush = [&](int anchor, const float (&v)[GS]) {
+    if (anchor < 0 || anchor >= k) return;
+#pragma unroll
+    for (int g = 0; g < GS; ++g) {
+      if (v[g] == 0.f) continue;
+      if (anchor >= a0 && anchor < a1) {  // this CTA owns the anchor
+        atomicAdd(&Wt[(anchor - a0) * GS + g], v[g]);
+      } else {
+        const int owner = anchor / kc;
+        red_cluster(&Wt[(anchor - owner * kc) * GS + g], owner, v[g]);
+      }
+    }
+  };
 
   // ---- phase 2: tile blocks ----
+  // lane -> four consecutive stored tokens of the warp's 128-token region, every head
   bool overflow_risk = false;
   for (int tl = 0; tl < n_t; ++tl) {
     const int it = n_ka + tl;
@@ -751,148 +858,117 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     if (ok && !warp_failed(failed)) {
       const TileView tv = tile_view(st, meta[s], U, j0 + tl, P.cap);
       const float* rsb = reinterpret_cast<const float*>(st + P.o_rs);
-      uint8_t* pfb = const_cast<uint8_t*>(st) + P.o_pf;
-      const int t0 = warp * REG + chunk * LT;  // a multiple of LT: the chunk sits in one bitmap word
-      const int te = min(t0 + LT, tv.n);
-      if (t0 < te) {
+      const int t0 = warp * REG + 4 * lane;
+      // tail: the run that ends this lane's tokens (its anchor `key`), head: the run that
+      // starts them when it differs (multi)
+      uint32_t key = 0xFFFFFFFFu;
+      int hkey = -1;
+      bool multi = false;
+      float val[GS], headv[GS];
+#pragma unroll
+      for (int g = 0; g < GS; ++g) val[g] = headv[g] = 0.f;
+      if (t0 < tv.n) {
+        const uint4 ka = *reinterpret_cast<const uint4*>(tv.st + 4 * t0);
+        const uint4 va = *reinterpret_cast<const uint4*>(tv.st + 4 * (tv.n64 + t0));
+        const uint32_t ek[4] = {ka.x, ka.y, ka.z, ka.w}, ev[4] = {va.x, va.y, va.z, va.w};
         const int wi = t0 >> 6, sh = t0 & 63;
-        const uint64_t wk = tv.bm(0, wi), wv = tv.bm(1, wi);
-        const uint64_t below = (1ull << sh) - 1ull;
-        int rkn = tv.rk(0, wi) + __popcll(wk & below);  // record of the next key-residual token
-        int rvn = tv.rk(1, wi) + __popcll(wv & below);
-        const uint32_t bk = (uint32_t)(wk >> sh), bv = (uint32_t)(wv >> sh);
-        // value weights: the sum over the current run of equal value anchors, in a register
-        int cur = (int)(*reinterpret_cast<const uint32_t*>(tv.st + 4 * (tv.n64 + t0)) & 0xFFFFu);
-        float acc = 0.f;
-        auto flush = [&]() {
-          if (acc != 0.f && cur < k) {
-            if (cur >= a0 && cur < a1) {  // this CTA owns the anchor
-              atomicAdd(&Wt[(cur - a0) * GS + g_own], acc);
-            } else {
-              const int owner = cur / kc;
-              red_cluster(&Wt[(cur - owner * kc) * GS + g_own], owner, acc);
-            }
-          }
-        };
-        const uint32_t lmask = LT == 32 ? 0xFFFFFFFFu : ((1u << LT) - 1u);
-        const bool staged_all = rkn + __popc(bk & lmask) <= R && rvn + __popc(bv & lmask) <= R;
-        if (staged_all) {
-          // every record of the chunk is staged: no branch but the run change; tokens without a
-          // residual read record 0 and write their (zero) value operand to the spare group
-#pragma unroll 1
-          for (int q4 = t0; q4 < te; q4 += 4) {  // 16-byte loads; entries past n (< n64) read as 0
-            const uint4 ka = *reinterpret_cast<const uint4*>(tv.st + 4 * q4);
-            const uint4 va = *reinterpret_cast<const uint4*>(tv.st + 4 * (tv.n64 + q4));
-            const uint32_t ek[4] = {ka.x, ka.y, ka.z, ka.w}, ev[4] = {va.x, va.y, va.z, va.w};
+        const uint64_t wk = tv.bm(0, wi);
+        const uint32_t kbits = (uint32_t)(wk >> sh) & 0xFu;
+        int rkn = tv.rk(0, wi) + __popcll(wk & ((1ull << sh) - 1ull));
+        const int nvalid = min(4, tv.n - t0);
+        float cw[4][GS];
+        uint32_t av[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              if (q4 + e >= te) break;
-              const int bit = q4 + e - t0;
-              const int a = min((int)(ek[e] & 0xFFFFu), k - 1);  // indices are < k by construction
-              const uint32_t kb = (bk >> bit) & 1u, vb = (bv >> bit) & 1u;
-              const float rt = rsb[(kb ? rkn : 0) * GS + g_own];
-              rkn += (int)kb;
-              float x = fmaf(half_hi(ek[e]), SA[a * GS + g_own], kb ? rt : 0.f) - m_own;
-              overflow_risk |= x > 120.f;
-              const float p = exp2f(x);
-              l_part += p;
-              const int av = (int)(ev[e] & 0xFFFFu);
-              if (av != cur) {  // stored order: a new run of value anchor av
-                flush();
-                cur = av;
-                acc = 0.f;
-              }
-              acc = fmaf(p, half_hi(ev[e]), acc);
-              const int r = vb ? rvn : 0;
-              rvn += (int)vb;
-              uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.st + tv.sm_v + 4u * (uint32_t)r);
-              smn = vb ? smn : 0u;
-              pmin = fmaf(p, half_hi(smn), pmin);
-              __nv_bfloat16 hi, lo;
-              split_b(p * half_lo(smn), hi, lo);
-              const int grp = vb ? (r >> 4) : spare_grp, kk = r & 15;
-              const int comp = (kk >> 3) * 2, hf = kk & 1, cc = (kk & 7) >> 1;
-              unsigned short* dst = reinterpret_cast<unsigned short*>(pfb + grp * 512 + (4 * g_own + cc) * 16);
-              dst[comp * 2 + hf] = __bfloat16_as_ushort(hi);
-              dst[(comp + 1) * 2 + hf] = __bfloat16_as_ushort(lo);
-            }
-          }
-        } else {
-#pragma unroll 1
-          for (int q4 = t0; q4 < te; q4 += 4) {
-            const uint4 ka = *reinterpret_cast<const uint4*>(tv.st + 4 * q4);
-            const uint4 va = *reinterpret_cast<const uint4*>(tv.st + 4 * (tv.n64 + q4));
-            const uint32_t ek[4] = {ka.x, ka.y, ka.z, ka.w}, ev[4] = {va.x, va.y, va.z, va.w};
+        for (int e = 0; e < 4; ++e) {
+          const bool valid = e < nvalid;
+          const int a = min((int)(ek[e] & 0xFFFFu), k - 1);  // indices are < k by construction
+          float sa[GS], rt[GS];
+          load_row<GS>(SA + a * GS, sa);
+          const bool kb = (kbits >> e) & 1u;
+          const int r = rkn;
+          rkn += (int)kb;
+          if (kb && r >= R) {  // beyond the staged records (a locally dense tile): CUDA cores
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              if (q4 + e >= te) break;
-              const int a = min((int)(ek[e] & 0xFFFFu), k - 1);
-              float x = half_hi(ek[e]) * SA[a * GS + g_own];
-              const int bit = q4 + e - t0;
-              if ((bk >> bit) & 1u) {  // key residual term
-                const int r = rkn++;
-                x += r < R ? rsb[r * GS + g_own] : key_record_term(tv, r, qp_own, sq[g_own]);
-              }
-              x -= m_own;
-              overflow_risk |= x > 120.f;
-              const float p = exp2f(x);
-              l_part += p;
-              const int av = (int)(ev[e] & 0xFFFFu);
-              if (av != cur) {
-                flush();
-                cur = av;
-                acc = 0.f;
-              }
-              acc += p * half_hi(ev[e]);
-              if ((bv >> bit) & 1u) {  // value residual: A operand of its group, or beyond the staged ones
-                const int r = rvn++;
-                const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_v + 4u * (uint32_t)r));
-                const float scl = half_lo(smn), mn = half_hi(smn);
-                pmin += p * mn;
-                if (r < R) {
-                  const int grp = r >> 4, kk = r & 15;
-                  const int comp = (kk >> 3) * 2, hf = kk & 1, cc = (kk & 7) >> 1;
-                  __nv_bfloat16 hi, lo;
-                  split_b(p * scl, hi, lo);
-                  unsigned short* dst = reinterpret_cast<unsigned short*>(pfb + grp * 512 + (4 * g_own + cc) * 16);
-                  dst[comp * 2 + hf] = __bfloat16_as_ushort(hi);
-                  dst[(comp + 1) * 2 + hf] = __bfloat16_as_ushort(lo);
-                } else {
-                  value_record_add(tv, r, p * scl, accs + g_own * 128);
-                }
-              }
-            }
+            for (int g = 0; g < GS; ++g) rt[g] = key_record_term(tv, r, qp + g * 128, sq[g]);
+          } else {
+            load_row<GS>(rsb + (kb ? r : 0) * GS, rt);
           }
+          const float gk = half_hi(ek[e]), gv = half_hi(ev[e]);
+#pragma unroll
+          for (int g = 0; g < GS; ++g) {
+            const float x = fmaf(gk, sa[g], kb ? rt[g] : 0.f) - m_ref[g];
+            overflow_risk |= valid && x > 120.f;
+            const float p = valid ? exp2f(x) : 0.f;
+            l_part[g] += p;
+            cw[e][g] = p * gv;
+          }
+          av[e] = ev[e] & 0xFFFFu;
         }
-        flush();
+        // tokens past the tile join the last token's run with zero weight
+#pragma unroll
+        for (int e = 1; e < 4; ++e)
+          if (e >= nvalid) av[e] = av[e - 1];
+        hkey = (int)av[0];
+        key = av[3];
+        multi = av[0] != av[3];
+#pragma unroll
+        for (int g = 0; g < GS; ++g) {
+          float hs = 0.f, ts = 0.f;
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            hs += av[e] == av[0] ? cw[e][g] : 0.f;
+            ts += av[e] == av[3] ? cw[e][g] : 0.f;
+          }
+          val[g] = ts;
+          headv[g] = multi ? hs : 0.f;
+        }
+        if (multi) {  // runs strictly inside the lane's four tokens (rare)
+#pragma unroll
+          for (int e = 1; e < 3; ++e)
+            if (av[e] != av[0] && av[e] != av[3]) flush((int)av[e], cw[e]);
+        }
       }
+      // Runs across lanes (anchors never decrease from lane to lane): the next lane's head run
+      // continues this lane's tail run when their anchors match; a head run that does not
+      // continue the previous lane's tail is complete
+      const uint32_t pkey = __shfl_up_sync(0xffffffffu, key, 1);
+      const int nhkey = __shfl_down_sync(0xffffffffu, hkey, 1);
+      const bool nmulti = __shfl_down_sync(0xffffffffu, (int)multi, 1) != 0;
+#pragma unroll
+      for (int g = 0; g < GS; ++g) {
+        const float nh = __shfl_down_sync(0xffffffffu, headv[g], 1);
+        if (lane < 31 && nmulti && (uint32_t)nhkey == key) val[g] += nh;
+      }
+      if (multi && !(lane > 0 && pkey == (uint32_t)hkey)) flush(hkey, headv);
+      // segmented inclusive scan of the tail sums over lanes with equal anchors
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const uint32_t kd = __shfl_up_sync(0xffffffffu, key, d);
+#pragma unroll
+        for (int g = 0; g < GS; ++g) {
+          const float vd = __shfl_up_sync(0xffffffffu, val[g], d);
+          if (lane >= d && kd == key) val[g] += vd;
+        }
+      }
+      const uint32_t nkey = __shfl_down_sync(0xffffffffu, key, 1);
+      if (key != 0xFFFFFFFFu && (lane == 31 || nkey != key)) flush((int)key, val);
     }
     __syncwarp();
-    if (lane == 0) mbar_arrive(bar_p(s));
+    if (lane == 0) mbar_arrive(bar_empty(s));
   }
   if (overflow_risk) *failed = 1;  // a logit beyond 2^120 of the reference would overflow the sums
 
-  // ---- per-CTA totals: lanes with lane % GS == g hold head g ----
-  {
+  // ---- per-CTA totals ----
 #pragma unroll
-    for (int o = GS; o < 32; o <<= 1) {
-      l_part += __shfl_xor_sync(0xffffffffu, l_part, o);
-      pmin += __shfl_xor_sync(0xffffffffu, pmin, o);
-    }
-    if (lane < GS) {
-      red[warp * GS + lane] = l_part;
-      opart[warp * GS + lane] = pmin;  // scratch until phase 3
-    }
+  for (int g = 0; g < GS; ++g) {
+    const float sl = warp_sum(l_part[g]);
+    if (lane == 0) red[warp * GS + g] = sl;
   }
   tw_sync();
   if (tid < GS) {
-    float sl = 0.f, pm = 0.f;
-    for (int w = 0; w < NTW; ++w) {
-      sl += red[w * GS + tid];
-      pm += opart[w * GS + tid];
-    }
+    float sl = 0.f;
+    for (int w = 0; w < NTW; ++w) sl += red[w * GS + tid];
     cl[tid] = sl;
-    pms[tid] = pm;
   }
   tw_sync();
 
@@ -1057,12 +1133,12 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_misc = take((size_t)(NTW * GS + 6 * GS + 4) * 4);
   P.o_meta = take(8 * 8);
   P.o_bar = take(5 * 8 * 8);
+  P.o_pfb = take((size_t)2 * ((R + 15) / 16) * 512);
   // a stage: staged bytes (a tile block's head, or an anchor chunk), then the key-residual
-  // terms and the value-residual A operands of a tile
+  // terms of a tile
   const int sb = (int)align128((size_t)std::max(cap, CH * 256));
   P.o_rs = sb;
-  P.o_pf = (int)align128((size_t)sb + (size_t)R * GS * 4);
-  const int stage = (int)align128((size_t)P.o_pf + (size_t)((R + 15) / 16 + 1) * 512);
+  const int stage = (int)align128((size_t)sb + (size_t)R * GS * 4);
   P.o_ring = (int)off;
   const long long room = (long long)smem_optin - (long long)off;
   if (room < 2LL * stage) return false;
