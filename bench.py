@@ -63,11 +63,12 @@ def _tile_fixed(n):
 
 def unit_bytes(S, k, nk, nv, G):
     """Compressed bytes one decode step reads for one (request, KV head), plus its q and out
-    rows: anchors, tile table and tile blocks (record padding taken at its mean, 12 B per
-    tile; the benchmark itself reads the exact block sizes from the arena's tile tables)."""
+    rows: anchors, tile table and tile blocks (record padding taken at its mean: 12 B of
+    scale padding and 240 B of value-code group padding per tile; the benchmark itself
+    reads the exact block sizes from the arena's tile tables)."""
     nt = (S + TILE - 1) // TILE
     fixed = sum(_tile_fixed(min(TILE, S - j * TILE)) for j in range(nt))
-    return 512 * k + 4 * (nt + 1) + fixed + 36 * (nk + nv) + 12 * nt + 2 * (2 * G * 128)
+    return 512 * k + 4 * (nt + 1) + fixed + 36 * (nk + nv) + 252 * nt + 2 * (2 * G * 128)
 
 
 def arena_read_bytes(torch, akv, p, lens, arena):

@@ -144,7 +144,13 @@ typedef struct akv_arena_header {
  *   then            smv [nv] uint32   (padded to 16 B)
  *   then            cdk [nk][32] uint8  2-bit codes of the rotated key residual, code j in
  *                                     byte j/4, bits 2(j%4)..2(j%4)+1
- *   then            cdv [nv][32] uint8
+ *   then            cdv  value codes in groups of 16 records (the last group padded with
+ *                        zero codes): group G is 128 uint32 words; word
+ *                        32 (d/32) + 4 (d%8) + (d%32)/8 holds the code of dimension d of
+ *                        record 16 G + s at bits 2s..2s+1.  ceil(nv/16) * 512 bytes.
+ *                        (Dimension-major, because the value side sums over records:
+ *                        one 16-byte load gives a thread the codes of 16 records for
+ *                        the four dimensions it multiplies.)
  * Record r of a side belongs to the r-th token (in stored order) whose bit is set;
  * token t's record is rk[t/64] + popcount(bm[t/64] & ((1 << (t%64)) - 1)) (the O(1)
  * position-to-slot lookup of Appendix A.1, "Layout", local to the tile).

@@ -665,7 +665,16 @@ int or_arena_unpack(const uint8_t* arena, uint64_t bytes, int32_t u, or_unit* ou
     uint32_t cd_off[2];
     cd_off[0] = sm_off[1] + (uint32_t)(((4 * m[1] + 15) / 16) * 16);
     cd_off[1] = cd_off[0] + 32u * (uint32_t)m[0];
-    if (b0 + cd_off[1] + 32u * (uint32_t)m[1] != b1) return -1;
+    /* value codes: groups of 16 records, dimension-major (word 32 (d/32) + 4 (d%8) + (d%32)/8
+     * of a group holds dimension d, record slot s at bits 2s) */
+    uint32_t nvgrp = (uint32_t)((m[1] + 15) / 16);
+    if (b0 + cd_off[1] + 512u * nvgrp != b1) return -1;
+    for (int32_t sl = m[1]; sl < 16 * (int32_t)nvgrp; ++sl) /* padding slots hold zero codes */
+      for (int dd = 0; dd < 128; ++dd) {
+        uint32_t wd = rd32(blk + cd_off[1] + 512u * (uint32_t)(sl / 16) +
+                           4u * (uint32_t)(32 * (dd / 32) + 4 * (dd % 8) + (dd % 32) / 8));
+        if ((wd >> (2 * (sl % 16))) & 3u) return -1;
+      }
     if (cnt[0] + m[0] > nk || cnt[1] + m[1] > nv) return -1;
     int32_t r[2] = {0, 0};
     for (int32_t t = 0; t < n; ++t) {
@@ -684,7 +693,17 @@ int or_arena_unpack(const uint8_t* arena, uint64_t bytes, int32_t u, or_unit* ou
         uint32_t e = rd32(blk + sm_off[side] + 4ull * r[side]);
         (side ? out->scale_v : out->scale_k)[g] = (uint16_t)(e & 0xFFFFu);
         (side ? out->min_v : out->min_k)[g] = (uint16_t)(e >> 16);
-        memcpy((side ? out->codes_v : out->codes_k) + 32ull * g, blk + cd_off[side] + 32ull * r[side], 32);
+        if (side == 0) {
+          memcpy(out->codes_k + 32ull * g, blk + cd_off[0] + 32ull * r[0], 32);
+        } else {
+          uint8_t* rec = out->codes_v + 32ull * g;
+          memset(rec, 0, 32);
+          for (int dd = 0; dd < 128; ++dd) {
+            uint32_t wd = rd32(blk + cd_off[1] + 512u * (uint32_t)(r[1] / 16) +
+                               4u * (uint32_t)(32 * (dd / 32) + 4 * (dd % 8) + (dd % 32) / 8));
+            rec[dd / 4] |= (uint8_t)(((wd >> (2 * (r[1] % 16))) & 3u) << (2 * (dd % 4)));
+          }
+        }
         ++r[side];
       }
     }

@@ -80,10 +80,11 @@ akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out
       sh.nv = (int32_t)nv;
       const int32_t nt = (S + kTile - 1) / kTile;
       sh.nt = nt;
-      // tile blocks: fixed parts exactly, records and at most 24 bytes of padding per tile
+      // tile blocks: fixed parts exactly, records, at most 24 bytes of scale padding and
+      // 480 bytes of value-code group padding per tile
       uint64_t cap = 0;
       for (int32_t j = 0; j < nt; ++j) cap += tile_fixed_bytes(std::min(kTile, S - j * kTile));
-      cap += 36ull * (uint64_t)(nk + nv) + 24ull * (uint64_t)nt;
+      cap += 36ull * (uint64_t)(nk + nv) + 504ull * (uint64_t)nt;
       if (cap >= (1ull << 32)) return fail(AKV_ERR_UNSUPPORTED, "a unit's tile blocks could exceed 2^32 bytes");
       const uint64_t sizes[kNumSections] = {(uint64_t)k * 256, (uint64_t)k * 256, (uint64_t)k * 4,
                                             4ull * (uint64_t)(nt + 1), cap};
@@ -305,7 +306,14 @@ akv_status akv_cache_pack_host(const akv_params* p, const int32_t* ctx_lens_host
           const uint16_t sc = side ? in.scale_v[sl] : in.scale_k[sl];
           const uint16_t mn = side ? in.min_v[sl] : in.min_k[sl];
           sm[side][r[side]] = (uint32_t)sc | ((uint32_t)mn << 16);
-          std::memcpy(cd[side] + 32 * (size_t)r[side], (side ? in.codes_v : in.codes_k) + 32 * (size_t)sl, 32);
+          const uint8_t* src = (side ? in.codes_v : in.codes_k) + 32 * (size_t)sl;
+          if (side == 0) {
+            std::memcpy(cd[0] + 32 * (size_t)r[0], src, 32);
+          } else {  // dimension-major groups of 16 records
+            uint32_t* grp = (uint32_t*)(cd[1] + 512 * (size_t)(r[1] / 16));
+            for (int dd = 0; dd < 128; ++dd)
+              grp[value_code_word(dd)] |= (uint32_t)((src[dd / 4] >> (2 * (dd % 4))) & 3u) << (2 * (r[1] % 16));
+          }
           ++r[side];
         }
       }

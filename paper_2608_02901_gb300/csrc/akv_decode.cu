@@ -67,7 +67,6 @@ constexpr int REG = T / NTW;           // tokens of a tile per token warp
 static_assert(REG == 128, "a token lane's chunk (REG * GS / 32 tokens) lies in one bitmap word");
 static_assert(NTW % NVR == 0, "value-residual warps release a stage with NTW / NVR arrivals each");
 constexpr int CH = 64;                 // anchor rows per chunk item
-constexpr int ROWE = 80;               // stride of an expanded row of 32 codes (64 B + 16 B pad)
 constexpr int kMaxCluster = 16;
 constexpr unsigned kWaitLimit = 1u << 22;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -82,7 +81,7 @@ struct DecodeParams {
   float scale_log2;
   unsigned long long sign_lo, sign_hi;
   int R, NS, stage_bytes, cap;
-  int o_sa, o_w, o_qfa, o_qfk, o_qp, o_acc, o_opart, o_e, o_misc, o_meta, o_bar, o_ring;
+  int o_sa, o_w, o_qfa, o_qfk, o_qp, o_acc, o_opart, o_misc, o_meta, o_bar, o_ring;
   int o_pfb;       // value-residual operands, two buffers (tiles alternate)
   int o_rs;        // inside a stage
 };
@@ -206,6 +205,14 @@ __device__ __forceinline__ float half_lo(uint32_t w) {
 }
 __device__ __forceinline__ float half_hi(uint32_t w) { return __half2float(__ushort_as_half((unsigned short)(w >> 16))); }
 
+// 2^x with the hardware approximation (relative error near 2^-22; results below the
+// smallest normal flush to 0, which only drops weights under 2^-126 of the reference).
+__device__ __forceinline__ float exp2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -305,12 +312,13 @@ __device__ __noinline__ float key_record_term(const TileView& tv, int r, const f
   }
   return half_hi(smn) * sqg + half_lo(smn) * dot;
 }
-// accg += ps * c of value record r (rotated domain).
+// accg += ps * c of value record r (rotated domain); value codes are dimension-major
+// groups of 16 records.
 __device__ __noinline__ void value_record_add(const TileView& tv, int r, float ps, float* accg) {
-  for (int bb = 0; bb < 32; ++bb) {
-    const uint32_t byte = *tv.at(tv.cd_v + 32u * (uint32_t)r + (uint32_t)bb);
-#pragma unroll
-    for (int c = 0; c < 4; ++c) atomicAdd(&accg[4 * bb + c], ps * (float)((byte >> (2 * c)) & 3u));
+  const uint32_t base = tv.cd_v + 512u * (uint32_t)(r / 16);
+  for (int d = 0; d < 128; ++d) {
+    const uint32_t w = *reinterpret_cast<const uint32_t*>(tv.at(base + 4u * value_code_word(d)));
+    atomicAdd(&accg[d], ps * (float)((w >> (2 * (r % 16))) & 3u));
   }
 }
 
@@ -363,7 +371,6 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float* qp = reinterpret_cast<float*>(smem + P.o_qp);
   float* accs = reinterpret_cast<float*>(smem + P.o_acc);
   float* opart = reinterpret_cast<float*>(smem + P.o_opart);
-  uint8_t* ebuf = smem + P.o_e;
   float* red = reinterpret_cast<float*>(smem + P.o_misc);  // [NTW][GS]
   float* sq = red + NTW * GS;                             // [GS]
   float* mref = sq + GS;                                  // [GS]
@@ -556,7 +563,6 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     cluster_arrive();  // B1
     named_sync(3, NTW * 32 + NVR * 32);  // anchor-score table, references and accs are ready
     float accV[2][4][4] = {};  // two independent sets (alternate groups), summed at the end
-    uint8_t* ew = ebuf + vw * 2 * 16 * ROWE;
     // step-1 roles: record slot (lane % 16) of a group, heads hb, hb + 2, ... (hb = lane / 16)
     constexpr int HPL = GS >= 2 ? GS / 2 : 1;
     const int sl16 = lane & 15, hb = lane >> 4;
@@ -602,7 +608,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
               const int g = hb + 2 * i;
               float rt = 0.f;
               if (kb) rt = rk < R ? rsb[rk * GS + g] : key_record_term(tv, rk, qp + g * 128, sq[g]);
-              const float p = exp2f(fmaf(gk, SA[a * GS + g], rt) - mv[i]);  // as the token warps form it
+              const float p = exp2_approx(fmaf(gk, SA[a * GS + g], rt) - mv[i]);  // as the token warps form it
               pminv[i] = fmaf(p, mn, pminv[i]);
               const float ps = p * scl;
               if (r < R) {
@@ -625,37 +631,24 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       // other buffer (its previous tile)
       named_sync(4, NVR * 32);
       if (go) {
+        // B operand straight from the dimension-major code words: this lane's four words hold
+        // dimensions 32 vw + 8 nb + r8 (nb = 0..3) of 16 records; records 2c, 2c+1 feed b0,
+        // records 2c+8, 2c+9 feed b1
+        const uint32_t woff = tv.cd_v + 4u * (uint32_t)(32 * vw + 4 * r8);
         for (int grp = 0; grp * 16 < nV; grp += 2) {
-          const int n = lane >> 1, hh = lane & 1;
-#pragma unroll
-          for (int q = 0; q < 2; ++q) {
-            const int sl = (grp + q) * 16 + n;
-            uint32_t x = 0;
-            if (sl < nV) x = *reinterpret_cast<const uint32_t*>(tv.at(tv.cd_v + 32u * (uint32_t)sl + 8u * vw + 4u * hh));
-            const uint32_t lo = x & 0xFFFFu, y = lo | (lo << 14);  // code 2m at bit 4m, code 2m+1 at 4m + 16
-            const uint32_t hi = x >> 16, z = hi | (hi << 14);
-            uint8_t* e = ew + q * 16 * ROWE;
-            *reinterpret_cast<uint4*>(e + n * ROWE + hh * 32) =
-                make_uint4(codes2_to_b2(y), codes2_to_b2(y >> 4), codes2_to_b2(y >> 8), codes2_to_b2(y >> 12));
-            *reinterpret_cast<uint4*>(e + n * ROWE + hh * 32 + 16) =
-                make_uint4(codes2_to_b2(z), codes2_to_b2(z >> 4), codes2_to_b2(z >> 8), codes2_to_b2(z >> 12));
-          }
-          __syncwarp();
-          const int mi = lane >> 3, ri = lane & 7;
 #pragma unroll
           for (int q = 0; q < 2; ++q) {
             if ((grp + q) * 16 >= nV) break;  // warp-uniform
             const uint4 a = *reinterpret_cast<const uint4*>(pf + (grp + q) * 512 + lane * 16);
-            const uint8_t* e = ew + q * 16 * ROWE;
+            const uint4 w4 = *reinterpret_cast<const uint4*>(tv.at(woff + 512u * (uint32_t)(grp + q)));
+            const uint32_t wd[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-              uint32_t b00, b01, b10, b11;
-              ldsm_x4_trans(smem_u32(e + ((mi & 1) * 8 + ri) * ROWE + half * 32 + (mi >> 1) * 16), b00, b01, b10, b11);
-              mma_bf16(accV[q][2 * half], a.x, a.y, a.z, a.w, b00, b01);
-              mma_bf16(accV[q][2 * half + 1], a.x, a.y, a.z, a.w, b10, b11);
+            for (int nb = 0; nb < 4; ++nb) {
+              // codes of records 2c, 2c+1 (x0) and 2c+8, 2c+9 (x1) in the low four bits
+              const uint32_t x0 = (wd[nb] >> (4 * c4)) & 0xFu, x1 = (wd[nb] >> (4 * c4 + 16)) & 0xFu;
+              mma_bf16(accV[q][nb], a.x, a.y, a.z, a.w, codes2_to_b2(x0 | (x0 << 14)), codes2_to_b2(x1 | (x1 << 14)));
             }
           }
-          __syncwarp();
         }
       }
       __syncwarp();
@@ -898,7 +891,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
           for (int g = 0; g < GS; ++g) {
             const float x = fmaf(gk, sa[g], kb ? rt[g] : 0.f) - m_ref[g];
             overflow_risk |= valid && x > 120.f;
-            const float p = valid ? exp2f(x) : 0.f;
+            const float p = valid ? exp2_approx(x) : 0.f;
             l_part[g] += p;
             cw[e][g] = p * gv;
           }
@@ -1129,7 +1122,6 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_qp = take((size_t)GS * 128 * 4);
   P.o_acc = take((size_t)GS * 128 * 4);
   P.o_opart = take((size_t)std::max(GS * 128, NTW * GS) * 4);
-  P.o_e = take((size_t)NVR * 2 * 16 * ROWE);
   P.o_misc = take((size_t)(NTW * GS + 6 * GS + 4) * 4);
   P.o_meta = take(8 * 8);
   P.o_bar = take(5 * 8 * 8);

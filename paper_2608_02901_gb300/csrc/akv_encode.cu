@@ -650,7 +650,13 @@ __global__ void enc_quant(const EncArgs A) {
   const uint32_t cd_off = F + round16(4u * (uint32_t)nkj) + round16(4u * (uint32_t)nvj) +
                           (side ? 32u * (uint32_t)nkj : 0u) + 32u * (uint32_t)r;
   uint8_t* blk = const_cast<uint8_t*>(blkc);
-  blk[cd_off + lane] = (uint8_t)byte;
+  if (side == 0) {
+    blk[cd_off + lane] = (uint8_t)byte;
+  } else {  // value codes: dimension-major groups of 16 records
+    uint32_t* grp = reinterpret_cast<uint32_t*>(blk + cd_off - 32u * (uint32_t)r + 512u * (uint32_t)(r / 16));
+    for (int c = 0; c < 4; ++c)
+      atomicOr(&grp[value_code_word(4 * lane + c)], ((byte >> (2 * c)) & 3u) << (2 * (r % 16)));
+  }
   if (lane == 0) *reinterpret_cast<uint32_t*>(blk + sm_off) = sch | (mnh << 16);
 }
 

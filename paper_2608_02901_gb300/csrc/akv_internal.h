@@ -35,9 +35,14 @@ AKV_HD constexpr uint32_t tile_words(int n) { return (uint32_t)(n + 63) / 64u; }
 AKV_HD constexpr uint32_t tile_fixed_bytes(int n) {
   return 8u * 64u * tile_words(n) + 16u * tile_words(n) + 2u * round16(2u * tile_words(n));
 }
+// value codes: groups of 16 records, 512 bytes each (the last group padded)
+AKV_HD constexpr uint32_t value_code_bytes(int nv) { return 512u * (((uint32_t)nv + 15u) / 16u); }
 AKV_HD constexpr uint32_t tile_block_bytes(int n, int nk, int nv) {
-  return tile_fixed_bytes(n) + round16(4u * (uint32_t)nk) + round16(4u * (uint32_t)nv) + 32u * (uint32_t)(nk + nv);
+  return tile_fixed_bytes(n) + round16(4u * (uint32_t)nk) + round16(4u * (uint32_t)nv) + 32u * (uint32_t)nk +
+         value_code_bytes(nv);
 }
+// word of dimension d in a group of value codes
+AKV_HD constexpr uint32_t value_code_word(int d) { return 32u * (uint32_t)(d / 32) + 4u * (uint32_t)(d % 8) + (uint32_t)((d % 32) / 8); }
 
 // Section indices inside one unit segment, in storage order.
 enum Section { kAnchorK = 0, kAnchorV, kAnchorPos, kTileTable, kTiles, kNumSections };

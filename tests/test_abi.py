@@ -71,12 +71,13 @@ def test_layout_header_and_sections():
         assert (b, h) == (u // 2, u % 2) and S == lens[b] and nt == (S + 1023) // 1024
         offs = d[32:72].view(np.uint64)
         cap, data = (int(x) for x in d[72:88].view(np.uint64))
-        # fixed part of every tile (streams, bitmaps, rank words), records, <= 24 B padding per tile
+        # fixed part of every tile (streams, bitmaps, rank words), records, <= 24 B of scale
+        # padding and <= 480 B of value-code group padding per tile
         fixed = 0
         for j in range(nt):
             nw = (min(1024, S - 1024 * j) + 63) // 64
             fixed += 512 * nw + 16 * nw + 2 * ((2 * nw + 15) // 16 * 16)
-        assert cap == fixed + 36 * (nk + nv) + 24 * nt
+        assert cap == fixed + 36 * (nk + nv) + 504 * nt
         sizes = [k * 256, k * 256, 4 * k, 4 * (nt + 1), cap]
         assert offs[0] % 256 == 0
         for o, sz in zip(offs, sizes):
