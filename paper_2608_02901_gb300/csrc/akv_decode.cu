@@ -1190,9 +1190,11 @@ int plan_for(const Layout& L, const LaunchKey& key, int vunits, Plan* out, std::
   if (e != cudaSuccess) return (int)e;
   e = cudaFuncSetAttribute(akv_decode_kernel<GS>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (e != cudaSuccess) return (int)e;
-  // Cluster size: one CTA per SM for one wave, no more CTAs than tiles in the longest unit.
-  int C = 1;
-  while (C < kMaxCluster && (long long)vunits * (C * 2) <= di.sms && (C * 2) <= L.max_tiles) C *= 2;
+  // Cluster size: the most CTAs per unit such that every cluster is resident at once (one CTA
+  // per SM), no more CTAs than tiles in the longest unit.  Sizes are tried downwards one by
+  // one: a GPU whose processor clusters cannot hold 16 CTAs each may still hold 12 or 13.
+  int C = std::min<long long>(kMaxCluster, std::max<long long>(1, di.sms / std::max(1, vunits)));
+  C = std::max(1, std::min(C, L.max_tiles));
   if (key.cluster_env >= 1 && key.cluster_env <= kMaxCluster) C = key.cluster_env;
   Plan pl;
   for (;;) {
@@ -1214,7 +1216,7 @@ int plan_for(const Layout& L, const LaunchKey& key, int vunits, Plan* out, std::
     // prefer a size whose clusters all fit at once; an explicit override only needs one to fit
     if (e == cudaSuccess && (nclusters >= vunits || (key.cluster_env == C && nclusters >= 1))) break;
     cudaGetLastError();
-    C = (C & (C - 1)) ? C - 1 : C / 2;
+    C -= 1;
   }
   std::lock_guard<std::mutex> lk(mu);
   cache[key] = pl;
