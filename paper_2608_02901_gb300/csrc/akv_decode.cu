@@ -205,6 +205,36 @@ __device__ __forceinline__ float half_lo(uint32_t w) {
 }
 __device__ __forceinline__ float half_hi(uint32_t w) { return __half2float(__ushort_as_half((unsigned short)(w >> 16))); }
 
+// Packed pairs of fp32 (one instruction for both lanes of the pair).
+__device__ __forceinline__ float2 f2fma(float2 a, float2 b, float2 c) {
+  unsigned long long ra, rb, rc, rd;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(ra) : "f"(a.x), "f"(a.y));
+  asm("mov.b64 %0, {%1, %2};" : "=l"(rb) : "f"(b.x), "f"(b.y));
+  asm("mov.b64 %0, {%1, %2};" : "=l"(rc) : "f"(c.x), "f"(c.y));
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(rd) : "l"(ra), "l"(rb), "l"(rc));
+  float2 d;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(rd));
+  return d;
+}
+__device__ __forceinline__ float2 f2add(float2 a, float2 b) {
+  unsigned long long ra, rb, rd;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(ra) : "f"(a.x), "f"(a.y));
+  asm("mov.b64 %0, {%1, %2};" : "=l"(rb) : "f"(b.x), "f"(b.y));
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(rd) : "l"(ra), "l"(rb));
+  float2 d;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(rd));
+  return d;
+}
+__device__ __forceinline__ float2 f2mul(float2 a, float2 b) {
+  unsigned long long ra, rb, rd;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(ra) : "f"(a.x), "f"(a.y));
+  asm("mov.b64 %0, {%1, %2};" : "=l"(rb) : "f"(b.x), "f"(b.y));
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(rd) : "l"(ra), "l"(rb));
+  float2 d;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(rd));
+  return d;
+}
+
 // 2^x with the hardware approximation (relative error near 2^-22; results below the
 // smallest normal flush to 0, which only drops weights under 2^-126 of the reference).
 __device__ __forceinline__ float exp2_approx(float x) {
@@ -378,6 +408,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float* pms = cl + GS;                                   // [GS]
   float* ltot = pms + GS;                                 // [GS]
   volatile int* failed = reinterpret_cast<volatile int*>(ltot + GS);
+  // 16-byte rows: zeros (no key residual) and -inf (a token past the tile's end)
+  float* zrow = reinterpret_cast<float*>(smem + P.o_misc + (((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15));
+  float* ninfrow = zrow + 4;
   uint2* meta = reinterpret_cast<uint2*>(smem + P.o_meta);  // [NS] tile block offset, bytes
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + P.o_bar);
   uint8_t* ring = smem + P.o_ring;
@@ -696,6 +729,10 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   for (int e = tid; e < kc * GS; e += NTT) Wt[e] = 0.f;  // before B1: peers add into it only after B1
   for (int e = tid; e < ((R + 15) / 16) * 256; e += NTT) reinterpret_cast<uint32_t*>(smem + P.o_pfb)[e] = 0u;
   if (tid < GS) pms[tid] = 0.f;
+  if (tid < 4) {
+    zrow[tid] = 0.f;
+    ninfrow[tid] = -INFINITY;
+  }
   if (P.rotate) tw_wht_rows(qp, GS);
   else tw_sync();
   {
@@ -816,30 +853,29 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     tw_sync();
   }
   named_arrive(3, NTW * 32 + NVR * 32);  // the value-residual warps may use SA, mref and accs
-  float m_ref[GS], l_part[GS];
+  // pairs of heads for the packed arithmetic (GS = 1: one head, the pair's second lane idle)
+  constexpr int NP = GS >= 2 ? GS / 2 : 1;
+  float2 negm[NP], l2[NP];
 #pragma unroll
-  for (int g = 0; g < GS; ++g) {
-    m_ref[g] = mref[g];
-    l_part[g] = 0.f;
+  for (int i = 0; i < NP; ++i) {
+    negm[i] = make_float2(-mref[2 * i], GS >= 2 ? -mref[2 * i + 1] : 0.f);
+    l2[i] = make_float2(0.f, 0.f);
   }
   // Value weights of a run: one reduction per head into the anchor's owner CTA.
-  auto flush = [&](int anchor, const float (&v)[GS]) {
+  auto flush = [&](int anchor, const float2 (&v)[NP]) {
     if (anchor < 0 || anchor >= k) return;
+    const int owner = anchor >= a0 && anchor < a1 ? rank : anchor / kc;
 #pragma unroll
     for (int g = 0; g < GS; ++g) {
-      if (v[g] == 0.f) continue;
-      if (anchor >= a0 && anchor < a1) {  // this CTA owns the anchor
-        atomicAdd(&Wt[(anchor - a0) * GS + g], v[g]);
-      } else {
-        const int owner = anchor / kc;
-        red_cluster(&Wt[(anchor - owner * kc) * GS + g], owner, v[g]);
-      }
+      const float x = (g & 1) ? v[g >> 1].y : v[g >> 1].x;
+      if (x == 0.f) continue;
+      if (owner == rank) atomicAdd(&Wt[(anchor - a0) * GS + g], x);
+      else red_cluster(&Wt[(anchor - owner * kc) * GS + g], owner, x);
     }
   };
 
   // ---- phase 2: tile blocks ----
   // lane -> four consecutive stored tokens of the warp's 128-token region, every head
-  bool overflow_risk = false;
   for (int tl = 0; tl < n_t; ++tl) {
     const int it = n_ka + tl;
     const int s = it % NS;
@@ -857,9 +893,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       uint32_t key = 0xFFFFFFFFu;
       int hkey = -1;
       bool multi = false;
-      float val[GS], headv[GS];
+      float2 val[NP], headv[NP];
 #pragma unroll
-      for (int g = 0; g < GS; ++g) val[g] = headv[g] = 0.f;
+      for (int i = 0; i < NP; ++i) val[i] = headv[i] = make_float2(0.f, 0.f);
       if (t0 < tv.n) {
         const uint4 ka = *reinterpret_cast<const uint4*>(tv.st + 4 * t0);
         const uint4 va = *reinterpret_cast<const uint4*>(tv.st + 4 * (tv.n64 + t0));
@@ -869,11 +905,10 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         const uint32_t kbits = (uint32_t)(wk >> sh) & 0xFu;
         int rkn = tv.rk(0, wi) + __popcll(wk & ((1ull << sh) - 1ull));
         const int nvalid = min(4, tv.n - t0);
-        float cw[4][GS];
+        float2 cw[4][NP];
         uint32_t av[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          const bool valid = e < nvalid;
           const int a = min((int)(ek[e] & 0xFFFFu), k - 1);  // indices are < k by construction
           float sa[GS], rt[GS];
           load_row<GS>(SA + a * GS, sa);
@@ -883,17 +918,18 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
           if (kb && r >= R) {  // beyond the staged records (a locally dense tile): CUDA cores
 #pragma unroll
             for (int g = 0; g < GS; ++g) rt[g] = key_record_term(tv, r, qp + g * 128, sq[g]);
-          } else {
-            load_row<GS>(rsb + (kb ? r : 0) * GS, rt);
+          } else {  // the key-residual terms, zeros, or -inf for a token past the tile's end
+            load_row<GS>(e >= nvalid ? ninfrow : (kb ? rsb + r * GS : zrow), rt);
           }
           const float gk = half_hi(ek[e]), gv = half_hi(ev[e]);
 #pragma unroll
-          for (int g = 0; g < GS; ++g) {
-            const float x = fmaf(gk, sa[g], kb ? rt[g] : 0.f) - m_ref[g];
-            overflow_risk |= valid && x > 120.f;
-            const float p = valid ? exp2_approx(x) : 0.f;
-            l_part[g] += p;
-            cw[e][g] = p * gv;
+          for (int i = 0; i < NP; ++i) {
+            const float2 s2 = make_float2(sa[2 * i], GS >= 2 ? sa[2 * i + 1] : 0.f);
+            const float2 r2 = make_float2(rt[2 * i], GS >= 2 ? rt[2 * i + 1] : 0.f);
+            const float2 x = f2add(f2fma(make_float2(gk, gk), s2, r2), negm[i]);
+            const float2 p = make_float2(exp2_approx(x.x), GS >= 2 ? exp2_approx(x.y) : 0.f);
+            l2[i] = f2add(l2[i], p);
+            cw[e][i] = f2mul(p, make_float2(gv, gv));
           }
           av[e] = ev[e] & 0xFFFFu;
         }
@@ -904,16 +940,22 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         hkey = (int)av[0];
         key = av[3];
         multi = av[0] != av[3];
+        float hw[4], tw[4];  // 0/1 membership of the head run and the tail run
 #pragma unroll
-        for (int g = 0; g < GS; ++g) {
-          float hs = 0.f, ts = 0.f;
+        for (int e = 0; e < 4; ++e) {
+          hw[e] = av[e] == av[0] ? 1.f : 0.f;
+          tw[e] = av[e] == av[3] ? 1.f : 0.f;
+        }
+#pragma unroll
+        for (int i = 0; i < NP; ++i) {
+          float2 hs = make_float2(0.f, 0.f), ts = hs;
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            hs += av[e] == av[0] ? cw[e][g] : 0.f;
-            ts += av[e] == av[3] ? cw[e][g] : 0.f;
+            hs = f2fma(cw[e][i], make_float2(hw[e], hw[e]), hs);
+            ts = f2fma(cw[e][i], make_float2(tw[e], tw[e]), ts);
           }
-          val[g] = ts;
-          headv[g] = multi ? hs : 0.f;
+          val[i] = ts;
+          headv[i] = multi ? hs : make_float2(0.f, 0.f);
         }
         if (multi) {  // runs strictly inside the lane's four tokens (rare)
 #pragma unroll
@@ -927,20 +969,24 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       const uint32_t pkey = __shfl_up_sync(0xffffffffu, key, 1);
       const int nhkey = __shfl_down_sync(0xffffffffu, hkey, 1);
       const bool nmulti = __shfl_down_sync(0xffffffffu, (int)multi, 1) != 0;
+      const bool take_next = lane < 31 && nmulti && (uint32_t)nhkey == key;
 #pragma unroll
-      for (int g = 0; g < GS; ++g) {
-        const float nh = __shfl_down_sync(0xffffffffu, headv[g], 1);
-        if (lane < 31 && nmulti && (uint32_t)nhkey == key) val[g] += nh;
+      for (int i = 0; i < NP; ++i) {
+        const float2 nh = make_float2(__shfl_down_sync(0xffffffffu, headv[i].x, 1),
+                                      __shfl_down_sync(0xffffffffu, headv[i].y, 1));
+        if (take_next) val[i] = f2add(val[i], nh);
       }
       if (multi && !(lane > 0 && pkey == (uint32_t)hkey)) flush(hkey, headv);
       // segmented inclusive scan of the tail sums over lanes with equal anchors
 #pragma unroll
       for (int d = 1; d < 32; d <<= 1) {
         const uint32_t kd = __shfl_up_sync(0xffffffffu, key, d);
+        const bool add = lane >= d && kd == key;
 #pragma unroll
-        for (int g = 0; g < GS; ++g) {
-          const float vd = __shfl_up_sync(0xffffffffu, val[g], d);
-          if (lane >= d && kd == key) val[g] += vd;
+        for (int i = 0; i < NP; ++i) {
+          const float2 vd = make_float2(__shfl_up_sync(0xffffffffu, val[i].x, d),
+                                        __shfl_up_sync(0xffffffffu, val[i].y, d));
+          if (add) val[i] = f2add(val[i], vd);
         }
       }
       const uint32_t nkey = __shfl_down_sync(0xffffffffu, key, 1);
@@ -949,12 +995,16 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     __syncwarp();
     if (lane == 0) mbar_arrive(bar_empty(s));
   }
-  if (overflow_risk) *failed = 1;  // a logit beyond 2^120 of the reference would overflow the sums
+  // a logit so far above the reference that the sums overflow leaves a non-finite normaliser
+  bool overflow_risk = false;
+#pragma unroll
+  for (int i = 0; i < NP; ++i) overflow_risk |= !(l2[i].x < INFINITY) || !(l2[i].y < INFINITY);
+  if (overflow_risk) *failed = 1;
 
   // ---- per-CTA totals ----
 #pragma unroll
   for (int g = 0; g < GS; ++g) {
-    const float sl = warp_sum(l_part[g]);
+    const float sl = warp_sum((g & 1) ? l2[g >> 1].y : l2[g >> 1].x);
     if (lane == 0) red[warp * GS + g] = sl;
   }
   tw_sync();
@@ -1122,7 +1172,7 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_qp = take((size_t)GS * 128 * 4);
   P.o_acc = take((size_t)GS * 128 * 4);
   P.o_opart = take((size_t)std::max(GS * 128, NTW * GS) * 4);
-  P.o_misc = take((size_t)(NTW * GS + 6 * GS + 4) * 4);
+  P.o_misc = take((size_t)(((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15) + 32);
   P.o_meta = take(8 * 8);
   P.o_bar = take(5 * 8 * 8);
   P.o_pfb = take((size_t)2 * ((R + 15) / 16) * 512);
