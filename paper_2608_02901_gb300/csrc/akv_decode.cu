@@ -83,6 +83,7 @@ struct DecodeParams {
   int R, NS, stage_bytes, cap;
   int o_sa, o_w, o_qfa, o_qfk, o_qp, o_acc, o_opart, o_misc, o_meta, o_bar, o_ring;
   int o_pfb;       // value-residual operands, two buffers (tiles alternate)
+  int o_vmap;      // per value-residual warp: token of each staged value record
   int o_rs;        // inside a stage
 };
 
@@ -623,10 +624,23 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         tv = tile_view(stage(s), meta[s], U, j0 + tl, P.cap);
         nV = min(tv.nv, R);
         const float* rsb = reinterpret_cast<const float*>(stage(s) + P.o_rs);
+        // token of each staged value record, from the bitmap: one 32-bit half word per lane
+        uint16_t* vmap = reinterpret_cast<uint16_t*>(smem + P.o_vmap) + vw * R;
+        if (lane < 2 * tv.nw) {
+          const int w = lane >> 1, hw = lane & 1;
+          const uint64_t word = tv.bm(1, w);
+          uint32_t bits = hw ? (uint32_t)(word >> 32) : (uint32_t)word;
+          int rr = tv.rk(1, w) + (hw ? __popc((uint32_t)word) : 0);
+          while (bits && rr < R) {
+            vmap[rr++] = (uint16_t)(64 * w + 32 * hw + __ffs(bits) - 1);
+            bits &= bits - 1u;
+          }
+        }
+        __syncwarp();
         for (int grp = vw; grp * 16 < tv.nv; grp += NVR) {
           const int r = grp * 16 + sl16;
           if (r < tv.nv && head_lane) {
-            const int t = value_record_token(tv, r);
+            const int t = r < R ? (int)vmap[r] : value_record_token(tv, r);
             const uint32_t ek = reinterpret_cast<const uint32_t*>(tv.st)[t];
             const int a = min((int)(ek & 0xFFFFu), k - 1);
             const float gk = half_hi(ek);
@@ -1176,6 +1190,7 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_meta = take(8 * 8);
   P.o_bar = take(5 * 8 * 8);
   P.o_pfb = take((size_t)2 * ((R + 15) / 16) * 512);
+  P.o_vmap = take((size_t)NVR * R * 2);
   // a stage: staged bytes (a tile block's head, or an anchor chunk), then the key-residual
   // terms of a tile
   const int sb = (int)align128((size_t)std::max(cap, CH * 256));
