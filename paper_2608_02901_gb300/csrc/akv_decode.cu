@@ -398,7 +398,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float* SA = reinterpret_cast<float*>(smem + P.o_sa);  // [k][GS] anchor scores (log2 units)
   float* Wt = reinterpret_cast<float*>(smem + P.o_w);   // [kc][GS] value weights of owned anchors
   uint2* qfa = reinterpret_cast<uint2*>(smem + P.o_qfa);
-  uint4* qfk = reinterpret_cast<uint4*>(smem + P.o_qfk);
+  uint2* qfk = reinterpret_cast<uint2*>(smem + P.o_qfk);
   float* qp = reinterpret_cast<float*>(smem + P.o_qp);
   float* accs = reinterpret_cast<float*>(smem + P.o_acc);
   float* opart = reinterpret_cast<float*>(smem + P.o_opart);
@@ -513,15 +513,18 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   }
 
   // =========================== key-residual warps ================================
-  // q' . c for the staged key records of each tile, 8 records per mma group, fragments
-  // of q' (fp16 high and low parts) held in registers.
+  // q' . c for the staged key records of each tile on tensor cores: A = the 2-bit codes of
+  // 16 records (rows), converted in registers; B = q' (columns: heads as fp16 high parts, then
+  // low parts), fragments held in registers.  k order within a 16-dim step: the pair (2c, 2c+1)
+  // is dims (2c, 2c+8), the pair (2c+8, 2c+9) is dims (2c+1, 2c+9), so one shift of a code word
+  // gives both codes of a pair at bits 0 and 16.
   if (warp >= W_KRES && warp < W_KRES + NKR) {
     const int kw = warp - W_KRES;
     cluster_arrive();  // B1
     named_sync(2, NTW * 32 + NKR * 32);  // q' fragments written by the token warps
-    uint4 af[8];
+    uint2 bf[8];
 #pragma unroll
-    for (int ks = 0; ks < 8; ++ks) af[ks] = qfk[ks * 32 + lane];
+    for (int ks = 0; ks < 8; ++ks) bf[ks] = qfk[ks * 32 + lane];
     bool ok = true;
     for (int tl = 0; tl < n_t; ++tl) {
       const int s = (n_ka + tl) % NS;
@@ -533,41 +536,54 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         const TileView tv = tile_view(stage(s), meta[s], U, j0 + tl, P.cap);
         const int nK = min(tv.nk, R);
         float* rs = reinterpret_cast<float*>(stage(s) + P.o_rs);
-        // two groups of 8 records at a time, each as two independent mma chains
-        for (int g8 = kw; g8 * 8 < nK; g8 += 2 * NKR) {
-          const int gsel[2] = {g8, g8 + NKR};
-          uint32_t wd[2][8];
+        // two groups of 16 records at a time, each as two independent mma chains
+        for (int g16 = kw; g16 * 16 < nK; g16 += 2 * NKR) {
+          uint32_t wd[2][2][8];  // [group][record r8 / r8 + 8][16-dim step]
 #pragma unroll
-          for (int q = 0; q < 2; ++q) {
-            const int sl = gsel[q] * 8 + r8;  // the record whose codes this lane feeds (B column r8)
-            uint4 w0 = make_uint4(0u, 0u, 0u, 0u), w1 = w0;
-            if (sl < nK) {
-              w0 = *reinterpret_cast<const uint4*>(tv.at(tv.cd_k + 32u * (uint32_t)sl));
-              w1 = *reinterpret_cast<const uint4*>(tv.at(tv.cd_k + 32u * (uint32_t)sl + 16u));
+          for (int q = 0; q < 2; ++q)
+#pragma unroll
+            for (int hr = 0; hr < 2; ++hr) {
+              const int sl = (g16 + q * NKR) * 16 + r8 + 8 * hr;
+              uint4 w0 = make_uint4(0u, 0u, 0u, 0u), w1 = w0;
+              if (sl < nK) {
+                w0 = *reinterpret_cast<const uint4*>(tv.at(tv.cd_k + 32u * (uint32_t)sl));
+                w1 = *reinterpret_cast<const uint4*>(tv.at(tv.cd_k + 32u * (uint32_t)sl + 16u));
+              }
+              wd[q][hr][0] = w0.x; wd[q][hr][1] = w0.y; wd[q][hr][2] = w0.z; wd[q][hr][3] = w0.w;
+              wd[q][hr][4] = w1.x; wd[q][hr][5] = w1.y; wd[q][hr][6] = w1.z; wd[q][hr][7] = w1.w;
             }
-            wd[q][0] = w0.x; wd[q][1] = w0.y; wd[q][2] = w0.z; wd[q][3] = w0.w;
-            wd[q][4] = w1.x; wd[q][5] = w1.y; wd[q][6] = w1.z; wd[q][7] = w1.w;
-          }
           float d[2][2][4] = {};
 #pragma unroll
           for (int ks = 0; ks < 8; ++ks)
 #pragma unroll
             for (int q = 0; q < 2; ++q) {
-              const uint32_t x = wd[q][ks] >> (4 * c4);
-              mma_f16(d[q][ks & 1], af[ks], codes2_to_h2(x), codes2_to_h2(x >> 2));
+              const uint32_t xa = wd[q][0][ks] >> (4 * c4), xb = wd[q][1][ks] >> (4 * c4);
+              const uint4 a = make_uint4(codes2_to_h2(xa), codes2_to_h2(xb), codes2_to_h2(xa >> 2), codes2_to_h2(xb >> 2));
+              mma_f16(d[q][ks & 1], a, bf[ks].x, bf[ks].y);
             }
-          if (r8 < GS) {  // D rows r8 (high parts) and r8 + 8 (low parts), columns 2c, 2c+1
+          // columns 2c, 2c+1: high parts of heads 2c, 2c+1 (c < 2) or low parts (c >= 2)
 #pragma unroll
-            for (int q = 0; q < 2; ++q)
+          for (int q = 0; q < 2; ++q) {
+            float v[4];
 #pragma unroll
-              for (int e2 = 0; e2 < 2; ++e2) {
-                const int sl2 = gsel[q] * 8 + 2 * c4 + e2;
-                if (sl2 < nK) {
-                  const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_k + 4u * (uint32_t)sl2));
-                  const float dot = (d[q][0][e2] + d[q][1][e2]) + (d[q][0][2 + e2] + d[q][1][2 + e2]);
-                  rs[sl2 * GS + r8] = half_hi(smn) * sq[r8] + half_lo(smn) * dot;
+            for (int e = 0; e < 4; ++e) {
+              v[e] = d[q][0][e] + d[q][1][e];
+              v[e] += __shfl_xor_sync(0xffffffffu, v[e], 2);
+            }
+            if (c4 < 2) {
+#pragma unroll
+              for (int hr = 0; hr < 2; ++hr) {
+                const int sl = (g16 + q * NKR) * 16 + r8 + 8 * hr;
+                if (sl < nK) {
+                  const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_k + 4u * (uint32_t)sl));
+#pragma unroll
+                  for (int e = 0; e < 2; ++e) {
+                    const int g = 2 * c4 + e;
+                    if (g < GS) rs[sl * GS + g] = half_hi(smn) * sq[g] + half_lo(smn) * v[2 * hr + e];
+                  }
                 }
               }
+            }
           }
         }
       }
@@ -763,23 +779,24 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   {
     // fragment (k-step ks, lane ln): one per token thread (8 k-steps x 32 lanes)
     const int ks = tid >> 5, ln = tid & 31, g = ln >> 2, c = ln & 3;
-    uint2 fa = make_uint2(0u, 0u);
-    uint4 fk = make_uint4(0u, 0u, 0u, 0u);
+    uint2 fa = make_uint2(0u, 0u), fk = make_uint2(0u, 0u);
     if (g < GS) {
       // anchor-score B operand: q in bf16, k order permuted so a thread's dims are contiguous
       const __nv_bfloat16* qr = P.q + qrow0 + (size_t)g * 128;
       const int d0 = 32 * (ks >> 1) + 8 * c + 4 * (ks & 1);
       fa.x = pack_b2(qr[d0], qr[d0 + 1]);
       fa.y = pack_b2(qr[d0 + 2], qr[d0 + 3]);
-      // key-residual A operand: rows g = q' high parts, rows g + 8 = low parts; k index pairs
-      // (2c, 2c+1) <-> coords (16ks + 2c, 16ks + 2c + 8), (2c+8, 2c+9) <-> (16ks + 2c + 1, 16ks + 2c + 9)
-      const float* x = qp + g * 128 + 16 * ks + 2 * c;
-      const __half h0 = __float2half_rn(x[0]), h8 = __float2half_rn(x[8]);
-      const __half h1 = __float2half_rn(x[1]), h9 = __float2half_rn(x[9]);
-      fk.x = pack_h2(h0, h8);
-      fk.y = pack_h2(__float2half_rn(x[0] - __half2float(h0)), __float2half_rn(x[8] - __half2float(h8)));
-      fk.z = pack_h2(h1, h9);
-      fk.w = pack_h2(__float2half_rn(x[1] - __half2float(h1)), __float2half_rn(x[9] - __half2float(h9)));
+    }
+    if ((g & 3) < GS) {
+      // key-residual B operand, column g: head g % 4, fp16 high part (g < 4) or low part;
+      // k pairs (2c, 2c+1) <-> dims (16ks + 2c, 16ks + 2c + 8), (2c+8, 2c+9) <-> (16ks + 2c + 1, 16ks + 2c + 9)
+      const float* x = qp + (g & 3) * 128 + 16 * ks + 2 * c;
+      auto part = [&](float v) {
+        const __half hi = __float2half_rn(v);
+        return g < 4 ? hi : __float2half_rn(v - __half2float(hi));
+      };
+      fk.x = pack_h2(part(x[0]), part(x[8]));
+      fk.y = pack_h2(part(x[1]), part(x[9]));
     }
     qfa[ks * 32 + ln] = fa;
     qfk[ks * 32 + ln] = fk;
@@ -1182,7 +1199,7 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_sa = take((size_t)L.max_k * GS * 4);
   P.o_w = take((size_t)kc_max * GS * 4);
   P.o_qfa = take(8 * 32 * 8);
-  P.o_qfk = take(8 * 32 * 16);
+  P.o_qfk = take(8 * 32 * 8);
   P.o_qp = take((size_t)GS * 128 * 4);
   P.o_acc = take((size_t)GS * 128 * 4);
   P.o_opart = take((size_t)std::max(GS * 128, NTW * GS) * 4);
