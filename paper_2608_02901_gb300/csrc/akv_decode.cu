@@ -45,6 +45,7 @@
 #include <mutex>
 #include <string>
 #include <tuple>
+#include <type_traits>
 
 #include "akv_internal.h"
 
@@ -83,8 +84,7 @@ struct DecodeParams {
   int R, NS, stage_bytes, cap;
   int o_sa, o_w, o_qfa, o_qfk, o_qp, o_acc, o_opart, o_misc, o_meta, o_bar, o_ring;
   int o_pfb;       // value-residual operands, two buffers (tiles alternate)
-  int o_vmap;      // per value-residual warp: token of each staged value record
-  int o_rs;        // inside a stage
+  int o_rs, o_pv;  // inside a stage: key-residual terms, p of the value-record tokens
 };
 
 // ---- device helpers ---------------------------------------------------------------
@@ -353,6 +353,18 @@ __device__ __noinline__ void value_record_add(const TileView& tv, int r, float p
   }
 }
 
+// GS probabilities (pairs) as one row of GS floats (16-, 8- or 4-byte aligned).
+template <int GS, int NP>
+__device__ __forceinline__ void store_row(float* p, const float2 (&v)[NP]) {
+  if constexpr (GS == 4) {
+    *reinterpret_cast<float4*>(p) = make_float4(v[0].x, v[0].y, v[1].x, v[1].y);
+  } else if constexpr (GS == 2) {
+    *reinterpret_cast<float2*>(p) = v[0];
+  } else {
+    p[0] = v[0].x;
+  }
+}
+
 // A row of GS consecutive floats (16-, 8- or 4-byte aligned) into registers.
 template <int GS>
 __device__ __forceinline__ void load_row(const float* p, float (&out)[GS]) {
@@ -365,21 +377,6 @@ __device__ __forceinline__ void load_row(const float* p, float (&out)[GS]) {
   } else {
     out[0] = p[0];
   }
-}
-
-// Token t of the tile (index in stored order) holding value record r: the r-th set bit
-// of the value bitmap, found from the rank words.
-__device__ __forceinline__ int value_record_token(const TileView& tv, int r) {
-  int w = 0;
-#pragma unroll
-  for (int step = 8; step; step >>= 1)
-    if (w + step < tv.nw && tv.rk(1, w + step) <= r) w += step;
-  const int rem = r - tv.rk(1, w);
-  const uint64_t word = tv.bm(1, w);
-  const uint32_t lo = (uint32_t)word, hi = (uint32_t)(word >> 32);
-  const int plo = __popc(lo);
-  const int bit = rem < plo ? (int)__fns(lo, 0, rem + 1) : 32 + (int)__fns(hi, 0, rem - plo + 1);
-  return 64 * w + bit;
 }
 
 template <int GS>
@@ -418,12 +415,13 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   const int NS = P.NS;
   // per stage: an anchor chunk landed (full_c) / a tile block landed (full_t); stage free
   // again (empty: all token and value-residual warps are done with it); key-residual
-  // terms ready (rs).  Chunk items and tiles complete different barriers, so every waiter
-  // sees every phase it waits on.
+  // terms ready (rs); probabilities of the value-record tokens written (p).  Chunk items and
+  // tiles complete different barriers, so every waiter sees every phase it waits on.
   auto bar_full_c = [&](int s) { return smem_u32(bars + s); };
   auto bar_full_t = [&](int s) { return smem_u32(bars + NS + s); };
   auto bar_empty = [&](int s) { return smem_u32(bars + 2 * NS + s); };
   auto bar_rs = [&](int s) { return smem_u32(bars + 3 * NS + s); };
+  auto bar_p = [&](int s) { return smem_u32(bars + 4 * NS + s); };
   auto stage = [&](int s) { return ring + (size_t)s * P.stage_bytes; };
 
   // this CTA's anchors (it owns their value weights) and tile blocks
@@ -450,6 +448,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       mbar_init(bar_full_t(s), 1);
       mbar_init(bar_empty(s), NTW + NVR);
       mbar_init(bar_rs(s), NKR);
+      mbar_init(bar_p(s), NTW);
     }
     *failed = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -601,13 +600,12 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   }
 
   // =========================== value-residual warps ==============================
-  // Per tile, for the value records only: the token's probability p (recomputed from the
-  // anchor scores and the key-residual terms), then sum over records of (p scale) c on
-  // tensor cores (bf16 operands: p scale as high + low parts, codes exact), in the rotated
-  // domain.  Step 1: each warp builds the A operands of every NVR-th group of 16 records
-  // into a shared buffer (two buffers, tiles alternate); step 2: each warp multiplies all
-  // groups into the 32 coordinates 32 vw .. 32 vw + 31 it owns.  Records beyond the staged
-  // count are added on CUDA cores in step 1.
+  // Per tile, for the staged value records: sum over records of (p scale) c on tensor cores
+  // (bf16 operands: p scale as high + low parts, codes exact), in the rotated domain, with p
+  // as the token warps stored it.  Step 1: each warp builds the A operands of every NVR-th
+  // group of 16 records into a shared buffer (two buffers, tiles alternate); step 2: each
+  // warp multiplies all groups into the 32 coordinates 32 vw .. 32 vw + 31 it owns.  The token
+  // warps add records beyond the staged count themselves, on CUDA cores.
   if (warp >= W_VRES && warp < W_VRES + NVR) {
     const int vw = warp - W_VRES;
     cluster_arrive();  // B1
@@ -617,19 +615,16 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     constexpr int HPL = GS >= 2 ? GS / 2 : 1;
     const int sl16 = lane & 15, hb = lane >> 4;
     const bool head_lane = hb < GS;
-    float mv[HPL], pminv[HPL];
+    float pminv[HPL];
 #pragma unroll
-    for (int i = 0; i < HPL; ++i) {
-      mv[i] = head_lane ? mref[hb + 2 * i] : 0.f;
-      pminv[i] = 0.f;
-    }
+    for (int i = 0; i < HPL; ++i) pminv[i] = 0.f;
     const int ngrp_st = (R + 15) / 16;
     bool ok = true;
     for (int tl = 0; tl < n_t; ++tl) {
       const int s = (n_ka + tl) % NS;
       const uint32_t par = (uint32_t)(tl / NS) & 1u;
       if (ok && !warp_failed(failed)) {
-        ok = mbar_wait_w(bar_full_t(s), par) && mbar_wait_w(bar_rs(s), par);
+        ok = mbar_wait_w(bar_full_t(s), par) && mbar_wait_w(bar_p(s), par);
         if (!ok) *failed = 1;
       }
       const bool go = ok && !warp_failed(failed);
@@ -639,53 +634,25 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       if (go) {
         tv = tile_view(stage(s), meta[s], U, j0 + tl, P.cap);
         nV = min(tv.nv, R);
-        const float* rsb = reinterpret_cast<const float*>(stage(s) + P.o_rs);
-        // token of each staged value record, from the bitmap: one 32-bit half word per lane
-        uint16_t* vmap = reinterpret_cast<uint16_t*>(smem + P.o_vmap) + vw * R;
-        if (lane < 2 * tv.nw) {
-          const int w = lane >> 1, hw = lane & 1;
-          const uint64_t word = tv.bm(1, w);
-          uint32_t bits = hw ? (uint32_t)(word >> 32) : (uint32_t)word;
-          int rr = tv.rk(1, w) + (hw ? __popc((uint32_t)word) : 0);
-          while (bits && rr < R) {
-            vmap[rr++] = (uint16_t)(64 * w + 32 * hw + __ffs(bits) - 1);
-            bits &= bits - 1u;
-          }
-        }
-        __syncwarp();
-        for (int grp = vw; grp * 16 < tv.nv; grp += NVR) {
+        const float* pvb = reinterpret_cast<const float*>(stage(s) + P.o_pv);
+        for (int grp = vw; grp * 16 < nV; grp += NVR) {
           const int r = grp * 16 + sl16;
-          if (r < tv.nv && head_lane) {
-            const int t = r < R ? (int)vmap[r] : value_record_token(tv, r);
-            const uint32_t ek = reinterpret_cast<const uint32_t*>(tv.st)[t];
-            const int a = min((int)(ek & 0xFFFFu), k - 1);
-            const float gk = half_hi(ek);
-            const int wi = t >> 6;
-            const uint64_t wk = tv.bm(0, wi);
-            const bool kb = (wk >> (t & 63)) & 1ull;
-            const int rk = tv.rk(0, wi) + __popcll(wk & ((1ull << (t & 63)) - 1ull));
+          if (r < nV && head_lane) {
             const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_v + 4u * (uint32_t)r));
             const float scl = half_lo(smn), mn = half_hi(smn);
 #pragma unroll
             for (int i = 0; i < HPL; ++i) {
               const int g = hb + 2 * i;
-              float rt = 0.f;
-              if (kb) rt = rk < R ? rsb[rk * GS + g] : key_record_term(tv, rk, qp + g * 128, sq[g]);
-              const float p = exp2_approx(fmaf(gk, SA[a * GS + g], rt) - mv[i]);  // as the token warps form it
+              const float p = pvb[r * GS + g];
               pminv[i] = fmaf(p, mn, pminv[i]);
-              const float ps = p * scl;
-              if (r < R) {
-                // A-operand place of (record r, head g): group r / 16, lane 4 g + (r % 8) / 2,
-                // register 2 ((r / 8) % 2) (high part) or + 1 (low part), half r % 2
-                __nv_bfloat16 phi, plo;
-                split_b(ps, phi, plo);
-                unsigned short* dst = reinterpret_cast<unsigned short*>(
-                    pf + grp * 512 + (4 * g + ((r & 7) >> 1)) * 16 + ((r >> 3) & 1) * 8 + (r & 1) * 2);
-                dst[0] = __bfloat16_as_ushort(phi);
-                dst[2] = __bfloat16_as_ushort(plo);
-              } else {
-                value_record_add(tv, r, ps, accs + g * 128);
-              }
+              // A-operand place of (record r, head g): group r / 16, lane 4 g + (r % 8) / 2,
+              // register 2 ((r / 8) % 2) (high part) or + 1 (low part), half r % 2
+              __nv_bfloat16 phi, plo;
+              split_b(p * scl, phi, plo);
+              unsigned short* dst = reinterpret_cast<unsigned short*>(
+                  pf + grp * 512 + (4 * g + ((r & 7) >> 1)) * 16 + ((r >> 3) & 1) * 8 + (r & 1) * 2);
+              dst[0] = __bfloat16_as_ushort(phi);
+              dst[2] = __bfloat16_as_ushort(plo);
             }
           }
         }
@@ -932,27 +899,33 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         const uint4 va = *reinterpret_cast<const uint4*>(tv.st + 4 * (tv.n64 + t0));
         const uint32_t ek[4] = {ka.x, ka.y, ka.z, ka.w}, ev[4] = {va.x, va.y, va.z, va.w};
         const int wi = t0 >> 6, sh = t0 & 63;
-        const uint64_t wk = tv.bm(0, wi);
-        const uint32_t kbits = (uint32_t)(wk >> sh) & 0xFu;
+        const uint64_t wk = tv.bm(0, wi), wv = tv.bm(1, wi);
+        const uint32_t kbits = (uint32_t)(wk >> sh) & 0xFu, vbits = (uint32_t)(wv >> sh) & 0xFu;
         int rkn = tv.rk(0, wi) + __popcll(wk & ((1ull << sh) - 1ull));
+        int rvn = tv.rk(1, wi) + __popcll(wv & ((1ull << sh) - 1ull));
+        float* pvb = reinterpret_cast<float*>(const_cast<uint8_t*>(st) + P.o_pv);
         const int nvalid = min(4, tv.n - t0);
         float2 cw[4][NP];
         uint32_t av[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
+        // one token: logits, p, l, run weights and, for a value record, its p (every record
+        // staged: tokens without a value record write the spare row R; otherwise the records
+        // beyond the staged ones take the CUDA-core paths)
+        auto token = [&](int e, auto dense) {
+          constexpr bool kDense = decltype(dense)::value;
           const int a = min((int)(ek[e] & 0xFFFFu), k - 1);  // indices are < k by construction
           float sa[GS], rt[GS];
           load_row<GS>(SA + a * GS, sa);
           const bool kb = (kbits >> e) & 1u;
           const int r = rkn;
           rkn += (int)kb;
-          if (kb && r >= R) {  // beyond the staged records (a locally dense tile): CUDA cores
+          if (kDense && kb && r >= R) {
 #pragma unroll
             for (int g = 0; g < GS; ++g) rt[g] = key_record_term(tv, r, qp + g * 128, sq[g]);
           } else {  // the key-residual terms, zeros, or -inf for a token past the tile's end
             load_row<GS>(e >= nvalid ? ninfrow : (kb ? rsb + r * GS : zrow), rt);
           }
           const float gk = half_hi(ek[e]), gv = half_hi(ev[e]);
+          float2 pe[NP];
 #pragma unroll
           for (int i = 0; i < NP; ++i) {
             const float2 s2 = make_float2(sa[2 * i], GS >= 2 ? sa[2 * i + 1] : 0.f);
@@ -961,8 +934,34 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             const float2 p = make_float2(exp2_approx(x.x), GS >= 2 ? exp2_approx(x.y) : 0.f);
             l2[i] = f2add(l2[i], p);
             cw[e][i] = f2mul(p, make_float2(gv, gv));
+            pe[i] = p;
           }
           av[e] = ev[e] & 0xFFFFu;
+          const bool vb = (vbits >> e) & 1u;
+          const int rv = rvn;
+          rvn += (int)vb;
+          if (!kDense) {
+            store_row<GS>(pvb + (vb ? rv : R) * GS, pe);
+          } else if (vb) {
+            if (rv < R) {
+              store_row<GS>(pvb + rv * GS, pe);
+            } else {  // beyond the staged records (a locally dense tile): CUDA cores
+              const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_v + 4u * (uint32_t)rv));
+#pragma unroll
+              for (int g = 0; g < GS; ++g) {
+                const float pg = (g & 1) ? pe[g >> 1].y : pe[g >> 1].x;
+                value_record_add(tv, rv, pg * half_lo(smn), accs + g * 128);
+                atomicAdd(&pms[g], pg * half_hi(smn));
+              }
+            }
+          }
+        };
+        if (tv.nk <= R && tv.nv <= R) {
+#pragma unroll
+          for (int e = 0; e < 4; ++e) token(e, std::false_type{});
+        } else {
+#pragma unroll
+          for (int e = 0; e < 4; ++e) token(e, std::true_type{});
         }
         // tokens past the tile join the last token's run with zero weight
 #pragma unroll
@@ -1024,7 +1023,10 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       if (key != 0xFFFFFFFFu && (lane == 31 || nkey != key)) flush((int)key, val);
     }
     __syncwarp();
-    if (lane == 0) mbar_arrive(bar_empty(s));
+    if (lane == 0) {
+      mbar_arrive(bar_p(s));
+      mbar_arrive(bar_empty(s));
+    }
   }
   // a logit so far above the reference that the sums overflow leaves a non-finite normaliser
   bool overflow_risk = false;
@@ -1207,12 +1209,12 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_meta = take(8 * 8);
   P.o_bar = take(5 * 8 * 8);
   P.o_pfb = take((size_t)2 * ((R + 15) / 16) * 512);
-  P.o_vmap = take((size_t)NVR * R * 2);
   // a stage: staged bytes (a tile block's head, or an anchor chunk), then the key-residual
   // terms of a tile
   const int sb = (int)align128((size_t)std::max(cap, CH * 256));
   P.o_rs = sb;
-  const int stage = (int)align128((size_t)sb + (size_t)R * GS * 4);
+  P.o_pv = (int)align128((size_t)sb + (size_t)R * GS * 4);
+  const int stage = (int)align128((size_t)P.o_pv + (size_t)(R + 1) * GS * 4);  // row R: spare
   P.o_ring = (int)off;
   const long long room = (long long)smem_optin - (long long)off;
   if (room < 2LL * stage) return false;
