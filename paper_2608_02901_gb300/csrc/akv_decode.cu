@@ -57,12 +57,17 @@ namespace {
 // warp roles
 constexpr int NTW = 8;                 // token warps (warps 0 .. 7)
 constexpr int NTT = NTW * 32;          // token threads
-constexpr int W_KRES = NTW;            // key-residual warps
-constexpr int NKR = 2;
-constexpr int W_VRES = W_KRES + NKR;   // value-residual warps
-constexpr int NVR = 4;
-constexpr int W_PROD = W_VRES + NVR;   // producer warp
+constexpr int NKR = 2;                 // key-residual warps: 10, 11
+constexpr int NVR = 4;                 // value-residual warps: 8, 9, 12, 13
+constexpr int W_PROD = NTW + NKR + NVR;  // producer warp (14)
 constexpr int NT = (W_PROD + 1) * 32;  // 480 threads
+// A warp issues on sub-partition (warp % 4): the roles are placed so that each sub-partition
+// carries two token warps and one residual warp (the producer joins sub-partition 2).
+__device__ __forceinline__ int kres_index(int warp) { return warp == 10 ? 0 : warp == 11 ? 1 : -1; }
+__device__ __forceinline__ int vres_index(int warp) {
+  return warp == 8 ? 0 : warp == 9 ? 1 : warp == 12 ? 2 : warp == 13 ? 3 : -1;
+}
+static_assert(NTW == 8 && NKR == 2 && NVR == 4, "role placement above assumes 8 + 2 + 4 + 1 warps");
 constexpr int T = kTile;               // tokens per tile block
 constexpr int REG = T / NTW;           // tokens of a tile per token warp
 static_assert(REG == 128, "a token lane's chunk (REG * GS / 32 tokens) lies in one bitmap word");
@@ -517,8 +522,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   // low parts), fragments held in registers.  k order within a 16-dim step: the pair (2c, 2c+1)
   // is dims (2c, 2c+8), the pair (2c+8, 2c+9) is dims (2c+1, 2c+9), so one shift of a code word
   // gives both codes of a pair at bits 0 and 16.
-  if (warp >= W_KRES && warp < W_KRES + NKR) {
-    const int kw = warp - W_KRES;
+  if (kres_index(warp) >= 0) {
+    const int kw = kres_index(warp);
     cluster_arrive();  // B1
     named_sync(2, NTW * 32 + NKR * 32);  // q' fragments written by the token warps
     uint2 bf[8];
@@ -606,8 +611,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   // group of 16 records into a shared buffer (two buffers, tiles alternate); step 2: each
   // warp multiplies all groups into the 32 coordinates 32 vw .. 32 vw + 31 it owns.  The token
   // warps add records beyond the staged count themselves, on CUDA cores.
-  if (warp >= W_VRES && warp < W_VRES + NVR) {
-    const int vw = warp - W_VRES;
+  if (vres_index(warp) >= 0) {
+    const int vw = vres_index(warp);
     cluster_arrive();  // B1
     named_sync(3, NTW * 32 + NVR * 32);  // anchor-score table, references and accs are ready
     float accV[2][4][4] = {};  // two independent sets (alternate groups), summed at the end
