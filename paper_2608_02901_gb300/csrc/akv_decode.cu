@@ -540,56 +540,65 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         const TileView tv = tile_view(stage(s), meta[s], U, j0 + tl, P.cap);
         const int nK = min(tv.nk, R);
         float* rs = reinterpret_cast<float*>(stage(s) + P.o_rs);
-        // two groups of 16 records at a time, each as two independent mma chains
-        for (int g16 = kw; g16 * 16 < nK; g16 += 2 * NKR) {
-          uint32_t wd[2][2][8];  // [group][record r8 / r8 + 8][16-dim step]
+        // records addressed in shared memory when the whole block is staged (the common case)
+        auto groups = [&](auto staged_all) {
+          auto rec = [&](uint32_t off) -> const uint8_t* {
+            if constexpr (decltype(staged_all)::value) return tv.st + off;
+            else return tv.at(off);
+          };
+          // two groups of 16 records at a time, each as two independent mma chains
+          for (int g16 = kw; g16 * 16 < nK; g16 += 2 * NKR) {
+            uint32_t wd[2][2][8];  // [group][record r8 / r8 + 8][16-dim step]
 #pragma unroll
-          for (int q = 0; q < 2; ++q)
-#pragma unroll
-            for (int hr = 0; hr < 2; ++hr) {
-              const int sl = (g16 + q * NKR) * 16 + r8 + 8 * hr;
-              uint4 w0 = make_uint4(0u, 0u, 0u, 0u), w1 = w0;
-              if (sl < nK) {
-                w0 = *reinterpret_cast<const uint4*>(tv.at(tv.cd_k + 32u * (uint32_t)sl));
-                w1 = *reinterpret_cast<const uint4*>(tv.at(tv.cd_k + 32u * (uint32_t)sl + 16u));
-              }
-              wd[q][hr][0] = w0.x; wd[q][hr][1] = w0.y; wd[q][hr][2] = w0.z; wd[q][hr][3] = w0.w;
-              wd[q][hr][4] = w1.x; wd[q][hr][5] = w1.y; wd[q][hr][6] = w1.z; wd[q][hr][7] = w1.w;
-            }
-          float d[2][2][4] = {};
-#pragma unroll
-          for (int ks = 0; ks < 8; ++ks)
-#pragma unroll
-            for (int q = 0; q < 2; ++q) {
-              const uint32_t xa = wd[q][0][ks] >> (4 * c4), xb = wd[q][1][ks] >> (4 * c4);
-              const uint4 a = make_uint4(codes2_to_h2(xa), codes2_to_h2(xb), codes2_to_h2(xa >> 2), codes2_to_h2(xb >> 2));
-              mma_f16(d[q][ks & 1], a, bf[ks].x, bf[ks].y);
-            }
-          // columns 2c, 2c+1: high parts of heads 2c, 2c+1 (c < 2) or low parts (c >= 2)
-#pragma unroll
-          for (int q = 0; q < 2; ++q) {
-            float v[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              v[e] = d[q][0][e] + d[q][1][e];
-              v[e] += __shfl_xor_sync(0xffffffffu, v[e], 2);
-            }
-            if (c4 < 2) {
+            for (int q = 0; q < 2; ++q)
 #pragma unroll
               for (int hr = 0; hr < 2; ++hr) {
                 const int sl = (g16 + q * NKR) * 16 + r8 + 8 * hr;
+                uint4 w0 = make_uint4(0u, 0u, 0u, 0u), w1 = w0;
                 if (sl < nK) {
-                  const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_k + 4u * (uint32_t)sl));
+                  w0 = *reinterpret_cast<const uint4*>(rec(tv.cd_k + 32u * (uint32_t)sl));
+                  w1 = *reinterpret_cast<const uint4*>(rec(tv.cd_k + 32u * (uint32_t)sl + 16u));
+                }
+                wd[q][hr][0] = w0.x; wd[q][hr][1] = w0.y; wd[q][hr][2] = w0.z; wd[q][hr][3] = w0.w;
+                wd[q][hr][4] = w1.x; wd[q][hr][5] = w1.y; wd[q][hr][6] = w1.z; wd[q][hr][7] = w1.w;
+              }
+            float d[2][2][4] = {};
 #pragma unroll
-                  for (int e = 0; e < 2; ++e) {
-                    const int g = 2 * c4 + e;
-                    if (g < GS) rs[sl * GS + g] = half_hi(smn) * sq[g] + half_lo(smn) * v[2 * hr + e];
+            for (int ks = 0; ks < 8; ++ks)
+#pragma unroll
+              for (int q = 0; q < 2; ++q) {
+                const uint32_t xa = wd[q][0][ks] >> (4 * c4), xb = wd[q][1][ks] >> (4 * c4);
+                const uint4 a = make_uint4(codes2_to_h2(xa), codes2_to_h2(xb), codes2_to_h2(xa >> 2), codes2_to_h2(xb >> 2));
+                mma_f16(d[q][ks & 1], a, bf[ks].x, bf[ks].y);
+              }
+            // columns 2c, 2c+1: high parts of heads 2c, 2c+1 (c < 2) or low parts (c >= 2)
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              float v[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                v[e] = d[q][0][e] + d[q][1][e];
+                v[e] += __shfl_xor_sync(0xffffffffu, v[e], 2);
+              }
+              if (c4 < 2) {
+#pragma unroll
+                for (int hr = 0; hr < 2; ++hr) {
+                  const int sl = (g16 + q * NKR) * 16 + r8 + 8 * hr;
+                  if (sl < nK) {
+                    const uint32_t smn = *reinterpret_cast<const uint32_t*>(rec(tv.sm_k + 4u * (uint32_t)sl));
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                      const int g = 2 * c4 + e;
+                      if (g < GS) rs[sl * GS + g] = half_hi(smn) * sq[g] + half_lo(smn) * v[2 * hr + e];
+                    }
                   }
                 }
               }
             }
           }
-        }
+        };
+        if (tv.staged == meta[s].y) groups(std::true_type{});
+        else groups(std::false_type{});
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_rs(s));
@@ -669,22 +678,30 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         // B operand straight from the dimension-major code words: this lane's four words hold
         // dimensions 32 vw + 8 nb + r8 (nb = 0..3) of 16 records; records 2c, 2c+1 feed b0,
         // records 2c+8, 2c+9 feed b1
-        const uint32_t woff = tv.cd_v + 4u * (uint32_t)(32 * vw + 4 * r8);
-        for (int grp = 0; grp * 16 < nV; grp += 2) {
+        auto groups = [&](auto staged_all) {  // code words in shared memory when all staged
+          auto rec = [&](uint32_t off) -> const uint8_t* {
+            if constexpr (decltype(staged_all)::value) return tv.st + off;
+            else return tv.at(off);
+          };
+          const uint32_t woff = tv.cd_v + 4u * (uint32_t)(32 * vw + 4 * r8);
+          for (int grp = 0; grp * 16 < nV; grp += 2) {
 #pragma unroll
-          for (int q = 0; q < 2; ++q) {
-            if ((grp + q) * 16 >= nV) break;  // warp-uniform
-            const uint4 a = *reinterpret_cast<const uint4*>(pf + (grp + q) * 512 + lane * 16);
-            const uint4 w4 = *reinterpret_cast<const uint4*>(tv.at(woff + 512u * (uint32_t)(grp + q)));
-            const uint32_t wd[4] = {w4.x, w4.y, w4.z, w4.w};
+            for (int q = 0; q < 2; ++q) {
+              if ((grp + q) * 16 >= nV) break;  // warp-uniform
+              const uint4 a = *reinterpret_cast<const uint4*>(pf + (grp + q) * 512 + lane * 16);
+              const uint4 w4 = *reinterpret_cast<const uint4*>(rec(woff + 512u * (uint32_t)(grp + q)));
+              const uint32_t wd[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
-            for (int nb = 0; nb < 4; ++nb) {
-              // codes of records 2c, 2c+1 (x0) and 2c+8, 2c+9 (x1) in the low four bits
-              const uint32_t x0 = (wd[nb] >> (4 * c4)) & 0xFu, x1 = (wd[nb] >> (4 * c4 + 16)) & 0xFu;
-              mma_bf16(accV[q][nb], a.x, a.y, a.z, a.w, codes2_to_b2(x0 | (x0 << 14)), codes2_to_b2(x1 | (x1 << 14)));
+              for (int nb = 0; nb < 4; ++nb) {
+                // codes of records 2c, 2c+1 (x0) and 2c+8, 2c+9 (x1) in the low four bits
+                const uint32_t x0 = (wd[nb] >> (4 * c4)) & 0xFu, x1 = (wd[nb] >> (4 * c4 + 16)) & 0xFu;
+                mma_bf16(accV[q][nb], a.x, a.y, a.z, a.w, codes2_to_b2(x0 | (x0 << 14)), codes2_to_b2(x1 | (x1 << 14)));
+              }
             }
           }
-        }
+        };
+        if (tv.staged == meta[s].y) groups(std::true_type{});
+        else groups(std::false_type{});
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_empty(s));
