@@ -147,7 +147,9 @@ typedef struct akv_arena_header {
  *   then            cdv  value codes in groups of 16 records (the last group padded with
  *                        zero codes): group G is 128 uint32 words; word
  *                        32 (d/32) + 4 (d%8) + (d%32)/8 holds the code of dimension d of
- *                        record 16 G + s at bits 2s..2s+1.  ceil(nv/16) * 512 bytes.
+ *                        record 16 G + s at bits 2 (s/2) + 16 (s%2) .. +1 (even records
+ *                        in the low half word, odd ones in the high half).
+ *                        ceil(nv/16) * 512 bytes.
  *                        (Dimension-major, because the value side sums over records:
  *                        one 16-byte load gives a thread the codes of 16 records for
  *                        the four dimensions it multiplies.)

@@ -666,14 +666,14 @@ int or_arena_unpack(const uint8_t* arena, uint64_t bytes, int32_t u, or_unit* ou
     cd_off[0] = sm_off[1] + (uint32_t)(((4 * m[1] + 15) / 16) * 16);
     cd_off[1] = cd_off[0] + 32u * (uint32_t)m[0];
     /* value codes: groups of 16 records, dimension-major (word 32 (d/32) + 4 (d%8) + (d%32)/8
-     * of a group holds dimension d, record slot s at bits 2s) */
+     * of a group holds dimension d, record slot s at bits 2 (s/2) + 16 (s%2)) */
     uint32_t nvgrp = (uint32_t)((m[1] + 15) / 16);
     if (b0 + cd_off[1] + 512u * nvgrp != b1) return -1;
     for (int32_t sl = m[1]; sl < 16 * (int32_t)nvgrp; ++sl) /* padding slots hold zero codes */
       for (int dd = 0; dd < 128; ++dd) {
         uint32_t wd = rd32(blk + cd_off[1] + 512u * (uint32_t)(sl / 16) +
                            4u * (uint32_t)(32 * (dd / 32) + 4 * (dd % 8) + (dd % 32) / 8));
-        if ((wd >> (2 * (sl % 16))) & 3u) return -1;
+        if ((wd >> (2 * ((sl % 16) / 2) + 16 * (sl % 2))) & 3u) return -1;
       }
     if (cnt[0] + m[0] > nk || cnt[1] + m[1] > nv) return -1;
     int32_t r[2] = {0, 0};
@@ -701,7 +701,7 @@ int or_arena_unpack(const uint8_t* arena, uint64_t bytes, int32_t u, or_unit* ou
           for (int dd = 0; dd < 128; ++dd) {
             uint32_t wd = rd32(blk + cd_off[1] + 512u * (uint32_t)(r[1] / 16) +
                                4u * (uint32_t)(32 * (dd / 32) + 4 * (dd % 8) + (dd % 32) / 8));
-            rec[dd / 4] |= (uint8_t)(((wd >> (2 * (r[1] % 16))) & 3u) << (2 * (dd % 4)));
+            rec[dd / 4] |= (uint8_t)(((wd >> (2 * ((r[1] % 16) / 2) + 16 * (r[1] % 2))) & 3u) << (2 * (dd % 4)));
           }
         }
         ++r[side];

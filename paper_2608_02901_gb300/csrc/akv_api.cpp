@@ -312,7 +312,7 @@ akv_status akv_cache_pack_host(const akv_params* p, const int32_t* ctx_lens_host
           } else {  // dimension-major groups of 16 records
             uint32_t* grp = (uint32_t*)(cd[1] + 512 * (size_t)(r[1] / 16));
             for (int dd = 0; dd < 128; ++dd)
-              grp[value_code_word(dd)] |= (uint32_t)((src[dd / 4] >> (2 * (dd % 4))) & 3u) << (2 * (r[1] % 16));
+              grp[value_code_word(dd)] |= (uint32_t)((src[dd / 4] >> (2 * (dd % 4))) & 3u) << value_code_bit(r[1] % 16);
           }
           ++r[side];
         }

@@ -354,7 +354,7 @@ __device__ __noinline__ void value_record_add(const TileView& tv, int r, float p
   const uint32_t base = tv.cd_v + 512u * (uint32_t)(r / 16);
   for (int d = 0; d < 128; ++d) {
     const uint32_t w = *reinterpret_cast<const uint32_t*>(tv.at(base + 4u * value_code_word(d)));
-    atomicAdd(&accg[d], ps * (float)((w >> (2 * (r % 16))) & 3u));
+    atomicAdd(&accg[d], ps * (float)((w >> value_code_bit(r % 16)) & 3u));
   }
 }
 
@@ -652,7 +652,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         for (int grp = vw; grp * 16 < nV; grp += NVR) {
           const int r = grp * 16 + sl16;
           if (r < nV && head_lane) {
-            const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_v + 4u * (uint32_t)r));
+            const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.staged == meta[s].y ? tv.st + tv.sm_v + 4u * (uint32_t)r
+                                                                                            : tv.at(tv.sm_v + 4u * (uint32_t)r));
             const float scl = half_lo(smn), mn = half_hi(smn);
 #pragma unroll
             for (int i = 0; i < HPL; ++i) {
@@ -693,9 +694,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
               const uint32_t wd[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
               for (int nb = 0; nb < 4; ++nb) {
-                // codes of records 2c, 2c+1 (x0) and 2c+8, 2c+9 (x1) in the low four bits
-                const uint32_t x0 = (wd[nb] >> (4 * c4)) & 0xFu, x1 = (wd[nb] >> (4 * c4 + 16)) & 0xFu;
-                mma_bf16(accV[q][nb], a.x, a.y, a.z, a.w, codes2_to_b2(x0 | (x0 << 14)), codes2_to_b2(x1 | (x1 << 14)));
+                // records 2c, 2c+1 at bits 2c and 2c + 16, records 2c+8, 2c+9 eight bits higher
+                const uint32_t x = wd[nb] >> (2 * c4);
+                mma_bf16(accV[q][nb], a.x, a.y, a.z, a.w, codes2_to_b2(x), codes2_to_b2(x >> 8));
               }
             }
           }

@@ -655,7 +655,7 @@ __global__ void enc_quant(const EncArgs A) {
   } else {  // value codes: dimension-major groups of 16 records
     uint32_t* grp = reinterpret_cast<uint32_t*>(blk + cd_off - 32u * (uint32_t)r + 512u * (uint32_t)(r / 16));
     for (int c = 0; c < 4; ++c)
-      atomicOr(&grp[value_code_word(4 * lane + c)], ((byte >> (2 * c)) & 3u) << (2 * (r % 16)));
+      atomicOr(&grp[value_code_word(4 * lane + c)], ((byte >> (2 * c)) & 3u) << value_code_bit(r % 16));
   }
   if (lane == 0) *reinterpret_cast<uint32_t*>(blk + sm_off) = sch | (mnh << 16);
 }

@@ -43,6 +43,8 @@ AKV_HD constexpr uint32_t tile_block_bytes(int n, int nk, int nv) {
 }
 // word of dimension d in a group of value codes
 AKV_HD constexpr uint32_t value_code_word(int d) { return 32u * (uint32_t)(d / 32) + 4u * (uint32_t)(d % 8) + (uint32_t)((d % 32) / 8); }
+// bit of record slot s (0..15) in a value-code word: even slots in the low half word
+AKV_HD constexpr uint32_t value_code_bit(int s) { return 2u * (uint32_t)(s / 2) + 16u * (uint32_t)(s % 2); }
 
 // Section indices inside one unit segment, in storage order.
 enum Section { kAnchorK = 0, kAnchorV, kAnchorPos, kTileTable, kTiles, kNumSections };
