@@ -72,7 +72,7 @@ constexpr int T = kTile;               // tokens per tile block
 constexpr int REG = T / NTW;           // tokens of a tile per token warp
 static_assert(REG == 128, "a token lane's chunk (REG * GS / 32 tokens) lies in one bitmap word");
 static_assert(NTW % NVR == 0, "value-residual warps release a stage with NTW / NVR arrivals each");
-constexpr int CH = 64;                 // anchor rows per chunk item
+constexpr int CH = 80;                 // anchor rows per chunk item (a multiple of 16)
 constexpr int kMaxCluster = 16;
 constexpr unsigned kWaitLimit = 1u << 22;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -807,14 +807,15 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   };
 
   // ---- phase 1: anchor scores of this CTA's slice (bf16 tensor cores) ----
-  // warp -> 16-row block (warp / 2) of the 64-row chunk, half of the 128 dims (warp % 2);
-  // rows are swizzled in 16-byte chunks by (row % 8) = r8
+  // work item (16-row block rb, half kh of the 128 dims) -> warp item % NTW; rows are
+  // swizzled in 16-byte chunks by (row % 8) = r8
   for (int it = 0; it < n_ka; ++it) {
     const uint8_t* st = wait_item(it);
     if (ok && !warp_failed(failed)) {
       const int r0 = a0 + it * CH, nr = min(a1 - r0, CH);
-      const int rb = warp >> 1, kh = warp & 1;
-      if (16 * rb < nr) {
+      for (int item = warp; item < 2 * (CH / 16); item += NTW) {
+        const int rb = item >> 1, kh = item & 1;
+        if (16 * rb >= nr) break;
         float d[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int jj = 0; jj < 2; ++jj) {
@@ -842,11 +843,22 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   tw_sync();
   cluster_arrive();  // B1
   cluster_wait();
-  // every entry outside this CTA's slice comes from the peer that owns its anchor
-#pragma unroll 4
-  for (int e = tid; e < k * GS; e += NTT) {
-    const int r = (e / GS) / kc;
-    if (r != rank) SA[e] = cluster.map_shared_rank(SA, r)[e];
+  // every row outside this CTA's slice comes from the peer that owns its anchor: four rows
+  // per thread in flight at a time
+  for (int a4 = tid; a4 < k; a4 += 4 * NTT) {
+    float row[4][GS];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int a = a4 + j * NTT, r = a / kc;
+      if (a < k && r != rank) load_row<GS>(cluster.map_shared_rank(SA, r) + a * GS, row[j]);
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int a = a4 + j * NTT;
+      if (a < k && a / kc != rank)
+#pragma unroll
+        for (int g = 0; g < GS; ++g) SA[a * GS + g] = row[j][g];
+    }
   }
   tw_sync();
   // Reference for the exponentials: the largest anchor score per query row.  Anchors are
@@ -1087,7 +1099,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     const uint8_t* st = wait_item(it);
     if (ok && !warp_failed(failed)) {
       const int r0 = a0 + ci * CH, nr = min(a1 - r0, CH);
-      for (int blk = 0; blk < 4 && 16 * blk < nr; ++blk) {
+      for (int blk = 0; blk < CH / 16 && 16 * blk < nr; ++blk) {
         const int mi = lane >> 3, ri = lane & 7;
         const int row = 16 * blk + (mi & 1) * 8 + ri;
         const int cc = (2 * warp + (mi >> 1)) ^ ri;  // row % 8 == ri
