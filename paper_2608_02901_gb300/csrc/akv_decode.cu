@@ -430,7 +430,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   auto stage = [&](int s) { return ring + (size_t)s * P.stage_bytes; };
 
   // this CTA's anchors (it owns their value weights) and tile blocks
-  const int kc = ((k + C - 1) / C + 15) / 16 * 16;
+  // ceil(k / C) anchors each: their runs lie in about the tiles this CTA reads, so most value
+  // weights are reduced locally
+  const int kc = (k + C - 1) / C;
   const int a0 = min(k, rank * kc), a1 = min(k, a0 + kc);
   const int j0 = (int)((long long)rank * U.nt / C), j1 = (int)((long long)(rank + 1) * U.nt / C);
   const int n_ka = (a1 - a0 + CH - 1) / CH;
@@ -808,7 +810,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 
   // ---- phase 1: anchor scores of this CTA's slice (bf16 tensor cores) ----
   // work item (16-row block rb, half kh of the 128 dims) -> warp item % NTW; rows are
-  // swizzled in 16-byte chunks by (row % 8) = r8
+  // swizzled in 16-byte chunks by (absolute row % 8)
   for (int it = 0; it < n_ka; ++it) {
     const uint8_t* st = wait_item(it);
     if (ok && !warp_failed(failed)) {
@@ -819,7 +821,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         float d[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int jj = 0; jj < 2; ++jj) {
-          const int j = 2 * kh + jj, cc = (4 * j + c4) ^ r8;
+          const int j = 2 * kh + jj, cc = (4 * j + c4) ^ ((r0 + r8) & 7);  // rows r8, r8 + 8: same swizzle
           const uint4 lo = *reinterpret_cast<const uint4*>(st + (16 * rb + r8) * 256 + 16 * cc);
           const uint4 hi = *reinterpret_cast<const uint4*>(st + (16 * rb + r8 + 8) * 256 + 16 * cc);
           const uint2 b0 = qfa[(2 * j) * 32 + lane], b1 = qfa[(2 * j + 1) * 32 + lane];
@@ -1102,7 +1104,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       for (int blk = 0; blk < CH / 16 && 16 * blk < nr; ++blk) {
         const int mi = lane >> 3, ri = lane & 7;
         const int row = 16 * blk + (mi & 1) * 8 + ri;
-        const int cc = (2 * warp + (mi >> 1)) ^ ri;  // row % 8 == ri
+        const int cc = (2 * warp + (mi >> 1)) ^ ((r0 + ri) & 7);  // absolute row % 8
         uint32_t b00, b01, b10, b11;
         ldsm_x4_trans(smem_u32(st + row * 256 + 16 * cc), b00, b01, b10, b11);
         // rows past the slice hold stale bytes: clear their halves of B
@@ -1226,7 +1228,7 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   DecodeParams& P = pl.P;
   // staged bytes of a tile: all of a tile with at most R records per side
   const int cap = (int)(F_MAX + 2 * round16(4u * (uint32_t)R) + 64u * (uint32_t)R);
-  const int kc_max = ((L.max_k + C - 1) / C + 15) / 16 * 16;
+  const int kc_max = (L.max_k + C - 1) / C;
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t o = off;
