@@ -74,7 +74,7 @@ static_assert(REG == 128, "a token lane's chunk (REG * GS / 32 tokens) lies in o
 static_assert(NTW % NVR == 0, "value-residual warps release a stage with NTW / NVR arrivals each");
 constexpr int CH = 80;                 // anchor rows per chunk item (a multiple of 16)
 constexpr int kMaxCluster = 16;
-constexpr unsigned kWaitLimit = 1u << 22;
+constexpr unsigned long long kWaitNs = 2000000000ull;  // an mbarrier wait gives up after 2 s
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint32_t F_MAX = tile_fixed_bytes(T);  // streams, bitmaps, rank words of a full tile
 
@@ -109,6 +109,9 @@ __device__ __forceinline__ void mbar_arrive_cnt(uint32_t bar, uint32_t count) {
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
+// Test for completion of the phase with the given parity (the hardware may hold the thread
+// for a short while before answering no).  A longer sleep hint measured slower: waking on
+// completion lags behind polling.
 __device__ __forceinline__ uint32_t mbar_try(uint32_t bar, uint32_t parity) {
   uint32_t done;
   asm volatile(
@@ -118,22 +121,32 @@ __device__ __forceinline__ uint32_t mbar_try(uint32_t bar, uint32_t parity) {
       : "memory");
   return done;
 }
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
 // Bounded wait of one thread for completion of the phase with the given parity; false if
-// the bound ran out.
+// kWaitNs passed first.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-  for (unsigned i = 0; i < kWaitLimit; ++i)
+  if (mbar_try(bar, parity)) return true;
+  const unsigned long long t0 = global_ns();
+  do {
     if (mbar_try(bar, parity)) return true;
+  } while (global_ns() - t0 < kWaitNs);
   return false;
 }
 // The same by a whole warp: every lane observes the completion itself (its acquire), and
-// all lanes return together with the same result.
+// all lanes return together with the same result (the clock is lane 0's).
 __device__ __forceinline__ bool mbar_wait_w(uint32_t bar, uint32_t parity) {
-  uint32_t done = 0;
-  for (unsigned i = 0; i < kWaitLimit; ++i) {
+  uint32_t done = mbar_try(bar, parity);
+  if (__all_sync(0xffffffffu, done)) return true;
+  const unsigned long long t0 = global_ns();
+  for (;;) {
     if (!done) done = mbar_try(bar, parity);
     if (__all_sync(0xffffffffu, done)) return true;
+    if (__shfl_sync(0xffffffffu, global_ns() - t0 >= kWaitNs ? 1 : 0, 0)) return false;
   }
-  return false;
 }
 // The CTA's failure flag as lane 0 reads it, the same for every lane of the warp.
 __device__ __forceinline__ bool warp_failed(const volatile int* failed) {
@@ -153,6 +166,10 @@ __device__ __forceinline__ void named_arrive(int id, int n) {
 }
 __device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
+// Reduction (no return value) into this CTA's shared memory.
+__device__ __forceinline__ void red_local(float* p, float v) {
+  asm volatile("red.shared.add.f32 [%0], %1;" ::"r"(smem_u32(p)), "f"(v) : "memory");
+}
 // Reduction into shared memory of CTA `rank` of the cluster (possibly this one).
 __device__ __forceinline__ void red_cluster(float* local, int rank, float v) {
   uint32_t remote;
@@ -897,15 +914,19 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     l2[i] = make_float2(0.f, 0.f);
   }
   // Value weights of a run: one reduction per head into the anchor's owner CTA.
+  // The owner is nearly always this CTA (its anchors are the ones its tiles hold), so the
+  // branch is taken once per run, not per head.
   auto flush = [&](int anchor, const float2 (&v)[NP]) {
     if (anchor < 0 || anchor >= k) return;
-    const int owner = anchor >= a0 && anchor < a1 ? rank : anchor / kc;
+    if (anchor >= a0 && anchor < a1) {
+      float* w = &Wt[(anchor - a0) * GS];
 #pragma unroll
-    for (int g = 0; g < GS; ++g) {
-      const float x = (g & 1) ? v[g >> 1].y : v[g >> 1].x;
-      if (x == 0.f) continue;
-      if (owner == rank) atomicAdd(&Wt[(anchor - a0) * GS + g], x);
-      else red_cluster(&Wt[(anchor - owner * kc) * GS + g], owner, x);
+      for (int g = 0; g < GS; ++g) red_local(w + g, (g & 1) ? v[g >> 1].y : v[g >> 1].x);
+    } else {
+      const int owner = anchor / kc;
+      float* w = &Wt[(anchor - owner * kc) * GS];
+#pragma unroll
+      for (int g = 0; g < GS; ++g) red_cluster(w + g, owner, (g & 1) ? v[g >> 1].y : v[g >> 1].x);
     }
   };
 
@@ -919,6 +940,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       ok = mbar_wait_w(bar_rs(s), item_phase(it) & 1u);
       if (!ok) *failed = 1;
     }
+    bool released = false;
     if (ok && !warp_failed(failed)) {
       const TileView tv = tile_view(st, meta[s], U, j0 + tl, P.cap);
       const float* rsb = reinterpret_cast<const float*>(st + P.o_rs);
@@ -1030,6 +1052,14 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             if (av[e] != av[0] && av[e] != av[3]) flush((int)av[e], cw[e]);
         }
       }
+      // the stage is not read again: release it before the reductions, which then never
+      // delay the hand-over to the value-residual warps and the producer
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(bar_p(s));
+        mbar_arrive(bar_empty(s));
+      }
+      released = true;
       // Runs across lanes (anchors never decrease from lane to lane): the next lane's head run
       // continues this lane's tail run when their anchors match; a head run that does not
       // continue the previous lane's tail is complete
@@ -1059,10 +1089,12 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       const uint32_t nkey = __shfl_down_sync(0xffffffffu, key, 1);
       if (key != 0xFFFFFFFFu && (lane == 31 || nkey != key)) flush((int)key, val);
     }
-    __syncwarp();
-    if (lane == 0) {
-      mbar_arrive(bar_p(s));
-      mbar_arrive(bar_empty(s));
+    if (!released) {  // a failed CTA still hands the stage on (warp-uniform)
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(bar_p(s));
+        mbar_arrive(bar_empty(s));
+      }
     }
   }
   // a logit so far above the reference that the sums overflow leaves a non-finite normaliser
