@@ -196,16 +196,17 @@ __device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t& r0, uint3
                : "r"(addr));
 }
 
-// Two 2-bit codes, at bits 0-1 and 16-17 of x, as an fp16 pair of exact small
-// integers: OR them into the mantissa of 1024.0 (0x6400), then subtract 1024.
-__device__ __forceinline__ uint32_t codes2_to_h2(uint32_t x) {
-  uint32_t t, r;
+// Two 2-bit codes c, at bits 0-1 and 16-17 of x, as the fp16 pair 1024 + c: OR them into
+// the mantissa of 1024.0 (0x6400, unit spacing), one logic op.  A product with these
+// operands carries 1024 x (sum of the other operand), taken off once per head.
+__device__ __forceinline__ uint32_t codes2_to_h1024(uint32_t x) {
+  uint32_t t;
   asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(t) : "r"(x), "r"(0x00030003u), "r"(0x64006400u));
-  asm("sub.f16x2 %0, %1, %2;" : "=r"(r) : "r"(t), "r"(0x64006400u));
-  return r;
+  return t;
 }
-// The same as a bf16 pair: OR into the mantissa of 128.0 (0x4300, unit spacing), then
-// t * 1 - 128 (exact).
+// Two 2-bit codes as the exact bf16 pair c: OR into the mantissa of 128.0 (0x4300, unit
+// spacing), then t * 1 - 128.  (The value-residual sum runs over many more products than a
+// key term, so it keeps exact operands: an offset there would cost fp32 accuracy.)
 __device__ __forceinline__ uint32_t codes2_to_b2(uint32_t x) {
   uint32_t t, r;
   asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(t) : "r"(x), "r"(0x00030003u), "r"(0x43004300u));
@@ -427,7 +428,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float* cl = mref + GS;                                  // [GS]
   float* pms = cl + GS;                                   // [GS]
   float* ltot = pms + GS;                                 // [GS]
-  volatile int* failed = reinterpret_cast<volatile int*>(ltot + GS);
+  float* kofs = ltot + GS;  // [GS] 1024 x sum of q' (high + low fp16 parts): the key codes' offset
+  volatile int* failed = reinterpret_cast<volatile int*>(kofs + GS);
   // 16-byte rows: zeros (no key residual) and -inf (a token past the tile's end)
   float* zrow = reinterpret_cast<float*>(smem + P.o_misc + (((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15));
   float* ninfrow = zrow + 4;
@@ -465,6 +467,20 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     return (uint32_t)(ka_on_s + cj / NS);
   };
   auto is_tile = [&](int it) { return it >= n_ka && it < n_ka + n_t; };
+  // Stage and phase parity of the tiles in order, without divisions: tile tl is item n_ka + tl
+  // on stage (n_ka + tl) % NS, and its parity on the tile barriers is (tl / NS) & 1.
+  struct TileCursor {
+    int s, cnt, ns;
+    uint32_t par;
+    __device__ void next() {
+      s = s + 1 == ns ? 0 : s + 1;
+      if (++cnt == ns) {
+        cnt = 0;
+        par ^= 1u;
+      }
+    }
+  };
+  const TileCursor cursor0{n_ka % NS, 0, NS, 0u};
 
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
@@ -484,14 +500,18 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     cluster_arrive();  // B1: this warp never blocks on anything behind B1 before it waits on B1
     bool ok = true, b1_done = false;
     int issued = 0;
-    for (int it = 0; it < n_items; ++it) {
+    int s = 0;
+    uint32_t use = 0;  // it = NS use + s
+    for (int it = 0; it < n_items; ++it, ++s) {
+      if (s == NS) {
+        s = 0;
+        ++use;
+      }
       if (it == n_ka + n_t) {  // anchor values are consumed after B2: let B1 complete, arrive on B2
         cluster_wait();
         cluster_arrive();
         b1_done = true;
       }
-      const int s = it % NS;
-      const uint32_t use = (uint32_t)(it / NS);
       if (it >= NS) ok = mbar_wait_w(bar_empty(s), (use - 1) & 1u);
       if (!ok || warp_failed(failed)) {
         *failed = 1;
@@ -549,10 +569,11 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
     for (int ks = 0; ks < 8; ++ks) bf[ks] = qfk[ks * 32 + lane];
     bool ok = true;
-    for (int tl = 0; tl < n_t; ++tl) {
-      const int s = (n_ka + tl) % NS;
+    TileCursor cur = cursor0;
+    for (int tl = 0; tl < n_t; ++tl, cur.next()) {
+      const int s = cur.s;
       if (ok && !warp_failed(failed)) {
-        ok = mbar_wait_w(bar_full_t(s), (uint32_t)(tl / NS) & 1u);
+        ok = mbar_wait_w(bar_full_t(s), cur.par);
         if (!ok) *failed = 1;
       }
       if (ok && !warp_failed(failed)) {
@@ -587,7 +608,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
               for (int q = 0; q < 2; ++q) {
                 const uint32_t xa = wd[q][0][ks] >> (4 * c4), xb = wd[q][1][ks] >> (4 * c4);
-                const uint4 a = make_uint4(codes2_to_h2(xa), codes2_to_h2(xb), codes2_to_h2(xa >> 2), codes2_to_h2(xb >> 2));
+                const uint4 a = make_uint4(codes2_to_h1024(xa), codes2_to_h1024(xb), codes2_to_h1024(xa >> 2), codes2_to_h1024(xb >> 2));
                 mma_f16(d[q][ks & 1], a, bf[ks].x, bf[ks].y);
               }
             // columns 2c, 2c+1: high parts of heads 2c, 2c+1 (c < 2) or low parts (c >= 2)
@@ -608,7 +629,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
                     for (int e = 0; e < 2; ++e) {
                       const int g = 2 * c4 + e;
-                      if (g < GS) rs[sl * GS + g] = half_hi(smn) * sq[g] + half_lo(smn) * v[2 * hr + e];
+                      if (g < GS) rs[sl * GS + g] = half_hi(smn) * sq[g] + half_lo(smn) * (v[2 * hr + e] - kofs[g]);
                     }
                   }
                 }
@@ -653,9 +674,10 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     for (int i = 0; i < HPL; ++i) pminv[i] = 0.f;
     const int ngrp_st = (R + 15) / 16;
     bool ok = true;
-    for (int tl = 0; tl < n_t; ++tl) {
-      const int s = (n_ka + tl) % NS;
-      const uint32_t par = (uint32_t)(tl / NS) & 1u;
+    TileCursor cur = cursor0;
+    for (int tl = 0; tl < n_t; ++tl, cur.next()) {
+      const int s = cur.s;
+      const uint32_t par = cur.par;
       if (ok && !warp_failed(failed)) {
         ok = mbar_wait_w(bar_full_t(s), par) && mbar_wait_w(bar_p(s), par);
         if (!ok) *failed = 1;
@@ -670,19 +692,23 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         const float* pvb = reinterpret_cast<const float*>(stage(s) + P.o_pv);
         for (int grp = vw; grp * 16 < nV; grp += NVR) {
           const int r = grp * 16 + sl16;
-          if (r < nV && head_lane) {
-            const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.staged == meta[s].y ? tv.st + tv.sm_v + 4u * (uint32_t)r
-                                                                                            : tv.at(tv.sm_v + 4u * (uint32_t)r));
+          // slots past the last record get zero operands
+          if (head_lane) {
+            const bool rec_ok = r < nV;
+            uint32_t smn = 0u;
+            if (rec_ok)
+              smn = *reinterpret_cast<const uint32_t*>(tv.staged == meta[s].y ? tv.st + tv.sm_v + 4u * (uint32_t)r
+                                                                             : tv.at(tv.sm_v + 4u * (uint32_t)r));
             const float scl = half_lo(smn), mn = half_hi(smn);
 #pragma unroll
             for (int i = 0; i < HPL; ++i) {
               const int g = hb + 2 * i;
-              const float p = pvb[r * GS + g];
-              pminv[i] = fmaf(p, mn, pminv[i]);
+              const float p = rec_ok ? pvb[r * GS + g] : 0.f;
               // A-operand place of (record r, head g): group r / 16, lane 4 g + (r % 8) / 2,
               // register 2 ((r / 8) % 2) (high part) or + 1 (low part), half r % 2
               __nv_bfloat16 phi, plo;
               split_b(p * scl, phi, plo);
+              pminv[i] = fmaf(p, mn, pminv[i]);
               unsigned short* dst = reinterpret_cast<unsigned short*>(
                   pf + grp * 512 + (4 * g + ((r & 7) >> 1)) * 16 + ((r >> 3) & 1) * 8 + (r & 1) * 2);
               dst[0] = __bfloat16_as_ushort(phi);
@@ -767,7 +793,10 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   for (int e = a0 * GS + tid; e < a1 * GS; e += NTT) SA[e] = 0.f;
   for (int e = tid; e < kc * GS; e += NTT) Wt[e] = 0.f;  // before B1: peers add into it only after B1
   for (int e = tid; e < ((R + 15) / 16) * 256; e += NTT) reinterpret_cast<uint32_t*>(smem + P.o_pfb)[e] = 0u;
-  if (tid < GS) pms[tid] = 0.f;
+  if (tid < GS) {
+    pms[tid] = 0.f;
+    kofs[tid] = 0.f;
+  }
   if (tid < 4) {
     zrow[tid] = 0.f;
     ninfrow[tid] = -INFINITY;
@@ -804,8 +833,10 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         const __half hi = __float2half_rn(v);
         return g < 4 ? hi : __float2half_rn(v - __half2float(hi));
       };
-      fk.x = pack_h2(part(x[0]), part(x[8]));
-      fk.y = pack_h2(part(x[1]), part(x[9]));
+      const __half h0 = part(x[0]), h8 = part(x[8]), h1 = part(x[1]), h9 = part(x[9]);
+      fk.x = pack_h2(h0, h8);
+      fk.y = pack_h2(h1, h9);
+      red_local(&kofs[g & 3], 1024.f * ((__half2float(h0) + __half2float(h8)) + (__half2float(h1) + __half2float(h9))));
     }
     qfa[ks * 32 + ln] = fa;
     qfk[ks * 32 + ln] = fk;
@@ -932,12 +963,12 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 
   // ---- phase 2: tile blocks ----
   // lane -> four consecutive stored tokens of the warp's 128-token region, every head
-  for (int tl = 0; tl < n_t; ++tl) {
-    const int it = n_ka + tl;
-    const int s = it % NS;
-    const uint8_t* st = wait_item(it);
+  TileCursor cur = cursor0;
+  for (int tl = 0; tl < n_t; ++tl, cur.next()) {
+    const int s = cur.s;
+    const uint8_t* st = stage(s);
     if (ok && !warp_failed(failed)) {
-      ok = mbar_wait_w(bar_rs(s), item_phase(it) & 1u);
+      ok = mbar_wait_w(bar_full_t(s), cur.par) && mbar_wait_w(bar_rs(s), cur.par);
       if (!ok) *failed = 1;
     }
     bool released = false;
