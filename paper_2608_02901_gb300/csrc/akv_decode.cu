@@ -90,6 +90,7 @@ struct DecodeParams {
   int o_sa, o_w, o_qfa, o_qfk, o_qp, o_acc, o_opart, o_misc, o_meta, o_bar, o_ring;
   int o_pfb;       // value-residual operands, two buffers (tiles alternate)
   int o_rs, o_pv;  // inside a stage: key-residual terms, p of the value-record tokens
+  int o_mslot;     // [kMaxCluster][GS] largest anchor score of each CTA's slice, per head
 };
 
 // ---- device helpers ---------------------------------------------------------------
@@ -127,14 +128,14 @@ __device__ __forceinline__ unsigned long long global_ns() {
   return t;
 }
 // Bounded wait of one thread for completion of the phase with the given parity; false if
-// kWaitNs passed first.
+// kWaitNs passed first (the clock is read every 64 tries, so a try costs a few instructions).
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   if (mbar_try(bar, parity)) return true;
   const unsigned long long t0 = global_ns();
-  do {
+  for (unsigned i = 1;; ++i) {
     if (mbar_try(bar, parity)) return true;
-  } while (global_ns() - t0 < kWaitNs);
-  return false;
+    if ((i & 63u) == 0 && global_ns() - t0 >= kWaitNs) return false;
+  }
 }
 // The same by a whole warp: every lane observes the completion itself (its acquire), and
 // all lanes return together with the same result (the clock is lane 0's).
@@ -142,10 +143,10 @@ __device__ __forceinline__ bool mbar_wait_w(uint32_t bar, uint32_t parity) {
   uint32_t done = mbar_try(bar, parity);
   if (__all_sync(0xffffffffu, done)) return true;
   const unsigned long long t0 = global_ns();
-  for (;;) {
+  for (unsigned i = 1;; ++i) {
     if (!done) done = mbar_try(bar, parity);
     if (__all_sync(0xffffffffu, done)) return true;
-    if (__shfl_sync(0xffffffffu, global_ns() - t0 >= kWaitNs ? 1 : 0, 0)) return false;
+    if ((i & 63u) == 0 && __shfl_sync(0xffffffffu, global_ns() - t0 >= kWaitNs ? 1 : 0, 0)) return false;
   }
 }
 // The CTA's failure flag as lane 0 reads it, the same for every lane of the warp.
@@ -166,6 +167,23 @@ __device__ __forceinline__ void named_arrive(int id, int n) {
 }
 __device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
+// A row of GS floats (16-, 8- or 4-byte aligned) stored into the same place in the shared
+// memory of CTA `rank` of the cluster.
+template <int GS>
+__device__ __forceinline__ void st_cluster_row(const float* local, int rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  if constexpr (GS == 4) {
+    const float4 v = *reinterpret_cast<const float4*>(local);
+    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(remote), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+                 : "memory");
+  } else if constexpr (GS == 2) {
+    const float2 v = *reinterpret_cast<const float2*>(local);
+    asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(remote), "f"(v.x), "f"(v.y) : "memory");
+  } else {
+    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(local[0]) : "memory");
+  }
+}
 // Reduction (no return value) into this CTA's shared memory.
 __device__ __forceinline__ void red_local(float* p, float v) {
   asm volatile("red.shared.add.f32 [%0], %1;" ::"r"(smem_u32(p)), "f"(v) : "memory");
@@ -278,21 +296,29 @@ __device__ __forceinline__ float warp_max(float v) {
   return v;
 }
 
-// Unnormalised 128-point Walsh-Hadamard transform of `rows` rows in shared
-// memory, by the token warps.
-__device__ void tw_wht_rows(float* v, int rows) {
-  for (int h = 1; h < 128; h <<= 1) {
-    tw_sync();
-    for (int e = threadIdx.x; e < rows * 64; e += NTT) {
-      const int r = e >> 6, pr = e & 63;
-      const int j = (pr / h) * 2 * h + (pr % h);
-      float* x = v + r * 128;
-      const float a = x[j], b = x[j + h];
-      x[j] = a + b;
-      x[j + h] = a - b;
+// Unnormalised 128-point Walsh-Hadamard transform of one row held by a warp, lane l holding
+// elements 4 l .. 4 l + 3: two butterfly stages inside the lane, five across lanes.
+__device__ __forceinline__ void warp_wht128(float (&x)[4], int lane) {
+  const float a0 = x[0] + x[1], a1 = x[0] - x[1], a2 = x[2] + x[3], a3 = x[2] - x[3];
+  x[0] = a0 + a2;
+  x[1] = a1 + a3;
+  x[2] = a0 - a2;
+  x[3] = a1 - a3;
+#pragma unroll
+  for (int m = 1; m < 32; m <<= 1) {  // stage of distance 4 m: partner lane l ^ m
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float v = __shfl_xor_sync(0xffffffffu, x[j], m);
+      x[j] = (lane & m) ? v - x[j] : x[j] + v;
     }
   }
-  tw_sync();
+}
+// The rotation's signs s_j of dims 4 l .. 4 l + 3 applied to x.
+__device__ __forceinline__ void apply_signs(float (&x)[4], int lane, unsigned long long lo, unsigned long long hi) {
+  const unsigned long long sb = lane < 16 ? lo : hi;
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    if ((sb >> ((4 * lane + j) & 63)) & 1ull) x[j] = -x[j];
 }
 
 // Sections of one unit.
@@ -434,6 +460,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float* zrow = reinterpret_cast<float*>(smem + P.o_misc + (((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15));
   float* ninfrow = zrow + 4;
   uint2* meta = reinterpret_cast<uint2*>(smem + P.o_meta);  // [NS] tile block offset, bytes
+  float* mslot = reinterpret_cast<float*>(smem + P.o_mslot);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + P.o_bar);
   uint8_t* ring = smem + P.o_ring;
   const int NS = P.NS;
@@ -494,11 +521,25 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
+  // B0: every CTA of the cluster has started (its shared memory may take remote stores)
+  cluster_arrive();
+  // first element of this CTA's query (and output) rows, computed where used
+  auto qrow_base = [&]() -> size_t {
+    const int b = u / P.n_kv_heads, h = u % P.n_kv_heads;
+    return ((size_t)b * P.n_q_heads + (size_t)h * P.G + (size_t)hg * GS) * 128;
+  };
 
   // =========================== producer warp ===================================
   if (warp == W_PROD) {
-    cluster_arrive();  // B1: this warp never blocks on anything behind B1 before it waits on B1
-    bool ok = true, b1_done = false;
+    // The first NS items need no free stage.  Before the first wait for one (a stage whose
+    // tile is consumed only after B1) this warp passes B0 and arrives on B1.
+    bool ok = true, b1_arrived = false, b1_done = false;
+    const int b1_at = min(NS, n_ka + n_t);
+    auto arrive_b1 = [&]() {
+      cluster_wait();  // B0
+      cluster_arrive();  // B1
+      b1_arrived = true;
+    };
     int issued = 0;
     int s = 0;
     uint32_t use = 0;  // it = NS use + s
@@ -507,6 +548,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         s = 0;
         ++use;
       }
+      if (it == b1_at) arrive_b1();
       if (it == n_ka + n_t) {  // anchor values are consumed after B2: let B1 complete, arrive on B2
         cluster_wait();
         cluster_arrive();
@@ -538,6 +580,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       issued = it + 1;
       __syncwarp();
     }
+    if (!b1_arrived) arrive_b1();
     if (!b1_done) {
       cluster_wait();
       cluster_arrive();
@@ -563,8 +606,55 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   // gives both codes of a pair at bits 0 and 16.
   if (kres_index(warp) >= 0) {
     const int kw = kres_index(warp);
+    cluster_wait();    // B0
     cluster_arrive();  // B1
-    named_sync(2, NTW * 32 + NKR * 32);  // q' fragments written by the token warps
+    // ---- the rotated query (off the token warps' way to the anchor scores) ----
+    // row g (warp g % NKR): signs, 128-point Walsh-Hadamard transform in registers, scale ->
+    // q' (Appendix A.1, Eq. 12) into qp, its sum into sq
+    if (kw == 0 && lane < GS) kofs[lane] = 0.f;
+    const float f = P.rotate ? P.scale_log2 * (1.0f / 128.0f) : P.scale_log2;
+    for (int g = kw; g < GS; g += NKR) {
+      const uint2 raw = *reinterpret_cast<const uint2*>(P.q + qrow_base() + (size_t)g * 128 + 4 * lane);
+      float x[4] = {__bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.x & 0xFFFFu))),
+                    __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.x >> 16))),
+                    __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.y & 0xFFFFu))),
+                    __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.y >> 16)))};
+      if (P.rotate) {
+        apply_signs(x, lane, P.sign_lo, P.sign_hi);
+        warp_wht128(x, lane);
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) x[j] *= f;
+      *reinterpret_cast<float4*>(qp + g * 128 + 4 * lane) = make_float4(x[0], x[1], x[2], x[3]);
+      const float sg = warp_sum((x[0] + x[1]) + (x[2] + x[3]));
+      if (lane == 0) sq[g] = sg;
+    }
+    named_sync(5, NKR * 32);
+    // key-residual B fragments (k-step ks, lane): column c = lane / 4 is head c % 4 as the fp16
+    // high part (c < 4) or low part; k pairs (2t, 2t+1) <-> dims (16ks + 2t, 16ks + 2t + 8),
+    // (2t+8, 2t+9) <-> (16ks + 2t + 1, 16ks + 2t + 9), t = lane % 4.  kofs sums them (x 1024).
+    {
+      const int g = lane >> 2, c = lane & 3;
+      float part_sum = 0.f;
+      for (int ks = kw; ks < 8; ks += NKR) {
+        uint2 fk = make_uint2(0u, 0u);
+        if ((g & 3) < GS) {
+          const float* x = qp + (g & 3) * 128 + 16 * ks + 2 * c;
+          auto part = [&](float v) {
+            const __half hi = __float2half_rn(v);
+            return g < 4 ? hi : __float2half_rn(v - __half2float(hi));
+          };
+          const __half h0 = part(x[0]), h8 = part(x[8]), h1 = part(x[1]), h9 = part(x[9]);
+          fk.x = pack_h2(h0, h8);
+          fk.y = pack_h2(h1, h9);
+          part_sum += (__half2float(h0) + __half2float(h8)) + (__half2float(h1) + __half2float(h9));
+        }
+        qfk[ks * 32 + lane] = fk;
+      }
+      if ((g & 3) < GS) red_local(&kofs[g & 3], 1024.f * part_sum);
+    }
+    named_sync(5, NKR * 32);
+    named_arrive(2, NTW * 32 + NKR * 32);  // the token warps may use qp and sq
     uint2 bf[8];
 #pragma unroll
     for (int ks = 0; ks < 8; ++ks) bf[ks] = qfk[ks * 32 + lane];
@@ -662,6 +752,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   // warps add records beyond the staged count themselves, on CUDA cores.
   if (vres_index(warp) >= 0) {
     const int vw = vres_index(warp);
+    cluster_wait();    // B0
     cluster_arrive();  // B1
     named_sync(3, NTW * 32 + NVR * 32);  // anchor-score table, references and accs are ready
     float accV[2][4][4] = {};  // two independent sets (alternate groups), summed at the end
@@ -779,70 +870,29 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   }
 
   // =========================== token warps =======================================
-  const int b = u / P.n_kv_heads, h = u % P.n_kv_heads;
-  const size_t qrow0 = ((size_t)b * P.n_q_heads + (size_t)h * P.G + (size_t)hg * GS) * 128;
-
-  // ---- phase 0: query rows, rotated query, tensor-core fragments ----
-  for (int e = tid; e < GS * 128; e += NTT) {
-    const int j = e & 127;
-    const float x = __bfloat162float(P.q[qrow0 + e]);
-    const unsigned long long sb = j < 64 ? P.sign_lo : P.sign_hi;
-    qp[e] = (P.rotate && ((sb >> (j & 63)) & 1ull)) ? -x : x;
-    accs[e] = 0.f;
-  }
+  // ---- phase 0: zeroed tables, anchor-score B fragments (the rotated query is the
+  // key-residual warps' job) ----
+  for (int e = tid; e < GS * 128; e += NTT) accs[e] = 0.f;
   for (int e = a0 * GS + tid; e < a1 * GS; e += NTT) SA[e] = 0.f;
   for (int e = tid; e < kc * GS; e += NTT) Wt[e] = 0.f;  // before B1: peers add into it only after B1
   for (int e = tid; e < ((R + 15) / 16) * 256; e += NTT) reinterpret_cast<uint32_t*>(smem + P.o_pfb)[e] = 0u;
-  if (tid < GS) {
-    pms[tid] = 0.f;
-    kofs[tid] = 0.f;
-  }
+  if (tid < GS) pms[tid] = 0.f;
   if (tid < 4) {
     zrow[tid] = 0.f;
     ninfrow[tid] = -INFINITY;
   }
-  if (P.rotate) tw_wht_rows(qp, GS);
-  else tw_sync();
   {
-    const float f = P.rotate ? P.scale_log2 * (1.0f / 128.0f) : P.scale_log2;
-    for (int e = tid; e < GS * 128; e += NTT) qp[e] *= f;
-  }
-  tw_sync();
-  if (warp < GS) {
-    float s = 0.f;
-    for (int j = lane; j < 128; j += 32) s += qp[warp * 128 + j];
-    s = warp_sum(s);
-    if (lane == 0) sq[warp] = s;
-  }
-  {
-    // fragment (k-step ks, lane ln): one per token thread (8 k-steps x 32 lanes)
+    // fragment (k-step ks, lane ln): one per token thread (8 k-steps x 32 lanes); q in bf16,
+    // k order permuted so that a thread's dims are contiguous
     const int ks = tid >> 5, ln = tid & 31, g = ln >> 2, c = ln & 3;
-    uint2 fa = make_uint2(0u, 0u), fk = make_uint2(0u, 0u);
+    uint2 fa = make_uint2(0u, 0u);
     if (g < GS) {
-      // anchor-score B operand: q in bf16, k order permuted so a thread's dims are contiguous
-      const __nv_bfloat16* qr = P.q + qrow0 + (size_t)g * 128;
-      const int d0 = 32 * (ks >> 1) + 8 * c + 4 * (ks & 1);
-      fa.x = pack_b2(qr[d0], qr[d0 + 1]);
-      fa.y = pack_b2(qr[d0 + 2], qr[d0 + 3]);
-    }
-    if ((g & 3) < GS) {
-      // key-residual B operand, column g: head g % 4, fp16 high part (g < 4) or low part;
-      // k pairs (2c, 2c+1) <-> dims (16ks + 2c, 16ks + 2c + 8), (2c+8, 2c+9) <-> (16ks + 2c + 1, 16ks + 2c + 9)
-      const float* x = qp + (g & 3) * 128 + 16 * ks + 2 * c;
-      auto part = [&](float v) {
-        const __half hi = __float2half_rn(v);
-        return g < 4 ? hi : __float2half_rn(v - __half2float(hi));
-      };
-      const __half h0 = part(x[0]), h8 = part(x[8]), h1 = part(x[1]), h9 = part(x[9]);
-      fk.x = pack_h2(h0, h8);
-      fk.y = pack_h2(h1, h9);
-      red_local(&kofs[g & 3], 1024.f * ((__half2float(h0) + __half2float(h8)) + (__half2float(h1) + __half2float(h9))));
+      const uint2 raw = *reinterpret_cast<const uint2*>(P.q + qrow_base() + (size_t)g * 128 + 32 * (ks >> 1) + 8 * c + 4 * (ks & 1));
+      fa = raw;  // dims d0 .. d0 + 3 as two bf16 pairs
     }
     qfa[ks * 32 + ln] = fa;
-    qfk[ks * 32 + ln] = fk;
   }
   tw_sync();
-  named_arrive(2, NTW * 32 + NKR * 32);  // the key-residual warps may read q' fragments and sq
 
   bool ok = true;
   auto wait_item = [&](int i) -> const uint8_t* {
@@ -891,37 +941,24 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     release_chunk(it);
   }
   tw_sync();
-  cluster_arrive();  // B1
-  cluster_wait();
-  // every row outside this CTA's slice comes from the peer that owns its anchor: four rows
-  // per thread in flight at a time
-  for (int a4 = tid; a4 < k; a4 += 4 * NTT) {
-    float row[4][GS];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int a = a4 + j * NTT, r = a / kc;
-      if (a < k && r != rank) load_row<GS>(cluster.map_shared_rank(SA, r) + a * GS, row[j]);
-    }
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int a = a4 + j * NTT;
-      if (a < k && a / kc != rank)
-#pragma unroll
-        for (int g = 0; g < GS; ++g) SA[a * GS + g] = row[j][g];
-    }
-  }
-  tw_sync();
-  // Reference for the exponentials: the largest anchor score per query row.  Anchors are
-  // tokens of the unit, so it never exceeds the true maximum logit; every CTA of the
-  // cluster holds the same table and so the same reference, which makes the cluster
-  // combine a plain sum.
+  // The slice goes into every peer's table (remote stores, done before B1 completes), and
+  // its largest score per head into slot `rank` of every CTA.  Reference for the exponentials:
+  // the largest anchor score per query row.  Anchors are tokens of the unit, so it never
+  // exceeds the true maximum logit; every CTA of the cluster takes the same reference, which
+  // makes the cluster combine a plain sum.
+  cluster_wait();  // B0: the peers have started
   {
     float mx[GS];
 #pragma unroll
     for (int g = 0; g < GS; ++g) mx[g] = -INFINITY;
-    for (int a = tid; a < k; a += NTT)
+    for (int a = a0 + tid; a < a1; a += NTT) {
+      float row[GS];
+      load_row<GS>(SA + a * GS, row);
 #pragma unroll
-      for (int g = 0; g < GS; ++g) mx[g] = fmaxf(mx[g], SA[a * GS + g]);
+      for (int g = 0; g < GS; ++g) mx[g] = fmaxf(mx[g], row[g]);
+      for (int r = 0; r < C; ++r)
+        if (r != rank) st_cluster_row<GS>(SA + a * GS, r);
+    }
 #pragma unroll
     for (int g = 0; g < GS; ++g) {
       const float m = warp_max(mx[g]);
@@ -931,10 +968,19 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     if (tid < GS) {
       float m = red[tid];
       for (int w = 1; w < NTW; ++w) m = fmaxf(m, red[w * GS + tid]);
-      mref[tid] = m;
+      mslot[rank * GS + tid] = m;
+      for (int r = 0; r < C; ++r)
+        if (r != rank) st_cluster_row<1>(mslot + rank * GS + tid, r);
     }
-    tw_sync();
   }
+  cluster_arrive();  // B1
+  cluster_wait();
+  if (tid < GS) {
+    float m = mslot[tid];
+    for (int r = 1; r < C; ++r) m = fmaxf(m, mslot[r * GS + tid]);
+    mref[tid] = m;
+  }
+  tw_sync();
   named_arrive(3, NTW * 32 + NVR * 32);  // the value-residual warps may use SA, mref and accs
   // pairs of heads for the packed arithmetic (GS = 1: one head, the pair's second lane idle)
   constexpr int NP = GS >= 2 ? GS / 2 : 1;
@@ -962,6 +1008,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   };
 
   // ---- phase 2: tile blocks ----
+  named_sync(2, NTW * 32 + NKR * 32);  // q' rows and their sums from the key-residual warps
   // lane -> four consecutive stored tokens of the warp's 128-token region, every head
   TileCursor cur = cursor0;
   for (int tl = 0; tl < n_t; ++tl, cur.next()) {
@@ -1200,18 +1247,19 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   }
   // this CTA's value residuals (staged records from the value-residual warps, overflow
   // records and sum p * min from the token warps), then the inverse rotation once
-  for (int e = tid; e < GS * 128; e += NTT) accs[e] += pms[e >> 7];
-  if (P.rotate) tw_wht_rows(accs, GS);
-  else tw_sync();
-  for (int e = tid; e < GS * 128; e += NTT) {
-    const int j = e & 127;
-    float r = accs[e];
+  // (warp g < GS: row g in registers; the inverse of q' = H (s o q) / 128 on the value side
+  // is s o H(.) / 128)
+  if (warp < GS) {
+    const float4 v = *reinterpret_cast<const float4*>(accs + warp * 128 + 4 * lane);
+    const float pm = pms[warp];
+    float x[4] = {v.x + pm, v.y + pm, v.z + pm, v.w + pm};
     if (P.rotate) {
-      const unsigned long long sb = j < 64 ? P.sign_lo : P.sign_hi;
-      r = ((sb >> (j & 63)) & 1ull) ? -r : r;
-      r *= (1.0f / 128.0f);
+      warp_wht128(x, lane);
+      apply_signs(x, lane, P.sign_lo, P.sign_hi);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) x[j] *= (1.0f / 128.0f);
     }
-    opart[e] = r;
+    *reinterpret_cast<float4*>(opart + warp * 128 + 4 * lane) = make_float4(x[0], x[1], x[2], x[3]);
   }
   tw_sync();
   if (r8 < GS) {
@@ -1239,7 +1287,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
       for (int r = 0; r < kMaxCluster; ++r) sum += v[r];
       const float y = bad ? __int_as_float(0x7FC00000) : sum / ltot[e >> 7];
-      const size_t o = qrow0 + e;
+      const size_t o = qrow_base() + e;
       P.out[o] = __float2bfloat16_rn(y);
       if (P.out_f32) P.out_f32[o] = y;
     }
@@ -1307,6 +1355,7 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_opart = take((size_t)std::max(GS * 128, NTW * GS) * 4);
   P.o_misc = take((size_t)(((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15) + 32);
   P.o_meta = take(8 * 8);
+  P.o_mslot = take((size_t)kMaxCluster * GS * 4);
   P.o_bar = take(5 * 8 * 8);
   P.o_pfb = take((size_t)2 * ((R + 15) / 16) * 512);
   // a stage: staged bytes (a tile block's head, or an anchor chunk), then the key-residual
