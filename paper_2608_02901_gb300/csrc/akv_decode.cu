@@ -91,6 +91,9 @@ struct DecodeParams {
   int o_pfb;       // value-residual operands, two buffers (tiles alternate)
   int o_rs, o_pv;  // inside a stage: key-residual terms, p of the value-record tokens
   int o_mslot;     // [kMaxCluster][GS] largest anchor score of each CTA's slice, per head
+  int o_lslot;     // [kMaxCluster][GS] each CTA's normaliser share
+  int o_fslot;     // [kMaxCluster] each CTA's failure flag
+  int o_ofin;      // [C][per] staging: partial output numerators of this CTA's share, per rank
 };
 
 // ---- device helpers ---------------------------------------------------------------
@@ -183,6 +186,19 @@ __device__ __forceinline__ void st_cluster_row(const float* local, int rank) {
   } else {
     asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(local[0]) : "memory");
   }
+}
+// v stored at the place of `local` in the shared memory of CTA `rank` of the cluster.
+__device__ __forceinline__ void st_cluster_v4(const float* local, int rank, float4 v) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(remote), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+               : "memory");
+}
+// An int stored into the same place in the shared memory of CTA `rank` of the cluster.
+__device__ __forceinline__ void st_cluster_int(const int* local, int rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("st.shared::cluster.s32 [%0], %1;" ::"r"(remote), "r"(local[0]) : "memory");
 }
 // Reduction (no return value) into this CTA's shared memory.
 __device__ __forceinline__ void red_local(float* p, float v) {
@@ -461,6 +477,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float* ninfrow = zrow + 4;
   uint2* meta = reinterpret_cast<uint2*>(smem + P.o_meta);  // [NS] tile block offset, bytes
   float* mslot = reinterpret_cast<float*>(smem + P.o_mslot);
+  float* lslot = reinterpret_cast<float*>(smem + P.o_lslot);
+  int* fslot = reinterpret_cast<int*>(smem + P.o_fslot);
+  float* ofin = reinterpret_cast<float*>(smem + P.o_ofin);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + P.o_bar);
   uint8_t* ring = smem + P.o_ring;
   const int NS = P.NS;
@@ -592,9 +611,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     __syncwarp();
     cluster_wait();  // B2
     cluster_arrive();
-    cluster_wait();  // B3
-    cluster_arrive();
-    cluster_wait();  // B4
+    cluster_wait();  // B3 (the last cluster barrier: nothing remote follows it)
     return;
   }
 
@@ -737,9 +754,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     cluster_arrive();
     cluster_wait();  // B2
     cluster_arrive();
-    cluster_wait();  // B3
-    cluster_arrive();
-    cluster_wait();  // B4
+    cluster_wait();  // B3 (the last cluster barrier: nothing remote follows it)
     return;
   }
 
@@ -863,9 +878,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     cluster_arrive();
     cluster_wait();  // B2
     cluster_arrive();
-    cluster_wait();  // B3
-    cluster_arrive();
-    cluster_wait();  // B4
+    cluster_wait();  // B3 (the last cluster barrier: nothing remote follows it)
     return;
   }
 
@@ -1188,19 +1201,21 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     if (lane == 0) red[warp * GS + g] = sl;
   }
   tw_sync();
-  if (tid < GS) {
+  if (tid < GS) {  // this CTA's normaliser share, into slot `rank` of every CTA
     float sl = 0.f;
     for (int w = 0; w < NTW; ++w) sl += red[w * GS + tid];
-    cl[tid] = sl;
+    lslot[rank * GS + tid] = sl;
+    for (int r = 0; r < C; ++r)
+      if (r != rank) st_cluster_row<1>(lslot + rank * GS + tid, r);
   }
   tw_sync();
 
   // ---- phase 3: combine across the cluster (one common reference: plain sums) ----
-  cluster_arrive();  // B2: every value-weight reduction into this CTA has landed
+  cluster_arrive();  // B2: every value-weight reduction and normaliser share has landed
   cluster_wait();
   if (tid < GS) {
     float Lt = 0.f;
-    for (int r = 0; r < C; ++r) Lt += cluster.map_shared_rank(cl, r)[tid];
+    for (int r = 0; r < C; ++r) Lt += lslot[r * GS + tid];
     ltot[tid] = Lt;
   }
   // weights of the owned anchors times their values (bf16 tensor cores, weights as hi + lo);
@@ -1271,29 +1286,39 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     }
   }
   tw_sync();
+  // Elements are shared out in blocks of `per` (a multiple of 4); each block of this CTA's
+  // partial output goes, as 16-byte remote stores, into slot `rank` of the staging rows of
+  // the CTA that writes it, and this CTA's failure flag into slot `rank` of every CTA.  After
+  // B3 no CTA touches another's shared memory, so none waits for the others before it exits.
+  const int E = GS * 128;
+  const int per = 4 * ((E / 4 + C - 1) / C);
+  for (int e = 4 * tid; e < E; e += 4 * NTT) {
+    const int owner = e / per;
+    float* dst = ofin + rank * per + (e - owner * per);  // the same place in the owner's rows
+    const float4 v = *reinterpret_cast<const float4*>(opart + e);
+    if (owner == rank) *reinterpret_cast<float4*>(dst) = v;
+    else st_cluster_v4(dst, owner, v);
+  }
+  if (tid == 0) {
+    fslot[rank] = *failed;
+    for (int r = 0; r < C; ++r)
+      if (r != rank) st_cluster_int(fslot + rank, r);
+  }
   cluster_arrive();  // B3
   cluster_wait();
   {
-    const int E = GS * 128;
-    const int per = (E + C - 1) / C;
     const int e0 = rank * per, e1 = min(E, e0 + per);
     bool bad = false;
-    for (int r = 0; r < C; ++r) bad |= cluster.map_shared_rank(const_cast<int*>(failed), r)[0] != 0;
+    for (int r = 0; r < C; ++r) bad |= fslot[r] != 0;
     for (int e = e0 + tid; e < e1; e += NTT) {
-      float v[kMaxCluster];
-#pragma unroll
-      for (int r = 0; r < kMaxCluster; ++r) v[r] = r < C ? cluster.map_shared_rank(opart, r)[e] : 0.f;
       float sum = 0.f;
-#pragma unroll
-      for (int r = 0; r < kMaxCluster; ++r) sum += v[r];
+      for (int r = 0; r < C; ++r) sum += ofin[r * per + (e - e0)];
       const float y = bad ? __int_as_float(0x7FC00000) : sum / ltot[e >> 7];
       const size_t o = qrow_base() + e;
       P.out[o] = __float2bfloat16_rn(y);
       if (P.out_f32) P.out_f32[o] = y;
     }
   }
-  cluster_arrive();  // B4
-  cluster_wait();
 }
 
 struct DeviceInfo {
@@ -1356,6 +1381,9 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_misc = take((size_t)(((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15) + 32);
   P.o_meta = take(8 * 8);
   P.o_mslot = take((size_t)kMaxCluster * GS * 4);
+  P.o_lslot = take((size_t)kMaxCluster * GS * 4);
+  P.o_fslot = take((size_t)kMaxCluster * 4);
+  P.o_ofin = take((size_t)(GS * 128 + 4 * kMaxCluster) * 4);  // C x per <= GS 128 + 4 C
   P.o_bar = take(5 * 8 * 8);
   P.o_pfb = take((size_t)2 * ((R + 15) / 16) * 512);
   // a stage: staged bytes (a tile block's head, or an anchor chunk), then the key-residual
