@@ -9,18 +9,20 @@
 //                     shared-memory stages, one bulk asynchronous copy per item, each
 //                     completing a transaction-counted mbarrier:
 //                     [anchor-key chunks] [tile blocks] [anchor-value chunks]
-//   2 key-residual warps  per tile: q' . c for the staged key records on tensor cores,
-//                     straight from the packed 2-bit codes (q' = H(s o q)/128,
-//                     Appendix A.1 Eq. 12, as fp16 high + low parts)
-//   8 token warps     phase 1: anchor scores S_A = q . k_a of the CTA's anchor slice
-//                     (bf16 tensor cores), gathered cluster-wide through DSMEM;
+//   2 key-residual warps  first the rotated query q' = H(s o q)/128 (Appendix A.1, Eq. 12;
+//                     a warp-local Walsh-Hadamard transform) and its fp16 high + low
+//                     fragments; then per tile: q' . c for the staged key records on tensor
+//                     cores, straight from the packed 2-bit codes
+//   8 token warps     phase 1: anchor scores S_A = q . k_a of the CTA's anchor slice (bf16
+//                     tensor cores), pushed into every peer's table (DSMEM stores);
 //                     per tile: logits gamma_i S_A[a(i)] + residual term, p = 2^(l - m),
-//                     value-residual operands, and the value weights
+//                     the value-residual warps' p, and the value weights
 //                     w[a] = sum_i p_i gamma_i (Eq. 3) -- tokens are stored sorted by
-//                     value anchor, so w is a sum over runs: a one-hot (anchors x tokens)
-//                     times (tokens x heads) product on the tensor cores, flushed into the
-//                     anchor's owner CTA with DSMEM reductions;
-//                     phase 3: the anchor-value product of the CTA's anchors, cluster combine
+//                     value anchor, so w is a sum over runs: per lane its head and tail
+//                     runs, merged across lanes by a warp segmented scan, one reduction
+//                     per run into the anchor's owner CTA (shared or DSMEM red);
+//                     phase 3: the anchor-value product of the CTA's anchors, the inverse
+//                     rotation of the value-residual sum, cluster combine
 //   4 value-residual warps  per tile: sum of (p scale) c over the staged value records on
 //                     tensor cores, in the rotated domain
 // Stages are handed between the roles with mbarriers, so different roles work on
@@ -90,6 +92,7 @@ struct DecodeParams {
   int o_sa, o_w, o_qfa, o_qfk, o_qp, o_acc, o_opart, o_misc, o_meta, o_bar, o_ring;
   int o_pfb;       // value-residual operands, two buffers (tiles alternate)
   int o_rs, o_pv;  // inside a stage: key-residual terms, p of the value-record tokens
+  int o_hdr;       // [NS][2] uint4: tile header per stage (put_header)
   int o_mslot;     // [kMaxCluster][GS] largest anchor score of each CTA's slice, per head
   int o_lslot;     // [kMaxCluster][GS] each CTA's normaliser share
   int o_fslot;     // [kMaxCluster] each CTA's failure flag
@@ -395,6 +398,34 @@ __device__ __forceinline__ TileView tile_view(const uint8_t* st, const uint2 met
   return v;
 }
 
+// A tile block's header as the key-residual warps publish it per stage (two 16-byte words:
+// block offset, block bytes, n | nw << 16, nk | nv << 16, then the four section offsets), so
+// that the token and value-residual warps skip the dependent loads of tile_view.
+__device__ __forceinline__ void put_header(uint4* hdr, const TileView& v, uint2 meta) {
+  const int lane = threadIdx.x & 31;
+  if (lane == 0)
+    hdr[0] = make_uint4(meta.x, meta.y, (uint32_t)v.n | ((uint32_t)v.nw << 16), (uint32_t)v.nk | ((uint32_t)v.nv << 16));
+  if (lane == 1) hdr[1] = make_uint4(v.sm_k, v.sm_v, v.cd_k, v.cd_v);
+}
+__device__ __forceinline__ TileView header_view(const uint8_t* st, const uint4* hdr, const UnitView& U, int cap, uint2* meta_out) {
+  const uint4 h0 = hdr[0], h1 = hdr[1];
+  TileView v;
+  v.st = st;
+  v.gb = U.tiles + h0.x;
+  v.staged = min(h0.y, (uint32_t)cap);
+  v.n = (int)(h0.z & 0xFFFFu);
+  v.nw = (int)(h0.z >> 16);
+  v.n64 = 64 * v.nw;
+  v.nk = (int)(h0.w & 0xFFFFu);
+  v.nv = (int)(h0.w >> 16);
+  v.sm_k = h1.x;
+  v.sm_v = h1.y;
+  v.cd_k = h1.z;
+  v.cd_v = h1.w;
+  *meta_out = make_uint2(h0.x, h0.y);
+  return v;
+}
+
 // Records beyond the staged count (a locally dense tile) take these rare paths on CUDA
 // cores, kept out of line so that the token loop stays small.
 // Key residual term scale (q'_g . c) + min sum(q'_g) of key record r.
@@ -477,6 +508,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float* ninfrow = zrow + 4;
   uint2* meta = reinterpret_cast<uint2*>(smem + P.o_meta);  // [NS] tile block offset, bytes
   float* mslot = reinterpret_cast<float*>(smem + P.o_mslot);
+  uint4* hdrs = reinterpret_cast<uint4*>(smem + P.o_hdr);  // [NS][2]
   float* lslot = reinterpret_cast<float*>(smem + P.o_lslot);
   int* fslot = reinterpret_cast<int*>(smem + P.o_fslot);
   float* ofin = reinterpret_cast<float*>(smem + P.o_ofin);
@@ -685,6 +717,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       }
       if (ok && !warp_failed(failed)) {
         const TileView tv = tile_view(stage(s), meta[s], U, j0 + tl, P.cap);
+        if (kw == 0) put_header(hdrs + 2 * s, tv, meta[s]);
         const int nK = min(tv.nk, R);
         float* rs = reinterpret_cast<float*>(stage(s) + P.o_rs);
         // records addressed in shared memory when the whole block is staged (the common case)
@@ -790,10 +823,11 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       }
       const bool go = ok && !warp_failed(failed);
       TileView tv;
+      uint2 mt = make_uint2(0u, 0u);  // block offset and bytes, from the header
       uint8_t* pf = smem + P.o_pfb + (tl & 1) * ngrp_st * 512;
       int nV = 0;
       if (go) {
-        tv = tile_view(stage(s), meta[s], U, j0 + tl, P.cap);
+        tv = header_view(stage(s), hdrs + 2 * s, U, P.cap, &mt);
         nV = min(tv.nv, R);
         const float* pvb = reinterpret_cast<const float*>(stage(s) + P.o_pv);
         for (int grp = vw; grp * 16 < nV; grp += NVR) {
@@ -803,7 +837,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             const bool rec_ok = r < nV;
             uint32_t smn = 0u;
             if (rec_ok)
-              smn = *reinterpret_cast<const uint32_t*>(tv.staged == meta[s].y ? tv.st + tv.sm_v + 4u * (uint32_t)r
+              smn = *reinterpret_cast<const uint32_t*>(tv.staged == mt.y ? tv.st + tv.sm_v + 4u * (uint32_t)r
                                                                              : tv.at(tv.sm_v + 4u * (uint32_t)r));
             const float scl = half_lo(smn), mn = half_hi(smn);
 #pragma unroll
@@ -852,7 +886,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             }
           }
         };
-        if (tv.staged == meta[s].y) groups(std::true_type{});
+        if (tv.staged == mt.y) groups(std::true_type{});
         else groups(std::false_type{});
       }
       __syncwarp();
@@ -1033,7 +1067,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     }
     bool released = false;
     if (ok && !warp_failed(failed)) {
-      const TileView tv = tile_view(st, meta[s], U, j0 + tl, P.cap);
+      uint2 mt;
+      const TileView tv = header_view(st, hdrs + 2 * s, U, P.cap, &mt);
       const float* rsb = reinterpret_cast<const float*>(st + P.o_rs);
       const int t0 = warp * REG + 4 * lane;
       // tail: the run that ends this lane's tokens (its anchor `key`), head: the run that
@@ -1380,6 +1415,7 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_opart = take((size_t)std::max(GS * 128, NTW * GS) * 4);
   P.o_misc = take((size_t)(((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15) + 32);
   P.o_meta = take(8 * 8);
+  P.o_hdr = take(8 * 32);
   P.o_mslot = take((size_t)kMaxCluster * GS * 4);
   P.o_lslot = take((size_t)kMaxCluster * GS * 4);
   P.o_fslot = take((size_t)kMaxCluster * 4);
