@@ -59,17 +59,23 @@ namespace {
 // warp roles
 constexpr int NTW = 8;                 // token warps (warps 0 .. 7)
 constexpr int NTT = NTW * 32;          // token threads
-constexpr int NKR = 2;                 // key-residual warps: 10, 11
+constexpr int NKR = 3;                 // key-residual warps: 10, 11, 15
 constexpr int NVR = 4;                 // value-residual warps: 8, 9, 12, 13
-constexpr int W_PROD = NTW + NKR + NVR;  // producer warp (14)
-constexpr int NT = (W_PROD + 1) * 32;  // 480 threads
-// A warp issues on sub-partition (warp % 4): the roles are placed so that each sub-partition
-// carries two token warps and one residual warp (the producer joins sub-partition 2).
-__device__ __forceinline__ int kres_index(int warp) { return warp == 10 ? 0 : warp == 11 ? 1 : -1; }
+constexpr int W_PROD = 14;             // producer warp
+constexpr int NT = 16 * 32;            // 512 threads: four warpgroups
+// A warp issues on sub-partition (warp % 4): each sub-partition carries two token warps and
+// two of the others.  In the reallocating kernel, warpgroups 0-1 (the token warps) raise
+// their register budget and warpgroups 2-3 lower theirs (setmaxnreg): 256 x kRegTok +
+// 256 x kRegRes equals 512 x 128, the launch's own total when the kernel was compiled to 128
+// registers a thread; the host launches it only then, so the raise never waits for registers
+// the block does not hold.
+constexpr int kRegTok = 152, kRegRes = 104;
+static_assert(2 * 128 * kRegTok + 2 * 128 * kRegRes == NT * 128, "register split must equal the launch total");
+__device__ __forceinline__ int kres_index(int warp) { return warp == 10 ? 0 : warp == 11 ? 1 : warp == 15 ? 2 : -1; }
 __device__ __forceinline__ int vres_index(int warp) {
   return warp == 8 ? 0 : warp == 9 ? 1 : warp == 12 ? 2 : warp == 13 ? 3 : -1;
 }
-static_assert(NTW == 8 && NKR == 2 && NVR == 4, "role placement above assumes 8 + 2 + 4 + 1 warps");
+static_assert(NTW == 8 && NKR == 3 && NVR == 4 && W_PROD == 14, "role placement above assumes 8 + 3 + 4 + 1 warps");
 constexpr int T = kTile;               // tokens per tile block
 constexpr int REG = T / NTW;           // tokens of a tile per token warp
 static_assert(REG == 128, "a token lane's chunk (REG * GS / 32 tokens) lies in one bitmap word");
@@ -475,7 +481,7 @@ __device__ __forceinline__ void load_row(const float* p, float (&out)[GS]) {
   }
 }
 
-template <int GS>
+template <int GS, bool RA>
 __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P) {
   extern __shared__ __align__(128) uint8_t smem[];
   cg::cluster_group cluster = cg::this_cluster();
@@ -572,6 +578,10 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
+  if constexpr (RA) {  // launched only when its register count is exactly 128 (decode_kernel)
+    if (warp < NTW) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegTok));
+    else asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegRes));
+  }
   // B0: every CTA of the cluster has started (its shared memory may take remote stores)
   cluster_arrive();
   // first element of this CTA's query (and output) rows, computed where used
@@ -1467,6 +1477,23 @@ struct LaunchKey {
   }
 };
 
+using KernelFn = void (*)(const DecodeParams);
+// The kernel for GS heads per CTA: for GS = 4 the register-reallocating one when its launch
+// register count is the 128 the split assumes (checked once), else the plain one.
+template <int GS>
+KernelFn decode_kernel() {
+  if constexpr (GS == 4) {
+    static const bool ra = [] {
+      cudaFuncAttributes a{};
+      return cudaFuncGetAttributes(&a, akv_decode_kernel<4, true>) == cudaSuccess && a.numRegs == 128;
+    }();
+    cudaGetLastError();
+    return ra ? akv_decode_kernel<4, true> : akv_decode_kernel<4, false>;
+  } else {
+    return akv_decode_kernel<GS, false>;
+  }
+}
+
 template <int GS>
 int plan_for(const Layout& L, const LaunchKey& key, int vunits, Plan* out, std::string* why) {
   static std::mutex mu;
@@ -1482,10 +1509,10 @@ int plan_for(const Layout& L, const LaunchKey& key, int vunits, Plan* out, std::
   const DeviceInfo di = device_info();
   // The attribute is per kernel, not per launch: raise it to the device limit
   // once, so that every cached configuration stays launchable.
-  cudaError_t e =
-      cudaFuncSetAttribute(akv_decode_kernel<GS>, cudaFuncAttributeMaxDynamicSharedMemorySize, di.smem_optin);
+  const KernelFn kfn = decode_kernel<GS>();
+  cudaError_t e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, di.smem_optin);
   if (e != cudaSuccess) return (int)e;
-  e = cudaFuncSetAttribute(akv_decode_kernel<GS>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  e = cudaFuncSetAttribute(kfn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (e != cudaSuccess) return (int)e;
   // Cluster size: the most CTAs per unit such that every cluster is resident at once (one CTA
   // per SM), no more CTAs than tiles in the longest unit.  Sizes are tried downwards one by
@@ -1509,7 +1536,7 @@ int plan_for(const Layout& L, const LaunchKey& key, int vunits, Plan* out, std::
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int nclusters = 0;
-    e = cudaOccupancyMaxActiveClusters(&nclusters, akv_decode_kernel<GS>, &cfg);
+    e = cudaOccupancyMaxActiveClusters(&nclusters, kfn, &cfg);
     // prefer a size whose clusters all fit at once; an explicit override only needs one to fit
     if (e == cudaSuccess && (nclusters >= vunits || (key.cluster_env == C && nclusters >= 1))) break;
     cudaGetLastError();
@@ -1562,7 +1589,7 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, akv_decode_kernel<GS>, P);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, decode_kernel<GS>(), P);
   if (e != cudaSuccess) return (int)e;
   return (int)cudaGetLastError();
 }
