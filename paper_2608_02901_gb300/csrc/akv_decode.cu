@@ -177,6 +177,11 @@ __device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sy
 __device__ __forceinline__ void named_arrive(int id, int n) {
   asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
+// Programmatic dependent launch: the next launch in the stream may start its prologue (it
+// only streams the cache, which no decode launch writes) while this one runs; a thread waits
+// for the preceding launch to complete before it reads the query or writes an output.
+__device__ __forceinline__ void pdl_allow_next() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait_prev() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 // A row of GS floats (16-, 8- or 4-byte aligned) stored into the same place in the shared
@@ -578,6 +583,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
+  pdl_allow_next();
   if constexpr (RA) {  // launched only when its register count is exactly 128 (decode_kernel)
     if (warp < NTW) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegTok));
     else asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegRes));
@@ -667,6 +673,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     const int kw = kres_index(warp);
     cluster_wait();    // B0
     cluster_arrive();  // B1
+    pdl_wait_prev();  // the query may come from the preceding launch
     // ---- the rotated query (off the token warps' way to the anchor scores) ----
     // row g (warp g % NKR): signs, 128-point Walsh-Hadamard transform in registers, scale ->
     // q' (Appendix A.1, Eq. 12) into qp, its sum into sq
@@ -938,6 +945,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     zrow[tid] = 0.f;
     ninfrow[tid] = -INFINITY;
   }
+  pdl_wait_prev();  // the query and the outputs may be the preceding launch's
   {
     // fragment (k-step ks, lane ln): one per token thread (8 k-steps x 32 lanes); q in bf16,
     // k order permuted so that a thread's dims are contiguous
@@ -1582,13 +1590,16 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   cfg.blockDim = dim3(NT, 1, 1);
   cfg.dynamicSmemBytes = pl.smem;
   cfg.stream = (cudaStream_t)stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = pl.C;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  // the launch may overlap the tail of a preceding decode launch (griddepcontrol in the kernel)
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   cudaError_t e = cudaLaunchKernelEx(&cfg, decode_kernel<GS>(), P);
   if (e != cudaSuccess) return (int)e;
   return (int)cudaGetLastError();
