@@ -319,11 +319,10 @@ akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_len
  * Errors: AKV_ERR_INVALID (null/misaligned pointers, bad sizes),
  * AKV_ERR_UNSUPPORTED (k * G beyond the shared-memory tables of this build),
  * AKV_ERR_CUDA (launch failure).
- * Ordering: the launch is a programmatic dependent launch.  When the preceding work
- * in the stream is another akv_decode_attn launch, this one may start streaming its
- * arena before that launch ends (a decode launch never writes an arena); it reads q
- * and writes out/out_f32 only after the preceding launch has completed.  After any
- * other kind of preceding work it starts in ordinary stream order.
+ * Ordering: the launch is a programmatic dependent launch: it may be scheduled and set
+ * up its on-chip state while a preceding akv_decode_attn launch in the same stream
+ * drains, but it reads the arena and q, and writes out/out_f32, only after all
+ * preceding work in the stream has completed (ordinary stream semantics for data).
  */
 akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,
                            size_t arena_bytes, const void* q, void* out, float* out_f32, float sm_scale,

@@ -64,13 +64,7 @@ constexpr int NVR = 4;                 // value-residual warps: 8, 9, 12, 13
 constexpr int W_PROD = 14;             // producer warp
 constexpr int NT = 16 * 32;            // 512 threads: four warpgroups
 // A warp issues on sub-partition (warp % 4): each sub-partition carries two token warps and
-// two of the others.  In the reallocating kernel, warpgroups 0-1 (the token warps) raise
-// their register budget and warpgroups 2-3 lower theirs (setmaxnreg): 256 x kRegTok +
-// 256 x kRegRes equals 512 x 128, the launch's own total when the kernel was compiled to 128
-// registers a thread; the host launches it only then, so the raise never waits for registers
-// the block does not hold.
-constexpr int kRegTok = 152, kRegRes = 104;
-static_assert(2 * 128 * kRegTok + 2 * 128 * kRegRes == NT * 128, "register split must equal the launch total");
+// two of the others.
 __device__ __forceinline__ int kres_index(int warp) { return warp == 10 ? 0 : warp == 11 ? 1 : warp == 15 ? 2 : -1; }
 __device__ __forceinline__ int vres_index(int warp) {
   return warp == 8 ? 0 : warp == 9 ? 1 : warp == 12 ? 2 : warp == 13 ? 3 : -1;
@@ -177,9 +171,9 @@ __device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sy
 __device__ __forceinline__ void named_arrive(int id, int n) {
   asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
-// Programmatic dependent launch: the next launch in the stream may start its prologue (it
-// only streams the cache, which no decode launch writes) while this one runs; a thread waits
-// for the preceding launch to complete before it reads the query or writes an output.
+// Programmatic dependent launch: the next launch in the stream may be scheduled, and set up
+// its shared memory and barriers, while this one runs; before it reads the cache
+// or the query, or writes an output, every thread waits for the preceding work to complete.
 __device__ __forceinline__ void pdl_allow_next() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 __device__ __forceinline__ void pdl_wait_prev() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
@@ -486,7 +480,7 @@ __device__ __forceinline__ void load_row(const float* p, float (&out)[GS]) {
   }
 }
 
-template <int GS, bool RA>
+template <int GS>
 __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P) {
   extern __shared__ __align__(128) uint8_t smem[];
   cg::cluster_group cluster = cg::this_cluster();
@@ -496,9 +490,6 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   const int u = vu / P.nhg, hg = vu % P.nhg;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c4 = lane & 3, r8 = lane >> 2;
-  const UnitView U = unit_view(P.arena, u);
-  const int k = U.k;
-
   float* SA = reinterpret_cast<float*>(smem + P.o_sa);  // [k][GS] anchor scores (log2 units)
   float* Wt = reinterpret_cast<float*>(smem + P.o_w);   // [kc][GS] value weights of owned anchors
   uint2* qfa = reinterpret_cast<uint2*>(smem + P.o_qfa);
@@ -537,6 +528,26 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   auto bar_p = [&](int s) { return smem_u32(bars + 4 * NS + s); };
   auto stage = [&](int s) { return ring + (size_t)s * P.stage_bytes; };
 
+
+  if (tid == 0) {
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(bar_full_c(s), 1);  // the producer's expect_tx arrival; bytes complete the phase
+      mbar_init(bar_full_t(s), 1);
+      mbar_init(bar_empty(s), NTW + NVR);
+      mbar_init(bar_rs(s), NKR);
+      mbar_init(bar_p(s), NTW);
+    }
+    *failed = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  pdl_allow_next();
+  // Everything above touches only this CTA's shared memory; from here on the launch reads
+  // the cache and the query, and writes outputs: first the preceding work must be complete.
+  pdl_wait_prev();
+  const UnitView U = unit_view(P.arena, u);
+  const int k = U.k;
+
   // this CTA's anchors (it owns their value weights) and tile blocks
   // ceil(k / C) anchors each: their runs lie in about the tiles this CTA reads, so most value
   // weights are reduced locally
@@ -570,24 +581,6 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     }
   };
   const TileCursor cursor0{n_ka % NS, 0, NS, 0u};
-
-  if (tid == 0) {
-    for (int s = 0; s < NS; ++s) {
-      mbar_init(bar_full_c(s), 1);  // the producer's expect_tx arrival; bytes complete the phase
-      mbar_init(bar_full_t(s), 1);
-      mbar_init(bar_empty(s), NTW + NVR);
-      mbar_init(bar_rs(s), NKR);
-      mbar_init(bar_p(s), NTW);
-    }
-    *failed = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  __syncthreads();
-  pdl_allow_next();
-  if constexpr (RA) {  // launched only when its register count is exactly 128 (decode_kernel)
-    if (warp < NTW) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegTok));
-    else asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegRes));
-  }
   // B0: every CTA of the cluster has started (its shared memory may take remote stores)
   cluster_arrive();
   // first element of this CTA's query (and output) rows, computed where used
@@ -673,7 +666,6 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     const int kw = kres_index(warp);
     cluster_wait();    // B0
     cluster_arrive();  // B1
-    pdl_wait_prev();  // the query may come from the preceding launch
     // ---- the rotated query (off the token warps' way to the anchor scores) ----
     // row g (warp g % NKR): signs, 128-point Walsh-Hadamard transform in registers, scale ->
     // q' (Appendix A.1, Eq. 12) into qp, its sum into sq
@@ -945,7 +937,6 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     zrow[tid] = 0.f;
     ninfrow[tid] = -INFINITY;
   }
-  pdl_wait_prev();  // the query and the outputs may be the preceding launch's
   {
     // fragment (k-step ks, lane ln): one per token thread (8 k-steps x 32 lanes); q in bf16,
     // k order permuted so that a thread's dims are contiguous
@@ -1486,20 +1477,9 @@ struct LaunchKey {
 };
 
 using KernelFn = void (*)(const DecodeParams);
-// The kernel for GS heads per CTA: for GS = 4 the register-reallocating one when its launch
-// register count is the 128 the split assumes (checked once), else the plain one.
 template <int GS>
 KernelFn decode_kernel() {
-  if constexpr (GS == 4) {
-    static const bool ra = [] {
-      cudaFuncAttributes a{};
-      return cudaFuncGetAttributes(&a, akv_decode_kernel<4, true>) == cudaSuccess && a.numRegs == 128;
-    }();
-    cudaGetLastError();
-    return ra ? akv_decode_kernel<4, true> : akv_decode_kernel<4, false>;
-  } else {
-    return akv_decode_kernel<GS, false>;
-  }
+  return akv_decode_kernel<GS>;
 }
 
 template <int GS>
