@@ -238,13 +238,16 @@ __device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t& r0, uint3
                : "r"(addr));
 }
 
-// Two 2-bit codes c, at bits 0-1 and 16-17 of x, as the fp16 pair 1024 + c: OR them into
-// the mantissa of 1024.0 (0x6400, unit spacing), one logic op.  A product with these
-// operands carries 1024 x (sum of the other operand), taken off once per head.
-__device__ __forceinline__ uint32_t codes2_to_h1024(uint32_t x) {
-  uint32_t t;
+// Two 2-bit codes, at bits 0-1 and 16-17 of x, as an fp16 pair of exact small integers: OR
+// them into the mantissa of 1024.0 (0x6400, unit spacing), then subtract 1024.  (Leaving the
+// 1024 in and taking 1024 x sum(q') off afterwards saves the subtraction but costs the
+// tensor-core sums about two decimal digits: they do not hold full fp32 precision against an
+// offset that large.)
+__device__ __forceinline__ uint32_t codes2_to_h2(uint32_t x) {
+  uint32_t t, r;
   asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(t) : "r"(x), "r"(0x00030003u), "r"(0x64006400u));
-  return t;
+  asm("sub.f16x2 %0, %1, %2;" : "=r"(r) : "r"(t), "r"(0x64006400u));
+  return r;
 }
 // Two 2-bit codes as the exact bf16 pair c: OR into the mantissa of 128.0 (0x4300, unit
 // spacing), then t * 1 - 128.  (The value-residual sum runs over many more products than a
@@ -503,8 +506,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float* cl = mref + GS;                                  // [GS]
   float* pms = cl + GS;                                   // [GS]
   float* ltot = pms + GS;                                 // [GS]
-  float* kofs = ltot + GS;  // [GS] 1024 x sum of q' (high + low fp16 parts): the key codes' offset
-  volatile int* failed = reinterpret_cast<volatile int*>(kofs + GS);
+  volatile int* failed = reinterpret_cast<volatile int*>(ltot + GS);
   // 16-byte rows: zeros (no key residual) and -inf (a token past the tile's end)
   float* zrow = reinterpret_cast<float*>(smem + P.o_misc + (((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15));
   float* ninfrow = zrow + 4;
@@ -669,7 +671,6 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     // ---- the rotated query (off the token warps' way to the anchor scores) ----
     // row g (warp g % NKR): signs, 128-point Walsh-Hadamard transform in registers, scale ->
     // q' (Appendix A.1, Eq. 12) into qp, its sum into sq
-    if (kw == 0 && lane < GS) kofs[lane] = 0.f;
     const float f = P.rotate ? P.scale_log2 * (1.0f / 128.0f) : P.scale_log2;
     for (int g = kw; g < GS; g += NKR) {
       const uint2 raw = *reinterpret_cast<const uint2*>(P.q + qrow_base() + (size_t)g * 128 + 4 * lane);
@@ -690,10 +691,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     named_sync(5, NKR * 32);
     // key-residual B fragments (k-step ks, lane): column c = lane / 4 is head c % 4 as the fp16
     // high part (c < 4) or low part; k pairs (2t, 2t+1) <-> dims (16ks + 2t, 16ks + 2t + 8),
-    // (2t+8, 2t+9) <-> (16ks + 2t + 1, 16ks + 2t + 9), t = lane % 4.  kofs sums them (x 1024).
+    // (2t+8, 2t+9) <-> (16ks + 2t + 1, 16ks + 2t + 9), t = lane % 4.
     {
       const int g = lane >> 2, c = lane & 3;
-      float part_sum = 0.f;
       for (int ks = kw; ks < 8; ks += NKR) {
         uint2 fk = make_uint2(0u, 0u);
         if ((g & 3) < GS) {
@@ -705,11 +705,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
           const __half h0 = part(x[0]), h8 = part(x[8]), h1 = part(x[1]), h9 = part(x[9]);
           fk.x = pack_h2(h0, h8);
           fk.y = pack_h2(h1, h9);
-          part_sum += (__half2float(h0) + __half2float(h8)) + (__half2float(h1) + __half2float(h9));
         }
         qfk[ks * 32 + lane] = fk;
       }
-      if ((g & 3) < GS) red_local(&kofs[g & 3], 1024.f * part_sum);
     }
     named_sync(5, NKR * 32);
     named_arrive(2, NTW * 32 + NKR * 32);  // the token warps may use qp and sq
@@ -757,7 +755,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
               for (int q = 0; q < 2; ++q) {
                 const uint32_t xa = wd[q][0][ks] >> (4 * c4), xb = wd[q][1][ks] >> (4 * c4);
-                const uint4 a = make_uint4(codes2_to_h1024(xa), codes2_to_h1024(xb), codes2_to_h1024(xa >> 2), codes2_to_h1024(xb >> 2));
+                const uint4 a = make_uint4(codes2_to_h2(xa), codes2_to_h2(xb), codes2_to_h2(xa >> 2), codes2_to_h2(xb >> 2));
                 mma_f16(d[q][ks & 1], a, bf[ks].x, bf[ks].y);
               }
             // columns 2c, 2c+1: high parts of heads 2c, 2c+1 (c < 2) or low parts (c >= 2)
@@ -778,7 +776,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
                     for (int e = 0; e < 2; ++e) {
                       const int g = 2 * c4 + e;
-                      if (g < GS) rs[sl * GS + g] = half_hi(smn) * sq[g] + half_lo(smn) * (v[2 * hr + e] - kofs[g]);
+                      if (g < GS) rs[sl * GS + g] = half_hi(smn) * sq[g] + half_lo(smn) * v[2 * hr + e];
                     }
                   }
                 }

@@ -73,22 +73,25 @@ def test_many_units_cluster_sizes(dev, monkeypatch):
         _run_seeded(dev, p, [8192, 3000, 6001, 700], qseed=int(c))
 
 
-def test_tiny_encoded_config(dev):
-    """configs[0]-shaped case: S=4096, one KV head, G=1, encoded on the GPU."""
+@pytest.mark.parametrize("H,G", [(1, 1), (2, 4)])
+def test_tiny_encoded_config(dev, H, G):
+    """configs[0]-shaped case (S=4096, one KV head, G=1) and a 2-head G=4 variant, encoded on
+    the GPU: clustered keys and values with real residual structure, where the key-residual
+    products need every bit of their fp32 accumulation at sm_scale = 1."""
     S = 4096
-    p = akv.Params(batch=1, n_kv_heads=1, n_q_heads=1, seed=7, rot_seed=11)
-    K, V = gen.clustered_batch(1, 1, [S], seed=42)
+    p = akv.Params(batch=1, n_kv_heads=H, n_q_heads=H * G, seed=7, rot_seed=11)
+    K, V = gen.clustered_batch(1, H, [S], seed=42)
     a_bytes, w_bytes = akv.akv_cache_size(p, [S])
     arena = torch.empty(a_bytes, dtype=torch.uint8, device=dev)
     ws = torch.empty(w_bytes, dtype=torch.uint8, device=dev)
     akv.akv_encode(p, [S], to_dev_u16(K, torch, dev), to_dev_u16(V, torch, dev), arena, ws)
     units = oracle.unpack_arena(arena.cpu().numpy())
-    for t in range(4):
+    for qseed in (1, 100, 101, 102, 103):
         for sm in (1.0, 1 / math.sqrt(128)):
-            q = gen.queries(1, seed=100 + t)
+            q = gen.queries(H * G, seed=qseed)
             out, out32 = decode_on_gpu(torch, p, [S], arena, q, sm)
             ref = oracle_decode(p, units, q, sm)
-            check_outputs(out, out32, ref, "tiny")
+            check_outputs(out, out32, ref, f"tiny H={H} G={G} q={qseed} sm={sm:.3f}")
 
 
 def test_8b_32k_encoded(dev):
@@ -132,3 +135,41 @@ def test_locally_dense_residuals_exceed_staging(dev):
     for G in (1, 4, 8):
         p = akv.Params(batch=2, n_kv_heads=2, n_q_heads=2 * G, seed=31)
         _run_seeded(dev, p, [6000, 3000], mutate=mutate)
+
+
+def test_back_to_back_launches_follow_stream_order(dev):
+    """Consecutive decode launches in one stream overlap their set-up (programmatic dependent
+    launch) but not their data: a launch whose query is the previous launch's output, and a
+    launch that overwrites a buffer an earlier one read, both see stream order."""
+    p = akv.Params(batch=2, n_kv_heads=2, n_q_heads=8, seed=3, rot_seed=77)
+    lens = [6001, 3000]
+    ua = seeded_units(p, lens, seed=5)
+    ub = seeded_units(p, lens, seed=6)
+    arena_a = torch.from_numpy(akv.akv_cache_pack_host(p, lens, [akv.unit_host_from_logical(u) for u in ua])).to(dev)
+    arena_b = torch.from_numpy(akv.akv_cache_pack_host(p, lens, [akv.unit_host_from_logical(u) for u in ub])).to(dev)
+    q0 = gen.queries(p.batch * p.n_q_heads, seed=17)
+    shape = (p.batch, p.n_q_heads, 128)
+    q0_dev = to_dev_u16(q0.reshape(shape), torch, dev)
+    x = torch.empty(shape, dtype=torch.bfloat16, device=dev)
+    y = torch.empty_like(x)
+    z = torch.empty_like(x)
+    y32 = torch.empty(shape, dtype=torch.float32, device=dev)
+    z32 = torch.empty_like(y32)
+    x32 = torch.empty_like(y32)
+    akv.akv_decode_attn(p, lens, arena_a, q0_dev, x)            # x = attn(A, q0)
+    akv.akv_decode_attn(p, lens, arena_b, x, y, y32)            # reads x as its query
+    akv.akv_decode_attn(p, lens, arena_a, y, z, z32)            # reads y as its query
+    akv.akv_decode_attn(p, lens, arena_b, q0_dev, x, x32)       # overwrites x after y's launch read it
+    torch.cuda.synchronize()
+    oa = [oracle_unit(u) for u in ua]
+    ob = [oracle_unit(u) for u in ub]
+    # z from the y this chain produced (exact input), and the final x from q0
+    y_bits = y.view(torch.int16).cpu().numpy().astype(np.uint16).reshape(-1, 128)
+    check_outputs(z.float().cpu().numpy(), z32.cpu().numpy(), oracle_decode(p, oa, y_bits, 1.0), where="z = attn(A, y)")
+    check_outputs(x.float().cpu().numpy(), x32.cpu().numpy(), oracle_decode(p, ob, q0, 1.0), where="x = attn(B, q0)")
+    # y from the bf16 rounding of the oracle's attn(A, q0): a launch that read x before the first
+    # one finished would be far off; a last-place difference in x moves y well within 5e-3
+    x1 = gen.bf16_bits(oracle_decode(p, oa, q0, 1.0)).reshape(-1, 128)
+    y_ref = oracle_decode(p, ob, x1, 1.0)
+    assert np.all(np.isfinite(y32.cpu().numpy()))
+    assert np.abs(y32.cpu().numpy().astype(np.float64) - y_ref).max() <= 5e-3
