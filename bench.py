@@ -36,6 +36,25 @@ WORKLOADS = {
     "8b-128k": (4, 8, 32, 131072, "seeded"),
     "70b-128k": (8, 8, 64, 131072, "seeded"),
 }
+# Budget and ragged-batch sweep at the 8B shape: 16 requests, contexts uniform in [8192, 131072]
+# (one fixed draw), anchor fraction a % and residual-slot fraction r % per side.
+SWEEP_BATCH = 16
+SWEEP_POINTS = {f"sweep-a{a}-r{r}": (a / 100.0, r / 100.0) for a in (1, 2, 4) for r in (0, 5, 10, 20)}
+for _name in SWEEP_POINTS:
+    WORKLOADS[_name] = (SWEEP_BATCH, 8, 32, 0, "seeded")
+
+
+def workload_lens(name: str, B: int, S: int) -> list:
+    """Context length per request: S for the fixed workloads, the ragged draw for the sweep."""
+    if name in SWEEP_POINTS:
+        return [int(x) for x in np.random.default_rng(15).integers(8192, 131073, size=B)]
+    return [S] * B
+
+
+def workload_params(akv, name: str, **kw):
+    """akv.Params of a workload (the sweep points set their budgets)."""
+    fa, fr = SWEEP_POINTS.get(name, (0.02, 0.10))
+    return akv.Params(anchor_frac=fa, res_frac_k=fr, res_frac_v=fr, **kw)
 N_LAYERS = 32
 N_TOKENS = 64
 DEC_KERNEL_SRC = os.path.join(ROOT, "paper_2608_02901_gb300", "csrc", "akv_decode.cu")
@@ -174,10 +193,17 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def kernel_traffic():
-    """DRAM bytes per decode launch from the committed ncu summary, if it matches the current kernel source."""
+TRAFFIC_PROFILES = {"8b-32k": "akv_decode_8b32k_ncu.md", "8b-128k": "akv_decode_8b128k_ncu.md"}
+
+
+def kernel_traffic(workload: str):
+    """DRAM bytes per decode launch from the committed ncu summary of this workload, if there is one
+    and it matches the current kernel source (the 8B-128K capture runs 2 of the 8 cycled layers,
+    same per-launch bytes)."""
     src_hash = hashlib.sha256(open(DEC_KERNEL_SRC, "rb").read()).hexdigest()[:16]
-    path = os.path.join(ROOT, "profiles", "akv_decode_8b32k_ncu.md")
+    if workload not in TRAFFIC_PROFILES:
+        return None
+    path = os.path.join(ROOT, "profiles", TRAFFIC_PROFILES[workload])
     if not os.path.exists(path):
         return None
     vals = {}
@@ -235,8 +261,9 @@ def run_akv(args, rank, world, local):
 
     dev = torch.device("cuda", local)
     B, H, Hq, S, source = WORKLOADS[args.workload]
-    lens = [S] * B
-    p = akv.Params(batch=B, n_kv_heads=H, n_q_heads=Hq, seed=rank_seed(11, rank), rot_seed=0x5EED)
+    lens = workload_lens(args.workload, B, S)
+    p = workload_params(akv, args.workload, batch=B, n_kv_heads=H, n_q_heads=Hq, seed=rank_seed(11, rank),
+                        rot_seed=0x5EED)
     layers = args.layers
     arenas, arena_bytes, step_bytes = build_layers(torch, akv, gen, p, lens, layers, source, dev, rank)
     n_tok = N_TOKENS
@@ -330,7 +357,7 @@ def run_akv(args, rank, world, local):
     peak = float(peaks.get("hbm_gbs", 6800.0))
     achieved = step_bytes / (sec / args.steps) / 1e9  # per launch: one decode kernel per step
     roofline = {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak, "unit": "GB/s",
-                "frac": round(achieved / peak, 4), "traffic": kernel_traffic(),
+                "frac": round(achieved / peak, 4), "traffic": kernel_traffic(args.workload),
                 "peak_source": "measured" if "hbm_gbs" in peaks else "fallback",
                 "bytes_per_launch": round(step_bytes), "frac_of_8tbs": round(achieved / 8000.0, 4)}
 
@@ -343,7 +370,8 @@ def run_akv(args, rank, world, local):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 6),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded clustered K/V, encoded on GPU)" if source == "encoded" else "synthetic (seeded cache)",
-        "config": {"workload": args.workload, "batch": B, "n_kv_heads": H, "n_q_heads": Hq, "context": S,
+        "config": {"workload": args.workload, "batch": B, "n_kv_heads": H, "n_q_heads": Hq,
+                   "context": S if args.workload not in SWEEP_POINTS else f"ragged U[8192, 131072]: {lens}",
                    "anchor_frac": p.anchor_frac, "res_frac": p.res_frac_k, "layers_cycled": layers,
                    "fresh_queries": N_TOKENS, "arena_bytes_per_layer": arena_bytes,
                    "l2": f"inputs larger than L2: {layers} distinct layer caches, {layers * arena_bytes / 1e6:.0f} MB cycled",
@@ -389,8 +417,9 @@ def run_reference(args, rank, world, local):
     import oracle
     import paper_2608_02901_gb300 as akv_params_only  # Params/shape helpers are pure host code
     B, H, Hq, S, source = WORKLOADS[args.workload]
+    S = max(workload_lens(args.workload, B, S))  # the longest request of a ragged batch
     G = Hq // H
-    p = akv_params_only.Params(batch=1, n_kv_heads=1, n_q_heads=G, seed=11, rot_seed=0x5EED)
+    p = workload_params(akv_params_only, args.workload, batch=1, n_kv_heads=1, n_q_heads=G, seed=11, rot_seed=0x5EED)
     # one (request, KV head) unit of the workload; each step attends one query group over a prefix of it
     k, nk, nv = oracle.unit_shape(S, p.anchor_frac, p.res_frac_k, p.res_frac_v, p.window)
     if source == "encoded":

@@ -45,6 +45,8 @@
 #include <cstdlib>
 #include <map>
 #include <mutex>
+#include <queue>
+#include <vector>
 #include <string>
 #include <tuple>
 #include <type_traits>
@@ -1449,17 +1451,42 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   return true;
 }
 
-bool make_plan(const Layout& L, int GS, int C, int smem_optin, Plan* out, std::string* why) {
-  // records staged per tile and side: 1.35x the densest unit's mean plus slack, at most 320;
-  // records of a denser tile beyond these are read from global memory by the token warps.
-  // Fewer if the ring would hold less than two stages.
-  int R = (int)(T * max_density(L) * 1.35) + 32;
-  R = std::min(320, std::max(16, (R + 15) & ~15));
-  for (; R >= 16; R -= 16)
+// Records staged per tile and side: 1.35x the densest unit's mean plus slack, at most 320;
+// records of a denser tile beyond these take the CUDA-core paths, which cost far more.
+int full_r(const Layout& L) {
+  const int R = (int)(T * max_density(L) * 1.35) + 32;
+  return std::min(320, std::max(16, (R + 15) & ~15));
+}
+
+// full_only: only the full staged count; else fewer records when the ring would otherwise hold
+// less than two stages (the last resort: most records then take the CUDA-core paths).
+bool make_plan(const Layout& L, int GS, int C, int smem_optin, Plan* out, std::string* why, bool full_only = false) {
+  for (int R = full_r(L); R >= (full_only ? full_r(L) : 16); R -= 16)
     if (make_plan_r(L, GS, C, R, smem_optin, out)) return true;
   *why = "shared memory: anchor tables of k = " + std::to_string(L.max_k) + " with " + std::to_string(GS) +
          " query heads per CTA leave room for fewer than 2 pipeline stages";
   return false;
+}
+
+// Estimated makespan, in tile times, of a launch with clusters of C CTAs of which nc can be
+// resident at once: clusters start in launch order (unit-major, then head group) on the first
+// free slot, and a cluster lasts as long as its CTA with the most tiles, plus a fixed cost
+// (query preparation, cluster barriers, combine: about six tiles) and its anchor chunks.
+double estimate_makespan(const Layout& L, int nhg, int C, int nc) {
+  constexpr double kFixed = 6.0, kPerChunk = 0.3;
+  std::priority_queue<double, std::vector<double>, std::greater<double>> slots;
+  for (int i = 0; i < nc; ++i) slots.push(0.0);
+  double end = 0.0;
+  for (const auto& s : L.shape) {
+    const double cost = (double)((s.nt + C - 1) / C) + kFixed + kPerChunk * (double)(((s.k + C - 1) / C + CH - 1) / CH);
+    for (int g = 0; g < nhg; ++g) {
+      const double t = slots.top() + cost;
+      slots.pop();
+      slots.push(t);
+      end = std::max(end, t);
+    }
+  }
+  return end;
 }
 
 // Launch configuration per (device, G, units, lengths, density, cluster override):
@@ -1503,13 +1530,13 @@ int plan_for(const Layout& L, const LaunchKey& key, int vunits, Plan* out, std::
   // Cluster size: the most CTAs per unit such that every cluster is resident at once (one CTA
   // per SM), no more CTAs than tiles in the longest unit.  Sizes are tried downwards one by
   // one: a GPU whose processor clusters cannot hold 16 CTAs each may still hold 12 or 13.
-  int C = std::min<long long>(kMaxCluster, std::max<long long>(1, di.sms / std::max(1, vunits)));
-  C = std::max(1, std::min(C, L.max_tiles));
-  if (key.cluster_env >= 1 && key.cluster_env <= kMaxCluster) C = key.cluster_env;
-  Plan pl;
-  for (;;) {
-    if (!make_plan(L, GS, C, di.smem_optin, &pl, why)) return -1;
-    if (C == 1) break;
+  // A size whose tables leave room for the full staged count comes first: the value-weight table
+  // shrinks with C (ceil(k / C) anchors), so when it is too large at every all-resident size a
+  // larger C is taken even if its clusters run in more than one wave; only when no size fits is
+  // the staged count cut.
+  const int C0 = std::max(1, std::min<int>(std::min<long long>(kMaxCluster, std::max<long long>(1, di.sms / std::max(1, vunits))),
+                                           L.max_tiles));
+  auto clusters_fit = [&](int C, const Plan& pl) -> int {  // clusters resident at once (C > 1)
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(C * vunits), 1, 1);
     cfg.blockDim = dim3(NT, 1, 1);
@@ -1522,11 +1549,40 @@ int plan_for(const Layout& L, const LaunchKey& key, int vunits, Plan* out, std::
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int nclusters = 0;
-    e = cudaOccupancyMaxActiveClusters(&nclusters, kfn, &cfg);
-    // prefer a size whose clusters all fit at once; an explicit override only needs one to fit
-    if (e == cudaSuccess && (nclusters >= vunits || (key.cluster_env == C && nclusters >= 1))) break;
-    cudaGetLastError();
-    C -= 1;
+    if (cudaOccupancyMaxActiveClusters(&nclusters, kfn, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      return 0;
+    }
+    return nclusters;
+  };
+  Plan pl;
+  int C = 0;
+  if (key.cluster_env >= 1 && key.cluster_env <= kMaxCluster) {  // requested size, or the next that fits once
+    for (int c = key.cluster_env; c >= 1 && !C; --c)
+      if (make_plan(L, GS, c, di.smem_optin, &pl, why) && (c == 1 || clusters_fit(c, pl) >= 1)) C = c;
+    if (!C) return -1;
+  } else {
+    // 1. among the sizes whose tables leave room for the full staged count, the one with the
+    //    shortest estimated makespan (estimate_makespan; resident clusters from the occupancy
+    //    query, so sizes whose clusters cannot all be resident pay for their extra waves)
+    double best = 0.0;
+    for (int c = std::min(kMaxCluster, std::max(1, L.max_tiles)); c >= 1; --c) {
+      Plan cand;
+      std::string w;
+      if (!make_plan(L, GS, c, di.smem_optin, &cand, &w, true)) continue;
+      const int nc = c == 1 ? di.sms : clusters_fit(c, cand);
+      if (nc < 1) continue;
+      const double t = estimate_makespan(L, vunits / (int)L.shape.size(), c, nc);
+      if (!C || t < best * 0.97) {  // near-ties keep the larger size: the anchor work spreads wider
+        C = c;
+        best = t;
+        pl = cand;
+      }
+    }
+    // 2. else a cut staged count at the largest all-resident size
+    for (int c = C0; c >= 1 && !C; --c)
+      if (make_plan(L, GS, c, di.smem_optin, &pl, why) && (c == 1 || clusters_fit(c, pl) >= vunits)) C = c;
+    if (!C) return -1;
   }
   std::lock_guard<std::mutex> lk(mu);
   cache[key] = pl;
