@@ -235,13 +235,32 @@ def akv_decode_workspace_size(p: Params, ctx_lens) -> int:
     return w.value
 
 
+# The marshalled (params, lengths) of recent decode calls: a decode loop repeats them, and
+# building the ctypes structures dominates the binding's share of a call.
+_DECODE_ARGS: dict = {}
+
+
+def _decode_args(p: Params, ctx_lens):
+    key = (p.batch, p.n_kv_heads, p.n_q_heads, p.head_dim, p.anchor_frac, p.res_frac_k, p.res_frac_v, p.window,
+           p.seed, p.rot_seed, p.rotate, tuple(int(x) for x in ctx_lens))
+    ent = _DECODE_ARGS.get(key)
+    if ent is None:
+        if len(_DECODE_ARGS) >= 64:
+            _DECODE_ARGS.clear()
+        pc = p.c()
+        lens = _lens(ctx_lens)
+        ent = (pc, lens, ctypes.byref(pc), _i32p(lens))
+        _DECODE_ARGS[key] = ent
+    return ent[2], ent[3]
+
+
 def akv_decode_attn(p: Params, ctx_lens, arena, q, out, out_f32=None, sm_scale: float = 1.0, ws=None, stream=None):
     """q, out: CUDA bf16 [B][H_q][128]; out_f32 optional fp32 of the same shape."""
-    lens = _lens(ctx_lens)
+    pref, lref = _decode_args(p, ctx_lens)
     ws_bytes = 0 if ws is None else ws.numel() * ws.element_size()
-    _check(lib().akv_decode_attn(ctypes.byref(p.c()), _i32p(lens), _dev_ptr(arena),
-                                 arena.numel() * arena.element_size(), _dev_ptr(q), _dev_ptr(out),
-                                 _dev_ptr(out_f32), float(sm_scale), _dev_ptr(ws), ws_bytes, _stream_ptr(stream)),
+    _check(lib().akv_decode_attn(pref, lref, _dev_ptr(arena), arena.numel() * arena.element_size(), _dev_ptr(q),
+                                 _dev_ptr(out), _dev_ptr(out_f32), float(sm_scale), _dev_ptr(ws), ws_bytes,
+                                 _stream_ptr(stream)),
            "akv_decode_attn")
 
 
