@@ -180,13 +180,20 @@ __device__ __forceinline__ void pdl_allow_next() { asm volatile("griddepcontrol.
 __device__ __forceinline__ void pdl_wait_prev() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
-// A row of GS floats (16-, 8- or 4-byte aligned) stored into the same place in the shared
+// A row of GS floats (16-byte aligned for GS >= 4, else 8 or 4) stored into the same place in the shared
 // memory of CTA `rank` of the cluster.
 template <int GS>
 __device__ __forceinline__ void st_cluster_row(const float* local, int rank) {
   uint32_t remote;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
-  if constexpr (GS == 4) {
+  if constexpr (GS == 8) {
+    const float4 v = *reinterpret_cast<const float4*>(local), w = *reinterpret_cast<const float4*>(local + 4);
+    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(remote), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+                 : "memory");
+    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(remote + 16u), "f"(w.x), "f"(w.y), "f"(w.z),
+                 "f"(w.w)
+                 : "memory");
+  } else if constexpr (GS == 4) {
     const float4 v = *reinterpret_cast<const float4*>(local);
     asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(remote), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
                  : "memory");
@@ -459,10 +466,13 @@ __device__ __noinline__ void value_record_add(const TileView& tv, int r, float p
   }
 }
 
-// GS probabilities (pairs) as one row of GS floats (16-, 8- or 4-byte aligned).
+// GS probabilities (pairs) as one row of GS floats (16-byte aligned for GS >= 4, else 8 or 4).
 template <int GS, int NP>
 __device__ __forceinline__ void store_row(float* p, const float2 (&v)[NP]) {
-  if constexpr (GS == 4) {
+  if constexpr (GS == 8) {
+    *reinterpret_cast<float4*>(p) = make_float4(v[0].x, v[0].y, v[1].x, v[1].y);
+    *reinterpret_cast<float4*>(p + 4) = make_float4(v[2].x, v[2].y, v[3].x, v[3].y);
+  } else if constexpr (GS == 4) {
     *reinterpret_cast<float4*>(p) = make_float4(v[0].x, v[0].y, v[1].x, v[1].y);
   } else if constexpr (GS == 2) {
     *reinterpret_cast<float2*>(p) = v[0];
@@ -471,10 +481,14 @@ __device__ __forceinline__ void store_row(float* p, const float2 (&v)[NP]) {
   }
 }
 
-// A row of GS consecutive floats (16-, 8- or 4-byte aligned) into registers.
+// A row of GS consecutive floats (16-byte aligned for GS >= 4, else 8 or 4) into registers.
 template <int GS>
 __device__ __forceinline__ void load_row(const float* p, float (&out)[GS]) {
-  if constexpr (GS == 4) {
+  if constexpr (GS == 8) {
+    const float4 v = *reinterpret_cast<const float4*>(p), w = *reinterpret_cast<const float4*>(p + 4);
+    out[0] = v.x; out[1] = v.y; out[2] = v.z; out[3] = v.w;
+    out[4] = w.x; out[5] = w.y; out[6] = w.z; out[7] = w.w;
+  } else if constexpr (GS == 4) {
     const float4 v = *reinterpret_cast<const float4*>(p);
     out[0] = v.x; out[1] = v.y; out[2] = v.z; out[3] = v.w;
   } else if constexpr (GS == 2) {
@@ -509,9 +523,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float* pms = cl + GS;                                   // [GS]
   float* ltot = pms + GS;                                 // [GS]
   volatile int* failed = reinterpret_cast<volatile int*>(ltot + GS);
-  // 16-byte rows: zeros (no key residual) and -inf (a token past the tile's end)
+  // rows of max(GS, 4) floats: zeros (no key residual) and -inf (a token past the tile's end)
   float* zrow = reinterpret_cast<float*>(smem + P.o_misc + (((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15));
-  float* ninfrow = zrow + 4;
+  float* ninfrow = zrow + (GS > 4 ? GS : 4);
   uint2* meta = reinterpret_cast<uint2*>(smem + P.o_meta);  // [NS] tile block offset, bytes
   float* mslot = reinterpret_cast<float*>(smem + P.o_mslot);
   uint4* hdrs = reinterpret_cast<uint4*>(smem + P.o_hdr);  // [NS][2]
@@ -692,30 +706,38 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     }
     named_sync(5, NKR * 32);
     // key-residual B fragments (k-step ks, lane): column c = lane / 4 is head c % 4 as the fp16
-    // high part (c < 4) or low part; k pairs (2t, 2t+1) <-> dims (16ks + 2t, 16ks + 2t + 8),
-    // (2t+8, 2t+9) <-> (16ks + 2t + 1, 16ks + 2t + 9), t = lane % 4.
+    // high part (c < 4) or low part -- for GS = 8, set hl (0: high parts, 1: low parts) of
+    // head c; k pairs (2t, 2t+1) <-> dims (16ks + 2t, 16ks + 2t + 8), (2t+8, 2t+9) <->
+    // (16ks + 2t + 1, 16ks + 2t + 9), t = lane % 4.
     {
       const int g = lane >> 2, c = lane & 3;
-      for (int ks = kw; ks < 8; ks += NKR) {
-        uint2 fk = make_uint2(0u, 0u);
-        if ((g & 3) < GS) {
-          const float* x = qp + (g & 3) * 128 + 16 * ks + 2 * c;
-          auto part = [&](float v) {
-            const __half hi = __float2half_rn(v);
-            return g < 4 ? hi : __float2half_rn(v - __half2float(hi));
-          };
-          const __half h0 = part(x[0]), h8 = part(x[8]), h1 = part(x[1]), h9 = part(x[9]);
-          fk.x = pack_h2(h0, h8);
-          fk.y = pack_h2(h1, h9);
+      for (int ks = kw; ks < 8; ks += NKR)
+#pragma unroll
+        for (int hl = 0; hl < (GS == 8 ? 2 : 1); ++hl) {
+          uint2 fk = make_uint2(0u, 0u);
+          const int head = GS == 8 ? g : (g & 3);
+          const bool low = GS == 8 ? hl == 1 : g >= 4;
+          if (head < GS) {
+            const float* x = qp + head * 128 + 16 * ks + 2 * c;
+            auto part = [&](float v) {
+              const __half hi = __float2half_rn(v);
+              return low ? __float2half_rn(v - __half2float(hi)) : hi;
+            };
+            const __half h0 = part(x[0]), h8 = part(x[8]), h1 = part(x[1]), h9 = part(x[9]);
+            fk.x = pack_h2(h0, h8);
+            fk.y = pack_h2(h1, h9);
+          }
+          qfk[hl * 256 + ks * 32 + lane] = fk;
         }
-        qfk[ks * 32 + lane] = fk;
-      }
     }
     named_sync(5, NKR * 32);
     named_arrive(2, NTW * 32 + NKR * 32);  // the token warps may use qp and sq
-    uint2 bf[8];
+    constexpr int NBF = GS == 8 ? 2 : 1;  // fragment sets: GS = 8 keeps high and low parts apart
+    uint2 bf[NBF][8];
 #pragma unroll
-    for (int ks = 0; ks < 8; ++ks) bf[ks] = qfk[ks * 32 + lane];
+    for (int hl = 0; hl < NBF; ++hl)
+#pragma unroll
+      for (int ks = 0; ks < 8; ++ks) bf[hl][ks] = qfk[hl * 256 + ks * 32 + lane];
     bool ok = true;
     TileCursor cur = cursor0;
     for (int tl = 0; tl < n_t; ++tl, cur.next()) {
@@ -751,6 +773,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
                 wd[q][hr][0] = w0.x; wd[q][hr][1] = w0.y; wd[q][hr][2] = w0.z; wd[q][hr][3] = w0.w;
                 wd[q][hr][4] = w1.x; wd[q][hr][5] = w1.y; wd[q][hr][6] = w1.z; wd[q][hr][7] = w1.w;
               }
+            // two independent chains per group: alternate k-steps, or (GS = 8) high and low parts
             float d[2][2][4] = {};
 #pragma unroll
             for (int ks = 0; ks < 8; ++ks)
@@ -758,18 +781,24 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
               for (int q = 0; q < 2; ++q) {
                 const uint32_t xa = wd[q][0][ks] >> (4 * c4), xb = wd[q][1][ks] >> (4 * c4);
                 const uint4 a = make_uint4(codes2_to_h2(xa), codes2_to_h2(xb), codes2_to_h2(xa >> 2), codes2_to_h2(xb >> 2));
-                mma_f16(d[q][ks & 1], a, bf[ks].x, bf[ks].y);
+                if constexpr (GS == 8) {
+                  mma_f16(d[q][0], a, bf[0][ks].x, bf[0][ks].y);
+                  mma_f16(d[q][1], a, bf[NBF - 1][ks].x, bf[NBF - 1][ks].y);
+                } else {
+                  mma_f16(d[q][ks & 1], a, bf[0][ks].x, bf[0][ks].y);
+                }
               }
-            // columns 2c, 2c+1: high parts of heads 2c, 2c+1 (c < 2) or low parts (c >= 2)
+            // columns 2c, 2c+1: heads 2c, 2c+1 (GS = 8: high + low parts of the two chains);
+            // otherwise high parts of heads 2c, 2c+1 (c < 2) or low parts (c >= 2)
 #pragma unroll
             for (int q = 0; q < 2; ++q) {
               float v[4];
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
                 v[e] = d[q][0][e] + d[q][1][e];
-                v[e] += __shfl_xor_sync(0xffffffffu, v[e], 2);
+                if constexpr (GS != 8) v[e] += __shfl_xor_sync(0xffffffffu, v[e], 2);
               }
-              if (c4 < 2) {
+              if (GS == 8 || c4 < 2) {
 #pragma unroll
                 for (int hr = 0; hr < 2; ++hr) {
                   const int sl = (g16 + q * NKR) * 16 + r8 + 8 * hr;
@@ -933,7 +962,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   for (int e = tid; e < kc * GS; e += NTT) Wt[e] = 0.f;  // before B1: peers add into it only after B1
   for (int e = tid; e < ((R + 15) / 16) * 256; e += NTT) reinterpret_cast<uint32_t*>(smem + P.o_pfb)[e] = 0u;
   if (tid < GS) pms[tid] = 0.f;
-  if (tid < 4) {
+  if (tid < (GS > 4 ? GS : 4)) {
     zrow[tid] = 0.f;
     ninfrow[tid] = -INFINITY;
   }
@@ -1418,11 +1447,11 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_sa = take((size_t)L.max_k * GS * 4);
   P.o_w = take((size_t)kc_max * GS * 4);
   P.o_qfa = take(8 * 32 * 8);
-  P.o_qfk = take(8 * 32 * 8);
+  P.o_qfk = take((GS == 8 ? 2 : 1) * 8 * 32 * 8);  // [hi, lo for GS = 8][k-step][lane]
   P.o_qp = take((size_t)GS * 128 * 4);
   P.o_acc = take((size_t)GS * 128 * 4);
   P.o_opart = take((size_t)std::max(GS * 128, NTW * GS) * 4);
-  P.o_misc = take((size_t)(((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15) + 32);
+  P.o_misc = take((size_t)(((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15) + 2 * 4 * std::max(GS, 4));
   P.o_meta = take(8 * 8);
   P.o_hdr = take(8 * 32);
   P.o_mslot = take((size_t)kMaxCluster * GS * 4);
@@ -1643,12 +1672,18 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
 
 int launch_decode(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
                   float sm_scale, void* stream, std::string* why) {
-  // a CTA serves up to 4 query heads of its KV head (group size 8: two CTA groups per unit)
+  // a CTA serves all G query heads of its KV head; for G = 8, when the anchor tables of eight
+  // heads leave no room for the pipeline, two CTA groups of four heads each
   switch (L.G) {
     case 1: return launch_g<1>(L, p, arena, q, out, out_f32, sm_scale, stream, why);
     case 2: return launch_g<2>(L, p, arena, q, out, out_f32, sm_scale, stream, why);
-    case 4:
-    case 8: return launch_g<4>(L, p, arena, q, out, out_f32, sm_scale, stream, why);
+    case 4: return launch_g<4>(L, p, arena, q, out, out_f32, sm_scale, stream, why);
+    case 8: {
+      const int e = launch_g<8>(L, p, arena, q, out, out_f32, sm_scale, stream, why);
+      if (e != -1) return e;
+      why->clear();
+      return launch_g<4>(L, p, arena, q, out, out_f32, sm_scale, stream, why);
+    }
   }
   *why = "unsupported group size";
   return -1;
