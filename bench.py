@@ -69,6 +69,9 @@ def parse():
     ap.add_argument("--workload", default="8b-32k", choices=sorted(WORKLOADS))
     ap.add_argument("--layers", type=int, default=N_LAYERS)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--dense-context", action="store_true",
+                    help="context only: torch scaled-dot-product attention decoding over the dense bf16 K/V of the same "
+                         "shapes (a library kernel, not this repository's path)")
     return ap.parse_args()
 
 
@@ -481,11 +484,69 @@ def _prefix_unit(oracle, u, P):
     return sub
 
 
+def run_dense_context(args, rank, world, local):
+    """Dense bf16 decode attention over the uncompressed K/V of the workload's shapes, timed the way
+    the main line is (CUDA graph, events, inputs larger than L2): the cost the compressed cache is
+    compared against.  Random data: only the time is of interest."""
+    import torch
+    import torch.nn.functional as F
+    if rank != 0:
+        return
+    dev = torch.device("cuda", local)
+    B, H, Hq, S, _ = WORKLOADS[args.workload]
+    lens = workload_lens(args.workload, B, S)
+    Smax = max(lens)
+    per_layer = 2 * B * H * Smax * 128 * 2
+    layers = max(1, min(args.layers, int(math.ceil(400e6 / per_layer))))  # > 3x L2 in total
+    g = torch.Generator(device=dev)
+    g.manual_seed(5)
+    Ks = [torch.randn((B, H, Smax, 128), generator=g, device=dev, dtype=torch.bfloat16) for _ in range(layers)]
+    Vs = [torch.randn((B, H, Smax, 128), generator=g, device=dev, dtype=torch.bfloat16) for _ in range(layers)]
+    q = torch.randn((B, Hq, 1, 128), generator=g, device=dev, dtype=torch.bfloat16) / math.sqrt(128)
+    mask = None
+    if len(set(lens)) > 1:  # ragged batch: positions past a request's length masked out
+        pos = torch.arange(Smax, device=dev)
+        mask = (pos[None, None, None, :] < torch.tensor(lens, device=dev)[:, None, None, None])
+    outs = torch.empty((B, Hq, 1, 128), device=dev, dtype=torch.bfloat16)
+
+    def step(i):
+        outs.copy_(F.scaled_dot_product_attention(q, Ks[i % layers], Vs[i % layers], attn_mask=mask, scale=1.0,
+                                                  enable_gqa=True))
+
+    for i in range(max(3, layers)):
+        step(i)
+    torch.cuda.synchronize()
+    stream = torch.cuda.Stream(device=dev)
+    n = max(layers, 64)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for i in range(n):
+            step(i)
+    graph.replay()
+    torch.cuda.synchronize()
+    reps = max(1, args.steps // n)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record()
+        for _ in range(reps):
+            graph.replay()
+        e1.record()
+    torch.cuda.synchronize()
+    us = e0.elapsed_time(e1) * 1e3 / (reps * n)
+    dense_bytes = sum(2 * H * L * 128 * 2 for L in lens)
+    print(json.dumps({"impl": "dense-sdpa-context", "workload": args.workload, "us_per_step": round(us, 3),
+                      "dense_bytes_per_step": dense_bytes, "GB/s": round(dense_bytes / (us * 1e-6) / 1e9, 1),
+                      "layers_cycled": layers, "note": "torch scaled_dot_product_attention on dense bf16 K/V "
+                      "(library kernel, context only)"}), flush=True)
+
+
 def main():
     args = parse()
     rank, world, local = dist_setup(args)
     try:
-        if args.impl == "reference":
+        if args.dense_context:
+            run_dense_context(args, rank, world, local)
+        elif args.impl == "reference":
             run_reference(args, rank, world, local)
         else:
             run_akv(args, rank, world, local)
