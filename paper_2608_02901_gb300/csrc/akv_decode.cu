@@ -99,6 +99,7 @@ struct DecodeParams {
   int o_lslot;     // [kMaxCluster][GS] each CTA's normaliser share
   int o_fslot;     // [kMaxCluster] each CTA's failure flag
   int o_ofin;      // [C][per] staging: partial output numerators of this CTA's share, per rank
+  int drop_last;   // test hook: the producer withholds its item n_items - drop_last (0: none)
 };
 
 // ---- device helpers ---------------------------------------------------------------
@@ -637,7 +638,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         *failed = 1;
         break;
       }
-      if (lane == 0) {
+      if (lane == 0 && it != n_items - P.drop_last) {  // (drop_last: a test withholds one item)
         const uint32_t dst = smem_u32(stage(s));
         if (!is_tile(it)) {
           const bool val = it >= n_ka + n_t;
@@ -1629,6 +1630,11 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   cudaGetDevice(&dev);
   int cenv = 0;
   if (const char* env = std::getenv("AKV_CLUSTER")) cenv = std::atoi(env);
+  // test hook (failure detection): with AKV_DEBUG_DROP_LAST=1 every CTA withholds the last item
+  // of its stream (its stage is not used again), so the waits on it run out after their bound
+  // and the outputs become NaN
+  int drop = 0;
+  if (const char* env = std::getenv("AKV_DEBUG_DROP_LAST")) drop = std::max(0, std::atoi(env));
   const LaunchKey key{dev, L.G, units, L.max_len, L.max_k, cenv, (long long)(max_density(L) * 1e6)};
   Plan pl;
   int err = plan_for<GS>(L, key, vunits, &pl, why);
@@ -1647,6 +1653,7 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   P.sign_lo = L.header.sign_bits[0];
   P.sign_hi = L.header.sign_bits[1];
   P.cluster = pl.C;
+  P.drop_last = drop;
 
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(pl.C * vunits), 1, 1);

@@ -193,3 +193,24 @@ def test_large_anchor_tables_take_larger_clusters(dev):
     ref = oracle_decode(p, [oracle_unit(u) for u in units], q, 1.0, sel=sel)
     rows = np.repeat(sel.astype(bool), p.G).reshape(p.batch, p.n_q_heads)
     check_outputs(out[rows], out32[rows], ref[rows], where="large anchor tables")
+
+
+def test_withheld_item_times_out_to_nan_and_context_survives(dev, monkeypatch):
+    """Failure detection without a GPU fault: with the test hook every CTA withholds the last
+    item of its stream, so the waits on it run out after their bound (about 2 s).  The call
+    returns, the outputs are NaN, and the next call on the same context is correct."""
+    import time
+    p = akv.Params(batch=1, n_kv_heads=2, n_q_heads=8, seed=3, rot_seed=77)
+    lens = [5000]
+    units = seeded_units(p, lens, seed=5)
+    arena = torch.from_numpy(akv.akv_cache_pack_host(p, lens, [akv.unit_host_from_logical(u) for u in units])).to(dev)
+    q = gen.queries(p.batch * p.n_q_heads, seed=17)
+    monkeypatch.setenv("AKV_DEBUG_DROP_LAST", "1")
+    t0 = time.perf_counter()
+    out, out32 = decode_on_gpu(torch, p, lens, arena, q, 1.0)
+    waited = time.perf_counter() - t0
+    monkeypatch.delenv("AKV_DEBUG_DROP_LAST")
+    assert np.all(np.isnan(out32)) and np.all(np.isnan(out))
+    assert waited > 1.0, waited
+    out, out32 = decode_on_gpu(torch, p, lens, arena, q, 1.0)
+    check_outputs(out, out32, oracle_decode(p, [oracle_unit(u) for u in units], q, 1.0), where="after the timed-out call")
