@@ -1,15 +1,16 @@
 // Split-K decode attention read directly from the AnchorKV compressed cache.
 //
-// One thread-block cluster per (request, KV head, group of up to 4 query heads); its C
-// CTAs split the unit's tile blocks and its anchors.  Eq. 3 is folded into Eq. 4: no key
-// or value row is ever rebuilt in memory.
+// One thread-block cluster per (request, KV head) -- for G = 8, when eight heads' tables do
+// not fit, per (request, KV head, four query heads); its C CTAs split the unit's tile blocks
+// and its anchors.  Eq. 3 is folded into Eq. 4: no key or value row is ever rebuilt in
+// memory.
 //
-// Warp-specialised CTA (15 warps):
+// Warp-specialised CTA (16 warps):
 //   producer warp     one elected lane streams a sequence of items through a ring of
 //                     shared-memory stages, one bulk asynchronous copy per item, each
 //                     completing a transaction-counted mbarrier:
 //                     [anchor-key chunks] [tile blocks] [anchor-value chunks]
-//   2 key-residual warps  first the rotated query q' = H(s o q)/128 (Appendix A.1, Eq. 12;
+//   3 key-residual warps  first the rotated query q' = H(s o q)/128 (Appendix A.1, Eq. 12;
 //                     a warp-local Walsh-Hadamard transform) and its fp16 high + low
 //                     fragments; then per tile: q' . c for the staged key records on tensor
 //                     cores, straight from the packed 2-bit codes
