@@ -20,9 +20,11 @@
 //                     the value-residual warps' p, and the value weights
 //                     w[a] = sum_i p_i gamma_i (Eq. 3) -- tokens are stored sorted by
 //                     value anchor, so w is a sum over runs: per lane its head and tail
-//                     runs, merged across lanes by a warp segmented scan, one reduction
-//                     per run into the anchor's owner CTA (shared or DSMEM red);
-//                     phase 3: the anchor-value product of the CTA's anchors, the inverse
+//                     runs, merged across lanes by a warp segmented scan, one shared-memory
+//                     reduction per run into the CTA's own table of the value slots its
+//                     tiles cover (a slot at the edge of two CTAs' tiles gets a share in
+//                     each: the products add up);
+//                     phase 3: the anchor-value product over those slots, the inverse
 //                     rotation of the value-residual sum, cluster combine
 //   4 value-residual warps  per tile: sum of (p scale) c over the staged value records on
 //                     tensor cores, in the rotated domain
@@ -100,7 +102,9 @@ struct DecodeParams {
   int o_lslot;     // [kMaxCluster][GS] each CTA's normaliser share
   int o_fslot;     // [kMaxCluster] each CTA's failure flag
   int o_ofin;      // [C][per] staging: partial output numerators of this CTA's share, per rank
-  int drop_last;   // test hook: the producer withholds its item n_items - drop_last (0: none)
+  int drop_last;   // test hook: the producer withholds its tile item n_kas + n_t - drop_last (0: none)
+  int o_ovf;       // [GS][128] anchor-value products of runs beyond the value-weight table
+  int wrows;       // rows of the value-weight table (value slots o0 .. o0 + wrows - 1)
 };
 
 // ---- device helpers ---------------------------------------------------------------
@@ -223,13 +227,6 @@ __device__ __forceinline__ void st_cluster_int(const int* local, int rank) {
 __device__ __forceinline__ void red_local(float* p, float v) {
   asm volatile("red.shared.add.f32 [%0], %1;" ::"r"(smem_u32(p)), "f"(v) : "memory");
 }
-// Reduction into shared memory of CTA `rank` of the cluster (possibly this one).
-__device__ __forceinline__ void red_cluster(float* local, int rank, float v) {
-  uint32_t remote;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
-  asm volatile("red.shared::cluster.add.f32 [%0], %1;" ::"r"(remote), "f"(v) : "memory");
-}
-
 __device__ __forceinline__ void mma_f16(float (&d)[4], const uint4& a, uint32_t b0, uint32_t b1) {
   asm volatile(
       "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
@@ -512,7 +509,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c4 = lane & 3, r8 = lane >> 2;
   float* SA = reinterpret_cast<float*>(smem + P.o_sa);  // [k][GS] anchor scores (log2 units)
-  float* Wt = reinterpret_cast<float*>(smem + P.o_w);   // [kc][GS] value weights of owned anchors
+  float* Wt = reinterpret_cast<float*>(smem + P.o_w);   // [wrows][GS] value weights of covered slots
   uint2* qfa = reinterpret_cast<uint2*>(smem + P.o_qfa);
   uint2* qfk = reinterpret_cast<uint2*>(smem + P.o_qfk);
   float* qp = reinterpret_cast<float*>(smem + P.o_qp);
@@ -536,6 +533,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float* ofin = reinterpret_cast<float*>(smem + P.o_ofin);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + P.o_bar);
   uint8_t* ring = smem + P.o_ring;
+  float* ovf = reinterpret_cast<float*>(smem + P.o_ovf);
   const int NS = P.NS;
   // per stage: an anchor chunk landed (full_c) / a tile block landed (full_t); stage free
   // again (empty: all token and value-residual warps are done with it); key-residual
@@ -568,27 +566,28 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   const UnitView U = unit_view(P.arena, u);
   const int k = U.k;
 
-  // this CTA's anchors (it owns their value weights) and tile blocks
-  // ceil(k / C) anchors each: their runs lie in about the tiles this CTA reads, so most value
-  // weights are reduced locally
+  // This CTA's stream of items: the anchor-key chunks of its score slice (ceil(k / C) anchors),
+  // its tile blocks, then the anchor-value chunks of the value slots its tiles cover.  Tokens
+  // are stored in value-slot order, so those slots run from the slot of its first stored token,
+  // o0, to that of its last; it weights them with its own tokens only, and the products of the
+  // CTAs whose ranges meet at a slot add up to that slot's share of the output.
   const int kc = (k + C - 1) / C;
   const int a0 = min(k, rank * kc), a1 = min(k, a0 + kc);
   const int j0 = (int)((long long)rank * U.nt / C), j1 = (int)((long long)(rank + 1) * U.nt / C);
-  const int n_ka = (a1 - a0 + CH - 1) / CH;
+  const int n_kas = (a1 - a0 + CH - 1) / CH;
   const int n_t = j1 - j0;
-  const int n_items = 2 * n_ka + n_t;
   const int R = P.R;
   // phase index, on its stage's barrier, of item `it` (anchor chunks and tiles counted apart)
   auto item_phase = [&](int it) -> uint32_t {
-    if (it < n_ka) return (uint32_t)(it / NS);
-    if (it < n_ka + n_t) return (uint32_t)((it - n_ka) / NS);
-    const int s = it % NS, cj = it - n_ka - n_t;
-    const int ka_on_s = n_ka > s ? (n_ka - 1 - s) / NS + 1 : 0;
+    if (it < n_kas) return (uint32_t)(it / NS);
+    if (it < n_kas + n_t) return (uint32_t)((it - n_kas) / NS);
+    const int s = it % NS, cj = it - n_kas - n_t;
+    const int ka_on_s = n_kas > s ? (n_kas - 1 - s) / NS + 1 : 0;
     return (uint32_t)(ka_on_s + cj / NS);
   };
-  auto is_tile = [&](int it) { return it >= n_ka && it < n_ka + n_t; };
-  // Stage and phase parity of the tiles in order, without divisions: tile tl is item n_ka + tl
-  // on stage (n_ka + tl) % NS, and its parity on the tile barriers is (tl / NS) & 1.
+  auto is_tile = [&](int it) { return it >= n_kas && it < n_kas + n_t; };
+  // Stage and phase parity of the tiles in order, without divisions: tile tl is item n_kas + tl
+  // on stage (n_kas + tl) % NS, and its parity on the tile barriers is (tl / NS) & 1.
   struct TileCursor {
     int s, cnt, ns;
     uint32_t par;
@@ -600,7 +599,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       }
     }
   };
-  const TileCursor cursor0{n_ka % NS, 0, NS, 0u};
+  const TileCursor cursor0{n_kas % NS, 0, NS, 0u};
   // B0: every CTA of the cluster has started (its shared memory may take remote stores)
   cluster_arrive();
   // first element of this CTA's query (and output) rows, computed where used
@@ -614,7 +613,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     // The first NS items need no free stage.  Before the first wait for one (a stage whose
     // tile is consumed only after B1) this warp passes B0 and arrives on B1.
     bool ok = true, b1_arrived = false, b1_done = false;
-    const int b1_at = min(NS, n_ka + n_t);
+    const int n_front = n_kas + n_t;
+    const int b1_at = min(NS, n_front);
     auto arrive_b1 = [&]() {
       cluster_wait();  // B0
       cluster_arrive();  // B1
@@ -623,13 +623,28 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     int issued = 0;
     int s = 0;
     uint32_t use = 0;  // it = NS use + s
-    for (int it = 0; it < n_items; ++it, ++s) {
+    // value words of the first and the last stored token (lane 0, read as their tiles are
+    // issued), then the covered slots [o0, oe) and their chunks, from item n_front on
+    uint32_t w_first = 0, w_last = 0;
+    int o0 = 0, oe = 0, n_kao = 0;
+    for (int it = 0;; ++it, ++s) {
+      if (it == n_front) {
+        int f = 0, e = 0;
+        if (lane == 0 && n_t > 0) {
+          f = (int)(w_first & 0xFFFFu);
+          e = min(k, min((int)(w_last & 0xFFFFu) + 1, f + P.wrows));
+        }
+        o0 = __shfl_sync(0xffffffffu, f, 0);
+        oe = __shfl_sync(0xffffffffu, e, 0);
+        n_kao = oe > o0 ? (oe - o0 + CH - 1) / CH : 0;
+      }
+      if (it >= n_front + n_kao) break;
       if (s == NS) {
         s = 0;
         ++use;
       }
       if (it == b1_at) arrive_b1();
-      if (it == n_ka + n_t) {  // anchor values are consumed after B2: let B1 complete, arrive on B2
+      if (it == n_front) {  // anchor values are consumed after B2: let B1 complete, arrive on B2
         cluster_wait();
         cluster_arrive();
         b1_done = true;
@@ -639,23 +654,30 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         *failed = 1;
         break;
       }
-      if (lane == 0 && it != n_items - P.drop_last) {  // (drop_last: a test withholds one item)
+      // (drop_last: a test withholds one tile)
+      if (lane == 0 && !(P.drop_last > 0 && it == n_front - P.drop_last)) {
         const uint32_t dst = smem_u32(stage(s));
         if (!is_tile(it)) {
-          const bool val = it >= n_ka + n_t;
-          const int ci = val ? it - n_ka - n_t : it;
-          const int r0 = a0 + ci * CH, nr = min(a1 - r0, CH);
+          const bool val = it >= n_front;
+          const int r0 = val ? o0 + (it - n_front) * CH : a0 + it * CH;
+          const int nr = min((val ? oe : a1) - r0, CH);
           const uint32_t bytes = (uint32_t)nr * 256u;
           mbar_expect_tx(bar_full_c(s), bytes);
           bulk_g2s(dst, (val ? U.AV : U.AK) + (size_t)r0 * 256, bytes, bar_full_c(s));
         } else {
-          const int j = j0 + it - n_ka;
+          const int j = j0 + it - n_kas;
           const uint32_t b0 = U.table[j], blk = U.table[j + 1] - b0;
           const uint32_t bytes = min(blk, (uint32_t)P.cap);
           meta[s] = make_uint2(b0, blk);
           mbar_expect_tx(bar_full_t(s), bytes);
           bulk_g2s(dst, U.tiles + b0, bytes, bar_full_t(s));
         }
+      }
+      if (lane == 0 && is_tile(it) && (it == n_kas || it == n_front - 1)) {
+        const int j = j0 + it - n_kas, n = min(T, U.S - j * T);
+        const uint8_t* vs = U.tiles + U.table[j] + 4 * ((n + 63) & ~63);  // the value stream
+        if (it == n_kas) w_first = *reinterpret_cast<const uint32_t*>(vs);
+        if (it == n_front - 1) w_last = *reinterpret_cast<const uint32_t*>(vs + 4 * (n - 1));
       }
       issued = it + 1;
       __syncwarp();
@@ -959,9 +981,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   // =========================== token warps =======================================
   // ---- phase 0: zeroed tables, anchor-score B fragments (the rotated query is the
   // key-residual warps' job) ----
-  for (int e = tid; e < GS * 128; e += NTT) accs[e] = 0.f;
+  for (int e = tid; e < GS * 128; e += NTT) accs[e] = ovf[e] = 0.f;
   for (int e = a0 * GS + tid; e < a1 * GS; e += NTT) SA[e] = 0.f;
-  for (int e = tid; e < kc * GS; e += NTT) Wt[e] = 0.f;  // before B1: peers add into it only after B1
+  for (int e = tid; e < P.wrows * GS; e += NTT) Wt[e] = 0.f;
   for (int e = tid; e < ((R + 15) / 16) * 256; e += NTT) reinterpret_cast<uint32_t*>(smem + P.o_pfb)[e] = 0u;
   if (tid < GS) pms[tid] = 0.f;
   if (tid < (GS > 4 ? GS : 4)) {
@@ -996,7 +1018,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   // ---- phase 1: anchor scores of this CTA's slice (bf16 tensor cores) ----
   // work item (16-row block rb, half kh of the 128 dims) -> warp item % NTW; rows are
   // swizzled in 16-byte chunks by (absolute row % 8)
-  for (int it = 0; it < n_ka; ++it) {
+  for (int it = 0; it < n_kas; ++it) {
     const uint8_t* st = wait_item(it);
     if (ok && !warp_failed(failed)) {
       const int r0 = a0 + it * CH, nr = min(a1 - r0, CH);
@@ -1077,20 +1099,27 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     negm[i] = make_float2(-mref[2 * i], GS >= 2 ? -mref[2 * i + 1] : 0.f);
     l2[i] = make_float2(0.f, 0.f);
   }
-  // Value weights of a run: one reduction per head into the anchor's owner CTA.
-  // The owner is nearly always this CTA (its anchors are the ones its tiles hold), so the
-  // branch is taken once per run, not per head.
+  // Value weights of a run: one reduction per head into this CTA's table, whose row i is value
+  // slot o0 + i (o0: the slot of this CTA's first stored token, so no run lies below it).  A run
+  // beyond the table's wrows rows (tiles that cover more slots than it holds: rare) takes its
+  // anchor's value row from global memory and adds its products into ovf on CUDA cores.
+  int o0 = 0, o_last = -1;  // value slots of this CTA's first and last stored tokens
   auto flush = [&](int anchor, const float2 (&v)[NP]) {
-    if (anchor < 0 || anchor >= k) return;
-    if (anchor >= a0 && anchor < a1) {
-      float* w = &Wt[(anchor - a0) * GS];
+    const int i = anchor - o0;
+    if (anchor >= k || i < 0) return;
+    if (i < P.wrows) {
+      float* w = &Wt[i * GS];
 #pragma unroll
       for (int g = 0; g < GS; ++g) red_local(w + g, (g & 1) ? v[g >> 1].y : v[g >> 1].x);
     } else {
-      const int owner = anchor / kc;
-      float* w = &Wt[(anchor - owner * kc) * GS];
+      // (kept compact: this code sits in the token loop but almost never runs)
+      const uint8_t* row = U.AV + (size_t)anchor * 256;
+#pragma unroll 1
+      for (int d = 0; d < 128; ++d) {  // dim d: element d % 8 of chunk d / 8, stored at (d / 8) ^ (row % 8)
+        const float x = __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(row + 16 * ((d >> 3) ^ (anchor & 7)) + 2 * (d & 7)));
 #pragma unroll
-      for (int g = 0; g < GS; ++g) red_cluster(w + g, owner, (g & 1) ? v[g >> 1].y : v[g >> 1].x);
+        for (int g = 0; g < GS; ++g) atomicAdd(&ovf[g * 128 + d], ((g & 1) ? v[g >> 1].y : v[g >> 1].x) * x);
+      }
     }
   };
 
@@ -1111,6 +1140,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       const TileView tv = header_view(st, hdrs + 2 * s, U, P.cap, &mt);
       const float* rsb = reinterpret_cast<const float*>(st + P.o_rs);
       const int t0 = warp * REG + 4 * lane;
+      if (tl == 0) o0 = (int)(*reinterpret_cast<const uint32_t*>(tv.st + 4 * tv.n64) & 0xFFFFu);
+      if (tl == n_t - 1) o_last = (int)(*reinterpret_cast<const uint32_t*>(tv.st + 4 * (tv.n64 + tv.n - 1)) & 0xFFFFu);
       // tail: the run that ends this lane's tokens (its anchor `key`), head: the run that
       // starts them when it differs (multi)
       uint32_t key = 0xFFFFFFFFu;
@@ -1286,21 +1317,24 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   tw_sync();
 
   // ---- phase 3: combine across the cluster (one common reference: plain sums) ----
-  cluster_arrive();  // B2: every value-weight reduction and normaliser share has landed
+  cluster_arrive();  // B2: every normaliser share has landed
   cluster_wait();
   if (tid < GS) {
     float Lt = 0.f;
     for (int r = 0; r < C; ++r) Lt += lslot[r * GS + tid];
     ltot[tid] = Lt;
   }
-  // weights of the owned anchors times their values (bf16 tensor cores, weights as hi + lo);
+  // weights of the covered slots times their values (bf16 tensor cores, weights as hi + lo);
   // warp -> dims 16 warp .. 16 warp + 15
   float oacc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-  for (int ci = 0; ci < n_ka; ++ci) {
-    const int it = n_ka + n_t + ci;
+  // (the producer derives the same covered slots [o0, oe) from the same two tokens)
+  const int oe = n_t > 0 ? min(k, min(o_last + 1, o0 + P.wrows)) : 0;
+  const int n_kao = oe > o0 ? (oe - o0 + CH - 1) / CH : 0;
+  for (int ci = 0; ci < n_kao; ++ci) {
+    const int it = n_kas + n_t + ci;
     const uint8_t* st = wait_item(it);
     if (ok && !warp_failed(failed)) {
-      const int r0 = a0 + ci * CH, nr = min(a1 - r0, CH);
+      const int r0 = o0 + ci * CH, nr = min(oe - r0, CH);
       for (int blk = 0; blk < CH / 16 && 16 * blk < nr; ++blk) {
         const int mi = lane >> 3, ri = lane & 7;
         const int row = 16 * blk + (mi & 1) * 8 + ri;
@@ -1321,7 +1355,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
           __nv_bfloat16 hi[4], lo[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            const float w = kk[e] < nr ? Wt[(r0 - a0 + kk[e]) * GS + r8] : 0.f;
+            const float w = kk[e] < nr ? Wt[(r0 - o0 + kk[e]) * GS + r8] : 0.f;
             split_b(w, hi[e], lo[e]);
           }
           ah0 = pack_b2(hi[0], hi[1]);
@@ -1360,6 +1394,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       opart[r8 * 128 + col + 1] += oacc[nb][1] + oacc[nb][3];
     }
   }
+  tw_sync();
+  for (int e = tid; e < GS * 128; e += NTT) opart[e] += ovf[e];
   tw_sync();
   // Elements are shared out in blocks of `per` (a multiple of 4); each block of this CTA's
   // partial output goes, as 16-byte remote stores, into slot `rank` of the staging rows of
@@ -1440,38 +1476,52 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   // staged bytes of a tile: all of a tile with at most R records per side
   const int cap = (int)(F_MAX + 2 * round16(4u * (uint32_t)R) + 64u * (uint32_t)R);
   const int kc_max = (L.max_k + C - 1) / C;
-  size_t off = 0;
-  auto take = [&](size_t bytes) {
-    const size_t o = off;
-    off = align128(off + bytes);
-    return (int)o;
-  };
-  P.o_sa = take((size_t)L.max_k * GS * 4);
-  P.o_w = take((size_t)kc_max * GS * 4);
-  P.o_qfa = take(8 * 32 * 8);
-  P.o_qfk = take((GS == 8 ? 2 : 1) * 8 * 32 * 8);  // [hi, lo for GS = 8][k-step][lane]
-  P.o_qp = take((size_t)GS * 128 * 4);
-  P.o_acc = take((size_t)GS * 128 * 4);
-  P.o_opart = take((size_t)std::max(GS * 128, NTW * GS) * 4);
-  P.o_misc = take((size_t)(((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15) + 2 * 4 * std::max(GS, 4));
-  P.o_meta = take(8 * 8);
-  P.o_hdr = take(8 * 32);
-  P.o_mslot = take((size_t)kMaxCluster * GS * 4);
-  P.o_lslot = take((size_t)kMaxCluster * GS * 4);
-  P.o_fslot = take((size_t)kMaxCluster * 4);
-  P.o_ofin = take((size_t)(GS * 128 + 4 * kMaxCluster) * 4);  // C x per <= GS 128 + 4 C
-  P.o_bar = take(5 * 8 * 8);
-  P.o_pfb = take((size_t)2 * ((R + 15) / 16) * 512);
   // a stage: staged bytes (a tile block's head, or an anchor chunk), then the key-residual
   // terms of a tile
   const int sb = (int)align128((size_t)std::max(cap, CH * 256));
   P.o_rs = sb;
   P.o_pv = (int)align128((size_t)sb + (size_t)R * GS * 4);
   const int stage = (int)align128((size_t)P.o_pv + (size_t)(R + 1) * GS * 4);  // row R: spare
-  P.o_ring = (int)off;
-  const long long room = (long long)smem_optin - (long long)off;
+  // The value-weight table holds kc_max + 2 m rows, for the value slots a CTA's tiles cover
+  // (about kc_max, more where runs are uneven): m takes what the ring leaves of the shared
+  // memory (at most kc_max).
+  auto layout = [&](int m) -> bool {
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+      const size_t o = off;
+      off = align128(off + bytes);
+      return (int)o;
+    };
+    P.wrows = kc_max + 2 * m;
+    P.o_sa = take((size_t)L.max_k * GS * 4);
+    P.o_w = take((size_t)P.wrows * GS * 4);
+    P.o_qfa = take(8 * 32 * 8);
+    P.o_qfk = take((GS == 8 ? 2 : 1) * 8 * 32 * 8);  // [hi, lo for GS = 8][k-step][lane]
+    P.o_qp = take((size_t)GS * 128 * 4);
+    P.o_acc = take((size_t)GS * 128 * 4);
+    P.o_opart = take((size_t)std::max(GS * 128, NTW * GS) * 4);
+    P.o_misc = take((size_t)(((NTW * GS + 6 * GS + 4) * 4 + 15) & ~15) + 2 * 4 * std::max(GS, 4));
+    P.o_meta = take(8 * 8);
+    P.o_hdr = take(8 * 32);
+    P.o_mslot = take((size_t)kMaxCluster * GS * 4);
+    P.o_lslot = take((size_t)kMaxCluster * GS * 4);
+    P.o_fslot = take((size_t)kMaxCluster * 4);
+    P.o_ofin = take((size_t)(GS * 128 + 4 * kMaxCluster) * 4);  // C x per <= GS 128 + 4 C
+    P.o_bar = take(5 * 8 * 8);
+    P.o_ovf = take((size_t)GS * 128 * 4);
+    P.o_pfb = take((size_t)2 * ((R + 15) / 16) * 512);
+    P.o_ring = (int)off;
+    return true;
+  };
+  layout(0);
+  const long long room = (long long)smem_optin - (long long)P.o_ring;
   if (room < 2LL * stage) return false;
   const int NS = (int)std::min<long long>(8, room / stage);
+  // the margin: whole 128-byte steps of the table within what NS stages leave over
+  const long long spare = room - (long long)NS * stage;
+  const int m = (int)std::min<long long>(kc_max, std::max<long long>(0, (spare - 128) / (2LL * GS * 4)));
+  layout(m);
+  if ((long long)P.o_ring + (long long)NS * stage > (long long)smem_optin) return false;
   P.NS = NS;
   P.stage_bytes = stage;
   P.R = R;
@@ -1631,7 +1681,7 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   cudaGetDevice(&dev);
   int cenv = 0;
   if (const char* env = std::getenv("AKV_CLUSTER")) cenv = std::atoi(env);
-  // test hook (failure detection): with AKV_DEBUG_DROP_LAST=1 every CTA withholds the last item
+  // test hook (failure detection): with AKV_DEBUG_DROP_LAST=1 every CTA withholds the last tile
   // of its stream (its stage is not used again), so the waits on it run out after their bound
   // and the outputs become NaN
   int drop = 0;

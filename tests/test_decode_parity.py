@@ -137,6 +137,23 @@ def test_locally_dense_residuals_exceed_staging(dev):
         _run_seeded(dev, p, [6000, 3000], mutate=mutate)
 
 
+def test_tiles_covering_more_value_slots_than_the_weight_table(dev, monkeypatch):
+    """Every non-anchor token on the last value anchor: stored in value-slot order, the first
+    tile then holds one token of each of about a thousand anchors, more value slots than its
+    CTA's value-weight table rows, so most of its runs take the path that adds their
+    anchor-value products on CUDA cores; the CTAs whose tiles hold the long last run share
+    that slot, each with its own tokens' weights."""
+    def mutate(u, d):
+        non = np.setdiff1d(np.arange(d["S"]), d["anchor_pos"])
+        d["idx_v"] = d["idx_v"].copy()
+        d["idx_v"][non] = d["k"] - 1
+    for c in ("4", "8"):
+        monkeypatch.setenv("AKV_CLUSTER", c)
+        for G in (1, 4):
+            p = akv.Params(batch=1, n_kv_heads=2, n_q_heads=2 * G, anchor_frac=0.2, seed=41)
+            _run_seeded(dev, p, [6000], mutate=mutate, qseed=int(c) + G)
+
+
 def test_back_to_back_launches_follow_stream_order(dev):
     """Consecutive decode launches in one stream overlap their set-up (programmatic dependent
     launch) but not their data: a launch whose query is the previous launch's output, and a
@@ -197,7 +214,7 @@ def test_large_anchor_tables_take_larger_clusters(dev):
 
 def test_withheld_item_times_out_to_nan_and_context_survives(dev, monkeypatch):
     """Failure detection without a GPU fault: with the test hook every CTA withholds the last
-    item of its stream, so the waits on it run out after their bound (about 2 s).  The call
+    tile of its stream, so the waits on it run out after their bound (about 2 s).  The call
     returns, the outputs are NaN, and the next call on the same context is correct."""
     import time
     p = akv.Params(batch=1, n_kv_heads=2, n_q_heads=8, seed=3, rot_seed=77)
