@@ -1482,9 +1482,15 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
   P.o_rs = sb;
   P.o_pv = (int)align128((size_t)sb + (size_t)R * GS * 4);
   const int stage = (int)align128((size_t)P.o_pv + (size_t)(R + 1) * GS * 4);  // row R: spare
-  // The value-weight table holds kc_max + 2 m rows, for the value slots a CTA's tiles cover
-  // (about kc_max, more where runs are uneven): m takes what the ring leaves of the shared
-  // memory (at most kc_max).
+  // The value-weight table holds kt + 2 m rows for the value slots a CTA's tiles cover: kt, the
+  // larger tile share of a CTA (where C does not divide a unit's tiles) times the unit's slots
+  // per tile, plus the slot a first run continues; m, a margin for uneven runs, takes what the
+  // ring leaves of the shared memory (at most kc_max).
+  int kt = 1;
+  for (const auto& sh : L.shape) {
+    const long long tmax = (sh.nt + C - 1) / C;
+    kt = std::max(kt, (int)(((long long)sh.k * tmax + sh.nt - 1) / std::max(1, sh.nt)) + 1);
+  }
   auto layout = [&](int m) -> bool {
     size_t off = 0;
     auto take = [&](size_t bytes) {
@@ -1492,7 +1498,7 @@ bool make_plan_r(const Layout& L, int GS, int C, int R, int smem_optin, Plan* ou
       off = align128(off + bytes);
       return (int)o;
     };
-    P.wrows = kc_max + 2 * m;
+    P.wrows = kt + 2 * m;
     P.o_sa = take((size_t)L.max_k * GS * 4);
     P.o_w = take((size_t)P.wrows * GS * 4);
     P.o_qfa = take(8 * 32 * 8);
