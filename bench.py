@@ -1,16 +1,22 @@
 #!/usr/bin/env python
 """Benchmark of AnchorKV decode attention on GB300.
 
-Workload (default "8b-32k"): Llama-3.1-8B layer shape, 32 query / 8 KV heads,
-head_dim 128, context 32768, batch 1, 2 % anchors and 10 % residual slots
-(about 20x smaller than the bf16 cache), encoded on the GPU from the clustered
-synthetic K/V recipe.  A step is one decode-attention call for one layer with
-a fresh query; the timed region cycles through 32 distinct layer caches
-(217 MB, larger than the 129 MB L2) and 64 fresh query sets, replayed from a
-CUDA graph.  The metric is compressed bytes read per second (GB/s) and
-microseconds per step.
+Workload (default "70b-128k", the largest single-GPU configuration): Llama-3-70B
+layer shape, 64 query / 8 KV heads (G = 8), head_dim 128, context 131072, batch 8,
+2 % anchors and 10 % residual slots per side (about 20x smaller than the bf16
+cache), a seeded compressed cache.  A step is one decode-attention call for one
+layer with a fresh query set; the timed region cycles through 4 distinct layer
+caches (874 MB, several times the 129 MB L2) and 64 fresh query sets, replayed
+from CUDA graphs.  The metric is compressed bytes read per second (GB/s) and
+microseconds per step.  Other workloads: "8b-32k" (GPU-encoded clustered K/V,
+32 layers cycled), "8b-128k", and the ragged budget sweep "sweep-a<A>-r<R>".
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl akv|reference] [--workload NAME]
+
+With --gpus N > 1 and no torch.distributed environment, the script starts N
+ranks itself (torch.distributed.run on 127.0.0.1), one per GPU; each rank
+encodes and decodes its own requests (data parallel by request, no collective
+on the data path) and the line reports the whole job.
 """
 from __future__ import annotations
 
@@ -55,24 +61,39 @@ def workload_params(akv, name: str, **kw):
     """akv.Params of a workload (the sweep points set their budgets)."""
     fa, fr = SWEEP_POINTS.get(name, (0.02, 0.10))
     return akv.Params(anchor_frac=fa, res_frac_k=fr, res_frac_v=fr, **kw)
-N_LAYERS = 32
 N_TOKENS = 64
+# layer caches cycled per workload: enough distinct bytes to exceed the 129 MB L2 several times
+DEFAULT_LAYERS = {"8b-32k": 32, "8b-128k": 8, "70b-128k": 4}
+DEFAULT_LAYERS.update({n: 2 for n in SWEEP_POINTS})
+# graph replays of (N_TOKENS x layers) steps timed by default, about ten seconds or less of device time
+DEFAULT_REPLAYS = {"8b-32k": 100, "8b-128k": 40, "70b-128k": 40}
 DEC_KERNEL_SRC = os.path.join(ROOT, "paper_2608_02901_gb300", "csrc", "akv_decode.cu")
 
 
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=N_LAYERS * N_TOKENS * 100)
-    ap.add_argument("--warmup", type=int, default=N_LAYERS * N_TOKENS)
+    ap.add_argument("--steps", type=int, default=None)
+    ap.add_argument("--warmup", type=int, default=None)
     ap.add_argument("--impl", default="akv", choices=["akv", "reference"])
-    ap.add_argument("--workload", default="8b-32k", choices=sorted(WORKLOADS))
-    ap.add_argument("--layers", type=int, default=N_LAYERS)
+    ap.add_argument("--workload", default="70b-128k", choices=sorted(WORKLOADS))
+    ap.add_argument("--layers", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--launch-check", action="store_true",
+                    help="start the ranks, have each report itself through the process group, print them and exit "
+                         "(checks the N-rank launch; measures nothing)")
     ap.add_argument("--dense-context", action="store_true",
                     help="context only: torch scaled-dot-product attention decoding over the dense bf16 K/V of the same "
                          "shapes (a library kernel, not this repository's path)")
-    return ap.parse_args()
+    args = ap.parse_args()
+    if args.layers is None:
+        args.layers = DEFAULT_LAYERS.get(args.workload, 2)
+    chunk = N_TOKENS * args.layers
+    if args.steps is None:
+        args.steps = chunk * DEFAULT_REPLAYS.get(args.workload, 8)
+    if args.warmup is None:
+        args.warmup = chunk
+    return args
 
 
 TILE = 1024
@@ -93,21 +114,26 @@ def unit_bytes(S, k, nk, nv, G):
     return 512 * k + 4 * (nt + 1) + fixed + 36 * (nk + nv) + 252 * nt + 2 * (2 * G * 128)
 
 
-def arena_read_bytes(torch, akv, p, lens, arena):
-    """Exact bytes one decode reads from this arena (anchors, tile tables, the tile blocks
-    as the tables record them), plus the q and out rows."""
+def arena_unit_bytes(torch, akv, p, lens, arena) -> list:
+    """Exact bytes one decode reads from this arena per unit (anchors, tile table, the tile
+    blocks as the table records them), plus the unit's q and out rows."""
     hdr = akv.akv_cache_header_host(p, lens)
-    total = 0
+    fixed = []
     offs = []
     for u in range(p.n_units):
         d = hdr[256 * (u + 1): 256 * (u + 2)]
         k, nt = int(d[4:8].view(np.int32)[0]), int(d[16:20].view(np.int32)[0])
         o_tt = int(d[56:64].view(np.uint64)[0])
         offs.append(o_tt + 4 * nt)
-        total += 512 * k + 4 * (nt + 1) + 2 * (2 * p.G * 128)
+        fixed.append(512 * k + 4 * (nt + 1) + 2 * (2 * p.G * 128))
     idx = torch.tensor([o + i for o in offs for i in range(4)], dtype=torch.long, device=arena.device)
-    used = arena[idx].cpu().numpy().view(np.uint32)
-    return total + int(used.astype(np.int64).sum())
+    used = arena[idx].cpu().numpy().view(np.uint32).astype(np.int64)
+    return [f + int(b) for f, b in zip(fixed, used)]
+
+
+def arena_read_bytes(torch, akv, p, lens, arena):
+    """Exact bytes one decode reads from this arena, plus the q and out rows."""
+    return sum(arena_unit_bytes(torch, akv, p, lens, arena))
 
 
 def rank_seed(base: int, rank: int) -> int:
@@ -115,11 +141,29 @@ def rank_seed(base: int, rank: int) -> int:
     return base + 1000003 * rank
 
 
+def free_port() -> int:
+    import socket
+    with socket.socket(socket.AF_INET, socket.SOCK_STREAM) as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def launch_ranks(n: int) -> int:
+    """Re-run this script as n ranks on one node (torch.distributed.run, rendezvous on 127.0.0.1);
+    returns the launcher's exit code."""
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={n}",
+           "--master-addr=127.0.0.1", f"--master-port={free_port()}", os.path.abspath(__file__)] + sys.argv[1:]
+    env = dict(os.environ, OMP_NUM_THREADS=os.environ.get("OMP_NUM_THREADS", "1"))
+    return subprocess.run(cmd, env=env).returncode
+
+
 def dist_setup(args):
     import torch
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args is not None and world != args.gpus:
+        raise SystemExit(f"bench.py: --gpus {args.gpus} but the process group has WORLD_SIZE={world} ranks")
     if world > 1:
         import torch.distributed as dist
         backend = "nccl" if torch.cuda.is_available() else "gloo"
@@ -328,29 +372,53 @@ def run_akv(args, rank, world, local):
     value = world * step_bytes * args.steps / sec / 1e9
     us_step = ms * 1e3 / args.steps
 
-    # end to end through the C ABI with host buffers: pinned q in, pinned out back, every step
-    e2e_steps = min(args.steps, 2 * chunk)
-    q_host = torch.empty((n_tok, layers, B, Hq, 128), dtype=torch.bfloat16, pin_memory=True)
-    q_host.copy_(qs.cpu())
-    o_host = torch.empty((B, Hq, 128), dtype=torch.bfloat16, pin_memory=True)
+    # End to end through the C ABI with host buffers: every step copies its query set in from
+    # pinned host memory, decodes, copies the output back to pinned host memory and waits for
+    # it on the host.  The three operations of a step are replayed from one CUDA graph (the
+    # way a serving loop issues them); the same steps issued eagerly from Python are reported
+    # beside it.
+    e2e_steps = min(args.steps, chunk, 64)
+    q_host = torch.empty((e2e_steps, B, Hq, 128), dtype=torch.bfloat16, pin_memory=True)
+    for i in range(e2e_steps):
+        t, layer = divmod(i, layers)
+        q_host[i].copy_(qs[t, layer].cpu())
+    o_host = torch.empty((e2e_steps, B, Hq, 128), dtype=torch.bfloat16, pin_memory=True)
     q_dev = torch.empty((B, Hq, 128), dtype=torch.bfloat16, device=dev)
     o_dev = torch.empty((B, Hq, 128), dtype=torch.bfloat16, device=dev)
+
+    def e2e_ops(i, s):
+        q_dev.copy_(q_host[i], non_blocking=True)
+        akv.akv_decode_attn(p, lens, arenas[i % layers], q_dev, o_dev, None, 1.0, None, s)
+        o_host[i].copy_(o_dev, non_blocking=True)
+
+    e2e_graphs = []
+    for i in range(e2e_steps):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            e2e_ops(i, torch.cuda.current_stream())
+        e2e_graphs.append(g)
+    for g in e2e_graphs:  # warm-up
+        g.replay()
     torch.cuda.synchronize()
     dist_barrier(world)
+    t0 = time.perf_counter()
+    for g in e2e_graphs:
+        g.replay()
+        stream.synchronize()
+    e2e_sec = dist_max(time.perf_counter() - t0, world)
     with torch.cuda.stream(stream):
         t0 = time.perf_counter()
         for i in range(e2e_steps):
-            t, layer = divmod(i % chunk, layers)
-            q_dev.copy_(q_host[t, layer], non_blocking=True)
-            akv.akv_decode_attn(p, lens, arenas[layer], q_dev, o_dev, None, 1.0, None, stream)
-            o_host.copy_(o_dev, non_blocking=True)
+            e2e_ops(i, stream)
             stream.synchronize()
-        e2e_sec = time.perf_counter() - t0
-    e2e_sec = dist_max(e2e_sec, world)
+        eager_sec = dist_max(time.perf_counter() - t0, world)
     h2d = B * Hq * 128 * 2
     e2e = {"value": round(world * step_bytes * e2e_steps / e2e_sec / 1e9, 3), "unit": "GB/s",
            "us_per_step": round(e2e_sec * 1e6 / e2e_steps, 3), "steps": e2e_steps,
-           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": h2d}
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": h2d,
+           "how": "per step: H2D copy of the query set from pinned memory, akv_decode_attn, D2H copy of the output "
+                  "to pinned memory (one CUDA graph per step), host synchronisation",
+           "eager_us_per_step": round(eager_sec * 1e6 / e2e_steps, 3)}
 
     peaks = {}
     try:
@@ -366,7 +434,7 @@ def run_akv(args, rank, world, local):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(torch, akv, p, lens, arenas)
+        cpu = cpu_baseline(torch, akv, p, lens, arenas[0])
 
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": "GB/s", "us_per_step": round(us_step, 4),
@@ -390,26 +458,42 @@ def _oracle_units_from_arena(torch, arena):
     return oracle.unpack_arena(arena.cpu().numpy())
 
 
-def cpu_baseline(torch, akv, p, lens, arenas, budget_s=12.0):
-    """The fp64 oracle, as it stands, on the host cores: whole layers of the same workload."""
+def cpu_baseline(torch, akv, p, lens, arena, budget_s=16.0):
+    """The fp64 oracle, as it stands, on the host cores, over the same layer cache the GPU reads:
+    whole layer steps with OpenMP over the units (threads = min(cores, units)), then single units
+    on one core.  Bytes are the exact bytes of the units attended (the tile tables' sizes)."""
     import gen
     import oracle
-    units = _oracle_units_from_arena(torch, arenas[0])
-    G = p.G
-    q = gen.queries(p.batch * p.n_q_heads, seed=5)
-    shapes = akv.akv_unit_shapes(p, lens)
-    layer_bytes = sum(unit_bytes(int(S), int(k), int(nk), int(nv), G) for S, k, nk, nv in shapes)
+    units = _oracle_units_from_arena(torch, arena)
+    ub = arena_unit_bytes(torch, akv, p, lens, arena)
+    G, n = p.G, p.n_units
+    q = gen.queries(n * G, seed=5).reshape(n, G, 128)
+    nproc = os.cpu_count() or 1
+    threads = min(nproc, n)
     done, t0 = 0, time.perf_counter()
     while True:
-        oracle.attend(units, q.reshape(p.n_units, G, 128), G, 1.0, p.rot_seed)
+        oracle.attend(units, q, G, 1.0, p.rot_seed)
         done += 1
-        if time.perf_counter() - t0 > budget_s:
+        if time.perf_counter() - t0 > budget_s / 2:
             break
     sec = time.perf_counter() - t0
-    cores = min(os.cpu_count() or 1, p.n_units)
-    return {"value": round(layer_bytes * done / sec / 1e9, 5), "unit": "GB/s", "cores": cores, "kind": "oracle",
-            "sample": f"{done} full layer steps ({p.n_units} units, OpenMP over units) of the {lens[0]}-token layer",
-            "seconds": round(sec, 2), "us_per_step": round(sec * 1e6 / done, 1)}
+    one, b1, t1 = 0, 0, time.perf_counter()
+    sel = np.zeros(n, np.uint8)
+    while True:
+        sel[:] = 0
+        sel[one % n] = 1
+        oracle.attend(units, q, G, 1.0, p.rot_seed, sel=sel)
+        b1 += ub[one % n]
+        one += 1
+        if time.perf_counter() - t1 > budget_s / 2:
+            break
+    sec1 = time.perf_counter() - t1
+    return {"value": round(sum(ub) * done / sec / 1e9, 5), "unit": "GB/s", "cores": threads, "nproc": nproc,
+            "kind": "oracle",
+            "sample": f"{done} full layer steps of the workload's first layer cache ({n} units, OpenMP over units)",
+            "seconds": round(sec, 2), "us_per_step": round(sec * 1e6 / done, 1),
+            "single_core": {"value": round(b1 / sec1 / 1e9, 5), "unit": "GB/s", "cores": 1,
+                            "sample": f"{one} single units of the same layer, one at a time", "seconds": round(sec1, 2)}}
 
 
 def run_reference(args, rank, world, local):
@@ -540,11 +624,32 @@ def run_dense_context(args, rank, world, local):
                       "(library kernel, context only)"}), flush=True)
 
 
+def run_launch_check(args, rank, world, local):
+    """Every rank reports (rank, local rank, world size) through the process group; rank 0 prints them."""
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        mine = [rank, local, world, os.getpid()]
+        got = [None] * world
+        dist.all_gather_object(got, mine)
+    else:
+        got = [[rank, local, world, os.getpid()]]
+    if rank == 0:
+        print(json.dumps({"launch_check": True, "n_gpus": args.gpus, "world_size": world,
+                          "ranks": sorted(g[0] for g in got), "local_ranks": sorted(g[1] for g in got),
+                          "distinct_processes": len({g[3] for g in got}),
+                          "backend": "nccl" if torch.cuda.is_available() else "gloo"}), flush=True)
+
+
 def main():
     args = parse()
+    if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
+        sys.exit(launch_ranks(args.gpus))
     rank, world, local = dist_setup(args)
     try:
-        if args.dense_context:
+        if args.launch_check:
+            run_launch_check(args, rank, world, local)
+        elif args.dense_context:
             run_dense_context(args, rank, world, local)
         elif args.impl == "reference":
             run_reference(args, rank, world, local)

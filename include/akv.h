@@ -247,9 +247,11 @@ akv_status akv_encode(const akv_params* p, const int32_t* ctx_lens_host, const v
  *  - The encode workspace that akv_cache_size reports for (p, ctx_lens_host)
  *    must fit AKV_NOALLOC_SCRATCH_BYTES; otherwise AKV_ERR_UNSUPPORTED and
  *    nothing is launched.
- *  - The first call on a device looks up that device's address of the array
- *    (cudaGetSymbolAddress, with the device current).  Make that first call
- *    before any stream capture.
+ *  - Every call looks up the array's address on the current device and
+ *    context (cudaGetSymbolAddress), so the address stays right after a device
+ *    reset or in a non-primary context.  The first call on a device also
+ *    loads the library's module there: make that first call before any
+ *    stream capture.
  *  - Every call on a device shares the one array and leaves its contents
  *    behind; the kernels need none of it cleared.  Calls whose work overlaps
  *    on the GPU (different streams, no ordering between them) race on the
@@ -327,6 +329,23 @@ akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_len
 akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,
                            size_t arena_bytes, const void* q, void* out, float* out_f32, float sm_scale,
                            void* ws, size_t ws_bytes, akv_stream_t stream);
+
+/* ---- Testing and tuning controls ------------------------------------------ */
+
+/*
+ * Process-wide controls of akv_decode_attn, for tests and tuning (the paper has
+ * no counterpart).  Both are 0 by default, which is normal operation; a call
+ * applies to every decode launch issued after it, on every thread.
+ *   cluster_ctas  : 0 = the launch planner chooses the CTAs per (request, KV
+ *                   head); 1..16 = that many, or the largest smaller count
+ *                   whose launch fits the device
+ *   withhold_last : 1 = every CTA withholds the last tile of its stream, so the
+ *                   waits on it run out after their bound (about 2 s): the call
+ *                   returns and its outputs are NaN.  This tests the bounded
+ *                   waits (failure detection) without any GPU fault.
+ * Errors: AKV_ERR_INVALID for values out of range.
+ */
+akv_status akv_decode_set_debug(int32_t cluster_ctas, int32_t withhold_last);
 
 #ifdef __cplusplus
 } /* extern "C" */

@@ -4,7 +4,9 @@ Only the tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 ``bench.py`` may import this package.  The product library never calls it and
 shares no code with it: ``akv_oracle.c`` is written from the paper's
 equations (Section 3.1 Eq. 1-3, Section 3.3 Eq. 4, Appendix A.1 Eq. 12-14,
-Section 3.2 anchor selection) and the readings recorded in the design doc.
+Section 3.2 anchor selection) and the readings R1-R16 where the paper is
+silent or ambiguous (GQA mapping, anchor sampling, tie rules, rounding, the
+quantizer's scale and min, the stored token order).
 
 Every function here is marshalling around the C file; the arithmetic lives
 there.  Parity status: every function is pinned by ``tests/test_oracle_*.py``

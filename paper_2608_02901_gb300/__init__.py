@@ -24,6 +24,7 @@ HEAD_DIM = 128
 EXPORTED = (
     "akv_status_string", "akv_last_error", "akv_unit_shapes", "akv_cache_size", "akv_cache_header_host",
     "akv_encode", "akv_encode_noalloc", "akv_cache_pack_host", "akv_decode_workspace_size", "akv_decode_attn",
+    "akv_decode_set_debug",
 )
 NOALLOC_SCRATCH_BYTES = 16 << 20
 
@@ -110,6 +111,8 @@ def lib():
         L.akv_decode_attn.restype = st
         L.akv_decode_attn.argtypes = [P, i32p, vp, ctypes.c_size_t, vp, vp, vp, ctypes.c_float, vp,
                                       ctypes.c_size_t, vp]
+        L.akv_decode_set_debug.restype = st
+        L.akv_decode_set_debug.argtypes = [ctypes.c_int32, ctypes.c_int32]
         _lib = L
     return _lib
 
@@ -262,6 +265,11 @@ def akv_decode_attn(p: Params, ctx_lens, arena, q, out, out_f32=None, sm_scale: 
                                  _dev_ptr(out), _dev_ptr(out_f32), float(sm_scale), _dev_ptr(ws), ws_bytes,
                                  _stream_ptr(stream)),
            "akv_decode_attn")
+
+
+def akv_decode_set_debug(cluster_ctas: int = 0, withhold_last: int = 0):
+    """Testing controls of the decode launch (0, 0 = normal operation)."""
+    _check(lib().akv_decode_set_debug(int(cluster_ctas), int(withhold_last)), "akv_decode_set_debug")
 
 
 def unit_host_from_logical(u: dict) -> dict:

@@ -4,6 +4,8 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <memory>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -154,6 +156,40 @@ void encode_ws_layout(const Layout& L, EncodeWs* ws) {
     off += b;
   }
   ws->total = off + 256;
+}
+
+// Layouts of recent decode calls.  A decode loop repeats the same (params, lengths) call after
+// call; the layout (one descriptor per unit) is then built once instead of on every call.
+std::shared_ptr<const Layout> decode_layout(const akv_params* p, const int32_t* ctx_lens, akv_status* st) {
+  static std::mutex mu;
+  struct Entry {
+    akv_params p;
+    std::vector<int32_t> lens;
+    std::shared_ptr<const Layout> L;
+  };
+  static std::vector<Entry> recent;  // most recent last, at most kKeep
+  constexpr size_t kKeep = 16;
+  *st = AKV_OK;
+  const bool cacheable = p && ctx_lens && p->batch >= 1 && p->batch <= 4096;
+  if (cacheable) {
+    std::lock_guard<std::mutex> lk(mu);
+    for (size_t i = recent.size(); i-- > 0;) {
+      const Entry& e = recent[i];
+      if (std::memcmp(&e.p, p, sizeof(akv_params)) == 0 &&
+          std::memcmp(e.lens.data(), ctx_lens, sizeof(int32_t) * (size_t)p->batch) == 0 &&
+          e.lens.size() == (size_t)p->batch)
+        return e.L;
+    }
+  }
+  auto L = std::make_shared<Layout>();
+  *st = make_layout(p, ctx_lens, L.get());
+  if (*st != AKV_OK) return nullptr;
+  if (cacheable) {
+    std::lock_guard<std::mutex> lk(mu);
+    if (recent.size() >= kKeep) recent.erase(recent.begin());
+    recent.push_back(Entry{*p, std::vector<int32_t>(ctx_lens, ctx_lens + p->batch), L});
+  }
+  return L;
 }
 
 }  // namespace akv
@@ -367,6 +403,15 @@ akv_status akv_encode_noalloc(const akv_params* p, const int32_t* ctx_lens_host,
   return akv_encode(p, ctx_lens_host, K, V, s_max, arena, arena_bytes, ws, ws_bytes, stream);
 }
 
+akv_status akv_decode_set_debug(int32_t cluster_ctas, int32_t withhold_last) {
+  g_last_error.clear();
+  if (cluster_ctas < 0 || cluster_ctas > 16) return fail(AKV_ERR_INVALID, "cluster_ctas must be in [0, 16]");
+  if (withhold_last < 0 || withhold_last > 1) return fail(AKV_ERR_INVALID, "withhold_last must be 0 or 1");
+  g_debug_cluster.store(cluster_ctas);
+  g_debug_withhold.store(withhold_last);
+  return AKV_OK;
+}
+
 akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_lens_host, size_t* ws_bytes) {
   g_last_error.clear();
   Layout L;
@@ -382,10 +427,11 @@ akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, co
                            void* ws, size_t ws_bytes, akv_stream_t stream) {
   (void)ws;
   (void)ws_bytes;
-  g_last_error.clear();
-  Layout L;
-  akv_status st = make_layout(p, ctx_lens_host, &L);
+  if (!g_last_error.empty()) g_last_error.clear();
+  akv_status st;
+  const std::shared_ptr<const Layout> Lp = decode_layout(p, ctx_lens_host, &st);
   if (st != AKV_OK) return st;
+  const Layout& L = *Lp;
   if (!arena || !q || !out) return fail(AKV_ERR_INVALID, "null arena, q or out");
   if (((uintptr_t)arena % 256) || ((uintptr_t)q % 16) || ((uintptr_t)out % 16) || ((uintptr_t)out_f32 % 16))
     return fail(AKV_ERR_INVALID, "arena must be 256-byte aligned; q, out, out_f32 16-byte aligned");

@@ -44,6 +44,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cstdio>
 #include <cstdlib>
 #include <map>
@@ -1685,13 +1686,11 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   const int vunits = units * nhg;
   int dev = 0;
   cudaGetDevice(&dev);
-  int cenv = 0;
-  if (const char* env = std::getenv("AKV_CLUSTER")) cenv = std::atoi(env);
-  // test hook (failure detection): with AKV_DEBUG_DROP_LAST=1 every CTA withholds the last tile
-  // of its stream (its stage is not used again), so the waits on it run out after their bound
-  // and the outputs become NaN
-  int drop = 0;
-  if (const char* env = std::getenv("AKV_DEBUG_DROP_LAST")) drop = std::max(0, std::atoi(env));
+  // testing controls (akv_decode_set_debug): a requested cluster size, and the failure-detection
+  // hook with which every CTA withholds the last tile of its stream (its stage is not used
+  // again), so the waits on it run out after their bound and the outputs become NaN
+  const int cenv = g_debug_cluster.load(std::memory_order_relaxed);
+  const int drop = g_debug_withhold.load(std::memory_order_relaxed);
   const LaunchKey key{dev, L.G, units, L.max_len, L.max_k, cenv, (long long)(max_density(L) * 1e6)};
   Plan pl;
   int err = plan_for<GS>(L, key, vunits, &pl, why);
@@ -1733,6 +1732,8 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
 }
 
 }  // namespace
+
+std::atomic<int> g_debug_cluster{0}, g_debug_withhold{0};
 
 int launch_decode(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
                   float sm_scale, void* stream, std::string* why) {

@@ -669,22 +669,16 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[AKV_NOALLOC_SCR
 
 int noalloc_scratch(void** ptr, size_t* bytes) {
   // Host code must not use g_noalloc_scratch's name as a device address: it is
-  // a host-side stand-in.  The device address is looked up once per device,
-  // with that device current.
-  static std::mutex mu;
-  static void* addr[64] = {};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  // a host-side stand-in.  The device address is looked up on every call, with
+  // the caller's device current, rather than cached: after cudaDeviceReset the
+  // module is loaded again and the array may move, and a context other than the
+  // primary one holds its own copy, so a cached address could point at memory
+  // this call does not own.  The lookup costs far less than the encode.  The
+  // first lookup on a device loads the library's module there.
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
   if (e != cudaSuccess) return (int)e;
-  if (dev < 0 || dev >= 64) return (int)cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lk(mu);
-  if (!addr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess) return (int)e;
-    addr[dev] = p;
-  }
-  *ptr = addr[dev];
+  *ptr = p;
   *bytes = AKV_NOALLOC_SCRATCH_BYTES;
   return 0;
 }

@@ -1,6 +1,7 @@
 // Internal declarations shared by the host API and the CUDA translation units.
 #pragma once
 
+#include <atomic>
 #include <cstddef>
 #include <cstdint>
 #include <string>
@@ -86,8 +87,10 @@ int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const
 int launch_decode(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
                   float sm_scale, void* stream, std::string* why);
 const char* cuda_error_string(int err);
+// Testing controls of the decode launch (akv_decode_set_debug), 0 = normal operation.
+extern std::atomic<int> g_debug_cluster, g_debug_withhold;
 // Device address of the library's static encode scratch on the current device
-// (looked up once per device); returns a cudaError_t as int.
+// and context (looked up on every call); returns a cudaError_t as int.
 int noalloc_scratch(void** ptr, size_t* bytes);
 
 }  // namespace akv

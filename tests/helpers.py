@@ -7,7 +7,7 @@ import gen
 import oracle
 import paper_2608_02901_gb300 as akv
 
-# Parity bar (written out in DESIGN.md, "Parity bar"):
+# Parity bar (derived from the arithmetic of the kernel):
 #  * fp32 output vs the fp64 oracle: max-abs <= 1e-4 * max(1, |y|).  The kernel
 #    accumulates in fp32 over <= 2^17 terms of magnitude <= 1 with hardware exp2;
 #    1e-4 is ~100x the expected error and 50x tighter than the 5e-3 target.
@@ -19,6 +19,9 @@ import paper_2608_02901_gb300 as akv
 F32_MAX_ABS = 1e-4
 BF16_MAX_ABS = 5e-3
 BF16_MEAN_ABS = 5e-4
+# (case, bf16 max-abs, bf16 mean-abs, fp32 max-abs, widened bar needed) of every parity check
+# this session, printed in pytest's terminal summary (tests/conftest.py)
+PARITY_LOG: list = []
 
 
 def bf16_half_ulp(y: np.ndarray) -> np.ndarray:
@@ -47,6 +50,8 @@ def check_outputs(out_bf16: np.ndarray, out_f32: np.ndarray, ref: np.ndarray, wh
     hu = bf16_half_ulp(ref)
     assert np.all(e16 <= np.maximum(BF16_MAX_ABS, hu + tol32)), f"{where}: bf16 max err {e16.max():.3e}"
     assert e16.mean() <= max(BF16_MEAN_ABS, hu.mean()), f"{where}: bf16 mean err {e16.mean():.3e}"
+    widened = bool(e16.max() > BF16_MAX_ABS or e16.mean() > BF16_MEAN_ABS)
+    PARITY_LOG.append((where or "?", float(e16.max()), float(e16.mean()), float(e32.max()), widened))
     return e16.max(), e16.mean(), e32.max()
 
 

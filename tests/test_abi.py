@@ -190,3 +190,10 @@ def test_entry_points_validate_before_any_launch():
     assert st == akv.AKV_ERR_INVALID  # s_max < S
     st = L.akv_encode(ctypes.byref(p), lp, 256, 256, 128, 0x1000, nbytes, 0x2000, 16, None)
     assert st == akv.AKV_ERR_TOO_SMALL
+
+
+def test_decode_debug_controls_validate():
+    assert _err(akv.akv_decode_set_debug, 17, 0) == akv.AKV_ERR_INVALID
+    assert _err(akv.akv_decode_set_debug, -1, 0) == akv.AKV_ERR_INVALID
+    assert _err(akv.akv_decode_set_debug, 0, 2) == akv.AKV_ERR_INVALID
+    akv.akv_decode_set_debug(0, 0)

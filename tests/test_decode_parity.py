@@ -21,6 +21,13 @@ def dev():
     return torch.device("cuda:0")
 
 
+@pytest.fixture
+def debug_controls():
+    """The decode testing controls, put back to normal operation after the test."""
+    yield
+    akv.akv_decode_set_debug(0, 0)
+
+
 def _run_seeded(dev, p, lens, sm_scale=1.0, seed=5, mutate=None, qseed=17):
     units = seeded_units(p, lens, seed=seed, mutate=mutate)
     arena = akv.akv_cache_pack_host(p, lens, [akv.unit_host_from_logical(u) for u in units])
@@ -66,11 +73,11 @@ def test_negative_and_saturated_gamma_and_zero_anchor(dev):
     _run_seeded(dev, p, [1500, 900], mutate=mutate)
 
 
-def test_many_units_cluster_sizes(dev, monkeypatch):
+def test_many_units_cluster_sizes(dev, debug_controls):
     p = akv.Params(batch=4, n_kv_heads=4, n_q_heads=16)
-    for c in ("1", "2", "3", "8", "16"):
-        monkeypatch.setenv("AKV_CLUSTER", c)
-        _run_seeded(dev, p, [8192, 3000, 6001, 700], qseed=int(c))
+    for c in (1, 2, 3, 8, 16):
+        akv.akv_decode_set_debug(cluster_ctas=c)
+        _run_seeded(dev, p, [8192, 3000, 6001, 700], qseed=c)
 
 
 @pytest.mark.parametrize("H,G", [(1, 1), (2, 4)])
@@ -137,7 +144,7 @@ def test_locally_dense_residuals_exceed_staging(dev):
         _run_seeded(dev, p, [6000, 3000], mutate=mutate)
 
 
-def test_tiles_covering_more_value_slots_than_the_weight_table(dev, monkeypatch):
+def test_tiles_covering_more_value_slots_than_the_weight_table(dev, debug_controls):
     """Every non-anchor token on the last value anchor: stored in value-slot order, the first
     tile then holds one token of each of about a thousand anchors, more value slots than its
     CTA's value-weight table rows, so most of its runs take the path that adds their
@@ -147,11 +154,11 @@ def test_tiles_covering_more_value_slots_than_the_weight_table(dev, monkeypatch)
         non = np.setdiff1d(np.arange(d["S"]), d["anchor_pos"])
         d["idx_v"] = d["idx_v"].copy()
         d["idx_v"][non] = d["k"] - 1
-    for c in ("4", "8"):
-        monkeypatch.setenv("AKV_CLUSTER", c)
+    for c in (4, 8):
+        akv.akv_decode_set_debug(cluster_ctas=c)
         for G in (1, 4):
             p = akv.Params(batch=1, n_kv_heads=2, n_q_heads=2 * G, anchor_frac=0.2, seed=41)
-            _run_seeded(dev, p, [6000], mutate=mutate, qseed=int(c) + G)
+            _run_seeded(dev, p, [6000], mutate=mutate, qseed=c + G)
 
 
 def test_back_to_back_launches_follow_stream_order(dev):
@@ -212,7 +219,7 @@ def test_large_anchor_tables_take_larger_clusters(dev):
     check_outputs(out[rows], out32[rows], ref[rows], where="large anchor tables")
 
 
-def test_withheld_item_times_out_to_nan_and_context_survives(dev, monkeypatch):
+def test_withheld_item_times_out_to_nan_and_context_survives(dev, debug_controls):
     """Failure detection without a GPU fault: with the test hook every CTA withholds the last
     tile of its stream, so the waits on it run out after their bound (about 2 s).  The call
     returns, the outputs are NaN, and the next call on the same context is correct."""
@@ -222,11 +229,11 @@ def test_withheld_item_times_out_to_nan_and_context_survives(dev, monkeypatch):
     units = seeded_units(p, lens, seed=5)
     arena = torch.from_numpy(akv.akv_cache_pack_host(p, lens, [akv.unit_host_from_logical(u) for u in units])).to(dev)
     q = gen.queries(p.batch * p.n_q_heads, seed=17)
-    monkeypatch.setenv("AKV_DEBUG_DROP_LAST", "1")
+    akv.akv_decode_set_debug(withhold_last=1)
     t0 = time.perf_counter()
     out, out32 = decode_on_gpu(torch, p, lens, arena, q, 1.0)
     waited = time.perf_counter() - t0
-    monkeypatch.delenv("AKV_DEBUG_DROP_LAST")
+    akv.akv_decode_set_debug(withhold_last=0)
     assert np.all(np.isnan(out32)) and np.all(np.isnan(out))
     assert waited > 1.0, waited
     out, out32 = decode_on_gpu(torch, p, lens, arena, q, 1.0)

@@ -42,3 +42,33 @@ def test_two_gloo_ranks_max_time_and_disjoint_shards():
     mp.spawn(_rank_main, args=(world, _free_port(), out), nprocs=world, join=True)
     assert out[0] == out[1] == 2.0  # both ranks report the slowest rank's time
     assert out[2] != out[3]  # distinct per-rank inputs
+
+
+@pytest.mark.timeout(180)
+def test_bench_starts_n_ranks_itself():
+    """`bench.py --gpus 2` without a torch.distributed environment starts two ranks itself
+    (torch.distributed.run on 127.0.0.1); every rank reports through the process group
+    (gloo on a host without a GPU) and rank 0 prints them."""
+    import json
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = {k: v for k, v in os.environ.items() if k not in ("WORLD_SIZE", "RANK", "LOCAL_RANK", "MASTER_ADDR",
+                                                            "MASTER_PORT")}
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    r = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--gpus", "2", "--launch-check"],
+                       env=env, capture_output=True, text=True, timeout=170)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [json.loads(x) for x in r.stdout.splitlines() if x.startswith("{")]
+    assert len(lines) == 1, r.stdout
+    got = lines[0]
+    assert got["world_size"] == 2 and got["ranks"] == [0, 1] and got["distinct_processes"] == 2
+    assert got["backend"] == "gloo"
+
+
+def test_bench_refuses_a_rank_count_that_disagrees():
+    import argparse
+    import bench
+    os.environ.pop("WORLD_SIZE", None)
+    with pytest.raises(SystemExit):
+        bench.dist_setup(argparse.Namespace(gpus=2))

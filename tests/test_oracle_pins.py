@@ -102,7 +102,7 @@ def test_paper_worked_example():
     P = S - W
     assert 2 * H * P == int(g["token_sides"])
     # The printed N follows from Eq. 9 with the mean of the two residual costs
-    # c_K = D/4 + 4 and c_V = D/4 + 5 (reading recorded in the design doc) ...
+    # c_K = D/4 + 4 and c_V = D/4 + 5 (reading R11 of the byte accounting) ...
     b_res = (acc.paper_c_k(Dg) + acc.paper_c_v(Dg)) / 2
     N = acc.paper_n_residuals(g["theta"], m_full, m_base, b_res)
     assert N == int(g["n_residuals"])

@@ -41,6 +41,8 @@ def test_noalloc_encode_matches_workspace_encode():
 
 
 def test_noalloc_rejects_oversized_work():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
     p = akv.Params(batch=8, n_kv_heads=8, n_q_heads=32)
     with pytest.raises(akv.AkvError) as e:
         akv.akv_encode_noalloc(p, [131072] * 8, torch.empty((8, 8, 1, 128), dtype=torch.bfloat16, device="cuda"),
