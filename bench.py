@@ -240,13 +240,14 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
-TRAFFIC_PROFILES = {"8b-32k": "akv_decode_8b32k_ncu.md", "8b-128k": "akv_decode_8b128k_ncu.md"}
+TRAFFIC_PROFILES = {"8b-32k": "akv_decode_8b32k_ncu.md", "8b-128k": "akv_decode_8b128k_ncu.md",
+                    "70b-128k": "akv_decode_70b128k_ncu.md"}
 
 
 def kernel_traffic(workload: str):
     """DRAM bytes per decode launch from the committed ncu summary of this workload, if there is one
-    and it matches the current kernel source (the 8B-128K capture runs 2 of the 8 cycled layers,
-    same per-launch bytes)."""
+    and it matches the current kernel source (the 128K captures cycle fewer layers than the benchmark;
+    every launch reads one layer either way, so the bytes per launch are the same)."""
     src_hash = hashlib.sha256(open(DEC_KERNEL_SRC, "rb").read()).hexdigest()[:16]
     if workload not in TRAFFIC_PROFILES:
         return None
@@ -397,15 +398,17 @@ def run_akv(args, rank, world, local):
         with torch.cuda.graph(g, stream=stream):
             e2e_ops(i, torch.cuda.current_stream())
         e2e_graphs.append(g)
-    for g in e2e_graphs:  # warm-up
-        g.replay()
-    torch.cuda.synchronize()
-    dist_barrier(world)
-    t0 = time.perf_counter()
-    for g in e2e_graphs:
-        g.replay()
+    with torch.cuda.stream(stream):  # replays run on the current stream: make it the one waited on
+        for g in e2e_graphs:  # warm-up
+            g.replay()
         stream.synchronize()
-    e2e_sec = dist_max(time.perf_counter() - t0, world)
+    dist_barrier(world)
+    with torch.cuda.stream(stream):
+        t0 = time.perf_counter()
+        for g in e2e_graphs:
+            g.replay()
+            stream.synchronize()
+        e2e_sec = dist_max(time.perf_counter() - t0, world)
     with torch.cuda.stream(stream):
         t0 = time.perf_counter()
         for i in range(e2e_steps):
