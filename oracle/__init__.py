@@ -79,6 +79,15 @@ def lib():
             L.or_quantize_residual.argtypes = [vp, u64, ctypes.c_int, vp, vp, vp]
             L.or_arena_shape.restype = ctypes.c_int
             L.or_arena_shape.argtypes = [vp, u64, i32, vp]
+            L.or_exp_neg.restype = dbl
+            L.or_exp_neg.argtypes = [dbl]
+            L.or_selector_scores_unit.argtypes = [i32, i32, i32, i32, vp, vp, vp]
+            L.or_budget_n.restype = ctypes.c_int64
+            L.or_budget_n.argtypes = [dbl, i32, i32, i32, i32]
+            L.or_utilities_unit.argtypes = [ctypes.POINTER(_OrUnit), vp, vp, vp, i32, vp, vp]
+            L.or_encode_select_batch.restype = ctypes.c_int
+            L.or_encode_select_batch.argtypes = [vp, vp, vp, i32, i32, i32, i32, i32, ctypes.c_float, ctypes.c_float,
+                                                 i32, u64, u64, ctypes.c_int, vp]
             L.or_arena_unpack.restype = ctypes.c_int
             L.or_arena_unpack.argtypes = [vp, u64, i32, ctypes.POINTER(_OrUnit)]
             _lib = L
@@ -200,6 +209,76 @@ def encode(K: np.ndarray, V: np.ndarray, ctx_lens, n_kv_heads: int, f_a: float, 
     if rc != 0:
         raise RuntimeError("oracle encode failed")
     return units
+
+
+# ---- the paper's full selection (Algorithm 1; Section 3.2-3.4, Appendix A.2) ----------
+
+def exp_neg(x: float) -> float:
+    """e^x for x <= 0 by the oracle's Cody-Waite + Taylor evaluation."""
+    return float(lib().or_exp_neg(float(x)))
+
+
+def selector_scores(K: np.ndarray, Q: np.ndarray, W: int, kappa: int) -> np.ndarray:
+    """Appendix A.2 selector scores of positions [0, S - min(W, S)) of one unit:
+    K bf16 bits [S][128], Q bf16 bits [m][128] (the observation rows)."""
+    K = np.ascontiguousarray(K, dtype=np.uint16)
+    Q = np.ascontiguousarray(Q, dtype=np.uint16)
+    S, m = K.shape[0], Q.shape[0]
+    out = np.zeros(max(0, S - min(W, S)), np.float64)
+    lib().or_selector_scores_unit(S, W, m, kappa, _p(K), _p(Q), _p(out) if out.size else None)
+    return out
+
+
+def budget_n(theta: float, S: int, H: int, W: int, k: int) -> int:
+    """Eq. 9 residual count of one layer with the Appendix A.1 accounting."""
+    return int(lib().or_budget_n(float(theta), S, H, W, k))
+
+
+def utilities(unit: "Unit", K: np.ndarray, V: np.ndarray, Q: np.ndarray):
+    """Eq. 6 utilities (u^K, u^V) of every position of a unit given its anchors and
+    coefficients; anchors get -1."""
+    K = np.ascontiguousarray(K, dtype=np.uint16)
+    V = np.ascontiguousarray(V, dtype=np.uint16)
+    Q = np.ascontiguousarray(Q, dtype=np.uint16)
+    uk = np.zeros(unit.S, np.float64)
+    uv = np.zeros(unit.S, np.float64)
+    s = unit.c_struct()
+    lib().or_utilities_unit(ctypes.byref(s), _p(K), _p(V), _p(Q), Q.shape[0], _p(uk), _p(uv))
+    return uk, uv
+
+
+def encode_select(K: np.ndarray, V: np.ndarray, Q: np.ndarray, ctx_lens, n_kv_heads: int, f_a: float, W: int,
+                  theta: float, rho: float, kappa: int, seed: int, rot_seed: int, rotate: bool = True) -> list:
+    """Algorithm 1 with the paper's selection.  K, V bf16 bits [B][H][s_max][128];
+    Q bf16 bits [B][H][m][128], m = W G.  Returns B*H Units with per-unit residual counts."""
+    K = np.ascontiguousarray(K, dtype=np.uint16)
+    V = np.ascontiguousarray(V, dtype=np.uint16)
+    Q = np.ascontiguousarray(Q, dtype=np.uint16)
+    B, H, s_max, d = K.shape
+    m = Q.shape[2]
+    assert H == n_kv_heads and d == D and Q.shape[:2] == (B, H) and len(ctx_lens) == B
+    f32 = ctypes.c_float
+    units = []
+    for b in range(B):
+        S = int(ctx_lens[b])
+        k, _, _ = unit_shape(S, f_a, 0.0, 0.0, W)
+        N = budget_n(float(f32(theta).value), S, H, W, k)
+        cap_k, cap_v = min(N // 2, S - k), min(N - N // 2, S - k)
+        for h in range(H):
+            units.append(alloc_unit(S, k, cap_k, cap_v))
+    structs = (_OrUnit * len(units))(*[u.c_struct() for u in units])
+    rc = lib().or_encode_select_batch(_p(K), _p(V), _p(Q), s_max, B, H, m, W, theta, rho, kappa,
+                                      ctypes.c_uint64(seed), ctypes.c_uint64(rot_seed), int(bool(rotate)),
+                                      ctypes.cast(structs, ctypes.c_void_p))
+    if rc != 0:
+        raise RuntimeError("oracle select encode failed")
+    out = []
+    for u, s in zip(units, structs):
+        nk, nv = int(s.nk), int(s.nv)
+        out.append(Unit(u.S, u.k, nk, nv, u.anchor_k, u.anchor_v, u.anchor_pos, u.idx_k, u.gam_k, u.idx_v, u.gam_v,
+                        u.res_k[:nk].copy(), u.codes_k[:nk].copy(), u.scale_k[:nk].copy(), u.min_k[:nk].copy(),
+                        u.res_v[:nv].copy(), u.codes_v[:nv].copy(), u.scale_v[:nv].copy(), u.min_v[:nv].copy()))
+    return out
 
 
 def attend(units, q: np.ndarray, G: int, sm_scale: float, rot_seed: int, rotate: bool = True, sel=None) -> np.ndarray:

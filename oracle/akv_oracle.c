@@ -14,6 +14,13 @@
  *             A.1 Eq. 12 (randomized Hadamard rotation) and a 4-level
  *             2-bit quantizer with per-token fp16 scale and min; residual
  *             slots ranked by residual norm (Section 4.3, variant (ii)).
+ *   encode_select : Algorithm 1 with the paper's full selection: the last W
+ *             positions, a share rho of the other anchors by the selector
+ *             score of Appendix A.2 (observation queries' attention, average
+ *             pooled over kappa positions), the rest sampled uniformly; the
+ *             output-aware utilities of Eq. 6; the layer budget of Eq. 9
+ *             (Appendix A.1 accounting) split floor(N/2) keys, the rest
+ *             values, each side's top-N pooled over the layer's KV heads.
  *   attend  : Eq. 3 reconstruction of every key and value, then Eq. 4
  *             softmax attention, all in fp64, one token at a time.
  *   attend_factorized : the same attention regrouped by anchor (anchor
@@ -295,7 +302,7 @@ static void or_encode_side(int32_t S, int32_t k, int32_t nres, const uint16_t* X
   /* residual slots: the nres largest energies among non-anchors */
   qsort(cand, (size_t)ncand, sizeof(or_errpos), cmp_err_desc);
   for (int32_t t = 0; t < nres; ++t) res[t] = cand[t].pos;
-  qsort(res, (size_t)nres, sizeof(int32_t), cmp_i32);
+  if (nres > 0) qsort(res, (size_t)nres, sizeof(int32_t), cmp_i32);
   for (int32_t t = 0; t < nres; ++t) {
     int32_t i = res[t];
     const uint16_t* x = X + (size_t)i * OR_D;
@@ -484,6 +491,363 @@ void or_attend_unit(const or_unit* u, const uint16_t* q, int32_t G, double sm_sc
   free(logit);
   free(slot_k);
   free(slot_v);
+}
+
+/* ------------------------------------------------------------------------ */
+/* The paper's full selection (Algorithm 1): anchors scored by the          */
+/* observation queries (Section 3.2, Appendix A.2), output-aware residual   */
+/* utilities (Section 3.3, Eq. 6), the byte budget of Eq. 9 pooled over a   */
+/* layer's KV heads (Section 3.4).                                           */
+/* ------------------------------------------------------------------------ */
+
+/* e^x for x <= 0 by the Cody-Waite argument reduction and a Taylor series
+ * (Cody and Waite, "Software Manual for the Elementary Functions", 1980):
+ * n = rint(x / ln 2), r = (x - n c1) - n c2 with c1 + c2 = ln 2 (c1 holding
+ * the leading 32 bits, so n c1 is exact), then e^r = sum_{j<=22} r^j / j!
+ * by Horner's rule, then the factor 2^n.  Every step is one separately
+ * rounded IEEE operation in a fixed order, so any implementation of the same
+ * steps gives the same bits; its error is about 1 ulp (pinned against libm).
+ * Arguments below -700 give 0, so the scaling by 2^n never leaves the normal
+ * range (there it is exact). */
+double or_exp_neg(double x) {
+  if (!(x >= -700.0)) return 0.0;
+  const double c1 = 0.693147180559890330187045037746429443359375; /* 2^-32 grid */
+  const double c2 = 5.4979230187083711552420206887987e-14;
+  double n = rint(x / 0.6931471805599453094172321);
+  double r = (x - n * c1) - n * c2;
+  double y = 1.0;
+  for (int j = 22; j >= 1; --j) y = 1.0 + (r / (double)j) * y;
+  return ldexp(y, (int)n);
+}
+
+/* Exact attention of m query rows over the dense keys of one unit (Eq. 4,
+ * logits q.K_t / sqrt(D), softmax over all S positions): alpha [m][S].
+ * Sums run in position order. */
+static void or_obs_alpha(int32_t S, int32_t m, const uint16_t* K, const uint16_t* Q, double* alpha) {
+  const double inv = 1.0 / sqrt((double)OR_D);
+  double qd[OR_D];
+  for (int32_t w = 0; w < m; ++w) {
+    for (int j = 0; j < OR_D; ++j) qd[j] = or_bf16_to_double(Q[(size_t)w * OR_D + j]);
+    double* a = alpha + (size_t)w * S;
+    double mx = -INFINITY;
+    for (int32_t t = 0; t < S; ++t) {
+      double d = 0.0;
+      for (int j = 0; j < OR_D; ++j) d = d + qd[j] * or_bf16_to_double(K[(size_t)t * OR_D + j]);
+      a[t] = d * inv;
+      if (a[t] > mx) mx = a[t];
+    }
+    double den = 0.0;
+    for (int32_t t = 0; t < S; ++t) {
+      a[t] = or_exp_neg(a[t] - mx);
+      den = den + a[t];
+    }
+    for (int32_t t = 0; t < S; ++t) a[t] = a[t] / den;
+  }
+}
+
+/* Appendix A.2 selector score of the candidate positions t in [0, P), P = S - W:
+ * the m observation rows' attention averaged over the rows, then average
+ * pooling of odd width kappa centred on t, zero outside [0, P), divided by kappa. */
+void or_selector_scores(int32_t S, int32_t P, int32_t m, int32_t kappa, const double* alpha, double* score) {
+  double* mean = (double*)malloc(sizeof(double) * (size_t)(P > 0 ? P : 1));
+  for (int32_t t = 0; t < P; ++t) {
+    double acc = 0.0;
+    for (int32_t w = 0; w < m; ++w) acc = acc + alpha[(size_t)w * S + t];
+    mean[t] = acc / (double)m;
+  }
+  int32_t h = kappa / 2;
+  for (int32_t t = 0; t < P; ++t) {
+    double acc = 0.0;
+    for (int32_t j = t - h; j <= t + h; ++j)
+      if (j >= 0 && j < P) acc = acc + mean[j];
+    score[t] = acc / (double)kappa;
+  }
+  free(mean);
+}
+
+/* Exported for the pins: the selector scores of one unit from its keys and m observation rows. */
+void or_selector_scores_unit(int32_t S, int32_t W, int32_t m, int32_t kappa, const uint16_t* K, const uint16_t* Q,
+                             double* score) {
+  double* alpha = (double*)malloc(sizeof(double) * (size_t)m * (size_t)S + 1);
+  or_obs_alpha(S, m, K, Q, alpha);
+  int32_t w = W < S ? W : S;
+  or_selector_scores(S, S - w, m, kappa, alpha, score);
+  free(alpha);
+}
+
+typedef struct {
+  double u;
+  int32_t h, pos;
+} or_util;
+
+/* higher utility first; equal utilities: lower head, then lower position */
+static int cmp_util_desc(const void* a, const void* b) {
+  const or_util* x = (const or_util*)a;
+  const or_util* y = (const or_util*)b;
+  if (x->u > y->u) return -1;
+  if (x->u < y->u) return 1;
+  if (x->h != y->h) return (x->h < y->h) ? -1 : 1;
+  return (x->pos < y->pos) ? -1 : (x->pos > y->pos);
+}
+
+/* Eq. 11 fixed bytes M_base and Eq. 9 residual count N of one layer of H KV
+ * heads at context S (Appendix A.1 accounting: b_a = b_gamma = 2, residual
+ * cost b_res = (c_K + c_V) / 2 with c_K = D/4 + 4 and c_V = D/4 + 5). */
+int64_t or_budget_n(double theta, int32_t S, int32_t H, int32_t W, int32_t k) {
+  int32_t w = W < S ? W : S;
+  int64_t P = (int64_t)S - w;
+  int64_t words = (P + 63) / 64;
+  double m_full = 4.0 * (double)S * (double)H * (double)OR_D;
+  double m_base = (double)H * (4.0 * k * OR_D + 8.0 * (k - w) + 2.0 * (double)P * (2 + 2)) + 24.0 * H * words +
+                  8.0 * (H + 1) + 4.0 * (double)P;
+  double b_res = ((OR_D / 4 + 4) + (OR_D / 4 + 5)) / 2.0;
+  double n = floor((theta * m_full - m_base) / b_res);
+  return n > 0.0 ? (int64_t)n : 0;
+}
+
+/*
+ * Algorithm 1 for one request: K, V bf16 [H][s_max][128], Q the observation
+ * rows bf16 [H][m][128] (m = W G: the last W positions' queries of the G query
+ * heads of each KV head).  units[h] arrive with S and k set and arrays sized
+ * for at most min(N_side, S - k) residuals per side; nk and nv are set here.
+ */
+int or_encode_select_request(const uint16_t* K, const uint16_t* V, const uint16_t* Q, int32_t s_max, int32_t H, int32_t m,
+                             int32_t W, float theta, float rho, int32_t kappa, int32_t b, uint64_t seed,
+                             uint64_t rot_seed, int rotate, or_unit* units) {
+  int32_t S = units[0].S, k = units[0].k;
+  int32_t w = W < S ? W : S;
+  int32_t rest = k - w;
+  int32_t n_s = (m > 0 && rest > 0) ? (int32_t)floor((double)rho * (double)rest) : 0;
+  double sv[OR_D];
+  or_signs(rot_seed, sv);
+  double* alpha = (double*)malloc(sizeof(double) * (size_t)(m > 0 ? m : 1) * (size_t)S);
+  double* y = (double*)malloc(sizeof(double) * (size_t)(m > 0 ? m : 1) * OR_D);
+  or_util* cand[2];
+  int64_t ncand[2] = {0, 0};
+  cand[0] = (or_util*)malloc(sizeof(or_util) * (size_t)H * (size_t)S);
+  cand[1] = (or_util*)malloc(sizeof(or_util) * (size_t)H * (size_t)S);
+  int32_t** slot_of = (int32_t**)malloc(sizeof(int32_t*) * (size_t)H);
+  for (int32_t h = 0; h < H; ++h) {
+    or_unit* u = &units[h];
+    const uint16_t* Kh = K + (size_t)h * s_max * OR_D;
+    const uint16_t* Vh = V + (size_t)h * s_max * OR_D;
+    const uint16_t* Qh = Q + (size_t)h * (size_t)(m > 0 ? m : 0) * OR_D;
+    if (m > 0) or_obs_alpha(S, m, Kh, Qh, alpha);
+    /* anchor set: last w, top n_s by the selector score, the rest by the sampling hash */
+    char* is_anchor = (char*)calloc((size_t)S, 1);
+    int32_t P = S - w;
+    if (rest > 0) {
+      if (n_s > 0) {
+        double* score = (double*)malloc(sizeof(double) * (size_t)P);
+        or_selector_scores(S, P, m, kappa, alpha, score);
+        or_util* sc = (or_util*)malloc(sizeof(or_util) * (size_t)P);
+        for (int32_t t = 0; t < P; ++t) {
+          sc[t].u = score[t];
+          sc[t].h = 0;
+          sc[t].pos = t;
+        }
+        qsort(sc, (size_t)P, sizeof(or_util), cmp_util_desc);
+        for (int32_t t = 0; t < n_s; ++t) is_anchor[sc[t].pos] = 1;
+        free(sc);
+        free(score);
+      }
+      or_keypos* kp = (or_keypos*)malloc(sizeof(or_keypos) * (size_t)P);
+      uint64_t base = seed ^ ((uint64_t)b << 40) ^ ((uint64_t)h << 32);
+      int32_t np = 0;
+      for (int32_t p = 0; p < P; ++p) {
+        if (is_anchor[p]) continue;
+        kp[np].key = or_splitmix64(base ^ (uint64_t)p);
+        kp[np].pos = p;
+        ++np;
+      }
+      qsort(kp, (size_t)np, sizeof(or_keypos), cmp_key_asc);
+      for (int32_t t = 0; t < rest - n_s; ++t) is_anchor[kp[t].pos] = 1;
+      free(kp);
+    }
+    for (int32_t p = S - w; p < S; ++p) is_anchor[p] = 1;
+    slot_of[h] = (int32_t*)malloc(sizeof(int32_t) * (size_t)S);
+    int32_t t = 0;
+    for (int32_t p = 0; p < S; ++p) {
+      if (is_anchor[p]) {
+        u->anchor_pos[t] = p;
+        slot_of[h][p] = t++;
+      } else {
+        slot_of[h][p] = -1;
+      }
+    }
+    free(is_anchor);
+    if (t != k) return -1;
+    for (int32_t a = 0; a < k; ++a) {
+      memcpy(u->anchor_k + (size_t)a * OR_D, Kh + (size_t)u->anchor_pos[a] * OR_D, OR_D * 2);
+      memcpy(u->anchor_v + (size_t)a * OR_D, Vh + (size_t)u->anchor_pos[a] * OR_D, OR_D * 2);
+    }
+    /* assignment and coefficients (Eq. 1, Eq. 2), no residual slots yet */
+    or_encode_side(S, k, 0, Kh, u->anchor_pos, slot_of[h], sv, rotate, u->idx_k, u->gam_k, NULL, NULL, NULL, NULL);
+    or_encode_side(S, k, 0, Vh, u->anchor_pos, slot_of[h], sv, rotate, u->idx_v, u->gam_v, NULL, NULL, NULL, NULL);
+    /* exact outputs y^(w) of the observation rows (Eq. 4) */
+    for (int32_t ww = 0; ww < m; ++ww)
+      for (int j = 0; j < OR_D; ++j) {
+        double acc = 0.0;
+        for (int32_t p = 0; p < S; ++p)
+          acc = acc + alpha[(size_t)ww * S + p] * or_bf16_to_double(Vh[(size_t)p * OR_D + j]);
+        y[(size_t)ww * OR_D + j] = acc;
+      }
+    /* Eq. 6 utilities of the non-anchor positions, per side */
+    for (int32_t p = 0; p < S; ++p) {
+      if (slot_of[h][p] >= 0) continue;
+      double rk[OR_D], rv[OR_D], vt[OR_D];
+      double gk = or_fp16_to_double(u->gam_k[p]), gv = or_fp16_to_double(u->gam_v[p]);
+      const uint16_t* xk = Kh + (size_t)p * OR_D;
+      const uint16_t* xv = Vh + (size_t)p * OR_D;
+      const uint16_t* ak = u->anchor_k + (size_t)u->idx_k[p] * OR_D;
+      const uint16_t* av = u->anchor_v + (size_t)u->idx_v[p] * OR_D;
+      double ev = 0.0;
+      for (int j = 0; j < OR_D; ++j) {
+        rk[j] = or_bf16_to_double(xk[j]) - gk * or_bf16_to_double(ak[j]);
+        rv[j] = or_bf16_to_double(xv[j]) - gv * or_bf16_to_double(av[j]);
+        vt[j] = or_bf16_to_double(xv[j]);
+        ev = ev + rv[j] * rv[j];
+      }
+      double uk = 0.0, uv = 0.0;
+      for (int32_t ww = 0; ww < m; ++ww) {
+        double a = alpha[(size_t)ww * S + p];
+        double a2 = a * a;
+        double d = 0.0, dv = 0.0;
+        for (int j = 0; j < OR_D; ++j) {
+          d = d + or_bf16_to_double(Qh[(size_t)ww * OR_D + j]) * rk[j];
+          double c = vt[j] - y[(size_t)ww * OR_D + j];
+          dv = dv + c * c;
+        }
+        uk = uk + a2 * (d * d / (double)OR_D) * dv;
+        uv = uv + a2 * ev;
+      }
+      if (m > 0) {
+        uk = uk / (double)m;
+        uv = uv / (double)m;
+      }
+      cand[0][ncand[0]].u = uk;
+      cand[0][ncand[0]].h = h;
+      cand[0][ncand[0]].pos = p;
+      ++ncand[0];
+      cand[1][ncand[1]].u = uv;
+      cand[1][ncand[1]].h = h;
+      cand[1][ncand[1]].pos = p;
+      ++ncand[1];
+    }
+  }
+  /* Eq. 9 budget, keys floor(N / 2), values the rest; top N per side pooled over the heads */
+  int64_t N = or_budget_n((double)theta, S, H, W, k);
+  int64_t nside[2] = {N / 2, N - N / 2};
+  for (int side = 0; side < 2; ++side) {
+    if (nside[side] > ncand[side]) nside[side] = ncand[side];
+    qsort(cand[side], (size_t)ncand[side], sizeof(or_util), cmp_util_desc);
+    for (int32_t h = 0; h < H; ++h) {
+      if (side == 0) units[h].nk = 0;
+      else units[h].nv = 0;
+    }
+    for (int64_t i = 0; i < nside[side]; ++i) {
+      or_unit* u = &units[cand[side][i].h];
+      if (side == 0) u->res_k[u->nk++] = cand[side][i].pos;
+      else u->res_v[u->nv++] = cand[side][i].pos;
+    }
+  }
+  /* rotate and quantize the chosen residuals (Appendix A.1), positions ascending */
+  for (int32_t h = 0; h < H; ++h) {
+    or_unit* u = &units[h];
+    const uint16_t* Kh = K + (size_t)h * s_max * OR_D;
+    const uint16_t* Vh = V + (size_t)h * s_max * OR_D;
+    if (u->nk > 0) qsort(u->res_k, (size_t)u->nk, sizeof(int32_t), cmp_i32);
+    if (u->nv > 0) qsort(u->res_v, (size_t)u->nv, sizeof(int32_t), cmp_i32);
+    for (int side = 0; side < 2; ++side) {
+      int32_t n = side ? u->nv : u->nk;
+      const int32_t* res = side ? u->res_v : u->res_k;
+      const uint16_t* X = side ? Vh : Kh;
+      const uint16_t* A = side ? u->anchor_v : u->anchor_k;
+      const uint16_t* idx = side ? u->idx_v : u->idx_k;
+      const uint16_t* gam = side ? u->gam_v : u->gam_k;
+      for (int32_t i = 0; i < n; ++i) {
+        double r[OR_D];
+        int32_t p = res[i];
+        double g = or_fp16_to_double(gam[p]);
+        for (int j = 0; j < OR_D; ++j)
+          r[j] = or_bf16_to_double(X[(size_t)p * OR_D + j]) - g * or_bf16_to_double(A[(size_t)idx[p] * OR_D + j]);
+        if (side == 0) or_quantize(r, sv, rotate, u->codes_k + (size_t)i * 32, &u->scale_k[i], &u->min_k[i]);
+        else or_quantize(r, sv, rotate, u->codes_v + (size_t)i * 32, &u->scale_v[i], &u->min_v[i]);
+      }
+    }
+    free(slot_of[h]);
+  }
+  free(slot_of);
+  free(cand[0]);
+  free(cand[1]);
+  free(y);
+  free(alpha);
+  return 0;
+}
+
+/* Exported for the pins: Eq. 6 utilities of every position of one unit with
+ * given anchors and coefficients (anchors get -1).  K, V bf16 [S][128],
+ * Q bf16 [m][128]; uk, uv [S]. */
+void or_utilities_unit(const or_unit* u, const uint16_t* K, const uint16_t* V, const uint16_t* Q, int32_t m,
+                       double* uk, double* uv) {
+  int32_t S = u->S;
+  double* alpha = (double*)malloc(sizeof(double) * (size_t)(m > 0 ? m : 1) * (size_t)S);
+  double* y = (double*)malloc(sizeof(double) * (size_t)(m > 0 ? m : 1) * OR_D);
+  if (m > 0) or_obs_alpha(S, m, K, Q, alpha);
+  for (int32_t ww = 0; ww < m; ++ww)
+    for (int j = 0; j < OR_D; ++j) {
+      double acc = 0.0;
+      for (int32_t p = 0; p < S; ++p) acc = acc + alpha[(size_t)ww * S + p] * or_bf16_to_double(V[(size_t)p * OR_D + j]);
+      y[(size_t)ww * OR_D + j] = acc;
+    }
+  char* is_anchor = (char*)calloc((size_t)S, 1);
+  for (int32_t a = 0; a < u->k; ++a) is_anchor[u->anchor_pos[a]] = 1;
+  for (int32_t p = 0; p < S; ++p) {
+    if (is_anchor[p]) {
+      uk[p] = uv[p] = -1.0;
+      continue;
+    }
+    double rk[OR_D], ev = 0.0;
+    double gk = or_fp16_to_double(u->gam_k[p]), gv = or_fp16_to_double(u->gam_v[p]);
+    for (int j = 0; j < OR_D; ++j) {
+      rk[j] = or_bf16_to_double(K[(size_t)p * OR_D + j]) - gk * or_bf16_to_double(u->anchor_k[(size_t)u->idx_k[p] * OR_D + j]);
+      double rv = or_bf16_to_double(V[(size_t)p * OR_D + j]) - gv * or_bf16_to_double(u->anchor_v[(size_t)u->idx_v[p] * OR_D + j]);
+      ev = ev + rv * rv;
+    }
+    double a_k = 0.0, a_v = 0.0;
+    for (int32_t ww = 0; ww < m; ++ww) {
+      double a = alpha[(size_t)ww * S + p];
+      double d = 0.0, dv = 0.0;
+      for (int j = 0; j < OR_D; ++j) {
+        d = d + or_bf16_to_double(Q[(size_t)ww * OR_D + j]) * rk[j];
+        double c = or_bf16_to_double(V[(size_t)p * OR_D + j]) - y[(size_t)ww * OR_D + j];
+        dv = dv + c * c;
+      }
+      a_k = a_k + (a * a) * (d * d / (double)OR_D) * dv;
+      a_v = a_v + (a * a) * ev;
+    }
+    uk[p] = m > 0 ? a_k / (double)m : 0.0;
+    uv[p] = m > 0 ? a_v / (double)m : 0.0;
+  }
+  free(is_anchor);
+  free(y);
+  free(alpha);
+}
+
+/* Batched over requests: K, V [B][H][s_max][128], Q [B][H][m][128]; units [B*H]. */
+int or_encode_select_batch(const uint16_t* K, const uint16_t* V, const uint16_t* Q, int32_t s_max, int32_t B, int32_t H,
+                           int32_t m, int32_t W, float theta, float rho, int32_t kappa, uint64_t seed,
+                           uint64_t rot_seed, int rotate, or_unit* units) {
+  int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(| : bad)
+  for (int32_t b = 0; b < B; ++b) {
+    size_t off = (size_t)b * H * (size_t)s_max * OR_D;
+    size_t qoff = (size_t)b * H * (size_t)m * OR_D;
+    if (or_encode_select_request(K + off, V + off, Q + qoff, s_max, H, m, W, theta, rho, kappa, b, seed, rot_seed,
+                                 rotate, units + (size_t)b * H) != 0)
+      bad |= 1;
+  }
+  return bad ? -1 : 0;
 }
 
 /* Batched definitional attention: q bf16 [n_units][G][128] (unit u = b*H + h
