@@ -15,6 +15,10 @@ clustered_kv  Keys and values of one (request, KV head): 64 centres
               channels by 8 (outlier channels).  Drawn in fp64, rounded to
               bf16 (round-to-nearest-even, direct from fp64).
 queries       q ~ N(0, I) / sqrt(128), rounded to bf16.
+observation_queries  the observation rows of the full selection (the queries of the last
+              W positions of the G query heads of each KV head; Section 3.2): each row
+              is 0.25 x one of the unit's keys, picked uniformly, plus N(0, I) noise, so
+              that its attention concentrates on that key's cluster, rounded to bf16.
 seeded_cache  A compressed cache drawn directly: the last W positions plus a
               uniform sample are anchors, anchor rows from clustered_kv,
               non-anchor indices uniform over the anchors, gamma ~ N(1, 0.1)
@@ -92,6 +96,19 @@ def queries(n_rows: int, seed: int, step: int = 0) -> np.ndarray:
     """n_rows query vectors, uint16 bf16 bits [n_rows][128]."""
     rng = _rng(seed, step, 0x5159)
     return bf16_bits(rng.standard_normal((n_rows, D)) / np.sqrt(D))
+
+
+def observation_queries(K: np.ndarray, ctx_lens, m: int, seed: int) -> np.ndarray:
+    """m observation rows per (request, KV head): uint16 bf16 bits [B][H][m][128]; K is the
+    uint16 [B][H][s_max][128] of clustered_batch."""
+    B, H = K.shape[:2]
+    out = np.zeros((B, H, m, D), np.uint16)
+    for b in range(B):
+        for h in range(H):
+            rng = _rng(seed, b * H + h, 0x0B5E)
+            t = rng.integers(0, int(ctx_lens[b]), size=m)
+            out[b, h] = bf16_bits(0.25 * bf16_to_f64(K[b, h, t]) + rng.standard_normal((m, D)))
+    return out
 
 
 def ragged_lens(B: int, lo: int, hi: int, seed: int) -> np.ndarray:

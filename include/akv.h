@@ -262,6 +262,70 @@ akv_status akv_encode(const akv_params* p, const int32_t* ctx_lens_host, const v
 akv_status akv_encode_noalloc(const akv_params* p, const int32_t* ctx_lens_host, const void* K, const void* V,
                               int32_t s_max, void* arena, size_t arena_bytes, akv_stream_t stream);
 
+/* ---- Encode with the paper's full selection ------------------------------ */
+
+/*
+ * The paper's full selection (Algorithm 1; Section 3.2 "Anchor selection",
+ * Appendix A.2; Section 3.3 Eq. 6; Section 3.4 Eq. 9):
+ *  - anchors: the last min(W, S) positions; floor(rho (k - W)) positions of
+ *    [0, S - W) with the highest selector score (the observation rows'
+ *    softmax attention, q.K / sqrt(D) over all S positions, averaged over the
+ *    m rows and average-pooled over kappa positions centred on each one, zero
+ *    outside [0, S - W), divided by kappa; ties: lower position); the rest
+ *    sampled uniformly as in akv_encode (smallest SplitMix64 hashes among the
+ *    positions not yet chosen);
+ *  - residual budget of each request's layer: N of Eq. 9 (Appendix A.1
+ *    accounting: anchors, metadata, 36.5 bytes per residual), keys floor(N/2),
+ *    values the rest;
+ *  - each side's N slots go to the positions with the highest utility of
+ *    Eq. 6 over all KV heads of the request (ties: lower head, then lower
+ *    position), so heads receive different counts:
+ *      u^K_t = 1/m sum_w alpha_wt^2 (q_w . r^K_t)^2 / D |V_t - y_w|^2,
+ *      u^V_t = 1/m sum_w alpha_wt^2 |r^V_t|^2,
+ *    with alpha_w, y_w the exact attention and output of observation row w.
+ * The anchor budget k comes from akv_params.anchor_frac and window as for
+ * akv_encode; res_frac_k and res_frac_v are not used.  Every decision is taken
+ * in fp64 with a fixed operation order (the exponential is evaluated by a
+ * Cody-Waite reduction and a Taylor series), so the packed bytes are
+ * reproducible bit for bit.
+ */
+typedef struct akv_select_params {
+  float theta;      /* retained fraction of the bf16 cache, in (0, 1] (Eq. 9) */
+  float rho;        /* share of the k - W non-window anchors picked by score, in [0, 1] (0.7) */
+  int32_t kappa;    /* pooling width of the selector score, odd, 1..255 (7) */
+  int32_t reserved; /* must be 0 */
+} akv_select_params;
+
+/*
+ * Arena and workspace bytes of akv_encode_select.  The arena reserves, per
+ * unit and side, room for min(N_side, S - k) residual records (the most the
+ * pooled budget can give one head); the workspace adds the observation rows'
+ * attention (8 m S bytes per unit).  m = W * G.
+ */
+akv_status akv_cache_size_select(const akv_params* p, const akv_select_params* sel, const int32_t* ctx_lens_host,
+                                 size_t* arena_bytes, size_t* encode_ws_bytes);
+
+/*
+ * Compresses K, V with the full selection.
+ *   K, V  : device bf16 [B][H][s_max][128], as for akv_encode
+ *   Q     : device bf16 [B][H][m][128], m = W * G: the observation rows of each
+ *           KV head, i.e. the queries of the last W positions of the G query
+ *           heads that read it (W >= 1)
+ *   arena, ws : sizes from akv_cache_size_select, 256-byte aligned
+ * The descriptors of the written arena hold each unit's chosen residual
+ * counts; akv_decode_attn reads such an arena like any other.  Its launch
+ * planner stages, per tile, the residual records that the akv_params
+ * fractions it is given suggest: pass fractions near the densities the
+ * selection chose (at most N / (2 H S) per side keeps the size check within
+ * this arena) for speed; records beyond the staged count are read from
+ * global memory, so any such fractions, 0 included, give the same results.
+ * Errors: as for akv_encode; AKV_ERR_INVALID for bad select parameters or
+ * W = 0 (no observation rows).
+ */
+akv_status akv_encode_select(const akv_params* p, const akv_select_params* sel, const int32_t* ctx_lens_host,
+                             const void* K, const void* V, const void* Q, int32_t s_max, void* arena, size_t arena_bytes,
+                             void* ws, size_t ws_bytes, akv_stream_t stream);
+
 /* ---- Host packer -------------------------------------------------------- */
 
 /*

@@ -606,141 +606,151 @@ int64_t or_budget_n(double theta, int32_t S, int32_t H, int32_t W, int32_t k) {
 }
 
 /*
- * Algorithm 1 for one request: K, V bf16 [H][s_max][128], Q the observation
- * rows bf16 [H][m][128] (m = W G: the last W positions' queries of the G query
- * heads of each KV head).  units[h] arrive with S and k set and arrays sized
- * for at most min(N_side, S - k) residuals per side; nk and nv are set here.
+ * Algorithm 1, per KV head: anchor set, assignment and coefficients, and the
+ * Eq. 6 utilities of its non-anchor positions.  K, V bf16 [S][128] (rows of
+ * one head, stride s_max), Q its m observation rows; u arrives with S and k
+ * set.  cand[side] receive one entry per non-anchor position (*ncand of them).
  */
-int or_encode_select_request(const uint16_t* K, const uint16_t* V, const uint16_t* Q, int32_t s_max, int32_t H, int32_t m,
-                             int32_t W, float theta, float rho, int32_t kappa, int32_t b, uint64_t seed,
-                             uint64_t rot_seed, int rotate, or_unit* units) {
-  int32_t S = units[0].S, k = units[0].k;
+static int or_select_head(const uint16_t* Kh, const uint16_t* Vh, const uint16_t* Qh, int32_t m, int32_t W, float rho,
+                          int32_t kappa, int32_t b, int32_t h, uint64_t seed, const double* sv, int rotate, or_unit* u,
+                          or_util* cand_k, or_util* cand_v, int64_t* ncand) {
+  int32_t S = u->S, k = u->k;
   int32_t w = W < S ? W : S;
   int32_t rest = k - w;
   int32_t n_s = (m > 0 && rest > 0) ? (int32_t)floor((double)rho * (double)rest) : 0;
-  double sv[OR_D];
-  or_signs(rot_seed, sv);
   double* alpha = (double*)malloc(sizeof(double) * (size_t)(m > 0 ? m : 1) * (size_t)S);
   double* y = (double*)malloc(sizeof(double) * (size_t)(m > 0 ? m : 1) * OR_D);
-  or_util* cand[2];
-  int64_t ncand[2] = {0, 0};
-  cand[0] = (or_util*)malloc(sizeof(or_util) * (size_t)H * (size_t)S);
-  cand[1] = (or_util*)malloc(sizeof(or_util) * (size_t)H * (size_t)S);
-  int32_t** slot_of = (int32_t**)malloc(sizeof(int32_t*) * (size_t)H);
-  for (int32_t h = 0; h < H; ++h) {
-    or_unit* u = &units[h];
-    const uint16_t* Kh = K + (size_t)h * s_max * OR_D;
-    const uint16_t* Vh = V + (size_t)h * s_max * OR_D;
-    const uint16_t* Qh = Q + (size_t)h * (size_t)(m > 0 ? m : 0) * OR_D;
-    if (m > 0) or_obs_alpha(S, m, Kh, Qh, alpha);
-    /* anchor set: last w, top n_s by the selector score, the rest by the sampling hash */
-    char* is_anchor = (char*)calloc((size_t)S, 1);
-    int32_t P = S - w;
-    if (rest > 0) {
-      if (n_s > 0) {
-        double* score = (double*)malloc(sizeof(double) * (size_t)P);
-        or_selector_scores(S, P, m, kappa, alpha, score);
-        or_util* sc = (or_util*)malloc(sizeof(or_util) * (size_t)P);
-        for (int32_t t = 0; t < P; ++t) {
-          sc[t].u = score[t];
-          sc[t].h = 0;
-          sc[t].pos = t;
-        }
-        qsort(sc, (size_t)P, sizeof(or_util), cmp_util_desc);
-        for (int32_t t = 0; t < n_s; ++t) is_anchor[sc[t].pos] = 1;
-        free(sc);
-        free(score);
+  if (m > 0) or_obs_alpha(S, m, Kh, Qh, alpha);
+  /* anchor set: last w, top n_s by the selector score, the rest by the sampling hash */
+  char* is_anchor = (char*)calloc((size_t)S, 1);
+  int32_t P = S - w;
+  if (rest > 0) {
+    if (n_s > 0) {
+      double* score = (double*)malloc(sizeof(double) * (size_t)P);
+      or_selector_scores(S, P, m, kappa, alpha, score);
+      or_util* sc = (or_util*)malloc(sizeof(or_util) * (size_t)P);
+      for (int32_t t = 0; t < P; ++t) {
+        sc[t].u = score[t];
+        sc[t].h = 0;
+        sc[t].pos = t;
       }
-      or_keypos* kp = (or_keypos*)malloc(sizeof(or_keypos) * (size_t)P);
-      uint64_t base = seed ^ ((uint64_t)b << 40) ^ ((uint64_t)h << 32);
-      int32_t np = 0;
-      for (int32_t p = 0; p < P; ++p) {
-        if (is_anchor[p]) continue;
-        kp[np].key = or_splitmix64(base ^ (uint64_t)p);
-        kp[np].pos = p;
-        ++np;
-      }
-      qsort(kp, (size_t)np, sizeof(or_keypos), cmp_key_asc);
-      for (int32_t t = 0; t < rest - n_s; ++t) is_anchor[kp[t].pos] = 1;
-      free(kp);
+      qsort(sc, (size_t)P, sizeof(or_util), cmp_util_desc);
+      for (int32_t t = 0; t < n_s; ++t) is_anchor[sc[t].pos] = 1;
+      free(sc);
+      free(score);
     }
-    for (int32_t p = S - w; p < S; ++p) is_anchor[p] = 1;
-    slot_of[h] = (int32_t*)malloc(sizeof(int32_t) * (size_t)S);
-    int32_t t = 0;
-    for (int32_t p = 0; p < S; ++p) {
-      if (is_anchor[p]) {
-        u->anchor_pos[t] = p;
-        slot_of[h][p] = t++;
-      } else {
-        slot_of[h][p] = -1;
-      }
+    or_keypos* kp = (or_keypos*)malloc(sizeof(or_keypos) * (size_t)P);
+    uint64_t base = seed ^ ((uint64_t)b << 40) ^ ((uint64_t)h << 32);
+    int32_t np = 0;
+    for (int32_t p = 0; p < P; ++p) {
+      if (is_anchor[p]) continue;
+      kp[np].key = or_splitmix64(base ^ (uint64_t)p);
+      kp[np].pos = p;
+      ++np;
     }
-    free(is_anchor);
-    if (t != k) return -1;
-    for (int32_t a = 0; a < k; ++a) {
-      memcpy(u->anchor_k + (size_t)a * OR_D, Kh + (size_t)u->anchor_pos[a] * OR_D, OR_D * 2);
-      memcpy(u->anchor_v + (size_t)a * OR_D, Vh + (size_t)u->anchor_pos[a] * OR_D, OR_D * 2);
-    }
-    /* assignment and coefficients (Eq. 1, Eq. 2), no residual slots yet */
-    or_encode_side(S, k, 0, Kh, u->anchor_pos, slot_of[h], sv, rotate, u->idx_k, u->gam_k, NULL, NULL, NULL, NULL);
-    or_encode_side(S, k, 0, Vh, u->anchor_pos, slot_of[h], sv, rotate, u->idx_v, u->gam_v, NULL, NULL, NULL, NULL);
-    /* exact outputs y^(w) of the observation rows (Eq. 4) */
-    for (int32_t ww = 0; ww < m; ++ww)
-      for (int j = 0; j < OR_D; ++j) {
-        double acc = 0.0;
-        for (int32_t p = 0; p < S; ++p)
-          acc = acc + alpha[(size_t)ww * S + p] * or_bf16_to_double(Vh[(size_t)p * OR_D + j]);
-        y[(size_t)ww * OR_D + j] = acc;
-      }
-    /* Eq. 6 utilities of the non-anchor positions, per side */
-    for (int32_t p = 0; p < S; ++p) {
-      if (slot_of[h][p] >= 0) continue;
-      double rk[OR_D], rv[OR_D], vt[OR_D];
-      double gk = or_fp16_to_double(u->gam_k[p]), gv = or_fp16_to_double(u->gam_v[p]);
-      const uint16_t* xk = Kh + (size_t)p * OR_D;
-      const uint16_t* xv = Vh + (size_t)p * OR_D;
-      const uint16_t* ak = u->anchor_k + (size_t)u->idx_k[p] * OR_D;
-      const uint16_t* av = u->anchor_v + (size_t)u->idx_v[p] * OR_D;
-      double ev = 0.0;
-      for (int j = 0; j < OR_D; ++j) {
-        rk[j] = or_bf16_to_double(xk[j]) - gk * or_bf16_to_double(ak[j]);
-        rv[j] = or_bf16_to_double(xv[j]) - gv * or_bf16_to_double(av[j]);
-        vt[j] = or_bf16_to_double(xv[j]);
-        ev = ev + rv[j] * rv[j];
-      }
-      double uk = 0.0, uv = 0.0;
-      for (int32_t ww = 0; ww < m; ++ww) {
-        double a = alpha[(size_t)ww * S + p];
-        double a2 = a * a;
-        double d = 0.0, dv = 0.0;
-        for (int j = 0; j < OR_D; ++j) {
-          d = d + or_bf16_to_double(Qh[(size_t)ww * OR_D + j]) * rk[j];
-          double c = vt[j] - y[(size_t)ww * OR_D + j];
-          dv = dv + c * c;
-        }
-        uk = uk + a2 * (d * d / (double)OR_D) * dv;
-        uv = uv + a2 * ev;
-      }
-      if (m > 0) {
-        uk = uk / (double)m;
-        uv = uv / (double)m;
-      }
-      cand[0][ncand[0]].u = uk;
-      cand[0][ncand[0]].h = h;
-      cand[0][ncand[0]].pos = p;
-      ++ncand[0];
-      cand[1][ncand[1]].u = uv;
-      cand[1][ncand[1]].h = h;
-      cand[1][ncand[1]].pos = p;
-      ++ncand[1];
+    qsort(kp, (size_t)np, sizeof(or_keypos), cmp_key_asc);
+    for (int32_t t = 0; t < rest - n_s; ++t) is_anchor[kp[t].pos] = 1;
+    free(kp);
+  }
+  for (int32_t p = S - w; p < S; ++p) is_anchor[p] = 1;
+  int32_t* slot_of = (int32_t*)malloc(sizeof(int32_t) * (size_t)S);
+  int32_t t = 0;
+  for (int32_t p = 0; p < S; ++p) {
+    if (is_anchor[p]) {
+      u->anchor_pos[t] = p;
+      slot_of[p] = t++;
+    } else {
+      slot_of[p] = -1;
     }
   }
-  /* Eq. 9 budget, keys floor(N / 2), values the rest; top N per side pooled over the heads */
+  free(is_anchor);
+  if (t != k) {
+    free(slot_of);
+    free(y);
+    free(alpha);
+    return -1;
+  }
+  for (int32_t a = 0; a < k; ++a) {
+    memcpy(u->anchor_k + (size_t)a * OR_D, Kh + (size_t)u->anchor_pos[a] * OR_D, OR_D * 2);
+    memcpy(u->anchor_v + (size_t)a * OR_D, Vh + (size_t)u->anchor_pos[a] * OR_D, OR_D * 2);
+  }
+  /* assignment and coefficients (Eq. 1, Eq. 2), no residual slots yet */
+  or_encode_side(S, k, 0, Kh, u->anchor_pos, slot_of, sv, rotate, u->idx_k, u->gam_k, NULL, NULL, NULL, NULL);
+  or_encode_side(S, k, 0, Vh, u->anchor_pos, slot_of, sv, rotate, u->idx_v, u->gam_v, NULL, NULL, NULL, NULL);
+  /* exact outputs y^(w) of the observation rows (Eq. 4) */
+  for (int32_t ww = 0; ww < m; ++ww)
+    for (int j = 0; j < OR_D; ++j) {
+      double acc = 0.0;
+      for (int32_t p = 0; p < S; ++p)
+        acc = acc + alpha[(size_t)ww * S + p] * or_bf16_to_double(Vh[(size_t)p * OR_D + j]);
+      y[(size_t)ww * OR_D + j] = acc;
+    }
+  /* Eq. 6 utilities of the non-anchor positions, per side */
+  int64_t nc = 0;
+  for (int32_t p = 0; p < S; ++p) {
+    if (slot_of[p] >= 0) continue;
+    double rk[OR_D], rv[OR_D], vt[OR_D];
+    double gk = or_fp16_to_double(u->gam_k[p]), gv = or_fp16_to_double(u->gam_v[p]);
+    const uint16_t* xk = Kh + (size_t)p * OR_D;
+    const uint16_t* xv = Vh + (size_t)p * OR_D;
+    const uint16_t* ak = u->anchor_k + (size_t)u->idx_k[p] * OR_D;
+    const uint16_t* av = u->anchor_v + (size_t)u->idx_v[p] * OR_D;
+    double ev = 0.0;
+    for (int j = 0; j < OR_D; ++j) {
+      rk[j] = or_bf16_to_double(xk[j]) - gk * or_bf16_to_double(ak[j]);
+      rv[j] = or_bf16_to_double(xv[j]) - gv * or_bf16_to_double(av[j]);
+      vt[j] = or_bf16_to_double(xv[j]);
+      ev = ev + rv[j] * rv[j];
+    }
+    double uk = 0.0, uv = 0.0;
+    for (int32_t ww = 0; ww < m; ++ww) {
+      double a = alpha[(size_t)ww * S + p];
+      double a2 = a * a;
+      double d = 0.0, dv = 0.0;
+      for (int j = 0; j < OR_D; ++j) {
+        d = d + or_bf16_to_double(Qh[(size_t)ww * OR_D + j]) * rk[j];
+        double c = vt[j] - y[(size_t)ww * OR_D + j];
+        dv = dv + c * c;
+      }
+      uk = uk + a2 * (d * d / (double)OR_D) * dv;
+      uv = uv + a2 * ev;
+    }
+    if (m > 0) {
+      uk = uk / (double)m;
+      uv = uv / (double)m;
+    }
+    cand_k[nc].u = uk;
+    cand_k[nc].h = h;
+    cand_k[nc].pos = p;
+    cand_v[nc].u = uv;
+    cand_v[nc].h = h;
+    cand_v[nc].pos = p;
+    ++nc;
+  }
+  *ncand = nc;
+  free(slot_of);
+  free(y);
+  free(alpha);
+  return 0;
+}
+
+/* Algorithm 1, per request: the Eq. 9 budget, keys floor(N / 2) and values the
+ * rest, each side's top N pooled over the request's H heads (the candidates of
+ * head h at cand + h S), then rotation and quantization of the chosen residuals. */
+static void or_pool_request(const uint16_t* K, const uint16_t* V, int32_t s_max, int32_t H, int32_t W, float theta,
+                            const double* sv, int rotate, or_unit* units, or_util* cand[2], const int64_t* ncand) {
+  int32_t S = units[0].S, k = units[0].k;
   int64_t N = or_budget_n((double)theta, S, H, W, k);
   int64_t nside[2] = {N / 2, N - N / 2};
   for (int side = 0; side < 2; ++side) {
-    if (nside[side] > ncand[side]) nside[side] = ncand[side];
-    qsort(cand[side], (size_t)ncand[side], sizeof(or_util), cmp_util_desc);
+    /* gather the heads' candidates, then rank them */
+    int64_t tot = 0;
+    for (int32_t h = 0; h < H; ++h) {
+      memmove(cand[side] + tot, cand[side] + (size_t)h * S, sizeof(or_util) * (size_t)ncand[h]);
+      tot += ncand[h];
+    }
+    if (nside[side] > tot) nside[side] = tot;
+    qsort(cand[side], (size_t)tot, sizeof(or_util), cmp_util_desc);
     for (int32_t h = 0; h < H; ++h) {
       if (side == 0) units[h].nk = 0;
       else units[h].nv = 0;
@@ -775,14 +785,7 @@ int or_encode_select_request(const uint16_t* K, const uint16_t* V, const uint16_
         else or_quantize(r, sv, rotate, u->codes_v + (size_t)i * 32, &u->scale_v[i], &u->min_v[i]);
       }
     }
-    free(slot_of[h]);
   }
-  free(slot_of);
-  free(cand[0]);
-  free(cand[1]);
-  free(y);
-  free(alpha);
-  return 0;
 }
 
 /* Exported for the pins: Eq. 6 utilities of every position of one unit with
@@ -834,19 +837,49 @@ void or_utilities_unit(const or_unit* u, const uint16_t* K, const uint16_t* V, c
   free(alpha);
 }
 
-/* Batched over requests: K, V [B][H][s_max][128], Q [B][H][m][128]; units [B*H]. */
+/* Batched over requests: K, V [B][H][s_max][128], Q [B][H][m][128]; units [B*H]
+ * with S and k set and residual arrays sized min(N_side, S - k).  The heads
+ * run in parallel, then each request's pooling. */
 int or_encode_select_batch(const uint16_t* K, const uint16_t* V, const uint16_t* Q, int32_t s_max, int32_t B, int32_t H,
                            int32_t m, int32_t W, float theta, float rho, int32_t kappa, uint64_t seed,
                            uint64_t rot_seed, int rotate, or_unit* units) {
+  double sv[OR_D];
+  or_signs(rot_seed, sv);
+  int32_t n = B * H;
+  or_util** ck = (or_util**)malloc(sizeof(or_util*) * (size_t)B);
+  or_util** cv = (or_util**)malloc(sizeof(or_util*) * (size_t)B);
+  int64_t* ncand = (int64_t*)calloc((size_t)n, sizeof(int64_t));
+  for (int32_t b = 0; b < B; ++b) {
+    size_t S = (size_t)units[(size_t)b * H].S;
+    ck[b] = (or_util*)malloc(sizeof(or_util) * (size_t)H * S + 1);
+    cv[b] = (or_util*)malloc(sizeof(or_util) * (size_t)H * S + 1);
+  }
   int bad = 0;
 #pragma omp parallel for schedule(dynamic, 1) reduction(| : bad)
-  for (int32_t b = 0; b < B; ++b) {
-    size_t off = (size_t)b * H * (size_t)s_max * OR_D;
-    size_t qoff = (size_t)b * H * (size_t)m * OR_D;
-    if (or_encode_select_request(K + off, V + off, Q + qoff, s_max, H, m, W, theta, rho, kappa, b, seed, rot_seed,
-                                 rotate, units + (size_t)b * H) != 0)
+  for (int32_t u = 0; u < n; ++u) {
+    int32_t b = u / H, h = u % H;
+    size_t off = (size_t)u * (size_t)s_max * OR_D;
+    size_t S = (size_t)units[u].S;
+    if (or_select_head(K + off, V + off, Q + (size_t)u * (size_t)m * OR_D, m, W, rho, kappa, b, h, seed, sv, rotate,
+                       &units[u], ck[b] + (size_t)h * S, cv[b] + (size_t)h * S, &ncand[u]) != 0)
       bad |= 1;
   }
+  if (!bad) {
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int32_t b = 0; b < B; ++b) {
+      size_t off = (size_t)b * H * (size_t)s_max * OR_D;
+      or_util* cand[2] = {ck[b], cv[b]};
+      or_pool_request(K + off, V + off, s_max, H, W, theta, sv, rotate, units + (size_t)b * H, cand,
+                      ncand + (size_t)b * H);
+    }
+  }
+  for (int32_t b = 0; b < B; ++b) {
+    free(ck[b]);
+    free(cv[b]);
+  }
+  free(ck);
+  free(cv);
+  free(ncand);
   return bad ? -1 : 0;
 }
 

@@ -24,7 +24,7 @@ HEAD_DIM = 128
 EXPORTED = (
     "akv_status_string", "akv_last_error", "akv_unit_shapes", "akv_cache_size", "akv_cache_header_host",
     "akv_encode", "akv_encode_noalloc", "akv_cache_pack_host", "akv_decode_workspace_size", "akv_decode_attn",
-    "akv_decode_set_debug",
+    "akv_decode_set_debug", "akv_cache_size_select", "akv_encode_select",
 )
 NOALLOC_SCRATCH_BYTES = 16 << 20
 
@@ -40,6 +40,22 @@ class _Params(ctypes.Structure):
                 ("head_dim", ctypes.c_int32), ("anchor_frac", ctypes.c_float), ("res_frac_k", ctypes.c_float),
                 ("res_frac_v", ctypes.c_float), ("window", ctypes.c_int32), ("seed", ctypes.c_uint64),
                 ("rot_seed", ctypes.c_uint64), ("flags", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+
+
+class _SelectParams(ctypes.Structure):
+    _fields_ = [("theta", ctypes.c_float), ("rho", ctypes.c_float), ("kappa", ctypes.c_int32),
+                ("reserved", ctypes.c_int32)]
+
+
+@dataclass
+class SelectParams:
+    """The paper's full selection (see akv_select_params in include/akv.h)."""
+    theta: float = 0.05
+    rho: float = 0.7
+    kappa: int = 7
+
+    def c(self) -> _SelectParams:
+        return _SelectParams(self.theta, self.rho, self.kappa, 0)
 
 
 class _UnitHost(ctypes.Structure):
@@ -111,6 +127,12 @@ def lib():
         L.akv_decode_attn.restype = st
         L.akv_decode_attn.argtypes = [P, i32p, vp, ctypes.c_size_t, vp, vp, vp, ctypes.c_float, vp,
                                       ctypes.c_size_t, vp]
+        SP = ctypes.POINTER(_SelectParams)
+        L.akv_cache_size_select.restype = st
+        L.akv_cache_size_select.argtypes = [P, SP, i32p, sz, sz]
+        L.akv_encode_select.restype = st
+        L.akv_encode_select.argtypes = [P, SP, i32p, vp, vp, vp, ctypes.c_int32, vp, ctypes.c_size_t, vp,
+                                        ctypes.c_size_t, vp]
         L.akv_decode_set_debug.restype = st
         L.akv_decode_set_debug.argtypes = [ctypes.c_int32, ctypes.c_int32]
         _lib = L
@@ -205,6 +227,24 @@ def akv_encode_noalloc(p: Params, ctx_lens, K, V, arena, stream=None):
     _check(lib().akv_encode_noalloc(ctypes.byref(p.c()), _i32p(lens), _dev_ptr(K), _dev_ptr(V), s_max,
                                     _dev_ptr(arena), arena.numel() * arena.element_size(), _stream_ptr(stream)),
            "akv_encode_noalloc")
+
+
+def akv_cache_size_select(p: Params, sel: SelectParams, ctx_lens):
+    lens = _lens(ctx_lens)
+    a, w = ctypes.c_size_t(), ctypes.c_size_t()
+    _check(lib().akv_cache_size_select(ctypes.byref(p.c()), ctypes.byref(sel.c()), _i32p(lens), ctypes.byref(a),
+                                       ctypes.byref(w)), "akv_cache_size_select")
+    return a.value, w.value
+
+
+def akv_encode_select(p: Params, sel: SelectParams, ctx_lens, K, V, Q, arena, ws, stream=None):
+    """K, V: CUDA bf16 [B][H][s_max][128]; Q: CUDA bf16 [B][H][W*G][128] observation rows."""
+    lens = _lens(ctx_lens)
+    s_max = int(K.shape[2])
+    _check(lib().akv_encode_select(ctypes.byref(p.c()), ctypes.byref(sel.c()), _i32p(lens), _dev_ptr(K), _dev_ptr(V),
+                                   _dev_ptr(Q), s_max, _dev_ptr(arena), arena.numel() * arena.element_size(),
+                                   _dev_ptr(ws), ws.numel() * ws.element_size(), _stream_ptr(stream)),
+           "akv_encode_select")
 
 
 _UNIT_FIELDS = (("anchor_k", np.uint16), ("anchor_v", np.uint16), ("anchor_pos", np.int32), ("idx_k", np.uint16),

@@ -37,7 +37,7 @@ void rotation_signs(uint64_t rot_seed, uint64_t bits[2]) {
   bits[1] = splitmix64(rot_seed + 1);
 }
 
-akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out) {
+akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out, const akv_select_params* sel) {
   if (!p || !ctx_lens || !out) return fail(AKV_ERR_INVALID, "null params, ctx_lens or output");
   if (p->head_dim != kD) return fail(AKV_ERR_UNSUPPORTED, "head_dim must be 128");
   if (p->batch < 1 || p->n_kv_heads < 1 || p->n_q_heads < 1)
@@ -51,6 +51,16 @@ akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out
     return fail(AKV_ERR_INVALID, "fractions must be finite and in [0, 1]");
   if (p->window < 0) return fail(AKV_ERR_INVALID, "window must be >= 0");
   if (p->reserved != 0 || (p->flags & ~AKV_FLAG_ROTATE) != 0) return fail(AKV_ERR_INVALID, "unknown flags");
+  if (sel) {
+    if (!(std::isfinite(sel->theta) && sel->theta > 0.0f && sel->theta <= 1.0f))
+      return fail(AKV_ERR_INVALID, "theta must be in (0, 1]");
+    if (!(std::isfinite(sel->rho) && sel->rho >= 0.0f && sel->rho <= 1.0f))
+      return fail(AKV_ERR_INVALID, "rho must be in [0, 1]");
+    if (sel->kappa < 1 || sel->kappa > 255 || sel->kappa % 2 == 0)
+      return fail(AKV_ERR_INVALID, "kappa must be odd and in [1, 255]");
+    if (sel->reserved != 0) return fail(AKV_ERR_INVALID, "reserved select field must be 0");
+    if (p->window < 1) return fail(AKV_ERR_INVALID, "the full selection needs W >= 1 observation positions");
+  }
 
   Layout& L = *out;
   L = Layout();
@@ -69,6 +79,11 @@ akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out
     if (k > S) k = S;
     int64_t nk = (int64_t)std::floor((double)p->res_frac_k * (double)S);
     int64_t nv = (int64_t)std::floor((double)p->res_frac_v * (double)S);
+    if (sel) {  // capacities: the most the request's pooled budget can give one head
+      const int64_t N = budget_residuals(sel->theta, S, p->n_kv_heads, p->window, (int32_t)std::min<int64_t>(k, S));
+      nk = N / 2;
+      nv = N - N / 2;
+    }
     if (nk > S - k) nk = S - k;
     if (nv > S - k) nv = S - k;
     if (k < 1) return fail(AKV_ERR_INVALID, "anchor budget is zero (window 0 and anchor_frac * S < 1)");
@@ -130,7 +145,7 @@ akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out
   return AKV_OK;
 }
 
-void encode_ws_layout(const Layout& L, EncodeWs* ws) {
+void encode_ws_layout(const Layout& L, EncodeWs* ws, int32_t m_obs) {
   // Per unit: two u64 key arrays [S] (anchor hashes, then residual energies
   // per side), slot map i32 [S], residual positions i32 [N_K + N_V],
   // anchor norms (squared, and square roots) f64 [k] per side, 256 B control,
@@ -153,6 +168,10 @@ void encode_ws_layout(const Layout& L, EncodeWs* ws) {
     b += align_up((uint64_t)s.S * 4, 256) * 2;        // stored order and its inverse
     b += align_up((uint64_t)(s.k + 1) * 4, 256);      // value-anchor run starts
     b += align_up((uint64_t)s.nt * 8, 256);           // records per tile and side
+    if (m_obs > 0) {                                  // full selection: observation rows'
+      b += align_up((uint64_t)m_obs * s.S * 8, 256);  // attention alpha [m][S] f64
+      b += align_up((uint64_t)m_obs * kD * 8, 256);   // and exact outputs y [m][128] f64
+    }
     off += b;
   }
   ws->total = off + 256;
@@ -377,6 +396,46 @@ akv_status akv_encode(const akv_params* p, const int32_t* ctx_lens_host, const v
   encode_ws_layout(L, &W);
   if (ws_bytes < W.total) return fail(AKV_ERR_TOO_SMALL, "encode workspace shorter than akv_cache_size");
   int err = launch_encode(L, W, *p, K, V, s_max, arena, ws, (void*)stream);
+  if (err) return fail(AKV_ERR_CUDA, std::string("encode launch failed: ") + cuda_error_string(err));
+  return AKV_OK;
+}
+
+akv_status akv_cache_size_select(const akv_params* p, const akv_select_params* sel, const int32_t* ctx_lens_host,
+                                 size_t* arena_bytes, size_t* encode_ws_bytes) {
+  g_last_error.clear();
+  if (!sel) return fail(AKV_ERR_INVALID, "null select parameters");
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L, sel);
+  if (st != AKV_OK) return st;
+  if (arena_bytes) *arena_bytes = (size_t)L.total_bytes;
+  if (encode_ws_bytes) {
+    EncodeWs W;
+    encode_ws_layout(L, &W, p->window * L.G);
+    *encode_ws_bytes = (size_t)W.total;
+  }
+  return AKV_OK;
+}
+
+akv_status akv_encode_select(const akv_params* p, const akv_select_params* sel, const int32_t* ctx_lens_host,
+                             const void* K, const void* V, const void* Q, int32_t s_max, void* arena, size_t arena_bytes,
+                             void* ws, size_t ws_bytes, akv_stream_t stream) {
+  g_last_error.clear();
+  if (!sel) return fail(AKV_ERR_INVALID, "null select parameters");
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L, sel);
+  if (st != AKV_OK) return st;
+  if (!K || !V || !Q || !arena || !ws) return fail(AKV_ERR_INVALID, "null K, V, Q, arena or workspace");
+  if (((uintptr_t)arena % 256) || ((uintptr_t)ws % 256) || ((uintptr_t)K % 16) || ((uintptr_t)V % 16) ||
+      ((uintptr_t)Q % 16))
+    return fail(AKV_ERR_INVALID, "arena and workspace must be 256-byte aligned, K, V and Q 16-byte aligned");
+  if (s_max < L.max_len) return fail(AKV_ERR_INVALID, "s_max is smaller than the longest context");
+  if (L.shape.size() > 65535) return fail(AKV_ERR_UNSUPPORTED, "encode handles at most 65535 (request, head) units");
+  if (arena_bytes < L.total_bytes) return fail(AKV_ERR_TOO_SMALL, "arena shorter than akv_cache_size_select");
+  const int32_t m_obs = p->window * L.G;
+  EncodeWs W;
+  encode_ws_layout(L, &W, m_obs);
+  if (ws_bytes < W.total) return fail(AKV_ERR_TOO_SMALL, "encode workspace shorter than akv_cache_size_select");
+  int err = launch_encode(L, W, *p, K, V, s_max, arena, ws, (void*)stream, sel, Q, m_obs);
   if (err) return fail(AKV_ERR_CUDA, std::string("encode launch failed: ") + cuda_error_string(err));
   return AKV_OK;
 }

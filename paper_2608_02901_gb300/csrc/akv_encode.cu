@@ -45,6 +45,8 @@ struct EncUnitWs {
   int32_t* inv;       // [S] stored index of position i
   uint32_t* cursor;   // [k + 1] value-anchor counts, then start of each run
   uint32_t* tcnt;     // [2 * n_tiles] residual records per tile (keys, values)
+  double* alpha;      // full selection: [m][S] observation rows' attention
+  double* yobs;       // full selection: [m][128] their exact outputs
 };
 
 struct EncArgs {
@@ -60,6 +62,11 @@ struct EncArgs {
   int32_t rotate;
   uint64_t seed;
   unsigned long long sign_lo, sign_hi;
+  // full selection (m_obs > 0): observation rows Q [units][m_obs][128], pooling width,
+  // scored share, retained fraction
+  const __nv_bfloat16* Q;
+  int32_t m_obs, kappa;
+  float rho, theta;
 };
 
 __device__ __forceinline__ const akv_unit_desc* unit_desc(const EncArgs& A, int u) {
@@ -101,6 +108,10 @@ __device__ EncUnitWs unit_ws(const EncArgs& A, int u, const akv_unit_desc* d) {
   w.cursor = (uint32_t*)p;
   p += au((k + 1) * 4, 256);
   w.tcnt = (uint32_t*)p;
+  p += au((uint64_t)d->n_tiles * 8, 256);
+  w.alpha = (double*)p;
+  p += au((uint64_t)A.m_obs * S * 8, 256);
+  w.yobs = (double*)p;
   return w;
 }
 
@@ -146,17 +157,18 @@ __device__ uint32_t f64_to_fp16_bits(double x) {
   return sign | out;
 }
 
-// r-th smallest (1-based) of n 64-bit keys (optionally of their complements),
-// MSB-first radix select by 8-bit digits; returns the key and the rank of the
-// answer among keys equal to it (*rank_in_eq, 1-based).  Block-wide.
-__device__ uint64_t block_select(const uint64_t* keys, int n, uint32_t r, bool complement, uint32_t* hist,
-                                 uint32_t* bcast, uint32_t* rank_in_eq) {
+// r-th smallest (1-based) of the n 64-bit keys key_at(0 .. n-1) (optionally of their
+// complements), MSB-first radix select by 8-bit digits; returns the key and the rank of
+// the answer among keys equal to it (*rank_in_eq, 1-based).  Block-wide.
+template <class KeyAt>
+__device__ uint64_t block_select_f(KeyAt key_at, int64_t n, uint32_t r, bool complement, uint32_t* hist,
+                                   uint32_t* bcast, uint32_t* rank_in_eq) {
   uint64_t prefix = 0, mask = 0;
   for (int shift = 56; shift >= 0; shift -= 8) {
     for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
     __syncthreads();
-    for (int i = threadIdx.x; i < n; i += blockDim.x) {
-      uint64_t key = keys[i];
+    for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
+      uint64_t key = key_at(i);
       if (complement) key = ~key;
       if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
     }
@@ -181,6 +193,10 @@ __device__ uint64_t block_select(const uint64_t* keys, int n, uint32_t r, bool c
   }
   *rank_in_eq = r;
   return complement ? ~prefix : prefix;
+}
+__device__ uint64_t block_select(const uint64_t* keys, int n, uint32_t r, bool complement, uint32_t* hist,
+                                 uint32_t* bcast, uint32_t* rank_in_eq) {
+  return block_select_f([keys](int64_t i) { return keys[i]; }, n, r, complement, hist, bcast, rank_in_eq);
 }
 
 // Exclusive block scan of 0/1 flags for a block of 1024 threads; returns the
@@ -212,6 +228,12 @@ __device__ int block_scan_flag(int flag, int* warp_tot, int* total) {
 
 // ---- kernels -----------------------------------------------------------------
 
+// Anchors of the full selection picked by score: floor(rho (k - w)) (Section 3.2); none in
+// the plain encoder.
+__device__ __forceinline__ int n_scored(const EncArgs& A, int rest) {
+  return (A.m_obs > 0 && rest > 0) ? (int)floor((double)A.rho * (double)rest) : 0;
+}
+
 __global__ void enc_hash(const EncArgs A) {
   const int u = blockIdx.y;
   const akv_unit_desc* d = unit_desc(A, u);
@@ -221,7 +243,9 @@ __global__ void enc_hash(const EncArgs A) {
   EncUnitWs w = unit_ws(A, u, d);
   const int win = min(A.window, S);
   const uint64_t base = A.seed ^ ((uint64_t)d->b << 40) ^ ((uint64_t)d->h << 32);
-  w.key0[p] = (p < S - win) ? splitmix64_dev(base ^ (uint64_t)p) : ~0ull;
+  // (full selection: positions already chosen by their score take no part in the sampling)
+  const bool scored = A.m_obs > 0 && w.slot_of[p] == -2;
+  w.key0[p] = (p < S - win && !scored) ? splitmix64_dev(base ^ (uint64_t)p) : ~0ull;
 }
 
 __global__ void __launch_bounds__(1024) enc_anchors(const EncArgs A) {
@@ -233,7 +257,9 @@ __global__ void __launch_bounds__(1024) enc_anchors(const EncArgs A) {
   const int S = d->len, k = d->n_anchors;
   EncUnitWs w = unit_ws(A, u, d);
   const int win = min(A.window, S);
-  const int pool = S - win, rest = k - win;
+  const int pool = S - win;
+  // the sampled share: all k - w non-window anchors, less those the full selection scored
+  const int rest = k - win - n_scored(A, k - win);
   uint64_t thr = 0;
   bool any = rest > 0;
   if (any) {
@@ -245,7 +271,7 @@ __global__ void __launch_bounds__(1024) enc_anchors(const EncArgs A) {
   for (int c0 = 0; c0 < S; c0 += 1024) {
     const int p = c0 + threadIdx.x;
     int flag = 0;
-    if (p < S) flag = (p >= pool) || (any && w.key0[p] <= thr);
+    if (p < S) flag = (p >= pool) || (A.m_obs > 0 && w.slot_of[p] == -2) || (any && w.key0[p] <= thr);
     int tot;
     const int pre = block_scan_flag(flag, wt, &tot);
     if (p < S) {
@@ -571,11 +597,12 @@ __global__ void enc_quant(const EncArgs A) {
   __shared__ double vbuf[8][128];
   const int u = blockIdx.y, side = blockIdx.z;
   const akv_unit_desc* d = unit_desc(A, u);
-  const int N = side ? d->n_res_v : d->n_res_k;
+  EncUnitWs w = unit_ws(A, u, d);
+  // slots of this unit: the parameters' count, or the count the full selection chose
+  const int N = A.m_obs > 0 ? (int)w.ctrl[2 + side] : (side ? d->n_res_v : d->n_res_k);
   const int wi = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int s = blockIdx.x * 8 + wi;
   if (s >= N) return;
-  EncUnitWs w = unit_ws(A, u, d);
   const int p = w.res_pos[(side ? d->n_res_k : 0) + s];
   const uint32_t st = w.st[side][p];
   const int a = (int)(st & 0xFFFFu);
@@ -660,6 +687,283 @@ __global__ void enc_quant(const EncArgs A) {
   if (lane == 0) *reinterpret_cast<uint32_t*>(blk + sm_off) = sch | (mnh << 16);
 }
 
+// ---- the paper's full selection (Algorithm 1; Section 3.2-3.4, Appendix A.2) --------------
+// Each fp64 sum runs in a fixed order (positions, then rows, then dimensions ascending, one
+// thread per output), and the exponential is evaluated by fixed steps, so every decision
+// (scored anchors, pooled residual slots) comes out the same on any IEEE machine.
+
+// e^x for x <= 0: Cody-Waite argument reduction (ln 2 split into a 42-bit leading part,
+// whose product with n is exact, and the remainder), a degree-22 Taylor series of e^r by
+// Horner's rule, then the exact scaling by 2^n; about 1 ulp.  Arguments below -700 give 0.
+__device__ double exp_neg_dev(double x) {
+  if (!(x >= -700.0)) return 0.0;
+  const double ln2_hi = 0.693147180559890330187045037746429443359375;
+  const double ln2_lo = 5.4979230187083711552420206887987e-14;
+  const double n = rint(__ddiv_rn(x, 0.6931471805599453094172321));
+  const double r = __dsub_rn(__dsub_rn(x, __dmul_rn(n, ln2_hi)), __dmul_rn(n, ln2_lo));
+  double y = 1.0;
+  for (int j = 22; j >= 1; --j) y = __dadd_rn(1.0, __dmul_rn(__ddiv_rn(r, (double)j), y));
+  return ldexp(y, (int)n);
+}
+
+// Logits q_w . K_t / sqrt(D) of every observation row and position (Eq. 4), into alpha.
+__global__ void __launch_bounds__(128) enc_obs_logit(const EncArgs A) {
+  __shared__ double qs[128];
+  const int u = blockIdx.z, wr = blockIdx.y;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len;
+  const int t = blockIdx.x * 128 + threadIdx.x;
+  if (blockIdx.x * 128 >= S) return;
+  EncUnitWs w = unit_ws(A, u, d);
+  qs[threadIdx.x] = bf16_to_f64(A.Q[((size_t)u * A.m_obs + wr) * 128 + threadIdx.x]);
+  __syncthreads();
+  if (t >= S) return;
+  const __nv_bfloat16* X = A.K + ((size_t)u * A.s_max + t) * 128;
+  double acc = 0.0;
+  for (int j = 0; j < 128; ++j) acc = __dadd_rn(acc, __dmul_rn(qs[j], bf16_to_f64(X[j])));
+  w.alpha[(size_t)wr * S + t] = __dmul_rn(acc, __ddiv_rn(1.0, __dsqrt_rn(128.0)));
+}
+
+// Softmax of each observation row's logits over all S positions.
+__global__ void __launch_bounds__(1024) enc_obs_softmax(const EncArgs A) {
+  __shared__ double red[32];
+  __shared__ double den_s;
+  const int u = blockIdx.y, wr = blockIdx.x;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len;
+  EncUnitWs w = unit_ws(A, u, d);
+  double* a = w.alpha + (size_t)wr * S;
+  double mx = -INFINITY;
+  for (int t = threadIdx.x; t < S; t += blockDim.x) mx = fmax(mx, a[t]);
+  for (int o = 16; o > 0; o >>= 1) mx = fmax(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double m = red[0];
+    for (int i = 1; i < (int)(blockDim.x >> 5); ++i) m = fmax(m, red[i]);
+    red[0] = m;
+  }
+  __syncthreads();
+  mx = red[0];
+  for (int t = threadIdx.x; t < S; t += blockDim.x) a[t] = exp_neg_dev(__dsub_rn(a[t], mx));
+  __syncthreads();
+  if (threadIdx.x == 0) {  // the normaliser, summed in position order
+    double den = 0.0;
+    for (int t = 0; t < S; ++t) den = __dadd_rn(den, a[t]);
+    den_s = den;
+  }
+  __syncthreads();
+  const double den = den_s;
+  for (int t = threadIdx.x; t < S; t += blockDim.x) a[t] = __ddiv_rn(a[t], den);
+}
+
+// Exact output y_w = sum_t alpha_wt V_t of each observation row (positions in order).
+__global__ void __launch_bounds__(128) enc_obs_y(const EncArgs A) {
+  const int u = blockIdx.y, wr = blockIdx.x, j = threadIdx.x;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len;
+  EncUnitWs w = unit_ws(A, u, d);
+  const double* a = w.alpha + (size_t)wr * S;
+  const __nv_bfloat16* V = A.V + (size_t)u * A.s_max * 128;
+  double acc = 0.0;
+  for (int t = 0; t < S; ++t) acc = __dadd_rn(acc, __dmul_rn(a[t], bf16_to_f64(V[(size_t)t * 128 + j])));
+  w.yobs[wr * 128 + j] = acc;
+}
+
+// Selector score, step 1: the rows' attention averaged over the m rows (into key1 as fp64).
+__global__ void enc_score_mean(const EncArgs A) {
+  const int u = blockIdx.y;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len, P = S - min(A.window, S);
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= P) return;
+  EncUnitWs w = unit_ws(A, u, d);
+  double acc = 0.0;
+  for (int wr = 0; wr < A.m_obs; ++wr) acc = __dadd_rn(acc, w.alpha[(size_t)wr * S + t]);
+  w.key1[t] = (uint64_t)__double_as_longlong(__ddiv_rn(acc, (double)A.m_obs));
+}
+
+// Selector score, step 2: average pooling of width kappa centred on t over [0, P), zero
+// outside, divided by kappa (Appendix A.2); the score's bits into key0 (scores are >= 0,
+// so their bit patterns order like the values).
+__global__ void enc_score_pool(const EncArgs A) {
+  const int u = blockIdx.y;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len, P = S - min(A.window, S);
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= P) return;
+  EncUnitWs w = unit_ws(A, u, d);
+  const int h = A.kappa / 2;
+  double acc = 0.0;
+  for (int j = t - h; j <= t + h; ++j)
+    if (j >= 0 && j < P) acc = __dadd_rn(acc, __longlong_as_double((long long)w.key1[j]));
+  w.key0[t] = (uint64_t)__double_as_longlong(__ddiv_rn(acc, (double)A.kappa));
+}
+
+// The floor(rho (k - w)) highest scores (ties: lower position) become anchors: slot_of = -2
+// marks them for enc_hash and enc_anchors, every other position gets -1.
+__global__ void __launch_bounds__(1024) enc_score_pick(const EncArgs A) {
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t bc[2];
+  __shared__ int wt[33];
+  const int u = blockIdx.x;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len, k = d->n_anchors, win = min(A.window, S), P = S - win;
+  EncUnitWs w = unit_ws(A, u, d);
+  const int ns = n_scored(A, k - win);
+  uint64_t thr = ~0ull;
+  uint32_t need = 0;
+  if (ns > 0) thr = block_select(w.key0, P, (uint32_t)ns, true, hist, bc, &need);
+  int eq_seen = 0;
+  for (int c0 = 0; c0 < S; c0 += 1024) {
+    const int p = c0 + threadIdx.x;
+    const uint64_t kv = (p < P) ? w.key0[p] : 0ull;
+    const int is_eq = (ns > 0 && p < P && kv == thr) ? 1 : 0;
+    int eq_tot;
+    const int eq_pre = block_scan_flag(is_eq, wt, &eq_tot);
+    const int sel = (ns > 0 && p < P) && (kv > thr || (is_eq && (uint32_t)(eq_seen + eq_pre) < need));
+    eq_seen += eq_tot;
+    if (p < S) w.slot_of[p] = sel ? -2 : -1;
+    __syncthreads();
+  }
+}
+
+// Eq. 6 utilities of the non-anchor positions (one thread per position, rows and
+// dimensions in order): key0 = bits(u^K) + 1, key1 = bits(u^V) + 1, anchors 0.
+constexpr int UT_ROWS = 16;  // observation rows staged in shared memory at a time
+__global__ void __launch_bounds__(128) enc_util(const EncArgs A) {
+  __shared__ double qs[UT_ROWS][128];
+  __shared__ double ys[UT_ROWS][128];
+  const int u = blockIdx.y;
+  const akv_unit_desc* d = unit_desc(A, u);
+  const int S = d->len;
+  if (blockIdx.x * 128 >= S) return;
+  EncUnitWs w = unit_ws(A, u, d);
+  const int p = blockIdx.x * 128 + threadIdx.x;
+  const bool live = p < S && w.slot_of[p] < 0;
+  const int32_t* apos = reinterpret_cast<const int32_t*>(A.arena_c + d->off_anchor_pos);
+  const __nv_bfloat16 *xk = nullptr, *xv = nullptr, *ak = nullptr, *av = nullptr;
+  double gk = 0.0, gv = 0.0, ev = 0.0;
+  if (live) {
+    xk = A.K + ((size_t)u * A.s_max + p) * 128;
+    xv = A.V + ((size_t)u * A.s_max + p) * 128;
+    const uint32_t sk = w.st[0][p], sv = w.st[1][p];
+    ak = anchor_src(A, u, 0, apos, (int)(sk & 0xFFFFu));
+    av = anchor_src(A, u, 1, apos, (int)(sv & 0xFFFFu));
+    gk = fp16_bits_to_f64(sk >> 16);
+    gv = fp16_bits_to_f64(sv >> 16);
+    for (int j = 0; j < 128; ++j) {
+      const double rv = __dsub_rn(bf16_to_f64(xv[j]), __dmul_rn(gv, bf16_to_f64(av[j])));
+      ev = __dadd_rn(ev, __dmul_rn(rv, rv));
+    }
+  }
+  double uk = 0.0, uv = 0.0;
+  for (int w0 = 0; w0 < A.m_obs; w0 += UT_ROWS) {
+    const int nr = min(UT_ROWS, A.m_obs - w0);
+    __syncthreads();
+    for (int e = threadIdx.x; e < nr * 128; e += 128) {
+      qs[e >> 7][e & 127] = bf16_to_f64(A.Q[((size_t)u * A.m_obs + w0 + (e >> 7)) * 128 + (e & 127)]);
+      ys[e >> 7][e & 127] = w.yobs[(w0 + (e >> 7)) * 128 + (e & 127)];
+    }
+    __syncthreads();
+    if (!live) continue;
+    for (int r = 0; r < nr; ++r) {
+      const double a = w.alpha[(size_t)(w0 + r) * S + p];
+      const double a2 = __dmul_rn(a, a);
+      double dq = 0.0, dv = 0.0;
+      for (int j = 0; j < 128; ++j) {
+        const double rk = __dsub_rn(bf16_to_f64(xk[j]), __dmul_rn(gk, bf16_to_f64(ak[j])));
+        dq = __dadd_rn(dq, __dmul_rn(qs[r][j], rk));
+        const double c = __dsub_rn(bf16_to_f64(xv[j]), ys[r][j]);
+        dv = __dadd_rn(dv, __dmul_rn(c, c));
+      }
+      uk = __dadd_rn(uk, __dmul_rn(__dmul_rn(a2, __ddiv_rn(__dmul_rn(dq, dq), 128.0)), dv));
+      uv = __dadd_rn(uv, __dmul_rn(a2, ev));
+    }
+  }
+  if (p >= S) return;
+  if (!live) {
+    w.key0[p] = 0ull;
+    w.key1[p] = 0ull;
+    return;
+  }
+  uk = __ddiv_rn(uk, (double)A.m_obs);
+  uv = __ddiv_rn(uv, (double)A.m_obs);
+  w.key0[p] = (uint64_t)__double_as_longlong(uk) + 1ull;
+  w.key1[p] = (uint64_t)__double_as_longlong(uv) + 1ull;
+}
+
+// One block per request: the side's Eq. 9 share of the budget goes to the highest
+// utilities over all KV heads of the request (ties: lower head, then lower position) ->
+// per-unit flags, ascending slot lists and counts (ctrl[2 + side]).
+__global__ void __launch_bounds__(1024) enc_pool(const EncArgs A, int side) {
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t bc[2];
+  __shared__ int wt[33];
+  __shared__ const uint64_t* keys[256];
+  __shared__ int32_t* lists[256];
+  __shared__ uint32_t* ctrls[256];
+  __shared__ uint8_t* flags[256];
+  const int H = A.n_kv_heads, u0 = blockIdx.x * H;
+  const akv_unit_desc* d0 = unit_desc(A, u0);
+  const int S = d0->len, k = d0->n_anchors;
+  for (int h = threadIdx.x; h < H; h += blockDim.x) {
+    const akv_unit_desc* d = unit_desc(A, u0 + h);
+    EncUnitWs w = unit_ws(A, u0 + h, d);
+    keys[h] = side ? w.key1 : w.key0;
+    lists[h] = w.res_pos + (side ? d->n_res_k : 0);
+    ctrls[h] = w.ctrl;
+    flags[h] = w.flag;
+  }
+  __syncthreads();
+  const int64_t N = budget_residuals(A.theta, S, H, A.window, k);
+  const int64_t cand = (int64_t)H * (S - k);
+  int64_t want = side ? N - N / 2 : N / 2;
+  if (want > cand) want = cand;
+  const int64_t n = (int64_t)H * S;
+  auto key_at = [&](int64_t i) { return keys[i / S][i % S]; };
+  uint64_t thr = ~0ull;
+  uint32_t need = 0;
+  if (want > 0) thr = block_select_f(key_at, n, (uint32_t)want, true, hist, bc, &need);
+  int eq_seen = 0;
+  for (int h = 0; h < H; ++h) {
+    int base = 0;
+    for (int c0 = 0; c0 < S; c0 += 1024) {
+      const int p = c0 + threadIdx.x;
+      const uint64_t kv = p < S ? keys[h][p] : 0ull;
+      const int is_eq = (want > 0 && p < S && kv == thr) ? 1 : 0;
+      int eq_tot;
+      const int eq_pre = block_scan_flag(is_eq, wt, &eq_tot);
+      const int sel = (want > 0 && p < S) && (kv > thr || (is_eq && (uint32_t)(eq_seen + eq_pre) < need));
+      eq_seen += eq_tot;
+      int tot;
+      const int pre = block_scan_flag(sel, wt, &tot);
+      if (sel) lists[h][base + pre] = p;
+      // flags of both sides share bytes: the side-0 launch writes them, side 1 ORs its bit in
+      if (p < S) {
+        if (side == 0) flags[h][p] = (uint8_t)sel;
+        else if (sel) flags[h][p] |= 2u;
+      }
+      base += tot;
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) ctrls[h][2 + side] = (uint32_t)base;
+  }
+}
+
+// The arena descriptors take the residual counts the full selection chose (last launch:
+// every earlier kernel sizes its scratch from the reserved counts).
+__global__ void enc_set_counts(const EncArgs A, int units) {
+  const int u = blockIdx.x * blockDim.x + threadIdx.x;
+  if (u >= units) return;
+  const akv_unit_desc* d = unit_desc(A, u);
+  EncUnitWs w = unit_ws(A, u, d);
+  akv_unit_desc* dm = reinterpret_cast<akv_unit_desc*>(A.arena + 256) + u;
+  const int32_t nk = (int32_t)w.ctrl[2], nv = (int32_t)w.ctrl[3];
+  dm->n_res_k = nk;
+  dm->n_res_v = nv;
+}
+
 }  // namespace
 
 // Scratch of akv_encode_noalloc, for callers that cannot hand the library a
@@ -684,7 +988,7 @@ int noalloc_scratch(void** ptr, size_t* bytes) {
 }
 
 int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const void* K, const void* V, int32_t s_max,
-                  void* arena, void* ws, void* stream) {
+                  void* arena, void* ws, void* stream, const akv_select_params* sel, const void* Q, int32_t m_obs) {
   cudaStream_t st = (cudaStream_t)stream;
   const int units = (int)L.shape.size();
   cudaError_t e;
@@ -712,22 +1016,44 @@ int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const
   A.seed = p.seed;
   A.sign_lo = L.header.sign_bits[0];
   A.sign_hi = L.header.sign_bits[1];
+  const bool full = sel != nullptr && Q != nullptr && m_obs > 0;
+  A.Q = (const __nv_bfloat16*)Q;
+  A.m_obs = full ? m_obs : 0;
+  A.kappa = full ? sel->kappa : 1;
+  A.rho = full ? sel->rho : 0.0f;
+  A.theta = full ? sel->theta : 0.0f;
 
   const unsigned maxS = (unsigned)L.max_len;
+  if (full) {  // observation rows' attention, selector scores, the scored anchors
+    const unsigned m = (unsigned)m_obs;
+    enc_obs_logit<<<dim3((maxS + 127) / 128, m, units), 128, 0, st>>>(A);
+    enc_obs_softmax<<<dim3(m, units), 1024, 0, st>>>(A);
+    enc_obs_y<<<dim3(m, units), 128, 0, st>>>(A);
+    enc_score_mean<<<dim3((maxS + 255) / 256, units), 256, 0, st>>>(A);
+    enc_score_pool<<<dim3((maxS + 255) / 256, units), 256, 0, st>>>(A);
+    enc_score_pick<<<units, 1024, 0, st>>>(A);
+  }
   enc_hash<<<dim3((maxS + 255) / 256, units), 256, 0, st>>>(A);
   enc_anchors<<<units, 1024, 0, st>>>(A);
   enc_rows<<<dim3((unsigned)(L.max_k + 7) / 8, units), 256, 0, st>>>(A);
   if ((e = cudaFuncSetAttribute(enc_assign, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AS_SMEM)) != cudaSuccess)
     return (int)e;
   enc_assign<<<dim3((maxS + AS_POS - 1) / AS_POS, units, 2), AS_THREADS, AS_SMEM, st>>>(A);
-  enc_slots<<<units, 1024, 0, st>>>(A, 0);  // writes the flag bytes
-  enc_slots<<<units, 1024, 0, st>>>(A, 1);  // ORs the value bit in
+  if (full) {  // Eq. 6 utilities, then each side's pooled top-N per request
+    enc_util<<<dim3((maxS + 127) / 128, units), 128, 0, st>>>(A);
+    enc_pool<<<units / p.n_kv_heads, 1024, 0, st>>>(A, 0);  // writes the flag bytes
+    enc_pool<<<units / p.n_kv_heads, 1024, 0, st>>>(A, 1);  // ORs the value bit in
+  } else {
+    enc_slots<<<units, 1024, 0, st>>>(A, 0);  // writes the flag bytes
+    enc_slots<<<units, 1024, 0, st>>>(A, 1);  // ORs the value bit in
+  }
   enc_order<<<units, 1024, 0, st>>>(A);
   enc_tile_count<<<dim3((unsigned)L.max_tiles, units), kTile, 0, st>>>(A);
   enc_tile_table<<<(units + 127) / 128, 128, 0, st>>>(A, units);
   enc_tile_fill<<<dim3((unsigned)L.max_tiles, units), kTile, 0, st>>>(A);
   const int maxN = std::max(L.max_nk, L.max_nv);
   if (maxN > 0) enc_quant<<<dim3((unsigned)(maxN + 7) / 8, units, 2), 256, 0, st>>>(A);
+  if (full) enc_set_counts<<<(units + 127) / 128, 128, 0, st>>>(A, units);
   return (int)cudaGetLastError();
 }
 

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <atomic>
+#include <cmath>
 #include <cstddef>
 #include <cstdint>
 #include <string>
@@ -47,6 +48,27 @@ AKV_HD constexpr uint32_t value_code_word(int d) { return 32u * (uint32_t)(d / 3
 // bit of record slot s (0..15) in a value-code word: even slots in the low half word
 AKV_HD constexpr uint32_t value_code_bit(int s) { return 2u * (uint32_t)(s / 2) + 16u * (uint32_t)(s % 2); }
 
+// Eq. 9 residual count of one layer (one request's H KV heads at context S), with the fixed
+// bytes M_base of Eq. 11 and the residual cost of the Appendix A.1 accounting.  M_base per
+// head: bf16 anchor keys and values (4 k D bytes), int64 positions of the k - w non-window
+// anchors, a 2-byte index and a 2-byte coefficient per side for each of the P = S - w other
+// positions, and per side a 64-bit mask word and a 32-bit prefix word per 64 positions;
+// shared by the heads: H + 1 int64 head offsets and P int32 position ids.  M_full = 4 S H D
+// (bf16 keys and values).  One residual costs the mean of a key record (D/4 code bytes and
+// an fp32 scale) and a value record (one more byte of position).  Every term is an integer
+// below 2^53 except theta * M_full, so host and device evaluate it identically.  Keys take
+// floor(N / 2) slots, values the rest (Section 3.4).
+AKV_HD inline int64_t budget_residuals(float theta, int32_t S, int32_t H, int32_t W, int32_t k) {
+  const int64_t w = W < S ? W : S;
+  const int64_t P = (int64_t)S - w;
+  const int64_t m_full = 4ll * S * H * kD;
+  const int64_t m_base = (int64_t)H * (4ll * k * kD + 8ll * (k - w) + 8ll * P) + 24ll * H * ((P + 63) / 64) +
+                         8ll * (H + 1) + 4ll * P;
+  const double b_res = (double)((kD / 4 + 4) + (kD / 4 + 5)) / 2.0;
+  const double n = floor(((double)theta * (double)m_full - (double)m_base) / b_res);
+  return n > 0.0 ? (int64_t)n : 0;
+}
+
 // Section indices inside one unit segment, in storage order.
 enum Section { kAnchorK = 0, kAnchorV, kAnchorPos, kTileTable, kTiles, kNumSections };
 
@@ -66,8 +88,12 @@ struct Layout {
 // Records a failure text for akv_last_error() and returns the status.
 akv_status fail(akv_status s, const std::string& msg);
 
-// Validates parameters and context lengths and fills the layout.
-akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out);
+// Validates parameters and context lengths and fills the layout.  With `sel` (the
+// paper's full selection), each unit's residual capacity per side is the most the pooled
+// Eq. 9 budget of its request can give one head: min(N_side, S - k); the descriptors of an
+// encoded arena then hold the counts the selection chose.
+akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out,
+                       const akv_select_params* sel = nullptr);
 
 // 128-bit rotation sign mask: bit j set <=> s_j = -1.
 void rotation_signs(uint64_t rot_seed, uint64_t bits[2]);
@@ -79,11 +105,14 @@ struct EncodeWs {
   std::vector<uint64_t> unit_off;  // byte offset of each unit's scratch in ws
   uint64_t total = 0;
 };
-void encode_ws_layout(const Layout& L, EncodeWs* ws);
+// m_obs > 0: scratch of the full selection (observation rows' attention and outputs) as well.
+void encode_ws_layout(const Layout& L, EncodeWs* ws, int32_t m_obs = 0);
 
 // Kernel launchers (defined in the .cu files).  Return cudaError_t as int.
+// sel / Q non-null: the paper's full selection with m_obs observation rows per KV head.
 int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const void* K, const void* V, int32_t s_max,
-                  void* arena, void* ws, void* stream);
+                  void* arena, void* ws, void* stream, const akv_select_params* sel = nullptr,
+                  const void* Q = nullptr, int32_t m_obs = 0);
 int launch_decode(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
                   float sm_scale, void* stream, std::string* why);
 const char* cuda_error_string(int err);

@@ -197,3 +197,20 @@ def test_decode_debug_controls_validate():
     assert _err(akv.akv_decode_set_debug, -1, 0) == akv.AKV_ERR_INVALID
     assert _err(akv.akv_decode_set_debug, 0, 2) == akv.AKV_ERR_INVALID
     akv.akv_decode_set_debug(0, 0)
+
+
+def test_select_parameters_validate_and_size_the_pooled_capacity():
+    p = akv.Params(batch=2, n_kv_heads=4, n_q_heads=16, anchor_frac=0.02, res_frac_k=0.0, res_frac_v=0.0)
+    lens = [4096, 1000]
+    for bad in (akv.SelectParams(theta=0.0), akv.SelectParams(theta=1.5), akv.SelectParams(rho=-0.1),
+                akv.SelectParams(kappa=4), akv.SelectParams(kappa=0)):
+        assert _err(akv.akv_cache_size_select, p, bad, lens) == akv.AKV_ERR_INVALID
+    p0 = akv.Params(batch=2, n_kv_heads=4, n_q_heads=16, window=0, anchor_frac=0.02)
+    assert _err(akv.akv_cache_size_select, p0, akv.SelectParams(), lens) == akv.AKV_ERR_INVALID
+    sel = akv.SelectParams(theta=0.05)
+    a_sel, w_sel = akv.akv_cache_size_select(p, sel, lens)
+    a_plain, w_plain = akv.akv_cache_size(p, lens)
+    assert a_sel > a_plain and w_sel > w_plain  # residual room for the pooled budget; attention scratch
+    # each unit may hold up to its request's whole side budget (Eq. 9), capped by its non-anchors
+    hdr = akv.akv_cache_header_host(p, lens)  # plain layout: no residuals at fractions 0
+    assert int(hdr[256 + 8:256 + 12].view(np.int32)[0]) == 0
