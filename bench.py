@@ -111,7 +111,7 @@ def unit_bytes(S, k, nk, nv, G):
     reads the exact block sizes from the arena's tile tables)."""
     nt = (S + TILE - 1) // TILE
     fixed = sum(_tile_fixed(min(TILE, S - j * TILE)) for j in range(nt))
-    return 512 * k + 4 * (nt + 1) + fixed + 36 * (nk + nv) + 252 * nt + 2 * (2 * G * 128)
+    return 512 * k + 4 * (2 * nt + 1) + fixed + 36 * (nk + nv) + 252 * nt + 2 * (2 * G * 128)
 
 
 def arena_unit_bytes(torch, akv, p, lens, arena) -> list:
@@ -125,7 +125,7 @@ def arena_unit_bytes(torch, akv, p, lens, arena) -> list:
         k, nt = int(d[4:8].view(np.int32)[0]), int(d[16:20].view(np.int32)[0])
         o_tt = int(d[56:64].view(np.uint64)[0])
         offs.append(o_tt + 4 * nt)
-        fixed.append(512 * k + 4 * (nt + 1) + 2 * (2 * p.G * 128))
+        fixed.append(512 * k + 4 * (2 * nt + 1) + 2 * (2 * p.G * 128))
     idx = torch.tensor([o + i for o in offs for i in range(4)], dtype=torch.long, device=arena.device)
     used = arena[idx].cpu().numpy().view(np.uint32).astype(np.int64)
     return [f + int(b) for f, b in zip(fixed, used)]
@@ -319,9 +319,12 @@ def run_akv(args, rank, world, local):
     out = torch.empty((n_tok, layers, B, Hq, 128), dtype=torch.bfloat16, device=dev)
     chunk = n_tok * layers
 
+    # one decode workspace (anchor scores, partial sums) serves every call: they are stream-ordered
+    dws = torch.empty(akv.akv_decode_workspace_size(p, lens), dtype=torch.uint8, device=dev)
+
     def step(i, stream=None):
         t, layer = divmod(i % chunk, layers)
-        akv.akv_decode_attn(p, lens, arenas[layer], qs[t, layer], out[t, layer], None, 1.0, None, stream)
+        akv.akv_decode_attn(p, lens, arenas[layer], qs[t, layer], out[t, layer], None, 1.0, dws, stream)
 
     # warm-up (also sets kernel attributes before capture)
     for i in range(min(args.warmup, chunk)):
@@ -389,7 +392,7 @@ def run_akv(args, rank, world, local):
 
     def e2e_ops(i, s):
         q_dev.copy_(q_host[i], non_blocking=True)
-        akv.akv_decode_attn(p, lens, arenas[i % layers], q_dev, o_dev, None, 1.0, None, s)
+        akv.akv_decode_attn(p, lens, arenas[i % layers], q_dev, o_dev, None, 1.0, dws, s)
         o_host[i].copy_(o_dev, non_blocking=True)
 
     e2e_graphs = []

@@ -54,7 +54,7 @@ typedef enum akv_status {
 #define AKV_HEAD_DIM 128
 #define AKV_FLAG_ROTATE 1u /* residuals carry the randomized Hadamard rotation (Appendix A.1, Eq. 12) */
 #define AKV_ARENA_MAGIC 0x32564B41u /* "AKV2" */
-#define AKV_ARENA_VERSION 2u
+#define AKV_ARENA_VERSION 3u
 #define AKV_MAX_ANCHORS 65535 /* anchor indices are uint16 (Table 1, b_a = 2) */
 #define AKV_TILE_TOKENS 1024  /* tokens per tile block of the packed token stream */
 
@@ -126,7 +126,11 @@ typedef struct akv_arena_header {
  *   anchor_v   [k][128] bf16  anchor values, same swizzle
  *   anchor_pos [k] int32      anchor positions (not read by decode)
  *   tile_table [n_tiles + 1] uint32  byte offset of tile block j from off_tiles
- *                             (multiples of 16); entry n_tiles = bytes used
+ *                             (multiples of 16); entry n_tiles = bytes used;
+ *              then [n_tiles] uint32  value-slot range of tile j: the a_V slot of its
+ *                             first stored token in bits 0-15, of its last in bits
+ *                             16-31 (the anchor-value rows its tokens weight, known
+ *                             before the block is read)
  *   tiles                     n_tiles = ceil(S / AKV_TILE_TOKENS) tile blocks
  *
  * Tile block j holds the stored tokens [j T, min(S, (j+1) T)), T = AKV_TILE_TOKENS:
@@ -364,8 +368,11 @@ akv_status akv_cache_pack_host(const akv_params* p, const int32_t* ctx_lens_host
 /* ---- Decode ------------------------------------------------------------- */
 
 /*
- * Bytes of device workspace akv_decode_attn needs (0 for the cluster kernel
- * of this build; callers should still query it).
+ * Bytes of device workspace akv_decode_attn needs for these parameters and
+ * context lengths: the anchor scores of every unit (4 G bytes per anchor),
+ * their maxima per chunk of 64 anchors, one arrival counter per unit, and
+ * the partial sums of the CTAs that share a unit (about 8.5 KB per query head
+ * and (CTA or unit) slot, at most 256 CTAs).  Contents on entry are ignored.
  */
 akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_lens_host, size_t* ws_bytes);
 
@@ -381,14 +388,18 @@ akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_len
  *   q         : device bf16 [B][H_q][128]
  *   out       : device bf16 [B][H_q][128], round-to-nearest-even of the fp32 result
  *   out_f32   : device fp32 [B][H_q][128] or NULL
- *   ws        : device workspace of >= akv_decode_workspace_size bytes (may be NULL if 0)
- * Errors: AKV_ERR_INVALID (null/misaligned pointers, bad sizes),
- * AKV_ERR_UNSUPPORTED (k * G beyond the shared-memory tables of this build),
+ *   ws        : device workspace, 256-byte aligned, of >= akv_decode_workspace_size
+ *               bytes; calls that overlap on the GPU need separate workspaces
+ * Two launches: the anchor scores of every unit, then the decode itself, one CTA
+ * per SM over equal shares of all units' tile blocks.
+ * Errors: AKV_ERR_INVALID (null/misaligned pointers, bad sizes), AKV_ERR_TOO_SMALL
+ * (arena or workspace short), AKV_ERR_UNSUPPORTED (no shared-memory plan fits),
  * AKV_ERR_CUDA (launch failure).
- * Ordering: the launch is a programmatic dependent launch: it may be scheduled and set
- * up its on-chip state while a preceding akv_decode_attn launch in the same stream
- * drains, but it reads the arena and q, and writes out/out_f32, only after all
- * preceding work in the stream has completed (ordinary stream semantics for data).
+ * Ordering: both launches are programmatic dependent launches: each may be scheduled
+ * and set up its on-chip state while the preceding launch in the stream drains, but
+ * reads the arena, q and the workspace, and writes out/out_f32 and the workspace,
+ * only after all preceding work in the stream has completed (ordinary stream
+ * semantics for data).
  */
 akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,
                            size_t arena_bytes, const void* q, void* out, float* out_f32, float sm_scale,
@@ -400,16 +411,17 @@ akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, co
  * Process-wide controls of akv_decode_attn, for tests and tuning (the paper has
  * no counterpart).  Both are 0 by default, which is normal operation; a call
  * applies to every decode launch issued after it, on every thread.
- *   cluster_ctas  : 0 = the launch planner chooses the CTAs per (request, KV
- *                   head); 1..16 = that many, or the largest smaller count
- *                   whose launch fits the device
- *   withhold_last : 1 = every CTA withholds the last tile of its stream, so the
- *                   waits on it run out after their bound (about 2 s): the call
- *                   returns and its outputs are NaN.  This tests the bounded
- *                   waits (failure detection) without any GPU fault.
+ *   ctas          : 0 = one decode CTA per SM; 1..256 = that many CTAs (at most
+ *                   one per tile block), which moves the boundaries of the ranges
+ *                   of tile blocks the CTAs share out
+ *   withhold_last : 1 = every CTA withholds the last tile block of its range, so
+ *                   the waits on it run out after their bound (about 2 s): the
+ *                   call returns and the outputs of the units of those tiles are
+ *                   NaN.  This tests the bounded waits (failure detection) without
+ *                   any GPU fault.
  * Errors: AKV_ERR_INVALID for values out of range.
  */
-akv_status akv_decode_set_debug(int32_t cluster_ctas, int32_t withhold_last);
+akv_status akv_decode_set_debug(int32_t ctas, int32_t withhold_last);
 
 #ifdef __cplusplus
 } /* extern "C" */

@@ -1001,7 +1001,7 @@ static uint64_t rd64(const uint8_t* p) {
 
 /* Returns 0 and the shape of unit u, or -1 on a malformed arena. */
 int or_arena_shape(const uint8_t* arena, uint64_t bytes, int32_t u, int32_t* shape4) {
-  if (bytes < 256 || rd32(arena) != 0x32564B41u || rd32(arena + 4) != 2u || rd32(arena + 104) != 1024u) return -1;
+  if (bytes < 256 || rd32(arena) != 0x32564B41u || rd32(arena + 4) != 3u || rd32(arena + 104) != 1024u) return -1;
   int32_t n_units = (int32_t)rd32(arena + 72);
   uint64_t doff = rd64(arena + 80);
   if (u < 0 || u >= n_units || doff + 256ull * (uint64_t)(u + 1) > bytes) return -1;
@@ -1027,7 +1027,7 @@ int or_arena_unpack(const uint8_t* arena, uint64_t bytes, int32_t u, or_unit* ou
   uint64_t o_ak = rd64(d + 32), o_av = rd64(d + 40), o_ap = rd64(d + 48), o_tt = rd64(d + 56), o_ti = rd64(d + 64);
   uint64_t cap = rd64(d + 72);
   if (o_ak + 256ull * k > bytes || o_av + 256ull * k > bytes || o_ap + 4ull * k > bytes ||
-      o_tt + 4ull * (nt + 1) > bytes || o_ti + cap > bytes || (o_ak % 16) || (o_av % 16) || (o_ti % 16))
+      o_tt + 4ull * (2 * nt + 1) > bytes || o_ti + cap > bytes || (o_ak % 16) || (o_av % 16) || (o_ti % 16))
     return -1;
   for (int32_t a = 0; a < k; ++a)
     for (int c = 0; c < 16; ++c) {
@@ -1106,6 +1106,9 @@ int or_arena_unpack(const uint8_t* arena, uint64_t bytes, int32_t u, or_unit* ou
     }
     for (int32_t t = n; t < n64; ++t)
       if (rd32(kst + 4ull * t) || rd32(vst + 4ull * t)) return -1;
+    /* the tile's value-slot range word: slots of its first and last stored tokens */
+    if (rd32(arena + o_tt + 4ull * (nt + 1 + j)) != ((rd32(vst) & 0xFFFFu) | ((rd32(vst + 4ull * (n - 1)) & 0xFFFFu) << 16)))
+      return -1;
     cnt[0] += m[0];
     cnt[1] += m[1];
   }

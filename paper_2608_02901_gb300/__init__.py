@@ -298,18 +298,24 @@ def _decode_args(p: Params, ctx_lens):
 
 
 def akv_decode_attn(p: Params, ctx_lens, arena, q, out, out_f32=None, sm_scale: float = 1.0, ws=None, stream=None):
-    """q, out: CUDA bf16 [B][H_q][128]; out_f32 optional fp32 of the same shape."""
+    """q, out: CUDA bf16 [B][H_q][128]; out_f32 optional fp32 of the same shape.
+    ws: CUDA uint8 workspace of akv_decode_workspace_size bytes; when None, one is taken
+    from torch's allocator on out's device for this call."""
     pref, lref = _decode_args(p, ctx_lens)
-    ws_bytes = 0 if ws is None else ws.numel() * ws.element_size()
+    if ws is None:
+        import torch
+        ws = torch.empty(akv_decode_workspace_size(p, ctx_lens), dtype=torch.uint8, device=out.device)
+    ws_bytes = ws.numel() * ws.element_size()
     _check(lib().akv_decode_attn(pref, lref, _dev_ptr(arena), arena.numel() * arena.element_size(), _dev_ptr(q),
                                  _dev_ptr(out), _dev_ptr(out_f32), float(sm_scale), _dev_ptr(ws), ws_bytes,
                                  _stream_ptr(stream)),
            "akv_decode_attn")
 
 
-def akv_decode_set_debug(cluster_ctas: int = 0, withhold_last: int = 0):
-    """Testing controls of the decode launch (0, 0 = normal operation)."""
-    _check(lib().akv_decode_set_debug(int(cluster_ctas), int(withhold_last)), "akv_decode_set_debug")
+def akv_decode_set_debug(ctas: int = 0, withhold_last: int = 0):
+    """Testing controls of the decode launch (0, 0 = normal operation): the number of decode
+    CTAs (0 = one per SM), and withholding each CTA's last tile block."""
+    _check(lib().akv_decode_set_debug(int(ctas), int(withhold_last)), "akv_decode_set_debug")
 
 
 def unit_host_from_logical(u: dict) -> dict:

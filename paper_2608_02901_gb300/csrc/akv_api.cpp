@@ -104,7 +104,7 @@ akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out
       cap += 36ull * (uint64_t)(nk + nv) + 504ull * (uint64_t)nt;
       if (cap >= (1ull << 32)) return fail(AKV_ERR_UNSUPPORTED, "a unit's tile blocks could exceed 2^32 bytes");
       const uint64_t sizes[kNumSections] = {(uint64_t)k * 256, (uint64_t)k * 256, (uint64_t)k * 4,
-                                            4ull * (uint64_t)(nt + 1), cap};
+                                            tile_table_bytes(nt), cap};
       akv_unit_desc& d = L.desc[u];
       std::memset(&d, 0, sizeof(d));
       d.len = S;
@@ -335,6 +335,7 @@ akv_status akv_cache_pack_host(const akv_params* p, const int32_t* ctx_lens_host
       for (int32_t t = 0; t < n; ++t)
         for (int side = 0; side < 2; ++side) cnt[side] += slot[side][(size_t)perm[(size_t)(t0 + t)]] >= 0;
       table[j] = off;
+      table[sh.nt + 1 + j] = (uint32_t)in.idx_v[perm[(size_t)t0]] | ((uint32_t)in.idx_v[perm[(size_t)(t0 + n - 1)]] << 16);
       if ((uint64_t)off + tile_block_bytes(n, cnt[0], cnt[1]) > d.tiles_capacity)
         return fail(AKV_ERR_INVALID, "tile blocks exceed their reserved capacity");  // cannot happen: bound
       uint8_t* blk = tiles + off;
@@ -462,11 +463,11 @@ akv_status akv_encode_noalloc(const akv_params* p, const int32_t* ctx_lens_host,
   return akv_encode(p, ctx_lens_host, K, V, s_max, arena, arena_bytes, ws, ws_bytes, stream);
 }
 
-akv_status akv_decode_set_debug(int32_t cluster_ctas, int32_t withhold_last) {
+akv_status akv_decode_set_debug(int32_t ctas, int32_t withhold_last) {
   g_last_error.clear();
-  if (cluster_ctas < 0 || cluster_ctas > 16) return fail(AKV_ERR_INVALID, "cluster_ctas must be in [0, 16]");
+  if (ctas < 0 || ctas > 256) return fail(AKV_ERR_INVALID, "ctas must be in [0, 256]");
   if (withhold_last < 0 || withhold_last > 1) return fail(AKV_ERR_INVALID, "withhold_last must be 0 or 1");
-  g_debug_cluster.store(cluster_ctas);
+  g_debug_cluster.store(ctas);
   g_debug_withhold.store(withhold_last);
   return AKV_OK;
 }
@@ -477,15 +478,13 @@ akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_len
   akv_status st = make_layout(p, ctx_lens_host, &L);
   if (st != AKV_OK) return st;
   if (!ws_bytes) return fail(AKV_ERR_INVALID, "null ws_bytes");
-  *ws_bytes = 0;
+  *ws_bytes = decode_ws_layout(L).total;
   return AKV_OK;
 }
 
 akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,
                            size_t arena_bytes, const void* q, void* out, float* out_f32, float sm_scale,
                            void* ws, size_t ws_bytes, akv_stream_t stream) {
-  (void)ws;
-  (void)ws_bytes;
   if (!g_last_error.empty()) g_last_error.clear();
   akv_status st;
   const std::shared_ptr<const Layout> Lp = decode_layout(p, ctx_lens_host, &st);
@@ -496,8 +495,10 @@ akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, co
     return fail(AKV_ERR_INVALID, "arena must be 256-byte aligned; q, out, out_f32 16-byte aligned");
   if (arena_bytes < L.total_bytes) return fail(AKV_ERR_TOO_SMALL, "arena shorter than akv_cache_size");
   if (!std::isfinite(sm_scale)) return fail(AKV_ERR_INVALID, "sm_scale must be finite");
+  if (!ws || ((uintptr_t)ws % 256)) return fail(AKV_ERR_INVALID, "decode workspace must be non-null and 256-byte aligned");
+  if (ws_bytes < decode_ws_layout(L).total) return fail(AKV_ERR_TOO_SMALL, "decode workspace shorter than akv_decode_workspace_size");
   std::string why;
-  int err = launch_decode(L, *p, arena, q, out, out_f32, sm_scale, (void*)stream, &why);
+  int err = launch_decode(L, *p, arena, q, out, out_f32, sm_scale, ws, (void*)stream, &why);
   if (err == -1) return fail(AKV_ERR_UNSUPPORTED, why);
   if (err) return fail(AKV_ERR_CUDA, std::string("decode launch failed: ") + cuda_error_string(err) + " " + why);
   return AKV_OK;

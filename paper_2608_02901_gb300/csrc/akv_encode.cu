@@ -550,6 +550,9 @@ __global__ void enc_tile_table(const EncArgs A, int units) {
   for (int j = 0; j < d->n_tiles; ++j) {
     table[j] = off;
     off += tile_block_bytes(tile_len(d->len, j), (int)w.tcnt[2 * j], (int)w.tcnt[2 * j + 1]);
+    // value slots of the tile's first and last stored tokens
+    const int t0 = j * kTile, t1 = t0 + tile_len(d->len, j) - 1;
+    table[d->n_tiles + 1 + j] = (w.st[1][w.perm[t0]] & 0xFFFFu) | ((w.st[1][w.perm[t1]] & 0xFFFFu) << 16);
   }
   table[d->n_tiles] = off;
 }

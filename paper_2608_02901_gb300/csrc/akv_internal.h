@@ -43,6 +43,8 @@ AKV_HD constexpr uint32_t tile_block_bytes(int n, int nk, int nv) {
   return tile_fixed_bytes(n) + round16(4u * (uint32_t)nk) + round16(4u * (uint32_t)nv) + 32u * (uint32_t)nk +
          value_code_bytes(nv);
 }
+// tile table section: n_tiles + 1 block offsets, then one value-slot range word per tile
+AKV_HD constexpr uint64_t tile_table_bytes(int nt) { return 4ull * (uint64_t)(2 * nt + 1); }
 // word of dimension d in a group of value codes
 AKV_HD constexpr uint32_t value_code_word(int d) { return 32u * (uint32_t)(d / 32) + 4u * (uint32_t)(d % 8) + (uint32_t)((d % 32) / 8); }
 // bit of record slot s (0..15) in a value-code word: even slots in the low half word
@@ -113,8 +115,14 @@ void encode_ws_layout(const Layout& L, EncodeWs* ws, int32_t m_obs = 0);
 int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const void* K, const void* V, int32_t s_max,
                   void* arena, void* ws, void* stream, const akv_select_params* sel = nullptr,
                   const void* Q = nullptr, int32_t m_obs = 0);
+// Decode workspace (device): anchor scores [units][ka][G] f32, chunk maxima, arrival counters,
+// partial slots; byte offsets from the workspace base (256-byte aligned).
+struct DecodeWs {
+  size_t o_sa = 0, o_cmax = 0, o_cnt = 0, o_part = 0, total = 0;
+};
+DecodeWs decode_ws_layout(const Layout& L);
 int launch_decode(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
-                  float sm_scale, void* stream, std::string* why);
+                  float sm_scale, void* ws, void* stream, std::string* why);
 const char* cuda_error_string(int err);
 // Testing controls of the decode launch (akv_decode_set_debug), 0 = normal operation.
 extern std::atomic<int> g_debug_cluster, g_debug_withhold;

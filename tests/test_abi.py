@@ -56,7 +56,7 @@ def test_layout_header_and_sections():
     p = akv.Params(batch=4, n_kv_heads=2, n_q_heads=8, seed=3, rot_seed=9)
     arena_bytes, ws_bytes = akv.akv_cache_size(p, lens)
     hdr = akv.akv_cache_header_host(p, lens)
-    assert hdr[:4].view(np.uint32)[0] == 0x32564B41 and hdr[4:8].view(np.uint32)[0] == 2
+    assert hdr[:4].view(np.uint32)[0] == 0x32564B41 and hdr[4:8].view(np.uint32)[0] == 3
     assert hdr[8:16].view(np.uint64)[0] == arena_bytes
     assert hdr[72:76].view(np.int32)[0] == 8 and hdr[76:80].view(np.int32)[0] == 5000
     assert hdr[104:108].view(np.int32)[0] == 1024
@@ -78,12 +78,13 @@ def test_layout_header_and_sections():
             nw = (min(1024, S - 1024 * j) + 63) // 64
             fixed += 512 * nw + 16 * nw + 2 * ((2 * nw + 15) // 16 * 16)
         assert cap == fixed + 36 * (nk + nv) + 504 * nt
-        sizes = [k * 256, k * 256, 4 * k, 4 * (nt + 1), cap]
+        # tile table: nt + 1 block offsets and one value-slot range word per tile
+        sizes = [k * 256, k * 256, 4 * k, 4 * (2 * nt + 1), cap]
         assert offs[0] % 256 == 0
         for o, sz in zip(offs, sizes):
             assert o % 128 == 0 and o >= prev_end
             prev_end = o + sz
-        assert data == 512 * k + 4 * (nt + 1) + cap
+        assert data == 512 * k + 4 * (2 * nt + 1) + cap
     assert prev_end <= arena_bytes
     assert ws_bytes > 0
 
@@ -153,7 +154,7 @@ def test_parameter_validation():
     assert _err(akv.akv_cache_size, akv.Params(**base), [0]) == akv.AKV_ERR_INVALID
     assert _err(akv.akv_cache_size, akv.Params(**base, window=0, anchor_frac=0.0), [100]) == akv.AKV_ERR_INVALID
     assert _err(akv.akv_cache_size, akv.Params(**base, anchor_frac=0.02), [4_000_000]) == akv.AKV_ERR_UNSUPPORTED
-    assert akv.akv_decode_workspace_size(akv.Params(**base), [100]) == 0
+    assert akv.akv_decode_workspace_size(akv.Params(**base), [100]) > 0
 
 
 def test_pack_rejects_bad_arrays():
@@ -184,6 +185,13 @@ def test_entry_points_validate_before_any_launch():
     assert st == akv.AKV_ERR_TOO_SMALL
     st = L.akv_decode_attn(ctypes.byref(p), lp, 0x1000, nbytes, 256, 256, None, float("inf"), None, 0, None)
     assert st == akv.AKV_ERR_INVALID
+    wbytes = akv.akv_decode_workspace_size(akv.Params(batch=1, n_kv_heads=1, n_q_heads=1), lens)
+    st = L.akv_decode_attn(ctypes.byref(p), lp, 0x1000, nbytes, 256, 256, None, 1.0, None, wbytes, None)
+    assert st == akv.AKV_ERR_INVALID and "workspace" in akv.akv_last_error()
+    st = L.akv_decode_attn(ctypes.byref(p), lp, 0x1000, nbytes, 256, 256, None, 1.0, 0x3000 + 16, wbytes, None)
+    assert st == akv.AKV_ERR_INVALID
+    st = L.akv_decode_attn(ctypes.byref(p), lp, 0x1000, nbytes, 256, 256, None, 1.0, 0x3000, wbytes - 1, None)
+    assert st == akv.AKV_ERR_TOO_SMALL
     st = L.akv_encode(ctypes.byref(p), lp, None, 256, 128, 0x1000, nbytes, 0x2000, 1 << 20, None)
     assert st == akv.AKV_ERR_INVALID
     st = L.akv_encode(ctypes.byref(p), lp, 256, 256, 50, 0x1000, nbytes, 0x2000, 1 << 20, None)
@@ -193,7 +201,7 @@ def test_entry_points_validate_before_any_launch():
 
 
 def test_decode_debug_controls_validate():
-    assert _err(akv.akv_decode_set_debug, 17, 0) == akv.AKV_ERR_INVALID
+    assert _err(akv.akv_decode_set_debug, 257, 0) == akv.AKV_ERR_INVALID
     assert _err(akv.akv_decode_set_debug, -1, 0) == akv.AKV_ERR_INVALID
     assert _err(akv.akv_decode_set_debug, 0, 2) == akv.AKV_ERR_INVALID
     akv.akv_decode_set_debug(0, 0)

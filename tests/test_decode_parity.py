@@ -73,10 +73,12 @@ def test_negative_and_saturated_gamma_and_zero_anchor(dev):
     _run_seeded(dev, p, [1500, 900], mutate=mutate)
 
 
-def test_many_units_cluster_sizes(dev, debug_controls):
+def test_many_units_cta_counts(dev, debug_controls):
+    """The tile blocks of 16 units (ragged) split over 1 .. 37 CTAs: ranges that start and end
+    inside units, CTAs that cross several units, units shared by several CTAs."""
     p = akv.Params(batch=4, n_kv_heads=4, n_q_heads=16)
-    for c in (1, 2, 3, 8, 16):
-        akv.akv_decode_set_debug(cluster_ctas=c)
+    for c in (1, 2, 3, 8, 16, 37):
+        akv.akv_decode_set_debug(ctas=c)
         _run_seeded(dev, p, [8192, 3000, 6001, 700], qseed=c)
 
 
@@ -146,16 +148,16 @@ def test_locally_dense_residuals_exceed_staging(dev):
 
 def test_tiles_covering_more_value_slots_than_the_weight_table(dev, debug_controls):
     """Every non-anchor token on the last value anchor: stored in value-slot order, the first
-    tile then holds one token of each of about a thousand anchors, more value slots than its
-    CTA's value-weight table rows, so most of its runs take the path that adds their
-    anchor-value products on CUDA cores; the CTAs whose tiles hold the long last run share
+    tile then holds one token of each of about a thousand anchors, more value slots than the
+    anchor-value rows staged with a tile, so most of its runs take the path that adds their
+    anchor-value products on CUDA cores; the tiles (and CTAs) that hold the long last run share
     that slot, each with its own tokens' weights."""
     def mutate(u, d):
         non = np.setdiff1d(np.arange(d["S"]), d["anchor_pos"])
         d["idx_v"] = d["idx_v"].copy()
         d["idx_v"][non] = d["k"] - 1
     for c in (4, 8):
-        akv.akv_decode_set_debug(cluster_ctas=c)
+        akv.akv_decode_set_debug(ctas=c)
         for G in (1, 4):
             p = akv.Params(batch=1, n_kv_heads=2, n_q_heads=2 * G, anchor_frac=0.2, seed=41)
             _run_seeded(dev, p, [6000], mutate=mutate, qseed=c + G)
@@ -199,12 +201,12 @@ def test_back_to_back_launches_follow_stream_order(dev):
     assert np.abs(y32.cpu().numpy().astype(np.float64) - y_ref).max() <= 5e-3
 
 
-def test_large_anchor_tables_take_larger_clusters(dev):
-    """80 units with 5243 anchors each: at one CTA per unit the anchor-score and value-weight
-    tables leave no room for the full staged record count, so the launch takes clusters of two
-    or more (more than one wave) rather than pushing most records onto the CUDA-core paths.
-    Checked against the oracle on a sample of units; all outputs finite."""
-    p = akv.Params(batch=40, n_kv_heads=2, n_q_heads=8, anchor_frac=0.16, res_frac_k=0.1, res_frac_v=0.1, seed=4,
+@pytest.mark.parametrize("G", [4, 8])
+def test_large_anchor_tables(dev, G):
+    """80 units with 5243 anchors each: 84 KB of anchor scores per unit at G = 4 (staged in shared
+    memory next to the pipeline), 168 KB at G = 8 (beyond it: the token gathers read the
+    workspace table).  Checked against the oracle on a sample of units; all outputs finite."""
+    p = akv.Params(batch=40, n_kv_heads=2, n_q_heads=2 * G, anchor_frac=0.16, res_frac_k=0.1, res_frac_v=0.1, seed=4,
                    rot_seed=9)
     lens = [32768] * p.batch
     units = seeded_units(p, lens, seed=12)
@@ -216,13 +218,14 @@ def test_large_anchor_tables_take_larger_clusters(dev):
     sel[[0, 37, 79]] = 1
     ref = oracle_decode(p, [oracle_unit(u) for u in units], q, 1.0, sel=sel)
     rows = np.repeat(sel.astype(bool), p.G).reshape(p.batch, p.n_q_heads)
-    check_outputs(out[rows], out32[rows], ref[rows], where="large anchor tables")
+    check_outputs(out[rows], out32[rows], ref[rows], where=f"large anchor tables G={G}")
 
 
 def test_withheld_item_times_out_to_nan_and_context_survives(dev, debug_controls):
     """Failure detection without a GPU fault: with the test hook every CTA withholds the last
-    tile of its stream, so the waits on it run out after their bound (about 2 s).  The call
-    returns, the outputs are NaN, and the next call on the same context is correct."""
+    tile of its range (here every CTA has one tile), so the waits on it run out after their
+    bound (about 2 s).  The call returns, the outputs are NaN, and the next call on the same
+    context is correct."""
     import time
     p = akv.Params(batch=1, n_kv_heads=2, n_q_heads=8, seed=3, rot_seed=77)
     lens = [5000]
