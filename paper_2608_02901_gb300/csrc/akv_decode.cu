@@ -59,14 +59,12 @@ namespace {
 
 constexpr int NG = 2;               // tile groups per CTA: tiles in processing at once
 constexpr int WPG = 4;              // warps per group
-constexpr int NCW = NG * WPG;       // compute warps 0 .. 7
-constexpr int W_PROD = NCW;         // producer warp
-constexpr int NT = (NCW + 1) * 32;  // 288 threads
+constexpr int NCW = NG * WPG;       // warps 0 .. 7; two per SM sub-partition, so 255 registers each
+constexpr int NT = NCW * 32;        // 256 threads
 constexpr int T = kTile;            // tokens per tile block
 constexpr int LCH = T / (WPG * 32); // consecutive stored tokens per lane
 static_assert(LCH == 8, "a lane's tokens are one byte of a bitmap word");
-constexpr int NSLOT = 8;            // stage descriptors; a multiple of NG, so a slot always serves one group
-static_assert(NSLOT % NG == 0, "slot reuse must stay within one group");
+constexpr int NSG = 4;              // tiles a group has in flight at most (its stage descriptors)
 constexpr int kMaxGrid = 256;       // CTAs of the decode launch at most
 constexpr int CHA = 64;             // anchors per score-kernel CTA (4 warps x 16 rows)
 constexpr int kRingSlack = 4096;    // shared memory after the ring: the masked rows of the last
@@ -245,27 +243,6 @@ __device__ __forceinline__ float half_lo(uint32_t w) {
 }
 __device__ __forceinline__ float half_hi(uint32_t w) { return __half2float(__ushort_as_half((unsigned short)(w >> 16))); }
 
-// Packed pairs of fp32 (one instruction for both lanes of the pair).
-__device__ __forceinline__ float2 f2fma(float2 a, float2 b, float2 c) {
-  unsigned long long ra, rb, rc, rd;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(ra) : "f"(a.x), "f"(a.y));
-  asm("mov.b64 %0, {%1, %2};" : "=l"(rb) : "f"(b.x), "f"(b.y));
-  asm("mov.b64 %0, {%1, %2};" : "=l"(rc) : "f"(c.x), "f"(c.y));
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(rd) : "l"(ra), "l"(rb), "l"(rc));
-  float2 d;
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(rd));
-  return d;
-}
-__device__ __forceinline__ float2 f2add(float2 a, float2 b) {
-  unsigned long long ra, rb, rd;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(ra) : "f"(a.x), "f"(a.y));
-  asm("mov.b64 %0, {%1, %2};" : "=l"(rb) : "f"(b.x), "f"(b.y));
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(rd) : "l"(ra), "l"(rb));
-  float2 d;
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(rd));
-  return d;
-}
-
 // 2^x with the hardware approximation (relative error near 2^-22; results below the
 // smallest normal flush to 0, which only drops weights under 2^-126 of the reference).
 __device__ __forceinline__ float exp2_approx(float x) {
@@ -376,7 +353,7 @@ __device__ __forceinline__ TileView tile_view(const uint8_t* st, const Meta& mt,
 // Records beyond the staged ones (a locally dense tile) take these rare paths on CUDA
 // cores, kept out of line so that the token loop stays small.
 // Key residual term scale (q'_g . c) + min sum(q'_g) of key record r.
-__device__ __noinline__ float key_record_term(const TileView& tv, int r, const float* qpg, float sqg) {
+__device__ __noinline__ float key_record_term(const TileView tv, int r, const float* qpg, float sqg) {
   const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_k + 4u * (uint32_t)r));
   float dot = 0.f;
   for (int bb = 0; bb < 32; ++bb) {
@@ -388,7 +365,7 @@ __device__ __noinline__ float key_record_term(const TileView& tv, int r, const f
 }
 // accg += p (min + scale c) of value record r, in the rotated domain (value codes are
 // dimension-major groups of 16 records).
-__device__ __noinline__ void value_record_add(const TileView& tv, int r, float p, float* accg) {
+__device__ __noinline__ void value_record_add(const TileView tv, int r, float p, float* accg) {
   const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_v + 4u * (uint32_t)r));
   const float ps = p * half_lo(smn), pm = p * half_hi(smn);
   const uint32_t base = tv.cd_v + 512u * (uint32_t)(r / 16);
@@ -406,6 +383,18 @@ __device__ __noinline__ void anchor_value_add(const uint8_t* AV, int anchor, con
     const float x = __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(row + 16 * ((d >> 3) ^ (anchor & 7)) + 2 * (d & 7)));
 #pragma unroll
     for (int g = 0; g < GS; ++g) atomicAdd(&ov[g * 128 + d], acc[g] * x);
+  }
+}
+
+// N consecutive 32-bit words (4 N-byte aligned) from shared memory.
+template <int N>
+__device__ __forceinline__ void load_words(const uint8_t* p, uint32_t (&w)[N]) {
+  if constexpr (N == 4) {
+    const uint4 v = *reinterpret_cast<const uint4*>(p);
+    w[0] = v.x; w[1] = v.y; w[2] = v.z; w[3] = v.w;
+  } else {
+    const uint2 v = *reinterpret_cast<const uint2*>(p);
+    w[0] = v.x; w[1] = v.y;
   }
 }
 
@@ -523,23 +512,57 @@ __device__ void combine_unit(const DecodeParams& P, int u, int first, int nseg, 
   const int lane = threadIdx.x & 31;
   constexpr int PF = part_floats(GS);
   const size_t ob = qrow_base(u, P.n_kv_heads, P.n_q_heads);
+  const int ns = nseg * (NG + 1);  // slots: CTA first + c, then its groups and its overflow slot
+  auto slot = [&](int s) { return P.part + ((size_t)(first + s / (NG + 1) + u) * (NG + 1) + s % (NG + 1)) * PF; };
+  // normalisers, sums of p min and failure flags of every slot: lanes in parallel, then a
+  // fixed-order reduction (lane order, then a butterfly)
+  float Lh[GS], PMh[GS];
+#pragma unroll
+  for (int g = 0; g < GS; ++g) Lh[g] = PMh[g] = 0.f;
+  bool bad = false;
+  for (int s = lane; s < ns; s += 32) {
+    const float* sp = slot(s);
+    bad |= __ldcg(sp + part_flag(GS)) != 0.f;
+    if (s % (NG + 1) < NG)
+#pragma unroll
+      for (int w = 0; w < WPG; ++w)
+#pragma unroll
+        for (int g = 0; g < GS; ++g) {
+          Lh[g] += __ldcg(sp + 256 * GS + w * GS + g);
+          PMh[g] += __ldcg(sp + 256 * GS + WPG * GS + w * GS + g);
+        }
+  }
+  bad = __any_sync(0xffffffffu, bad);
+#pragma unroll
+  for (int g = 0; g < GS; ++g) {
+    Lh[g] = warp_sum(Lh[g]);
+    PMh[g] = warp_sum(PMh[g]);
+  }
   for (int h = widx; h < GS; h += nw) {
     float4 a = make_float4(0.f, 0.f, 0.f, 0.f), r = a;
+    for (int s0 = 0; s0 < ns; s0 += 4) {  // four slots' loads in flight at a time
+      float4 xa[4], xr[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        xa[j] = xr[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (s0 + j < ns) {
+          const float* sp = slot(s0 + j);
+          xa[j] = __ldcg(reinterpret_cast<const float4*>(sp + h * 128 + 4 * lane));
+          xr[j] = __ldcg(reinterpret_cast<const float4*>(sp + GS * 128 + h * 128 + 4 * lane));
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        a.x += xa[j].x; a.y += xa[j].y; a.z += xa[j].z; a.w += xa[j].w;
+        r.x += xr[j].x; r.y += xr[j].y; r.z += xr[j].z; r.w += xr[j].w;
+      }
+    }
     float L = 0.f, PM = 0.f;
-    bool bad = false;
-    for (int c = first; c < first + nseg; ++c)
-      for (int j = 0; j <= NG; ++j) {
-        const float* sp = P.part + ((size_t)(c + u) * (NG + 1) + j) * PF;
-        const float4 x = __ldcg(reinterpret_cast<const float4*>(sp + h * 128 + 4 * lane));
-        const float4 y = __ldcg(reinterpret_cast<const float4*>(sp + GS * 128 + h * 128 + 4 * lane));
-        a.x += x.x; a.y += x.y; a.z += x.z; a.w += x.w;
-        r.x += y.x; r.y += y.y; r.z += y.z; r.w += y.w;
-        if (j < NG)
-          for (int w = 0; w < WPG; ++w) {
-            L += __ldcg(sp + 256 * GS + w * GS + h);
-            PM += __ldcg(sp + 256 * GS + WPG * GS + w * GS + h);
-          }
-        bad |= __ldcg(sp + part_flag(GS)) != 0.f;
+#pragma unroll
+    for (int g = 0; g < GS; ++g)
+      if (g == h) {
+        L = Lh[g];
+        PM = PMh[g];
       }
     float x[4] = {r.x + PM, r.y + PM, r.z + PM, r.w + PM};
     if (P.rotate) {
@@ -548,15 +571,15 @@ __device__ void combine_unit(const DecodeParams& P, int u, int first, int nseg, 
 #pragma unroll
       for (int e = 0; e < 4; ++e) x[e] *= (1.0f / 128.0f);
     }
-    bad |= !(L < INFINITY);  // a logit so far above the reference that the sums overflowed
+    const bool badh = bad || !(L < INFINITY);  // a logit so far above the reference that the sums overflowed
     const float yv[4] = {a.x + x[0], a.y + x[1], a.z + x[2], a.w + x[3]};
     const size_t o = ob + (size_t)h * 128 + 4 * lane;
+    float y[4];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const float y = bad ? __int_as_float(0x7FC00000) : yv[e] / L;
-      P.out[o + e] = __float2bfloat16_rn(y);
-      if (P.out_f32) P.out_f32[o + e] = y;
-    }
+    for (int e = 0; e < 4; ++e) y[e] = badh ? __int_as_float(0x7FC00000) : yv[e] / L;
+    *reinterpret_cast<uint2*>(P.out + o) = make_uint2(pack_b2(__float2bfloat16_rn(y[0]), __float2bfloat16_rn(y[1])),
+                                                      pack_b2(__float2bfloat16_rn(y[2]), __float2bfloat16_rn(y[3])));
+    if (P.out_f32) *reinterpret_cast<float4*>(P.out_f32 + o) = make_float4(y[0], y[1], y[2], y[3]);
   }
 }
 
@@ -568,6 +591,131 @@ __device__ __forceinline__ bool count_in(const DecodeParams& P, int u, int nseg)
   const bool last = old == (unsigned)((NG + 1) * nseg - 1);
   if (last) __threadfence();
   return last;
+}
+
+// Probabilities of one token for every head: p_g = 2^(gamma S_A[a][g] + rt_g) (rt: the key-residual
+// term minus m, or -m), added into the normaliser sums.
+template <int GS, int NP>
+__device__ __forceinline__ void head_probs(float gk, const float (&sa)[GS], const float (&rt)[GS], float2 (&pe)[NP],
+                                           float2 (&l2)[NP]) {
+  if constexpr (GS == 1) {
+    const float p = exp2_approx(fmaf(gk, sa[0], rt[0]));
+    pe[0] = make_float2(p, 0.f);
+    l2[0].x += p;
+  } else {
+    const float2 gk2 = make_float2(gk, gk);
+#pragma unroll
+    for (int i2 = 0; i2 < NP; ++i2) {
+      const float2 x = __ffma2_rn(gk2, make_float2(sa[2 * i2], sa[2 * i2 + 1]), make_float2(rt[2 * i2], rt[2 * i2 + 1]));
+      pe[i2] = make_float2(exp2_approx(x.x), exp2_approx(x.y));
+      l2[i2] = __fadd2_rn(l2[i2], pe[i2]);
+    }
+  }
+}
+
+// A lane's tokens of a tile: bitmap bytes and first record indices.
+struct TokLane {
+  uint32_t kbits, vbits;
+  int rk, rv, t0;
+};
+// What the general token path reads of its tile.
+struct TokTile {
+  TileView tv;
+  uint32_t lo, nrows;
+  const float* SAt;   // anchor scores [k][GS]
+  const float* rows;  // [0,8): -m, [8,16): -inf, [16,24): sum q'
+  const float* qp;    // [GS][128] rotated query
+  float* pv;          // [R][8] p rows of the value records
+  float* W;           // [X][GS] the tile's value weights
+  float* ovf;         // [2][GS][128] overflow sums
+  float* lsum;        // [GS] the group's normaliser contributions of this path
+  const uint8_t* AV;  // the unit's anchor values (global)
+  int k, nKs, nVs;
+};
+
+// The general token path (kept out of line: a tile with records beyond the staged ones, runs
+// beyond the staged anchor-value rows, or a lane past the tile's end): the same arithmetic as
+// the fast path, with the rare cases on CUDA cores.  Everything is passed by value and the
+// normaliser goes to shared memory, so that no variable of the caller has its address taken
+// (it would then live in local memory, whose lines the small L1 here does not keep).
+template <int GS>
+__device__ __noinline__ void token_chunk_general(const TokTile tt, const TokLane tl) {
+  constexpr int NP = GS >= 2 ? GS / 2 : 1;
+  const TileView& tv = tt.tv;
+  const uint8_t* st = tv.st;
+  const int t0 = tl.t0;
+  const int nvalid = min(LCH, tv.n - t0);
+  const float* rsb = reinterpret_cast<const float*>(st + tv.cd_k);
+  const float* negrow = tt.rows;
+  const float* ninfrow = tt.rows + 8;
+  const uint32_t lo = tt.lo;
+  const int nrows = (int)tt.nrows;
+  int rkn = tl.rk, rvn = tl.rv;
+  float2 l2[NP];
+#pragma unroll
+  for (int i2 = 0; i2 < NP; ++i2) l2[i2] = make_float2(0.f, 0.f);
+  uint32_t key = *reinterpret_cast<const uint32_t*>(st + 4 * (tv.n64 + t0)) & 0xFFFFu;
+  float2 acc[NP];
+#pragma unroll
+  for (int i2 = 0; i2 < NP; ++i2) acc[i2] = make_float2(0.f, 0.f);
+  auto flush = [&](uint32_t kk, const float2 (&v)[NP]) {
+    const int ix = (int)(kk - lo);
+    float vv[GS];
+#pragma unroll
+    for (int g = 0; g < GS; ++g) vv[g] = (g & 1) ? v[g >> 1].y : v[g >> 1].x;
+    if (ix < nrows) {
+      float* w = tt.W + ix * GS;
+#pragma unroll
+      for (int g = 0; g < GS; ++g) red_local(w + g, vv[g]);
+    } else {  // beyond the staged anchor-value rows: its products on CUDA cores
+      anchor_value_add<GS>(tt.AV, (int)kk, vv, tt.ovf);
+    }
+  };
+  for (int e = 0; e < LCH; ++e) {
+    const uint32_t ek = e < nvalid ? *reinterpret_cast<const uint32_t*>(st + 4 * (t0 + e)) : 0u;
+    const uint32_t ev = e < nvalid ? *reinterpret_cast<const uint32_t*>(st + 4 * (tv.n64 + t0 + e)) : 0u;
+    const int a = min((int)(ek & 0xFFFFu), tt.k - 1);
+    float sa[GS], rt[GS];
+    load_row<GS>(tt.SAt + a * GS, sa);
+    const bool kb = (tl.kbits >> e) & 1u;
+    const int r = rkn;
+    rkn += (int)kb;
+    if (kb && r >= tt.nKs && e < nvalid) {  // beyond the staged records
+#pragma unroll
+      for (int g = 0; g < GS; ++g) rt[g] = key_record_term(tv, r, tt.qp + g * 128, tt.rows[16 + g]) + tt.rows[g];
+    } else {  // the key-residual terms, -m, or -inf for a token past the tile's end
+      load_row<GS>(e >= nvalid ? ninfrow : (kb ? rsb + r * 8 : negrow), rt);
+    }
+    const float gk = half_hi(ek), gv = half_hi(ev);
+    float2 pe[NP];
+    head_probs<GS, NP>(gk, sa, rt, pe, l2);
+    const bool vb = (tl.vbits >> e) & 1u;
+    const int rv = rvn;
+    rvn += (int)vb;
+    if (vb && e < nvalid) {
+      if (rv < tt.nVs) {
+        store_row<GS>(tt.pv + rv * 8, pe);
+      } else {  // beyond the staged records
+#pragma unroll
+        for (int g = 0; g < GS; ++g)
+          value_record_add(tv, rv, (g & 1) ? pe[g >> 1].y : pe[g >> 1].x, tt.ovf + GS * 128 + g * 128);
+      }
+    }
+    // tokens past the tile join the current run with zero weight
+    const uint32_t av = e < nvalid ? (ev & 0xFFFFu) : key;
+    if (av != key) {
+      flush(key, acc);
+      key = av;
+#pragma unroll
+      for (int i2 = 0; i2 < NP; ++i2) acc[i2] = make_float2(0.f, 0.f);
+    }
+    const float2 gv2 = make_float2(gv, gv);
+#pragma unroll
+    for (int i2 = 0; i2 < NP; ++i2) acc[i2] = __ffma2_rn(pe[i2], gv2, acc[i2]);
+  }
+  flush(key, acc);
+#pragma unroll
+  for (int g = 0; g < GS; ++g) red_local(tt.lsum + g, (g & 1) ? l2[g >> 1].y : l2[g >> 1].x);
 }
 
 // ================================ decode ============================================
@@ -586,20 +734,17 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float* SAs = reinterpret_cast<float*>(smem + P.o_sa);
   float* ovf = reinterpret_cast<float*>(smem + P.o_ovf);  // [2][GS][128]: anchor-value and value-residual overflow sums
   uint8_t* ring = smem + P.o_ring;
-  // per slot: block + anchor rows landed (full), slot free again (empty: its group's warps are
-  // done); per unit: its anchor-score table landed (sa_full), compute warps done with it (sa_free)
-  auto bar_full = [&](int s) { return smem_u32(bars + s); };
-  auto bar_empty = [&](int s) { return smem_u32(bars + NSLOT + s); };
-  const uint32_t bar_sa_full = smem_u32(bars + 2 * NSLOT), bar_sa_free = smem_u32(bars + 2 * NSLOT + 1);
+  // per group and slot: a tile block and its anchor-value rows landed (full); per unit: its
+  // anchor-score table landed (sa_full; a plain arrival when the table stays in global memory)
+  auto bar_full = [&](int g, int s) { return smem_u32(bars + g * NSG + s); };
+  const uint32_t bar_sa_full = smem_u32(bars + NG * NSG);
+  int* segcnt = reinterpret_cast<int*>(smem + P.o_misc + 4);  // groups done with a segment, in total
 
   if (tid == 0) {
-    for (int s = 0; s < NSLOT; ++s) {
-      mbar_init(bar_full(s), 1);
-      mbar_init(bar_empty(s), WPG);
-    }
+    for (int s = 0; s < NG * NSG; ++s) mbar_init(smem_u32(bars + s), 1);
     mbar_init(bar_sa_full, 1);
-    mbar_init(bar_sa_free, NCW);
     *failed = 0;
+    *segcnt = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   for (int e = tid; e < 2 * GS * 128; e += NT) ovf[e] = 0.f;
@@ -644,122 +789,26 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     return true;
   };
 
-  // =========================== producer warp ===================================
-  if (warp == W_PROD) {
-    struct InFlight {
-      int i;
-      uint32_t a, e;
-    };
-    InFlight fq[NSLOT];  // tiles whose slot may not be free yet, oldest first (lane 0)
-    int qh = 0, qn = 0;
-    uint32_t head = 0;
-    int n_cta_tiles = (int)(B1 - B0);
-    Seg sg;
-    seg_begin(sg);
-    int sigma = 0, prev_u = -1, prev_first = 0, prev_nseg = 0;
-    // the overflow sums of a finished segment into this CTA's third slot of its unit, then the
-    // unit's counter (whole warp)
-    auto flush_ovf = [&](int u, int first, int nseg) {
-      float* dst = P.part + ((size_t)(c + u) * (NG + 1) + NG) * PF;
-      for (int e = 4 * lane; e < GS * 128; e += 128) {
-        float4* oa = reinterpret_cast<float4*>(ovf + e);
-        float4* orr = reinterpret_cast<float4*>(ovf + GS * 128 + e);
-        *reinterpret_cast<float4*>(dst + e) = *oa;
-        *reinterpret_cast<float4*>(dst + GS * 128 + e) = *orr;
-        *oa = make_float4(0.f, 0.f, 0.f, 0.f);
-        *orr = make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-      if (lane == 0) dst[part_flag(GS)] = *failed ? 1.f : 0.f;
-      __syncwarp();
-      int last = 0;
-      if (lane == 0) last = count_in(P, u, nseg) ? 1 : 0;
-      if (__shfl_sync(0xffffffffu, last, 0)) {
-        __threadfence();
-        combine_unit<GS>(P, u, first, nseg, 0, 1);
-      }
-    };
-    for (;; ++sigma) {
-      const UnitView U = unit_view(P.arena, sg.u);
-      if (sigma > 0) {
-        // every compute warp is done with the previous unit's anchor scores and overflow sums
-        if (!warp_failed(failed) && !mbar_wait_w(bar_sa_free, (uint32_t)(sigma - 1) & 1u)) *failed = 1;
-        flush_ovf(prev_u, prev_first, prev_nseg);
-      }
-      if (lane == 0) {
-        if (P.smem_sa && !*failed) {
-          const uint32_t bytes = round16(4u * (uint32_t)(U.k * GS));
-          mbar_expect_tx(bar_sa_full, bytes);
-          bulk_g2s(smem_u32(SAs), P.sa + (size_t)sg.u * P.ka_stride * GS, bytes, bar_sa_full);
-        } else {
-          mbar_arrive(bar_sa_full);  // the unit's start, for the compute warps
-        }
-      }
-      for (int j = sg.jb; j < sg.je; ++j) {
-        const int i = sg.ib + (j - sg.jb), s = i % NSLOT;
-        if (lane == 0 && !*failed) {
-          const uint32_t blk0 = U.table[j], blkn = U.table[j + 1] - blk0, sr = U.table[U.nt + 1 + j];
-          const uint32_t lo = sr & 0xFFFFu, hi = sr >> 16;
-          const uint32_t staged = min(blkn, (uint32_t)P.cap);
-          const uint32_t nrows = min(hi - lo + 1u, (uint32_t)P.X);
-          const uint32_t sz = staged + 256u * nrows;
-          if (head + sz > (uint32_t)P.ring_bytes) head = 0;
-          const uint32_t a = head;
-          // wait for the in-flight tiles whose bytes overlap [a, a + sz), and for the slot's
-          // previous tile, oldest first
-          int last = -1;
-          for (int t = 0; t < qn; ++t) {
-            const InFlight& f = fq[(qh + t) % NSLOT];
-            if (f.a < a + sz && a < f.e) last = t;
-          }
-          if (qn == NSLOT && last < 0) last = 0;
-          bool ok = true;
-          for (int t = 0; t <= last && ok; ++t) {
-            const InFlight& f = fq[qh];
-            ok = mbar_wait(bar_empty(f.i % NSLOT), (uint32_t)(f.i / NSLOT) & 1u);
-            qh = (qh + 1) % NSLOT;
-            --qn;
-          }
-          if (!ok) {
-            *failed = 1;
-          } else {
-            head = a + sz;
-            fq[(qh + qn) % NSLOT] = InFlight{i, a, a + sz};
-            ++qn;
-            meta[s] = Meta{a, blk0, blkn, staged, lo, nrows, (uint32_t)j, 0u};
-            // (drop_last: a test withholds the last tile of the range)
-            if (!(P.drop_last > 0 && i == n_cta_tiles - P.drop_last)) {
-              mbar_expect_tx(bar_full(s), sz);
-              bulk_g2s(smem_u32(ring + a), U.tiles + blk0, staged, bar_full(s));
-              if (nrows) bulk_g2s(smem_u32(ring + a + staged), U.AV + (size_t)lo * 256, 256u * nrows, bar_full(s));
-            } else {
-              fq[(qh + qn - 1) % NSLOT].e = fq[(qh + qn - 1) % NSLOT].a;  // nothing in flight there
-            }
-          }
-        }
-        __syncwarp();
-      }
-      prev_u = sg.u;
-      prev_first = sg.first;
-      prev_nseg = sg.nseg;
-      if (!seg_next(sg)) break;
+  // the first unit's anchor-score table (later ones: the group that finishes the previous unit last)
+  auto start_table = [&](int u) {
+    const int k = unit_desc(P.arena, u)->n_anchors;
+    if (P.smem_sa && !*failed) {
+      const uint32_t bytes = round16(4u * (uint32_t)(k * GS));
+      mbar_expect_tx(bar_sa_full, bytes);
+      bulk_g2s(smem_u32(SAs), P.sa + (size_t)u * P.ka_stride * GS, bytes, bar_sa_full);
+    } else {
+      mbar_arrive(bar_sa_full);  // the unit's start, for the warps that wait on it
     }
-    if (!warp_failed(failed) && !mbar_wait_w(bar_sa_free, (uint32_t)sigma & 1u)) *failed = 1;
-    flush_ovf(prev_u, prev_first, prev_nseg);
-    // every copy this warp started has landed before the CTA may exit (bounded)
-    if (lane == 0)
-      for (int t = 0; t < qn; ++t) {
-        const InFlight& f = fq[(qh + t) % NSLOT];
-        if (f.e > f.a) mbar_wait(bar_full(f.i % NSLOT), (uint32_t)(f.i / NSLOT) & 1u);
-      }
-    if (lane == 0 && P.smem_sa) mbar_wait(bar_sa_full, (uint32_t)sigma & 1u);
-    return;
-  }
+  };
+  if (tid == 0) start_table(P.cta_unit[c]);
+  const int n_cta_tiles = (int)(B1 - B0);
 
   // =========================== compute groups ==================================
   const int grp = warp / WPG, wg = warp % WPG, gt = tid - grp * WPG * 32;
   uint8_t* GB = smem + P.o_grp + grp * P.grp_bytes;
   float* qp = reinterpret_cast<float*>(GB + P.g_qp);      // [GS][128] rotated query q'
-  float* rows = reinterpret_cast<float*>(GB + P.g_rows);  // [0,8): -m, [8,16): -inf, [16,24): sum q', [24,32): m
+  float* rows = reinterpret_cast<float*>(GB + P.g_rows);  // [0,8): -m, [8,16): -inf, [16,24): sum q', [24,32): m,
+                                                          // [32,40): normaliser share of the general token path
   int* lastf = reinterpret_cast<int*>(GB + P.g_red);
   float* wb = reinterpret_cast<float*>(GB + P.g_wb);      // [2][X][GS] value weights of a tile's slots
   float* pv = reinterpret_cast<float*>(GB + P.g_pv);      // [R][8] p rows of the value records, then A operands
@@ -771,10 +820,91 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   float accA[4][4], accR[4][4];  // anchor-value and value-residual sums, dims 32 wg .. 32 wg + 31
   float2 l2[NP];
   float pminv[HPL];
-  int lt = 0;  // this group's tiles so far (weight-table buffer parity)
+  int lt = 0;  // this group's tiles so far (weight-table buffer parity, stage descriptor)
+
+  // ---- the group as its own producer (warp wg = 0; lane 0 issues the copies) ----
+  // Its tiles are the CTA's tiles i = grp, grp + NG, ...; each goes, with the anchor-value rows
+  // of the value slots it covers, into this group's half of the ring, oldest first: the tile
+  // table entries of the next tile to issue are read one issue ahead, so a copy never waits on
+  // a global load.
+  const uint32_t RH = (uint32_t)P.ring_bytes / NG, rbase = (uint32_t)grp * RH;
+  Meta* gmeta = meta + grp * NSG;
+  Seg si;                         // segment of the next tile to issue
+  int ii = grp;                   // CTA-local index of the next tile to issue
+  int nis = 0, nrel = 0;          // tiles issued, tiles released (group-local)
+  uint32_t head = 0, used = 0;    // ring bytes: next free place, bytes in flight
+  uint32_t pe0 = 0, pe1 = 0, pe2 = 0;  // table entries of tile ii: block offset, next offset, slot range
+  int pj = 0;
+  const uint8_t* ptiles = nullptr;
+  const uint8_t* pav = nullptr;
+  auto prefetch = [&]() {
+    if (ii >= n_cta_tiles) return;
+    while (ii >= si.ib + (si.je - si.jb)) seg_next(si);
+    const UnitView V = unit_view(P.arena, si.u);
+    pj = si.jb + (ii - si.ib);
+    pe0 = V.table[pj];
+    pe1 = V.table[pj + 1];
+    pe2 = V.table[V.nt + 1 + pj];
+    ptiles = V.tiles;
+    pav = V.AV;
+  };
+  auto issue_more = [&]() {
+    while (ii < n_cta_tiles && nis - nrel < NSG && !warp_failed(failed)) {
+      const uint32_t blkn = pe1 - pe0, lo = pe2 & 0xFFFFu, hi = pe2 >> 16;
+      const uint32_t staged = min(blkn, (uint32_t)P.cap);
+      const uint32_t nrows = min(hi - lo + 1u, (uint32_t)P.X);
+      const uint32_t sz = staged + 256u * nrows;
+      uint32_t at = 0;
+      bool fits = true;
+      if (used == 0) {
+        at = 0;
+      } else {
+        const uint32_t tail = gmeta[nrel % NSG].ring_off - rbase;  // the oldest tile in flight
+        if (head > tail) {
+          if (head + sz <= RH) at = head;
+          else if (sz <= tail) at = 0;
+          else fits = false;
+        } else if (head < tail) {
+          at = head;
+          fits = head + sz <= tail;
+        } else {
+          fits = false;
+        }
+      }
+      if (!fits) break;
+      const int sl = nis % NSG;
+      if (lane == 0) {
+        gmeta[sl] = Meta{rbase + at, pe0, blkn, staged, lo, nrows, (uint32_t)pj, sz};
+        // (drop_last: a test withholds the last tile of the range)
+        if (P.drop_last > 0 && ii == n_cta_tiles - P.drop_last) {
+          gmeta[sl].nrows |= 0x80000000u;  // withheld: nothing in flight
+        } else {
+          const uint32_t bar = bar_full(grp, sl);
+          mbar_expect_tx(bar, sz);
+          bulk_g2s(smem_u32(ring + rbase + at), ptiles + pe0, staged, bar);
+          if (nrows) bulk_g2s(smem_u32(ring + rbase + at + staged), pav + (size_t)lo * 256, 256u * nrows, bar);
+        }
+      }
+      __syncwarp();
+      head = at + sz;
+      used += sz;
+      ++nis;
+      ii += NG;
+      prefetch();
+    }
+  };
+  auto release_to = [&](int upto) {  // this group's tiles before `upto` are done with
+    for (; nrel < upto; ++nrel) used -= gmeta[nrel % NSG].pad;
+  };
+  if (wg == 0) {
+    seg_begin(si);
+    prefetch();
+    issue_more();
+  }
   Seg sg;
   seg_begin(sg);
-  for (int sigma = 0;; ++sigma) {
+  int sigma = 0;
+  for (;; ++sigma) {
     const UnitView U = unit_view(P.arena, sg.u);
     const int k = U.k;
     // ---- segment set-up: q' rows (warp wg: heads wg, wg + 4), their sums, the reference m ----
@@ -804,6 +934,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
           rows[8 + g] = -INFINITY;
           rows[16 + g] = sg_;
           rows[24 + g] = m;
+          rows[32 + g] = 0.f;  // normaliser share of the general token path
         }
       }
     }
@@ -851,19 +982,21 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     const int i_end = sg.ib + (sg.je - sg.jb);
     int i0 = sg.ib + ((grp - sg.ib % NG) + NG) % NG;  // this group's first tile of the segment
     for (int i = i0; i < i_end; i += NG, ++lt) {
-      const int s = i % NSLOT;
-      const bool go = !warp_failed(failed) && mbar_wait_w(bar_full(s), (uint32_t)(i / NSLOT) & 1u);
+      const bool go = !warp_failed(failed) && mbar_wait_w(bar_full(grp, lt % NSG), (uint32_t)(lt / NSG) & 1u);
       if (!go) *failed = 1;
-      const Meta mt = meta[s];
+      const Meta mt = gmeta[lt % NSG];
       const uint8_t* st = ring + mt.ring_off;
       TileView tv;
       int nKs = 0, nVs = 0;
+      bool fast_tile = false;
       float* W = wb + (lt & 1) * P.X * GS;
       if (go) {
         tv = tile_view(st, mt, U);
         const uint32_t codes_staged = tv.staged > tv.cd_k ? (tv.staged - tv.cd_k) / 32u : 0u;
         nKs = min(min(tv.nk, P.R), (int)codes_staged);
         nVs = min(tv.nv, P.R);
+        fast_tile = nKs == tv.nk && nVs == tv.nv &&
+                    (int)(((reinterpret_cast<const uint32_t*>(st + 4 * tv.n64))[tv.n - 1] & 0xFFFFu) - mt.lo) < (int)mt.nrows;
         for (int e = gt; e < P.X * GS; e += WPG * 32) W[e] = 0.f;
         // ---- key residuals: q' . c of the staged key records, tensor cores; the terms
         // scale (q' . c) + min sum(q') - m are written over the records' codes ----
@@ -926,97 +1059,127 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         }
       }
       gsync();  // (A) key-residual terms written, weight table zeroed
+      if (wg == 0) {  // every warp is done with the group's previous tile: its bytes take new ones
+        release_to(lt);
+        issue_more();
+        // the next tile did not fit beside this one (the ring's free bytes are split): it is
+        // issued once this tile is done (rare)
+        if (lane == 0) lastf[2] = (nis <= lt + 1 && ii < n_cta_tiles) ? 1 : 0;
+      }
       if (go) {
         // ---- tokens: lane -> stored tokens t0 .. t0 + 7, every head ----
         const int t0 = wg * (32 * LCH) + LCH * lane;
+        TokLane tl;
         if (t0 < tv.n) {
-          const int nvalid = min(LCH, tv.n - t0);
-          const uint4 ka0 = *reinterpret_cast<const uint4*>(st + 4 * t0);
-          const uint4 ka1 = *reinterpret_cast<const uint4*>(st + 4 * t0 + 16);
-          const uint4 va0 = *reinterpret_cast<const uint4*>(st + 4 * (tv.n64 + t0));
-          const uint4 va1 = *reinterpret_cast<const uint4*>(st + 4 * (tv.n64 + t0) + 16);
-          const uint32_t ek[LCH] = {ka0.x, ka0.y, ka0.z, ka0.w, ka1.x, ka1.y, ka1.z, ka1.w};
-          const uint32_t ev[LCH] = {va0.x, va0.y, va0.z, va0.w, va1.x, va1.y, va1.z, va1.w};
           const int wi = t0 >> 6, sh = t0 & 63;
           const uint64_t wk = tv.bm(0, wi), wv = tv.bm(1, wi);
-          const uint32_t kbits = (uint32_t)(wk >> sh) & 0xFFu, vbits = (uint32_t)(wv >> sh) & 0xFFu;
-          int rkn = tv.rk(0, wi) + __popcll(wk & ((1ull << sh) - 1ull));
-          int rvn = tv.rk(1, wi) + __popcll(wv & ((1ull << sh) - 1ull));
+          tl.kbits = (uint32_t)(wk >> sh) & 0xFFu;
+          tl.vbits = (uint32_t)(wv >> sh) & 0xFFu;
+          tl.rk = tv.rk(0, wi) + __popcll(wk & ((1ull << sh) - 1ull));
+          tl.rv = tv.rk(1, wi) + __popcll(wv & ((1ull << sh) - 1ull));
+          tl.t0 = t0;
+        }
+        if (fast_tile && tv.n == T) {  // warp-uniform
+          // A full tile, every record staged, every run on a staged anchor-value row.  No shared
+          // atomics: a run that starts and ends inside a lane's tokens is stored as it is (no
+          // other lane has its slot); runs that cross lanes are merged by a segmented scan.
           const float* rsb = reinterpret_cast<const float*>(st + tv.cd_k);
-          const float* negrow = rows;
-          const float* ninfrow = rows + 8;
           const uint32_t lo = mt.lo;
-          const int nrows = (int)mt.nrows;
-          uint32_t key = ev[0] & 0xFFFFu;  // value slot of the run being summed
-          float2 acc[NP];
+          const int km1 = k - 1;
+          uint32_t kb8 = tl.kbits, vb8 = tl.vbits;
+          int rk = tl.rk, rv = tl.rv;
+          uint32_t key = *reinterpret_cast<const uint32_t*>(st + 4 * (tv.n64 + t0)) & 0xFFFFu;
+          uint32_t hk = key;  // the lane's first run (its head), kept for the merge
+          bool multi = false;  // the lane's tokens hold more than one run
+          float2 acc[NP], hs[NP];
 #pragma unroll
-          for (int i2 = 0; i2 < NP; ++i2) acc[i2] = make_float2(0.f, 0.f);
-          // a finished run's weights into the tile's table (or, beyond its staged rows, its
-          // anchor-value products into the overflow sums)
-          auto flush = [&](uint32_t kk, const float2 (&v)[NP]) {
-            const int ix = (int)(kk - lo);
-            if (ix < nrows) {
-              float* w = W + ix * GS;
+          for (int i2 = 0; i2 < NP; ++i2) acc[i2] = hs[i2] = make_float2(0.f, 0.f);
+          constexpr int TPI = GS == 8 ? 2 : 4;  // tokens per step (live registers at GS = 8)
+#pragma unroll 1
+          for (int qd = 0; qd < LCH / TPI; ++qd) {
+            uint32_t ek[TPI], ev[TPI];
+            load_words<TPI>(st + 4 * (t0 + TPI * qd), ek);
+            load_words<TPI>(st + 4 * (tv.n64 + t0 + TPI * qd), ev);
 #pragma unroll
-              for (int g = 0; g < GS; ++g) red_local(w + g, (g & 1) ? v[g >> 1].y : v[g >> 1].x);
-            } else {
-              float vv[GS];
+            for (int e = 0; e < TPI; ++e) {
+              const int a = min((int)(ek[e] & 0xFFFFu), km1);  // indices are < k by construction
+              float sa[GS], rt[GS];
+              load_row<GS>(SAt + a * GS, sa);
+              const bool kb = kb8 & 1u;
+              kb8 >>= 1;
+              load_row<GS>(kb ? rsb + rk * 8 : rows, rt);  // the key-residual terms, or -m
+              rk += (int)kb;
+              const float gk = half_hi(ek[e]), gv = half_hi(ev[e]);
+              float2 pe[NP];
+              head_probs<GS, NP>(gk, sa, rt, pe, l2);
+              const bool vb = vb8 & 1u;
+              vb8 >>= 1;
+              if (vb) store_row<GS>(pv + rv * 8, pe);
+              rv += (int)vb;
+              const uint32_t av = ev[e] & 0xFFFFu;
+              if (av != key) {  // the run of `key` ends inside this lane
+                if (!multi) {   // the lane's first run: it may continue the previous lane's
 #pragma unroll
-              for (int g = 0; g < GS; ++g) vv[g] = (g & 1) ? v[g >> 1].y : v[g >> 1].x;
-              anchor_value_add<GS>(U.AV, (int)kk, vv, ovf);
-            }
-          };
+                  for (int i2 = 0; i2 < NP; ++i2) hs[i2] = acc[i2];
+                } else {        // started and ended here: its slot is this lane's alone
+                  store_row<GS>(W + (int)(key - lo) * GS, acc);
+                }
+                multi = true;
+                key = av;
 #pragma unroll
-          for (int e = 0; e < LCH; ++e) {
-            const int a = min((int)(ek[e] & 0xFFFFu), k - 1);  // indices are < k by construction
-            float sa[GS], rt[GS];
-            load_row<GS>(SAt + a * GS, sa);
-            const bool kb = (kbits >> e) & 1u;
-            const int r = rkn;
-            rkn += (int)kb;
-            if (kb && r >= nKs && e < nvalid) {  // beyond the staged records: CUDA cores (rare)
-#pragma unroll
-              for (int g = 0; g < GS; ++g) rt[g] = key_record_term(tv, r, qp + g * 128, rows[16 + g]) + rows[g];
-            } else {  // the key-residual terms, -m, or -inf for a token past the tile's end
-              load_row<GS>(e >= nvalid ? ninfrow : (kb ? rsb + r * 8 : negrow), rt);
-            }
-            const float gk = half_hi(ek[e]), gv = half_hi(ev[e]);
-            float2 pe[NP], cw[NP];
-#pragma unroll
-            for (int i2 = 0; i2 < NP; ++i2) {
-              const float2 s2 = make_float2(sa[2 * i2], GS >= 2 ? sa[2 * i2 + 1] : 0.f);
-              const float2 r2 = make_float2(rt[2 * i2], GS >= 2 ? rt[2 * i2 + 1] : -INFINITY);
-              const float2 x = f2fma(make_float2(gk, gk), s2, r2);
-              const float2 p = make_float2(exp2_approx(x.x), GS >= 2 ? exp2_approx(x.y) : 0.f);
-              l2[i2] = f2add(l2[i2], p);
-              cw[i2] = make_float2(p.x * gv, p.y * gv);
-              pe[i2] = p;
-            }
-            const bool vb = (vbits >> e) & 1u;
-            const int rv = rvn;
-            rvn += (int)vb;
-            if (vb && e < nvalid) {
-              if (rv < nVs) {
-                store_row<GS>(pv + rv * 8, pe);
-              } else {  // beyond the staged records: CUDA cores (rare)
-#pragma unroll
-                for (int g = 0; g < GS; ++g)
-                  value_record_add(tv, rv, (g & 1) ? pe[g >> 1].y : pe[g >> 1].x, ovf + GS * 128 + g * 128);
+                for (int i2 = 0; i2 < NP; ++i2) acc[i2] = make_float2(0.f, 0.f);
               }
-            }
-            // tokens past the tile join the current run with zero weight
-            const uint32_t av = e < nvalid ? (ev[e] & 0xFFFFu) : key;
-            if (av != key) {
-              flush(key, acc);
-              key = av;
+              const float2 gv2 = make_float2(gv, gv);
 #pragma unroll
-              for (int i2 = 0; i2 < NP; ++i2) acc[i2] = cw[i2];
-            } else {
-#pragma unroll
-              for (int i2 = 0; i2 < NP; ++i2) acc[i2] = f2add(acc[i2], cw[i2]);
+              for (int i2 = 0; i2 < NP; ++i2) acc[i2] = __ffma2_rn(pe[i2], gv2, acc[i2]);
             }
           }
-          flush(key, acc);
+          // merge across lanes: the next lane's head continues this lane's last run when their
+          // slots match; a head that does not continue the previous lane's run is complete
+          const uint32_t ptk = __shfl_up_sync(0xffffffffu, key, 1);
+          const uint32_t nhk = __shfl_down_sync(0xffffffffu, hk, 1);
+          const bool nmulti = __shfl_down_sync(0xffffffffu, (int)multi, 1) != 0;
+          const bool take_next = lane < 31 && nmulti && nhk == key;
+#pragma unroll
+          for (int i2 = 0; i2 < NP; ++i2) {
+            const float2 nh = make_float2(__shfl_down_sync(0xffffffffu, hs[i2].x, 1),
+                                          __shfl_down_sync(0xffffffffu, hs[i2].y, 1));
+            if (take_next) acc[i2] = __fadd2_rn(acc[i2], nh);
+          }
+          if (multi && !(lane > 0 && ptk == hk)) {
+            float* w = W + (int)(hk - lo) * GS;
+            if (lane == 0) {  // may continue the previous warp's last run
+#pragma unroll
+              for (int g = 0; g < GS; ++g) red_local(w + g, (g & 1) ? hs[g >> 1].y : hs[g >> 1].x);
+            } else {
+              store_row<GS>(w, hs);
+            }
+          }
+          // segmented inclusive scan of the last runs over lanes with equal slots
+#pragma unroll
+          for (int d = 1; d < 32; d <<= 1) {
+            const uint32_t kd = __shfl_up_sync(0xffffffffu, key, d);
+            const bool add = lane >= d && kd == key;
+#pragma unroll
+            for (int i2 = 0; i2 < NP; ++i2) {
+              const float2 vd = make_float2(__shfl_up_sync(0xffffffffu, acc[i2].x, d),
+                                            __shfl_up_sync(0xffffffffu, acc[i2].y, d));
+              if (add) acc[i2] = __fadd2_rn(acc[i2], vd);
+            }
+          }
+          const uint32_t nkey = __shfl_down_sync(0xffffffffu, key, 1);
+          const uint32_t key0 = __shfl_sync(0xffffffffu, key, 0);
+          if (lane == 31 || nkey != key) {  // the last lane of a segment holds its total
+            float* w = W + (int)(key - lo) * GS;
+            if (lane == 31 || key == key0) {  // the warp's first or last run: shared with a neighbour warp
+#pragma unroll
+              for (int g = 0; g < GS; ++g) red_local(w + g, (g & 1) ? acc[g >> 1].y : acc[g >> 1].x);
+            } else {
+              store_row<GS>(w, acc);
+            }
+          }
+        } else if (t0 < tv.n) {
+          token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, rows + 32, U.AV, k, nKs, nVs}, tl);
         }
       }
       gsync();  // (B) the tile's weights and p rows are complete
@@ -1112,12 +1275,14 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
           }
         }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(bar_empty(s));
+      if (lastf[2]) {  // (written before barrier C by warp 0, the same for every warp)
+        gsync();
+        if (wg == 0) {
+          release_to(lt + 1);
+          issue_more();
+        }
+      }
     }
-    // this warp is done with the unit's anchor scores and overflow sums
-    __syncwarp();
-    if (lane == 0) mbar_arrive(bar_sa_free);
 
     // ---- the group's partial for this unit into its slot, then the unit's counter ----
     {
@@ -1135,7 +1300,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
       for (int g = 0; g < GS; ++g) {
         const float sl = warp_sum((g & 1) ? l2[g >> 1].y : l2[g >> 1].x);
-        if (lane == 0) dst[256 * GS + wg * GS + g] = sl;
+        if (lane == 0) dst[256 * GS + wg * GS + g] = sl + (wg == 0 ? rows[32 + g] : 0.f);
       }
 #pragma unroll
       for (int i2 = 0; i2 < HPL; ++i2) {
@@ -1155,9 +1320,54 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         __threadfence();
         combine_unit<GS>(P, sg.u, sg.first, sg.nseg, wg, WPG);
       }
-      gsync();  // lastf and the set-up buffers are reused by the next segment
+      gsync();  // lastf is reused below
     }
-    if (!seg_next(sg)) break;
+    if (wg == 0) {  // the segment's last tile is done with: top the ring up
+      release_to(lt);
+      issue_more();
+    }
+    // ---- the group that finishes the segment last (the other has finished its tiles and its
+    // overflow sums) stores the CTA's overflow sums into the third slot, counts it in, and
+    // starts the next unit's anchor-score table ----
+    if (gt == 0) {
+      __threadfence_block();
+      lastf[1] = atomicAdd(segcnt, 1) % NG == NG - 1 ? 1 : 0;
+      __threadfence_block();
+    }
+    gsync();
+    const bool has_next = sg.t0 + sg.je < B1;
+    if (lastf[1]) {
+      float* dst = P.part + ((size_t)(c + sg.u) * (NG + 1) + NG) * PF;
+      for (int e = 4 * gt; e < GS * 128; e += 4 * WPG * 32) {
+        float4* oa = reinterpret_cast<float4*>(ovf + e);
+        float4* orr = reinterpret_cast<float4*>(ovf + GS * 128 + e);
+        *reinterpret_cast<float4*>(dst + e) = *oa;
+        *reinterpret_cast<float4*>(dst + GS * 128 + e) = *orr;
+        *oa = make_float4(0.f, 0.f, 0.f, 0.f);
+        *orr = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+      gsync();
+      if (gt == 0) {
+        dst[part_flag(GS)] = *failed ? 1.f : 0.f;
+        lastf[0] = count_in(P, sg.u, sg.nseg) ? 1 : 0;
+        if (has_next) start_table(sg.u + 1);  // the overflow sums are clear for it
+      }
+      gsync();
+      if (lastf[0]) {
+        __threadfence();
+        combine_unit<GS>(P, sg.u, sg.first, sg.nseg, wg, WPG);
+      }
+    }
+    gsync();  // lastf and the set-up buffers are reused by the next segment
+    if (!has_next) break;
+    seg_next(sg);
+  }
+  // every copy this group started has landed before the CTA may exit (bounded; they all have
+  // unless a wait ran out)
+  if (wg == 0 && lane == 0) {
+    for (int t = max(0, nis - NSG); t < nis; ++t)
+      if (!(gmeta[t % NSG].nrows >> 31)) mbar_wait(bar_full(grp, t % NSG), (uint32_t)(t / NSG) & 1u);
+    if (grp == 0) mbar_wait(bar_sa_full, (uint32_t)sigma & 1u);
   }
 }
 
@@ -1217,7 +1427,7 @@ struct Plan {
 };
 
 // Shared-memory carve-up for (R, X, table in shared memory or not); false if the ring
-// would hold fewer than `min_tiles` of the largest staged tiles.
+// would hold fewer than `min_tiles` of the largest staged tiles per group.
 bool make_plan_rx(const Layout& L, int GS, int R, int X, bool smem_sa, int smem_optin, int min_tiles, Plan* out) {
   DecodeParams& P = out->P;
   P.R = R;
@@ -1231,8 +1441,8 @@ bool make_plan_rx(const Layout& L, int GS, int R, int X, bool smem_sa, int smem_
     off = align128(off + bytes);
     return (int)o;
   };
-  P.o_bar = take((2 * NSLOT + 2) * 8);
-  P.o_meta = take(NSLOT * sizeof(Meta));
+  P.o_bar = take((NG * NSG + 1) * 8);
+  P.o_meta = take(NG * NSG * sizeof(Meta));
   P.o_misc = take(16);
   P.o_sa = take(smem_sa ? (size_t)P.ka_stride * GS * 4 : 0);
   P.o_ovf = take((size_t)2 * GS * 128 * 4);
@@ -1244,7 +1454,7 @@ bool make_plan_rx(const Layout& L, int GS, int R, int X, bool smem_sa, int smem_
     return (int)o;
   };
   P.g_qp = gtake((size_t)GS * 128 * 4);
-  P.g_rows = gtake(32 * 4);
+  P.g_rows = gtake(48 * 4);
   P.g_red = gtake(16);
   P.g_wb = gtake((size_t)2 * X * GS * 4);
   P.g_pv = gtake((size_t)R * 32);
@@ -1254,26 +1464,26 @@ bool make_plan_rx(const Layout& L, int GS, int R, int X, bool smem_sa, int smem_
   P.o_ring = (int)off;
   const long long room = (long long)smem_optin - (long long)P.o_ring - kRingSlack;
   const long long tile_max = (long long)P.cap + 256LL * X;
-  if (room < (long long)min_tiles * tile_max) return false;
+  if (room / NG < (long long)min_tiles * tile_max) return false;  // each group's half of the ring
   P.ring_bytes = (int)(room & ~127LL);
   out->smem = (size_t)P.o_ring + (size_t)P.ring_bytes + kRingSlack;
   return true;
 }
 
 // Preference: the anchor-score table in shared memory (the token gathers' fast path), with
-// room for three, then two of the largest staged tiles, staged counts trimmed from their full
-// values towards the mean (records first, then anchor-value rows: a run beyond those takes
-// the slowest fallback); then the table in global memory (gathers through L1 and L2) the
-// same way; then anything that holds two tiles, then one.
+// room for two, then one of the largest staged tiles in each group's half of the ring, staged
+// counts trimmed from their full values towards the mean (records first, then anchor-value
+// rows: a run beyond those takes the slowest fallback); then the table in global memory
+// (gathers through L1 and L2) the same way; then anything that holds one tile per group.
 bool make_plan(const Layout& L, int GS, int smem_optin, Plan* out, std::string* why) {
   const int R0 = full_r(L), X0 = full_x(L);
   const int Rmin = std::max(16, ((R0 * 3 / 4) + 15) & ~15), Xmin = std::max(16, ((X0 * 3 / 4) + 15) & ~15);
   for (int sa = 1; sa >= 0; --sa)
-    for (int min_tiles : {3, 2})
+    for (int min_tiles : {2, 1})
       for (int X = X0; X >= Xmin; X -= 16)
         for (int R = R0; R >= Rmin; R -= 16)
           if (make_plan_rx(L, GS, R, X, sa == 1, smem_optin, min_tiles, out)) return true;
-  for (int min_tiles : {2, 1})
+  for (int min_tiles : {1})
     for (int X = X0; X >= 16; X -= 16)
       for (int R = R0; R >= 16; R -= 16)
         if (make_plan_rx(L, GS, R, X, false, smem_optin, min_tiles, out)) return true;
