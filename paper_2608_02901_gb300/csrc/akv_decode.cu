@@ -386,6 +386,33 @@ __device__ __noinline__ void anchor_value_add(const uint8_t* AV, int anchor, con
   }
 }
 
+// Anchor-score table of a unit, ka rows: [a][GS] floats, except at GS = 8, where heads 0-3 and
+// 4-7 are two arrays [2][ka][4]: a gathered 16-byte half-row then lies in any of the eight
+// 16-byte bank groups of shared memory (a 32-byte row would start in only four of them).
+template <int GS>
+__device__ __forceinline__ size_t sa_at(int a, int g, int ka) {
+  if constexpr (GS == 8) return (size_t)(g >> 2) * ka * 4 + (size_t)a * 4 + (g & 3);
+  else return (size_t)a * GS + g;
+}
+template <int GS>
+__device__ __forceinline__ void load_sa_row(const float* t, int a, int ka, float (&out)[GS]) {
+  if constexpr (GS == 8) {
+    const float4 v = *reinterpret_cast<const float4*>(t + a * 4), w = *reinterpret_cast<const float4*>(t + (ka + a) * 4);
+    out[0] = v.x; out[1] = v.y; out[2] = v.z; out[3] = v.w;
+    out[4] = w.x; out[5] = w.y; out[6] = w.z; out[7] = w.w;
+  } else {
+    if constexpr (GS == 4) {
+      const float4 v = *reinterpret_cast<const float4*>(t + a * 4);
+      out[0] = v.x; out[1] = v.y; out[2] = v.z; out[3] = v.w;
+    } else if constexpr (GS == 2) {
+      const float2 v = *reinterpret_cast<const float2*>(t + a * 2);
+      out[0] = v.x; out[1] = v.y;
+    } else {
+      out[0] = t[a];
+    }
+  }
+}
+
 // N consecutive 32-bit words (4 N-byte aligned) from shared memory.
 template <int N>
 __device__ __forceinline__ void load_words(const uint8_t* p, uint32_t (&w)[N]) {
@@ -477,11 +504,11 @@ __global__ void __launch_bounds__(128) akv_scores_kernel(const ScoreParams P) {
       if (a < k) {
         const float s0 = dd[2 * h] * P.scale_log2, s1 = dd[2 * h + 1] * P.scale_log2;
         if (g0 < GS) {
-          sa[(size_t)a * GS + g0] = s0;
+          sa[sa_at<GS>(a, g0, P.ka_stride)] = s0;
           mx0 = fmaxf(mx0, s0);
         }
         if (g0 + 1 < GS) {
-          sa[(size_t)a * GS + g0 + 1] = s1;
+          sa[sa_at<GS>(a, g0 + 1, P.ka_stride)] = s1;
           mx1 = fmaxf(mx1, s1);
         }
       }
@@ -630,7 +657,7 @@ struct TokTile {
   float* ovf;         // [2][GS][128] overflow sums
   float* lsum;        // [GS] the group's normaliser contributions of this path
   const uint8_t* AV;  // the unit's anchor values (global)
-  int k, nKs, nVs;
+  int k, nKs, nVs, ka;
 };
 
 // The general token path (kept out of line: a tile with records beyond the staged ones, runs
@@ -676,15 +703,21 @@ __device__ __noinline__ void token_chunk_general(const TokTile tt, const TokLane
     const uint32_t ev = e < nvalid ? *reinterpret_cast<const uint32_t*>(st + 4 * (tv.n64 + t0 + e)) : 0u;
     const int a = min((int)(ek & 0xFFFFu), tt.k - 1);
     float sa[GS], rt[GS];
-    load_row<GS>(tt.SAt + a * GS, sa);
+    load_sa_row<GS>(tt.SAt, a, tt.ka, sa);
     const bool kb = (tl.kbits >> e) & 1u;
     const int r = rkn;
     rkn += (int)kb;
     if (kb && r >= tt.nKs && e < nvalid) {  // beyond the staged records
 #pragma unroll
       for (int g = 0; g < GS; ++g) rt[g] = key_record_term(tv, r, tt.qp + g * 128, tt.rows[16 + g]) + tt.rows[g];
-    } else {  // the key-residual terms, -m, or -inf for a token past the tile's end
-      load_row<GS>(e >= nvalid ? ninfrow : (kb ? rsb + r * 8 : negrow), rt);
+    } else {  // the key-residual terms minus m, -m, or -inf for a token past the tile's end
+      load_row<GS>(e >= nvalid ? ninfrow : negrow, rt);
+      if (kb && e < nvalid) {
+        float rs[GS];
+        load_row<GS>(rsb + r * 8, rs);
+#pragma unroll
+        for (int g = 0; g < GS; ++g) rt[g] += rs[g];
+      }
     }
     const float gk = half_hi(ek), gv = half_hi(ev);
     float2 pe[NP];
@@ -793,9 +826,17 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   auto start_table = [&](int u) {
     const int k = unit_desc(P.arena, u)->n_anchors;
     if (P.smem_sa && !*failed) {
-      const uint32_t bytes = round16(4u * (uint32_t)(k * GS));
-      mbar_expect_tx(bar_sa_full, bytes);
-      bulk_g2s(smem_u32(SAs), P.sa + (size_t)u * P.ka_stride * GS, bytes, bar_sa_full);
+      const float* src = P.sa + (size_t)u * P.ka_stride * GS;
+      if (GS == 8) {  // the two four-head arrays, k rows of each
+        const uint32_t half = 16u * (uint32_t)k;
+        mbar_expect_tx(bar_sa_full, 2 * half);
+        bulk_g2s(smem_u32(SAs), src, half, bar_sa_full);
+        bulk_g2s(smem_u32(SAs + (size_t)P.ka_stride * 4), src + (size_t)P.ka_stride * 4, half, bar_sa_full);
+      } else {
+        const uint32_t bytes = round16(4u * (uint32_t)(k * GS));
+        mbar_expect_tx(bar_sa_full, bytes);
+        bulk_g2s(smem_u32(SAs), src, bytes, bar_sa_full);
+      }
     } else {
       mbar_arrive(bar_sa_full);  // the unit's start, for the warps that wait on it
     }
@@ -827,9 +868,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   // of the value slots it covers, into this group's half of the ring, oldest first: the tile
   // table entries of the next tile to issue are read one issue ahead, so a copy never waits on
   // a global load.
-  const uint32_t RH = (uint32_t)P.ring_bytes / NG, rbase = (uint32_t)grp * RH;
+  const uint32_t RH = ((uint32_t)P.ring_bytes / NG) & ~127u, rbase = (uint32_t)grp * RH;  // 128-byte aligned halves
   Meta* gmeta = meta + grp * NSG;
-  Seg si;                         // segment of the next tile to issue
+  Seg si{};                       // segment of the next tile to issue
   int ii = grp;                   // CTA-local index of the next tile to issue
   int nis = 0, nrel = 0;          // tiles issued, tiles released (group-local)
   uint32_t head = 0, used = 0;    // ring bytes: next free place, bytes in flight
@@ -1050,7 +1091,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
                   for (int e = 0; e < 2; ++e) {
                     const int g = 2 * c4 + e;
-                    if (g < GS) rsb[sl * 8 + g] = half_hi(smn) * rows[16 + g] + half_lo(smn) * v[2 * hr + e] + rows[g];
+                    if (g < GS) rsb[sl * 8 + g] = half_hi(smn) * rows[16 + g] + half_lo(smn) * v[2 * hr + e];
                   }
                 }
               }
@@ -1094,7 +1135,12 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
           float2 acc[NP], hs[NP];
 #pragma unroll
           for (int i2 = 0; i2 < NP; ++i2) acc[i2] = hs[i2] = make_float2(0.f, 0.f);
-          constexpr int TPI = GS == 8 ? 2 : 4;  // tokens per step (live registers at GS = 8)
+          float2 negm2[NP];  // -m: the logit offset of every token
+#pragma unroll
+          for (int i2 = 0; i2 < NP; ++i2) negm2[i2] = make_float2(rows[2 * i2], GS >= 2 ? rows[2 * i2 + 1] : 0.f);
+          constexpr int TPI = 4;  // stream words per load (16 bytes)
+          // the table pointer as shared memory (32-bit addressing, shared loads) or global memory
+          auto token_loop = [&](const float* SAtab) {
 #pragma unroll 1
           for (int qd = 0; qd < LCH / TPI; ++qd) {
             uint32_t ek[TPI], ev[TPI];
@@ -1103,48 +1149,67 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
             for (int e = 0; e < TPI; ++e) {
               const int a = min((int)(ek[e] & 0xFFFFu), km1);  // indices are < k by construction
-              float sa[GS], rt[GS];
-              load_row<GS>(SAt + a * GS, sa);
+              float sa[GS];
+              load_sa_row<GS>(SAtab, a, P.ka_stride, sa);
               const bool kb = kb8 & 1u;
               kb8 >>= 1;
-              load_row<GS>(kb ? rsb + rk * 8 : rows, rt);  // the key-residual terms, or -m
-              rk += (int)kb;
               const float gk = half_hi(ek[e]), gv = half_hi(ev[e]);
+              // logits gamma S_A - m, plus the key-residual term for the lanes whose token has one
+              float2 x[NP];
+              const float2 gk2 = make_float2(gk, gk);
+#pragma unroll
+              for (int i2 = 0; i2 < NP; ++i2)
+                x[i2] = __ffma2_rn(gk2, make_float2(sa[2 * i2], GS >= 2 ? sa[2 * i2 + 1] : 0.f), negm2[i2]);
+              if (kb) {
+                float rs[GS];
+                load_row<GS>(rsb + rk * 8, rs);
+#pragma unroll
+                for (int i2 = 0; i2 < NP; ++i2) x[i2] = __fadd2_rn(x[i2], make_float2(rs[2 * i2], GS >= 2 ? rs[2 * i2 + 1] : 0.f));
+              }
+              rk += (int)kb;
               float2 pe[NP];
-              head_probs<GS, NP>(gk, sa, rt, pe, l2);
+#pragma unroll
+              for (int i2 = 0; i2 < NP; ++i2) {
+                pe[i2] = make_float2(exp2_approx(x[i2].x), GS >= 2 ? exp2_approx(x[i2].y) : 0.f);
+                l2[i2] = __fadd2_rn(l2[i2], pe[i2]);
+              }
               const bool vb = vb8 & 1u;
               vb8 >>= 1;
               if (vb) store_row<GS>(pv + rv * 8, pe);
               rv += (int)vb;
+              // the run of `key` ends here when the slot changes (branch-free): the lane's first
+              // run is kept as its head (it may continue the previous lane's); a later one started
+              // and ended in this lane, so its slot is this lane's alone and is stored as it is
               const uint32_t av = ev[e] & 0xFFFFu;
-              if (av != key) {  // the run of `key` ends inside this lane
-                if (!multi) {   // the lane's first run: it may continue the previous lane's
-#pragma unroll
-                  for (int i2 = 0; i2 < NP; ++i2) hs[i2] = acc[i2];
-                } else {        // started and ended here: its slot is this lane's alone
-                  store_row<GS>(W + (int)(key - lo) * GS, acc);
-                }
-                multi = true;
-                key = av;
-#pragma unroll
-                for (int i2 = 0; i2 < NP; ++i2) acc[i2] = make_float2(0.f, 0.f);
-              }
+              const bool chg = av != key;
+              if (chg && multi) store_row<GS>(W + (int)(key - lo) * GS, acc);
+              const float f_first = (chg && !multi) ? 1.f : 0.f, f_keep = chg ? 0.f : 1.f;
+              const float2 first2 = make_float2(f_first, f_first), keep2 = make_float2(f_keep, f_keep);
               const float2 gv2 = make_float2(gv, gv);
 #pragma unroll
-              for (int i2 = 0; i2 < NP; ++i2) acc[i2] = __ffma2_rn(pe[i2], gv2, acc[i2]);
+              for (int i2 = 0; i2 < NP; ++i2) {
+                hs[i2] = __ffma2_rn(acc[i2], first2, hs[i2]);
+                acc[i2] = __ffma2_rn(pe[i2], gv2, __fmul2_rn(acc[i2], keep2));
+              }
+              multi |= chg;
+              key = av;
             }
           }
+          };
+          if (P.smem_sa) token_loop(SAs);
+          else token_loop(P.sa + (size_t)sg.u * P.ka_stride * GS);
           // merge across lanes: the next lane's head continues this lane's last run when their
           // slots match; a head that does not continue the previous lane's run is complete
           const uint32_t ptk = __shfl_up_sync(0xffffffffu, key, 1);
           const uint32_t nhk = __shfl_down_sync(0xffffffffu, hk, 1);
           const bool nmulti = __shfl_down_sync(0xffffffffu, (int)multi, 1) != 0;
-          const bool take_next = lane < 31 && nmulti && nhk == key;
+          const float f_tn = (lane < 31 && nmulti && nhk == key) ? 1.f : 0.f;
+          const float2 tn2 = make_float2(f_tn, f_tn);
 #pragma unroll
           for (int i2 = 0; i2 < NP; ++i2) {
             const float2 nh = make_float2(__shfl_down_sync(0xffffffffu, hs[i2].x, 1),
                                           __shfl_down_sync(0xffffffffu, hs[i2].y, 1));
-            if (take_next) acc[i2] = __fadd2_rn(acc[i2], nh);
+            acc[i2] = __ffma2_rn(nh, tn2, acc[i2]);
           }
           if (multi && !(lane > 0 && ptk == hk)) {
             float* w = W + (int)(hk - lo) * GS;
@@ -1159,12 +1224,13 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
           for (int d = 1; d < 32; d <<= 1) {
             const uint32_t kd = __shfl_up_sync(0xffffffffu, key, d);
-            const bool add = lane >= d && kd == key;
+            const float f_add = (lane >= d && kd == key) ? 1.f : 0.f;
+            const float2 add2 = make_float2(f_add, f_add);
 #pragma unroll
             for (int i2 = 0; i2 < NP; ++i2) {
               const float2 vd = make_float2(__shfl_up_sync(0xffffffffu, acc[i2].x, d),
                                             __shfl_up_sync(0xffffffffu, acc[i2].y, d));
-              if (add) acc[i2] = __fadd2_rn(acc[i2], vd);
+              acc[i2] = __ffma2_rn(vd, add2, acc[i2]);
             }
           }
           const uint32_t nkey = __shfl_down_sync(0xffffffffu, key, 1);
@@ -1179,7 +1245,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             }
           }
         } else if (t0 < tv.n) {
-          token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, rows + 32, U.AV, k, nKs, nVs}, tl);
+          token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, rows + 32, U.AV, k, nKs, nVs, P.ka_stride}, tl);
         }
       }
       gsync();  // (B) the tile's weights and p rows are complete
@@ -1464,7 +1530,7 @@ bool make_plan_rx(const Layout& L, int GS, int R, int X, bool smem_sa, int smem_
   P.o_ring = (int)off;
   const long long room = (long long)smem_optin - (long long)P.o_ring - kRingSlack;
   const long long tile_max = (long long)P.cap + 256LL * X;
-  if (room / NG < (long long)min_tiles * tile_max) return false;  // each group's half of the ring
+  if (((room / NG) & ~127LL) < (long long)min_tiles * tile_max) return false;  // each group's part of the ring
   P.ring_bytes = (int)(room & ~127LL);
   out->smem = (size_t)P.o_ring + (size_t)P.ring_bytes + kRingSlack;
   return true;
