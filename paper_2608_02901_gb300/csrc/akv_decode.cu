@@ -73,9 +73,11 @@ constexpr unsigned long long kWaitNs = 2000000000ull;  // an mbarrier wait gives
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint32_t F_MAX = tile_fixed_bytes(T);  // streams, bitmaps, rank words of a full tile
 
-// floats of one partial slot: A [GS][128], R [GS][128], l [WPG][GS], pm [WPG][GS], flag, pad
-__host__ __device__ constexpr int part_floats(int GS) { return 256 * GS + 2 * WPG * GS + 4; }
-__host__ __device__ constexpr int part_flag(int GS) { return 256 * GS + 2 * WPG * GS; }
+// floats of one CTA's partial slot for a unit: numerator y [GS][128] (the inverse rotation already
+// applied), normaliser l [GS] (8 places), failure flag, pad to 16 bytes
+__host__ __device__ constexpr int part_floats(int GS) { return 128 * GS + 12; }
+__host__ __device__ constexpr int part_l(int GS) { return 128 * GS; }
+__host__ __device__ constexpr int part_flag(int GS) { return 128 * GS + 8; }
 
 struct ScoreParams {
   const uint8_t* arena;
@@ -539,67 +541,40 @@ __device__ void combine_unit(const DecodeParams& P, int u, int first, int nseg, 
   const int lane = threadIdx.x & 31;
   constexpr int PF = part_floats(GS);
   const size_t ob = qrow_base(u, P.n_kv_heads, P.n_q_heads);
-  const int ns = nseg * (NG + 1);  // slots: CTA first + c, then its groups and its overflow slot
-  auto slot = [&](int s) { return P.part + ((size_t)(first + s / (NG + 1) + u) * (NG + 1) + s % (NG + 1)) * PF; };
-  // normalisers, sums of p min and failure flags of every slot: lanes in parallel, then a
-  // fixed-order reduction (lane order, then a butterfly)
-  float Lh[GS], PMh[GS];
+  auto slot = [&](int s) { return P.part + (size_t)(first + s + u) * PF; };  // CTA first + s
+  // normalisers and failure flags of every slot: lanes in parallel, then a fixed-order reduction
+  float Lh[GS];
 #pragma unroll
-  for (int g = 0; g < GS; ++g) Lh[g] = PMh[g] = 0.f;
+  for (int g = 0; g < GS; ++g) Lh[g] = 0.f;
   bool bad = false;
-  for (int s = lane; s < ns; s += 32) {
+  for (int s = lane; s < nseg; s += 32) {
     const float* sp = slot(s);
     bad |= __ldcg(sp + part_flag(GS)) != 0.f;
-    if (s % (NG + 1) < NG)
 #pragma unroll
-      for (int w = 0; w < WPG; ++w)
-#pragma unroll
-        for (int g = 0; g < GS; ++g) {
-          Lh[g] += __ldcg(sp + 256 * GS + w * GS + g);
-          PMh[g] += __ldcg(sp + 256 * GS + WPG * GS + w * GS + g);
-        }
+    for (int g = 0; g < GS; ++g) Lh[g] += __ldcg(sp + part_l(GS) + g);
   }
   bad = __any_sync(0xffffffffu, bad);
 #pragma unroll
-  for (int g = 0; g < GS; ++g) {
-    Lh[g] = warp_sum(Lh[g]);
-    PMh[g] = warp_sum(PMh[g]);
-  }
+  for (int g = 0; g < GS; ++g) Lh[g] = warp_sum(Lh[g]);
   for (int h = widx; h < GS; h += nw) {
-    float4 a = make_float4(0.f, 0.f, 0.f, 0.f), r = a;
-    for (int s0 = 0; s0 < ns; s0 += 4) {  // four slots' loads in flight at a time
-      float4 xa[4], xr[4];
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int s0 = 0; s0 < nseg; s0 += 8) {  // eight slots' loads in flight at a time
+      float4 xa[8];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        xa[j] = xr[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (s0 + j < ns) {
-          const float* sp = slot(s0 + j);
-          xa[j] = __ldcg(reinterpret_cast<const float4*>(sp + h * 128 + 4 * lane));
-          xr[j] = __ldcg(reinterpret_cast<const float4*>(sp + GS * 128 + h * 128 + 4 * lane));
-        }
-      }
+      for (int j = 0; j < 8; ++j)
+        xa[j] = s0 + j < nseg ? __ldcg(reinterpret_cast<const float4*>(slot(s0 + j) + h * 128 + 4 * lane))
+                              : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
+      for (int j = 0; j < 8; ++j) {
         a.x += xa[j].x; a.y += xa[j].y; a.z += xa[j].z; a.w += xa[j].w;
-        r.x += xr[j].x; r.y += xr[j].y; r.z += xr[j].z; r.w += xr[j].w;
       }
     }
-    float L = 0.f, PM = 0.f;
+    float L = 0.f;
 #pragma unroll
     for (int g = 0; g < GS; ++g)
-      if (g == h) {
-        L = Lh[g];
-        PM = PMh[g];
-      }
-    float x[4] = {r.x + PM, r.y + PM, r.z + PM, r.w + PM};
-    if (P.rotate) {
-      warp_wht128(x, lane);
-      apply_signs(x, lane, P.sign_lo, P.sign_hi);
-#pragma unroll
-      for (int e = 0; e < 4; ++e) x[e] *= (1.0f / 128.0f);
-    }
+      if (g == h) L = Lh[g];
     const bool badh = bad || !(L < INFINITY);  // a logit so far above the reference that the sums overflowed
-    const float yv[4] = {a.x + x[0], a.y + x[1], a.z + x[2], a.w + x[3]};
+    const float yv[4] = {a.x, a.y, a.z, a.w};
     const size_t o = ob + (size_t)h * 128 + 4 * lane;
     float y[4];
 #pragma unroll
@@ -615,7 +590,7 @@ __device__ void combine_unit(const DecodeParams& P, int u, int first, int nseg, 
 __device__ __forceinline__ bool count_in(const DecodeParams& P, int u, int nseg) {
   __threadfence();
   const unsigned old = atomicAdd(P.cnt + u, 1u);
-  const bool last = old == (unsigned)((NG + 1) * nseg - 1);
+  const bool last = old == (unsigned)(nseg - 1);
   if (last) __threadfence();
   return last;
 }
@@ -655,7 +630,7 @@ struct TokTile {
   float* pv;          // [R][8] p rows of the value records
   float* W;           // [X][GS] the tile's value weights
   float* ovf;         // [2][GS][128] overflow sums
-  float* lsum;        // [GS] the group's normaliser contributions of this path
+  float* lsum;        // [GS] the CTA's normaliser sums (this path adds its share there)
   const uint8_t* AV;  // the unit's anchor values (global)
   int k, nKs, nVs, ka;
 };
@@ -780,7 +755,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     *segcnt = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  for (int e = tid; e < 2 * GS * 128; e += NT) ovf[e] = 0.f;
+  for (int e = tid; e < 2 * GS * 128 + 16; e += NT) ovf[e] = 0.f;  // (the CTA's sums start at zero)
   // zeroed p rows: rows past a tile's records are read (and multiplied by zero codes)
   for (int gi = 0; gi < NG; ++gi) {
     float* pvz = reinterpret_cast<float*>(smem + P.o_grp + gi * P.grp_bytes + P.g_pv);
@@ -848,8 +823,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   const int grp = warp / WPG, wg = warp % WPG, gt = tid - grp * WPG * 32;
   uint8_t* GB = smem + P.o_grp + grp * P.grp_bytes;
   float* qp = reinterpret_cast<float*>(GB + P.g_qp);      // [GS][128] rotated query q'
-  float* rows = reinterpret_cast<float*>(GB + P.g_rows);  // [0,8): -m, [8,16): -inf, [16,24): sum q', [24,32): m,
-                                                          // [32,40): normaliser share of the general token path
+  float* rows = reinterpret_cast<float*>(GB + P.g_rows);  // [0,8): -m, [8,16): -inf, [16,24): sum q', [24,32): m
   int* lastf = reinterpret_cast<int*>(GB + P.g_red);
   float* wb = reinterpret_cast<float*>(GB + P.g_wb);      // [2][X][GS] value weights of a tile's slots
   float* pv = reinterpret_cast<float*>(GB + P.g_pv);      // [R][8] p rows of the value records, then A operands
@@ -975,7 +949,6 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
           rows[8 + g] = -INFINITY;
           rows[16 + g] = sg_;
           rows[24 + g] = m;
-          rows[32 + g] = 0.f;  // normaliser share of the general token path
         }
       }
     }
@@ -1245,7 +1218,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             }
           }
         } else if (t0 < tv.n) {
-          token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, rows + 32, U.AV, k, nKs, nVs, P.ka_stride}, tl);
+          token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, ovf + 2 * GS * 128, U.AV, k, nKs, nVs, P.ka_stride}, tl);
         }
       }
       gsync();  // (B) the tile's weights and p rows are complete
@@ -1350,23 +1323,25 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       }
     }
 
-    // ---- the group's partial for this unit into its slot, then the unit's counter ----
+    // ---- the group's sums for this unit into the CTA's sums in shared memory (anchor-value and
+    // rotated value-residual numerators, normaliser, sum of p min); the overflow paths added there
+    // already.  Adds of the two groups meet only element by element. ----
+    float* cl = ovf + 2 * GS * 128;  // [8] normaliser, then [8] sum of p min, per head
     {
-      float* dst = P.part + ((size_t)(c + sg.u) * (NG + 1) + grp) * PF;
       if (r8 < GS) {
 #pragma unroll
         for (int nb = 0; nb < 4; ++nb) {
           const int col = 32 * wg + 8 * nb + 2 * c4;
-          *reinterpret_cast<float2*>(dst + r8 * 128 + col) =
-              make_float2(accA[nb][0] + accA[nb][2], accA[nb][1] + accA[nb][3]);
-          *reinterpret_cast<float2*>(dst + GS * 128 + r8 * 128 + col) =
-              make_float2(accR[nb][0] + accR[nb][2], accR[nb][1] + accR[nb][3]);
+          red_local(ovf + r8 * 128 + col, accA[nb][0] + accA[nb][2]);
+          red_local(ovf + r8 * 128 + col + 1, accA[nb][1] + accA[nb][3]);
+          red_local(ovf + GS * 128 + r8 * 128 + col, accR[nb][0] + accR[nb][2]);
+          red_local(ovf + GS * 128 + r8 * 128 + col + 1, accR[nb][1] + accR[nb][3]);
         }
       }
 #pragma unroll
       for (int g = 0; g < GS; ++g) {
         const float sl = warp_sum((g & 1) ? l2[g >> 1].y : l2[g >> 1].x);
-        if (lane == 0) dst[256 * GS + wg * GS + g] = sl + (wg == 0 ? rows[32 + g] : 0.f);
+        if (lane == 0) red_local(cl + g, sl);
       }
 #pragma unroll
       for (int i2 = 0; i2 < HPL; ++i2) {
@@ -1374,27 +1349,18 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
         for (int o = 1; o < 16; o <<= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
         const int g = (lane >> 4) + 2 * i2;
-        if ((lane & 15) == 0 && g < GS) dst[256 * GS + WPG * GS + wg * GS + g] = v;
+        if ((lane & 15) == 0 && g < GS) red_local(cl + 8 + g, v);
       }
-      gsync();
-      if (gt == 0) {
-        dst[part_flag(GS)] = *failed ? 1.f : 0.f;
-        *lastf = count_in(P, sg.u, sg.nseg) ? 1 : 0;
-      }
-      gsync();
-      if (*lastf) {
-        __threadfence();
-        combine_unit<GS>(P, sg.u, sg.first, sg.nseg, wg, WPG);
-      }
-      gsync();  // lastf is reused below
     }
     if (wg == 0) {  // the segment's last tile is done with: top the ring up
       release_to(lt);
       issue_more();
     }
-    // ---- the group that finishes the segment last (the other has finished its tiles and its
-    // overflow sums) stores the CTA's overflow sums into the third slot, counts it in, and
-    // starts the next unit's anchor-score table ----
+    // ---- the group that finishes the segment last (the other has added its sums) turns the
+    // CTA's sums into its slot of the unit: the value-residual part gets its sum of p min and the
+    // inverse rotation (s o H(.) / 128, once per head and CTA), the anchor-value part is added;
+    // then it clears the sums, counts the slot in, and starts the next unit's anchor scores ----
+    gsync();
     if (gt == 0) {
       __threadfence_block();
       lastf[1] = atomicAdd(segcnt, 1) % NG == NG - 1 ? 1 : 0;
@@ -1403,20 +1369,34 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     gsync();
     const bool has_next = sg.t0 + sg.je < B1;
     if (lastf[1]) {
-      float* dst = P.part + ((size_t)(c + sg.u) * (NG + 1) + NG) * PF;
-      for (int e = 4 * gt; e < GS * 128; e += 4 * WPG * 32) {
-        float4* oa = reinterpret_cast<float4*>(ovf + e);
-        float4* orr = reinterpret_cast<float4*>(ovf + GS * 128 + e);
-        *reinterpret_cast<float4*>(dst + e) = *oa;
-        *reinterpret_cast<float4*>(dst + GS * 128 + e) = *orr;
+      float* dst = P.part + (size_t)(c + sg.u) * PF;
+      for (int h = wg; h < GS; h += WPG) {
+        float4* oa = reinterpret_cast<float4*>(ovf + h * 128 + 4 * lane);
+        float4* orr = reinterpret_cast<float4*>(ovf + GS * 128 + h * 128 + 4 * lane);
+        const float4 va = *oa, vr = *orr;
+        const float pm = cl[8 + h];
+        float x[4] = {vr.x + pm, vr.y + pm, vr.z + pm, vr.w + pm};
+        if (P.rotate) {
+          warp_wht128(x, lane);
+          apply_signs(x, lane, P.sign_lo, P.sign_hi);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) x[e] *= (1.0f / 128.0f);
+        }
+        *reinterpret_cast<float4*>(dst + h * 128 + 4 * lane) = make_float4(va.x + x[0], va.y + x[1], va.z + x[2], va.w + x[3]);
         *oa = make_float4(0.f, 0.f, 0.f, 0.f);
         *orr = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+      gsync();
+      if (gt < GS) {
+        dst[part_l(GS) + gt] = cl[gt];
+        cl[gt] = 0.f;
+        cl[8 + gt] = 0.f;
       }
       gsync();
       if (gt == 0) {
         dst[part_flag(GS)] = *failed ? 1.f : 0.f;
         lastf[0] = count_in(P, sg.u, sg.nseg) ? 1 : 0;
-        if (has_next) start_table(sg.u + 1);  // the overflow sums are clear for it
+        if (has_next) start_table(sg.u + 1);  // the CTA's sums are clear for it
       }
       gsync();
       if (lastf[0]) {
@@ -1511,7 +1491,7 @@ bool make_plan_rx(const Layout& L, int GS, int R, int X, bool smem_sa, int smem_
   P.o_meta = take(NG * NSG * sizeof(Meta));
   P.o_misc = take(16);
   P.o_sa = take(smem_sa ? (size_t)P.ka_stride * GS * 4 : 0);
-  P.o_ovf = take((size_t)2 * GS * 128 * 4);
+  P.o_ovf = take((size_t)2 * GS * 128 * 4 + 2 * 8 * 4);  // + normaliser and sum of p min per head
   // a group's block: q' rows, small rows, last flag, two weight tables, p rows / A operands
   size_t g = 0;
   auto gtake = [&](size_t bytes) {
@@ -1520,7 +1500,7 @@ bool make_plan_rx(const Layout& L, int GS, int R, int X, bool smem_sa, int smem_
     return (int)o;
   };
   P.g_qp = gtake((size_t)GS * 128 * 4);
-  P.g_rows = gtake(48 * 4);
+  P.g_rows = gtake(32 * 4);
   P.g_red = gtake(16);
   P.g_wb = gtake((size_t)2 * X * GS * 4);
   P.g_pv = gtake((size_t)R * 32);
@@ -1598,7 +1578,7 @@ DecodeWs decode_ws_layout(const Layout& L) {
   w.o_sa = take(units * ka * (size_t)L.G * 4);
   w.o_cmax = take(units * nch * (size_t)L.G * 4);
   w.o_cnt = take(units * 4);
-  w.o_part = take((size_t)(kMaxGrid + units) * (NG + 1) * (size_t)part_floats(L.G) * 4);
+  w.o_part = take((size_t)(kMaxGrid + units) * (size_t)part_floats(L.G) * 4);
   w.total = off;
   return w;
 }
