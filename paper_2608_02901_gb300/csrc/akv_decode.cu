@@ -79,9 +79,16 @@ __host__ __device__ constexpr int part_floats(int GS) { return 128 * GS + 12; }
 __host__ __device__ constexpr int part_l(int GS) { return 128 * GS; }
 __host__ __device__ constexpr int part_flag(int GS) { return 128 * GS + 8; }
 
+// Bytes of a unit's query header (from the score kernel): the rotated query q' [GS][128] f32, its
+// sums [8] f32, and the key-residual mma B fragments [GS == 8 ? 2 : 1][8][32] uint2.
+__host__ __device__ constexpr int hdr_bytes(int GS) { return GS * 512 + 32 + (GS == 8 ? 2 : 1) * 2048; }
+
 struct ScoreParams {
   const uint8_t* arena;
   const __nv_bfloat16* q;
+  uint8_t* uh;     // [units] query headers, uh_stride bytes apart
+  int uh_stride, rotate;
+  unsigned long long sign_lo, sign_hi;
   float* sa;      // [units][ka_stride][G] anchor scores (log2 units)
   float* cmax;    // [units][n_ch][G] largest score of each chunk of CHA anchors
   unsigned* cnt;  // [units] arrival counters of the decode launch, zeroed here
@@ -102,6 +109,8 @@ struct DecodeParams {
   const float* cmax;
   float* part;
   unsigned* cnt;
+  const uint8_t* uh;  // query headers (score kernel)
+  int uh_stride;
   long long ttot;  // tiles of all units
   int grid, n_kv_heads, n_q_heads, rotate, ka_stride, n_ch;
   float scale_log2;
@@ -530,6 +539,57 @@ __global__ void __launch_bounds__(128) akv_scores_kernel(const ScoreParams P) {
     const int g = threadIdx.x;
     P.cmax[((size_t)u * P.n_ch + ch) * GS + g] = fmaxf(fmaxf(wmax[0][g], wmax[1][g]), fmaxf(wmax[2][g], wmax[3][g]));
   }
+  if (ch != 0) return;
+  // ---- the unit's query header (chunk 0): rotated query q' = H(s o q) / 128, scaled to log2
+  // units (Appendix A.1, Eq. 12; warp-local Walsh-Hadamard transform), its sums, and the
+  // key-residual mma B fragments: column n = lane / 4 is head n as the fp16 high part (set 0) and
+  // low part (set 1) for GS = 8, else head n % 4 high (n < 4) or low (n >= 4); k pairs (2t, 2t+1)
+  // <-> dims (16 ks + 2t, 16 ks + 2t + 8), (2t+8, 2t+9) <-> (16 ks + 2t + 1, 16 ks + 2t + 9) ----
+  constexpr int NBF = GS == 8 ? 2 : 1;
+  __shared__ __align__(16) float qs[8 * 128];
+  uint8_t* H = P.uh + (size_t)u * P.uh_stride;
+  float* hq = reinterpret_cast<float*>(H);
+  float* hs = hq + GS * 128;
+  uint2* hf = reinterpret_cast<uint2*>(hs + 8);
+  const size_t qb = qrow_base(u, P.n_kv_heads, P.n_q_heads);
+  const float f = P.rotate ? P.scale_log2 * (1.0f / 128.0f) : P.scale_log2;
+  for (int g = warp; g < GS; g += 4) {
+    const uint2 raw = *reinterpret_cast<const uint2*>(P.q + qb + (size_t)g * 128 + 4 * lane);
+    float x[4] = {__bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.x & 0xFFFFu))),
+                  __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.x >> 16))),
+                  __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.y & 0xFFFFu))),
+                  __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.y >> 16)))};
+    if (P.rotate) {
+      apply_signs(x, lane, P.sign_lo, P.sign_hi);
+      warp_wht128(x, lane);
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) x[j] *= f;
+    const float4 v = make_float4(x[0], x[1], x[2], x[3]);
+    *reinterpret_cast<float4*>(qs + g * 128 + 4 * lane) = v;
+    *reinterpret_cast<float4*>(hq + g * 128 + 4 * lane) = v;
+    const float sg = warp_sum((x[0] + x[1]) + (x[2] + x[3]));
+    if (lane == 0) hs[g] = sg;
+  }
+  if (threadIdx.x >= GS && threadIdx.x < 8) hs[threadIdx.x] = 0.f;
+  __syncthreads();
+  const int gcol = lane >> 2, cc = lane & 3;
+  for (int idx = warp; idx < NBF * 8; idx += 4) {
+    const int hl = idx >> 3, ks = idx & 7;
+    uint2 fk = make_uint2(0u, 0u);
+    const int head = GS == 8 ? gcol : (gcol & 3);
+    const bool low = GS == 8 ? hl == 1 : gcol >= 4;
+    if (head < GS) {
+      const float* x = qs + head * 128 + 16 * ks + 2 * cc;
+      auto part = [&](float v) {
+        const __half hi = __float2half_rn(v);
+        return low ? __float2half_rn(v - __half2float(hi)) : hi;
+      };
+      fk.x = pack_h2(part(x[0]), part(x[8]));
+      fk.y = pack_h2(part(x[1]), part(x[9]));
+    }
+    hf[(hl * 8 + ks) * 32 + lane] = fk;
+  }
 }
 
 // ============================ the unit's output ====================================
@@ -684,7 +744,7 @@ __device__ __noinline__ void token_chunk_general(const TokTile tt, const TokLane
     rkn += (int)kb;
     if (kb && r >= tt.nKs && e < nvalid) {  // beyond the staged records
 #pragma unroll
-      for (int g = 0; g < GS; ++g) rt[g] = key_record_term(tv, r, tt.qp + g * 128, tt.rows[16 + g]) + tt.rows[g];
+      for (int g = 0; g < GS; ++g) rt[g] = key_record_term(tv, r, tt.qp + g * 128, tt.qp[GS * 128 + g]) + tt.rows[g];
     } else {  // the key-residual terms minus m, -m, or -inf for a token past the tile's end
       load_row<GS>(e >= nvalid ? ninfrow : negrow, rt);
       if (kb && e < nvalid) {
@@ -746,11 +806,11 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   // anchor-score table landed (sa_full; a plain arrival when the table stays in global memory)
   auto bar_full = [&](int g, int s) { return smem_u32(bars + g * NSG + s); };
   const uint32_t bar_sa_full = smem_u32(bars + NG * NSG);
+  auto bar_hdr = [&](int g) { return smem_u32(bars + NG * NSG + 1 + g); };  // a group's query header landed
   int* segcnt = reinterpret_cast<int*>(smem + P.o_misc + 4);  // groups done with a segment, in total
 
   if (tid == 0) {
-    for (int s = 0; s < NG * NSG; ++s) mbar_init(smem_u32(bars + s), 1);
-    mbar_init(bar_sa_full, 1);
+    for (int s = 0; s < NG * NSG + 1 + NG; ++s) mbar_init(smem_u32(bars + s), 1);
     *failed = 0;
     *segcnt = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -823,7 +883,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   const int grp = warp / WPG, wg = warp % WPG, gt = tid - grp * WPG * 32;
   uint8_t* GB = smem + P.o_grp + grp * P.grp_bytes;
   float* qp = reinterpret_cast<float*>(GB + P.g_qp);      // [GS][128] rotated query q'
-  float* rows = reinterpret_cast<float*>(GB + P.g_rows);  // [0,8): -m, [8,16): -inf, [16,24): sum q', [24,32): m
+  float* sq = qp + GS * 128;                              // [8] sums of q' per head
+  float* rows = reinterpret_cast<float*>(GB + P.g_rows);  // [0,8): -m, [8,16): -inf, [24,32): m
   int* lastf = reinterpret_cast<int*>(GB + P.g_red);
   float* wb = reinterpret_cast<float*>(GB + P.g_wb);      // [2][X][GS] value weights of a tile's slots
   float* pv = reinterpret_cast<float*>(GB + P.g_pv);      // [R][8] p rows of the value records, then A operands
@@ -922,34 +983,26 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   for (;; ++sigma) {
     const UnitView U = unit_view(P.arena, sg.u);
     const int k = U.k;
-    // ---- segment set-up: q' rows (warp wg: heads wg, wg + 4), their sums, the reference m ----
-    {
-      const size_t qb = qrow_base(sg.u, P.n_kv_heads, P.n_q_heads);
-      const float f = P.rotate ? P.scale_log2 * (1.0f / 128.0f) : P.scale_log2;
-      for (int g = wg; g < GS; g += WPG) {
-        const uint2 raw = *reinterpret_cast<const uint2*>(P.q + qb + (size_t)g * 128 + 4 * lane);
-        float x[4] = {__bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.x & 0xFFFFu))),
-                      __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.x >> 16))),
-                      __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.y & 0xFFFFu))),
-                      __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.y >> 16)))};
-        if (P.rotate) {
-          apply_signs(x, lane, P.sign_lo, P.sign_hi);
-          warp_wht128(x, lane);
-        }
-#pragma unroll
-        for (int j = 0; j < 4; ++j) x[j] *= f;
-        *reinterpret_cast<float4*>(qp + g * 128 + 4 * lane) = make_float4(x[0], x[1], x[2], x[3]);
-        const float sg_ = warp_sum((x[0] + x[1]) + (x[2] + x[3]));
-        float m = -INFINITY;
-        const int nch = (k + CHA - 1) / CHA;
-        for (int ch = lane; ch < nch; ch += 32) m = fmaxf(m, P.cmax[((size_t)sg.u * P.n_ch + ch) * GS + g]);
-        m = warp_max(m);
-        if (lane == 0) {
-          rows[g] = -m;
-          rows[8 + g] = -INFINITY;
-          rows[16 + g] = sg_;
-          rows[24 + g] = m;
-        }
+    // ---- segment set-up: the unit's query header (q', its sums, key-residual fragments, from
+    // the score kernel) by one bulk copy; meanwhile the reference m of each head from the chunk
+    // maxima (warp wg: heads wg, wg + 4) ----
+    if (wg == 0 && lane == 0) {
+      if (!*failed) {
+        mbar_expect_tx(bar_hdr(grp), (uint32_t)hdr_bytes(GS));
+        bulk_g2s(smem_u32(qp), P.uh + (size_t)sg.u * P.uh_stride, (uint32_t)hdr_bytes(GS), bar_hdr(grp));
+      } else {
+        mbar_arrive(bar_hdr(grp));
+      }
+    }
+    for (int g = wg; g < GS; g += WPG) {
+      float m = -INFINITY;
+      const int nch = (k + CHA - 1) / CHA;
+      for (int ch = lane; ch < nch; ch += 32) m = fmaxf(m, P.cmax[((size_t)sg.u * P.n_ch + ch) * GS + g]);
+      m = warp_max(m);
+      if (lane == 0) {
+        rows[g] = -m;
+        rows[8 + g] = -INFINITY;
+        rows[24 + g] = m;
       }
     }
 #pragma unroll
@@ -963,34 +1016,11 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     for (int i = 0; i < NP; ++i) l2[i] = make_float2(0.f, 0.f);
 #pragma unroll
     for (int i = 0; i < HPL; ++i) pminv[i] = 0.f;
-    gsync();
-    // key-residual B fragments (k-step ks): column n = lane / 4 is head n as the fp16 high part
-    // (set 0) and low part (set 1) for GS = 8, else head n % 4 high (n < 4) or low (n >= 4);
-    // k pairs (2t, 2t+1) <-> dims (16 ks + 2t, 16 ks + 2t + 8), (2t+8, 2t+9) <-> (16 ks + 2t + 1,
-    // 16 ks + 2t + 9), t = lane % 4; warp wg builds k-steps wg, wg + 4
-    {
-      const int gcol = lane >> 2, cc = lane & 3;
-#pragma unroll
-      for (int hl = 0; hl < NBF; ++hl)
-        for (int ks = wg; ks < 8; ks += WPG) {
-          uint2 fk = make_uint2(0u, 0u);
-          const int head = GS == 8 ? gcol : (gcol & 3);
-          const bool low = GS == 8 ? hl == 1 : gcol >= 4;
-          if (head < GS) {
-            const float* x = qp + head * 128 + 16 * ks + 2 * cc;
-            auto part = [&](float v) {
-              const __half hi = __float2half_rn(v);
-              return low ? __float2half_rn(v - __half2float(hi)) : hi;
-            };
-            fk.x = pack_h2(part(x[0]), part(x[8]));
-            fk.y = pack_h2(part(x[1]), part(x[9]));
-          }
-          qf[(hl * 8 + ks) * 32 + lane] = fk;
-        }
-    }
-    // the unit's anchor-score table (every warp waits, tiles or not, so its phase count stays right)
+    // the header, then the unit's anchor-score table (every warp waits on both, tiles or not, so
+    // the phase counts stay right)
+    if (!warp_failed(failed) && !mbar_wait_w(bar_hdr(grp), (uint32_t)sigma & 1u)) *failed = 1;
     if (!warp_failed(failed) && !mbar_wait_w(bar_sa_full, (uint32_t)sigma & 1u)) *failed = 1;
-    gsync();  // fragments built
+    gsync();  // m of every head written
     const float* SAt = P.smem_sa ? SAs : P.sa + (size_t)sg.u * P.ka_stride * GS;
 
     const int i_end = sg.ib + (sg.je - sg.jb);
@@ -1064,7 +1094,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
                   for (int e = 0; e < 2; ++e) {
                     const int g = 2 * c4 + e;
-                    if (g < GS) rsb[sl * 8 + g] = half_hi(smn) * rows[16 + g] + half_lo(smn) * v[2 * hr + e];
+                    if (g < GS) rsb[sl * 8 + g] = half_hi(smn) * sq[g] + half_lo(smn) * v[2 * hr + e];
                   }
                 }
               }
@@ -1413,6 +1443,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   if (wg == 0 && lane == 0) {
     for (int t = max(0, nis - NSG); t < nis; ++t)
       if (!(gmeta[t % NSG].nrows >> 31)) mbar_wait(bar_full(grp, t % NSG), (uint32_t)(t / NSG) & 1u);
+    mbar_wait(bar_hdr(grp), (uint32_t)sigma & 1u);
     if (grp == 0) mbar_wait(bar_sa_full, (uint32_t)sigma & 1u);
   }
 }
@@ -1487,7 +1518,7 @@ bool make_plan_rx(const Layout& L, int GS, int R, int X, bool smem_sa, int smem_
     off = align128(off + bytes);
     return (int)o;
   };
-  P.o_bar = take((NG * NSG + 1) * 8);
+  P.o_bar = take((NG * NSG + 1 + NG) * 8);
   P.o_meta = take(NG * NSG * sizeof(Meta));
   P.o_misc = take(16);
   P.o_sa = take(smem_sa ? (size_t)P.ka_stride * GS * 4 : 0);
@@ -1499,12 +1530,12 @@ bool make_plan_rx(const Layout& L, int GS, int R, int X, bool smem_sa, int smem_
     g = align128(g + bytes);
     return (int)o;
   };
-  P.g_qp = gtake((size_t)GS * 128 * 4);
+  P.g_qp = gtake((size_t)hdr_bytes(GS));  // the unit's query header: q', its sums, B fragments
+  P.g_qf = P.g_qp + GS * 512 + 32;
   P.g_rows = gtake(32 * 4);
   P.g_red = gtake(16);
   P.g_wb = gtake((size_t)2 * X * GS * 4);
   P.g_pv = gtake((size_t)R * 32);
-  P.g_qf = gtake((size_t)(GS == 8 ? 2 : 1) * 8 * 32 * 8);
   P.grp_bytes = (int)g;
   P.o_grp = take((size_t)NG * g);
   P.o_ring = (int)off;
@@ -1576,6 +1607,7 @@ DecodeWs decode_ws_layout(const Layout& L) {
     return o;
   };
   w.o_sa = take(units * ka * (size_t)L.G * 4);
+  w.o_uh = take(units * (size_t)((hdr_bytes(L.G) + 255) & ~255));
   w.o_cmax = take(units * nch * (size_t)L.G * 4);
   w.o_cnt = take(units * 4);
   w.o_part = take((size_t)(kMaxGrid + units) * (size_t)part_floats(L.G) * 4);
@@ -1644,6 +1676,8 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   P.cmax = (const float*)(wsb + W.o_cmax);
   P.part = (float*)(wsb + W.o_part);
   P.cnt = (unsigned*)(wsb + W.o_cnt);
+  P.uh = wsb + W.o_uh;
+  P.uh_stride = (hdr_bytes(GS) + 255) & ~255;
   P.n_kv_heads = p.n_kv_heads;
   P.n_q_heads = p.n_q_heads;
   P.rotate = (p.flags & AKV_FLAG_ROTATE) ? 1 : 0;
@@ -1664,6 +1698,11 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   S.ka_stride = P.ka_stride;
   S.n_ch = P.n_ch;
   S.scale_log2 = P.scale_log2;
+  S.uh = wsb + W.o_uh;
+  S.uh_stride = P.uh_stride;
+  S.rotate = P.rotate;
+  S.sign_lo = P.sign_lo;
+  S.sign_hi = P.sign_hi;
 
   cudaLaunchAttribute attr[1];
   // each launch may overlap the tail of the preceding one (griddepcontrol in the kernels)

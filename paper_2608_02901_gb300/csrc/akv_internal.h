@@ -115,10 +115,10 @@ void encode_ws_layout(const Layout& L, EncodeWs* ws, int32_t m_obs = 0);
 int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const void* K, const void* V, int32_t s_max,
                   void* arena, void* ws, void* stream, const akv_select_params* sel = nullptr,
                   const void* Q = nullptr, int32_t m_obs = 0);
-// Decode workspace (device): anchor scores [units][ka][G] f32, chunk maxima, arrival counters,
-// partial slots; byte offsets from the workspace base (256-byte aligned).
+// Decode workspace (device): anchor scores [units][ka][G] f32, query headers, chunk maxima,
+// arrival counters, partial slots; byte offsets from the workspace base (256-byte aligned).
 struct DecodeWs {
-  size_t o_sa = 0, o_cmax = 0, o_cnt = 0, o_part = 0, total = 0;
+  size_t o_sa = 0, o_uh = 0, o_cmax = 0, o_cnt = 0, o_part = 0, total = 0;
 };
 DecodeWs decode_ws_layout(const Layout& L);
 int launch_decode(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
