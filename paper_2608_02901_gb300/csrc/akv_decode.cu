@@ -88,6 +88,7 @@ struct ScoreParams {
   const __nv_bfloat16* q;
   uint8_t* uh;     // [units] query headers, uh_stride bytes apart
   int uh_stride, rotate;
+  int prefetch_l2; // 1: the arena fits the L2 cache; every unit's decode data is prefetched into it
   unsigned long long sign_lo, sign_hi;
   float* sa;      // [units][ka_stride][G] anchor scores (log2 units)
   float* cmax;    // [units][n_ch][G] largest score of each chunk of CHA anchors
@@ -115,7 +116,7 @@ struct DecodeParams {
   int grid, n_kv_heads, n_q_heads, rotate, ka_stride, n_ch;
   float scale_log2;
   unsigned long long sign_lo, sign_hi;
-  int R;           // records per side and tile that are staged and handled on tensor cores
+  int R;           // value records per tile handled on tensor cores (their p rows); sizes the staging cap
   int X;           // anchor-value rows per tile that are staged (the weight table's rows)
   int cap;         // staged bytes of a tile block at most
   int ring_bytes, drop_last, smem_sa;
@@ -213,6 +214,11 @@ __device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t& r0, uint3
                : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                : "r"(addr));
 }
+// Asynchronous prefetch of [p, p + bytes) into the L2 cache (16-byte aligned, a multiple of 16).
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
 // 16 bytes of read-only global data, not kept in L1 (streamed once)
 __device__ __forceinline__ uint4 ldg_stream(const void* p) {
   uint4 v;
@@ -361,27 +367,36 @@ __device__ __forceinline__ TileView tile_view(const uint8_t* st, const Meta& mt,
   return v;
 }
 
-// Records beyond the staged ones (a locally dense tile) take these rare paths on CUDA
-// cores, kept out of line so that the token loop stays small.
-// Key residual term scale (q'_g . c) + min sum(q'_g) of key record r.
-__device__ __noinline__ float key_record_term(const TileView tv, int r, const float* qpg, float sqg) {
-  const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_k + 4u * (uint32_t)r));
+// Bytes of a tile block at offset `off`: shared memory for its first `staged` bytes, else the
+// block in global memory.
+__device__ __forceinline__ const uint8_t* blk_at(const uint8_t* st, const uint8_t* gb, uint32_t staged, uint32_t off) {
+  return off < staged ? st + off : gb + off;
+}
+// Records beyond the staged ones (a locally dense tile whose codes did not fit the staging
+// cap) take these rare paths on CUDA cores, kept out of line so that the token loop stays
+// small.  Their arguments are plain pointers and offsets: a struct passed by value would be
+// built in local memory at every call.
+// Key residual term scale (q'_g . c) + min sum(q'_g) of the key record whose scale-min word
+// is at `smn_off` and whose codes start at `cd_off`.
+__device__ __noinline__ float key_record_term(const uint8_t* st, const uint8_t* gb, uint32_t staged, uint32_t smn_off,
+                                              uint32_t cd_off, const float* qpg, float sqg) {
+  const uint32_t smn = *reinterpret_cast<const uint32_t*>(blk_at(st, gb, staged, smn_off));
   float dot = 0.f;
   for (int bb = 0; bb < 32; ++bb) {
-    const uint32_t byte = *tv.at(tv.cd_k + 32u * (uint32_t)r + (uint32_t)bb);
+    const uint32_t byte = *blk_at(st, gb, staged, cd_off + (uint32_t)bb);
 #pragma unroll
     for (int c = 0; c < 4; ++c) dot += qpg[4 * bb + c] * (float)((byte >> (2 * c)) & 3u);
   }
   return half_hi(smn) * sqg + half_lo(smn) * dot;
 }
 // accg += p (min + scale c) of value record r, in the rotated domain (value codes are
-// dimension-major groups of 16 records).
-__device__ __noinline__ void value_record_add(const TileView tv, int r, float p, float* accg) {
-  const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_v + 4u * (uint32_t)r));
+// dimension-major groups of 16 records; the group of r starts at `grp_off`).
+__device__ __noinline__ void value_record_add(const uint8_t* st, const uint8_t* gb, uint32_t staged, uint32_t smn_off,
+                                              uint32_t grp_off, int r, float p, float* accg) {
+  const uint32_t smn = *reinterpret_cast<const uint32_t*>(blk_at(st, gb, staged, smn_off));
   const float ps = p * half_lo(smn), pm = p * half_hi(smn);
-  const uint32_t base = tv.cd_v + 512u * (uint32_t)(r / 16);
   for (int d = 0; d < 128; ++d) {
-    const uint32_t w = *reinterpret_cast<const uint32_t*>(tv.at(base + 4u * value_code_word(d)));
+    const uint32_t w = *reinterpret_cast<const uint32_t*>(blk_at(st, gb, staged, grp_off + 4u * value_code_word(d)));
     atomicAdd(&accg[d], fmaf(ps, (float)((w >> value_code_bit(r % 16)) & 3u), pm));
   }
 }
@@ -483,6 +498,14 @@ __global__ void __launch_bounds__(128) akv_scores_kernel(const ScoreParams P) {
   const akv_unit_desc* d = unit_desc(P.arena, u);
   const int k = d->n_anchors;
   if (ch == 0 && threadIdx.x == 0) P.cnt[u] = 0u;
+  if (P.prefetch_l2 && threadIdx.x == 0) {
+    // the decode launch's reads of this unit (anchor values, tile table, tile blocks: one range
+    // of the arena) start from L2 instead of a chain of cold HBM reads; chunk ch takes its share
+    const uint64_t b0 = d->off_anchor_v, b1 = d->off_tiles + d->tiles_capacity;
+    const uint64_t per = (((b1 - b0) + P.n_ch - 1) / P.n_ch + 15) & ~15ull;
+    const uint64_t s0 = b0 + per * ch, s1 = (s0 + per < b1 ? s0 + per : b1) & ~15ull;
+    for (uint64_t a = s0; a < s1; a += (1ull << 20)) prefetch_l2(P.arena + a, (uint32_t)(s1 - a < (1ull << 20) ? s1 - a : (1ull << 20)));
+  }
   const int a0 = ch * CHA + 16 * warp;
   float mx0 = -INFINITY, mx1 = -INFINITY;  // heads 2 c4, 2 c4 + 1
   if (a0 < k) {
@@ -690,29 +713,46 @@ struct TokTile {
   float* pv;          // [R][8] p rows of the value records
   float* W;           // [X][GS] the tile's value weights
   float* ovf;         // [2][GS][128] overflow sums
-  float* lsum;        // [GS] the CTA's normaliser sums (this path adds its share there)
   const uint8_t* AV;  // the unit's anchor values (global)
   int k, nKs, nVs, ka;
 };
 
 // The general token path (kept out of line: a tile with records beyond the staged ones, runs
 // beyond the staged anchor-value rows, or a lane past the tile's end): the same arithmetic as
-// the fast path, with the rare cases on CUDA cores.  Everything is passed by value and the
-// normaliser goes to shared memory, so that no variable of the caller has its address taken
-// (it would then live in local memory, whose lines the small L1 here does not keep).
+// the fast path, with the rare cases on CUDA cores; it returns the lane's share of the
+// normaliser (a shared-memory sum would take every lane's addition on the same words).  The
+// arguments arrive by value and are copied into locals first: the shared-memory reductions below clobber memory, so a field read
+// through the argument itself would be reloaded from its local-memory copy (L2 latency, the
+// L1 here being small) after every reduction.
+template <int NP>
+struct LShare {
+  float2 v[NP];
+};
 template <int GS>
-__device__ __noinline__ void token_chunk_general(const TokTile tt, const TokLane tl) {
+__device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const TokTile tt_arg, const TokLane tl_arg) {
   constexpr int NP = GS >= 2 ? GS / 2 : 1;
-  const TileView& tv = tt.tv;
+  const TokTile tt = tt_arg;
+  const TokLane tl = tl_arg;
+  const TileView tv = tt.tv;
   const uint8_t* st = tv.st;
+  const uint8_t* gb = tv.gb;
+  const uint32_t staged = tv.staged;
   const int t0 = tl.t0;
   const int nvalid = min(LCH, tv.n - t0);
   const float* rsb = reinterpret_cast<const float*>(st + tv.cd_k);
   const float* negrow = tt.rows;
   const float* ninfrow = tt.rows + 8;
+  const float* qp = tt.qp;
+  const float* SAt = tt.SAt;
+  float* W = tt.W;
+  float* pv = tt.pv;
+  float* ovf = tt.ovf;
+  const uint8_t* AV = tt.AV;
+  const int k = tt.k, nKs = tt.nKs, nVs = tt.nVs, ka = tt.ka;
   const uint32_t lo = tt.lo;
   const int nrows = (int)tt.nrows;
   int rkn = tl.rk, rvn = tl.rv;
+  const uint32_t kbits = tl.kbits, vbits = tl.vbits;
   float2 l2[NP];
 #pragma unroll
   for (int i2 = 0; i2 < NP; ++i2) l2[i2] = make_float2(0.f, 0.f);
@@ -726,25 +766,28 @@ __device__ __noinline__ void token_chunk_general(const TokTile tt, const TokLane
 #pragma unroll
     for (int g = 0; g < GS; ++g) vv[g] = (g & 1) ? v[g >> 1].y : v[g >> 1].x;
     if (ix < nrows) {
-      float* w = tt.W + ix * GS;
+      float* w = W + ix * GS;
 #pragma unroll
       for (int g = 0; g < GS; ++g) red_local(w + g, vv[g]);
     } else {  // beyond the staged anchor-value rows: its products on CUDA cores
-      anchor_value_add<GS>(tt.AV, (int)kk, vv, tt.ovf);
+      anchor_value_add<GS>(AV, (int)kk, vv, ovf);
     }
   };
   for (int e = 0; e < LCH; ++e) {
     const uint32_t ek = e < nvalid ? *reinterpret_cast<const uint32_t*>(st + 4 * (t0 + e)) : 0u;
     const uint32_t ev = e < nvalid ? *reinterpret_cast<const uint32_t*>(st + 4 * (tv.n64 + t0 + e)) : 0u;
-    const int a = min((int)(ek & 0xFFFFu), tt.k - 1);
+    const int a = min((int)(ek & 0xFFFFu), k - 1);
     float sa[GS], rt[GS];
-    load_sa_row<GS>(tt.SAt, a, tt.ka, sa);
-    const bool kb = (tl.kbits >> e) & 1u;
+    load_sa_row<GS>(SAt, a, ka, sa);
+    const bool kb = (kbits >> e) & 1u;
     const int r = rkn;
     rkn += (int)kb;
-    if (kb && r >= tt.nKs && e < nvalid) {  // beyond the staged records
+    if (kb && r >= nKs && e < nvalid) {  // beyond the staged records
 #pragma unroll
-      for (int g = 0; g < GS; ++g) rt[g] = key_record_term(tv, r, tt.qp + g * 128, tt.qp[GS * 128 + g]) + tt.rows[g];
+      for (int g = 0; g < GS; ++g)
+        rt[g] = key_record_term(st, gb, staged, tv.sm_k + 4u * (uint32_t)r, tv.cd_k + 32u * (uint32_t)r, qp + g * 128,
+                                qp[GS * 128 + g]) +
+                negrow[g];
     } else {  // the key-residual terms minus m, -m, or -inf for a token past the tile's end
       load_row<GS>(e >= nvalid ? ninfrow : negrow, rt);
       if (kb && e < nvalid) {
@@ -757,16 +800,17 @@ __device__ __noinline__ void token_chunk_general(const TokTile tt, const TokLane
     const float gk = half_hi(ek), gv = half_hi(ev);
     float2 pe[NP];
     head_probs<GS, NP>(gk, sa, rt, pe, l2);
-    const bool vb = (tl.vbits >> e) & 1u;
+    const bool vb = (vbits >> e) & 1u;
     const int rv = rvn;
     rvn += (int)vb;
     if (vb && e < nvalid) {
-      if (rv < tt.nVs) {
-        store_row<GS>(tt.pv + rv * 8, pe);
+      if (rv < nVs) {
+        store_row<GS>(pv + rv * 8, pe);
       } else {  // beyond the staged records
 #pragma unroll
         for (int g = 0; g < GS; ++g)
-          value_record_add(tv, rv, (g & 1) ? pe[g >> 1].y : pe[g >> 1].x, tt.ovf + GS * 128 + g * 128);
+          value_record_add(st, gb, staged, tv.sm_v + 4u * (uint32_t)rv, tv.cd_v + 512u * (uint32_t)(rv / 16), rv,
+                           (g & 1) ? pe[g >> 1].y : pe[g >> 1].x, ovf + GS * 128 + g * 128);
       }
     }
     // tokens past the tile join the current run with zero weight
@@ -782,8 +826,10 @@ __device__ __noinline__ void token_chunk_general(const TokTile tt, const TokLane
     for (int i2 = 0; i2 < NP; ++i2) acc[i2] = __ffma2_rn(pe[i2], gv2, acc[i2]);
   }
   flush(key, acc);
+  LShare<NP> ls;
 #pragma unroll
-  for (int g = 0; g < GS; ++g) red_local(tt.lsum + g, (g & 1) ? l2[g >> 1].y : l2[g >> 1].x);
+  for (int i2 = 0; i2 < NP; ++i2) ls.v[i2] = l2[i2];
+  return ls;
 }
 
 // ================================ decode ============================================
@@ -1037,7 +1083,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       if (go) {
         tv = tile_view(st, mt, U);
         const uint32_t codes_staged = tv.staged > tv.cd_k ? (tv.staged - tv.cd_k) / 32u : 0u;
-        nKs = min(min(tv.nk, P.R), (int)codes_staged);
+        nKs = min(tv.nk, (int)codes_staged);  // their terms go over their own codes: no cap but staging
         nVs = min(tv.nv, P.R);
         fast_tile = nKs == tv.nk && nVs == tv.nv &&
                     (int)(((reinterpret_cast<const uint32_t*>(st + 4 * tv.n64))[tv.n - 1] & 0xFFFFu) - mt.lo) < (int)mt.nrows;
@@ -1248,7 +1294,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             }
           }
         } else if (t0 < tv.n) {
-          token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, ovf + 2 * GS * 128, U.AV, k, nKs, nVs, P.ka_stride}, tl);
+          const auto ls = token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, U.AV, k, nKs, nVs, P.ka_stride}, tl);
+#pragma unroll
+          for (int i2 = 0; i2 < NP; ++i2) l2[i2] = __fadd2_rn(l2[i2], ls.v[i2]);
         }
       }
       gsync();  // (B) the tile's weights and p rows are complete
@@ -1703,6 +1751,8 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   S.rotate = P.rotate;
   S.sign_lo = P.sign_lo;
   S.sign_hi = P.sign_hi;
+  // small arenas (a few layers fit the 129 MB L2 several times over) are prefetched into L2
+  S.prefetch_l2 = L.total_bytes <= (64ull << 20) ? 1 : 0;
 
   cudaLaunchAttribute attr[1];
   // each launch may overlap the tail of the preceding one (griddepcontrol in the kernels)

@@ -134,16 +134,42 @@ def test_ragged_sweep_points(dev):
         _run_seeded(dev, p, lens, seed=int(fa * 1000 + fr * 100))
 
 
+def _stored_non_anchor(d):
+    """Non-anchor positions in stored order: tokens are stored sorted by value-anchor slot
+    (stable, so by position within a slot), and tiles are runs of 1024 stored tokens."""
+    order = np.argsort(d["idx_v"], kind="stable")
+    is_anchor = np.zeros(d["S"], bool)
+    is_anchor[d["anchor_pos"]] = True
+    return order[~is_anchor[order]]
+
+
 def test_locally_dense_residuals_exceed_staging(dev):
-    """All residual slots packed into a few tiles: those tiles hold far more slots than the
-    kernel stages per tile (sized from the mean density), so the overflow paths run."""
+    """Key residuals on the first non-anchor tokens in stored order, value residuals on the
+    last: the first tile holds about 600 key records and the last about 600 value records, far
+    more than the kernel stages per tile (sized from the mean density), so the key records
+    whose codes fall beyond the staged bytes and the value records beyond the staged count
+    take the CUDA-core paths."""
     def mutate(u, d):
-        non = np.setdiff1d(np.arange(d["S"]), d["anchor_pos"])
+        non = _stored_non_anchor(d)
         d["res_k"] = np.sort(non[: d["nk"]]).astype(np.int32)
         d["res_v"] = np.sort(non[len(non) - d["nv"]:]).astype(np.int32)
     for G in (1, 4, 8):
         p = akv.Params(batch=2, n_kv_heads=2, n_q_heads=2 * G, seed=31)
         _run_seeded(dev, p, [6000, 3000], mutate=mutate)
+
+
+def test_key_records_beyond_the_value_staging_count(dev):
+    """Key residuals on every fourth non-anchor token in stored order (about 250 a tile, 2.5x
+    the mean): more key records than the value records a tile stages, yet their codes fit the
+    tile's staging, so they stay on the tensor-core path; the value residuals sit in the last
+    tiles, beyond their staged count."""
+    def mutate(u, d):
+        non = _stored_non_anchor(d)
+        d["res_k"] = np.sort(non[::4][: d["nk"]]).astype(np.int32)
+        d["res_v"] = np.sort(non[len(non) - d["nv"]:]).astype(np.int32)
+    for G in (4, 8):
+        p = akv.Params(batch=2, n_kv_heads=2, n_q_heads=2 * G, seed=37)
+        _run_seeded(dev, p, [6000, 9000], mutate=mutate, qseed=G)
 
 
 def test_tiles_covering_more_value_slots_than_the_weight_table(dev, debug_controls):
