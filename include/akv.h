@@ -395,11 +395,8 @@ akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_len
  * Errors: AKV_ERR_INVALID (null/misaligned pointers, bad sizes), AKV_ERR_TOO_SMALL
  * (arena or workspace short), AKV_ERR_UNSUPPORTED (no shared-memory plan fits),
  * AKV_ERR_CUDA (launch failure).
- * Ordering: both launches are programmatic dependent launches: each may be scheduled
- * and set up its on-chip state while the preceding launch in the stream drains, but
- * reads the arena, q and the workspace, and writes out/out_f32 and the workspace,
- * only after all preceding work in the stream has completed (ordinary stream
- * semantics for data).
+ * Ordering: both launches are ordinary launches on `stream`: they start after all
+ * preceding work in the stream and complete before any later work starts.
  */
 akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,
                            size_t arena_bytes, const void* q, void* out, float* out_f32, float sm_scale,
@@ -422,6 +419,20 @@ akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, co
  * Errors: AKV_ERR_INVALID for values out of range.
  */
 akv_status akv_decode_set_debug(int32_t ctas, int32_t withhold_last);
+
+/*
+ * Timing aid (process-wide, like akv_decode_set_debug): with non-null events, every
+ * later akv_decode_attn call records `after_scores` on its stream right after its
+ * first launch (the anchor scores) and `after_decode` right after its second (the
+ * decode), so that a caller who records an event before the call can time each
+ * launch with cudaEventElapsedTime.  Nothing is skipped or changed in the work.
+ *   after_scores, after_decode : cudaEvent_t handles created by the caller (both
+ *                                null = off; ownership stays with the caller, who
+ *                                must clear them before destroying the events)
+ * Errors: AKV_ERR_INVALID if exactly one of the two is null.  A failed record makes
+ * the decode call return AKV_ERR_CUDA.
+ */
+akv_status akv_decode_set_events(void* after_scores, void* after_decode);
 
 #ifdef __cplusplus
 } /* extern "C" */

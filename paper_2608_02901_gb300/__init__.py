@@ -24,7 +24,7 @@ HEAD_DIM = 128
 EXPORTED = (
     "akv_status_string", "akv_last_error", "akv_unit_shapes", "akv_cache_size", "akv_cache_header_host",
     "akv_encode", "akv_encode_noalloc", "akv_cache_pack_host", "akv_decode_workspace_size", "akv_decode_attn",
-    "akv_decode_set_debug", "akv_cache_size_select", "akv_encode_select",
+    "akv_decode_set_debug", "akv_decode_set_events", "akv_cache_size_select", "akv_encode_select",
 )
 NOALLOC_SCRATCH_BYTES = 16 << 20
 
@@ -135,6 +135,8 @@ def lib():
                                         ctypes.c_size_t, vp]
         L.akv_decode_set_debug.restype = st
         L.akv_decode_set_debug.argtypes = [ctypes.c_int32, ctypes.c_int32]
+        L.akv_decode_set_events.restype = st
+        L.akv_decode_set_events.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
         _lib = L
     return _lib
 
@@ -316,6 +318,15 @@ def akv_decode_set_debug(ctas: int = 0, withhold_last: int = 0):
     """Testing controls of the decode launch (0, 0 = normal operation): the number of decode
     CTAs (0 = one per SM), and withholding each CTA's last tile block."""
     _check(lib().akv_decode_set_debug(int(ctas), int(withhold_last)), "akv_decode_set_debug")
+
+
+def akv_decode_set_events(after_scores=None, after_decode=None):
+    """Timing aid: torch.cuda.Event objects (already recorded once, so that their CUDA events
+    exist) that every later decode call records after its score launch and after its decode
+    launch; call with no arguments to clear."""
+    a = ctypes.c_void_p(after_scores.cuda_event) if after_scores is not None else None
+    b = ctypes.c_void_p(after_decode.cuda_event) if after_decode is not None else None
+    _check(lib().akv_decode_set_events(a, b), "akv_decode_set_events")
 
 
 def unit_host_from_logical(u: dict) -> dict:

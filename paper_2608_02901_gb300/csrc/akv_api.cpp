@@ -472,6 +472,14 @@ akv_status akv_decode_set_debug(int32_t ctas, int32_t withhold_last) {
   return AKV_OK;
 }
 
+akv_status akv_decode_set_events(void* after_scores, void* after_decode) {
+  g_last_error.clear();
+  if ((after_scores == nullptr) != (after_decode == nullptr))
+    return fail(AKV_ERR_INVALID, "both events must be given, or neither");
+  set_decode_events(after_scores, after_decode);
+  return AKV_OK;
+}
+
 akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_lens_host, size_t* ws_bytes) {
   g_last_error.clear();
   Layout L;

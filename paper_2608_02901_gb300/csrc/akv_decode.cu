@@ -1,36 +1,42 @@
 // Decode attention read directly from the AnchorKV compressed cache (Eq. 3 folded into
-// Eq. 4: no key or value row is ever rebuilt in memory).  Two launches per call:
+// Eq. 4: no key or value row is ever rebuilt in memory).  Two launches per call, in stream
+// order:
 //
 // 1. akv_scores_kernel.  The anchor scores S_A[a][g] = q_g . k_a of every anchor of every
-//    unit, once per anchor (Eq. 2-3), bf16 tensor cores, in log2 units with sm_scale
-//    folded in, into the workspace; with the largest score per query head of each chunk of
-//    64 anchors.  It streams the anchor keys, a fifth of the compressed bytes, at full width.
+//    unit, once per anchor (Eq. 2-3), bf16 tensor cores, in log2 units with sm_scale folded
+//    in, into the workspace, with the largest score per query head of each chunk of 64
+//    anchors.  It streams the anchor keys, a fifth of the compressed bytes, at full width.
+//    Its first chunk of each unit also writes the unit's query header (the rotated query
+//    q' = H(s o q)/128 of Appendix A.1 Eq. 12, its sums per head, and q' as tensor-core
+//    fragments for the key residuals) and zeroes the unit's arrival counter.
 //
 // 2. akv_decode_kernel.  Persistent: one CTA per SM.  The tile blocks of all units, in unit
 //    order, are split into equal contiguous ranges, one per CTA (stream-K): a unit's tiles may
-//    lie in several CTAs and a CTA's range may cross units (its segments).  Per CTA:
-//      producer warp   one lane streams each tile block, followed by the anchor-value rows of
-//                      the value slots the tile covers (the tile table records the range),
-//                      into a byte ring of shared memory with one bulk asynchronous copy
-//                      each, completing a transaction-counted mbarrier; per segment it also
-//                      copies the unit's anchor-score table and flushes the CTA's overflow sums;
-//      2 groups of 4 warps  each group takes every other tile of the range, end to end:
-//        key residuals  q' . c of the staged key records on tensor cores (q' = H(s o q)/128,
-//                       Appendix A.1 Eq. 12), written over the records' codes;
-//        tokens         each lane 8 consecutive stored tokens, every head: logits
-//                       gamma_i S_A[a(i)] + residual term, p = 2^(l - m), the normaliser,
-//                       p rows of the value records, and the value weights
-//                       w[a] = sum_i p_i gamma_i (Eq. 3): tokens are stored sorted by value
-//                       anchor, so a lane sums a run in registers and adds it into the
-//                       tile's weight table when the anchor changes;
-//        value side     the value-residual sum (p scale) c over the records and the
-//                       anchor-value product w^T V_A over the tile's slots, both on tensor
-//                       cores (weights and p scale as bf16 high + low parts, codes exact),
-//                       accumulated in registers across the segment's tiles.
-//    At the end of a segment every group (and the producer, for the overflow sums) stores its
-//    partial numerator and normaliser into its own workspace slot and counts itself in on the
-//    unit's counter; the one that completes the count sums the unit's slots in a fixed order,
-//    applies the inverse rotation once (Appendix E.1) and writes the output.
+//    lie in several CTAs and a CTA's range may cross units (its segments).  A CTA has two
+//    groups of four warps; each group takes every other tile of the range, end to end:
+//      staging        the group's warp 0 issues its own tiles into its half of a byte ring of
+//                     shared memory: one bulk asynchronous copy of the tile block and one of
+//                     the anchor-value rows of the value slots the tile covers (the tile
+//                     table records the range), completing a transaction-counted mbarrier;
+//                     table entries are read one issue ahead;
+//      key residuals  q' . c of the tile's staged key records on tensor cores, the terms
+//                     scale (q' . c) + min sum(q') written over the records' own codes;
+//      tokens         each lane 8 consecutive stored tokens, every head: logits
+//                     gamma_i S_A[a(i)] + residual term, p = 2^(l - m), the normaliser, p
+//                     rows of the value records, and the value weights w[a] = sum_i p_i
+//                     gamma_i (Eq. 3): tokens are stored sorted by value anchor, so runs
+//                     inside a lane are summed in registers and stored, and runs across
+//                     lanes merged by a warp segmented scan, without shared atomics;
+//      value side     the value-residual sum (p scale) c over the records and the anchor-
+//                     value product w^T V_A over the tile's slots, both on tensor cores
+//                     (weights and p scale as bf16 high + low parts, codes exact),
+//                     accumulated in registers across the segment's tiles.
+//    At the end of a segment both groups add their sums into the CTA's shared sums; the group
+//    that finishes last applies the inverse rotation once (Appendix E.1), stores the CTA's
+//    partial numerator and normaliser into its workspace slot for the unit, and counts it in
+//    on the unit's counter; the CTA that completes the count sums the unit's slots in a fixed
+//    order and writes the output.  Tiles denser than the staged counts, and runs on value
+//    slots beyond a tile's staged anchor-value rows, take CUDA-core paths.
 //
 // The exponent reference m is the largest anchor score of each query row.  Anchors are
 // tokens of the unit, so it is a lower bound of the largest logit (sums cannot overflow unless
@@ -88,7 +94,6 @@ struct ScoreParams {
   const __nv_bfloat16* q;
   uint8_t* uh;     // [units] query headers, uh_stride bytes apart
   int uh_stride, rotate;
-  int prefetch_l2; // 1: the arena fits the L2 cache; every unit's decode data is prefetched into it
   unsigned long long sign_lo, sign_hi;
   float* sa;      // [units][ka_stride][G] anchor scores (log2 units)
   float* cmax;    // [units][n_ch][G] largest score of each chunk of CHA anchors
@@ -188,10 +193,6 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
                : "memory");
 }
 __device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
-// Programmatic dependent launch: the next launch in the stream may be scheduled while this
-// one runs; before it reads inputs or writes outputs, a launch waits for the preceding work.
-__device__ __forceinline__ void pdl_allow_next() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
-__device__ __forceinline__ void pdl_wait_prev() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 // Reduction (no return value) into this CTA's shared memory.
 __device__ __forceinline__ void red_local(float* p, float v) {
   asm volatile("red.shared.add.f32 [%0], %1;" ::"r"(smem_u32(p)), "f"(v) : "memory");
@@ -213,10 +214,6 @@ __device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t& r0, uint3
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
                : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                : "r"(addr));
-}
-// Asynchronous prefetch of [p, p + bytes) into the L2 cache (16-byte aligned, a multiple of 16).
-__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
 // 16 bytes of read-only global data, not kept in L1 (streamed once)
@@ -490,22 +487,12 @@ __device__ __forceinline__ void load_row(const float* p, float (&out)[GS]) {
 // contiguous: thread (r8, c4) of k-pair step j holds dims 32 j + 8 c4 .. + 7 of rows r8, r8 + 8).
 template <int GS>
 __global__ void __launch_bounds__(128) akv_scores_kernel(const ScoreParams P) {
-  pdl_wait_prev();
-  pdl_allow_next();
   __shared__ float wmax[4][8];
   const int u = blockIdx.x / P.n_ch, ch = blockIdx.x % P.n_ch;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, r8 = lane >> 2, c4 = lane & 3;
   const akv_unit_desc* d = unit_desc(P.arena, u);
   const int k = d->n_anchors;
   if (ch == 0 && threadIdx.x == 0) P.cnt[u] = 0u;
-  if (P.prefetch_l2 && threadIdx.x == 0) {
-    // the decode launch's reads of this unit (anchor values, tile table, tile blocks: one range
-    // of the arena) start from L2 instead of a chain of cold HBM reads; chunk ch takes its share
-    const uint64_t b0 = d->off_anchor_v, b1 = d->off_tiles + d->tiles_capacity;
-    const uint64_t per = (((b1 - b0) + P.n_ch - 1) / P.n_ch + 15) & ~15ull;
-    const uint64_t s0 = b0 + per * ch, s1 = (s0 + per < b1 ? s0 + per : b1) & ~15ull;
-    for (uint64_t a = s0; a < s1; a += (1ull << 20)) prefetch_l2(P.arena + a, (uint32_t)(s1 - a < (1ull << 20) ? s1 - a : (1ull << 20)));
-  }
   const int a0 = ch * CHA + 16 * warp;
   float mx0 = -INFINITY, mx1 = -INFINITY;  // heads 2 c4, 2 c4 + 1
   if (a0 < k) {
@@ -868,10 +855,6 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     for (int e = tid; e < P.R * 8; e += NT) pvz[e] = 0.f;
   }
   __syncthreads();
-  pdl_allow_next();
-  // Everything above touches only this CTA's shared memory; from here on the launch reads
-  // the cache, the query and the anchor scores, and writes outputs.
-  pdl_wait_prev();
 
   // This CTA's range of the concatenated tiles, walked as segments (one per unit it touches).
   const long long B0 = (long long)c * P.ttot / P.grid, B1 = (long long)(c + 1) * P.ttot / P.grid;
@@ -1641,6 +1624,15 @@ struct LaunchKey {
 }  // namespace
 
 std::atomic<int> g_debug_cluster{0}, g_debug_withhold{0};
+namespace {
+std::mutex g_events_mu;
+cudaEvent_t g_ev_scores = nullptr, g_ev_decode = nullptr;
+}  // namespace
+void set_decode_events(void* after_scores, void* after_decode) {
+  std::lock_guard<std::mutex> lk(g_events_mu);
+  g_ev_scores = (cudaEvent_t)after_scores;
+  g_ev_decode = (cudaEvent_t)after_decode;
+}
 
 // Workspace of a decode call: anchor scores, chunk maxima, arrival counters, partial slots.
 DecodeWs decode_ws_layout(const Layout& L) {
@@ -1751,22 +1743,20 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   S.rotate = P.rotate;
   S.sign_lo = P.sign_lo;
   S.sign_hi = P.sign_hi;
-  // small arenas (a few layers fit the 129 MB L2 several times over) are prefetched into L2
-  S.prefetch_l2 = L.total_bytes <= (64ull << 20) ? 1 : 0;
-
-  cudaLaunchAttribute attr[1];
-  // each launch may overlap the tail of the preceding one (griddepcontrol in the kernels)
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(units * P.n_ch), 1, 1);
   cfg.blockDim = dim3(128, 1, 1);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = (cudaStream_t)stream;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cudaEvent_t ev_scores = nullptr, ev_decode = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(g_events_mu);
+    ev_scores = g_ev_scores;
+    ev_decode = g_ev_decode;
+  }
   cudaError_t e = cudaLaunchKernelEx(&cfg, score_kernel<GS>(), S);
   if (e != cudaSuccess) return (int)e;
+  if (ev_scores && (e = cudaEventRecord(ev_scores, cfg.stream)) != cudaSuccess) return (int)e;
   cfg.gridDim = dim3((unsigned)pl.grid, 1, 1);
   cfg.blockDim = dim3(NT, 1, 1);
   cfg.dynamicSmemBytes = pl.smem;
@@ -1779,6 +1769,7 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
            std::to_string(fa.maxDynamicSharedSizeBytes) + ", grid " + std::to_string(pl.grid) + ")";
     return (int)e;
   }
+  if (ev_decode && (e = cudaEventRecord(ev_decode, cfg.stream)) != cudaSuccess) return (int)e;
   return (int)cudaGetLastError();
 }
 

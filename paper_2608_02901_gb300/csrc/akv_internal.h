@@ -126,6 +126,9 @@ int launch_decode(const Layout& L, const akv_params& p, const void* arena, const
 const char* cuda_error_string(int err);
 // Testing controls of the decode launch (akv_decode_set_debug), 0 = normal operation.
 extern std::atomic<int> g_debug_cluster, g_debug_withhold;
+// Timing aid of the decode launch (akv_decode_set_events): events recorded after each of
+// its two launches; both null = off.
+void set_decode_events(void* after_scores, void* after_decode);
 // Device address of the library's static encode scratch on the current device
 // and context (looked up on every call); returns a cudaError_t as int.
 int noalloc_scratch(void** ptr, size_t* bytes);

@@ -205,6 +205,8 @@ def test_decode_debug_controls_validate():
     assert _err(akv.akv_decode_set_debug, -1, 0) == akv.AKV_ERR_INVALID
     assert _err(akv.akv_decode_set_debug, 0, 2) == akv.AKV_ERR_INVALID
     akv.akv_decode_set_debug(0, 0)
+    assert akv.lib().akv_decode_set_events(ctypes.c_void_p(16), None) == akv.AKV_ERR_INVALID
+    assert akv.lib().akv_decode_set_events(None, None) == akv.AKV_OK
 
 
 def test_select_parameters_validate_and_size_the_pooled_capacity():

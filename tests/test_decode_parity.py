@@ -190,9 +190,8 @@ def test_tiles_covering_more_value_slots_than_the_weight_table(dev, debug_contro
 
 
 def test_back_to_back_launches_follow_stream_order(dev):
-    """Consecutive decode launches in one stream overlap their set-up (programmatic dependent
-    launch) but not their data: a launch whose query is the previous launch's output, and a
-    launch that overwrites a buffer an earlier one read, both see stream order."""
+    """Consecutive decode calls in one stream see stream order: a call whose query is the
+    previous call's output, and a call that overwrites a buffer an earlier one read."""
     p = akv.Params(batch=2, n_kv_heads=2, n_q_heads=8, seed=3, rot_seed=77)
     lens = [6001, 3000]
     ua = seeded_units(p, lens, seed=5)
