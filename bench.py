@@ -79,6 +79,9 @@ def parse():
     ap.add_argument("--workload", default="70b-128k", choices=sorted(WORKLOADS))
     ap.add_argument("--layers", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--suffix", type=int, default=0,
+                    help="exact dense suffix: this many generated tokens per request, kept in bf16 and attended in "
+                         "the same softmax (0 = none)")
     ap.add_argument("--launch-check", action="store_true",
                     help="start the ranks, have each report itself through the process group, print them and exit "
                          "(checks the N-rank launch; measures nothing)")
@@ -359,12 +362,25 @@ def run_akv(args, rank, world, local):
     out = torch.empty((n_tok, layers, B, Hq, 128), dtype=torch.bfloat16, device=dev)
     chunk = n_tok * layers
 
+    # the exact dense suffix of each layer (generated tokens in bf16), the same length for every request
+    sfx = [None] * layers
+    suffix_bytes = 0
+    if args.suffix > 0:
+        for layer in range(layers):
+            kv = gen.queries_torch(2 * B * H * args.suffix, seed=5000 + 97 * layer + rank, device=dev)
+            kv = kv.view(2, B, H, args.suffix, 128)
+            sfx[layer] = akv.Suffix(kv[0].contiguous(), kv[1].contiguous(),
+                                    torch.full((B,), args.suffix, dtype=torch.int32, device=dev))
+        suffix_bytes = B * H * args.suffix * 2 * 256  # key and value rows, read by the score launch
+        step_bytes += suffix_bytes
+
     # one decode workspace (anchor scores, partial sums) serves every call: they are stream-ordered
-    dws = torch.empty(akv.akv_decode_workspace_size(p, lens), dtype=torch.uint8, device=dev)
+    dws = torch.empty(akv.akv_decode_workspace_size(p, lens, args.suffix), dtype=torch.uint8, device=dev)
 
     def step(i, stream=None):
         t, layer = divmod(i % chunk, layers)
-        akv.akv_decode_attn(p, lens, arenas[layer], qs[t, layer], out[t, layer], None, 1.0, dws, stream)
+        akv.akv_decode_attn(p, lens, arenas[layer], qs[t, layer], out[t, layer], None, 1.0, dws, stream,
+                            suffix=sfx[layer])
 
     # warm-up (also sets kernel attributes before capture)
     for i in range(min(args.warmup, chunk)):
@@ -416,7 +432,7 @@ def run_akv(args, rank, world, local):
     # each launch of the step on its own, after the timed region (same layers, same order)
     us_scores, us_decode = time_launches(torch, akv, step, min(args.steps, max(chunk, 256)), stream)
     kb = [arena_kernel_bytes(torch, akv, p, lens, a) for a in arenas]
-    scores_bytes = sum(b[0] for b in kb) / len(kb)
+    scores_bytes = sum(b[0] for b in kb) / len(kb) + suffix_bytes
     decode_bytes = sum(b[1] for b in kb) / len(kb)
     value = world * step_bytes * args.steps / sec / 1e9
     us_step = ms * 1e3 / args.steps
@@ -437,7 +453,7 @@ def run_akv(args, rank, world, local):
 
     def e2e_ops(i, s):
         q_dev.copy_(q_host[i], non_blocking=True)
-        akv.akv_decode_attn(p, lens, arenas[i % layers], q_dev, o_dev, None, 1.0, dws, s)
+        akv.akv_decode_attn(p, lens, arenas[i % layers], q_dev, o_dev, None, 1.0, dws, s, suffix=sfx[i % layers])
         o_host[i].copy_(o_dev, non_blocking=True)
 
     e2e_graphs = []
@@ -506,6 +522,7 @@ def run_akv(args, rank, world, local):
         "config": {"workload": args.workload, "batch": B, "n_kv_heads": H, "n_q_heads": Hq,
                    "context": S if args.workload not in SWEEP_POINTS else f"ragged U[8192, 131072]: {lens}",
                    "anchor_frac": p.anchor_frac, "res_frac": p.res_frac_k, "layers_cycled": layers,
+                   "suffix_tokens": args.suffix,
                    "fresh_queries": N_TOKENS, "arena_bytes_per_layer": arena_bytes,
                    "l2": f"inputs larger than L2: {layers} distinct layer caches, {layers * arena_bytes / 1e6:.0f} MB cycled",
                    "timing": "CUDA graph replay, CUDA events on the launching stream", "parallelism": f"dp{world}"},

@@ -402,6 +402,70 @@ akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, co
                            size_t arena_bytes, const void* q, void* out, float* out_f32, float sm_scale,
                            void* ws, size_t ws_bytes, akv_stream_t stream);
 
+/* ---- Exact dense suffix (generated tokens) -------------------------------- */
+
+/*
+ * Tokens produced during decoding stay exact: their keys and values are
+ * appended in bf16 to a dense suffix and never compressed, and the compressed
+ * prefix and the suffix are attended in one softmax (Appendix E.1, the combine
+ * kernel; Appendix E.2, generated tokens).  The suffix is caller-owned device
+ * memory; its lengths live on the device, so that an append and a decode can be
+ * replayed from one CUDA graph step after step.
+ *   K, V : device bf16 [B][H_kv][cap][128]: row t of (request b, KV head h) at
+ *          ((b H_kv + h) cap + t) 128 elements (keys as the caller's model uses
+ *          them, the same as the keys given to akv_encode)
+ *   len  : device int32 [B]: the tokens held by each request, 0 .. cap; rows at
+ *          or past len are never read
+ *   cap  : tokens per (request, KV head), 1 .. AKV_MAX_SUFFIX
+ */
+#define AKV_MAX_SUFFIX (1 << 20)
+typedef struct akv_suffix {
+  const void* K;
+  const void* V;
+  const int32_t* len;
+  int32_t cap;
+} akv_suffix;
+
+/*
+ * Workspace of akv_decode_attn_suffix for a suffix of at most suffix_cap tokens
+ * per request: akv_decode_workspace_size's, plus one partial slot (about
+ * 0.5 KB per query head) per unit and chunk of 64 suffix tokens.  suffix_cap 0
+ * gives akv_decode_workspace_size's value.
+ * Errors: AKV_ERR_INVALID (bad parameters, suffix_cap < 0 or > AKV_MAX_SUFFIX).
+ */
+akv_status akv_decode_workspace_size_suffix(const akv_params* p, const int32_t* ctx_lens_host, int32_t suffix_cap,
+                                            size_t* ws_bytes);
+
+/*
+ * akv_decode_attn over the compressed prefix and the dense suffix together:
+ * for request b with n = suffix->len[b] suffix tokens,
+ *     out = sum_{i < S_b} w_i x^V_i + sum_{t < n} w_{S_b + t} V_suf[t],
+ *     w = softmax over the S_b + n logits sm_scale q . x^K_i and sm_scale q . K_suf[t].
+ * suffix NULL is akv_decode_attn.  The score launch also scores each chunk of
+ * 64 suffix tokens and sums its values under the chunk's own maximum; the unit's
+ * combine rescales those partials to the common maximum (one softmax, exactly).
+ *   ws : >= akv_decode_workspace_size_suffix(p, ctx_lens_host, suffix->cap)
+ * Errors: those of akv_decode_attn, and AKV_ERR_INVALID for a suffix with null
+ * or misaligned pointers (K, V 16-byte aligned; len 4-byte) or cap out of range.
+ * Lengths above cap are taken as cap.
+ */
+akv_status akv_decode_attn_suffix(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,
+                                  size_t arena_bytes, const void* q, void* out, float* out_f32, float sm_scale,
+                                  const akv_suffix* suffix, void* ws, size_t ws_bytes, akv_stream_t stream);
+
+/*
+ * The append path (Appendix E.2): one new token per request.  For every request b
+ * with len[b] < cap, rows K_new[b][h] and V_new[b][h] (device bf16 [B][H_kv][128])
+ * are copied to row len[b] of (b, h) in K_suf and V_suf, and len[b] is then
+ * incremented, on the device.  A request whose suffix is full (len[b] >= cap) is
+ * left unchanged; its len stays at cap, which is how the caller sees it.
+ * One launch on `stream`; the lengths are read and written only by it.
+ * Errors: AKV_ERR_INVALID (bad parameters, null or misaligned pointers: rows
+ * 16-byte aligned, len 4-byte aligned; cap out of range), AKV_ERR_CUDA.
+ */
+akv_status akv_suffix_append(const akv_params* p, const void* K_new, const void* V_new, void* K_suf, void* V_suf,
+                             int32_t* len, int32_t cap, akv_stream_t stream);
+
 /* ---- Testing and tuning controls ------------------------------------------ */
 
 /*

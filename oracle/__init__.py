@@ -74,6 +74,7 @@ def lib():
             L.or_encode_batch.argtypes = [vp, vp, i32, i32, i32, i32, u64, u64, ctypes.c_int, vp]
             L.or_attend_unit.argtypes = [ctypes.POINTER(_OrUnit), vp, i32, dbl, u64, ctypes.c_int, vp]
             L.or_attend_batch.argtypes = [vp, i32, vp, i32, dbl, u64, ctypes.c_int, vp, vp]
+            L.or_attend_batch_suffix.argtypes = [vp, i32, i32, vp, i32, dbl, u64, ctypes.c_int, vp, vp, vp, i32, vp]
             L.or_attend_factorized.argtypes = [ctypes.POINTER(_OrUnit), vp, i32, dbl, u64, ctypes.c_int, vp]
             L.or_reconstruct_side.argtypes = [i32, vp, vp, vp, i32, vp, vp, vp, vp, u64, ctypes.c_int, vp]
             L.or_quantize_residual.argtypes = [vp, u64, ctypes.c_int, vp, vp, vp]
@@ -294,6 +295,26 @@ def attend(units, q: np.ndarray, G: int, sm_scale: float, rot_seed: int, rotate:
         selp = _p(sel_arr)
     lib().or_attend_batch(ctypes.cast(structs, ctypes.c_void_p), n, _p(q), G, float(sm_scale),
                           ctypes.c_uint64(rot_seed), int(bool(rotate)), selp, _p(out))
+    return out
+
+
+def attend_suffix(units, q: np.ndarray, G: int, H: int, sm_scale: float, rot_seed: int, ksuf: np.ndarray,
+                  vsuf: np.ndarray, suf_len, rotate: bool = True) -> np.ndarray:
+    """Attention over each unit's compressed positions and the first suf_len[b] rows of its exact
+    dense suffix, in one softmax (Appendix E.1, E.2).  ksuf, vsuf: uint16 bf16 bits
+    [n_units][cap][128] (unit u = b*H + h); suf_len: int [B].  Returns fp64 [n_units][G][128]."""
+    n = len(units)
+    q = np.ascontiguousarray(q, dtype=np.uint16).reshape(n, G, D)
+    ksuf = np.ascontiguousarray(ksuf, dtype=np.uint16)
+    vsuf = np.ascontiguousarray(vsuf, dtype=np.uint16)
+    assert ksuf.shape == vsuf.shape and ksuf.shape[0] == n and ksuf.shape[2] == D
+    lens = np.ascontiguousarray(np.minimum(np.asarray(suf_len, dtype=np.int32), ksuf.shape[1]), dtype=np.int32)
+    assert lens.shape == (n // H,)
+    out = np.zeros((n, G, D), np.float64)
+    structs = (_OrUnit * n)(*[u.c_struct() for u in units])
+    lib().or_attend_batch_suffix(ctypes.cast(structs, ctypes.c_void_p), n, H, _p(q), G, float(sm_scale),
+                                 ctypes.c_uint64(rot_seed), int(bool(rotate)), _p(ksuf), _p(vsuf), _p(lens),
+                                 int(ksuf.shape[1]), _p(out))
     return out
 
 

@@ -22,7 +22,9 @@
  *             (Appendix A.1 accounting) split floor(N/2) keys, the rest
  *             values, each side's top-N pooled over the layer's KV heads.
  *   attend  : Eq. 3 reconstruction of every key and value, then Eq. 4
- *             softmax attention, all in fp64, one token at a time.
+ *             softmax attention, all in fp64, one token at a time; with an
+ *             exact dense suffix (Appendix E.1 and E.2: generated tokens kept
+ *             in bf16) the suffix tokens join the same softmax.
  *   attend_factorized : the same attention regrouped by anchor (anchor
  *             scores computed once, value weights summed per anchor, inverse
  *             rotation applied once after accumulation -- Section 4.4 and
@@ -428,12 +430,16 @@ void or_reconstruct_side(int32_t S, const uint16_t* anchors, const uint16_t* idx
   }
 }
 
-/* Definitional attention for one unit: G query rows (bf16 bits [G][128]),
- * out [G][128] fp64.  Each key and value is rebuilt per Eq. 3 and the
- * softmax of Eq. 4 is taken over all S positions. */
-void or_attend_unit(const or_unit* u, const uint16_t* q, int32_t G, double sm_scale, uint64_t rot_seed, int rotate,
-                    double* out) {
+/* Definitional attention for one unit with an exact dense suffix: G query
+ * rows (bf16 bits [G][128]), out [G][128] fp64.  Each key and value of the
+ * S compressed positions is rebuilt per Eq. 3; the nsuf suffix tokens (bf16
+ * rows ksuf, vsuf [nsuf][128], kept exact: Appendix E.2) follow them, and the
+ * softmax of Eq. 4 is taken over all S + nsuf positions at once (the combine
+ * of Appendix E.1 attends both under the same softmax). */
+void or_attend_unit_suffix(const or_unit* u, const uint16_t* q, int32_t G, double sm_scale, uint64_t rot_seed,
+                           int rotate, const uint16_t* ksuf, const uint16_t* vsuf, int32_t nsuf, double* out) {
   int32_t S = u->S;
+  int32_t n = S + nsuf; /* positions of the softmax */
   double s[OR_D];
   or_signs(rot_seed, s);
   int32_t* slot_k = (int32_t*)malloc(sizeof(int32_t) * (size_t)S);
@@ -441,18 +447,22 @@ void or_attend_unit(const or_unit* u, const uint16_t* q, int32_t G, double sm_sc
   for (int32_t i = 0; i < S; ++i) slot_k[i] = slot_v[i] = -1;
   for (int32_t t = 0; t < u->nk; ++t) slot_k[u->res_k[t]] = t;
   for (int32_t t = 0; t < u->nv; ++t) slot_v[u->res_v[t]] = t;
-  double* logit = (double*)malloc(sizeof(double) * (size_t)S * (size_t)G);
+  double* logit = (double*)malloc(sizeof(double) * (size_t)n * (size_t)G);
   double x[OR_D], rt[OR_D], qd[8][OR_D];
   for (int32_t g = 0; g < G; ++g)
     for (int j = 0; j < OR_D; ++j) qd[g][j] = or_bf16_to_double(q[(size_t)g * OR_D + j]);
-  for (int32_t i = 0; i < S; ++i) {
-    double gk = or_fp16_to_double(u->gam_k[i]);
-    const uint16_t* xa = u->anchor_k + (size_t)u->idx_k[i] * OR_D;
-    for (int j = 0; j < OR_D; ++j) x[j] = gk * or_bf16_to_double(xa[j]);
-    if (slot_k[i] >= 0) {
-      int32_t t = slot_k[i];
-      or_dequant_residual(u->codes_k + (size_t)t * 32, u->scale_k[t], u->min_k[t], s, rotate, rt);
-      for (int j = 0; j < OR_D; ++j) x[j] += rt[j];
+  for (int32_t i = 0; i < n; ++i) {
+    if (i < S) {
+      double gk = or_fp16_to_double(u->gam_k[i]);
+      const uint16_t* xa = u->anchor_k + (size_t)u->idx_k[i] * OR_D;
+      for (int j = 0; j < OR_D; ++j) x[j] = gk * or_bf16_to_double(xa[j]);
+      if (slot_k[i] >= 0) {
+        int32_t t = slot_k[i];
+        or_dequant_residual(u->codes_k + (size_t)t * 32, u->scale_k[t], u->min_k[t], s, rotate, rt);
+        for (int j = 0; j < OR_D; ++j) x[j] += rt[j];
+      }
+    } else {
+      for (int j = 0; j < OR_D; ++j) x[j] = or_bf16_to_double(ksuf[(size_t)(i - S) * OR_D + j]);
     }
     for (int32_t g = 0; g < G; ++g) {
       double d = 0.0;
@@ -462,26 +472,30 @@ void or_attend_unit(const or_unit* u, const uint16_t* q, int32_t G, double sm_sc
   }
   for (int32_t g = 0; g < G; ++g) {
     double m = -INFINITY;
-    for (int32_t i = 0; i < S; ++i)
+    for (int32_t i = 0; i < n; ++i)
       if (logit[(size_t)i * G + g] > m) m = logit[(size_t)i * G + g];
     double den = 0.0;
-    for (int32_t i = 0; i < S; ++i) {
+    for (int32_t i = 0; i < n; ++i) {
       double e = exp(logit[(size_t)i * G + g] - m);
       logit[(size_t)i * G + g] = e;
       den += e;
     }
-    for (int32_t i = 0; i < S; ++i) logit[(size_t)i * G + g] /= den;
+    for (int32_t i = 0; i < n; ++i) logit[(size_t)i * G + g] /= den;
   }
   for (int32_t g = 0; g < G; ++g)
     for (int j = 0; j < OR_D; ++j) out[(size_t)g * OR_D + j] = 0.0;
-  for (int32_t i = 0; i < S; ++i) {
-    double gv = or_fp16_to_double(u->gam_v[i]);
-    const uint16_t* xa = u->anchor_v + (size_t)u->idx_v[i] * OR_D;
-    for (int j = 0; j < OR_D; ++j) x[j] = gv * or_bf16_to_double(xa[j]);
-    if (slot_v[i] >= 0) {
-      int32_t t = slot_v[i];
-      or_dequant_residual(u->codes_v + (size_t)t * 32, u->scale_v[t], u->min_v[t], s, rotate, rt);
-      for (int j = 0; j < OR_D; ++j) x[j] += rt[j];
+  for (int32_t i = 0; i < n; ++i) {
+    if (i < S) {
+      double gv = or_fp16_to_double(u->gam_v[i]);
+      const uint16_t* xa = u->anchor_v + (size_t)u->idx_v[i] * OR_D;
+      for (int j = 0; j < OR_D; ++j) x[j] = gv * or_bf16_to_double(xa[j]);
+      if (slot_v[i] >= 0) {
+        int32_t t = slot_v[i];
+        or_dequant_residual(u->codes_v + (size_t)t * 32, u->scale_v[t], u->min_v[t], s, rotate, rt);
+        for (int j = 0; j < OR_D; ++j) x[j] += rt[j];
+      }
+    } else {
+      for (int j = 0; j < OR_D; ++j) x[j] = or_bf16_to_double(vsuf[(size_t)(i - S) * OR_D + j]);
     }
     for (int32_t g = 0; g < G; ++g) {
       double a = logit[(size_t)i * G + g];
@@ -491,6 +505,13 @@ void or_attend_unit(const or_unit* u, const uint16_t* q, int32_t G, double sm_sc
   free(logit);
   free(slot_k);
   free(slot_v);
+}
+
+/* Definitional attention for one unit (no suffix): the softmax of Eq. 4 over
+ * its S positions, each key and value rebuilt per Eq. 3. */
+void or_attend_unit(const or_unit* u, const uint16_t* q, int32_t G, double sm_scale, uint64_t rot_seed, int rotate,
+                    double* out) {
+  or_attend_unit_suffix(u, q, G, sm_scale, rot_seed, rotate, NULL, NULL, 0, out);
 }
 
 /* ------------------------------------------------------------------------ */
@@ -892,6 +913,20 @@ void or_attend_batch(const or_unit* units, int32_t n_units, const uint16_t* q, i
   for (int32_t u = 0; u < n_units; ++u) {
     if (sel && !sel[u]) continue;
     or_attend_unit(&units[u], q + (size_t)u * G * OR_D, G, sm_scale, rot_seed, rotate, out + (size_t)u * G * OR_D);
+  }
+}
+
+/* Batched attention with exact dense suffixes: unit u = b*H + h attends its
+ * S positions and the first suf_len[b] rows of its suffix block, rows
+ * ksuf/vsuf + (u * suf_cap + t) * 128 (bf16). */
+void or_attend_batch_suffix(const or_unit* units, int32_t n_units, int32_t H, const uint16_t* q, int32_t G,
+                            double sm_scale, uint64_t rot_seed, int rotate, const uint16_t* ksuf, const uint16_t* vsuf,
+                            const int32_t* suf_len, int32_t suf_cap, double* out) {
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int32_t u = 0; u < n_units; ++u) {
+    const size_t base = (size_t)u * (size_t)suf_cap * OR_D;
+    or_attend_unit_suffix(&units[u], q + (size_t)u * G * OR_D, G, sm_scale, rot_seed, rotate, ksuf + base, vsuf + base,
+                          suf_len[u / H], out + (size_t)u * G * OR_D);
   }
 }
 

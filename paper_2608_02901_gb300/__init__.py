@@ -25,7 +25,9 @@ EXPORTED = (
     "akv_status_string", "akv_last_error", "akv_unit_shapes", "akv_cache_size", "akv_cache_header_host",
     "akv_encode", "akv_encode_noalloc", "akv_cache_pack_host", "akv_decode_workspace_size", "akv_decode_attn",
     "akv_decode_set_debug", "akv_decode_set_events", "akv_cache_size_select", "akv_encode_select",
+    "akv_decode_workspace_size_suffix", "akv_decode_attn_suffix", "akv_suffix_append",
 )
+AKV_MAX_SUFFIX = 1 << 20
 NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
@@ -56,6 +58,10 @@ class SelectParams:
 
     def c(self) -> _SelectParams:
         return _SelectParams(self.theta, self.rho, self.kappa, 0)
+
+
+class _Suffix(ctypes.Structure):
+    _fields_ = [("K", ctypes.c_void_p), ("V", ctypes.c_void_p), ("len", ctypes.c_void_p), ("cap", ctypes.c_int32)]
 
 
 class _UnitHost(ctypes.Structure):
@@ -137,6 +143,13 @@ def lib():
         L.akv_decode_set_debug.argtypes = [ctypes.c_int32, ctypes.c_int32]
         L.akv_decode_set_events.restype = st
         L.akv_decode_set_events.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+        L.akv_decode_workspace_size_suffix.restype = st
+        L.akv_decode_workspace_size_suffix.argtypes = [P, i32p, ctypes.c_int32, sz]
+        L.akv_decode_attn_suffix.restype = st
+        L.akv_decode_attn_suffix.argtypes = [P, i32p, vp, ctypes.c_size_t, vp, vp, vp, ctypes.c_float,
+                                             ctypes.POINTER(_Suffix), vp, ctypes.c_size_t, vp]
+        L.akv_suffix_append.restype = st
+        L.akv_suffix_append.argtypes = [P, vp, vp, vp, vp, vp, ctypes.c_int32, vp]
         _lib = L
     return _lib
 
@@ -272,11 +285,13 @@ def akv_cache_pack_host(p: Params, ctx_lens, units) -> np.ndarray:
     return out
 
 
-def akv_decode_workspace_size(p: Params, ctx_lens) -> int:
+def akv_decode_workspace_size(p: Params, ctx_lens, suffix_cap: int = 0) -> int:
+    """Decode workspace bytes; with suffix_cap > 0, for akv_decode_attn with a dense suffix of at
+    most that many tokens per request."""
     lens = _lens(ctx_lens)
     w = ctypes.c_size_t()
-    _check(lib().akv_decode_workspace_size(ctypes.byref(p.c()), _i32p(lens), ctypes.byref(w)),
-           "akv_decode_workspace_size")
+    _check(lib().akv_decode_workspace_size_suffix(ctypes.byref(p.c()), _i32p(lens), int(suffix_cap), ctypes.byref(w)),
+           "akv_decode_workspace_size_suffix")
     return w.value
 
 
@@ -299,19 +314,52 @@ def _decode_args(p: Params, ctx_lens):
     return ent[2], ent[3]
 
 
-def akv_decode_attn(p: Params, ctx_lens, arena, q, out, out_f32=None, sm_scale: float = 1.0, ws=None, stream=None):
+def akv_decode_attn(p: Params, ctx_lens, arena, q, out, out_f32=None, sm_scale: float = 1.0, ws=None, stream=None,
+                    suffix=None):
     """q, out: CUDA bf16 [B][H_q][128]; out_f32 optional fp32 of the same shape.
-    ws: CUDA uint8 workspace of akv_decode_workspace_size bytes; when None, one is taken
-    from torch's allocator on out's device for this call."""
+    suffix: optional Suffix (the exact dense suffix attended in the same softmax).
+    ws: CUDA uint8 workspace of akv_decode_workspace_size(p, ctx_lens, suffix.cap) bytes; when
+    None, one is taken from torch's allocator on out's device for this call."""
     pref, lref = _decode_args(p, ctx_lens)
     if ws is None:
         import torch
-        ws = torch.empty(akv_decode_workspace_size(p, ctx_lens), dtype=torch.uint8, device=out.device)
+        ws = torch.empty(akv_decode_workspace_size(p, ctx_lens, suffix.cap if suffix is not None else 0),
+                         dtype=torch.uint8, device=out.device)
     ws_bytes = ws.numel() * ws.element_size()
-    _check(lib().akv_decode_attn(pref, lref, _dev_ptr(arena), arena.numel() * arena.element_size(), _dev_ptr(q),
-                                 _dev_ptr(out), _dev_ptr(out_f32), float(sm_scale), _dev_ptr(ws), ws_bytes,
-                                 _stream_ptr(stream)),
-           "akv_decode_attn")
+    args = (pref, lref, _dev_ptr(arena), arena.numel() * arena.element_size(), _dev_ptr(q), _dev_ptr(out),
+            _dev_ptr(out_f32), float(sm_scale))
+    if suffix is None:
+        _check(lib().akv_decode_attn(*args, _dev_ptr(ws), ws_bytes, _stream_ptr(stream)), "akv_decode_attn")
+    else:
+        _check(lib().akv_decode_attn_suffix(*args, ctypes.byref(suffix.c()), _dev_ptr(ws), ws_bytes,
+                                            _stream_ptr(stream)), "akv_decode_attn_suffix")
+
+
+class Suffix:
+    """The exact dense suffix of a batch (generated tokens): CUDA bf16 K and V [B][H_kv][cap][128]
+    and CUDA int32 lengths [B] (tokens held per request), all owned by the caller."""
+
+    def __init__(self, K, V, lens):
+        if K.dim() != 4 or tuple(K.shape) != tuple(V.shape) or K.shape[3] != HEAD_DIM:
+            raise ValueError("suffix K and V must be [B][H_kv][cap][128] of the same shape")
+        if str(K.dtype) != "torch.bfloat16" or str(V.dtype) != "torch.bfloat16" or str(lens.dtype) != "torch.int32":
+            raise ValueError("suffix K, V must be bf16 and lens int32")
+        if lens.numel() != K.shape[0]:
+            raise ValueError("suffix lens must hold one length per request")
+        self.K, self.V, self.lens = K, V, lens
+        self.cap = int(K.shape[2])
+        self._c = _Suffix(_dev_ptr(K), _dev_ptr(V), _dev_ptr(lens), self.cap)
+
+    def c(self):
+        return self._c
+
+
+def akv_suffix_append(p: Params, K_new, V_new, suffix: "Suffix", stream=None):
+    """Appends one token per request (K_new, V_new: CUDA bf16 [B][H_kv][128]) at each request's
+    length, on the device; requests whose suffix is full are left unchanged."""
+    _check(lib().akv_suffix_append(ctypes.byref(p.c()), _dev_ptr(K_new), _dev_ptr(V_new), _dev_ptr(suffix.K),
+                                   _dev_ptr(suffix.V), _dev_ptr(suffix.lens), suffix.cap, _stream_ptr(stream)),
+           "akv_suffix_append")
 
 
 def akv_decode_set_debug(ctas: int = 0, withhold_last: int = 0):

@@ -481,18 +481,31 @@ akv_status akv_decode_set_events(void* after_scores, void* after_decode) {
 }
 
 akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_lens_host, size_t* ws_bytes) {
+  return akv_decode_workspace_size_suffix(p, ctx_lens_host, 0, ws_bytes);
+}
+
+akv_status akv_decode_workspace_size_suffix(const akv_params* p, const int32_t* ctx_lens_host, int32_t suffix_cap,
+                                            size_t* ws_bytes) {
   g_last_error.clear();
   Layout L;
   akv_status st = make_layout(p, ctx_lens_host, &L);
   if (st != AKV_OK) return st;
   if (!ws_bytes) return fail(AKV_ERR_INVALID, "null ws_bytes");
-  *ws_bytes = decode_ws_layout(L).total;
+  if (suffix_cap < 0 || suffix_cap > AKV_MAX_SUFFIX) return fail(AKV_ERR_INVALID, "suffix_cap out of range");
+  *ws_bytes = decode_ws_layout(L, suffix_cap).total;
   return AKV_OK;
 }
 
 akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,
                            size_t arena_bytes, const void* q, void* out, float* out_f32, float sm_scale,
                            void* ws, size_t ws_bytes, akv_stream_t stream) {
+  return akv_decode_attn_suffix(p, ctx_lens_host, arena, arena_bytes, q, out, out_f32, sm_scale, nullptr, ws, ws_bytes,
+                                stream);
+}
+
+akv_status akv_decode_attn_suffix(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,
+                                  size_t arena_bytes, const void* q, void* out, float* out_f32, float sm_scale,
+                                  const akv_suffix* suffix, void* ws, size_t ws_bytes, akv_stream_t stream) {
   if (!g_last_error.empty()) g_last_error.clear();
   akv_status st;
   const std::shared_ptr<const Layout> Lp = decode_layout(p, ctx_lens_host, &st);
@@ -503,12 +516,40 @@ akv_status akv_decode_attn(const akv_params* p, const int32_t* ctx_lens_host, co
     return fail(AKV_ERR_INVALID, "arena must be 256-byte aligned; q, out, out_f32 16-byte aligned");
   if (arena_bytes < L.total_bytes) return fail(AKV_ERR_TOO_SMALL, "arena shorter than akv_cache_size");
   if (!std::isfinite(sm_scale)) return fail(AKV_ERR_INVALID, "sm_scale must be finite");
+  DecodeSuffix sfx;
+  if (suffix) {
+    if (!suffix->K || !suffix->V || !suffix->len) return fail(AKV_ERR_INVALID, "suffix: null K, V or len");
+    if (((uintptr_t)suffix->K % 16) || ((uintptr_t)suffix->V % 16) || ((uintptr_t)suffix->len % 4))
+      return fail(AKV_ERR_INVALID, "suffix: K and V must be 16-byte aligned, len 4-byte aligned");
+    if (suffix->cap < 1 || suffix->cap > AKV_MAX_SUFFIX) return fail(AKV_ERR_INVALID, "suffix: cap out of range");
+    sfx.K = suffix->K;
+    sfx.V = suffix->V;
+    sfx.len = suffix->len;
+    sfx.cap = suffix->cap;
+  }
   if (!ws || ((uintptr_t)ws % 256)) return fail(AKV_ERR_INVALID, "decode workspace must be non-null and 256-byte aligned");
-  if (ws_bytes < decode_ws_layout(L).total) return fail(AKV_ERR_TOO_SMALL, "decode workspace shorter than akv_decode_workspace_size");
+  if (ws_bytes < decode_ws_layout(L, sfx.cap).total)
+    return fail(AKV_ERR_TOO_SMALL, "decode workspace shorter than akv_decode_workspace_size(_suffix)");
   std::string why;
-  int err = launch_decode(L, *p, arena, q, out, out_f32, sm_scale, ws, (void*)stream, &why);
+  int err = launch_decode(L, *p, arena, q, out, out_f32, sm_scale, sfx, ws, (void*)stream, &why);
   if (err == -1) return fail(AKV_ERR_UNSUPPORTED, why);
   if (err) return fail(AKV_ERR_CUDA, std::string("decode launch failed: ") + cuda_error_string(err) + " " + why);
+  return AKV_OK;
+}
+
+akv_status akv_suffix_append(const akv_params* p, const void* K_new, const void* V_new, void* K_suf, void* V_suf,
+                             int32_t* len, int32_t cap, akv_stream_t stream) {
+  g_last_error.clear();
+  if (!p) return fail(AKV_ERR_INVALID, "null params");
+  if (p->batch < 1 || p->n_kv_heads < 1 || p->head_dim != AKV_HEAD_DIM)
+    return fail(AKV_ERR_INVALID, "batch and n_kv_heads must be >= 1, head_dim 128");
+  if (!K_new || !V_new || !K_suf || !V_suf || !len) return fail(AKV_ERR_INVALID, "null pointer");
+  if (((uintptr_t)K_new % 16) || ((uintptr_t)V_new % 16) || ((uintptr_t)K_suf % 16) || ((uintptr_t)V_suf % 16) ||
+      ((uintptr_t)len % 4))
+    return fail(AKV_ERR_INVALID, "rows must be 16-byte aligned, len 4-byte aligned");
+  if (cap < 1 || cap > AKV_MAX_SUFFIX) return fail(AKV_ERR_INVALID, "cap out of range");
+  const int err = launch_suffix_append(p->batch, p->n_kv_heads, K_new, V_new, K_suf, V_suf, len, cap, (void*)stream);
+  if (err) return fail(AKV_ERR_CUDA, std::string("suffix append launch failed: ") + cuda_error_string(err));
   return AKV_OK;
 }
 

@@ -89,6 +89,13 @@ __host__ __device__ constexpr int part_flag(int GS) { return 128 * GS + 8; }
 // sums [8] f32, and the key-residual mma B fragments [GS == 8 ? 2 : 1][8][32] uint2.
 __host__ __device__ constexpr int hdr_bytes(int GS) { return GS * 512 + 32 + (GS == 8 ? 2 : 1) * 2048; }
 
+// Dense suffix: tokens per chunk, and the floats of a chunk's partial slot: the value sum
+// o [GS][128] under the chunk's own maximum, its normaliser l [8] and that maximum m [8] (log2 units).
+constexpr int SCH = kSuffixChunk;
+__host__ __device__ constexpr int suf_floats(int GS) { return 128 * GS + 16; }
+__host__ __device__ constexpr int suf_l(int GS) { return 128 * GS; }
+__host__ __device__ constexpr int suf_m(int GS) { return 128 * GS + 8; }
+
 struct ScoreParams {
   const uint8_t* arena;
   const __nv_bfloat16* q;
@@ -100,6 +107,13 @@ struct ScoreParams {
   unsigned* cnt;  // [units] arrival counters of the decode launch, zeroed here
   int n_kv_heads, n_q_heads, G, ka_stride, n_ch;
   float scale_log2;
+  // dense suffix (null ksuf: none): rows [units][suf_cap][128], lengths per request, n_sch
+  // chunks of SCH tokens per unit, each a partial slot of suf_floats(G) floats
+  const __nv_bfloat16* ksuf;
+  const __nv_bfloat16* vsuf;
+  const int32_t* suf_len;
+  float* suf_part;
+  int suf_cap, n_sch;
 };
 
 struct Meta {  // a staged tile, as the producer recorded it
@@ -127,6 +141,9 @@ struct DecodeParams {
   int ring_bytes, drop_last, smem_sa;
   int o_bar, o_meta, o_misc, o_sa, o_ovf, o_grp, grp_bytes, o_ring;
   int g_qp, g_rows, g_red, g_wb, g_pv, g_qf;  // offsets inside a group's block
+  const float* suf_part;   // dense suffix partials [units][n_sch][suf_floats] (null: no suffix)
+  const int32_t* suf_len;  // suffix tokens per request
+  int suf_cap, n_sch;
   int cta_unit[kMaxGrid];  // first unit of each CTA's range
   int cta_tile[kMaxGrid];  // its first tile inside that unit
 };
@@ -485,10 +502,115 @@ __device__ __forceinline__ void load_row(const float* p, float (&out)[GS]) {
 // from global memory into the mma A fragments (rows are stored swizzled in 16-byte chunks by
 // slot % 8; the k order is permuted the same way in A and B so that a thread's dims are
 // contiguous: thread (r8, c4) of k-pair step j holds dims 32 j + 8 c4 .. + 7 of rows r8, r8 + 8).
+// Dense suffix chunk sc of unit u (Appendix E.1 and E.2): suffix tokens j0 .. j0 + 63 of its
+// request, scored against the unit's GS query rows on tensor cores (rows plain [token][128] bf16;
+// the same permuted k order as the anchor chunks), p = 2^(s - m_c) under the chunk's own maximum
+// m_c, then o[g][d] = sum_t p_t[g] V[t][d] (thread d) and l[g] = sum_t p_t[g] into the chunk's
+// partial slot.  Chunks at or past the request's length write nothing (the combine reads the
+// chunks below it only).
+template <int GS>
+__device__ __forceinline__ void suffix_chunk(const ScoreParams& P, int u, int sc) {
+  __shared__ float ps[SCH][8];
+  __shared__ float wm[4][8];
+  __shared__ float mc[8];
+  __shared__ __align__(16) __nv_bfloat16 vsm[SCH][128];
+  const int len = max(0, min(P.suf_len[u / P.n_kv_heads], P.suf_cap));
+  const int j0 = sc * SCH;
+  if (j0 >= len) return;
+  const int nv = min(SCH, len - j0);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, r8 = lane >> 2, c4 = lane & 3;
+  const uint8_t* Kr = reinterpret_cast<const uint8_t*>(P.ksuf) + (size_t)u * P.suf_cap * 256;
+  const uint8_t* Vr = reinterpret_cast<const uint8_t*>(P.vsuf) + (size_t)u * P.suf_cap * 256;
+  // the chunk's value rows, all in flight at once (row t / 16 + 8 i, 16-byte column t % 16),
+  // while the keys are scored
+  uint4 vrow[SCH / 8];
+#pragma unroll
+  for (int i = 0; i < SCH / 8; ++i) {
+    const int row = tid / 16 + 8 * i;
+    vrow[i] = row < nv ? ldg_stream(Vr + (size_t)(j0 + row) * 256 + 16 * (tid % 16)) : make_uint4(0u, 0u, 0u, 0u);
+  }
+  const size_t qb = qrow_base(u, P.n_kv_heads, P.n_q_heads);
+  uint2 bq[8];
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks)
+    bq[ks] = r8 < GS ? *reinterpret_cast<const uint2*>(P.q + qb + (size_t)r8 * 128 + 32 * (ks >> 1) + 8 * c4 + 4 * (ks & 1))
+                     : make_uint2(0u, 0u);
+  const int t0 = j0 + 16 * warp;
+  const int ra = min(t0 + r8, len - 1), rb = min(t0 + r8 + 8, len - 1);
+  uint4 lo[4], hi[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int cc = 4 * j + c4;
+    lo[j] = ldg_stream(Kr + (size_t)ra * 256 + 16 * cc);
+    hi[j] = ldg_stream(Kr + (size_t)rb * 256 + 16 * cc);
+  }
+  float dd[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    mma_bf16(dd, lo[j].x, hi[j].x, lo[j].y, hi[j].y, bq[2 * j].x, bq[2 * j].y);
+    mma_bf16(dd, lo[j].z, hi[j].z, lo[j].w, hi[j].w, bq[2 * j + 1].x, bq[2 * j + 1].y);
+  }
+  const int g0 = 2 * c4;
+  float sv[2][2];
+  float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const bool ok = t0 + r8 + 8 * h < len;
+    sv[h][0] = ok && g0 < GS ? dd[2 * h] * P.scale_log2 : -INFINITY;
+    sv[h][1] = ok && g0 + 1 < GS ? dd[2 * h + 1] * P.scale_log2 : -INFINITY;
+    mx0 = fmaxf(mx0, sv[h][0]);
+    mx1 = fmaxf(mx1, sv[h][1]);
+  }
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) {
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+  }
+  if (lane < 4) {
+    wm[warp][2 * lane] = mx0;
+    wm[warp][2 * lane + 1] = mx1;
+  }
+#pragma unroll
+  for (int i = 0; i < SCH / 8; ++i) *reinterpret_cast<uint4*>(&vsm[tid / 16 + 8 * i][8 * (tid % 16)]) = vrow[i];
+  __syncthreads();
+  if (tid < 8) mc[tid] = fmaxf(fmaxf(wm[0][tid], wm[1][tid]), fmaxf(wm[2][tid], wm[3][tid]));
+  __syncthreads();
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int row = 16 * warp + r8 + 8 * h;
+    if (g0 < GS) ps[row][g0] = sv[h][0] > -INFINITY ? exp2_approx(sv[h][0] - mc[g0]) : 0.f;
+    if (g0 + 1 < GS) ps[row][g0 + 1] = sv[h][1] > -INFINITY ? exp2_approx(sv[h][1] - mc[g0 + 1]) : 0.f;
+  }
+  __syncthreads();
+  float o[GS];
+#pragma unroll
+  for (int g = 0; g < GS; ++g) o[g] = 0.f;
+  for (int j = 0; j < nv; ++j) {  // thread tid: dimension tid of every row
+    const float v = __bfloat162float(vsm[j][tid]);
+#pragma unroll
+    for (int g = 0; g < GS; ++g) o[g] = fmaf(ps[j][g], v, o[g]);
+  }
+  float* dst = P.suf_part + ((size_t)u * P.n_sch + sc) * suf_floats(GS);
+#pragma unroll
+  for (int g = 0; g < GS; ++g) dst[g * 128 + tid] = o[g];
+  if (tid < GS) {
+    float l = 0.f;
+    for (int j = 0; j < nv; ++j) l += ps[j][tid];
+    dst[suf_l(GS) + tid] = l;
+    dst[suf_m(GS) + tid] = mc[tid];
+  }
+}
+
+// Grid: per unit, n_ch anchor chunks then n_sch dense-suffix chunks.
 template <int GS>
 __global__ void __launch_bounds__(128) akv_scores_kernel(const ScoreParams P) {
   __shared__ float wmax[4][8];
-  const int u = blockIdx.x / P.n_ch, ch = blockIdx.x % P.n_ch;
+  const int per = P.n_ch + P.n_sch;
+  const int u = blockIdx.x / per, ch = blockIdx.x % per;
+  if (ch >= P.n_ch) {
+    suffix_chunk<GS>(P, u, ch - P.n_ch);
+    return;
+  }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, r8 = lane >> 2, c4 = lane & 3;
   const akv_unit_desc* d = unit_desc(P.arena, u);
   const int k = d->n_anchors;
@@ -643,6 +765,38 @@ __device__ void combine_unit(const DecodeParams& P, int u, int first, int nseg, 
 #pragma unroll
     for (int g = 0; g < GS; ++g)
       if (g == h) L = Lh[g];
+    if (P.suf_part) {  // the dense suffix joins the same softmax (Appendix E.1 and E.2)
+      const int len = max(0, min(P.suf_len[u / P.n_kv_heads], P.suf_cap));
+      if (len > 0) {
+        // the compressed part's reference m (the unit's largest anchor score), the common maximum
+        // M over it and the chunks' maxima, and every part rescaled to M
+        const int nch = (unit_desc(P.arena, u)->n_anchors + CHA - 1) / CHA;
+        float m = -INFINITY;
+        for (int ch = lane; ch < nch; ch += 32) m = fmaxf(m, P.cmax[((size_t)u * P.n_ch + ch) * GS + h]);
+        m = warp_max(m);
+        const float* sp0 = P.suf_part + (size_t)u * P.n_sch * suf_floats(GS);
+        const int nsc = (len + SCH - 1) / SCH;
+        float M = m;
+        for (int c = lane; c < nsc; c += 32) M = fmaxf(M, sp0[(size_t)c * suf_floats(GS) + suf_m(GS) + h]);
+        M = warp_max(M);
+        const float f0 = exp2_approx(m - M);
+        a.x *= f0;
+        a.y *= f0;
+        a.z *= f0;
+        a.w *= f0;
+        L *= f0;
+        for (int c = 0; c < nsc; ++c) {
+          const float* sp = sp0 + (size_t)c * suf_floats(GS);
+          const float f = exp2_approx(sp[suf_m(GS) + h] - M);
+          const float4 o = *reinterpret_cast<const float4*>(sp + h * 128 + 4 * lane);
+          a.x = fmaf(f, o.x, a.x);
+          a.y = fmaf(f, o.y, a.y);
+          a.z = fmaf(f, o.z, a.z);
+          a.w = fmaf(f, o.w, a.w);
+          L = fmaf(f, sp[suf_l(GS) + h], L);
+        }
+      }
+    }
     const bool badh = bad || !(L < INFINITY);  // a logit so far above the reference that the sums overflowed
     const float yv[4] = {a.x, a.y, a.z, a.w};
     const size_t o = ob + (size_t)h * 128 + 4 * lane;
@@ -1635,7 +1789,7 @@ void set_decode_events(void* after_scores, void* after_decode) {
 }
 
 // Workspace of a decode call: anchor scores, chunk maxima, arrival counters, partial slots.
-DecodeWs decode_ws_layout(const Layout& L) {
+DecodeWs decode_ws_layout(const Layout& L, int32_t suffix_cap) {
   DecodeWs w;
   const size_t units = L.shape.size();
   const size_t ka = (size_t)((L.max_k + 3) & ~3);
@@ -1651,13 +1805,14 @@ DecodeWs decode_ws_layout(const Layout& L) {
   w.o_cmax = take(units * nch * (size_t)L.G * 4);
   w.o_cnt = take(units * 4);
   w.o_part = take((size_t)(kMaxGrid + units) * (size_t)part_floats(L.G) * 4);
+  w.o_suf = take(units * (size_t)((suffix_cap + SCH - 1) / SCH) * (size_t)suf_floats(L.G) * 4);
   w.total = off;
   return w;
 }
 
 template <int GS>
 int launch_g(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
-             float sm_scale, void* ws, void* stream, std::string* why) {
+             float sm_scale, const DecodeSuffix& sfx, void* ws, void* stream, std::string* why) {
   static std::mutex mu;
   static std::map<LaunchKey, Plan> cache;
   const int units = (int)L.shape.size();
@@ -1705,7 +1860,8 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
     std::lock_guard<std::mutex> lk(mu);
     cache[key] = pl;
   }
-  const DecodeWs W = decode_ws_layout(L);
+  const DecodeWs W = decode_ws_layout(L, sfx.cap);
+  const int n_sch = sfx.K ? (sfx.cap + SCH - 1) / SCH : 0;
   uint8_t* wsb = (uint8_t*)ws;
   DecodeParams& P = pl.P;
   P.arena = (const uint8_t*)arena;
@@ -1725,6 +1881,10 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   P.sign_lo = L.header.sign_bits[0];
   P.sign_hi = L.header.sign_bits[1];
   P.drop_last = drop;
+  P.suf_part = n_sch ? (const float*)(wsb + W.o_suf) : nullptr;
+  P.suf_len = sfx.len;
+  P.suf_cap = sfx.cap;
+  P.n_sch = n_sch;
 
   ScoreParams S;
   S.arena = P.arena;
@@ -1735,6 +1895,12 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   S.n_kv_heads = p.n_kv_heads;
   S.n_q_heads = p.n_q_heads;
   S.G = L.G;
+  S.ksuf = (const __nv_bfloat16*)sfx.K;
+  S.vsuf = (const __nv_bfloat16*)sfx.V;
+  S.suf_len = sfx.len;
+  S.suf_part = (float*)(wsb + W.o_suf);
+  S.suf_cap = sfx.cap;
+  S.n_sch = n_sch;
   S.ka_stride = P.ka_stride;
   S.n_ch = P.n_ch;
   S.scale_log2 = P.scale_log2;
@@ -1744,7 +1910,7 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   S.sign_lo = P.sign_lo;
   S.sign_hi = P.sign_hi;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(units * P.n_ch), 1, 1);
+  cfg.gridDim = dim3((unsigned)(units * (P.n_ch + n_sch)), 1, 1);
   cfg.blockDim = dim3(128, 1, 1);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = (cudaStream_t)stream;
@@ -1774,15 +1940,41 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
 }
 
 int launch_decode(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
-                  float sm_scale, void* ws, void* stream, std::string* why) {
+                  float sm_scale, const DecodeSuffix& sfx, void* ws, void* stream, std::string* why) {
   switch (L.G) {
-    case 1: return launch_g<1>(L, p, arena, q, out, out_f32, sm_scale, ws, stream, why);
-    case 2: return launch_g<2>(L, p, arena, q, out, out_f32, sm_scale, ws, stream, why);
-    case 4: return launch_g<4>(L, p, arena, q, out, out_f32, sm_scale, ws, stream, why);
-    case 8: return launch_g<8>(L, p, arena, q, out, out_f32, sm_scale, ws, stream, why);
+    case 1: return launch_g<1>(L, p, arena, q, out, out_f32, sm_scale, sfx, ws, stream, why);
+    case 2: return launch_g<2>(L, p, arena, q, out, out_f32, sm_scale, sfx, ws, stream, why);
+    case 4: return launch_g<4>(L, p, arena, q, out, out_f32, sm_scale, sfx, ws, stream, why);
+    case 8: return launch_g<8>(L, p, arena, q, out, out_f32, sm_scale, sfx, ws, stream, why);
   }
   *why = "unsupported group size";
   return -1;
+}
+
+// The append path of the dense suffix (Appendix E.2): CTA b copies the new key and value rows of
+// request b's KV heads to row len[b] of their suffix blocks, then counts the token in.  Every
+// thread reads len[b] before the barrier; thread 0 writes it after.
+__global__ void __launch_bounds__(256) akv_suffix_append_kernel(int H, const uint4* K_new, const uint4* V_new,
+                                                                 uint4* K_suf, uint4* V_suf, int32_t* len, int cap) {
+  const int b = blockIdx.x;
+  const int n = len[b];
+  const bool room = n >= 0 && n < cap;
+  if (room) {
+    for (int e = threadIdx.x; e < H * 16; e += blockDim.x) {  // 16 x 16 bytes per row
+      const size_t row = (size_t)b * H + e / 16;
+      K_suf[(row * cap + n) * 16 + e % 16] = K_new[row * 16 + e % 16];
+      V_suf[(row * cap + n) * 16 + e % 16] = V_new[row * 16 + e % 16];
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && room) len[b] = n + 1;
+}
+
+int launch_suffix_append(int32_t B, int32_t H, const void* K_new, const void* V_new, void* K_suf, void* V_suf,
+                         int32_t* len, int32_t cap, void* stream) {
+  akv_suffix_append_kernel<<<B, 256, 0, (cudaStream_t)stream>>>(H, (const uint4*)K_new, (const uint4*)V_new,
+                                                                (uint4*)K_suf, (uint4*)V_suf, len, cap);
+  return (int)cudaGetLastError();
 }
 
 const char* cuda_error_string(int err) { return cudaGetErrorString((cudaError_t)err); }

@@ -118,11 +118,25 @@ int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const
 // Decode workspace (device): anchor scores [units][ka][G] f32, query headers, chunk maxima,
 // arrival counters, partial slots; byte offsets from the workspace base (256-byte aligned).
 struct DecodeWs {
-  size_t o_sa = 0, o_uh = 0, o_cmax = 0, o_cnt = 0, o_part = 0, total = 0;
+  size_t o_sa = 0, o_uh = 0, o_cmax = 0, o_cnt = 0, o_part = 0, o_suf = 0, total = 0;
 };
-DecodeWs decode_ws_layout(const Layout& L);
+// The dense suffix of a decode call (akv_suffix): bf16 rows [B][H_kv][cap][128] and the tokens
+// held per request (device int32 [B]); null K = no suffix.
+struct DecodeSuffix {
+  const void* K = nullptr;
+  const void* V = nullptr;
+  const int32_t* len = nullptr;
+  int32_t cap = 0;
+};
+// Tokens per suffix chunk (one score-launch CTA each, one partial slot each).
+constexpr int kSuffixChunk = 64;
+// Workspace of a decode call whose suffix holds at most `suffix_cap` tokens per request.
+DecodeWs decode_ws_layout(const Layout& L, int32_t suffix_cap = 0);
 int launch_decode(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
-                  float sm_scale, void* ws, void* stream, std::string* why);
+                  float sm_scale, const DecodeSuffix& sfx, void* ws, void* stream, std::string* why);
+// Appends one token per request to the dense suffix (akv_suffix_append); returns a cudaError_t.
+int launch_suffix_append(int32_t B, int32_t H, const void* K_new, const void* V_new, void* K_suf, void* V_suf,
+                         int32_t* len, int32_t cap, void* stream);
 const char* cuda_error_string(int err);
 // Testing controls of the decode launch (akv_decode_set_debug), 0 = normal operation.
 extern std::atomic<int> g_debug_cluster, g_debug_withhold;

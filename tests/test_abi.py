@@ -198,6 +198,25 @@ def test_entry_points_validate_before_any_launch():
     assert st == akv.AKV_ERR_INVALID  # s_max < S
     st = L.akv_encode(ctypes.byref(p), lp, 256, 256, 128, 0x1000, nbytes, 0x2000, 16, None)
     assert st == akv.AKV_ERR_TOO_SMALL
+    # the dense suffix: pointers, capacity, and a workspace sized for the suffix's chunks
+    sp = ctypes.byref
+    S = akv._Suffix
+    wb = akv.akv_decode_workspace_size(akv.Params(batch=1, n_kv_heads=1, n_q_heads=1), lens)
+    ws_s = akv.akv_decode_workspace_size(akv.Params(batch=1, n_kv_heads=1, n_q_heads=1), lens, 1000)
+    assert ws_s > wb
+    for bad_sfx in (S(None, 0x5000, 0x6000, 10), S(0x4000, 0x5000, None, 10), S(0x4008, 0x5000, 0x6000, 10),
+                    S(0x4000, 0x5000, 0x6002, 10), S(0x4000, 0x5000, 0x6000, 0),
+                    S(0x4000, 0x5000, 0x6000, akv.AKV_MAX_SUFFIX + 1)):
+        st = L.akv_decode_attn_suffix(sp(p), lp, 0x1000, nbytes, 256, 256, None, 1.0, sp(bad_sfx), 0x3000, ws_s, None)
+        assert st == akv.AKV_ERR_INVALID, akv.akv_last_error()
+    st = L.akv_decode_attn_suffix(sp(p), lp, 0x1000, nbytes, 256, 256, None, 1.0, sp(S(0x4000, 0x5000, 0x6000, 1000)),
+                                  0x3000, ws_s - 1, None)
+    assert st == akv.AKV_ERR_TOO_SMALL
+    w = ctypes.c_size_t()
+    assert L.akv_decode_workspace_size_suffix(sp(p), lp, -1, sp(w)) == akv.AKV_ERR_INVALID
+    assert L.akv_suffix_append(sp(p), None, 0x2000, 0x3000, 0x4000, 0x5000, 8, None) == akv.AKV_ERR_INVALID
+    assert L.akv_suffix_append(sp(p), 0x1000, 0x2000, 0x3000, 0x4000, 0x5002, 8, None) == akv.AKV_ERR_INVALID
+    assert L.akv_suffix_append(sp(p), 0x1000, 0x2000, 0x3000, 0x4000, 0x5000, 0, None) == akv.AKV_ERR_INVALID
 
 
 def test_decode_debug_controls_validate():

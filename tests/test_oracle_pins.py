@@ -348,3 +348,79 @@ def test_zero_and_parallel_vectors():
     u = oracle.encode(K, V, [S], 1, 0.02, 0.1, 0.1, 32, 3, 11)[0]
     assert u.gam_k[10] == 0 and u.gam_v[11] == 0
     assert u.idx_k[12] == u.k - 1 and u.gam_k[12] == np.float16(-2.0).view(np.uint16)
+
+
+# ---- exact dense suffix (Appendix E.1, E.2): one softmax over prefix and suffix ----
+
+def _suffix_rows(n, seed, scale=1.0):
+    """bf16 bits [n][128] of clustered rows (a generated token's key or value)."""
+    K, V = gen.clustered_batch(1, 1, [max(n, 1)], seed=seed)
+    if scale != 1.0:
+        K = gen.bf16_bits(gen.bf16_to_f64(K) * scale)
+    return K[0, 0, :n], V[0, 0, :n]
+
+
+@pytest.mark.parametrize("n_suf", [1, 5, 70])
+@pytest.mark.parametrize("sm_scale", [1.0, 1 / math.sqrt(D)])
+def test_suffix_attend_matches_dense_bruteforce(tiny, n_suf, sm_scale):
+    """The compressed positions, rebuilt per Eq. 3, followed by the exact suffix rows, under one
+    softmax: equal to a dense softmax over the concatenated rows."""
+    _, _, u = tiny
+    ks, vs = _suffix_rows(n_suf, 900 + n_suf)
+    q = gen.queries(2, 77)
+    out = oracle.attend_suffix([u], q, 2, 1, sm_scale, PAR["rot_seed"], ks[None], vs[None], [n_suf])[0]
+    Kh = np.concatenate([oracle.reconstruct(u, "k", PAR["rot_seed"]), gen.bf16_to_f64(ks)])
+    Vh = np.concatenate([oracle.reconstruct(u, "v", PAR["rot_seed"]), gen.bf16_to_f64(vs)])
+    for g in range(2):
+        y, _ = _softmax_attend(Kh, Vh, gen.bf16_to_f64(q[g]), sm_scale)
+        assert np.allclose(out[g], y, rtol=0, atol=1e-12)
+
+
+def test_suffix_rows_past_the_length_are_ignored_and_empty_suffix_is_plain_attend(tiny):
+    _, _, u = tiny
+    ks, vs = _suffix_rows(40, 901)
+    q = gen.queries(4, 78)
+    plain = oracle.attend([u], q, 4, 1.0, PAR["rot_seed"])
+    empty = oracle.attend_suffix([u], q, 4, 1, 1.0, PAR["rot_seed"], ks[None], vs[None], [0])
+    assert np.array_equal(plain, empty)
+    short = oracle.attend_suffix([u], q, 4, 1, 1.0, PAR["rot_seed"], ks[None, :10], vs[None, :10], [10])
+    garbage = ks.copy()
+    garbage[10:] = 0x7F80  # +inf rows past the length must never be read
+    cut = oracle.attend_suffix([u], q, 4, 1, 1.0, PAR["rot_seed"], garbage[None], vs[None], [10])
+    assert np.array_equal(short, cut)
+
+
+def test_suffix_all_anchor_prefix_is_plain_softmax_over_the_input_rows():
+    """Every compressed position an anchor (S <= W): prefix and suffix are both exact, so the
+    result is textbook softmax attention over the input rows followed by the suffix rows; a suffix
+    whose logits dwarf the prefix's takes almost all the weight."""
+    S = 24
+    K, V = gen.clustered_batch(1, 1, [S], seed=5)
+    u = oracle.encode(K, V, [S], 1, 0.02, 0.1, 0.1, 32, 3, 11)[0]
+    for scale in (1.0, 8.0):
+        ks, vs = _suffix_rows(9, 902, scale)
+        q = gen.queries(1, 79)
+        out = oracle.attend_suffix([u], q, 1, 1, 1.0, 11, ks[None], vs[None], [9])[0, 0]
+        Kx = np.concatenate([gen.bf16_to_f64(K[0, 0]), gen.bf16_to_f64(ks)])
+        Vx = np.concatenate([gen.bf16_to_f64(V[0, 0]), gen.bf16_to_f64(vs)])
+        y, a = _softmax_attend(Kx, Vx, gen.bf16_to_f64(q[0]), 1.0)
+        assert np.allclose(out, y, rtol=0, atol=1e-13)
+    assert a[S:].sum() > 0.99  # the scaled suffix dominates
+
+
+def test_suffix_lengths_follow_requests_in_a_batch():
+    """Unit u = b*H + h takes request b's length: two requests, two KV heads, lengths 3 and 0."""
+    S, H = 300, 2
+    K, V = gen.clustered_batch(2, H, [S, S], seed=8)
+    units = oracle.encode(K, V, [S, S], H, 0.02, 0.1, 0.1, 32, 3, 11)
+    ks = np.zeros((4, 6, D), np.uint16)
+    vs = np.zeros((4, 6, D), np.uint16)
+    for u in range(4):
+        ks[u], vs[u] = _suffix_rows(6, 910 + u)
+    q = gen.queries(4 * 2, 80)
+    out = oracle.attend_suffix(units, q, 2, H, 1.0, 11, ks, vs, [3, 0])
+    plain = oracle.attend(units, q, 2, 1.0, 11)
+    for u in range(4):
+        ref = oracle.attend_suffix([units[u]], q.reshape(4, 2, D)[u], 2, 1, 1.0, 11, ks[u:u + 1, :3], vs[u:u + 1, :3],
+                                   [3]) if u < 2 else plain[u:u + 1]
+        assert np.array_equal(out[u:u + 1], ref)
