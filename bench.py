@@ -79,6 +79,8 @@ def parse():
     ap.add_argument("--workload", default="70b-128k", choices=sorted(WORKLOADS))
     ap.add_argument("--layers", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--codec", default="uniform", choices=["uniform", "lloyd"],
+                    help="residual codec: 4 uniform levels on [min, max], or the Lloyd-Max codebook (AKV_FLAG_LLOYD)")
     ap.add_argument("--suffix", type=int, default=0,
                     help="exact dense suffix: this many generated tokens per request, kept in bf16 and attended in "
                          "the same softmax (0 = none)")
@@ -354,7 +356,7 @@ def run_akv(args, rank, world, local):
     B, H, Hq, S, source = WORKLOADS[args.workload]
     lens = workload_lens(args.workload, B, S)
     p = workload_params(akv, args.workload, batch=B, n_kv_heads=H, n_q_heads=Hq, seed=rank_seed(11, rank),
-                        rot_seed=0x5EED)
+                        rot_seed=0x5EED, lloyd=args.codec == "lloyd")
     layers = args.layers
     arenas, arena_bytes, step_bytes = build_layers(torch, akv, gen, p, lens, layers, source, dev, rank)
     n_tok = N_TOKENS
@@ -522,7 +524,7 @@ def run_akv(args, rank, world, local):
         "config": {"workload": args.workload, "batch": B, "n_kv_heads": H, "n_q_heads": Hq,
                    "context": S if args.workload not in SWEEP_POINTS else f"ragged U[8192, 131072]: {lens}",
                    "anchor_frac": p.anchor_frac, "res_frac": p.res_frac_k, "layers_cycled": layers,
-                   "suffix_tokens": args.suffix,
+                   "suffix_tokens": args.suffix, "codec": args.codec,
                    "fresh_queries": N_TOKENS, "arena_bytes_per_layer": arena_bytes,
                    "l2": f"inputs larger than L2: {layers} distinct layer caches, {layers * arena_bytes / 1e6:.0f} MB cycled",
                    "timing": "CUDA graph replay, CUDA events on the launching stream", "parallelism": f"dp{world}"},

@@ -53,6 +53,14 @@ typedef enum akv_status {
 
 #define AKV_HEAD_DIM 128
 #define AKV_FLAG_ROTATE 1u /* residuals carry the randomized Hadamard rotation (Appendix A.1, Eq. 12) */
+/* Residual codec (Section 3.1, Appendix A.1 "Codebook"): without this flag, 4 uniform levels
+ * on [min, max] per token (c^ = min + code * scale, fp16 scale and min); with it, the
+ * four-level Lloyd-Max codebook of a unit Gaussian over a per-token RMS scale:
+ * scale = fp16(sqrt(sum_j v_j^2 / 128)) of the rotated residual v, min = 0, code = the
+ * decision region of v_j / scale (thresholds 0, +-0.98046875), c^ = scale * L[code] with
+ * L = {-1.5078125, -0.453125, 0.453125, 1.5078125} (Max's levels +-0.4528, +-1.5104 to 8
+ * significant bits, exact in bf16 and fp16).  Encode and decode must use the same flags. */
+#define AKV_FLAG_LLOYD 2u
 #define AKV_ARENA_MAGIC 0x32564B41u /* "AKV2" */
 #define AKV_ARENA_VERSION 3u
 #define AKV_MAX_ANCHORS 65535 /* anchor indices are uint16 (Table 1, b_a = 2) */

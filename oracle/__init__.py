@@ -78,6 +78,7 @@ def lib():
             L.or_attend_factorized.argtypes = [ctypes.POINTER(_OrUnit), vp, i32, dbl, u64, ctypes.c_int, vp]
             L.or_reconstruct_side.argtypes = [i32, vp, vp, vp, i32, vp, vp, vp, vp, u64, ctypes.c_int, vp]
             L.or_quantize_residual.argtypes = [vp, u64, ctypes.c_int, vp, vp, vp]
+            L.or_dequantize_residual.argtypes = [vp, ctypes.c_uint16, ctypes.c_uint16, u64, ctypes.c_int, vp]
             L.or_arena_shape.restype = ctypes.c_int
             L.or_arena_shape.argtypes = [vp, u64, i32, vp]
             L.or_exp_neg.restype = dbl
@@ -143,6 +144,11 @@ def alloc_unit(S: int, k: int, nk: int, nv: int) -> Unit:
 
 # ---- scalar helpers -------------------------------------------------------
 
+def _flags(rotate: bool, lloyd: bool) -> int:
+    """Codec flags of the C oracle: bit 0 the Hadamard rotation, bit 1 the Lloyd-Max codebook."""
+    return (1 if rotate else 0) | (2 if lloyd else 0)
+
+
 def splitmix64(x: int) -> int:
     return int(lib().or_splitmix64(ctypes.c_uint64(x & 0xFFFFFFFFFFFFFFFF)))
 
@@ -172,15 +178,39 @@ def wht128(v: np.ndarray) -> np.ndarray:
     return out
 
 
-def quantize_residual(r: np.ndarray, rot_seed: int, rotate: bool = True):
+def quantize_residual(r: np.ndarray, rot_seed: int, rotate: bool = True, lloyd: bool = False):
     """Rotate and quantize one residual; returns (codes[32] uint8, scale fp16 bits, min fp16 bits)."""
     r = np.ascontiguousarray(r, dtype=np.float64)
     assert r.shape == (D,)
     codes = np.zeros(32, np.uint8)
     sc = np.zeros(1, np.uint16)
     mn = np.zeros(1, np.uint16)
-    lib().or_quantize_residual(_p(r), ctypes.c_uint64(rot_seed), int(bool(rotate)), _p(codes), _p(sc), _p(mn))
+    lib().or_quantize_residual(_p(r), ctypes.c_uint64(rot_seed), _flags(rotate, lloyd), _p(codes), _p(sc), _p(mn))
     return codes, int(sc[0]), int(mn[0])
+
+
+def dequantize_residual(codes: np.ndarray, sc: int, mn: int, rot_seed: int, rotate: bool = True,
+                        lloyd: bool = False) -> np.ndarray:
+    """r~ = U^T C^-1(q) of one record (Eq. 14): fp64 [128]."""
+    codes = np.ascontiguousarray(codes, dtype=np.uint8)
+    out = np.zeros(D, np.float64)
+    lib().or_dequantize_residual(_p(codes), int(sc), int(mn), ctypes.c_uint64(rot_seed), _flags(rotate, lloyd),
+                                 _p(out))
+    return out
+
+
+def eta(residuals: np.ndarray, rot_seed: int, rotate: bool = True, lloyd: bool = False) -> float:
+    """Eq. 13: the relative squared distortion E||r - r~||^2 / ||r||^2 the codec leaves, as the mean
+    over the given residuals (fp64 [n][128], zero rows skipped) of ||r - r~||^2 / ||r||^2."""
+    vals = []
+    for r in np.asarray(residuals, np.float64):
+        nr = float(r @ r)
+        if nr == 0.0:
+            continue
+        codes, sc, mn = quantize_residual(r, rot_seed, rotate, lloyd)
+        e = r - dequantize_residual(codes, sc, mn, rot_seed, rotate, lloyd)
+        vals.append(float(e @ e) / nr)
+    return float(np.mean(vals))
 
 
 def unit_shape(S: int, f_a: float, f_rk: float, f_rv: float, W: int):
@@ -192,7 +222,7 @@ def unit_shape(S: int, f_a: float, f_rk: float, f_rv: float, W: int):
 # ---- encode / attend --------------------------------------------------------
 
 def encode(K: np.ndarray, V: np.ndarray, ctx_lens, n_kv_heads: int, f_a: float, f_rk: float, f_rv: float, W: int,
-           seed: int, rot_seed: int, rotate: bool = True) -> list:
+           seed: int, rot_seed: int, rotate: bool = True, lloyd: bool = False) -> list:
     """K, V: uint16 bf16 bits [B][H][s_max][128].  Returns B*H Units (u = b*H + h)."""
     K = np.ascontiguousarray(K, dtype=np.uint16)
     V = np.ascontiguousarray(V, dtype=np.uint16)
@@ -206,7 +236,7 @@ def encode(K: np.ndarray, V: np.ndarray, ctx_lens, n_kv_heads: int, f_a: float, 
             units.append(alloc_unit(S, *unit_shape(S, f_a, f_rk, f_rv, W)))
     structs = (_OrUnit * len(units))(*[u.c_struct() for u in units])
     rc = lib().or_encode_batch(_p(K), _p(V), s_max, len(units), H, W, ctypes.c_uint64(seed),
-                               ctypes.c_uint64(rot_seed), int(bool(rotate)), ctypes.cast(structs, ctypes.c_void_p))
+                               ctypes.c_uint64(rot_seed), _flags(rotate, lloyd), ctypes.cast(structs, ctypes.c_void_p))
     if rc != 0:
         raise RuntimeError("oracle encode failed")
     return units
@@ -249,7 +279,7 @@ def utilities(unit: "Unit", K: np.ndarray, V: np.ndarray, Q: np.ndarray):
 
 
 def encode_select(K: np.ndarray, V: np.ndarray, Q: np.ndarray, ctx_lens, n_kv_heads: int, f_a: float, W: int,
-                  theta: float, rho: float, kappa: int, seed: int, rot_seed: int, rotate: bool = True) -> list:
+                  theta: float, rho: float, kappa: int, seed: int, rot_seed: int, rotate: bool = True, lloyd: bool = False) -> list:
     """Algorithm 1 with the paper's selection.  K, V bf16 bits [B][H][s_max][128];
     Q bf16 bits [B][H][m][128], m = W G.  Returns B*H Units with per-unit residual counts."""
     K = np.ascontiguousarray(K, dtype=np.uint16)
@@ -269,7 +299,7 @@ def encode_select(K: np.ndarray, V: np.ndarray, Q: np.ndarray, ctx_lens, n_kv_he
             units.append(alloc_unit(S, k, cap_k, cap_v))
     structs = (_OrUnit * len(units))(*[u.c_struct() for u in units])
     rc = lib().or_encode_select_batch(_p(K), _p(V), _p(Q), s_max, B, H, m, W, theta, rho, kappa,
-                                      ctypes.c_uint64(seed), ctypes.c_uint64(rot_seed), int(bool(rotate)),
+                                      ctypes.c_uint64(seed), ctypes.c_uint64(rot_seed), _flags(rotate, lloyd),
                                       ctypes.cast(structs, ctypes.c_void_p))
     if rc != 0:
         raise RuntimeError("oracle select encode failed")
@@ -282,7 +312,7 @@ def encode_select(K: np.ndarray, V: np.ndarray, Q: np.ndarray, ctx_lens, n_kv_he
     return out
 
 
-def attend(units, q: np.ndarray, G: int, sm_scale: float, rot_seed: int, rotate: bool = True, sel=None) -> np.ndarray:
+def attend(units, q: np.ndarray, G: int, sm_scale: float, rot_seed: int, rotate: bool = True, lloyd: bool = False, sel=None) -> np.ndarray:
     """q: uint16 bf16 bits [n_units][G][128] (or [B][H_q][128]); returns fp64 of the same shape."""
     n = len(units)
     q = np.ascontiguousarray(q, dtype=np.uint16).reshape(n, G, D)
@@ -294,12 +324,12 @@ def attend(units, q: np.ndarray, G: int, sm_scale: float, rot_seed: int, rotate:
         assert sel_arr.shape == (n,)
         selp = _p(sel_arr)
     lib().or_attend_batch(ctypes.cast(structs, ctypes.c_void_p), n, _p(q), G, float(sm_scale),
-                          ctypes.c_uint64(rot_seed), int(bool(rotate)), selp, _p(out))
+                          ctypes.c_uint64(rot_seed), _flags(rotate, lloyd), selp, _p(out))
     return out
 
 
 def attend_suffix(units, q: np.ndarray, G: int, H: int, sm_scale: float, rot_seed: int, ksuf: np.ndarray,
-                  vsuf: np.ndarray, suf_len, rotate: bool = True) -> np.ndarray:
+                  vsuf: np.ndarray, suf_len, rotate: bool = True, lloyd: bool = False) -> np.ndarray:
     """Attention over each unit's compressed positions and the first suf_len[b] rows of its exact
     dense suffix, in one softmax (Appendix E.1, E.2).  ksuf, vsuf: uint16 bf16 bits
     [n_units][cap][128] (unit u = b*H + h); suf_len: int [B].  Returns fp64 [n_units][G][128]."""
@@ -313,21 +343,21 @@ def attend_suffix(units, q: np.ndarray, G: int, H: int, sm_scale: float, rot_see
     out = np.zeros((n, G, D), np.float64)
     structs = (_OrUnit * n)(*[u.c_struct() for u in units])
     lib().or_attend_batch_suffix(ctypes.cast(structs, ctypes.c_void_p), n, H, _p(q), G, float(sm_scale),
-                                 ctypes.c_uint64(rot_seed), int(bool(rotate)), _p(ksuf), _p(vsuf), _p(lens),
+                                 ctypes.c_uint64(rot_seed), _flags(rotate, lloyd), _p(ksuf), _p(vsuf), _p(lens),
                                  int(ksuf.shape[1]), _p(out))
     return out
 
 
-def attend_factorized(unit: Unit, q: np.ndarray, G: int, sm_scale: float, rot_seed: int, rotate: bool = True):
+def attend_factorized(unit: Unit, q: np.ndarray, G: int, sm_scale: float, rot_seed: int, rotate: bool = True, lloyd: bool = False):
     q = np.ascontiguousarray(q, dtype=np.uint16).reshape(G, D)
     out = np.zeros((G, D), np.float64)
     s = unit.c_struct()
     lib().or_attend_factorized(ctypes.byref(s), _p(q), G, float(sm_scale), ctypes.c_uint64(rot_seed),
-                               int(bool(rotate)), _p(out))
+                               _flags(rotate, lloyd), _p(out))
     return out
 
 
-def reconstruct(unit: Unit, side: str, rot_seed: int, rotate: bool = True) -> np.ndarray:
+def reconstruct(unit: Unit, side: str, rot_seed: int, rotate: bool = True, lloyd: bool = False) -> np.ndarray:
     """x^ of Eq. 3 for every position of one side ('k' or 'v'): fp64 [S][128]."""
     out = np.zeros((unit.S, D), np.float64)
     if side == "k":
@@ -336,7 +366,7 @@ def reconstruct(unit: Unit, side: str, rot_seed: int, rotate: bool = True) -> np
         arrs = (unit.anchor_v, unit.idx_v, unit.gam_v, unit.nv, unit.res_v, unit.codes_v, unit.scale_v, unit.min_v)
     anc, idx, gam, n, res, codes, sc, mn = arrs
     lib().or_reconstruct_side(unit.S, _p(anc), _p(idx), _p(gam), n, _p(res), _p(codes), _p(sc), _p(mn),
-                              ctypes.c_uint64(rot_seed), int(bool(rotate)), _p(out))
+                              ctypes.c_uint64(rot_seed), _flags(rotate, lloyd), _p(out))
     return out
 
 

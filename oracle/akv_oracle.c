@@ -12,7 +12,9 @@
  *             (projection coefficient, residual), Section 3.2 (last W
  *             positions are anchors, the rest sampled uniformly), Appendix
  *             A.1 Eq. 12 (randomized Hadamard rotation) and a 4-level
- *             2-bit quantizer with per-token fp16 scale and min; residual
+ *             2-bit quantizer: uniform with per-token fp16 scale and min, or
+ *             the Lloyd-Max codebook of Section 3.1 with a per-token RMS
+ *             scale; residual
  *             slots ranked by residual norm (Section 4.3, variant (ii)).
  *   encode_select : Algorithm 1 with the paper's full selection: the last W
  *             positions, a share rho of the other anchors by the selector
@@ -42,6 +44,22 @@
 #include <string.h>
 
 #define OR_D 128
+/* Codec flags (the library's AKV_FLAG_ROTATE and AKV_FLAG_LLOYD bits). */
+#define OR_ROTATE 1
+#define OR_LLOYD 2
+
+/* The four-level Lloyd-Max quantizer of a unit Gaussian source (Max 1960, the
+ * codebook of Section 3.1 and Appendix A.1): levels -1.5104, -0.4528, 0.4528,
+ * 1.5104, decision thresholds at their midpoints.  The levels are taken to 8
+ * significant bits (+-0.453125, +-1.5078125: exact in bf16 and fp16, so the
+ * decoder's tensor-core operands carry them unrounded) and the thresholds are
+ * the midpoints of those levels (0, +-0.98046875). */
+static const double OR_LM_LEVEL[4] = {-1.5078125, -0.453125, 0.453125, 1.5078125};
+#define OR_LM_T 0.98046875
+
+/* Reconstruction value of a 2-bit code: the code itself (uniform codec) or its
+ * Lloyd-Max level. */
+static double or_level(int flags, int c) { return (flags & OR_LLOYD) ? OR_LM_LEVEL[c] : (double)c; }
 
 /* ------------------------------------------------------------------------ */
 /* Scalar helpers                                                            */
@@ -199,13 +217,39 @@ static int cmp_i32(const void* a, const void* b) {
   return (x > y) - (x < y);
 }
 
-/* Quantize one residual (Appendix A.1 rotation, then 4-level uniform codes
- * on [min, max] with fp16 scale and min) and pack 4 codes per byte. */
-static void or_quantize(const double* r, const double* s, int rotate, uint8_t* codes, uint16_t* sc_out,
+/* Quantize one residual and pack 4 codes per byte (code j in byte j/4, bits
+ * 2(j%4)..+1).  Appendix A.1 rotation first (v = H(s o r), when flags has
+ * OR_ROTATE), then one of two codecs:
+ *   uniform  : 4-level uniform codes on [min, max] with fp16 scale and min,
+ *              c^_j = min + code_j scale;
+ *   Lloyd-Max: (OR_LLOYD) each coordinate divided by the per-token RMS scale
+ *              sigma = sqrt(sum_j v_j^2 / 128) (the rotated coordinates are
+ *              about N(0, sigma^2), Appendix A.1; the sum taken in index
+ *              order), fp16 scale, min 0, code = the Lloyd-Max decision region
+ *              of v_j / scale, c^_j = scale L[code]. */
+static void or_quantize(const double* r, const double* s, int flags, uint8_t* codes, uint16_t* sc_out,
                         uint16_t* mn_out) {
   double v[OR_D];
-  for (int j = 0; j < OR_D; ++j) v[j] = rotate ? s[j] * r[j] : r[j];
-  if (rotate) or_wht128(v);
+  for (int j = 0; j < OR_D; ++j) v[j] = (flags & OR_ROTATE) ? s[j] * r[j] : r[j];
+  if (flags & OR_ROTATE) or_wht128(v);
+  memset(codes, 0, 32);
+  if (flags & OR_LLOYD) {
+    double ss = 0.0;
+    for (int j = 0; j < OR_D; ++j) ss += v[j] * v[j];
+    uint16_t sc_h = or_fp16_from_double(sqrt(ss / (double)OR_D));
+    double sc = or_fp16_to_double(sc_h);
+    for (int j = 0; j < OR_D; ++j) {
+      int c = 2; /* a zero scale: every level reconstructs 0 */
+      if (sc != 0.0) {
+        double t = v[j] / sc;
+        c = t < -OR_LM_T ? 0 : (t < 0.0 ? 1 : (t < OR_LM_T ? 2 : 3));
+      }
+      codes[j / 4] |= (uint8_t)(c << (2 * (j % 4)));
+    }
+    *sc_out = sc_h;
+    *mn_out = 0;
+    return;
+  }
   double vmin = v[0], vmax = v[0];
   for (int j = 1; j < OR_D; ++j) {
     if (v[j] < vmin) vmin = v[j];
@@ -217,7 +261,6 @@ static void or_quantize(const double* r, const double* s, int rotate, uint8_t* c
   if (!(t > 0.0)) t = 0.0;
   uint16_t sc_h = or_fp16_from_double(t);
   double sc = or_fp16_to_double(sc_h);
-  memset(codes, 0, 32);
   for (int j = 0; j < OR_D; ++j) {
     int c = 0;
     if (sc != 0.0) {
@@ -233,16 +276,16 @@ static void or_quantize(const double* r, const double* s, int rotate, uint8_t* c
 }
 
 /* Exported for the quantizer pins: rotate (if set) and quantize one residual r[128]. */
-void or_quantize_residual(const double* r, uint64_t rot_seed, int rotate, uint8_t* codes, uint16_t* sc,
+void or_quantize_residual(const double* r, uint64_t rot_seed, int flags, uint8_t* codes, uint16_t* sc,
                           uint16_t* mn) {
   double s[OR_D];
   or_signs(rot_seed, s);
-  or_quantize(r, s, rotate, codes, sc, mn);
+  or_quantize(r, s, flags, codes, sc, mn);
 }
 
 /* Encode one side (keys or values) of one unit given the anchor set. */
 static void or_encode_side(int32_t S, int32_t k, int32_t nres, const uint16_t* X /*[S][128]*/,
-                           const int32_t* anchor_pos, const int32_t* slot_of, const double* s, int rotate,
+                           const int32_t* anchor_pos, const int32_t* slot_of, const double* s, int flags,
                            uint16_t* idx, uint16_t* gam, int32_t* res, uint8_t* codes, uint16_t* scale,
                            uint16_t* mins) {
   /* anchor rows as doubles (exact) and their squared norms */
@@ -317,7 +360,7 @@ static void or_encode_side(int32_t S, int32_t k, int32_t nres, const uint16_t* X
       double p = valid ? g * or_bf16_to_double(xa[j]) : 0.0;
       r[j] = or_bf16_to_double(x[j]) - p;
     }
-    or_quantize(r, s, rotate, codes + (size_t)t * 32, &scale[t], &mins[t]);
+    or_quantize(r, s, flags, codes + (size_t)t * 32, &scale[t], &mins[t]);
   }
   free(cand);
   free(xad);
@@ -330,7 +373,7 @@ static void or_encode_side(int32_t S, int32_t k, int32_t nres, const uint16_t* X
  * and sets u->S, k, nk, nv.
  */
 int or_encode_unit(const uint16_t* K, const uint16_t* V, int32_t b, int32_t h, int32_t W, uint64_t seed,
-                   uint64_t rot_seed, int rotate, or_unit* u) {
+                   uint64_t rot_seed, int flags, or_unit* u) {
   int32_t S = u->S, k = u->k;
   int32_t w = W < S ? W : S;
   /* Section 3.2: the last w positions are anchors; the k - w others are a
@@ -372,9 +415,9 @@ int or_encode_unit(const uint16_t* K, const uint16_t* V, int32_t b, int32_t h, i
   }
   double s[OR_D];
   or_signs(rot_seed, s);
-  or_encode_side(S, k, u->nk, K, u->anchor_pos, slot_of, s, rotate, u->idx_k, u->gam_k, u->res_k, u->codes_k,
+  or_encode_side(S, k, u->nk, K, u->anchor_pos, slot_of, s, flags, u->idx_k, u->gam_k, u->res_k, u->codes_k,
                  u->scale_k, u->min_k);
-  or_encode_side(S, k, u->nv, V, u->anchor_pos, slot_of, s, rotate, u->idx_v, u->gam_v, u->res_v, u->codes_v,
+  or_encode_side(S, k, u->nv, V, u->anchor_pos, slot_of, s, flags, u->idx_v, u->gam_v, u->res_v, u->codes_v,
                  u->scale_v, u->min_v);
   free(slot_of);
   free(is_anchor);
@@ -383,12 +426,12 @@ int or_encode_unit(const uint16_t* K, const uint16_t* V, int32_t b, int32_t h, i
 
 /* Batched encode: K, V are [n_units][s_max][128]; units[u] describe b = u / H, h = u % H. */
 int or_encode_batch(const uint16_t* K, const uint16_t* V, int32_t s_max, int32_t n_units, int32_t H, int32_t W,
-                    uint64_t seed, uint64_t rot_seed, int rotate, or_unit* units) {
+                    uint64_t seed, uint64_t rot_seed, int flags, or_unit* units) {
   int bad = 0;
 #pragma omp parallel for schedule(dynamic, 1) reduction(| : bad)
   for (int32_t u = 0; u < n_units; ++u) {
     size_t off = (size_t)u * (size_t)s_max * OR_D;
-    if (or_encode_unit(K + off, V + off, u / H, u % H, W, seed, rot_seed, rotate, &units[u]) != 0) bad |= 1;
+    if (or_encode_unit(K + off, V + off, u / H, u % H, W, seed, rot_seed, flags, &units[u]) != 0) bad |= 1;
   }
   return bad ? -1 : 0;
 }
@@ -398,25 +441,33 @@ int or_encode_batch(const uint16_t* K, const uint16_t* V, int32_t s_max, int32_t
 /* ------------------------------------------------------------------------ */
 
 /* r~ = U^T C^{-1}(q) of Eq. 14 with U = H diag(s) / sqrt(D): here the stored
- * codes dequantize to c^ = min + code * scale in the sqrt(D)-scaled rotated
- * domain, so r~ = s o (H c^) / D. */
-static void or_dequant_residual(const uint8_t* codes, uint16_t sc_h, uint16_t mn_h, const double* s, int rotate,
+ * codes dequantize to c^ = min + L(code) * scale in the sqrt(D)-scaled rotated
+ * domain (L(code) = code, or the Lloyd-Max level), so r~ = s o (H c^) / D. */
+static void or_dequant_residual(const uint8_t* codes, uint16_t sc_h, uint16_t mn_h, const double* s, int flags,
                                 double* out) {
   double sc = or_fp16_to_double(sc_h), mn = or_fp16_to_double(mn_h);
   for (int j = 0; j < OR_D; ++j) {
     int c = (codes[j / 4] >> (2 * (j % 4))) & 3;
-    out[j] = mn + (double)c * sc;
+    out[j] = mn + or_level(flags, c) * sc;
   }
-  if (rotate) {
+  if (flags & OR_ROTATE) {
     or_wht128(out);
     for (int j = 0; j < OR_D; ++j) out[j] = s[j] * out[j] / (double)OR_D;
   }
 }
 
+/* Exported for the codec pins: r~ of one record (codes [32], fp16 scale and min). */
+void or_dequantize_residual(const uint8_t* codes, uint16_t sc_h, uint16_t mn_h, uint64_t rot_seed, int flags,
+                            double* out) {
+  double s[OR_D];
+  or_signs(rot_seed, s);
+  or_dequant_residual(codes, sc_h, mn_h, s, flags, out);
+}
+
 /* x^_i of Eq. 3 for one side, for every position; out [S][128]. */
 void or_reconstruct_side(int32_t S, const uint16_t* anchors, const uint16_t* idx, const uint16_t* gam, int32_t nres,
                          const int32_t* res, const uint8_t* codes, const uint16_t* scale, const uint16_t* mins,
-                         uint64_t rot_seed, int rotate, double* out) {
+                         uint64_t rot_seed, int flags, double* out) {
   double s[OR_D], rt[OR_D];
   or_signs(rot_seed, s);
   for (int32_t i = 0; i < S; ++i) {
@@ -425,7 +476,7 @@ void or_reconstruct_side(int32_t S, const uint16_t* anchors, const uint16_t* idx
     for (int j = 0; j < OR_D; ++j) out[(size_t)i * OR_D + j] = g * or_bf16_to_double(xa[j]);
   }
   for (int32_t t = 0; t < nres; ++t) {
-    or_dequant_residual(codes + (size_t)t * 32, scale[t], mins[t], s, rotate, rt);
+    or_dequant_residual(codes + (size_t)t * 32, scale[t], mins[t], s, flags, rt);
     for (int j = 0; j < OR_D; ++j) out[(size_t)res[t] * OR_D + j] += rt[j];
   }
 }
@@ -437,7 +488,7 @@ void or_reconstruct_side(int32_t S, const uint16_t* anchors, const uint16_t* idx
  * softmax of Eq. 4 is taken over all S + nsuf positions at once (the combine
  * of Appendix E.1 attends both under the same softmax). */
 void or_attend_unit_suffix(const or_unit* u, const uint16_t* q, int32_t G, double sm_scale, uint64_t rot_seed,
-                           int rotate, const uint16_t* ksuf, const uint16_t* vsuf, int32_t nsuf, double* out) {
+                           int flags, const uint16_t* ksuf, const uint16_t* vsuf, int32_t nsuf, double* out) {
   int32_t S = u->S;
   int32_t n = S + nsuf; /* positions of the softmax */
   double s[OR_D];
@@ -458,7 +509,7 @@ void or_attend_unit_suffix(const or_unit* u, const uint16_t* q, int32_t G, doubl
       for (int j = 0; j < OR_D; ++j) x[j] = gk * or_bf16_to_double(xa[j]);
       if (slot_k[i] >= 0) {
         int32_t t = slot_k[i];
-        or_dequant_residual(u->codes_k + (size_t)t * 32, u->scale_k[t], u->min_k[t], s, rotate, rt);
+        or_dequant_residual(u->codes_k + (size_t)t * 32, u->scale_k[t], u->min_k[t], s, flags, rt);
         for (int j = 0; j < OR_D; ++j) x[j] += rt[j];
       }
     } else {
@@ -491,7 +542,7 @@ void or_attend_unit_suffix(const or_unit* u, const uint16_t* q, int32_t G, doubl
       for (int j = 0; j < OR_D; ++j) x[j] = gv * or_bf16_to_double(xa[j]);
       if (slot_v[i] >= 0) {
         int32_t t = slot_v[i];
-        or_dequant_residual(u->codes_v + (size_t)t * 32, u->scale_v[t], u->min_v[t], s, rotate, rt);
+        or_dequant_residual(u->codes_v + (size_t)t * 32, u->scale_v[t], u->min_v[t], s, flags, rt);
         for (int j = 0; j < OR_D; ++j) x[j] += rt[j];
       }
     } else {
@@ -509,9 +560,9 @@ void or_attend_unit_suffix(const or_unit* u, const uint16_t* q, int32_t G, doubl
 
 /* Definitional attention for one unit (no suffix): the softmax of Eq. 4 over
  * its S positions, each key and value rebuilt per Eq. 3. */
-void or_attend_unit(const or_unit* u, const uint16_t* q, int32_t G, double sm_scale, uint64_t rot_seed, int rotate,
+void or_attend_unit(const or_unit* u, const uint16_t* q, int32_t G, double sm_scale, uint64_t rot_seed, int flags,
                     double* out) {
-  or_attend_unit_suffix(u, q, G, sm_scale, rot_seed, rotate, NULL, NULL, 0, out);
+  or_attend_unit_suffix(u, q, G, sm_scale, rot_seed, flags, NULL, NULL, 0, out);
 }
 
 /* ------------------------------------------------------------------------ */
@@ -633,7 +684,7 @@ int64_t or_budget_n(double theta, int32_t S, int32_t H, int32_t W, int32_t k) {
  * set.  cand[side] receive one entry per non-anchor position (*ncand of them).
  */
 static int or_select_head(const uint16_t* Kh, const uint16_t* Vh, const uint16_t* Qh, int32_t m, int32_t W, float rho,
-                          int32_t kappa, int32_t b, int32_t h, uint64_t seed, const double* sv, int rotate, or_unit* u,
+                          int32_t kappa, int32_t b, int32_t h, uint64_t seed, const double* sv, int flags, or_unit* u,
                           or_util* cand_k, or_util* cand_v, int64_t* ncand) {
   int32_t S = u->S, k = u->k;
   int32_t w = W < S ? W : S;
@@ -696,8 +747,8 @@ static int or_select_head(const uint16_t* Kh, const uint16_t* Vh, const uint16_t
     memcpy(u->anchor_v + (size_t)a * OR_D, Vh + (size_t)u->anchor_pos[a] * OR_D, OR_D * 2);
   }
   /* assignment and coefficients (Eq. 1, Eq. 2), no residual slots yet */
-  or_encode_side(S, k, 0, Kh, u->anchor_pos, slot_of, sv, rotate, u->idx_k, u->gam_k, NULL, NULL, NULL, NULL);
-  or_encode_side(S, k, 0, Vh, u->anchor_pos, slot_of, sv, rotate, u->idx_v, u->gam_v, NULL, NULL, NULL, NULL);
+  or_encode_side(S, k, 0, Kh, u->anchor_pos, slot_of, sv, flags, u->idx_k, u->gam_k, NULL, NULL, NULL, NULL);
+  or_encode_side(S, k, 0, Vh, u->anchor_pos, slot_of, sv, flags, u->idx_v, u->gam_v, NULL, NULL, NULL, NULL);
   /* exact outputs y^(w) of the observation rows (Eq. 4) */
   for (int32_t ww = 0; ww < m; ++ww)
     for (int j = 0; j < OR_D; ++j) {
@@ -759,7 +810,7 @@ static int or_select_head(const uint16_t* Kh, const uint16_t* Vh, const uint16_t
  * rest, each side's top N pooled over the request's H heads (the candidates of
  * head h at cand + h S), then rotation and quantization of the chosen residuals. */
 static void or_pool_request(const uint16_t* K, const uint16_t* V, int32_t s_max, int32_t H, int32_t W, float theta,
-                            const double* sv, int rotate, or_unit* units, or_util* cand[2], const int64_t* ncand) {
+                            const double* sv, int flags, or_unit* units, or_util* cand[2], const int64_t* ncand) {
   int32_t S = units[0].S, k = units[0].k;
   int64_t N = or_budget_n((double)theta, S, H, W, k);
   int64_t nside[2] = {N / 2, N - N / 2};
@@ -802,8 +853,8 @@ static void or_pool_request(const uint16_t* K, const uint16_t* V, int32_t s_max,
         double g = or_fp16_to_double(gam[p]);
         for (int j = 0; j < OR_D; ++j)
           r[j] = or_bf16_to_double(X[(size_t)p * OR_D + j]) - g * or_bf16_to_double(A[(size_t)idx[p] * OR_D + j]);
-        if (side == 0) or_quantize(r, sv, rotate, u->codes_k + (size_t)i * 32, &u->scale_k[i], &u->min_k[i]);
-        else or_quantize(r, sv, rotate, u->codes_v + (size_t)i * 32, &u->scale_v[i], &u->min_v[i]);
+        if (side == 0) or_quantize(r, sv, flags, u->codes_k + (size_t)i * 32, &u->scale_k[i], &u->min_k[i]);
+        else or_quantize(r, sv, flags, u->codes_v + (size_t)i * 32, &u->scale_v[i], &u->min_v[i]);
       }
     }
   }
@@ -863,7 +914,7 @@ void or_utilities_unit(const or_unit* u, const uint16_t* K, const uint16_t* V, c
  * run in parallel, then each request's pooling. */
 int or_encode_select_batch(const uint16_t* K, const uint16_t* V, const uint16_t* Q, int32_t s_max, int32_t B, int32_t H,
                            int32_t m, int32_t W, float theta, float rho, int32_t kappa, uint64_t seed,
-                           uint64_t rot_seed, int rotate, or_unit* units) {
+                           uint64_t rot_seed, int flags, or_unit* units) {
   double sv[OR_D];
   or_signs(rot_seed, sv);
   int32_t n = B * H;
@@ -881,7 +932,7 @@ int or_encode_select_batch(const uint16_t* K, const uint16_t* V, const uint16_t*
     int32_t b = u / H, h = u % H;
     size_t off = (size_t)u * (size_t)s_max * OR_D;
     size_t S = (size_t)units[u].S;
-    if (or_select_head(K + off, V + off, Q + (size_t)u * (size_t)m * OR_D, m, W, rho, kappa, b, h, seed, sv, rotate,
+    if (or_select_head(K + off, V + off, Q + (size_t)u * (size_t)m * OR_D, m, W, rho, kappa, b, h, seed, sv, flags,
                        &units[u], ck[b] + (size_t)h * S, cv[b] + (size_t)h * S, &ncand[u]) != 0)
       bad |= 1;
   }
@@ -890,7 +941,7 @@ int or_encode_select_batch(const uint16_t* K, const uint16_t* V, const uint16_t*
     for (int32_t b = 0; b < B; ++b) {
       size_t off = (size_t)b * H * (size_t)s_max * OR_D;
       or_util* cand[2] = {ck[b], cv[b]};
-      or_pool_request(K + off, V + off, s_max, H, W, theta, sv, rotate, units + (size_t)b * H, cand,
+      or_pool_request(K + off, V + off, s_max, H, W, theta, sv, flags, units + (size_t)b * H, cand,
                       ncand + (size_t)b * H);
     }
   }
@@ -908,11 +959,11 @@ int or_encode_select_batch(const uint16_t* K, const uint16_t* V, const uint16_t*
  * owns query heads h*G .. h*G+G-1 of request b), out fp64 same shape.
  * Units with sel[u] == 0 are skipped (sel may be NULL). */
 void or_attend_batch(const or_unit* units, int32_t n_units, const uint16_t* q, int32_t G, double sm_scale,
-                     uint64_t rot_seed, int rotate, const uint8_t* sel, double* out) {
+                     uint64_t rot_seed, int flags, const uint8_t* sel, double* out) {
 #pragma omp parallel for schedule(dynamic, 1)
   for (int32_t u = 0; u < n_units; ++u) {
     if (sel && !sel[u]) continue;
-    or_attend_unit(&units[u], q + (size_t)u * G * OR_D, G, sm_scale, rot_seed, rotate, out + (size_t)u * G * OR_D);
+    or_attend_unit(&units[u], q + (size_t)u * G * OR_D, G, sm_scale, rot_seed, flags, out + (size_t)u * G * OR_D);
   }
 }
 
@@ -920,12 +971,12 @@ void or_attend_batch(const or_unit* units, int32_t n_units, const uint16_t* q, i
  * S positions and the first suf_len[b] rows of its suffix block, rows
  * ksuf/vsuf + (u * suf_cap + t) * 128 (bf16). */
 void or_attend_batch_suffix(const or_unit* units, int32_t n_units, int32_t H, const uint16_t* q, int32_t G,
-                            double sm_scale, uint64_t rot_seed, int rotate, const uint16_t* ksuf, const uint16_t* vsuf,
+                            double sm_scale, uint64_t rot_seed, int flags, const uint16_t* ksuf, const uint16_t* vsuf,
                             const int32_t* suf_len, int32_t suf_cap, double* out) {
 #pragma omp parallel for schedule(dynamic, 1)
   for (int32_t u = 0; u < n_units; ++u) {
     const size_t base = (size_t)u * (size_t)suf_cap * OR_D;
-    or_attend_unit_suffix(&units[u], q + (size_t)u * G * OR_D, G, sm_scale, rot_seed, rotate, ksuf + base, vsuf + base,
+    or_attend_unit_suffix(&units[u], q + (size_t)u * G * OR_D, G, sm_scale, rot_seed, flags, ksuf + base, vsuf + base,
                           suf_len[u / H], out + (size_t)u * G * OR_D);
   }
 }
@@ -934,15 +985,15 @@ void or_attend_batch_suffix(const or_unit* units, int32_t n_units, int32_t H, co
  * value weights summed per anchor before one product with the anchor values,
  * and the inverse rotation applied once to the accumulated residual codes. */
 void or_attend_factorized(const or_unit* u, const uint16_t* q, int32_t G, double sm_scale, uint64_t rot_seed,
-                          int rotate, double* out) {
+                          int flags, double* out) {
   int32_t S = u->S, k = u->k;
   double s[OR_D];
   or_signs(rot_seed, s);
   double qd[8][OR_D], qr[8][OR_D], qsum[8];
   for (int32_t g = 0; g < G; ++g) {
     for (int j = 0; j < OR_D; ++j) qd[g][j] = or_bf16_to_double(q[(size_t)g * OR_D + j]);
-    for (int j = 0; j < OR_D; ++j) qr[g][j] = rotate ? s[j] * qd[g][j] : qd[g][j];
-    if (rotate) {
+    for (int j = 0; j < OR_D; ++j) qr[g][j] = (flags & OR_ROTATE) ? s[j] * qd[g][j] : qd[g][j];
+    if (flags & OR_ROTATE) {
       or_wht128(qr[g]);
       for (int j = 0; j < OR_D; ++j) qr[g][j] /= (double)OR_D;
     }
@@ -965,7 +1016,8 @@ void or_attend_factorized(const or_unit* u, const uint16_t* q, int32_t G, double
     double sc = or_fp16_to_double(u->scale_k[t]), mn = or_fp16_to_double(u->min_k[t]);
     for (int32_t g = 0; g < G; ++g) {
       double d = 0.0;
-      for (int j = 0; j < OR_D; ++j) d += qr[g][j] * (double)((u->codes_k[(size_t)t * 32 + j / 4] >> (2 * (j % 4))) & 3);
+      for (int j = 0; j < OR_D; ++j)
+        d += qr[g][j] * or_level(flags, (u->codes_k[(size_t)t * 32 + j / 4] >> (2 * (j % 4))) & 3);
       lg[(size_t)i * G + g] += mn * qsum[g] + sc * d;
     }
   }
@@ -994,11 +1046,11 @@ void or_attend_factorized(const or_unit* u, const uint16_t* q, int32_t G, double
     for (int32_t g = 0; g < G; ++g) {
       double p = lg[(size_t)i * G + g];
       for (int j = 0; j < OR_D; ++j)
-        acc[g][j] += p * (mn + sc * (double)((u->codes_v[(size_t)t * 32 + j / 4] >> (2 * (j % 4))) & 3));
+        acc[g][j] += p * (mn + sc * or_level(flags, (u->codes_v[(size_t)t * 32 + j / 4] >> (2 * (j % 4))) & 3));
     }
   }
   for (int32_t g = 0; g < G; ++g) {
-    if (rotate) {
+    if (flags & OR_ROTATE) {
       or_wht128(acc[g]);
       for (int j = 0; j < OR_D; ++j) acc[g][j] = s[j] * acc[g][j] / (double)OR_D;
     }

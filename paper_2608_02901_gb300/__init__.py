@@ -19,6 +19,7 @@ LIB_PATH = os.path.join(_HERE, "libakv.so")
 
 AKV_OK, AKV_ERR_INVALID, AKV_ERR_UNSUPPORTED, AKV_ERR_TOO_SMALL, AKV_ERR_CUDA = range(5)
 AKV_FLAG_ROTATE = 1
+AKV_FLAG_LLOYD = 2
 HEAD_DIM = 128
 
 EXPORTED = (
@@ -84,6 +85,7 @@ class Params:
     rot_seed: int = 0x5EED
     rotate: bool = True
     head_dim: int = HEAD_DIM
+    lloyd: bool = False  # the Lloyd-Max residual codec (AKV_FLAG_LLOYD) instead of the uniform one
 
     @property
     def G(self) -> int:
@@ -96,7 +98,8 @@ class Params:
     def c(self) -> _Params:
         return _Params(self.batch, self.n_kv_heads, self.n_q_heads, self.head_dim, self.anchor_frac,
                        self.res_frac_k, self.res_frac_v, self.window, self.seed & (2**64 - 1),
-                       self.rot_seed & (2**64 - 1), AKV_FLAG_ROTATE if self.rotate else 0, 0)
+                       self.rot_seed & (2**64 - 1),
+                       (AKV_FLAG_ROTATE if self.rotate else 0) | (AKV_FLAG_LLOYD if self.lloyd else 0), 0)
 
 
 _lib = None
@@ -302,7 +305,7 @@ _DECODE_ARGS: dict = {}
 
 def _decode_args(p: Params, ctx_lens):
     key = (p.batch, p.n_kv_heads, p.n_q_heads, p.head_dim, p.anchor_frac, p.res_frac_k, p.res_frac_v, p.window,
-           p.seed, p.rot_seed, p.rotate, tuple(int(x) for x in ctx_lens))
+           p.seed, p.rot_seed, p.rotate, p.lloyd, tuple(int(x) for x in ctx_lens))
     ent = _DECODE_ARGS.get(key)
     if ent is None:
         if len(_DECODE_ARGS) >= 64:

@@ -50,7 +50,7 @@ akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out
   if (!frac_ok(p->anchor_frac) || !frac_ok(p->res_frac_k) || !frac_ok(p->res_frac_v))
     return fail(AKV_ERR_INVALID, "fractions must be finite and in [0, 1]");
   if (p->window < 0) return fail(AKV_ERR_INVALID, "window must be >= 0");
-  if (p->reserved != 0 || (p->flags & ~AKV_FLAG_ROTATE) != 0) return fail(AKV_ERR_INVALID, "unknown flags");
+  if (p->reserved != 0 || (p->flags & ~(AKV_FLAG_ROTATE | AKV_FLAG_LLOYD)) != 0) return fail(AKV_ERR_INVALID, "unknown flags");
   if (sel) {
     if (!(std::isfinite(sel->theta) && sel->theta > 0.0f && sel->theta <= 1.0f))
       return fail(AKV_ERR_INVALID, "theta must be in (0, 1]");

@@ -258,6 +258,38 @@ __device__ __forceinline__ uint32_t codes2_to_b2(uint32_t x) {
   asm("fma.rn.bf16x2 %0, %1, %2, %3;" : "=r"(r) : "r"(t), "r"(0x3F803F80u), "r"(0xC300C300u));
   return r;
 }
+// The Lloyd-Max codec (AKV_FLAG_LLOYD): a code c stands for level L[c] of
+// {-1.5078125, -0.453125, 0.453125, 1.5078125}.  Two codes (bits 0-1 and 16-17 of x) become a
+// 16-bit pair by a byte permutation out of the four-entry table held in two registers: the
+// selector nibbles 2c, 2c + 1 of both codes come from one integer multiply-add and one gather.
+__device__ __forceinline__ uint32_t lm_selector(uint32_t x) {
+  const uint32_t u = (x & 0x00030003u) * 0x22u + 0x00100010u;  // bytes 0 and 2: nibbles 2c, 2c + 1
+  uint32_t sel;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(sel) : "r"(u), "r"(0u), "r"(0x00000020u));
+  return sel;
+}
+__device__ __forceinline__ uint32_t lm_pair(uint32_t x, uint32_t tab_lo, uint32_t tab_hi) {
+  uint32_t r;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(tab_lo), "r"(tab_hi), "r"(lm_selector(x)));
+  return r;
+}
+// Code pair as the fp16 (key-residual A operand) or bf16 (value-residual B operand) pair of the
+// codec's reconstruction values: the codes themselves, or their Lloyd-Max levels (exact in both).
+template <int CODEC>
+__device__ __forceinline__ uint32_t code_pair_h2(uint32_t x) {
+  if constexpr (CODEC == 0) return codes2_to_h2(x);
+  else return lm_pair(x, 0xB740BE08u, 0x3E083740u);
+}
+template <int CODEC>
+__device__ __forceinline__ uint32_t code_pair_b2(uint32_t x) {
+  if constexpr (CODEC == 0) return codes2_to_b2(x);
+  else return lm_pair(x, 0xBEE8BFC1u, 0x3FC13EE8u);
+}
+// One code's reconstruction value on CUDA cores (the rare paths).
+__device__ __forceinline__ float code_level(uint32_t c, int lloyd) {
+  if (!lloyd) return (float)c;
+  return c == 0u ? -1.5078125f : (c == 1u ? -0.453125f : (c == 2u ? 0.453125f : 1.5078125f));
+}
 __device__ __forceinline__ uint32_t pack_h2(__half lo, __half hi) {
   return (uint32_t)__half_as_ushort(lo) | ((uint32_t)__half_as_ushort(hi) << 16);
 }
@@ -393,25 +425,25 @@ __device__ __forceinline__ const uint8_t* blk_at(const uint8_t* st, const uint8_
 // Key residual term scale (q'_g . c) + min sum(q'_g) of the key record whose scale-min word
 // is at `smn_off` and whose codes start at `cd_off`.
 __device__ __noinline__ float key_record_term(const uint8_t* st, const uint8_t* gb, uint32_t staged, uint32_t smn_off,
-                                              uint32_t cd_off, const float* qpg, float sqg) {
+                                              uint32_t cd_off, const float* qpg, float sqg, int lloyd) {
   const uint32_t smn = *reinterpret_cast<const uint32_t*>(blk_at(st, gb, staged, smn_off));
   float dot = 0.f;
   for (int bb = 0; bb < 32; ++bb) {
     const uint32_t byte = *blk_at(st, gb, staged, cd_off + (uint32_t)bb);
 #pragma unroll
-    for (int c = 0; c < 4; ++c) dot += qpg[4 * bb + c] * (float)((byte >> (2 * c)) & 3u);
+    for (int c = 0; c < 4; ++c) dot += qpg[4 * bb + c] * code_level((byte >> (2 * c)) & 3u, lloyd);
   }
   return half_hi(smn) * sqg + half_lo(smn) * dot;
 }
 // accg += p (min + scale c) of value record r, in the rotated domain (value codes are
 // dimension-major groups of 16 records; the group of r starts at `grp_off`).
 __device__ __noinline__ void value_record_add(const uint8_t* st, const uint8_t* gb, uint32_t staged, uint32_t smn_off,
-                                              uint32_t grp_off, int r, float p, float* accg) {
+                                              uint32_t grp_off, int r, float p, float* accg, int lloyd) {
   const uint32_t smn = *reinterpret_cast<const uint32_t*>(blk_at(st, gb, staged, smn_off));
   const float ps = p * half_lo(smn), pm = p * half_hi(smn);
   for (int d = 0; d < 128; ++d) {
     const uint32_t w = *reinterpret_cast<const uint32_t*>(blk_at(st, gb, staged, grp_off + 4u * value_code_word(d)));
-    atomicAdd(&accg[d], fmaf(ps, (float)((w >> value_code_bit(r % 16)) & 3u), pm));
+    atomicAdd(&accg[d], fmaf(ps, code_level((w >> value_code_bit(r % 16)) & 3u, lloyd), pm));
   }
 }
 // acc[g] x the anchor's value row (global memory, swizzled by the slot), added into ov[g][:]:
@@ -855,7 +887,7 @@ struct TokTile {
   float* W;           // [X][GS] the tile's value weights
   float* ovf;         // [2][GS][128] overflow sums
   const uint8_t* AV;  // the unit's anchor values (global)
-  int k, nKs, nVs, ka;
+  int k, nKs, nVs, ka, lloyd;
 };
 
 // The general token path (kept out of line: a tile with records beyond the staged ones, runs
@@ -889,7 +921,7 @@ __device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const
   float* pv = tt.pv;
   float* ovf = tt.ovf;
   const uint8_t* AV = tt.AV;
-  const int k = tt.k, nKs = tt.nKs, nVs = tt.nVs, ka = tt.ka;
+  const int k = tt.k, nKs = tt.nKs, nVs = tt.nVs, ka = tt.ka, lloyd = tt.lloyd;
   const uint32_t lo = tt.lo;
   const int nrows = (int)tt.nrows;
   int rkn = tl.rk, rvn = tl.rv;
@@ -927,7 +959,7 @@ __device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const
 #pragma unroll
       for (int g = 0; g < GS; ++g)
         rt[g] = key_record_term(st, gb, staged, tv.sm_k + 4u * (uint32_t)r, tv.cd_k + 32u * (uint32_t)r, qp + g * 128,
-                                qp[GS * 128 + g]) +
+                                qp[GS * 128 + g], lloyd) +
                 negrow[g];
     } else {  // the key-residual terms minus m, -m, or -inf for a token past the tile's end
       load_row<GS>(e >= nvalid ? ninfrow : negrow, rt);
@@ -951,7 +983,7 @@ __device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const
 #pragma unroll
         for (int g = 0; g < GS; ++g)
           value_record_add(st, gb, staged, tv.sm_v + 4u * (uint32_t)rv, tv.cd_v + 512u * (uint32_t)(rv / 16), rv,
-                           (g & 1) ? pe[g >> 1].y : pe[g >> 1].x, ovf + GS * 128 + g * 128);
+                           (g & 1) ? pe[g >> 1].y : pe[g >> 1].x, ovf + GS * 128 + g * 128, lloyd);
       }
     }
     // tokens past the tile join the current run with zero weight
@@ -974,7 +1006,8 @@ __device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const
 }
 
 // ================================ decode ============================================
-template <int GS>
+// CODEC: 0 = uniform codes (c^ = min + c scale), 1 = Lloyd-Max levels (c^ = scale L[c]).
+template <int GS, int CODEC>
 __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P) {
   extern __shared__ __align__(128) uint8_t smem[];
   constexpr int NP = GS >= 2 ? GS / 2 : 1;      // pairs of heads for the packed arithmetic
@@ -1250,7 +1283,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
             for (int q = 0; q < 2; ++q) {
               const uint32_t xa = wd[q][0][ks] >> (4 * c4), xb = wd[q][1][ks] >> (4 * c4);
-              const uint4 a = make_uint4(codes2_to_h2(xa), codes2_to_h2(xb), codes2_to_h2(xa >> 2), codes2_to_h2(xb >> 2));
+              const uint4 a = make_uint4(code_pair_h2<CODEC>(xa), code_pair_h2<CODEC>(xb), code_pair_h2<CODEC>(xa >> 2),
+                                         code_pair_h2<CODEC>(xb >> 2));
               if constexpr (GS == 8) {
                 mma_f16(d[q][0], a, b0.x, b0.y);
                 mma_f16(d[q][1], a, b1.x, b1.y);
@@ -1431,7 +1465,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             }
           }
         } else if (t0 < tv.n) {
-          const auto ls = token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, U.AV, k, nKs, nVs, P.ka_stride}, tl);
+          const auto ls = token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, U.AV, k, nKs, nVs, P.ka_stride, CODEC}, tl);
 #pragma unroll
           for (int i2 = 0; i2 < NP; ++i2) l2[i2] = __fadd2_rn(l2[i2], ls.v[i2]);
         }
@@ -1524,7 +1558,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             for (int nb = 0; nb < 4; ++nb) {
               // records 2c, 2c+1 at bits 2c and 2c + 16, records 2c+8, 2c+9 eight bits higher
               const uint32_t x = wd[nb] >> (2 * c4);
-              mma_bf16(accR[nb], a.x, a.y, a.z, a.w, codes2_to_b2(x), codes2_to_b2(x >> 8));
+              mma_bf16(accR[nb], a.x, a.y, a.z, a.w, code_pair_b2<CODEC>(x), code_pair_b2<CODEC>(x >> 8));
             }
           }
         }
@@ -1756,8 +1790,8 @@ bool make_plan(const Layout& L, int GS, int smem_optin, Plan* out, std::string* 
 using DecodeFn = void (*)(const DecodeParams);
 using ScoreFn = void (*)(const ScoreParams);
 template <int GS>
-DecodeFn decode_kernel() {
-  return akv_decode_kernel<GS>;
+DecodeFn decode_kernel(int codec) {
+  return codec ? akv_decode_kernel<GS, 1> : akv_decode_kernel<GS, 0>;
 }
 template <int GS>
 ScoreFn score_kernel() {
@@ -1767,11 +1801,11 @@ ScoreFn score_kernel() {
 // Launch configuration per (device, G, layout shape): computed once, then reused, so that a
 // call made during CUDA-graph capture only issues the launches.
 struct LaunchKey {
-  int dev, G, units, max_len, max_k, ctas;
+  int dev, G, codec, units, max_len, max_k, ctas;
   long long dens_key, adens_key, ttot;
   bool operator<(const LaunchKey& o) const {
-    return std::tie(dev, G, units, max_len, max_k, ctas, dens_key, adens_key, ttot) <
-           std::tie(o.dev, o.G, o.units, o.max_len, o.max_k, o.ctas, o.dens_key, o.adens_key, o.ttot);
+    return std::tie(dev, G, codec, units, max_len, max_k, ctas, dens_key, adens_key, ttot) <
+           std::tie(o.dev, o.G, o.codec, o.units, o.max_len, o.max_k, o.ctas, o.dens_key, o.adens_key, o.ttot);
   }
 };
 
@@ -1825,7 +1859,8 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   // after their bound and the outputs of its units become NaN
   const int ctas = g_debug_cluster.load(std::memory_order_relaxed);
   const int drop = g_debug_withhold.load(std::memory_order_relaxed);
-  const LaunchKey key{dev, L.G, units, L.max_len, L.max_k, ctas, (long long)(max_density(L) * 1e6),
+  const int codec = (p.flags & AKV_FLAG_LLOYD) ? 1 : 0;
+  const LaunchKey key{dev, L.G, codec, units, L.max_len, L.max_k, ctas, (long long)(max_density(L) * 1e6),
                       (long long)(max_anchor_density(L) * 1e6), ttot};
   Plan pl;
   bool have = false;
@@ -1839,7 +1874,7 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   }
   if (!have) {
     const DeviceInfo di = device_info();
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel<GS>(), cudaFuncAttributeMaxDynamicSharedMemorySize, di.smem_optin);
+    cudaError_t e = cudaFuncSetAttribute(decode_kernel<GS>(codec), cudaFuncAttributeMaxDynamicSharedMemorySize, di.smem_optin);
     if (e != cudaSuccess) return (int)e;
     if (!make_plan(L, GS, di.smem_optin, &pl, why)) return -1;
     int grid = (int)std::min<long long>(std::min(di.sms, kMaxGrid), ttot);
@@ -1926,10 +1961,10 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   cfg.gridDim = dim3((unsigned)pl.grid, 1, 1);
   cfg.blockDim = dim3(NT, 1, 1);
   cfg.dynamicSmemBytes = pl.smem;
-  e = cudaLaunchKernelEx(&cfg, decode_kernel<GS>(), P);
+  e = cudaLaunchKernelEx(&cfg, decode_kernel<GS>(codec), P);
   if (e != cudaSuccess) {
     cudaFuncAttributes fa{};
-    cudaFuncGetAttributes(&fa, decode_kernel<GS>());
+    cudaFuncGetAttributes(&fa, decode_kernel<GS>(codec));
     *why = "(decode kernel: " + std::to_string(fa.numRegs) + " registers, max " + std::to_string(fa.maxThreadsPerBlock) +
            " threads, " + std::to_string(pl.smem) + " B dynamic shared memory of " +
            std::to_string(fa.maxDynamicSharedSizeBytes) + ", grid " + std::to_string(pl.grid) + ")";

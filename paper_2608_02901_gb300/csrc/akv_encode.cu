@@ -30,6 +30,10 @@
 namespace akv {
 namespace {
 
+// The Lloyd-Max codec's outer decision threshold: the midpoint of its levels 0.453125 and
+// 1.5078125 (the Gaussian four-level Lloyd-Max levels 0.4528, 1.5104 to 8 significant bits).
+constexpr double kLloydT = 0.98046875;
+
 // Per-unit scratch pointers, derived from the workspace table the host writes.
 struct EncUnitWs {
   uint64_t* key0;     // [S] anchor hashes, then key residual energies
@@ -60,6 +64,7 @@ struct EncArgs {
   int32_t n_kv_heads;
   int32_t window;
   int32_t rotate;
+  int32_t lloyd;  // AKV_FLAG_LLOYD: the Lloyd-Max codec
   uint64_t seed;
   unsigned long long sign_lo, sign_hi;
   // full selection (m_obs > 0): observation rows Q [units][m_obs][128], pooling width,
@@ -635,37 +640,57 @@ __global__ void enc_quant(const EncArgs A) {
       __syncwarp();
     }
   }
-  // min / max with the first index winning ties (as a sequential scan does)
-  double mnv = v[4 * lane], mxv = mnv;
-  int mni = 4 * lane, mxi = mni;
-  for (int c = 1; c < 4; ++c) {
-    const double x = v[4 * lane + c];
-    if (x < mnv) { mnv = x; mni = 4 * lane + c; }
-    if (x > mxv) { mxv = x; mxi = 4 * lane + c; }
-  }
-  for (int o = 16; o > 0; o >>= 1) {
-    const double omn = __shfl_xor_sync(0xffffffffu, mnv, o);
-    const int omi = __shfl_xor_sync(0xffffffffu, mni, o);
-    const double omx = __shfl_xor_sync(0xffffffffu, mxv, o);
-    const int oxi = __shfl_xor_sync(0xffffffffu, mxi, o);
-    if (omn < mnv || (omn == mnv && omi < mni)) { mnv = omn; mni = omi; }
-    if (omx > mxv || (omx == mxv && oxi < mxi)) { mxv = omx; mxi = oxi; }
-  }
-  const uint32_t mnh = f64_to_fp16_bits(mnv);
-  const double mn = fp16_bits_to_f64(mnh);
-  double t = __ddiv_rn(__dsub_rn(mxv, mn), 3.0);
-  if (!(t > 0.0)) t = 0.0;
-  const uint32_t sch = f64_to_fp16_bits(t);
-  const double sc = fp16_bits_to_f64(sch);
-  uint32_t byte = 0;
-  for (int c = 0; c < 4; ++c) {
-    int code = 0;
-    if (sc != 0.0) {
-      double qv = rint(__ddiv_rn(__dsub_rn(v[4 * lane + c], mn), sc));
-      qv = fmin(fmax(qv, 0.0), 3.0);
-      code = (int)qv;
+  uint32_t mnh, sch, byte = 0;
+  if (A.lloyd) {
+    // Lloyd-Max codec (Section 3.1, Appendix A.1): per-token RMS scale fp16(sqrt(sum v^2 / 128)),
+    // the sum in index order (lane 0), min 0, codes by the decision regions of v / scale
+    double ss = 0.0;
+    if (lane == 0)
+      for (int j = 0; j < 128; ++j) ss = __dadd_rn(ss, __dmul_rn(v[j], v[j]));
+    ss = __shfl_sync(0xffffffffu, ss, 0);
+    sch = f64_to_fp16_bits(__dsqrt_rn(__ddiv_rn(ss, 128.0)));
+    mnh = 0u;
+    const double sc = fp16_bits_to_f64(sch);
+    for (int c = 0; c < 4; ++c) {
+      int code = 2;  // a zero scale: every level reconstructs 0
+      if (sc != 0.0) {
+        const double t = __ddiv_rn(v[4 * lane + c], sc);
+        code = t < -kLloydT ? 0 : (t < 0.0 ? 1 : (t < kLloydT ? 2 : 3));
+      }
+      byte |= (uint32_t)code << (2 * c);
     }
-    byte |= (uint32_t)code << (2 * c);
+  } else {
+    // min / max with the first index winning ties (as a sequential scan does)
+    double mnv = v[4 * lane], mxv = mnv;
+    int mni = 4 * lane, mxi = mni;
+    for (int c = 1; c < 4; ++c) {
+      const double x = v[4 * lane + c];
+      if (x < mnv) { mnv = x; mni = 4 * lane + c; }
+      if (x > mxv) { mxv = x; mxi = 4 * lane + c; }
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+      const double omn = __shfl_xor_sync(0xffffffffu, mnv, o);
+      const int omi = __shfl_xor_sync(0xffffffffu, mni, o);
+      const double omx = __shfl_xor_sync(0xffffffffu, mxv, o);
+      const int oxi = __shfl_xor_sync(0xffffffffu, mxi, o);
+      if (omn < mnv || (omn == mnv && omi < mni)) { mnv = omn; mni = omi; }
+      if (omx > mxv || (omx == mxv && oxi < mxi)) { mxv = omx; mxi = oxi; }
+    }
+    mnh = f64_to_fp16_bits(mnv);
+    const double mn = fp16_bits_to_f64(mnh);
+    double t = __ddiv_rn(__dsub_rn(mxv, mn), 3.0);
+    if (!(t > 0.0)) t = 0.0;
+    sch = f64_to_fp16_bits(t);
+    const double sc = fp16_bits_to_f64(sch);
+    for (int c = 0; c < 4; ++c) {
+      int code = 0;
+      if (sc != 0.0) {
+        double qv = rint(__ddiv_rn(__dsub_rn(v[4 * lane + c], mn), sc));
+        qv = fmin(fmax(qv, 0.0), 3.0);
+        code = (int)qv;
+      }
+      byte |= (uint32_t)code << (2 * c);
+    }
   }
   // record r of its tile: the rank of the token among the tile's tokens with this side's bit
   const int ts = w.inv[p], j = ts / kTile, tl = ts % kTile;
@@ -1016,6 +1041,7 @@ int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const
   A.n_kv_heads = p.n_kv_heads;
   A.window = p.window;
   A.rotate = (p.flags & AKV_FLAG_ROTATE) ? 1 : 0;
+  A.lloyd = (p.flags & AKV_FLAG_LLOYD) ? 1 : 0;
   A.seed = p.seed;
   A.sign_lo = L.header.sign_bits[0];
   A.sign_hi = L.header.sign_bits[1];

@@ -266,3 +266,30 @@ def test_withheld_item_times_out_to_nan_and_context_survives(dev, debug_controls
     assert waited > 1.0, waited
     out, out32 = decode_on_gpu(torch, p, lens, arena, q, 1.0)
     check_outputs(out, out32, oracle_decode(p, [oracle_unit(u) for u in units], q, 1.0), where="after the timed-out call")
+
+
+@pytest.mark.parametrize("G", [1, 4, 8])
+@pytest.mark.parametrize("fr", [(0.02, 0.1, 0.1), (0.02, 1.0, 1.0)])
+def test_lloyd_max_codec_seeded(dev, G, fr):
+    """The Lloyd-Max codec's levels on both tensor-core paths (key and value residuals) and, with
+    every token a residual, on the CUDA-core paths for records beyond the staged ones."""
+    p = akv.Params(batch=2, n_kv_heads=2, n_q_heads=2 * G, anchor_frac=fr[0], res_frac_k=fr[1], res_frac_v=fr[2],
+                   seed=12, rot_seed=13, lloyd=True)
+    _run_seeded(dev, p, [3000, 1100], qseed=G)
+
+
+@pytest.mark.parametrize("G", [4, 8])
+def test_lloyd_max_codec_encoded(dev, G):
+    """GPU encode with the Lloyd-Max codec, then decode, against the oracle reading the arena."""
+    S, H = 8192, 2
+    p = akv.Params(batch=1, n_kv_heads=H, n_q_heads=H * G, seed=7, rot_seed=11, lloyd=True)
+    K, V = gen.clustered_batch(1, H, [S], seed=44)
+    a_bytes, w_bytes = akv.akv_cache_size(p, [S])
+    arena = torch.empty(a_bytes, dtype=torch.uint8, device=dev)
+    ws = torch.empty(w_bytes, dtype=torch.uint8, device=dev)
+    akv.akv_encode(p, [S], to_dev_u16(K, torch, dev), to_dev_u16(V, torch, dev), arena, ws)
+    units = oracle.unpack_arena(arena.cpu().numpy())
+    for qseed in (1, 2):
+        q = gen.queries(H * G, seed=qseed)
+        out, out32 = decode_on_gpu(torch, p, [S], arena, q, 1.0)
+        check_outputs(out, out32, oracle_decode(p, units, q, 1.0), f"lloyd encoded G={G} q={qseed}")

@@ -25,7 +25,7 @@ def _encode_both(dev, p, lens, K, V):
     torch.cuda.synchronize()
     got = oracle.unpack_arena(arena.cpu().numpy())
     want = oracle.encode(K, V, lens, p.n_kv_heads, p.anchor_frac, p.res_frac_k, p.res_frac_v, p.window, p.seed,
-                         p.rot_seed, p.rotate)
+                         p.rot_seed, p.rotate, lloyd=p.lloyd)
     assert len(got) == len(want)
     for u, (g, w) in enumerate(zip(got, want)):
         assert (g.S, g.k, g.nk, g.nv) == (w.S, w.k, w.nk, w.nv)
@@ -76,3 +76,22 @@ def test_all_anchor_rows_zero(dev):
     K, V = K.copy(), V.copy()
     K[0, 0, 32:] = 0  # every anchor key is zero: no usable direction on the key side
     _encode_both(dev, p, lens, K, V)
+
+
+@pytest.mark.parametrize("rotate", [True, False])
+def test_lloyd_max_codec_bit_exact(dev, rotate):
+    """The Lloyd-Max codec (per-token RMS scale, min 0, decision-region codes), every residual
+    stored (res_frac 1), on clustered rows and ragged lengths."""
+    lens = [1, 700, 3000]
+    p = akv.Params(batch=3, n_kv_heads=2, n_q_heads=4, res_frac_k=1.0, res_frac_v=0.6, seed=5, rot_seed=9,
+                   rotate=rotate, lloyd=True)
+    K, V = gen.clustered_batch(3, 2, lens, seed=123)
+    got = _encode_both(dev, p, lens, K, V)
+    assert any(u.nk and not u.min_k.any() and u.scale_k.any() for u in got)  # min 0, scales stored
+
+
+def test_lloyd_max_codec_8b_32k_bit_exact(dev):
+    S = 32768
+    p = akv.Params(batch=1, n_kv_heads=8, n_q_heads=32, seed=1, rot_seed=2, lloyd=True)
+    K, V = gen.clustered_batch(1, 8, [S], seed=42)
+    _encode_both(dev, p, [S], K, V)

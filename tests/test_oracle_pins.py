@@ -424,3 +424,80 @@ def test_suffix_lengths_follow_requests_in_a_batch():
         ref = oracle.attend_suffix([units[u]], q.reshape(4, 2, D)[u], 2, 1, 1.0, 11, ks[u:u + 1, :3], vs[u:u + 1, :3],
                                    [3]) if u < 2 else plain[u:u + 1]
         assert np.array_equal(out[u:u + 1], ref)
+
+
+# ---- Lloyd-Max codec (Section 3.1, Appendix A.1 "Codebook"; distortion Eq. 13) ----
+
+# Max (1960): the four-level minimum-MSE quantizer of a unit Gaussian has levels +-0.4528,
+# +-1.5104 and thresholds 0, +-0.9816; the codec takes the levels to 8 significant bits.
+LM_LEVELS = np.array([-1.5078125, -0.453125, 0.453125, 1.5078125])
+
+
+def test_lloyd_levels_are_the_gaussian_lloyd_max_quantizer():
+    """The table is within 0.5 % of Max's levels, and those levels are the centroids of the unit
+    Gaussian over their own midpoint decision regions (the Lloyd condition), to 1e-3."""
+    import scipy.stats as st
+    assert np.allclose(LM_LEVELS, [-1.5104, -0.4528, 0.4528, 1.5104], rtol=5e-3)
+    t = 0.5 * (0.4528 + 1.5104)
+    for lo, hi, level in ((0.0, t, 0.4528), (t, np.inf, 1.5104)):
+        centroid = (st.norm.pdf(lo) - st.norm.pdf(hi)) / (st.norm.cdf(hi) - st.norm.cdf(lo))
+        assert abs(centroid - level) < 1e-3
+
+
+def test_lloyd_quantizer_without_rotation_hand_example():
+    # 48 coordinates of +-1.5 sigma and 80 of +-0.5 sigma: the RMS is exactly sigma = 0.75
+    # (fp16-exact); +-1.5 lies beyond the outer threshold, +-0.5 inside it
+    t = np.array([1.5] * 24 + [-1.5] * 24 + [0.5] * 40 + [-0.5] * 40)
+    rng = np.random.default_rng(4)
+    perm = rng.permutation(D)
+    r = 0.75 * t[perm]
+    codes, sc, mn = oracle.quantize_residual(r, rot_seed=5, rotate=False, lloyd=True)
+    assert sc == np.float16(0.75).view(np.uint16) and mn == 0
+    expect = np.where(t[perm] > 1, 3, np.where(t[perm] > 0, 2, np.where(t[perm] > -1, 1, 0)))
+    assert np.array_equal(codes, _pack(expect))
+    out = oracle.dequantize_residual(codes, sc, mn, rot_seed=5, rotate=False, lloyd=True)
+    assert np.array_equal(out, 0.75 * LM_LEVELS[expect])
+
+
+def test_lloyd_quantizer_with_rotation_matches_a_dense_hadamard():
+    """Codes of the rotated vector v = H (s o r) by the decision regions of v / fp16(RMS(v)), and
+    the record dequantized as s o (H (scale L[code])) / 128 with a dense Hadamard matrix."""
+    rng = np.random.default_rng(6)
+    s = oracle.signs(21)
+    H = scipy.linalg.hadamard(D).astype(np.float64)
+    for _ in range(20):
+        r = rng.standard_normal(D) * rng.uniform(0.01, 3.0)
+        codes, sc, mn = oracle.quantize_residual(r, rot_seed=21, rotate=True, lloyd=True)
+        v = H @ (s * r)
+        scale = float(np.float16(np.sqrt(np.sum(v * v) / D)))
+        assert sc == np.float16(scale).view(np.uint16) and mn == 0
+        x = v / scale
+        expect = np.where(x < -0.98046875, 0, np.where(x < 0, 1, np.where(x < 0.98046875, 2, 3)))
+        assert np.array_equal(codes, _pack(expect))
+        out = oracle.dequantize_residual(codes, sc, mn, rot_seed=21, rotate=True, lloyd=True)
+        assert np.allclose(out, s * (H @ (scale * LM_LEVELS[expect])) / D, rtol=0, atol=1e-13)
+
+
+def test_lloyd_zero_residual():
+    codes, sc, mn = oracle.quantize_residual(np.zeros(D), rot_seed=1, rotate=True, lloyd=True)
+    assert sc == 0 and mn == 0
+    assert np.array_equal(codes, _pack([2] * D))
+    assert not oracle.dequantize_residual(codes, sc, mn, 1, True, True).any()
+
+
+def test_eta_of_each_codec_on_gaussian_residuals():
+    """Eq. 13 on rotated Gaussian residuals: the Lloyd-Max codec leaves about the Gaussian
+    four-level minimum MSE (0.1175, here from numerical integration of its own levels and
+    thresholds; the per-token RMS scale brings it slightly lower), the uniform min/max codec about
+    twice as much."""
+    import scipy.integrate as si
+    import scipy.stats as st
+    T = 0.98046875
+    mse = 2 * sum(si.quad(lambda x, L=L: (x - L) ** 2 * st.norm.pdf(x), lo, hi)[0]
+                  for lo, hi, L in ((0, T, 0.453125), (T, np.inf, 1.5078125)))
+    assert abs(mse - 0.1175) < 1e-3
+    R = np.random.default_rng(0).standard_normal((2000, D))
+    e_lm = oracle.eta(R, 11, True, True)
+    e_un = oracle.eta(R, 11, True, False)
+    assert abs(e_lm - mse) < 0.005
+    assert 1.8 * e_lm < e_un < 0.3

@@ -47,7 +47,7 @@ def _run(dev, p, lens, suf_lens, cap, sm_scale=1.0, seed=5, qseed=17, key_scale=
     akv.akv_decode_attn(p, lens, arena, qt, out, out32, sm_scale=sm_scale, suffix=sfx)
     torch.cuda.synchronize()
     ref = oracle.attend_suffix([oracle_unit(u) for u in units], q.reshape(p.n_units, p.G, 128), p.G, H, sm_scale,
-                               p.rot_seed, ks, vs, suf_lens, p.rotate).reshape(p.batch, p.n_q_heads, 128)
+                               p.rot_seed, ks, vs, suf_lens, p.rotate, lloyd=p.lloyd).reshape(p.batch, p.n_q_heads, 128)
     return check_outputs(out.float().cpu().numpy(), out32.cpu().numpy(), ref, where=where)
 
 
