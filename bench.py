@@ -81,6 +81,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--codec", default="uniform", choices=["uniform", "lloyd"],
                     help="residual codec: 4 uniform levels on [min, max], or the Lloyd-Max codebook (AKV_FLAG_LLOYD)")
+    ap.add_argument("--rope", action="store_true",
+                    help="pre-RoPE keys with RoPE applied at decode (AKV_FLAG_ROPE, base 500000)")
     ap.add_argument("--suffix", type=int, default=0,
                     help="exact dense suffix: this many generated tokens per request, kept in bf16 and attended in "
                          "the same softmax (0 = none)")
@@ -127,10 +129,11 @@ def arena_unit_bytes(torch, akv, p, lens, arena) -> list:
     offs = []
     for u in range(p.n_units):
         d = hdr[256 * (u + 1): 256 * (u + 2)]
-        k, nt = int(d[4:8].view(np.int32)[0]), int(d[16:20].view(np.int32)[0])
+        S, k, nt = int(d[0:4].view(np.int32)[0]), int(d[4:8].view(np.int32)[0]), int(d[16:20].view(np.int32)[0])
         o_tt = int(d[56:64].view(np.uint64)[0])
         offs.append(o_tt + 4 * nt)
-        fixed.append(512 * k + 4 * (2 * nt + 1) + 2 * (2 * p.G * 128))
+        # (RoPE at decode: plus the stored tokens' positions)
+        fixed.append(512 * k + 4 * (2 * nt + 1) + 2 * (2 * p.G * 128) + (4 * S if p.rope else 0))
     idx = torch.tensor([o + i for o in offs for i in range(4)], dtype=torch.long, device=arena.device)
     used = arena[idx].cpu().numpy().view(np.uint32).astype(np.int64)
     return [f + int(b) for f, b in zip(fixed, used)]
@@ -138,14 +141,17 @@ def arena_unit_bytes(torch, akv, p, lens, arena) -> list:
 
 def arena_kernel_bytes(torch, akv, p, lens, arena):
     """Algorithmic bytes of each of the decode call's two launches over this arena: the score
-    launch reads the anchor keys and the query rows; the decode launch reads the anchor values,
-    the tile table and the tile blocks, and writes the output rows (the anchor scores it passes
-    between them through the workspace are not counted)."""
+    launch reads the anchor keys and the query rows (with RoPE at decode, the logits launch also
+    the positions and key stream words); the decode launch the rest: anchor values, tile table,
+    tile blocks, output rows (what the launches pass through the workspace is not counted)."""
     hdr = akv.akv_cache_header_host(p, lens)
     k_sum = sum(int(hdr[256 * (u + 1) + 4: 256 * (u + 1) + 8].view(np.int32)[0]) for u in range(p.n_units))
+    s_sum = sum(int(hdr[256 * (u + 1): 256 * (u + 1) + 4].view(np.int32)[0]) for u in range(p.n_units))
     rows = p.n_units * 2 * p.G * 128
     total = arena_read_bytes(torch, akv, p, lens, arena)
     scores = 256 * k_sum + rows
+    if p.rope:  # the RoPE logits launch also reads every token's position and key stream word
+        scores += 8 * s_sum
     return scores, total - scores
 
 
@@ -356,7 +362,7 @@ def run_akv(args, rank, world, local):
     B, H, Hq, S, source = WORKLOADS[args.workload]
     lens = workload_lens(args.workload, B, S)
     p = workload_params(akv, args.workload, batch=B, n_kv_heads=H, n_q_heads=Hq, seed=rank_seed(11, rank),
-                        rot_seed=0x5EED, lloyd=args.codec == "lloyd")
+                        rot_seed=0x5EED, lloyd=args.codec == "lloyd", rope=args.rope)
     layers = args.layers
     arenas, arena_bytes, step_bytes = build_layers(torch, akv, gen, p, lens, layers, source, dev, rank)
     n_tok = N_TOKENS
@@ -524,7 +530,7 @@ def run_akv(args, rank, world, local):
         "config": {"workload": args.workload, "batch": B, "n_kv_heads": H, "n_q_heads": Hq,
                    "context": S if args.workload not in SWEEP_POINTS else f"ragged U[8192, 131072]: {lens}",
                    "anchor_frac": p.anchor_frac, "res_frac": p.res_frac_k, "layers_cycled": layers,
-                   "suffix_tokens": args.suffix, "codec": args.codec,
+                   "suffix_tokens": args.suffix, "codec": args.codec, "rope_at_decode": args.rope,
                    "fresh_queries": N_TOKENS, "arena_bytes_per_layer": arena_bytes,
                    "l2": f"inputs larger than L2: {layers} distinct layer caches, {layers * arena_bytes / 1e6:.0f} MB cycled",
                    "timing": "CUDA graph replay, CUDA events on the launching stream", "parallelism": f"dp{world}"},

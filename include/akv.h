@@ -61,8 +61,15 @@ typedef enum akv_status {
  * L = {-1.5078125, -0.453125, 0.453125, 1.5078125} (Max's levels +-0.4528, +-1.5104 to 8
  * significant bits, exact in bf16 and fp16).  Encode and decode must use the same flags. */
 #define AKV_FLAG_LLOYD 2u
+/* RoPE applied at decode (Section 3.2; Appendix E.1's score kernel): the keys given to the
+ * encoder are pre-RoPE and are compressed as they are; the arena keeps each stored token's
+ * original position (its index in the request: 0 .. S-1), and the decode scores token i at
+ * position p_i as q . R(p_i) x^_i, R(p) the rotate-half RoPE rotation of dimension pairs
+ * (j, j + 64) by the angle p theta_j, theta_j = rope_theta^(-2j/128).  q is given already
+ * rotated to its own position, as a model computes it.  rope_theta must be finite and > 1. */
+#define AKV_FLAG_ROPE 4u
 #define AKV_ARENA_MAGIC 0x32564B41u /* "AKV2" */
-#define AKV_ARENA_VERSION 3u
+#define AKV_ARENA_VERSION 4u
 #define AKV_MAX_ANCHORS 65535 /* anchor indices are uint16 (Table 1, b_a = 2) */
 #define AKV_TILE_TOKENS 1024  /* tokens per tile block of the packed token stream */
 
@@ -93,7 +100,7 @@ typedef struct akv_params {
   uint64_t seed;
   uint64_t rot_seed;
   uint32_t flags;
-  uint32_t reserved; /* must be 0 */
+  float rope_theta;   /* AKV_FLAG_ROPE: the RoPE base; 0 otherwise */
 } akv_params;
 
 /*
@@ -182,8 +189,9 @@ typedef struct akv_unit_desc {
   int32_t reserved0;
   uint64_t off_anchor_k, off_anchor_v, off_anchor_pos, off_tile_table, off_tiles;
   uint64_t tiles_capacity; /* bytes reserved for the tile blocks (an upper bound of their use) */
-  uint64_t data_bytes;     /* anchors + tile table + tiles_capacity: the most one decode reads */
-  uint8_t pad[256 - 32 - 7 * 8];
+  uint64_t data_bytes;     /* anchors + tile table + tiles_capacity (+ positions): the most one decode reads */
+  uint64_t off_pos;        /* AKV_FLAG_ROPE: u32 [S], the original position of each stored token; else 0 */
+  uint8_t pad[256 - 32 - 8 * 8];
 } akv_unit_desc;
 
 /* ---- Introspection ------------------------------------------------------ */
@@ -454,7 +462,8 @@ akv_status akv_decode_workspace_size_suffix(const akv_params* p, const int32_t* 
  * combine rescales those partials to the common maximum (one softmax, exactly).
  *   ws : >= akv_decode_workspace_size_suffix(p, ctx_lens_host, suffix->cap)
  * Errors: those of akv_decode_attn, and AKV_ERR_INVALID for a suffix with null
- * or misaligned pointers (K, V 16-byte aligned; len 4-byte) or cap out of range.
+ * or misaligned pointers (K, V 16-byte aligned; len 4-byte) or cap out of range;
+ * AKV_ERR_UNSUPPORTED for a suffix with AKV_FLAG_ROPE (not built).
  * Lengths above cap are taken as cap.
  */
 akv_status akv_decode_attn_suffix(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,

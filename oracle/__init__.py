@@ -46,7 +46,7 @@ class _OrUnit(ctypes.Structure):
     _fields_ = [("S", ctypes.c_int32), ("k", ctypes.c_int32), ("nk", ctypes.c_int32), ("nv", ctypes.c_int32)] + [
         (name, ctypes.c_void_p)
         for name in ("anchor_k", "anchor_v", "anchor_pos", "idx_k", "gam_k", "idx_v", "gam_v", "res_k", "codes_k",
-                     "scale_k", "min_k", "res_v", "codes_v", "scale_v", "min_v")
+                     "scale_k", "min_k", "res_v", "codes_v", "scale_v", "min_v", "pos")
     ]
 
 
@@ -73,8 +73,10 @@ def lib():
             L.or_encode_batch.restype = ctypes.c_int
             L.or_encode_batch.argtypes = [vp, vp, i32, i32, i32, i32, u64, u64, ctypes.c_int, vp]
             L.or_attend_unit.argtypes = [ctypes.POINTER(_OrUnit), vp, i32, dbl, u64, ctypes.c_int, vp]
-            L.or_attend_batch.argtypes = [vp, i32, vp, i32, dbl, u64, ctypes.c_int, vp, vp]
-            L.or_attend_batch_suffix.argtypes = [vp, i32, i32, vp, i32, dbl, u64, ctypes.c_int, vp, vp, vp, i32, vp]
+            L.or_attend_batch.argtypes = [vp, i32, vp, i32, dbl, u64, ctypes.c_int, dbl, vp, vp]
+            L.or_attend_batch_suffix.argtypes = [vp, i32, i32, vp, i32, dbl, u64, ctypes.c_int, dbl, vp, vp, vp, i32,
+                                                 vp]
+            L.or_rope.argtypes = [vp, ctypes.c_int64, dbl]
             L.or_attend_factorized.argtypes = [ctypes.POINTER(_OrUnit), vp, i32, dbl, u64, ctypes.c_int, vp]
             L.or_reconstruct_side.argtypes = [i32, vp, vp, vp, i32, vp, vp, vp, vp, u64, ctypes.c_int, vp]
             L.or_quantize_residual.argtypes = [vp, u64, ctypes.c_int, vp, vp, vp]
@@ -122,12 +124,15 @@ class Unit:
     codes_v: np.ndarray
     scale_v: np.ndarray
     min_v: np.ndarray
+    pos: np.ndarray = None  # [S] int32 position of index i (RoPE at decode); None: position i
 
     def c_struct(self) -> _OrUnit:
         s = _OrUnit(self.S, self.k, self.nk, self.nv)
         for name in ("anchor_k", "anchor_v", "anchor_pos", "idx_k", "gam_k", "idx_v", "gam_v", "res_k", "codes_k",
-                     "scale_k", "min_k", "res_v", "codes_v", "scale_v", "min_v"):
+                     "scale_k", "min_k", "res_v", "codes_v", "scale_v", "min_v", "pos"):
             arr = getattr(self, name)
+            if arr is None:
+                continue
             assert arr.flags.c_contiguous
             setattr(s, name, arr.ctypes.data if arr.size else None)
         return s
@@ -139,7 +144,7 @@ def alloc_unit(S: int, k: int, nk: int, nv: int) -> Unit:
                 z((k, D), np.uint16), z((k, D), np.uint16), z(k, np.int32),
                 z(S, np.uint16), z(S, np.uint16), z(S, np.uint16), z(S, np.uint16),
                 z(nk, np.int32), z((nk, 32), np.uint8), z(nk, np.uint16), z(nk, np.uint16),
-                z(nv, np.int32), z((nv, 32), np.uint8), z(nv, np.uint16), z(nv, np.uint16))
+                z(nv, np.int32), z((nv, 32), np.uint8), z(nv, np.uint16), z(nv, np.uint16), np.arange(S, dtype=np.int32))
 
 
 # ---- scalar helpers -------------------------------------------------------
@@ -175,6 +180,14 @@ def wht128(v: np.ndarray) -> np.ndarray:
     out = np.ascontiguousarray(v, dtype=np.float64).copy()
     assert out.shape == (D,)
     lib().or_wht128(_p(out))
+    return out
+
+
+def rope(x: np.ndarray, p: int, base: float) -> np.ndarray:
+    """The oracle's RoPE turn of one 128-vector to position p (rotate-half pairs (j, j + 64))."""
+    out = np.ascontiguousarray(x, dtype=np.float64).copy()
+    assert out.shape == (D,)
+    lib().or_rope(_p(out), int(p), float(base))
     return out
 
 
@@ -312,8 +325,10 @@ def encode_select(K: np.ndarray, V: np.ndarray, Q: np.ndarray, ctx_lens, n_kv_he
     return out
 
 
-def attend(units, q: np.ndarray, G: int, sm_scale: float, rot_seed: int, rotate: bool = True, lloyd: bool = False, sel=None) -> np.ndarray:
-    """q: uint16 bf16 bits [n_units][G][128] (or [B][H_q][128]); returns fp64 of the same shape."""
+def attend(units, q: np.ndarray, G: int, sm_scale: float, rot_seed: int, rotate: bool = True, lloyd: bool = False,
+           sel=None, rope_theta: float = 0.0) -> np.ndarray:
+    """q: uint16 bf16 bits [n_units][G][128] (or [B][H_q][128]); returns fp64 of the same shape.
+    rope_theta > 0: keys are pre-RoPE and each is turned to its position (unit.pos) first."""
     n = len(units)
     q = np.ascontiguousarray(q, dtype=np.uint16).reshape(n, G, D)
     out = np.zeros((n, G, D), np.float64)
@@ -324,12 +339,14 @@ def attend(units, q: np.ndarray, G: int, sm_scale: float, rot_seed: int, rotate:
         assert sel_arr.shape == (n,)
         selp = _p(sel_arr)
     lib().or_attend_batch(ctypes.cast(structs, ctypes.c_void_p), n, _p(q), G, float(sm_scale),
-                          ctypes.c_uint64(rot_seed), _flags(rotate, lloyd), selp, _p(out))
+                          ctypes.c_uint64(rot_seed), _flags(rotate, lloyd) | (4 if rope_theta > 0 else 0),
+                          float(rope_theta), selp, _p(out))
     return out
 
 
 def attend_suffix(units, q: np.ndarray, G: int, H: int, sm_scale: float, rot_seed: int, ksuf: np.ndarray,
-                  vsuf: np.ndarray, suf_len, rotate: bool = True, lloyd: bool = False) -> np.ndarray:
+                  vsuf: np.ndarray, suf_len, rotate: bool = True, lloyd: bool = False,
+                  rope_theta: float = 0.0) -> np.ndarray:
     """Attention over each unit's compressed positions and the first suf_len[b] rows of its exact
     dense suffix, in one softmax (Appendix E.1, E.2).  ksuf, vsuf: uint16 bf16 bits
     [n_units][cap][128] (unit u = b*H + h); suf_len: int [B].  Returns fp64 [n_units][G][128]."""
@@ -343,7 +360,8 @@ def attend_suffix(units, q: np.ndarray, G: int, H: int, sm_scale: float, rot_see
     out = np.zeros((n, G, D), np.float64)
     structs = (_OrUnit * n)(*[u.c_struct() for u in units])
     lib().or_attend_batch_suffix(ctypes.cast(structs, ctypes.c_void_p), n, H, _p(q), G, float(sm_scale),
-                                 ctypes.c_uint64(rot_seed), _flags(rotate, lloyd), _p(ksuf), _p(vsuf), _p(lens),
+                                 ctypes.c_uint64(rot_seed), _flags(rotate, lloyd) | (4 if rope_theta > 0 else 0),
+                                 float(rope_theta), _p(ksuf), _p(vsuf), _p(lens),
                                  int(ksuf.shape[1]), _p(out))
     return out
 

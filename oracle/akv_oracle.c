@@ -26,7 +26,8 @@
  *   attend  : Eq. 3 reconstruction of every key and value, then Eq. 4
  *             softmax attention, all in fp64, one token at a time; with an
  *             exact dense suffix (Appendix E.1 and E.2: generated tokens kept
- *             in bf16) the suffix tokens join the same softmax.
+ *             in bf16) the suffix tokens join the same softmax; with RoPE at
+ *             decode (Section 3.2) every key is turned to its position first.
  *   attend_factorized : the same attention regrouped by anchor (anchor
  *             scores computed once, value weights summed per anchor, inverse
  *             rotation applied once after accumulation -- Section 4.4 and
@@ -47,6 +48,7 @@
 /* Codec flags (the library's AKV_FLAG_ROTATE and AKV_FLAG_LLOYD bits). */
 #define OR_ROTATE 1
 #define OR_LLOYD 2
+#define OR_ROPE 4
 
 /* The four-level Lloyd-Max quantizer of a unit Gaussian source (Max 1960, the
  * codebook of Section 3.1 and Appendix A.1): levels -1.5104, -0.4528, 0.4528,
@@ -183,6 +185,7 @@ typedef struct or_unit {
   uint8_t* codes_v;
   uint16_t* scale_v;
   uint16_t* min_v;
+  int32_t* pos; /* [S] position of index i (RoPE at decode); NULL: position i */
 } or_unit;
 
 typedef struct {
@@ -481,6 +484,21 @@ void or_reconstruct_side(int32_t S, const uint16_t* anchors, const uint16_t* idx
   }
 }
 
+/* RoPE (Section 3.2: keys kept pre-RoPE, the rotation applied at decode): the
+ * rotate-half form, dimension pairs (j, j + 64) turned by the angle p theta_j
+ * with theta_j = base^(-2j/128):
+ *   y_j = x_j cos - x_{j+64} sin,   y_{j+64} = x_{j+64} cos + x_j sin. */
+void or_rope(double* x, int64_t p, double base) {
+  for (int j = 0; j < OR_D / 2; ++j) {
+    double th = pow(base, -2.0 * (double)j / (double)OR_D);
+    double a = (double)p * th;
+    double c = cos(a), sn = sin(a);
+    double x0 = x[j], x1 = x[j + OR_D / 2];
+    x[j] = x0 * c - x1 * sn;
+    x[j + OR_D / 2] = x1 * c + x0 * sn;
+  }
+}
+
 /* Definitional attention for one unit with an exact dense suffix: G query
  * rows (bf16 bits [G][128]), out [G][128] fp64.  Each key and value of the
  * S compressed positions is rebuilt per Eq. 3; the nsuf suffix tokens (bf16
@@ -488,7 +506,8 @@ void or_reconstruct_side(int32_t S, const uint16_t* anchors, const uint16_t* idx
  * softmax of Eq. 4 is taken over all S + nsuf positions at once (the combine
  * of Appendix E.1 attends both under the same softmax). */
 void or_attend_unit_suffix(const or_unit* u, const uint16_t* q, int32_t G, double sm_scale, uint64_t rot_seed,
-                           int flags, const uint16_t* ksuf, const uint16_t* vsuf, int32_t nsuf, double* out) {
+                           int flags, double rope_theta, const uint16_t* ksuf, const uint16_t* vsuf, int32_t nsuf,
+                           double* out) {
   int32_t S = u->S;
   int32_t n = S + nsuf; /* positions of the softmax */
   double s[OR_D];
@@ -515,6 +534,8 @@ void or_attend_unit_suffix(const or_unit* u, const uint16_t* q, int32_t G, doubl
     } else {
       for (int j = 0; j < OR_D; ++j) x[j] = or_bf16_to_double(ksuf[(size_t)(i - S) * OR_D + j]);
     }
+    if (flags & OR_ROPE) /* the key at its position: compressed i at pos[i], suffix t at S + t */
+      or_rope(x, i < S ? (u->pos ? u->pos[i] : i) : i, rope_theta);
     for (int32_t g = 0; g < G; ++g) {
       double d = 0.0;
       for (int j = 0; j < OR_D; ++j) d += qd[g][j] * x[j];
@@ -562,7 +583,7 @@ void or_attend_unit_suffix(const or_unit* u, const uint16_t* q, int32_t G, doubl
  * its S positions, each key and value rebuilt per Eq. 3. */
 void or_attend_unit(const or_unit* u, const uint16_t* q, int32_t G, double sm_scale, uint64_t rot_seed, int flags,
                     double* out) {
-  or_attend_unit_suffix(u, q, G, sm_scale, rot_seed, flags, NULL, NULL, 0, out);
+  or_attend_unit_suffix(u, q, G, sm_scale, rot_seed, flags, 0.0, NULL, NULL, 0, out);
 }
 
 /* ------------------------------------------------------------------------ */
@@ -959,11 +980,12 @@ int or_encode_select_batch(const uint16_t* K, const uint16_t* V, const uint16_t*
  * owns query heads h*G .. h*G+G-1 of request b), out fp64 same shape.
  * Units with sel[u] == 0 are skipped (sel may be NULL). */
 void or_attend_batch(const or_unit* units, int32_t n_units, const uint16_t* q, int32_t G, double sm_scale,
-                     uint64_t rot_seed, int flags, const uint8_t* sel, double* out) {
+                     uint64_t rot_seed, int flags, double rope_theta, const uint8_t* sel, double* out) {
 #pragma omp parallel for schedule(dynamic, 1)
   for (int32_t u = 0; u < n_units; ++u) {
     if (sel && !sel[u]) continue;
-    or_attend_unit(&units[u], q + (size_t)u * G * OR_D, G, sm_scale, rot_seed, flags, out + (size_t)u * G * OR_D);
+    or_attend_unit_suffix(&units[u], q + (size_t)u * G * OR_D, G, sm_scale, rot_seed, flags, rope_theta, NULL, NULL, 0,
+                          out + (size_t)u * G * OR_D);
   }
 }
 
@@ -971,12 +993,13 @@ void or_attend_batch(const or_unit* units, int32_t n_units, const uint16_t* q, i
  * S positions and the first suf_len[b] rows of its suffix block, rows
  * ksuf/vsuf + (u * suf_cap + t) * 128 (bf16). */
 void or_attend_batch_suffix(const or_unit* units, int32_t n_units, int32_t H, const uint16_t* q, int32_t G,
-                            double sm_scale, uint64_t rot_seed, int flags, const uint16_t* ksuf, const uint16_t* vsuf,
-                            const int32_t* suf_len, int32_t suf_cap, double* out) {
+                            double sm_scale, uint64_t rot_seed, int flags, double rope_theta, const uint16_t* ksuf,
+                            const uint16_t* vsuf, const int32_t* suf_len, int32_t suf_cap, double* out) {
 #pragma omp parallel for schedule(dynamic, 1)
   for (int32_t u = 0; u < n_units; ++u) {
     const size_t base = (size_t)u * (size_t)suf_cap * OR_D;
-    or_attend_unit_suffix(&units[u], q + (size_t)u * G * OR_D, G, sm_scale, rot_seed, flags, ksuf + base, vsuf + base,
+    or_attend_unit_suffix(&units[u], q + (size_t)u * G * OR_D, G, sm_scale, rot_seed, flags, rope_theta, ksuf + base,
+                          vsuf + base,
                           suf_len[u / H], out + (size_t)u * G * OR_D);
   }
 }
@@ -1072,9 +1095,9 @@ void or_attend_factorized(const or_unit* u, const uint16_t* q, int32_t G, double
 /* Header: magic u32 @0, version u32 @4, total_bytes u64 @8, params (56 B) @16,
  * n_units i32 @72, max_len i32 @76, desc_offset u64 @80, sign bits 2 x u64 @88.
  * Descriptor (256 B each at desc_offset + 256 u): len, k, n_res_k, n_res_v,
- * n_words, b, h, reserved (i32 each), then u64 offsets: anchor_k, anchor_v,
- * anchor_pos, stream_k, stream_v, bitmap_k, prefix_k, bitmap_v, prefix_v,
- * codes_k, scales_k, codes_v, scales_v, then data_bytes. */
+ * n_tiles, b, h, reserved (i32 each), then u64: offsets of anchor_k, anchor_v,
+ * anchor_pos, tile table, tile blocks; tiles capacity, data_bytes, and the
+ * offset of the positions (RoPE arenas). */
 static uint32_t rd32(const uint8_t* p) {
   uint32_t v;
   memcpy(&v, p, 4);
@@ -1088,7 +1111,7 @@ static uint64_t rd64(const uint8_t* p) {
 
 /* Returns 0 and the shape of unit u, or -1 on a malformed arena. */
 int or_arena_shape(const uint8_t* arena, uint64_t bytes, int32_t u, int32_t* shape4) {
-  if (bytes < 256 || rd32(arena) != 0x32564B41u || rd32(arena + 4) != 3u || rd32(arena + 104) != 1024u) return -1;
+  if (bytes < 256 || rd32(arena) != 0x32564B41u || rd32(arena + 4) != 4u || rd32(arena + 104) != 1024u) return -1;
   int32_t n_units = (int32_t)rd32(arena + 72);
   uint64_t doff = rd64(arena + 80);
   if (u < 0 || u >= n_units || doff + 256ull * (uint64_t)(u + 1) > bytes) return -1;
@@ -1200,5 +1223,24 @@ int or_arena_unpack(const uint8_t* arena, uint64_t bytes, int32_t u, or_unit* ou
     cnt[1] += m[1];
   }
   if (cnt[0] != nk || cnt[1] != nv) return -1;
+  /* RoPE arenas (flags @64 of the header) keep each stored token's original position: a
+   * permutation of 0 .. S-1, ascending among the tokens of one value slot (the stable sort) */
+  if (rd32(arena + 64) & OR_ROPE) {
+    uint64_t o_pos = rd64(d + 88);
+    if (o_pos == 0 || o_pos + 4ull * S > bytes) return -1;
+    uint8_t* seen = (uint8_t*)calloc((size_t)S, 1);
+    int bad = 0;
+    for (int32_t i = 0; i < S && !bad; ++i) {
+      uint32_t p = rd32(arena + o_pos + 4ull * i);
+      if (p >= (uint32_t)S || seen[p]) bad = 1;
+      else seen[p] = 1;
+      if (!bad && i > 0 && out->idx_v[i] == out->idx_v[i - 1] && p <= rd32(arena + o_pos + 4ull * (i - 1))) bad = 1;
+      if (!bad && out->pos) out->pos[i] = (int32_t)p;
+    }
+    free(seen);
+    if (bad) return -1;
+  } else if (out->pos) {
+    for (int32_t i = 0; i < S; ++i) out->pos[i] = -1; /* positions are not stored */
+  }
   return 0;
 }

@@ -20,6 +20,7 @@ LIB_PATH = os.path.join(_HERE, "libakv.so")
 AKV_OK, AKV_ERR_INVALID, AKV_ERR_UNSUPPORTED, AKV_ERR_TOO_SMALL, AKV_ERR_CUDA = range(5)
 AKV_FLAG_ROTATE = 1
 AKV_FLAG_LLOYD = 2
+AKV_FLAG_ROPE = 4
 HEAD_DIM = 128
 
 EXPORTED = (
@@ -42,7 +43,7 @@ class _Params(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32), ("n_q_heads", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32), ("anchor_frac", ctypes.c_float), ("res_frac_k", ctypes.c_float),
                 ("res_frac_v", ctypes.c_float), ("window", ctypes.c_int32), ("seed", ctypes.c_uint64),
-                ("rot_seed", ctypes.c_uint64), ("flags", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+                ("rot_seed", ctypes.c_uint64), ("flags", ctypes.c_uint32), ("rope_theta", ctypes.c_float)]
 
 
 class _SelectParams(ctypes.Structure):
@@ -86,6 +87,8 @@ class Params:
     rotate: bool = True
     head_dim: int = HEAD_DIM
     lloyd: bool = False  # the Lloyd-Max residual codec (AKV_FLAG_LLOYD) instead of the uniform one
+    rope: bool = False  # pre-RoPE keys, RoPE applied at decode (AKV_FLAG_ROPE)
+    rope_theta: float = 500000.0
 
     @property
     def G(self) -> int:
@@ -99,7 +102,8 @@ class Params:
         return _Params(self.batch, self.n_kv_heads, self.n_q_heads, self.head_dim, self.anchor_frac,
                        self.res_frac_k, self.res_frac_v, self.window, self.seed & (2**64 - 1),
                        self.rot_seed & (2**64 - 1),
-                       (AKV_FLAG_ROTATE if self.rotate else 0) | (AKV_FLAG_LLOYD if self.lloyd else 0), 0)
+                       (AKV_FLAG_ROTATE if self.rotate else 0) | (AKV_FLAG_LLOYD if self.lloyd else 0) |
+                       (AKV_FLAG_ROPE if self.rope else 0), float(self.rope_theta) if self.rope else 0.0)
 
 
 _lib = None
@@ -305,7 +309,7 @@ _DECODE_ARGS: dict = {}
 
 def _decode_args(p: Params, ctx_lens):
     key = (p.batch, p.n_kv_heads, p.n_q_heads, p.head_dim, p.anchor_frac, p.res_frac_k, p.res_frac_v, p.window,
-           p.seed, p.rot_seed, p.rotate, p.lloyd, tuple(int(x) for x in ctx_lens))
+           p.seed, p.rot_seed, p.rotate, p.lloyd, p.rope, p.rope_theta, tuple(int(x) for x in ctx_lens))
     ent = _DECODE_ARGS.get(key)
     if ent is None:
         if len(_DECODE_ARGS) >= 64:

@@ -50,7 +50,9 @@ akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out
   if (!frac_ok(p->anchor_frac) || !frac_ok(p->res_frac_k) || !frac_ok(p->res_frac_v))
     return fail(AKV_ERR_INVALID, "fractions must be finite and in [0, 1]");
   if (p->window < 0) return fail(AKV_ERR_INVALID, "window must be >= 0");
-  if (p->reserved != 0 || (p->flags & ~(AKV_FLAG_ROTATE | AKV_FLAG_LLOYD)) != 0) return fail(AKV_ERR_INVALID, "unknown flags");
+  if ((p->flags & ~(AKV_FLAG_ROTATE | AKV_FLAG_LLOYD | AKV_FLAG_ROPE)) != 0) return fail(AKV_ERR_INVALID, "unknown flags");
+  if ((p->flags & AKV_FLAG_ROPE) ? !(std::isfinite(p->rope_theta) && p->rope_theta > 1.0f) : p->rope_theta != 0.0f)
+    return fail(AKV_ERR_INVALID, "rope_theta must be finite and > 1 with AKV_FLAG_ROPE, and 0 without it");
   if (sel) {
     if (!(std::isfinite(sel->theta) && sel->theta > 0.0f && sel->theta <= 1.0f))
       return fail(AKV_ERR_INVALID, "theta must be in (0, 1]");
@@ -123,6 +125,12 @@ akv_status make_layout(const akv_params* p, const int32_t* ctx_lens, Layout* out
       }
       d.tiles_capacity = cap;
       d.data_bytes = sizes[kAnchorK] + sizes[kAnchorV] + sizes[kTileTable] + cap;
+      if (p->flags & AKV_FLAG_ROPE) {  // original positions of the stored tokens
+        off = align_up(off, kSectionAlign);
+        d.off_pos = off;
+        off += (uint64_t)S * 4;
+        d.data_bytes += (uint64_t)S * 4;
+      }
       if (nt > L.max_tiles) L.max_tiles = nt;
       if (S > L.max_len) L.max_len = S;
       if (k > L.max_k) L.max_k = (int32_t)k;
@@ -324,6 +332,7 @@ akv_status akv_cache_pack_host(const akv_params* p, const int32_t* ctx_lens_host
     for (int32_t i = 0; i < S; ++i) ++start[(size_t)in.idx_v[i] + 1];
     for (int32_t a = 0; a < k; ++a) start[(size_t)a + 1] += start[(size_t)a];
     for (int32_t i = 0; i < S; ++i) perm[(size_t)start[in.idx_v[i]]++] = i;
+    if (d.off_pos) std::memcpy(A + d.off_pos, perm.data(), (size_t)S * 4);  // position of each stored token
     // tile blocks
     uint32_t* table = (uint32_t*)(A + d.off_tile_table);
     uint8_t* tiles = A + d.off_tiles;
@@ -517,6 +526,8 @@ akv_status akv_decode_attn_suffix(const akv_params* p, const int32_t* ctx_lens_h
   if (arena_bytes < L.total_bytes) return fail(AKV_ERR_TOO_SMALL, "arena shorter than akv_cache_size");
   if (!std::isfinite(sm_scale)) return fail(AKV_ERR_INVALID, "sm_scale must be finite");
   DecodeSuffix sfx;
+  if (suffix && (p->flags & AKV_FLAG_ROPE))
+    return fail(AKV_ERR_UNSUPPORTED, "a dense suffix with RoPE at decode is not supported");
   if (suffix) {
     if (!suffix->K || !suffix->V || !suffix->len) return fail(AKV_ERR_INVALID, "suffix: null K, V or len");
     if (((uintptr_t)suffix->K % 16) || ((uintptr_t)suffix->V % 16) || ((uintptr_t)suffix->len % 4))

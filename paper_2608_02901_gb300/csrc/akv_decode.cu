@@ -48,6 +48,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
 #include <atomic>
 #include <cstdio>
 #include <cstdlib>
@@ -116,6 +117,19 @@ struct ScoreParams {
   int suf_cap, n_sch;
 };
 
+// The RoPE logits launch (AKV_FLAG_ROPE): every stored token's logit per head.
+struct RopeParams {
+  const uint8_t* arena;
+  const __nv_bfloat16* q;
+  float* lg;      // [units][s_stride][G] logits (log2 units, sm_scale folded in), stored order
+  float* cmax;    // [units][n_tch][G] largest logit of each chunk of 64 stored tokens
+  unsigned* cnt;  // [units] arrival counters of the decode launch, zeroed here
+  int n_kv_heads, n_q_heads, rotate, lloyd, s_stride, n_tch;
+  float scale_log2;
+  unsigned long long sign_lo, sign_hi;
+  unsigned long long turn[64];  // theta_j / (2 pi) as a 64-bit binary fraction of a turn
+};
+
 struct Meta {  // a staged tile, as the producer recorded it
   uint32_t ring_off, blk_off, blk_bytes, staged, lo, nrows, j, pad;
 };
@@ -141,6 +155,8 @@ struct DecodeParams {
   int ring_bytes, drop_last, smem_sa;
   int o_bar, o_meta, o_misc, o_sa, o_ovf, o_grp, grp_bytes, o_ring;
   int g_qp, g_rows, g_red, g_wb, g_pv, g_qf;  // offsets inside a group's block
+  const float* lg;         // RoPE at decode: logits [units][s_stride][G] in stored order (else null)
+  int s_stride;
   const float* suf_part;   // dense suffix partials [units][n_sch][suf_floats] (null: no suffix)
   const int32_t* suf_len;  // suffix tokens per request
   int suf_cap, n_sch;
@@ -871,6 +887,169 @@ __device__ __forceinline__ void head_probs(float gk, const float (&sa)[GS], cons
   }
 }
 
+// ============================ RoPE at decode (AKV_FLAG_ROPE) ============================
+// Keys are stored pre-RoPE, so a token's score no longer factors through its anchor's score:
+// q . R(p_i) x^_i with x^_i = gamma_i x_a(i) + r~_i (Eq. 3) and R(p) the rotate-half RoPE turn
+// of dimension pairs (j, j + 64) by p theta_j (Section 3.2; Appendix E.1's score kernel rebuilds
+// keys and applies RoPE from the stored positions the same way).  CTA (unit u, chunk c): stored
+// tokens 64 c .. 64 c + 63; warp w rebuilds tokens 16 w .. 16 w + 15, lane l holding dimensions
+// 4 l .. 4 l + 3 (pair partners sit 16 lanes apart), into shared memory; then thread t sums
+// q_g . y over one half of the dimensions of token t % 64 for every head g.  The angle of pair j
+// at position p is taken as a binary fraction of a turn, p * turn_j mod 2^64 (exact integer
+// arithmetic), so the sine and cosine are evaluated on [0, 2 pi) whatever the position.
+template <int GS>
+__global__ void __launch_bounds__(128) akv_rope_logits_kernel(const RopeParams P) {
+  __shared__ __align__(16) float ys[64][132];  // rows 16-byte aligned; 128-bit reads conflict-free
+  __shared__ __align__(16) float qsm[8][128];
+  __shared__ float part[2][64][8];
+  __shared__ float wmx[2][8];
+  __shared__ unsigned long long turn[64];
+  const int u = blockIdx.x / P.n_tch, c = blockIdx.x % P.n_tch;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const akv_unit_desc* d = unit_desc(P.arena, u);
+  const int S = d->len, k = d->n_anchors;
+  if (c == 0 && tid == 0) P.cnt[u] = 0u;
+  const int ts0 = 64 * c;
+  if (ts0 >= S) return;  // past this unit's end (a shorter request)
+  const size_t qb = qrow_base(u, P.n_kv_heads, P.n_q_heads);
+  for (int e = tid; e < GS * 128; e += 128) qsm[e / 128][e % 128] = __bfloat162float(P.q[qb + e]);
+  if (tid < 64) turn[tid] = P.turn[tid];
+  // the chunk inside its tile block: one bitmap word (64 tokens) per side
+  const int j = ts0 / T, tl0 = ts0 % T;
+  const int n = min(T, S - j * T), nw = (int)tile_words(n), n64 = 64 * nw;
+  const uint8_t* blk = P.arena + d->off_tiles + reinterpret_cast<const uint32_t*>(P.arena + d->off_tile_table)[j];
+  const uint64_t* bm = reinterpret_cast<const uint64_t*>(blk + 8 * n64);
+  const uint16_t* rkk = reinterpret_cast<const uint16_t*>(blk + 8 * n64 + 16 * nw);
+  const uint16_t* rkv = reinterpret_cast<const uint16_t*>(blk + 8 * n64 + 16 * nw + round16(2u * nw));
+  const int nk = rkk[nw - 1] + __popcll(bm[nw - 1]), nv = rkv[nw - 1] + __popcll(bm[nw + nw - 1]);
+  const uint32_t F = tile_fixed_bytes(n);
+  const uint32_t sm_k = F, cd_k = F + round16(4u * (uint32_t)nk) + round16(4u * (uint32_t)nv);
+  const uint64_t word = bm[tl0 / 64];
+  const int rbase = rkk[tl0 / 64];
+  const uint8_t* AK = P.arena + d->off_anchor_k;
+  const uint32_t* pos = reinterpret_cast<const uint32_t*>(P.arena + d->off_pos);
+  __syncthreads();
+  // the warp's 16 tokens: lane i < 16 fetches token i's stream word and position; every lane then
+  // loads its 8 bytes of all 16 anchor rows, and the records of the tokens with a residual, before
+  // any arithmetic (the loads do not wait on one another)
+  const int tw = tl0 + 16 * warp;
+  const int nwt = max(0, min(16, n - tw));  // the warp's tokens inside the tile
+  uint32_t ek_l = 0u, pos_l = 0u;
+  if (lane < nwt) {
+    ek_l = reinterpret_cast<const uint32_t*>(blk)[tw + lane];
+    pos_l = pos[j * T + tw + lane];
+  }
+  uint2 xa[16];
+  uint32_t smn[16], cbyte[16];
+  const uint32_t wbits = (uint32_t)(word >> (tw % 64)) & 0xFFFFu;  // residual flags of the 16 tokens
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const uint32_t ek = __shfl_sync(0xffffffffu, ek_l, i);
+    const int a = min((int)(ek & 0xFFFFu), k - 1);
+    xa[i] = i < nwt ? *reinterpret_cast<const uint2*>(AK + (size_t)a * 256 + 16 * ((lane >> 1) ^ (a & 7)) + 8 * (lane & 1))
+                    : make_uint2(0u, 0u);
+    smn[i] = 0u;
+    cbyte[i] = 0u;
+    if (i < nwt && ((wbits >> i) & 1u)) {
+      const int r = rbase + __popcll(word & ((1ull << ((tw % 64) + i)) - 1ull));
+      smn[i] = *reinterpret_cast<const uint32_t*>(blk + sm_k + 4u * (uint32_t)r);
+      cbyte[i] = blk[cd_k + 32u * (uint32_t)r + (uint32_t)lane];
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {  // (fully unrolled: the per-token arrays stay in registers)
+    float y[4] = {0.f, 0.f, 0.f, 0.f};
+    const uint32_t ek = __shfl_sync(0xffffffffu, ek_l, i);
+    const uint32_t p = __shfl_sync(0xffffffffu, pos_l, i);
+    if (i < nwt) {  // (the same for the whole warp)
+      const float gk = half_hi(ek);
+      float x[4];
+      x[0] = gk * __bfloat162float(__ushort_as_bfloat16((unsigned short)(xa[i].x & 0xFFFFu)));
+      x[1] = gk * __bfloat162float(__ushort_as_bfloat16((unsigned short)(xa[i].x >> 16)));
+      x[2] = gk * __bfloat162float(__ushort_as_bfloat16((unsigned short)(xa[i].y & 0xFFFFu)));
+      x[3] = gk * __bfloat162float(__ushort_as_bfloat16((unsigned short)(xa[i].y >> 16)));
+      if ((wbits >> i) & 1u) {  // plus r~ = s o H(c^) / 128, c^ = min + scale L[code] (warp-uniform)
+        float cr[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          cr[e] = fmaf(half_lo(smn[i]), code_level((cbyte[i] >> (2 * e)) & 3u, P.lloyd), half_hi(smn[i]));
+        if (P.rotate) {
+          warp_wht128(cr, lane);
+          apply_signs(cr, lane, P.sign_lo, P.sign_hi);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) cr[e] *= (1.0f / 128.0f);
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) x[e] += cr[e];
+      }
+      // RoPE at the token's position: lanes 0-15 hold dims j < 64, lanes 16-31 their partners j + 64;
+      // the two halves each evaluate two of the four pairs' angles and trade them
+      float sn[4], cs[4];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int e = (lane < 16 ? 0 : 2) + h;
+        const unsigned long long ph = (unsigned long long)p * turn[(4 * lane + e) & 63];
+        __sincosf((float)(ph >> 40) * (6.2831853071795865f / 16777216.0f), &sn[e], &cs[e]);
+        const int eo = (lane < 16 ? 2 : 0) + h;
+        sn[eo] = 0.f;
+        cs[eo] = 0.f;
+      }
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {  // lanes < 16 receive pairs 2, 3; lanes >= 16 pairs 0, 1
+        const float so = __shfl_xor_sync(0xffffffffu, lane < 16 ? sn[h] : sn[2 + h], 16);
+        const float co = __shfl_xor_sync(0xffffffffu, lane < 16 ? cs[h] : cs[2 + h], 16);
+        if (lane < 16) {
+          sn[2 + h] = so;
+          cs[2 + h] = co;
+        } else {
+          sn[h] = so;
+          cs[h] = co;
+        }
+      }
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float xp = __shfl_xor_sync(0xffffffffu, x[e], 16);
+        y[e] = lane < 16 ? fmaf(x[e], cs[e], -xp * sn[e]) : fmaf(x[e], cs[e], xp * sn[e]);
+      }
+    }
+    *reinterpret_cast<float4*>(&ys[16 * warp + i][4 * lane]) = make_float4(y[0], y[1], y[2], y[3]);
+  }
+  __syncthreads();
+  // thread t: token t % 64, dimensions 64 (t / 64) .. + 63, every head
+  {
+    const int tk = tid & 63, hf = tid >> 6;
+    float acc[GS];
+#pragma unroll
+    for (int g = 0; g < GS; ++g) acc[g] = 0.f;
+#pragma unroll 4
+    for (int dd = 0; dd < 64; dd += 4) {
+      const float4 yv = *reinterpret_cast<const float4*>(&ys[tk][64 * hf + dd]);
+#pragma unroll
+      for (int g = 0; g < GS; ++g) {
+        const float4 qv = *reinterpret_cast<const float4*>(&qsm[g][64 * hf + dd]);  // (the same for the warp)
+        acc[g] = fmaf(yv.x, qv.x, fmaf(yv.y, qv.y, fmaf(yv.z, qv.z, fmaf(yv.w, qv.w, acc[g]))));
+      }
+    }
+#pragma unroll
+    for (int g = 0; g < GS; ++g) part[hf][tk][g] = acc[g];
+  }
+  __syncthreads();
+  if (tid < 64) {
+    const bool ok = ts0 + tid < S;
+    float* dst = P.lg + ((size_t)u * P.s_stride + ts0 + tid) * GS;
+#pragma unroll
+    for (int g = 0; g < GS; ++g) {
+      const float l = (part[0][tid][g] + part[1][tid][g]) * P.scale_log2;
+      if (ok) dst[g] = l;
+      float m = ok ? l : -INFINITY;
+      m = warp_max(m);
+      if (lane == 0) wmx[warp][g] = m;
+    }
+  }
+  __syncthreads();
+  if (tid < GS) P.cmax[((size_t)u * P.n_tch + c) * GS + tid] = fmaxf(wmx[0][tid], wmx[1][tid]);
+}
+
 // A lane's tokens of a tile: bitmap bytes and first record indices.
 struct TokLane {
   uint32_t kbits, vbits;
@@ -887,6 +1066,7 @@ struct TokTile {
   float* W;           // [X][GS] the tile's value weights
   float* ovf;         // [2][GS][128] overflow sums
   const uint8_t* AV;  // the unit's anchor values (global)
+  const float* lgt;   // RoPE at decode: the tile's logit rows [T][GS] (global), else null
   int k, nKs, nVs, ka, lloyd;
 };
 
@@ -921,6 +1101,7 @@ __device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const
   float* pv = tt.pv;
   float* ovf = tt.ovf;
   const uint8_t* AV = tt.AV;
+  const float* lgt = tt.lgt;
   const int k = tt.k, nKs = tt.nKs, nVs = tt.nVs, ka = tt.ka, lloyd = tt.lloyd;
   const uint32_t lo = tt.lo;
   const int nrows = (int)tt.nrows;
@@ -951,11 +1132,22 @@ __device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const
     const uint32_t ev = e < nvalid ? *reinterpret_cast<const uint32_t*>(st + 4 * (tv.n64 + t0 + e)) : 0u;
     const int a = min((int)(ek & 0xFFFFu), k - 1);
     float sa[GS], rt[GS];
-    load_sa_row<GS>(SAt, a, ka, sa);
+    if (lgt) {  // RoPE: the token's logits (no anchor-score table)
+#pragma unroll
+      for (int g = 0; g < GS; ++g) sa[g] = 0.f;
+    } else {
+      load_sa_row<GS>(SAt, a, ka, sa);
+    }
     const bool kb = (kbits >> e) & 1u;
     const int r = rkn;
     rkn += (int)kb;
-    if (kb && r >= nKs && e < nvalid) {  // beyond the staged records
+    if (lgt) {  // RoPE: the logits minus m, or -inf for a token past the tile's end
+      load_row<GS>(e >= nvalid ? ninfrow : negrow, rt);
+      if (e < nvalid) {
+#pragma unroll
+        for (int g = 0; g < GS; ++g) rt[g] += lgt[(t0 + e) * GS + g];
+      }
+    } else if (kb && r >= nKs && e < nvalid) {  // beyond the staged records
 #pragma unroll
       for (int g = 0; g < GS; ++g)
         rt[g] = key_record_term(st, gb, staged, tv.sm_k + 4u * (uint32_t)r, tv.cd_k + 32u * (uint32_t)r, qp + g * 128,
@@ -970,7 +1162,7 @@ __device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const
         for (int g = 0; g < GS; ++g) rt[g] += rs[g];
       }
     }
-    const float gk = half_hi(ek), gv = half_hi(ev);
+    const float gk = lgt ? 0.f : half_hi(ek), gv = half_hi(ev);
     float2 pe[NP];
     head_probs<GS, NP>(gk, sa, rt, pe, l2);
     const bool vb = (vbits >> e) & 1u;
@@ -1007,7 +1199,9 @@ __device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const
 
 // ================================ decode ============================================
 // CODEC: 0 = uniform codes (c^ = min + c scale), 1 = Lloyd-Max levels (c^ = scale L[c]).
-template <int GS, int CODEC>
+// ROPE: 1 = pre-RoPE keys: every token's logit comes from the RoPE logits launch (P.lg) instead
+// of gamma S_A plus its key-residual term; the key-residual phase has nothing to do.
+template <int GS, int CODEC, int ROPE>
 __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P) {
   extern __shared__ __align__(128) uint8_t smem[];
   constexpr int NP = GS >= 2 ? GS / 2 : 1;      // pairs of heads for the packed arithmetic
@@ -1203,7 +1397,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     // the score kernel) by one bulk copy; meanwhile the reference m of each head from the chunk
     // maxima (warp wg: heads wg, wg + 4) ----
     if (wg == 0 && lane == 0) {
-      if (!*failed) {
+      if (!*failed && !ROPE) {  // (RoPE: no key-side header is needed)
         mbar_expect_tx(bar_hdr(grp), (uint32_t)hdr_bytes(GS));
         bulk_g2s(smem_u32(qp), P.uh + (size_t)sg.u * P.uh_stride, (uint32_t)hdr_bytes(GS), bar_hdr(grp));
       } else {
@@ -1212,7 +1406,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
     }
     for (int g = wg; g < GS; g += WPG) {
       float m = -INFINITY;
-      const int nch = (k + CHA - 1) / CHA;
+      // the largest anchor score (a lower bound of the largest logit), or with RoPE the largest logit
+      const int nch = ROPE ? (U.S + 63) / 64 : (k + CHA - 1) / CHA;
       for (int ch = lane; ch < nch; ch += 32) m = fmaxf(m, P.cmax[((size_t)sg.u * P.n_ch + ch) * GS + g]);
       m = warp_max(m);
       if (lane == 0) {
@@ -1253,9 +1448,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
       if (go) {
         tv = tile_view(st, mt, U);
         const uint32_t codes_staged = tv.staged > tv.cd_k ? (tv.staged - tv.cd_k) / 32u : 0u;
-        nKs = min(tv.nk, (int)codes_staged);  // their terms go over their own codes: no cap but staging
+        nKs = ROPE ? 0 : min(tv.nk, (int)codes_staged);  // their terms go over their own codes: no cap but staging
         nVs = min(tv.nv, P.R);
-        fast_tile = nKs == tv.nk && nVs == tv.nv &&
+        fast_tile = (ROPE || nKs == tv.nk) && nVs == tv.nv &&
                     (int)(((reinterpret_cast<const uint32_t*>(st + 4 * tv.n64))[tv.n - 1] & 0xFFFFu) - mt.lo) < (int)mt.nrows;
         for (int e = gt; e < P.X * GS; e += WPG * 32) W[e] = 0.f;
         // ---- key residuals: q' . c of the staged key records, tensor cores; the terms
@@ -1359,6 +1554,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 #pragma unroll
           for (int i2 = 0; i2 < NP; ++i2) negm2[i2] = make_float2(rows[2 * i2], GS >= 2 ? rows[2 * i2 + 1] : 0.f);
           constexpr int TPI = 4;  // stream words per load (16 bytes)
+          // RoPE: the lane's tokens' logit rows (global, stored order)
+          const float* lgt = ROPE ? P.lg + ((size_t)sg.u * P.s_stride + (size_t)mt.j * T + t0) * GS : nullptr;
           // the table pointer as shared memory (32-bit addressing, shared loads) or global memory
           auto token_loop = [&](const float* SAtab) {
 #pragma unroll 1
@@ -1368,25 +1565,35 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             load_words<TPI>(st + 4 * (tv.n64 + t0 + TPI * qd), ev);
 #pragma unroll
             for (int e = 0; e < TPI; ++e) {
-              const int a = min((int)(ek[e] & 0xFFFFu), km1);  // indices are < k by construction
-              float sa[GS];
-              load_sa_row<GS>(SAtab, a, P.ka_stride, sa);
-              const bool kb = kb8 & 1u;
-              kb8 >>= 1;
-              const float gk = half_hi(ek[e]), gv = half_hi(ev[e]);
-              // logits gamma S_A - m, plus the key-residual term for the lanes whose token has one
+              const float gv = half_hi(ev[e]);
               float2 x[NP];
-              const float2 gk2 = make_float2(gk, gk);
+              if constexpr (ROPE) {  // the token's logits from the RoPE logits launch, minus m
+                float lr[GS];
+                load_row<GS>(lgt + (TPI * qd + e) * GS, lr);
 #pragma unroll
-              for (int i2 = 0; i2 < NP; ++i2)
-                x[i2] = __ffma2_rn(gk2, make_float2(sa[2 * i2], GS >= 2 ? sa[2 * i2 + 1] : 0.f), negm2[i2]);
-              if (kb) {
-                float rs[GS];
-                load_row<GS>(rsb + rk * 8, rs);
+                for (int i2 = 0; i2 < NP; ++i2)
+                  x[i2] = __fadd2_rn(make_float2(lr[2 * i2], GS >= 2 ? lr[2 * i2 + 1] : 0.f), negm2[i2]);
+              } else {
+                const int a = min((int)(ek[e] & 0xFFFFu), km1);  // indices are < k by construction
+                float sa[GS];
+                load_sa_row<GS>(SAtab, a, P.ka_stride, sa);
+                const bool kb = kb8 & 1u;
+                kb8 >>= 1;
+                const float gk = half_hi(ek[e]);
+                // logits gamma S_A - m, plus the key-residual term for the lanes whose token has one
+                const float2 gk2 = make_float2(gk, gk);
 #pragma unroll
-                for (int i2 = 0; i2 < NP; ++i2) x[i2] = __fadd2_rn(x[i2], make_float2(rs[2 * i2], GS >= 2 ? rs[2 * i2 + 1] : 0.f));
+                for (int i2 = 0; i2 < NP; ++i2)
+                  x[i2] = __ffma2_rn(gk2, make_float2(sa[2 * i2], GS >= 2 ? sa[2 * i2 + 1] : 0.f), negm2[i2]);
+                if (kb) {
+                  float rs[GS];
+                  load_row<GS>(rsb + rk * 8, rs);
+#pragma unroll
+                  for (int i2 = 0; i2 < NP; ++i2)
+                    x[i2] = __fadd2_rn(x[i2], make_float2(rs[2 * i2], GS >= 2 ? rs[2 * i2 + 1] : 0.f));
+                }
+                rk += (int)kb;
               }
-              rk += (int)kb;
               float2 pe[NP];
 #pragma unroll
               for (int i2 = 0; i2 < NP; ++i2) {
@@ -1416,8 +1623,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             }
           }
           };
-          if (P.smem_sa) token_loop(SAs);
-          else token_loop(P.sa + (size_t)sg.u * P.ka_stride * GS);
+          if (ROPE || !P.smem_sa) token_loop(P.sa + (size_t)sg.u * P.ka_stride * GS);  // (RoPE: no table read)
+          else token_loop(SAs);
           // merge across lanes: the next lane's head continues this lane's last run when their
           // slots match; a head that does not continue the previous lane's run is complete
           const uint32_t ptk = __shfl_up_sync(0xffffffffu, key, 1);
@@ -1465,7 +1672,9 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
             }
           }
         } else if (t0 < tv.n) {
-          const auto ls = token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, U.AV, k, nKs, nVs, P.ka_stride, CODEC}, tl);
+          const auto ls = token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, U.AV,
+                                                      ROPE ? P.lg + ((size_t)sg.u * P.s_stride + (size_t)mt.j * T) * GS : nullptr,
+                                                      k, nKs, nVs, P.ka_stride, CODEC}, tl);
 #pragma unroll
           for (int i2 = 0; i2 < NP; ++i2) l2[i2] = __fadd2_rn(l2[i2], ls.v[i2]);
         }
@@ -1771,10 +1980,11 @@ bool make_plan_rx(const Layout& L, int GS, int R, int X, bool smem_sa, int smem_
 // counts trimmed from their full values towards the mean (records first, then anchor-value
 // rows: a run beyond those takes the slowest fallback); then the table in global memory
 // (gathers through L1 and L2) the same way; then anything that holds one tile per group.
-bool make_plan(const Layout& L, int GS, int smem_optin, Plan* out, std::string* why) {
+// table false: no anchor-score table is read (RoPE at decode), so none is placed in shared memory.
+bool make_plan(const Layout& L, int GS, int smem_optin, bool table, Plan* out, std::string* why) {
   const int R0 = full_r(L), X0 = full_x(L);
   const int Rmin = std::max(16, ((R0 * 3 / 4) + 15) & ~15), Xmin = std::max(16, ((X0 * 3 / 4) + 15) & ~15);
-  for (int sa = 1; sa >= 0; --sa)
+  for (int sa = table ? 1 : 0; sa >= 0; --sa)
     for (int min_tiles : {2, 1})
       for (int X = X0; X >= Xmin; X -= 16)
         for (int R = R0; R >= Rmin; R -= 16)
@@ -1789,9 +1999,15 @@ bool make_plan(const Layout& L, int GS, int smem_optin, Plan* out, std::string* 
 
 using DecodeFn = void (*)(const DecodeParams);
 using ScoreFn = void (*)(const ScoreParams);
+using RopeFn = void (*)(const RopeParams);
 template <int GS>
-DecodeFn decode_kernel(int codec) {
-  return codec ? akv_decode_kernel<GS, 1> : akv_decode_kernel<GS, 0>;
+DecodeFn decode_kernel(int codec, int rope) {
+  if (rope) return codec ? akv_decode_kernel<GS, 1, 1> : akv_decode_kernel<GS, 0, 1>;
+  return codec ? akv_decode_kernel<GS, 1, 0> : akv_decode_kernel<GS, 0, 0>;
+}
+template <int GS>
+RopeFn rope_kernel() {
+  return akv_rope_logits_kernel<GS>;
 }
 template <int GS>
 ScoreFn score_kernel() {
@@ -1801,11 +2017,11 @@ ScoreFn score_kernel() {
 // Launch configuration per (device, G, layout shape): computed once, then reused, so that a
 // call made during CUDA-graph capture only issues the launches.
 struct LaunchKey {
-  int dev, G, codec, units, max_len, max_k, ctas;
+  int dev, G, codec, rope, units, max_len, max_k, ctas;
   long long dens_key, adens_key, ttot;
   bool operator<(const LaunchKey& o) const {
-    return std::tie(dev, G, codec, units, max_len, max_k, ctas, dens_key, adens_key, ttot) <
-           std::tie(o.dev, o.G, o.codec, o.units, o.max_len, o.max_k, o.ctas, o.dens_key, o.adens_key, o.ttot);
+    return std::tie(dev, G, codec, rope, units, max_len, max_k, ctas, dens_key, adens_key, ttot) <
+           std::tie(o.dev, o.G, o.codec, o.rope, o.units, o.max_len, o.max_k, o.ctas, o.dens_key, o.adens_key, o.ttot);
   }
 };
 
@@ -1834,9 +2050,13 @@ DecodeWs decode_ws_layout(const Layout& L, int32_t suffix_cap) {
     off = (off + bytes + 255) & ~(size_t)255;
     return o;
   };
-  w.o_sa = take(units * ka * (size_t)L.G * 4);
+  const bool rope = (L.header.params.flags & AKV_FLAG_ROPE) != 0;
+  const size_t s_stride = (size_t)((L.max_len + 63) & ~63);
+  w.o_sa = take(rope ? 0 : units * ka * (size_t)L.G * 4);
   w.o_uh = take(units * (size_t)((hdr_bytes(L.G) + 255) & ~255));
-  w.o_cmax = take(units * nch * (size_t)L.G * 4);
+  // chunk maxima: of 64 anchors, or with RoPE of 64 stored tokens
+  w.o_cmax = take(units * (rope ? s_stride / 64 : nch) * (size_t)L.G * 4);
+  w.o_lg = take(rope ? units * s_stride * (size_t)L.G * 4 : 0);  // RoPE: every token's logits
   w.o_cnt = take(units * 4);
   w.o_part = take((size_t)(kMaxGrid + units) * (size_t)part_floats(L.G) * 4);
   w.o_suf = take(units * (size_t)((suffix_cap + SCH - 1) / SCH) * (size_t)suf_floats(L.G) * 4);
@@ -1860,7 +2080,12 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   const int ctas = g_debug_cluster.load(std::memory_order_relaxed);
   const int drop = g_debug_withhold.load(std::memory_order_relaxed);
   const int codec = (p.flags & AKV_FLAG_LLOYD) ? 1 : 0;
-  const LaunchKey key{dev, L.G, codec, units, L.max_len, L.max_k, ctas, (long long)(max_density(L) * 1e6),
+  const int rope = (p.flags & AKV_FLAG_ROPE) ? 1 : 0;
+  if (rope && sfx.K) {
+    *why = "a dense suffix with RoPE at decode is not supported";
+    return -1;
+  }
+  const LaunchKey key{dev, L.G, codec, rope, units, L.max_len, L.max_k, ctas, (long long)(max_density(L) * 1e6),
                       (long long)(max_anchor_density(L) * 1e6), ttot};
   Plan pl;
   bool have = false;
@@ -1874,9 +2099,10 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   }
   if (!have) {
     const DeviceInfo di = device_info();
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel<GS>(codec), cudaFuncAttributeMaxDynamicSharedMemorySize, di.smem_optin);
+    cudaError_t e =
+        cudaFuncSetAttribute(decode_kernel<GS>(codec, rope), cudaFuncAttributeMaxDynamicSharedMemorySize, di.smem_optin);
     if (e != cudaSuccess) return (int)e;
-    if (!make_plan(L, GS, di.smem_optin, &pl, why)) return -1;
+    if (!make_plan(L, GS, di.smem_optin, !rope, &pl, why)) return -1;
     int grid = (int)std::min<long long>(std::min(di.sms, kMaxGrid), ttot);
     if (ctas > 0) grid = (int)std::min<long long>(ctas, ttot);
     pl.grid = grid;
@@ -1891,7 +2117,8 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
     }
     pl.P.ttot = ttot;
     pl.P.grid = grid;
-    pl.P.n_ch = (L.max_k + CHA - 1) / CHA;
+    // chunk maxima per unit: of 64 anchors, or with RoPE of 64 stored tokens
+    pl.P.n_ch = rope ? (L.max_len + 63) / 64 : (L.max_k + CHA - 1) / CHA;
     std::lock_guard<std::mutex> lk(mu);
     cache[key] = pl;
   }
@@ -1916,6 +2143,8 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   P.sign_lo = L.header.sign_bits[0];
   P.sign_hi = L.header.sign_bits[1];
   P.drop_last = drop;
+  P.lg = rope ? (const float*)(wsb + W.o_lg) : nullptr;
+  P.s_stride = (L.max_len + 63) & ~63;
   P.suf_part = n_sch ? (const float*)(wsb + W.o_suf) : nullptr;
   P.suf_len = sfx.len;
   P.suf_cap = sfx.cap;
@@ -1955,16 +2184,41 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
     ev_scores = g_ev_scores;
     ev_decode = g_ev_decode;
   }
-  cudaError_t e = cudaLaunchKernelEx(&cfg, score_kernel<GS>(), S);
+  cudaError_t e;
+  if (rope) {  // the logits of every stored token (no anchor scores)
+    RopeParams R;
+    R.arena = P.arena;
+    R.q = P.q;
+    R.lg = (float*)(wsb + W.o_lg);
+    R.cmax = (float*)(wsb + W.o_cmax);
+    R.cnt = P.cnt;
+    R.n_kv_heads = p.n_kv_heads;
+    R.n_q_heads = p.n_q_heads;
+    R.rotate = P.rotate;
+    R.lloyd = codec;
+    R.s_stride = P.s_stride;
+    R.n_tch = P.n_ch;
+    R.scale_log2 = P.scale_log2;
+    R.sign_lo = P.sign_lo;
+    R.sign_hi = P.sign_hi;
+    // theta_j / (2 pi) < 1 as a 64-bit binary fraction of a turn (truncated past 2^-64)
+    for (int j = 0; j < 64; ++j)
+      R.turn[j] = (unsigned long long)std::ldexp(
+          std::pow((double)p.rope_theta, -2.0 * (double)j / 128.0) / 6.283185307179586476925, 64);
+    cfg.gridDim = dim3((unsigned)(units * P.n_ch), 1, 1);
+    e = cudaLaunchKernelEx(&cfg, rope_kernel<GS>(), R);
+  } else {
+    e = cudaLaunchKernelEx(&cfg, score_kernel<GS>(), S);
+  }
   if (e != cudaSuccess) return (int)e;
   if (ev_scores && (e = cudaEventRecord(ev_scores, cfg.stream)) != cudaSuccess) return (int)e;
   cfg.gridDim = dim3((unsigned)pl.grid, 1, 1);
   cfg.blockDim = dim3(NT, 1, 1);
   cfg.dynamicSmemBytes = pl.smem;
-  e = cudaLaunchKernelEx(&cfg, decode_kernel<GS>(codec), P);
+  e = cudaLaunchKernelEx(&cfg, decode_kernel<GS>(codec, rope), P);
   if (e != cudaSuccess) {
     cudaFuncAttributes fa{};
-    cudaFuncGetAttributes(&fa, decode_kernel<GS>(codec));
+    cudaFuncGetAttributes(&fa, decode_kernel<GS>(codec, rope));
     *why = "(decode kernel: " + std::to_string(fa.numRegs) + " registers, max " + std::to_string(fa.maxThreadsPerBlock) +
            " threads, " + std::to_string(pl.smem) + " B dynamic shared memory of " +
            std::to_string(fa.maxDynamicSharedSizeBytes) + ", grid " + std::to_string(pl.grid) + ")";

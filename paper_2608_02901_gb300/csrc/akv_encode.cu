@@ -581,6 +581,7 @@ __global__ void __launch_bounds__(kTile) enc_tile_fill(const EncArgs A) {
     kst[t] = w.st[0][i];
     vst[t] = w.st[1][i];
     f = w.flag[i];
+    if (d->off_pos) reinterpret_cast<uint32_t*>(A.arena + d->off_pos)[j * kTile + t] = (uint32_t)i;  // RoPE positions
   }
   const unsigned bk = __ballot_sync(0xffffffffu, f & 1u), bv = __ballot_sync(0xffffffffu, f & 2u);
   if (lane == 0) {

@@ -118,7 +118,7 @@ int launch_encode(const Layout& L, const EncodeWs& W, const akv_params& p, const
 // Decode workspace (device): anchor scores [units][ka][G] f32, query headers, chunk maxima,
 // arrival counters, partial slots; byte offsets from the workspace base (256-byte aligned).
 struct DecodeWs {
-  size_t o_sa = 0, o_uh = 0, o_cmax = 0, o_cnt = 0, o_part = 0, o_suf = 0, total = 0;
+  size_t o_sa = 0, o_uh = 0, o_cmax = 0, o_cnt = 0, o_part = 0, o_suf = 0, o_lg = 0, total = 0;
 };
 // The dense suffix of a decode call (akv_suffix): bf16 rows [B][H_kv][cap][128] and the tokens
 // held per request (device int32 [B]); null K = no suffix.

@@ -126,5 +126,6 @@ def decode_on_gpu(torch, p: akv.Params, lens, arena_dev, q: np.ndarray, sm_scale
 
 def oracle_decode(p: akv.Params, units, q: np.ndarray, sm_scale: float, sel=None):
     G = p.G
-    ref = oracle.attend(units, q.reshape(p.n_units, G, 128), G, sm_scale, p.rot_seed, p.rotate, lloyd=p.lloyd, sel=sel)
+    ref = oracle.attend(units, q.reshape(p.n_units, G, 128), G, sm_scale, p.rot_seed, p.rotate, lloyd=p.lloyd, sel=sel,
+                        rope_theta=p.rope_theta if p.rope else 0.0)
     return ref.reshape(p.batch, p.n_q_heads, 128)

@@ -56,7 +56,7 @@ def test_layout_header_and_sections():
     p = akv.Params(batch=4, n_kv_heads=2, n_q_heads=8, seed=3, rot_seed=9)
     arena_bytes, ws_bytes = akv.akv_cache_size(p, lens)
     hdr = akv.akv_cache_header_host(p, lens)
-    assert hdr[:4].view(np.uint32)[0] == 0x32564B41 and hdr[4:8].view(np.uint32)[0] == 3
+    assert hdr[:4].view(np.uint32)[0] == 0x32564B41 and hdr[4:8].view(np.uint32)[0] == 4
     assert hdr[8:16].view(np.uint64)[0] == arena_bytes
     assert hdr[72:76].view(np.int32)[0] == 8 and hdr[76:80].view(np.int32)[0] == 5000
     assert hdr[104:108].view(np.int32)[0] == 1024
@@ -217,6 +217,20 @@ def test_entry_points_validate_before_any_launch():
     assert L.akv_suffix_append(sp(p), None, 0x2000, 0x3000, 0x4000, 0x5000, 8, None) == akv.AKV_ERR_INVALID
     assert L.akv_suffix_append(sp(p), 0x1000, 0x2000, 0x3000, 0x4000, 0x5002, 8, None) == akv.AKV_ERR_INVALID
     assert L.akv_suffix_append(sp(p), 0x1000, 0x2000, 0x3000, 0x4000, 0x5000, 0, None) == akv.AKV_ERR_INVALID
+    # RoPE at decode: the base must be given with the flag (and only with it); no suffix with it
+    pr = akv.Params(batch=1, n_kv_heads=1, n_q_heads=1, rope=True).c()
+    sz = ctypes.c_size_t()
+    assert L.akv_cache_size(sp(pr), lp, sp(sz), None) == akv.AKV_OK and sz.value > nbytes  # + positions
+    for theta in (0.0, 1.0, float("inf"), float("nan")):
+        bad = akv.Params(batch=1, n_kv_heads=1, n_q_heads=1, rope=True).c()
+        bad.rope_theta = theta
+        assert L.akv_cache_size(sp(bad), lp, sp(sz), None) == akv.AKV_ERR_INVALID
+    bad = akv.Params(batch=1, n_kv_heads=1, n_q_heads=1).c()
+    bad.rope_theta = 10000.0
+    assert L.akv_cache_size(sp(bad), lp, sp(sz), None) == akv.AKV_ERR_INVALID
+    st = L.akv_decode_attn_suffix(sp(pr), lp, 0x1000, sz.value, 256, 256, None, 1.0,
+                                  sp(S(0x4000, 0x5000, 0x6000, 1000)), 0x3000, 1 << 40, None)
+    assert st == akv.AKV_ERR_UNSUPPORTED
 
 
 def test_decode_debug_controls_validate():

@@ -293,3 +293,53 @@ def test_lloyd_max_codec_encoded(dev, G):
         q = gen.queries(H * G, seed=qseed)
         out, out32 = decode_on_gpu(torch, p, [S], arena, q, 1.0)
         check_outputs(out, out32, oracle_decode(p, units, q, 1.0), f"lloyd encoded G={G} q={qseed}")
+
+
+# ---- RoPE at decode (pre-RoPE keys, each token turned to its stored position) ----
+
+@pytest.mark.parametrize("G", [1, 2, 4, 8])
+def test_rope_seeded_ragged(dev, G):
+    """Seeded caches packed with their positions (the stored order's permutation), ragged lengths
+    (one token, partial chunks and tiles), both codecs."""
+    for lloyd, base in ((False, 10000.0), (True, 500000.0)):
+        p = akv.Params(batch=3, n_kv_heads=2, n_q_heads=2 * G, seed=21, rot_seed=22, rope=True, rope_theta=base,
+                       lloyd=lloyd)
+        _run_seeded(dev, p, [1, 777, 3000], qseed=G + int(lloyd))
+
+
+def test_rope_dense_residuals_and_cta_splits(dev, debug_controls):
+    """Every token a residual (the CUDA-core token path) and tile ranges split over few CTAs."""
+    p = akv.Params(batch=2, n_kv_heads=2, n_q_heads=8, anchor_frac=0.05, res_frac_k=1.0, res_frac_v=1.0, seed=23,
+                   rope=True)
+    _run_seeded(dev, p, [2500, 1200])
+    for c in (1, 3):
+        akv.akv_decode_set_debug(ctas=c)
+        _run_seeded(dev, p, [2500, 1200], qseed=c)
+
+
+def test_rope_long_context_positions(dev):
+    """128K positions: the angles of the fast pairs reach 1e5 radians; the integer turn keeps the
+    sine and cosine accurate at every position."""
+    S = 131072
+    p = akv.Params(batch=1, n_kv_heads=1, n_q_heads=4, seed=24, rope=True, rope_theta=500000.0)
+    _run_seeded(dev, p, [S], seed=9)
+
+
+def test_rope_encoded(dev):
+    """GPU encode of pre-RoPE clustered keys: the arena's positions (read back by the oracle's
+    reader) drive the rotation."""
+    S, H, G = 8192, 2, 4
+    p = akv.Params(batch=1, n_kv_heads=H, n_q_heads=H * G, seed=7, rot_seed=11, rope=True, rope_theta=500000.0)
+    K, V = gen.clustered_batch(1, H, [S], seed=45)
+    a_bytes, w_bytes = akv.akv_cache_size(p, [S])
+    arena = torch.empty(a_bytes, dtype=torch.uint8, device=dev)
+    ws = torch.empty(w_bytes, dtype=torch.uint8, device=dev)
+    akv.akv_encode(p, [S], to_dev_u16(K, torch, dev), to_dev_u16(V, torch, dev), arena, ws)
+    units = oracle.unpack_arena(arena.cpu().numpy())
+    want = oracle.encode(K, V, [S], H, p.anchor_frac, p.res_frac_k, p.res_frac_v, p.window, p.seed, p.rot_seed)
+    for g, w in zip(units, want):  # the stored tokens' positions: the stable sort of positions by value slot
+        assert np.array_equal(g.pos, np.argsort(w.idx_v, kind="stable"))
+    for qseed in (1, 2):
+        q = gen.queries(H * G, seed=qseed)
+        out, out32 = decode_on_gpu(torch, p, [S], arena, q, 1.0)
+        check_outputs(out, out32, oracle_decode(p, units, q, 1.0), f"rope encoded q={qseed}")

@@ -501,3 +501,53 @@ def test_eta_of_each_codec_on_gaussian_residuals():
     e_un = oracle.eta(R, 11, True, False)
     assert abs(e_lm - mse) < 0.005
     assert 1.8 * e_lm < e_un < 0.3
+
+
+# ---- RoPE at decode (Section 3.2: keys kept pre-RoPE, turned to their positions) ----
+
+def _rope_complex(X, pos, base):
+    """Rotate-half RoPE as complex multiplication: z_j = x_j + i x_{j+64} times e^{i p theta_j}."""
+    X = np.atleast_2d(np.asarray(X, np.float64))
+    th = base ** (-2.0 * np.arange(64) / 128.0)
+    z = (X[:, :64] + 1j * X[:, 64:]) * np.exp(1j * np.asarray(pos, np.float64)[:, None] * th[None, :])
+    return np.concatenate([z.real, z.imag], axis=1)
+
+
+@pytest.mark.parametrize("base", [10000.0, 500000.0])
+def test_rope_turn_is_the_complex_rotation(base):
+    rng = np.random.default_rng(8)
+    for p in (0, 1, 7, 4095, 131071, 1 << 20):
+        x = rng.standard_normal(D)
+        y = oracle.rope(x, p, base)
+        assert np.allclose(y, _rope_complex(x, [p], base)[0], rtol=0, atol=1e-9)
+        assert abs(np.linalg.norm(y) - np.linalg.norm(x)) < 1e-12  # a rotation
+
+
+@pytest.mark.parametrize("base", [10000.0, 500000.0])
+def test_rope_attend_matches_dense_bruteforce(tiny, base):
+    """Each reconstructed (pre-RoPE) key turned to its position, then Eq. 4 softmax: equal to a
+    dense softmax over the complex-rotated rows; positions from a permutation (stored order)."""
+    _, _, u = tiny
+    q = gen.queries(2, 81)
+    Kh = oracle.reconstruct(u, "k", PAR["rot_seed"])
+    Vh = oracle.reconstruct(u, "v", PAR["rot_seed"])
+    for pos in (np.arange(u.S, dtype=np.int32), np.random.default_rng(3).permutation(u.S).astype(np.int32)):
+        u.pos = pos
+        out = oracle.attend([u], q, 2, 1.0, PAR["rot_seed"], rope_theta=base)[0]
+        Kr = _rope_complex(Kh, pos, base)
+        for g in range(2):
+            y, _ = _softmax_attend(Kr, Vh, gen.bf16_to_f64(q[g]), 1.0)
+            assert np.allclose(out[g], y, rtol=0, atol=1e-10)
+    u.pos = np.arange(u.S, dtype=np.int32)
+
+
+def test_rope_at_position_zero_is_plain_attention(tiny):
+    _, _, u = tiny
+    q = gen.queries(4, 82)
+    plain = oracle.attend([u], q, 4, 1.0, PAR["rot_seed"])
+    u.pos = np.zeros(u.S, np.int32)
+    zero = oracle.attend([u], q, 4, 1.0, PAR["rot_seed"], rope_theta=500000.0)
+    u.pos = np.arange(u.S, dtype=np.int32)
+    assert np.array_equal(plain, zero)
+    moved = oracle.attend([u], q, 4, 1.0, PAR["rot_seed"], rope_theta=500000.0)
+    assert not np.allclose(plain, moved, rtol=0, atol=1e-6)
