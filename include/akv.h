@@ -381,6 +381,29 @@ typedef struct akv_unit_host {
 akv_status akv_cache_pack_host(const akv_params* p, const int32_t* ctx_lens_host, const akv_unit_host* units,
                                void* arena_host, size_t arena_bytes);
 
+/* ---- The paper's Table 1 layer layout (byte parity) ---------------------- */
+
+/*
+ * Appendix A.1 "Layout", Table 1: the tensors of one compressed layer, charging every byte, with
+ * P = S - W non-window positions:
+ *   anchor keys [H][k][128] bf16, anchor values [H][k][128] bf16, anchor positions [H][k-W] int64
+ *   (the non-window anchors), anchor index [2][H][P] u16 (b_a = 2), coefficient [2][H][P] fp16
+ *   (b_gamma = 2), residual mask [2][H][ceil(P/64)] u64 words, prefix counts [2][H][ceil(P/64)]
+ *   int32 (exclusive, within the head), head offsets [2][H+1] int32, position ids [P] int32, then
+ *   residual codes [N][32] (key records head by head in position order, then value records),
+ *   scales [N] fp32, value slot positions [N_V] u8 (position mod 64 of each value record).
+ * Its size is exactly M_base of Eq. 11 + N_K (D/4 + 4) + N_V (D/4 + 5): the accounting behind Eq. 9.
+ * It is an interchange layout, not read by the decode (whose own format is documented above).
+ * Table 1 stores one scale per record, so it needs AKV_FLAG_LLOYD (min = 0), and S >= W.
+ * One layer block per request, concatenated in request order.
+ */
+akv_status akv_table1_bytes(const akv_params* p, const int32_t* ctx_lens_host, size_t* bytes_per_request);
+/* Packs logical units (as for akv_cache_pack_host, minima 0) into the Table 1 layout in HOST memory.
+ * Errors: AKV_ERR_INVALID (null arrays, residual positions not ascending non-window positions, a
+ * nonzero min), AKV_ERR_UNSUPPORTED (not the Lloyd-Max codec, S < W), AKV_ERR_TOO_SMALL. */
+akv_status akv_pack_table1_host(const akv_params* p, const int32_t* ctx_lens_host, const akv_unit_host* units,
+                                void* out_host, size_t out_bytes);
+
 /* ---- Decode ------------------------------------------------------------- */
 
 /*

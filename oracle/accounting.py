@@ -57,3 +57,52 @@ def decode_read_bytes(S: int, k: int, nk: int, nv: int, G: int, D: int = 128) ->
     format_unit_bytes except the anchor positions, plus G bf16 query rows in
     and G bf16 output rows out."""
     return format_unit_bytes(S, k, nk, nv, D) - 4 * k + 2 * G * D * 2
+
+
+def read_table1(buf, S: int, H: int, W: int, k: int, nk, nv, D: int = 128) -> list:
+    """Independent reader of one request's layer in the paper's Table 1 layout (Appendix A.1):
+    returns per KV head a dict of the logical arrays (positions 0 .. P-1 for the per-position ones,
+    P = S - W), checking the prefix counts and head offsets against the masks."""
+    import numpy as np
+    b = np.frombuffer(bytes(buf), np.uint8)
+    P, nw = S - W, -(-(S - W) // 64)
+    at = 0
+
+    def take(n, dt, shape):
+        nonlocal at
+        a = b[at:at + n * np.dtype(dt).itemsize].view(dt).reshape(shape)
+        at += n * np.dtype(dt).itemsize
+        return a
+    ak = take(H * k * D, np.uint16, (H, k, D))
+    av = take(H * k * D, np.uint16, (H, k, D))
+    apos = take(H * (k - W), np.int64, (H, k - W))
+    idx = take(2 * H * P, np.uint16, (2, H, P))
+    gam = take(2 * H * P, np.uint16, (2, H, P))
+    mask = take(2 * H * nw, np.uint64, (2, H, nw))
+    pref = take(2 * H * nw, np.int32, (2, H, nw))
+    hoff = take(2 * (H + 1), np.int32, (2, H + 1))
+    ids = take(P, np.int32, (P,))
+    NK, NV = int(sum(nk)), int(sum(nv))
+    codes = take((NK + NV) * (D // 4), np.uint8, (NK + NV, D // 4))
+    scales = take(NK + NV, np.float32, (NK + NV,))
+    vslot = take(NV, np.uint8, (NV,))
+    assert at == b.size, "trailing or missing bytes"
+    assert np.array_equal(ids, np.arange(P))
+    out = []
+    for h in range(H):
+        u = dict(anchor_k=ak[h], anchor_v=av[h], anchor_pos=apos[h], idx_k=idx[0, h], gam_k=gam[0, h],
+                 idx_v=idx[1, h], gam_v=gam[1, h])
+        for side, name in ((0, "k"), (1, "v")):
+            bits = [(int(mask[side, h, w]) >> j) & 1 for w in range(nw) for j in range(64)]
+            pos = np.flatnonzero(np.array(bits[:P], bool)).astype(np.int32)
+            cnt = np.array([bin(int(m)).count("1") for m in mask[side, h]])
+            assert np.array_equal(pref[side, h], np.concatenate([[0], np.cumsum(cnt)[:-1]])), "prefix counts"
+            assert hoff[side, h + 1] - hoff[side, h] == pos.size, "head offsets"
+            first = (0 if side == 0 else NK) + int(hoff[side, h])
+            u["res_" + name] = pos
+            u["codes_" + name] = codes[first:first + pos.size]
+            u["scale_" + name] = scales[first:first + pos.size]
+            if side == 1:
+                u["vslot"] = vslot[int(hoff[1, h]):int(hoff[1, h]) + pos.size]
+        out.append(u)
+    return out

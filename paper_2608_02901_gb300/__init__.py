@@ -27,7 +27,8 @@ EXPORTED = (
     "akv_status_string", "akv_last_error", "akv_unit_shapes", "akv_cache_size", "akv_cache_header_host",
     "akv_encode", "akv_encode_noalloc", "akv_cache_pack_host", "akv_decode_workspace_size", "akv_decode_attn",
     "akv_decode_set_debug", "akv_decode_set_events", "akv_cache_size_select", "akv_encode_select",
-    "akv_decode_workspace_size_suffix", "akv_decode_attn_suffix", "akv_suffix_append",
+    "akv_decode_workspace_size_suffix", "akv_decode_attn_suffix", "akv_suffix_append", "akv_table1_bytes",
+    "akv_pack_table1_host",
 )
 AKV_MAX_SUFFIX = 1 << 20
 NOALLOC_SCRATCH_BYTES = 16 << 20
@@ -157,6 +158,10 @@ def lib():
                                              ctypes.POINTER(_Suffix), vp, ctypes.c_size_t, vp]
         L.akv_suffix_append.restype = st
         L.akv_suffix_append.argtypes = [P, vp, vp, vp, vp, vp, ctypes.c_int32, vp]
+        L.akv_table1_bytes.restype = st
+        L.akv_table1_bytes.argtypes = [P, i32p, ctypes.POINTER(ctypes.c_size_t)]
+        L.akv_pack_table1_host.restype = st
+        L.akv_pack_table1_host.argtypes = [P, i32p, ctypes.POINTER(_UnitHost), vp, ctypes.c_size_t]
         _lib = L
     return _lib
 
@@ -289,6 +294,32 @@ def akv_cache_pack_host(p: Params, ctx_lens, units) -> np.ndarray:
     out = np.zeros(arena_bytes, np.uint8)
     _check(lib().akv_cache_pack_host(ctypes.byref(p.c()), _i32p(lens), arr, out.ctypes.data, out.size),
            "akv_cache_pack_host")
+    return out
+
+
+def akv_table1_bytes(p: Params, ctx_lens) -> np.ndarray:
+    """Bytes of each request's layer in the paper's Table 1 layout (Lloyd-Max codec)."""
+    lens = _lens(ctx_lens)
+    out = np.zeros(p.batch, np.uint64)
+    _check(lib().akv_table1_bytes(ctypes.byref(p.c()), _i32p(lens),
+                                  out.ctypes.data_as(ctypes.POINTER(ctypes.c_size_t))), "akv_table1_bytes")
+    return out
+
+
+def akv_pack_table1_host(p: Params, ctx_lens, units) -> np.ndarray:
+    """units as for akv_cache_pack_host (minima 0); returns the requests' Table 1 layers, concatenated."""
+    lens = _lens(ctx_lens)
+    total = int(akv_table1_bytes(p, lens).sum())
+    keep = []
+    arr = (_UnitHost * len(units))()
+    for i, u in enumerate(units):
+        for name, dt in _UNIT_FIELDS:
+            a = np.ascontiguousarray(u[name], dtype=dt)
+            keep.append(a)
+            setattr(arr[i], name, a.ctypes.data if a.size else None)
+    out = np.zeros(total, np.uint8)
+    _check(lib().akv_pack_table1_host(ctypes.byref(p.c()), _i32p(lens), arr, out.ctypes.data, out.size),
+           "akv_pack_table1_host")
     return out
 
 

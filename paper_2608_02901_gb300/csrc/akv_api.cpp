@@ -489,6 +489,179 @@ akv_status akv_decode_set_events(void* after_scores, void* after_decode) {
   return AKV_OK;
 }
 
+// ---- The paper's Table 1 layer layout (byte parity with Appendix A.1) ----
+
+namespace {
+// Exact value of an fp16 bit pattern (every fp16 value is a float).
+float fp16_bits_to_float(uint16_t h) {
+  const int e = (h >> 10) & 31, m = h & 1023;
+  const float mag = e == 0 ? std::ldexp((float)m, -24) : (e == 31 ? (m ? NAN : INFINITY) : std::ldexp((float)(1024 + m), e - 25));
+  return (h & 0x8000) ? -mag : mag;
+}
+struct Table1Sizes {
+  uint64_t anchors, pos, stream, words, offsets, ids, codes, scales, vslots, total;
+};
+// Bytes of each Table 1 tensor of one request's layer (H units, context S, k anchors, N_K and N_V
+// residual records over its heads), with P = S - W the non-window positions.
+Table1Sizes table1_sizes(int64_t S, int64_t H, int64_t W, int64_t k, int64_t NK, int64_t NV) {
+  Table1Sizes t;
+  const int64_t P = S - W, nw = (P + 63) / 64;
+  t.anchors = (uint64_t)(H * k * 128 * 2);  // each of anchor keys and anchor values
+  t.pos = (uint64_t)(8 * H * (k - W));
+  t.stream = (uint64_t)(2 * H * P * 2);  // each of anchor index and coefficient
+  t.words = (uint64_t)(2 * H * nw * 8);  // residual mask
+  t.offsets = (uint64_t)(8 * (H + 1));
+  t.ids = (uint64_t)(4 * P);
+  t.codes = (uint64_t)((NK + NV) * 32);
+  t.scales = (uint64_t)((NK + NV) * 4);
+  t.vslots = (uint64_t)NV;
+  t.total = 2 * t.anchors + t.pos + 2 * t.stream + t.words + t.words / 2 + t.offsets + t.ids + t.codes + t.scales +
+            t.vslots;
+  return t;
+}
+// Table 1 needs every request's window inside its context and one scale per record (no min).
+akv_status table1_check(const akv_params* p, const Layout& L) {
+  if (!(p->flags & AKV_FLAG_LLOYD))
+    return fail(AKV_ERR_UNSUPPORTED, "the Table 1 layout stores one scale per record: the Lloyd-Max codec only");
+  for (const auto& sh : L.shape)
+    if (sh.S < p->window) return fail(AKV_ERR_UNSUPPORTED, "the Table 1 layout needs S >= W in every request");
+  return AKV_OK;
+}
+}  // namespace
+
+akv_status akv_table1_bytes(const akv_params* p, const int32_t* ctx_lens_host, size_t* bytes_per_request) {
+  g_last_error.clear();
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L);
+  if (st != AKV_OK) return st;
+  if (!bytes_per_request) return fail(AKV_ERR_INVALID, "null output");
+  if ((st = table1_check(p, L)) != AKV_OK) return st;
+  const int H = p->n_kv_heads;
+  for (int b = 0; b < p->batch; ++b) {
+    int64_t NK = 0, NV = 0;
+    for (int h = 0; h < H; ++h) {
+      NK += L.shape[(size_t)b * H + h].nk;
+      NV += L.shape[(size_t)b * H + h].nv;
+    }
+    const UnitShape& sh = L.shape[(size_t)b * H];
+    bytes_per_request[b] = (size_t)table1_sizes(sh.S, H, p->window, sh.k, NK, NV).total;
+  }
+  return AKV_OK;
+}
+
+akv_status akv_pack_table1_host(const akv_params* p, const int32_t* ctx_lens_host, const akv_unit_host* units,
+                                void* out_host, size_t out_bytes) {
+  g_last_error.clear();
+  Layout L;
+  akv_status st = make_layout(p, ctx_lens_host, &L);
+  if (st != AKV_OK) return st;
+  if (!units || !out_host) return fail(AKV_ERR_INVALID, "null units or output");
+  if ((st = table1_check(p, L)) != AKV_OK) return st;
+  const int H = p->n_kv_heads;
+  const int64_t W = p->window;
+  uint8_t* o = (uint8_t*)out_host;
+  size_t used = 0;
+  for (int b = 0; b < p->batch; ++b) {
+    const UnitShape& sh0 = L.shape[(size_t)b * H];
+    const int64_t S = sh0.S, k = sh0.k, P = S - W, nw = (P + 63) / 64;
+    int64_t NK = 0, NV = 0;
+    for (int h = 0; h < H; ++h) {
+      const akv_unit_host& in = units[(size_t)b * H + h];
+      const UnitShape& sh = L.shape[(size_t)b * H + h];
+      NK += sh.nk;
+      NV += sh.nv;
+      if (!in.anchor_k || !in.anchor_v || !in.anchor_pos || !in.idx_k || !in.gamma_k || !in.idx_v || !in.gamma_v ||
+          (sh.nk && (!in.res_pos_k || !in.codes_k || !in.scale_k || !in.min_k)) ||
+          (sh.nv && (!in.res_pos_v || !in.codes_v || !in.scale_v || !in.min_v)))
+        return fail(AKV_ERR_INVALID, "null array in unit " + std::to_string(b * H + h));
+    }
+    const Table1Sizes t = table1_sizes(S, H, W, k, NK, NV);
+    if (used + t.total > out_bytes) return fail(AKV_ERR_TOO_SMALL, "output shorter than akv_table1_bytes");
+    uint8_t* base = o + used;
+    size_t at = 0;
+    auto put = [&](const void* src, size_t n) {
+      std::memcpy(base + at, src, n);
+      at += n;
+    };
+    // anchor keys, anchor values: [H][k][128] bf16
+    for (int side = 0; side < 2; ++side)
+      for (int h = 0; h < H; ++h) put(side ? units[(size_t)b * H + h].anchor_v : units[(size_t)b * H + h].anchor_k, (size_t)k * 256);
+    // anchor positions [H][k - W] int64 (the non-window anchors: the first k - W slots)
+    for (int h = 0; h < H; ++h)
+      for (int64_t a = 0; a < k - W; ++a) {
+        const int64_t v = units[(size_t)b * H + h].anchor_pos[a];
+        put(&v, 8);
+      }
+    // anchor index and coefficient [2][H][P] (b_a = b_gamma = 2), positions 0 .. P-1
+    for (int side = 0; side < 2; ++side)
+      for (int h = 0; h < H; ++h) put(side ? units[(size_t)b * H + h].idx_v : units[(size_t)b * H + h].idx_k, (size_t)P * 2);
+    for (int side = 0; side < 2; ++side)
+      for (int h = 0; h < H; ++h)
+        put(side ? units[(size_t)b * H + h].gamma_v : units[(size_t)b * H + h].gamma_k, (size_t)P * 2);
+    // residual mask [2][H][nw] u64 and exclusive prefix counts [2][H][nw] i32 (within the head)
+    std::vector<uint64_t> mask((size_t)(2 * H * nw), 0);
+    for (int side = 0; side < 2; ++side)
+      for (int h = 0; h < H; ++h) {
+        const akv_unit_host& in = units[(size_t)b * H + h];
+        const int32_t n = side ? L.shape[(size_t)b * H + h].nv : L.shape[(size_t)b * H + h].nk;
+        const int32_t* rp = side ? in.res_pos_v : in.res_pos_k;
+        for (int32_t r = 0; r < n; ++r) {
+          if (rp[r] < 0 || rp[r] >= P || (r && rp[r] <= rp[r - 1]))
+            return fail(AKV_ERR_INVALID, "residual positions must be ascending non-window positions");
+          mask[(size_t)((side * H + h) * nw + rp[r] / 64)] |= 1ull << (rp[r] % 64);
+        }
+      }
+    put(mask.data(), mask.size() * 8);
+    for (int side = 0; side < 2; ++side)
+      for (int h = 0; h < H; ++h) {
+        int32_t run = 0;
+        for (int64_t wi = 0; wi < nw; ++wi) {
+          put(&run, 4);
+          run += __builtin_popcountll(mask[(size_t)((side * H + h) * nw + wi)]);
+        }
+      }
+    // head offsets [2][H + 1] i32: each side's records head by head
+    for (int side = 0; side < 2; ++side) {
+      int32_t off = 0;
+      for (int h = 0; h <= H; ++h) {
+        put(&off, 4);
+        if (h < H) off += side ? L.shape[(size_t)b * H + h].nv : L.shape[(size_t)b * H + h].nk;
+      }
+    }
+    // position ids [P] i32 (every non-window position is kept)
+    for (int32_t i = 0; i < (int32_t)P; ++i) put(&i, 4);
+    // residual codes [N][32]: key records head by head, then value records (position order);
+    // scales [N] fp32; value slot positions [N_V] u8 (position within its 64-position chunk)
+    for (int side = 0; side < 2; ++side)
+      for (int h = 0; h < H; ++h) {
+        const akv_unit_host& in = units[(size_t)b * H + h];
+        const int32_t n = side ? L.shape[(size_t)b * H + h].nv : L.shape[(size_t)b * H + h].nk;
+        put(side ? in.codes_v : in.codes_k, (size_t)n * 32);
+      }
+    for (int side = 0; side < 2; ++side)
+      for (int h = 0; h < H; ++h) {
+        const akv_unit_host& in = units[(size_t)b * H + h];
+        const int32_t n = side ? L.shape[(size_t)b * H + h].nv : L.shape[(size_t)b * H + h].nk;
+        for (int32_t r = 0; r < n; ++r) {
+          if ((side ? in.min_v : in.min_k)[r] & 0x7FFFu)
+            return fail(AKV_ERR_INVALID, "a record with a nonzero min: not a Lloyd-Max record");
+          const float sc = fp16_bits_to_float((side ? in.scale_v : in.scale_k)[r]);
+          put(&sc, 4);
+        }
+      }
+    for (int h = 0; h < H; ++h) {
+      const akv_unit_host& in = units[(size_t)b * H + h];
+      for (int32_t r = 0; r < L.shape[(size_t)b * H + h].nv; ++r) {
+        const uint8_t v = (uint8_t)(in.res_pos_v[r] % 64);
+        put(&v, 1);
+      }
+    }
+    if (at != t.total) return fail(AKV_ERR_INVALID, "internal: Table 1 sizes disagree");  // cannot happen
+    used += t.total;
+  }
+  return AKV_OK;
+}
+
 akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_lens_host, size_t* ws_bytes) {
   return akv_decode_workspace_size_suffix(p, ctx_lens_host, 0, ws_bytes);
 }

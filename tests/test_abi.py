@@ -257,3 +257,75 @@ def test_select_parameters_validate_and_size_the_pooled_capacity():
     # each unit may hold up to its request's whole side budget (Eq. 9), capped by its non-anchors
     hdr = akv.akv_cache_header_host(p, lens)  # plain layout: no residuals at fractions 0
     assert int(hdr[256 + 8:256 + 12].view(np.int32)[0]) == 0
+
+
+def _lloyd_units(p, lens, seed):
+    units = []
+    for u in helpers_seeded(p, lens, seed):
+        u["min_k"] = np.zeros_like(u["min_k"])
+        u["min_v"] = np.zeros_like(u["min_v"])
+        units.append(u)
+    return units
+
+
+def helpers_seeded(p, lens, seed):
+    from helpers import seeded_units
+    return seeded_units(p, lens, seed=seed)
+
+
+def test_table1_layout_has_the_paper_bytes_and_round_trips():
+    """Appendix A.1 Table 1: the packed layer has exactly M_base (Eq. 11) + N_K (D/4 + 4) + N_V (D/4 + 5)
+    bytes, and an independent reader gets every logical array back (value slot positions = p mod 64)."""
+    lens = [3000, 700]
+    p = akv.Params(batch=2, n_kv_heads=2, n_q_heads=4, seed=3, lloyd=True)
+    units = _lloyd_units(p, lens, 5)
+    shapes = akv.akv_unit_shapes(p, lens)
+    per_req = akv.akv_table1_bytes(p, lens)
+    blob = akv.akv_pack_table1_host(p, lens, [akv.unit_host_from_logical(u) for u in units])
+    at = 0
+    for b, S in enumerate(lens):
+        k = int(shapes[2 * b][1])
+        nk = [int(shapes[2 * b + h][2]) for h in range(2)]
+        nv = [int(shapes[2 * b + h][3]) for h in range(2)]
+        want = acc.paper_m_base(S, 2, 128, p.window, k) + sum(nk) * acc.paper_c_k(128) + sum(nv) * acc.paper_c_v(128)
+        assert int(per_req[b]) == want
+        heads = acc.read_table1(blob[at:at + want], S, 2, p.window, k, nk, nv)
+        at += want
+        P = S - p.window
+        for h, got in enumerate(heads):
+            u = units[2 * b + h]
+            assert np.array_equal(got["anchor_k"], u["anchor_k"]) and np.array_equal(got["anchor_v"], u["anchor_v"])
+            assert np.array_equal(got["anchor_pos"], u["anchor_pos"][:k - p.window])
+            for n in ("idx_k", "gam_k", "idx_v", "gam_v"):
+                assert np.array_equal(got[n], u[n][:P])
+            for side in ("k", "v"):
+                assert np.array_equal(got["res_" + side], u["res_" + side])
+                assert np.array_equal(got["codes_" + side], u["codes_" + side])
+                assert np.array_equal(got["scale_" + side], u["scale_" + side].view(np.float16).astype(np.float32))
+            assert np.array_equal(got["vslot"], u["res_v"] % 64)
+            # the window positions the layout leaves out are anchors of their own slot, gamma 1
+            assert np.array_equal(u["idx_k"][P:], np.arange(k - p.window, k)) and np.all(u["gam_k"][P:] == 0x3C00)
+    assert at == blob.size
+
+
+def test_table1_layout_of_the_worked_example_layer():
+    """The paper's worked example (S = 32K, H = 8, W = 32, k = 256, theta = 0.05: N = 91,056 residual
+    slots, 45,528 per side): the packed layer holds M_base (3.39 MB) + the residual bytes, within one
+    residual's bytes of theta M_full (6.71 MB)."""
+    S, H = 32768, 8
+    f = 5691 / 32768  # 45,528 / 8 records per head and side, exactly floor(f S)
+    p = akv.Params(batch=1, n_kv_heads=H, n_q_heads=H, anchor_frac=256 / 32768, res_frac_k=f, res_frac_v=f,
+                   lloyd=True)
+    shapes = akv.akv_unit_shapes(p, [S])
+    assert shapes[:, 1].tolist() == [256] * H and shapes[:, 2].sum() == 45528 and shapes[:, 3].sum() == 45528
+    n = int(akv.akv_table1_bytes(p, [S])[0])
+    m_full = acc.paper_m_full(S, H, 128)
+    assert n == acc.paper_m_base(S, H, 128, 32, 256) + 45528 * 36 + 45528 * 37
+    assert 0 <= 0.05 * m_full - n < 37
+    units = _lloyd_units(p, [S], 7)
+    assert akv.akv_pack_table1_host(p, [S], [akv.unit_host_from_logical(u) for u in units]).size == n
+
+
+def test_table1_layout_needs_the_lloyd_codec():
+    p = akv.Params(batch=1, n_kv_heads=1, n_q_heads=1)
+    assert _err(akv.akv_table1_bytes, p, [1000]) == akv.AKV_ERR_UNSUPPORTED
