@@ -74,6 +74,7 @@ static_assert(LCH == 8, "a lane's tokens are one byte of a bitmap word");
 constexpr int NSG = 4;              // tiles a group has in flight at most (its stage descriptors)
 constexpr int kMaxGrid = 256;       // CTAs of the decode launch at most
 constexpr int CHA = 64;             // anchors per score-kernel CTA (4 warps x 16 rows)
+constexpr int kOvl = 32;            // a tile's entries per overflow list (value records, anchor-value runs)
 constexpr int kRingSlack = 4096;    // shared memory after the ring: the masked rows of the last
                                     // 16-row block of staged anchor values are read from here
 constexpr unsigned long long kWaitNs = 2000000000ull;  // an mbarrier wait gives up after 2 s
@@ -154,7 +155,7 @@ struct DecodeParams {
   int cap;         // staged bytes of a tile block at most
   int ring_bytes, drop_last, smem_sa;
   int o_bar, o_meta, o_misc, o_sa, o_ovf, o_grp, grp_bytes, o_ring;
-  int g_qp, g_rows, g_red, g_wb, g_pv, g_qf;  // offsets inside a group's block
+  int g_qp, g_rows, g_red, g_wb, g_pv, g_qf, g_ovl;  // offsets inside a group's block
   const float* lg;         // RoPE at decode: logits [units][s_stride][G] in stored order (else null)
   int s_stride;
   const float* suf_part;   // dense suffix partials [units][n_sch][suf_floats] (null: no suffix)
@@ -893,16 +894,15 @@ __device__ __forceinline__ void head_probs(float gk, const float (&sa)[GS], cons
 // of dimension pairs (j, j + 64) by p theta_j (Section 3.2; Appendix E.1's score kernel rebuilds
 // keys and applies RoPE from the stored positions the same way).  CTA (unit u, chunk c): stored
 // tokens 64 c .. 64 c + 63; warp w rebuilds tokens 16 w .. 16 w + 15, lane l holding dimensions
-// 4 l .. 4 l + 3 (pair partners sit 16 lanes apart), into shared memory; then thread t sums
-// q_g . y over one half of the dimensions of token t % 64 for every head g.  The angle of pair j
+// 4 l .. 4 l + 3 (pair partners sit 16 lanes apart), into shared memory; then its 16 x G logits
+// come from tensor-core products (keys as fp16 high + low parts, q exact).  The angle of pair j
 // at position p is taken as a binary fraction of a turn, p * turn_j mod 2^64 (exact integer
 // arithmetic), so the sine and cosine are evaluated on [0, 2 pi) whatever the position.
 template <int GS>
 __global__ void __launch_bounds__(128) akv_rope_logits_kernel(const RopeParams P) {
   __shared__ __align__(16) float ys[64][132];  // rows 16-byte aligned; 128-bit reads conflict-free
   __shared__ __align__(16) float qsm[8][128];
-  __shared__ float part[2][64][8];
-  __shared__ float wmx[2][8];
+  __shared__ float wmx4[4][8];
   __shared__ unsigned long long turn[64];
   const int u = blockIdx.x / P.n_tch, c = blockIdx.x % P.n_tch;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -989,7 +989,7 @@ __global__ void __launch_bounds__(128) akv_rope_logits_kernel(const RopeParams P
       for (int h = 0; h < 2; ++h) {
         const int e = (lane < 16 ? 0 : 2) + h;
         const unsigned long long ph = (unsigned long long)p * turn[(4 * lane + e) & 63];
-        __sincosf((float)(ph >> 40) * (6.2831853071795865f / 16777216.0f), &sn[e], &cs[e]);
+        __sincosf((float)(uint32_t)(ph >> 40) * (6.2831853071795865f / 16777216.0f), &sn[e], &cs[e]);
         const int eo = (lane < 16 ? 2 : 0) + h;
         sn[eo] = 0.f;
         cs[eo] = 0.f;
@@ -1014,40 +1014,66 @@ __global__ void __launch_bounds__(128) akv_rope_logits_kernel(const RopeParams P
     }
     *reinterpret_cast<float4*>(&ys[16 * warp + i][4 * lane]) = make_float4(y[0], y[1], y[2], y[3]);
   }
-  __syncthreads();
-  // thread t: token t % 64, dimensions 64 (t / 64) .. + 63, every head
+  __syncwarp();
+  // the warp's 16 logits rows on tensor cores: A = its rotated keys (fp16 high and low parts, from
+  // shared memory), B = the query rows (exact in fp16), fp32 sums: D[token][head] (heads >= GS zero)
   {
-    const int tk = tid & 63, hf = tid >> 6;
-    float acc[GS];
+    const int r8 = lane >> 2, c4 = lane & 3;
+    float d[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int g = 0; g < GS; ++g) acc[g] = 0.f;
-#pragma unroll 4
-    for (int dd = 0; dd < 64; dd += 4) {
-      const float4 yv = *reinterpret_cast<const float4*>(&ys[tk][64 * hf + dd]);
+    for (int ks = 0; ks < 8; ++ks) {
+      const float* y0 = &ys[16 * warp + r8][16 * ks + 2 * c4];
+      const float* y1 = &ys[16 * warp + r8 + 8][16 * ks + 2 * c4];
+      const float2 v[4] = {*reinterpret_cast<const float2*>(y0), *reinterpret_cast<const float2*>(y1),
+                           *reinterpret_cast<const float2*>(y0 + 8), *reinterpret_cast<const float2*>(y1 + 8)};
+      uint32_t hi[4], lo[4];
 #pragma unroll
-      for (int g = 0; g < GS; ++g) {
-        const float4 qv = *reinterpret_cast<const float4*>(&qsm[g][64 * hf + dd]);  // (the same for the warp)
-        acc[g] = fmaf(yv.x, qv.x, fmaf(yv.y, qv.y, fmaf(yv.z, qv.z, fmaf(yv.w, qv.w, acc[g]))));
+      for (int e = 0; e < 4; ++e) {
+        const __half2 h = __float22half2_rn(v[e]);
+        const float2 hf = __half22float2(h);
+        const __half2 l = __float22half2_rn(make_float2(v[e].x - hf.x, v[e].y - hf.y));
+        hi[e] = *reinterpret_cast<const uint32_t*>(&h);
+        lo[e] = *reinterpret_cast<const uint32_t*>(&l);
+      }
+      const bool hv = r8 < GS;  // column n = r8 of B: head r8
+      const __half2 b0 = __float22half2_rn(hv ? make_float2(qsm[hv ? r8 : 0][16 * ks + 2 * c4], qsm[hv ? r8 : 0][16 * ks + 2 * c4 + 1])
+                                              : make_float2(0.f, 0.f));
+      const __half2 b1 = __float22half2_rn(hv ? make_float2(qsm[hv ? r8 : 0][16 * ks + 2 * c4 + 8], qsm[hv ? r8 : 0][16 * ks + 2 * c4 + 9])
+                                              : make_float2(0.f, 0.f));
+      const uint32_t ub0 = *reinterpret_cast<const uint32_t*>(&b0), ub1 = *reinterpret_cast<const uint32_t*>(&b1);
+      mma_f16(d, make_uint4(hi[0], hi[1], hi[2], hi[3]), ub0, ub1);
+      mma_f16(d, make_uint4(lo[0], lo[1], lo[2], lo[3]), ub0, ub1);
+    }
+    // D rows r8, r8 + 8 (tokens), columns 2 c4, 2 c4 + 1 (heads)
+    float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int hr = 0; hr < 2; ++hr) {
+      const int ts = ts0 + 16 * warp + r8 + 8 * hr;
+      const bool ok = ts < S;
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int g = 2 * c4 + e;
+        const float l = d[2 * hr + e] * P.scale_log2;
+        if (ok && g < GS) {
+          P.lg[((size_t)u * P.s_stride + ts) * GS + g] = l;
+          mx[e] = fmaxf(mx[e], l);
+        }
       }
     }
 #pragma unroll
-    for (int g = 0; g < GS; ++g) part[hf][tk][g] = acc[g];
-  }
-  __syncthreads();
-  if (tid < 64) {
-    const bool ok = ts0 + tid < S;
-    float* dst = P.lg + ((size_t)u * P.s_stride + ts0 + tid) * GS;
-#pragma unroll
-    for (int g = 0; g < GS; ++g) {
-      const float l = (part[0][tid][g] + part[1][tid][g]) * P.scale_log2;
-      if (ok) dst[g] = l;
-      float m = ok ? l : -INFINITY;
-      m = warp_max(m);
-      if (lane == 0) wmx[warp][g] = m;
+    for (int o = 4; o < 32; o <<= 1) {
+      mx[0] = fmaxf(mx[0], __shfl_xor_sync(0xffffffffu, mx[0], o));
+      mx[1] = fmaxf(mx[1], __shfl_xor_sync(0xffffffffu, mx[1], o));
+    }
+    if (lane < 4) {
+      wmx4[warp][2 * lane] = mx[0];
+      wmx4[warp][2 * lane + 1] = mx[1];
     }
   }
   __syncthreads();
-  if (tid < GS) P.cmax[((size_t)u * P.n_tch + c) * GS + tid] = fmaxf(wmx[0][tid], wmx[1][tid]);
+  if (tid < GS)
+    P.cmax[((size_t)u * P.n_tch + c) * GS + tid] =
+        fmaxf(fmaxf(wmx4[0][tid], wmx4[1][tid]), fmaxf(wmx4[2][tid], wmx4[3][tid]));
 }
 
 // A lane's tokens of a tile: bitmap bytes and first record indices.
@@ -1067,6 +1093,8 @@ struct TokTile {
   float* ovf;         // [2][GS][128] overflow sums
   const uint8_t* AV;  // the unit's anchor values (global)
   const float* lgt;   // RoPE at decode: the tile's logit rows [T][GS] (global), else null
+  int* ovl_n;         // the tile's overflow lists: value records beyond the staged ones, and runs
+  float* ovl;         // beyond the staged anchor-value rows, applied by the whole group after the tokens
   int k, nKs, nVs, ka, lloyd;
 };
 
@@ -1102,6 +1130,8 @@ __device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const
   float* ovf = tt.ovf;
   const uint8_t* AV = tt.AV;
   const float* lgt = tt.lgt;
+  int* ovl_n = tt.ovl_n;
+  float* ovl = tt.ovl;
   const int k = tt.k, nKs = tt.nKs, nVs = tt.nVs, ka = tt.ka, lloyd = tt.lloyd;
   const uint32_t lo = tt.lo;
   const int nrows = (int)tt.nrows;
@@ -1123,8 +1153,16 @@ __device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const
       float* w = W + ix * GS;
 #pragma unroll
       for (int g = 0; g < GS; ++g) red_local(w + g, vv[g]);
-    } else {  // beyond the staged anchor-value rows: its products on CUDA cores
-      anchor_value_add<GS>(AV, (int)kk, vv, ovf);
+    } else {  // beyond the staged anchor-value rows: listed for the group (else on CUDA cores here)
+      const int e = atomicAdd(ovl_n + 1, 1);
+      if (e < kOvl) {
+        float* en = ovl + (kOvl + e) * 9;
+        en[0] = __int_as_float((int)kk);
+#pragma unroll
+        for (int g = 0; g < GS; ++g) en[1 + g] = vv[g];
+      } else {
+        anchor_value_add<GS>(AV, (int)kk, vv, ovf);
+      }
     }
   };
   for (int e = 0; e < LCH; ++e) {
@@ -1171,11 +1209,19 @@ __device__ __noinline__ LShare<(GS >= 2 ? GS / 2 : 1)> token_chunk_general(const
     if (vb && e < nvalid) {
       if (rv < nVs) {
         store_row<GS>(pv + rv * 8, pe);
-      } else {  // beyond the staged records
+      } else {  // beyond the staged records: listed for the group (else on CUDA cores here)
+        const int en_i = atomicAdd(ovl_n, 1);
+        if (en_i < kOvl) {
+          float* en = ovl + en_i * 9;
+          en[0] = __int_as_float(rv);
 #pragma unroll
-        for (int g = 0; g < GS; ++g)
-          value_record_add(st, gb, staged, tv.sm_v + 4u * (uint32_t)rv, tv.cd_v + 512u * (uint32_t)(rv / 16), rv,
-                           (g & 1) ? pe[g >> 1].y : pe[g >> 1].x, ovf + GS * 128 + g * 128, lloyd);
+          for (int g = 0; g < GS; ++g) en[1 + g] = (g & 1) ? pe[g >> 1].y : pe[g >> 1].x;
+        } else {
+#pragma unroll
+          for (int g = 0; g < GS; ++g)
+            value_record_add(st, gb, staged, tv.sm_v + 4u * (uint32_t)rv, tv.cd_v + 512u * (uint32_t)(rv / 16), rv,
+                             (g & 1) ? pe[g >> 1].y : pe[g >> 1].x, ovf + GS * 128 + g * 128, lloyd);
+        }
       }
     }
     // tokens past the tile join the current run with zero weight
@@ -1298,6 +1344,8 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
   int* lastf = reinterpret_cast<int*>(GB + P.g_red);
   float* wb = reinterpret_cast<float*>(GB + P.g_wb);      // [2][X][GS] value weights of a tile's slots
   float* pv = reinterpret_cast<float*>(GB + P.g_pv);      // [R][8] p rows of the value records, then A operands
+  int* ovl_n = reinterpret_cast<int*>(GB + P.g_ovl);       // [2] entries in the two overflow lists
+  float* ovl = reinterpret_cast<float*>(GB + P.g_ovl + 16);  // [2][kOvl][9]: index bits, then p (or weights) per head
   uint2* qf = reinterpret_cast<uint2*>(GB + P.g_qf);      // [NBF][8][32] key-residual B fragments
   const int bar_id = 1 + grp;
   auto gsync = [&]() { named_sync(bar_id, WPG * 32); };
@@ -1453,6 +1501,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         fast_tile = (ROPE || nKs == tv.nk) && nVs == tv.nv &&
                     (int)(((reinterpret_cast<const uint32_t*>(st + 4 * tv.n64))[tv.n - 1] & 0xFFFFu) - mt.lo) < (int)mt.nrows;
         for (int e = gt; e < P.X * GS; e += WPG * 32) W[e] = 0.f;
+        if (gt < 2) ovl_n[gt] = 0;
         // ---- key residuals: q' . c of the staged key records, tensor cores; the terms
         // scale (q' . c) + min sum(q') - m are written over the records' codes ----
         float* rsb = reinterpret_cast<float*>(const_cast<uint8_t*>(st) + tv.cd_k);
@@ -1674,12 +1723,43 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
         } else if (t0 < tv.n) {
           const auto ls = token_chunk_general<GS>(TokTile{tv, mt.lo, mt.nrows, SAt, rows, qp, pv, W, ovf, U.AV,
                                                       ROPE ? P.lg + ((size_t)sg.u * P.s_stride + (size_t)mt.j * T) * GS : nullptr,
-                                                      k, nKs, nVs, P.ka_stride, CODEC}, tl);
+                                                      ovl_n, ovl, k, nKs, nVs, P.ka_stride, CODEC}, tl);
 #pragma unroll
           for (int i2 = 0; i2 < NP; ++i2) l2[i2] = __fadd2_rn(l2[i2], ls.v[i2]);
         }
       }
       gsync();  // (B) the tile's weights and p rows are complete
+      if (go && !fast_tile) {  // the overflow lists: thread gt takes dimension gt of every entry
+        const int nv_o = min(ovl_n[0], kOvl), na_o = min(ovl_n[1], kOvl);
+        if (nv_o + na_o > 0) {
+          float av[GS], aa[GS];
+#pragma unroll
+          for (int g = 0; g < GS; ++g) av[g] = aa[g] = 0.f;
+          for (int e = 0; e < nv_o; ++e) {  // p (min + scale L(c)) of a value record, rotated domain
+            const float* en = ovl + e * 9;
+            const uint32_t r = (uint32_t)__float_as_int(en[0]);
+            const uint32_t smn = *reinterpret_cast<const uint32_t*>(tv.at(tv.sm_v + 4u * r));
+            const uint32_t w = *reinterpret_cast<const uint32_t*>(tv.at(tv.cd_v + 512u * (r / 16u) + 4u * value_code_word(gt)));
+            const float val = fmaf(half_lo(smn), code_level((w >> value_code_bit((int)(r % 16u))) & 3u, CODEC), half_hi(smn));
+#pragma unroll
+            for (int g = 0; g < GS; ++g) av[g] = fmaf(en[1 + g], val, av[g]);
+          }
+          for (int e = 0; e < na_o; ++e) {  // weight x the anchor's value row (global, swizzled by the slot)
+            const float* en = ovl + (kOvl + e) * 9;
+            const int kk = __float_as_int(en[0]);
+            const uint8_t* row = U.AV + (size_t)kk * 256;
+            const float x = __bfloat162float(
+                *reinterpret_cast<const __nv_bfloat16*>(row + 16 * ((gt >> 3) ^ (kk & 7)) + 2 * (gt & 7)));
+#pragma unroll
+            for (int g = 0; g < GS; ++g) aa[g] = fmaf(en[1 + g], x, aa[g]);
+          }
+#pragma unroll
+          for (int g = 0; g < GS; ++g) {
+            if (nv_o) red_local(ovf + GS * 128 + g * 128 + gt, av[g]);
+            if (na_o) red_local(ovf + g * 128 + gt, aa[g]);
+          }
+        }
+      }
       if (go) {
         // ---- value operands: p scale as bf16 high + low parts in the mma A layout, written
         // over the p rows of the same 16 records; sum of p min per head ----
@@ -1964,6 +2044,7 @@ bool make_plan_rx(const Layout& L, int GS, int R, int X, bool smem_sa, int smem_
   P.g_red = gtake(16);
   P.g_wb = gtake((size_t)2 * X * GS * 4);
   P.g_pv = gtake((size_t)R * 32);
+  P.g_ovl = gtake((size_t)(16 + 2 * kOvl * 9 * 4));  // the tile's overflow lists (counts, then entries)
   P.grp_bytes = (int)g;
   P.o_grp = take((size_t)NG * g);
   P.o_ring = (int)off;

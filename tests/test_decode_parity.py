@@ -158,6 +158,17 @@ def test_locally_dense_residuals_exceed_staging(dev):
         _run_seeded(dev, p, [6000, 3000], mutate=mutate)
 
 
+def test_value_records_a_little_beyond_the_staged_count(dev):
+    """Value residuals on every fifth non-anchor token in stored order (about 205 a tile, R = 176
+    staged): each tile's few dozen extra records go through the group's overflow list."""
+    def mutate(u, d):
+        non = _stored_non_anchor(d)
+        d["res_v"] = np.sort(non[::5][: d["nv"]]).astype(np.int32)
+    for G in (1, 4, 8):
+        p = akv.Params(batch=2, n_kv_heads=2, n_q_heads=2 * G, seed=43)
+        _run_seeded(dev, p, [6000, 9000], mutate=mutate, qseed=G)
+
+
 def test_key_records_beyond_the_value_staging_count(dev):
     """Key residuals on every fourth non-anchor token in stored order (about 250 a tile, 2.5x
     the mean): more key records than the value records a tile stages, yet their codes fit the
