@@ -352,10 +352,11 @@ __device__ __forceinline__ void warp_wht128(float (&x)[4], int lane) {
   x[3] = a1 - a3;
 #pragma unroll
   for (int m = 1; m < 32; m <<= 1) {  // stage of distance 4 m: partner lane l ^ m
+    const float sg = (lane & m) ? -1.f : 1.f;  // v - x (upper partner) or x + v, one exact fma each
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const float v = __shfl_xor_sync(0xffffffffu, x[j], m);
-      x[j] = (lane & m) ? v - x[j] : x[j] + v;
+      x[j] = fmaf(sg, x[j], v);
     }
   }
 }
@@ -562,7 +563,9 @@ __device__ __forceinline__ void suffix_chunk(const ScoreParams& P, int u, int sc
   __shared__ float ps[SCH][8];
   __shared__ float wm[4][8];
   __shared__ float mc[8];
-  __shared__ __align__(16) __nv_bfloat16 vsm[SCH][128];
+  // the chunk's value rows: dynamic shared memory, requested only by launches with a suffix
+  extern __shared__ __align__(16) uint8_t score_dyn[];
+  __nv_bfloat16 (*vsm)[128] = reinterpret_cast<__nv_bfloat16 (*)[128]>(score_dyn);
   const int len = max(0, min(P.suf_len[u / P.n_kv_heads], P.suf_cap));
   const int j0 = sc * SCH;
   if (j0 >= len) return;
@@ -898,7 +901,7 @@ __device__ __forceinline__ void head_probs(float gk, const float (&sa)[GS], cons
 // come from tensor-core products (keys as fp16 high + low parts, q exact).  The angle of pair j
 // at position p is taken as a binary fraction of a turn, p * turn_j mod 2^64 (exact integer
 // arithmetic), so the sine and cosine are evaluated on [0, 2 pi) whatever the position.
-template <int GS>
+template <int GS, int CODEC>
 __global__ void __launch_bounds__(128) akv_rope_logits_kernel(const RopeParams P) {
   __shared__ __align__(16) float ys[64][132];  // rows 16-byte aligned; 128-bit reads conflict-free
   __shared__ __align__(16) float qsm[8][128];
@@ -929,6 +932,17 @@ __global__ void __launch_bounds__(128) akv_rope_logits_kernel(const RopeParams P
   const uint8_t* AK = P.arena + d->off_anchor_k;
   const uint32_t* pos = reinterpret_cast<const uint32_t*>(P.arena + d->off_pos);
   __syncthreads();
+  // per lane: the turns of the two pair angles it evaluates (lanes 0-15 pairs 0, 1 of their four,
+  // lanes 16-31 pairs 2, 3), the rotation signs of its dimensions with the 1/128 folded in
+  const bool low = lane < 16;
+  const unsigned long long tn0 = turn[(4 * lane + (low ? 0 : 2)) & 63], tn1 = turn[(4 * lane + (low ? 1 : 3)) & 63];
+  const float rsgn = low ? -1.f : 1.f;  // y = x cos - x' sin below the partner, x cos + x' sin above
+  float sgn128[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const unsigned long long sb = lane < 16 ? P.sign_lo : P.sign_hi;
+    sgn128[e] = (P.rotate ? (((sb >> ((4 * lane + e) & 63)) & 1ull) ? -1.f : 1.f) : 1.f) * (P.rotate ? 1.0f / 128.0f : 1.f);
+  }
   // the warp's 16 tokens: lane i < 16 fetches token i's stream word and position; every lane then
   // loads its 8 bytes of all 16 anchor rows, and the records of the tokens with a residual, before
   // any arithmetic (the loads do not wait on one another)
@@ -972,44 +986,28 @@ __global__ void __launch_bounds__(128) akv_rope_logits_kernel(const RopeParams P
         float cr[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e)
-          cr[e] = fmaf(half_lo(smn[i]), code_level((cbyte[i] >> (2 * e)) & 3u, P.lloyd), half_hi(smn[i]));
-        if (P.rotate) {
-          warp_wht128(cr, lane);
-          apply_signs(cr, lane, P.sign_lo, P.sign_hi);
+          cr[e] = fmaf(half_lo(smn[i]), code_level((cbyte[i] >> (2 * e)) & 3u, CODEC), half_hi(smn[i]));
+        if (P.rotate) warp_wht128(cr, lane);
 #pragma unroll
-          for (int e = 0; e < 4; ++e) cr[e] *= (1.0f / 128.0f);
-        }
-#pragma unroll
-        for (int e = 0; e < 4; ++e) x[e] += cr[e];
+        for (int e = 0; e < 4; ++e) x[e] = fmaf(cr[e], sgn128[e], x[e]);
       }
       // RoPE at the token's position: lanes 0-15 hold dims j < 64, lanes 16-31 their partners j + 64;
       // the two halves each evaluate two of the four pairs' angles and trade them
-      float sn[4], cs[4];
+      float sa[2], ca[2], sb[2], cb[2];
+      __sincosf((float)(uint32_t)(((unsigned long long)p * tn0) >> 40) * (6.2831853071795865f / 16777216.0f), &sa[0], &ca[0]);
+      __sincosf((float)(uint32_t)(((unsigned long long)p * tn1) >> 40) * (6.2831853071795865f / 16777216.0f), &sa[1], &ca[1]);
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int e = (lane < 16 ? 0 : 2) + h;
-        const unsigned long long ph = (unsigned long long)p * turn[(4 * lane + e) & 63];
-        __sincosf((float)(uint32_t)(ph >> 40) * (6.2831853071795865f / 16777216.0f), &sn[e], &cs[e]);
-        const int eo = (lane < 16 ? 2 : 0) + h;
-        sn[eo] = 0.f;
-        cs[eo] = 0.f;
+      for (int h = 0; h < 2; ++h) {  // the partner half's two angles
+        sb[h] = __shfl_xor_sync(0xffffffffu, sa[h], 16);
+        cb[h] = __shfl_xor_sync(0xffffffffu, ca[h], 16);
       }
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {  // lanes < 16 receive pairs 2, 3; lanes >= 16 pairs 0, 1
-        const float so = __shfl_xor_sync(0xffffffffu, lane < 16 ? sn[h] : sn[2 + h], 16);
-        const float co = __shfl_xor_sync(0xffffffffu, lane < 16 ? cs[h] : cs[2 + h], 16);
-        if (lane < 16) {
-          sn[2 + h] = so;
-          cs[2 + h] = co;
-        } else {
-          sn[h] = so;
-          cs[h] = co;
-        }
-      }
+      // pair e of this lane: pairs 0, 1 from the lower half's angles, pairs 2, 3 from the upper half's
+      const float sn[4] = {low ? sa[0] : sb[0], low ? sa[1] : sb[1], low ? sb[0] : sa[0], low ? sb[1] : sa[1]};
+      const float cs[4] = {low ? ca[0] : cb[0], low ? ca[1] : cb[1], low ? cb[0] : ca[0], low ? cb[1] : ca[1]};
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const float xp = __shfl_xor_sync(0xffffffffu, x[e], 16);
-        y[e] = lane < 16 ? fmaf(x[e], cs[e], -xp * sn[e]) : fmaf(x[e], cs[e], xp * sn[e]);
+        y[e] = fmaf(x[e], cs[e], rsgn * xp * sn[e]);
       }
     }
     *reinterpret_cast<float4*>(&ys[16 * warp + i][4 * lane]) = make_float4(y[0], y[1], y[2], y[3]);
@@ -2087,8 +2085,8 @@ DecodeFn decode_kernel(int codec, int rope) {
   return codec ? akv_decode_kernel<GS, 1, 0> : akv_decode_kernel<GS, 0, 0>;
 }
 template <int GS>
-RopeFn rope_kernel() {
-  return akv_rope_logits_kernel<GS>;
+RopeFn rope_kernel(int codec) {
+  return codec ? akv_rope_logits_kernel<GS, 1> : akv_rope_logits_kernel<GS, 0>;
 }
 template <int GS>
 ScoreFn score_kernel() {
@@ -2287,9 +2285,11 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
       R.turn[j] = (unsigned long long)std::ldexp(
           std::pow((double)p.rope_theta, -2.0 * (double)j / 128.0) / 6.283185307179586476925, 64);
     cfg.gridDim = dim3((unsigned)(units * P.n_ch), 1, 1);
-    e = cudaLaunchKernelEx(&cfg, rope_kernel<GS>(), R);
+    e = cudaLaunchKernelEx(&cfg, rope_kernel<GS>(codec), R);
   } else {
+    cfg.dynamicSmemBytes = n_sch ? (size_t)SCH * 256 : 0;  // a suffix chunk's value rows
     e = cudaLaunchKernelEx(&cfg, score_kernel<GS>(), S);
+    cfg.dynamicSmemBytes = 0;
   }
   if (e != cudaSuccess) return (int)e;
   if (ev_scores && (e = cudaEventRecord(ev_scores, cfg.stream)) != cudaSuccess) return (int)e;
