@@ -25,10 +25,11 @@ def dev():
     return torch.device("cuda:0")
 
 
-def _case(dev, lens, H, G, sel, anchor_frac=0.02, W=32, rotate=True, seed=3, check_decode=True):
+def _case(dev, lens, H, G, sel, anchor_frac=0.02, W=32, rotate=True, seed=3, check_decode=True, extra=None):
     B = len(lens)
+    extra = extra or {}  # further Params flags (codec, RoPE at decode)
     p = akv.Params(batch=B, n_kv_heads=H, n_q_heads=H * G, anchor_frac=anchor_frac, res_frac_k=0.0,
-                   res_frac_v=0.0, window=W, seed=seed, rot_seed=seed + 1, rotate=rotate)
+                   res_frac_v=0.0, window=W, seed=seed, rot_seed=seed + 1, rotate=rotate, **extra)
     K, V = gen.clustered_batch(B, H, lens, seed=seed)
     Q = gen.observation_queries(K, lens, W * G, seed=seed + 2)
     a_bytes, w_bytes = akv.akv_cache_size_select(p, sel, lens)
@@ -39,7 +40,7 @@ def _case(dev, lens, H, G, sel, anchor_frac=0.02, W=32, rotate=True, seed=3, che
     torch.cuda.synchronize()
     got = oracle.unpack_arena(arena.cpu().numpy())
     want = oracle.encode_select(K, V, Q, lens, H, anchor_frac, W, sel.theta, sel.rho, sel.kappa, p.seed, p.rot_seed,
-                                rotate)
+                                rotate, lloyd=p.lloyd)
     assert len(got) == len(want)
     for u, (g, w) in enumerate(zip(got, want)):
         assert (g.S, g.k, g.nk, g.nv) == (w.S, w.k, w.nk, w.nv), u
@@ -58,7 +59,7 @@ def _case(dev, lens, H, G, sel, anchor_frac=0.02, W=32, rotate=True, seed=3, che
         dk = min(0.999, sum(w.nk for w in want) / sum(w.S for w in want))
         dv = min(0.999, sum(w.nv for w in want) / sum(w.S for w in want))
         p_dens = akv.Params(batch=B, n_kv_heads=H, n_q_heads=H * G, anchor_frac=anchor_frac, res_frac_k=dk,
-                            res_frac_v=dv, window=W, seed=seed, rot_seed=seed + 1, rotate=rotate)
+                            res_frac_v=dv, window=W, seed=seed, rot_seed=seed + 1, rotate=rotate, **extra)
         for pd, sm in ((p_dens, 1.0), (p, 1.0 / np.sqrt(128.0))):
             out, out32 = decode_on_gpu(torch, pd, lens, arena, q, sm)
             check_outputs(out, out32, oracle_decode(pd, got, q, sm), where=f"select lens={lens} G={G} sm={sm:.3f}")
@@ -102,3 +103,10 @@ def test_select_8b_32k_shape(dev):
     the pooled budget over eight heads at full context (encode bytes only; the decode of such
     caches is covered by the smaller cases)."""
     _case(dev, [32768], 8, 4, akv.SelectParams(theta=0.05, rho=0.7, kappa=7), check_decode=False)
+
+
+def test_select_with_rope_positions_and_the_lloyd_max_codec(dev):
+    """The full selection writing a RoPE arena (the stored tokens' positions) with the Lloyd-Max
+    codec: bit-exact encode, then the RoPE decode against the oracle over the read-back units."""
+    _case(dev, [3000, 1500], 2, 4, akv.SelectParams(theta=0.06, rho=0.7, kappa=7), seed=11,
+          extra=dict(rope=True, lloyd=True))

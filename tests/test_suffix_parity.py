@@ -64,6 +64,11 @@ def test_suffix_decode_scales_and_full_capacity(dev, sm_scale):
     _run(dev, p, [4096, 1500], [128, 127], 128, sm_scale=sm_scale, where=f"suffix sm={sm_scale:.3f}")
 
 
+def test_suffix_with_the_lloyd_max_codec(dev):
+    p = akv.Params(batch=3, n_kv_heads=2, n_q_heads=16, seed=19, lloyd=True)
+    _run(dev, p, [2000, 4500, 700], [17, 64, 130], 160, where="suffix lloyd")
+
+
 def test_suffix_logits_far_above_the_anchor_reference(dev):
     """Suffix keys scaled up so their logits exceed every anchor score by far: the compressed part
     is rescaled to the suffix's maximum in the combine (and carries almost no weight)."""
