@@ -84,7 +84,7 @@ def test_many_units_cta_counts(dev, debug_controls):
 
 @pytest.mark.parametrize("H,G", [(1, 1), (2, 4)])
 def test_tiny_encoded_config(dev, H, G):
-    """configs[0]-shaped case (S=4096, one KV head, G=1) and a 2-head G=4 variant, encoded on
+    """The tiny workload's shape (S = 4096, one KV head, G = 1) and a 2-head G = 4 variant, encoded on
     the GPU: clustered keys and values with real residual structure, where the key-residual
     products need every bit of their fp32 accumulation at sm_scale = 1."""
     S = 4096
