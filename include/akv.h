@@ -480,13 +480,14 @@ akv_status akv_decode_workspace_size_suffix(const akv_params* p, const int32_t* 
  * for request b with n = suffix->len[b] suffix tokens,
  *     out = sum_{i < S_b} w_i x^V_i + sum_{t < n} w_{S_b + t} V_suf[t],
  *     w = softmax over the S_b + n logits sm_scale q . x^K_i and sm_scale q . K_suf[t].
- * suffix NULL is akv_decode_attn.  The score launch also scores each chunk of
- * 64 suffix tokens and sums its values under the chunk's own maximum; the unit's
- * combine rescales those partials to the common maximum (one softmax, exactly).
+ * suffix NULL is akv_decode_attn.  A third launch scores each chunk of 64 suffix
+ * tokens and sums its values under the chunk's own maximum; the unit's combine
+ * rescales those partials to the common maximum (one softmax, exactly).
  *   ws : >= akv_decode_workspace_size_suffix(p, ctx_lens_host, suffix->cap)
  * Errors: those of akv_decode_attn, and AKV_ERR_INVALID for a suffix with null
- * or misaligned pointers (K, V 16-byte aligned; len 4-byte) or cap out of range;
- * AKV_ERR_UNSUPPORTED for a suffix with AKV_FLAG_ROPE (not built).
+ * or misaligned pointers (K, V 16-byte aligned; len 4-byte) or cap out of range.
+ * With AKV_FLAG_ROPE the suffix keys are pre-RoPE too: suffix token t of request b sits at
+ * position S_b + t and is turned there before it is scored.
  * Lengths above cap are taken as cap.
  */
 akv_status akv_decode_attn_suffix(const akv_params* p, const int32_t* ctx_lens_host, const void* arena,

@@ -699,8 +699,6 @@ akv_status akv_decode_attn_suffix(const akv_params* p, const int32_t* ctx_lens_h
   if (arena_bytes < L.total_bytes) return fail(AKV_ERR_TOO_SMALL, "arena shorter than akv_cache_size");
   if (!std::isfinite(sm_scale)) return fail(AKV_ERR_INVALID, "sm_scale must be finite");
   DecodeSuffix sfx;
-  if (suffix && (p->flags & AKV_FLAG_ROPE))
-    return fail(AKV_ERR_UNSUPPORTED, "a dense suffix with RoPE at decode is not supported");
   if (suffix) {
     if (!suffix->K || !suffix->V || !suffix->len) return fail(AKV_ERR_INVALID, "suffix: null K, V or len");
     if (((uintptr_t)suffix->K % 16) || ((uintptr_t)suffix->V % 16) || ((uintptr_t)suffix->len % 4))

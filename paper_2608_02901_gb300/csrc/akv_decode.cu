@@ -116,6 +116,8 @@ struct ScoreParams {
   const int32_t* suf_len;
   float* suf_part;
   int suf_cap, n_sch;
+  // RoPE at decode (the suffix launch): suffix token t of a unit sits at position S + t
+  unsigned long long turn[64];  // theta_j / (2 pi) as a 64-bit binary fraction of a turn
 };
 
 // The RoPE logits launch (AKV_FLAG_ROPE): every stored token's logit per head.
@@ -557,8 +559,8 @@ __device__ __forceinline__ void load_row(const float* p, float (&out)[GS]) {
 // the same permuted k order as the anchor chunks), p = 2^(s - m_c) under the chunk's own maximum
 // m_c, then o[g][d] = sum_t p_t[g] V[t][d] (thread d) and l[g] = sum_t p_t[g] into the chunk's
 // partial slot.  Chunks at or past the request's length write nothing (the combine reads the
-// chunks below it only).
-template <int GS>
+// chunks below it only).  ROPE: the keys are pre-RoPE and turn to positions S + t first.
+template <int GS, bool ROPE>
 __device__ __forceinline__ void suffix_chunk(const ScoreParams& P, int u, int sc) {
   __shared__ float ps[SCH][8];
   __shared__ float wm[4][8];
@@ -597,10 +599,61 @@ __device__ __forceinline__ void suffix_chunk(const ScoreParams& P, int u, int sc
     hi[j] = ldg_stream(Kr + (size_t)rb * 256 + 16 * cc);
   }
   float dd[4] = {0.f, 0.f, 0.f, 0.f};
+  if constexpr (ROPE) {
+    // RoPE at positions S + t: a thread's chunks c4 + 4 j (j < 2) and c4 + 4 j + 8 hold the two
+    // members of pairs (d, d + 64), so each row turns in registers; the turned keys enter the
+    // products as bf16 high and low parts
+    const uint32_t S_u = (uint32_t)unit_desc(P.arena, u)->len;
+    uint4 kr[2][4];  // [row ra / rb][chunk j]: the loaded rows
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    mma_bf16(dd, lo[j].x, hi[j].x, lo[j].y, hi[j].y, bq[2 * j].x, bq[2 * j].y);
-    mma_bf16(dd, lo[j].z, hi[j].z, lo[j].w, hi[j].w, bq[2 * j + 1].x, bq[2 * j + 1].y);
+    for (int j = 0; j < 4; ++j) {
+      kr[0][j] = lo[j];
+      kr[1][j] = hi[j];
+    }
+    uint32_t khi[2][4][4], klo[2][4][4];  // [row][chunk][bf16 pair]
+#pragma unroll
+    for (int rr = 0; rr < 2; ++rr) {
+      const uint32_t p = S_u + (uint32_t)(rr ? rb : ra);
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const uint32_t* wa = reinterpret_cast<const uint32_t*>(&kr[rr][j]);
+        const uint32_t* wb = reinterpret_cast<const uint32_t*>(&kr[rr][j + 2]);
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          float ya[2], yb[2];
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            const int dim = 8 * (4 * j + c4) + 2 * w + hh;  // < 64; its partner is dim + 64
+            const float xa = __bfloat162float(__ushort_as_bfloat16((unsigned short)(hh ? wa[w] >> 16 : wa[w] & 0xFFFFu)));
+            const float xb = __bfloat162float(__ushort_as_bfloat16((unsigned short)(hh ? wb[w] >> 16 : wb[w] & 0xFFFFu)));
+            float sn, cs;
+            __sincosf((float)(uint32_t)(((unsigned long long)p * P.turn[dim]) >> 40) * (6.2831853071795865f / 16777216.0f), &sn, &cs);
+            ya[hh] = fmaf(xa, cs, -xb * sn);
+            yb[hh] = fmaf(xb, cs, xa * sn);
+          }
+          __nv_bfloat162 ha = __floats2bfloat162_rn(ya[0], ya[1]), hb = __floats2bfloat162_rn(yb[0], yb[1]);
+          const float2 fa = __bfloat1622float2(ha), fb = __bfloat1622float2(hb);
+          __nv_bfloat162 la = __floats2bfloat162_rn(ya[0] - fa.x, ya[1] - fa.y), lb = __floats2bfloat162_rn(yb[0] - fb.x, yb[1] - fb.y);
+          khi[rr][j][w] = *reinterpret_cast<const uint32_t*>(&ha);
+          khi[rr][j + 2][w] = *reinterpret_cast<const uint32_t*>(&hb);
+          klo[rr][j][w] = *reinterpret_cast<const uint32_t*>(&la);
+          klo[rr][j + 2][w] = *reinterpret_cast<const uint32_t*>(&lb);
+        }
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      mma_bf16(dd, khi[0][j][0], khi[1][j][0], khi[0][j][1], khi[1][j][1], bq[2 * j].x, bq[2 * j].y);
+      mma_bf16(dd, khi[0][j][2], khi[1][j][2], khi[0][j][3], khi[1][j][3], bq[2 * j + 1].x, bq[2 * j + 1].y);
+      mma_bf16(dd, klo[0][j][0], klo[1][j][0], klo[0][j][1], klo[1][j][1], bq[2 * j].x, bq[2 * j].y);
+      mma_bf16(dd, klo[0][j][2], klo[1][j][2], klo[0][j][3], klo[1][j][3], bq[2 * j + 1].x, bq[2 * j + 1].y);
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      mma_bf16(dd, lo[j].x, hi[j].x, lo[j].y, hi[j].y, bq[2 * j].x, bq[2 * j].y);
+      mma_bf16(dd, lo[j].z, hi[j].z, lo[j].w, hi[j].w, bq[2 * j + 1].x, bq[2 * j + 1].y);
+    }
   }
   const int g0 = 2 * c4;
   float sv[2][2];
@@ -653,15 +706,24 @@ __device__ __forceinline__ void suffix_chunk(const ScoreParams& P, int u, int sc
   }
 }
 
-// Grid: per unit, n_ch anchor chunks then n_sch dense-suffix chunks.
+// The dense suffix's chunks with RoPE at decode (grid: units x n_sch), a launch of its own after
+// the RoPE logits launch.
 template <int GS>
+__global__ void __launch_bounds__(128) akv_suffix_kernel(const ScoreParams P) {
+  suffix_chunk<GS, true>(P, blockIdx.x / P.n_sch, blockIdx.x % P.n_sch);
+}
+
+// Grid: per unit, n_ch anchor chunks, then (SUF) n_sch dense suffix chunks.
+template <int GS, bool SUF>
 __global__ void __launch_bounds__(128) akv_scores_kernel(const ScoreParams P) {
   __shared__ float wmax[4][8];
-  const int per = P.n_ch + P.n_sch;
+  const int per = P.n_ch + (SUF ? P.n_sch : 0);
   const int u = blockIdx.x / per, ch = blockIdx.x % per;
-  if (ch >= P.n_ch) {
-    suffix_chunk<GS>(P, u, ch - P.n_ch);
-    return;
+  if constexpr (SUF) {
+    if (ch >= P.n_ch) {
+      suffix_chunk<GS, false>(P, u, ch - P.n_ch);
+      return;
+    }
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, r8 = lane >> 2, c4 = lane & 3;
   const akv_unit_desc* d = unit_desc(P.arena, u);
@@ -822,7 +884,8 @@ __device__ void combine_unit(const DecodeParams& P, int u, int first, int nseg, 
       if (len > 0) {
         // the compressed part's reference m (the unit's largest anchor score), the common maximum
         // M over it and the chunks' maxima, and every part rescaled to M
-        const int nch = (unit_desc(P.arena, u)->n_anchors + CHA - 1) / CHA;
+        // (with RoPE at decode: the chunk maxima are those of every token's logit)
+        const int nch = P.lg ? (unit_desc(P.arena, u)->len + 63) / 64 : (unit_desc(P.arena, u)->n_anchors + CHA - 1) / CHA;
         float m = -INFINITY;
         for (int ch = lane; ch < nch; ch += 32) m = fmaxf(m, P.cmax[((size_t)u * P.n_ch + ch) * GS + h]);
         m = warp_max(m);
@@ -2089,8 +2152,12 @@ RopeFn rope_kernel(int codec) {
   return codec ? akv_rope_logits_kernel<GS, 1> : akv_rope_logits_kernel<GS, 0>;
 }
 template <int GS>
-ScoreFn score_kernel() {
-  return akv_scores_kernel<GS>;
+ScoreFn score_kernel(bool suffix) {
+  return suffix ? akv_scores_kernel<GS, true> : akv_scores_kernel<GS, false>;
+}
+template <int GS>
+ScoreFn suffix_kernel() {
+  return akv_suffix_kernel<GS>;
 }
 
 // Launch configuration per (device, G, layout shape): computed once, then reused, so that a
@@ -2160,10 +2227,6 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   const int drop = g_debug_withhold.load(std::memory_order_relaxed);
   const int codec = (p.flags & AKV_FLAG_LLOYD) ? 1 : 0;
   const int rope = (p.flags & AKV_FLAG_ROPE) ? 1 : 0;
-  if (rope && sfx.K) {
-    *why = "a dense suffix with RoPE at decode is not supported";
-    return -1;
-  }
   const LaunchKey key{dev, L.G, codec, rope, units, L.max_len, L.max_k, ctas, (long long)(max_density(L) * 1e6),
                       (long long)(max_anchor_density(L) * 1e6), ttot};
   Plan pl;
@@ -2253,7 +2316,7 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   S.sign_lo = P.sign_lo;
   S.sign_hi = P.sign_hi;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(units * (P.n_ch + n_sch)), 1, 1);
+  cfg.gridDim = dim3((unsigned)(units * P.n_ch), 1, 1);
   cfg.blockDim = dim3(128, 1, 1);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = (cudaStream_t)stream;
@@ -2286,9 +2349,18 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
           std::pow((double)p.rope_theta, -2.0 * (double)j / 128.0) / 6.283185307179586476925, 64);
     cfg.gridDim = dim3((unsigned)(units * P.n_ch), 1, 1);
     e = cudaLaunchKernelEx(&cfg, rope_kernel<GS>(codec), R);
+    for (int j = 0; j < 64; ++j) S.turn[j] = R.turn[j];
+    if (e == cudaSuccess && n_sch) {  // the suffix chunks, keys turned to positions S + t
+      cfg.gridDim = dim3((unsigned)(units * n_sch), 1, 1);
+      cfg.dynamicSmemBytes = (size_t)SCH * 256;  // a chunk's value rows
+      e = cudaLaunchKernelEx(&cfg, suffix_kernel<GS>(), S);
+      cfg.dynamicSmemBytes = 0;
+    }
   } else {
-    cfg.dynamicSmemBytes = n_sch ? (size_t)SCH * 256 : 0;  // a suffix chunk's value rows
-    e = cudaLaunchKernelEx(&cfg, score_kernel<GS>(), S);
+    // the suffix chunks (if any) share the grid with the anchor chunks
+    cfg.gridDim = dim3((unsigned)(units * (P.n_ch + n_sch)), 1, 1);
+    cfg.dynamicSmemBytes = n_sch ? (size_t)SCH * 256 : 0;
+    e = cudaLaunchKernelEx(&cfg, score_kernel<GS>(n_sch > 0), S);
     cfg.dynamicSmemBytes = 0;
   }
   if (e != cudaSuccess) return (int)e;

@@ -228,9 +228,11 @@ def test_entry_points_validate_before_any_launch():
     bad = akv.Params(batch=1, n_kv_heads=1, n_q_heads=1).c()
     bad.rope_theta = 10000.0
     assert L.akv_cache_size(sp(bad), lp, sp(sz), None) == akv.AKV_ERR_INVALID
+    # a suffix with RoPE: validated like any other (a short workspace is refused before any launch)
+    ws_r = akv.akv_decode_workspace_size(akv.Params(batch=1, n_kv_heads=1, n_q_heads=1, rope=True), lens, 1000)
     st = L.akv_decode_attn_suffix(sp(pr), lp, 0x1000, sz.value, 256, 256, None, 1.0,
-                                  sp(S(0x4000, 0x5000, 0x6000, 1000)), 0x3000, 1 << 40, None)
-    assert st == akv.AKV_ERR_UNSUPPORTED
+                                  sp(S(0x4000, 0x5000, 0x6000, 1000)), 0x3000, ws_r - 1, None)
+    assert st == akv.AKV_ERR_TOO_SMALL
 
 
 def test_decode_debug_controls_validate():

@@ -47,7 +47,8 @@ def _run(dev, p, lens, suf_lens, cap, sm_scale=1.0, seed=5, qseed=17, key_scale=
     akv.akv_decode_attn(p, lens, arena, qt, out, out32, sm_scale=sm_scale, suffix=sfx)
     torch.cuda.synchronize()
     ref = oracle.attend_suffix([oracle_unit(u) for u in units], q.reshape(p.n_units, p.G, 128), p.G, H, sm_scale,
-                               p.rot_seed, ks, vs, suf_lens, p.rotate, lloyd=p.lloyd).reshape(p.batch, p.n_q_heads, 128)
+                               p.rot_seed, ks, vs, suf_lens, p.rotate, lloyd=p.lloyd,
+                               rope_theta=p.rope_theta if p.rope else 0.0).reshape(p.batch, p.n_q_heads, 128)
     return check_outputs(out.float().cpu().numpy(), out32.cpu().numpy(), ref, where=where)
 
 
@@ -67,6 +68,14 @@ def test_suffix_decode_scales_and_full_capacity(dev, sm_scale):
 def test_suffix_with_the_lloyd_max_codec(dev):
     p = akv.Params(batch=3, n_kv_heads=2, n_q_heads=16, seed=19, lloyd=True)
     _run(dev, p, [2000, 4500, 700], [17, 64, 130], 160, where="suffix lloyd")
+
+
+@pytest.mark.parametrize("G", [1, 4, 8])
+def test_suffix_with_rope_at_decode(dev, G):
+    """Pre-RoPE suffix keys turned to positions S_b + t (after the request's compressed tokens),
+    in the same softmax as the RoPE-decoded prefix; ragged lengths, several chunks."""
+    p = akv.Params(batch=3, n_kv_heads=2, n_q_heads=2 * G, seed=23, rope=True, rope_theta=10000.0)
+    _run(dev, p, [2500, 700, 5000], [0, 65, 150], 150, where=f"suffix rope G={G}")
 
 
 def test_suffix_logits_far_above_the_anchor_reference(dev):
