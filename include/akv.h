@@ -423,14 +423,19 @@ akv_status akv_decode_workspace_size(const akv_params* p, const int32_t* ctx_len
  * over all S_b positions (no mask), with x^ reconstructed per Eq. 3.
  *
  *   arena     : device, as written by akv_encode or copied from akv_cache_pack_host
- *               for the same (p, ctx_lens_host)
+ *               for the same (p, ctx_lens_host), or by akv_encode_select
+ *   arena_bytes : the arena's whole size (akv_cache_size, or akv_cache_size_select
+ *               for a full-selection arena): the score launch reads anchor rows
+ *               through a tensor map of exactly this many bytes, and a unit whose
+ *               anchor rows lie outside it gets NaN outputs
  *   q         : device bf16 [B][H_q][128]
  *   out       : device bf16 [B][H_q][128], round-to-nearest-even of the fp32 result
  *   out_f32   : device fp32 [B][H_q][128] or NULL
  *   ws        : device workspace, 256-byte aligned, of >= akv_decode_workspace_size
  *               bytes; calls that overlap on the GPU need separate workspaces
- * Two launches: the anchor scores of every unit, then the decode itself, one CTA
- * per SM over equal shares of all units' tile blocks.
+ * Two launches: the anchor scores of every unit (persistent, tensor cores with
+ * tensor-memory accumulators, tiles of 128 anchors brought by tensor copies), then
+ * the decode itself, one CTA per SM over equal shares of all units' tile blocks.
  * Errors: AKV_ERR_INVALID (null/misaligned pointers, bad sizes), AKV_ERR_TOO_SMALL
  * (arena or workspace short), AKV_ERR_UNSUPPORTED (no shared-memory plan fits),
  * AKV_ERR_CUDA (launch failure).

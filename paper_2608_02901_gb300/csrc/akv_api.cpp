@@ -713,7 +713,7 @@ akv_status akv_decode_attn_suffix(const akv_params* p, const int32_t* ctx_lens_h
   if (ws_bytes < decode_ws_layout(L, sfx.cap).total)
     return fail(AKV_ERR_TOO_SMALL, "decode workspace shorter than akv_decode_workspace_size(_suffix)");
   std::string why;
-  int err = launch_decode(L, *p, arena, q, out, out_f32, sm_scale, sfx, ws, (void*)stream, &why);
+  int err = launch_decode(L, *p, arena, arena_bytes, q, out, out_f32, sm_scale, sfx, ws, (void*)stream, &why);
   if (err == -1) return fail(AKV_ERR_UNSUPPORTED, why);
   if (err) return fail(AKV_ERR_CUDA, std::string("decode launch failed: ") + cuda_error_string(err) + " " + why);
   return AKV_OK;

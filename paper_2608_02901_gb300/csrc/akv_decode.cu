@@ -1,14 +1,16 @@
 // Decode attention read directly from the AnchorKV compressed cache (Eq. 3 folded into
 // Eq. 4: no key or value row is ever rebuilt in memory).  Two launches per call, in stream
-// order:
+// order (three with a dense suffix, whose chunks take a launch of their own between them):
 //
-// 1. akv_scores_kernel.  The anchor scores S_A[a][g] = q_g . k_a of every anchor of every
-//    unit, once per anchor (Eq. 2-3), bf16 tensor cores, in log2 units with sm_scale folded
-//    in, into the workspace, with the largest score per query head of each chunk of 64
-//    anchors.  It streams the anchor keys, a fifth of the compressed bytes, at full width.
-//    Its first chunk of each unit also writes the unit's query header (the rotated query
-//    q' = H(s o q)/128 of Appendix A.1 Eq. 12, its sums per head, and q' as tensor-core
-//    fragments for the key residuals) and zeroes the unit's arrival counter.
+// 1. akv_scores_tc_kernel.  The anchor scores S_A[a][g] = q_g . k_a of every anchor of every
+//    unit, once per anchor (Eq. 2-3), in log2 units with sm_scale folded in, into the
+//    workspace, with the largest score per query head of each chunk of 64 anchors: tiles of
+//    128 anchors brought by tensor copies (TMA) into shared memory, products by tcgen05.mma
+//    into tensor memory, one persistent warp-specialised CTA per SM.  It streams the anchor
+//    keys, a fifth of the compressed bytes.  It also writes each unit's query header (the
+//    rotated query q' = H(s o q)/128 of Appendix A.1 Eq. 12, its sums per head, and q' as
+//    tensor-core fragments for the key residuals) and zeroes the unit's arrival counter.
+//    (With RoPE at decode akv_rope_logits_kernel takes its place.)
 //
 // 2. akv_decode_kernel.  Persistent: one CTA per SM.  The tile blocks of all units, in unit
 //    order, are split into equal contiguous ranges, one per CTA (stream-K): a unit's tiles may
@@ -43,6 +45,8 @@
 // a logit exceeds m by more than 2^120, which is flagged); every CTA of a unit takes the same
 // m, so partial sums combine by plain addition.  Every wait on an mbarrier is bounded; a wait
 // that runs out marks the CTA failed and the outputs of its units NaN.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
@@ -73,7 +77,21 @@ constexpr int LCH = T / (WPG * 32); // consecutive stored tokens per lane
 static_assert(LCH == 8, "a lane's tokens are one byte of a bitmap word");
 constexpr int NSG = 4;              // tiles a group has in flight at most (its stage descriptors)
 constexpr int kMaxGrid = 256;       // CTAs of the decode launch at most
-constexpr int CHA = 64;             // anchors per score-kernel CTA (4 warps x 16 rows)
+constexpr int CHA = 64;             // anchors per chunk maximum of the score launch
+// Score launch on tensor cores: a tile of 128 anchors (TMEM lanes) x 16 query rows (columns),
+// anchor rows and query rows brought by tensor copies into two 128-byte halves each
+constexpr int kScTile = 128;
+constexpr uint32_t kScHalfA = kScTile * 128;             // 128 rows x 64 bf16
+constexpr uint32_t kScHalfB = 16 * 128;                  // 16 rows x 64 bf16
+constexpr uint32_t kScStage = 2 * kScHalfA + 2 * kScHalfB;  // 36 KB, a multiple of 1024
+constexpr int kScStages = 6;                             // tiles in flight (one CTA per SM)
+constexpr int kScThreads = 192;  // warps 0-3 epilogue (TMEM lanes 32 w ..), 4 copies and products, 5 query headers
+constexpr int kScMaxTiles = 512;  // tiles of one CTA (its table in shared memory); the grid grows past this
+constexpr uint32_t kScDynSmem = kScStages * kScStage + 1024;  // + alignment of the first stage
+constexpr uint32_t kScTmemCols = 32;                     // two accumulators of 16 fp32 columns
+// Instruction descriptor of kind::f16: fp32 accumulator (bits 4-5 = 1), bf16 A and B (7-9 = 1,
+// 10-12 = 1), both K-major (15, 16 = 0), N / 8 (17-22), M / 16 (24-28).
+constexpr uint32_t kScIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((16u >> 3) << 17) | ((uint32_t)(kScTile >> 4) << 24);
 constexpr int kOvl = 32;            // a tile's entries per overflow list (value records, anchor-value runs)
 constexpr int kRingSlack = 4096;    // shared memory after the ring: the masked rows of the last
                                     // 16-row block of staged anchor values are read from here
@@ -116,6 +134,8 @@ struct ScoreParams {
   const int32_t* suf_len;
   float* suf_part;
   int suf_cap, n_sch;
+  int units, n_t;  // units; tiles of kScTile anchors per unit (the largest unit's)
+  long long arena_rows;  // 256-byte rows of the arena the anchor map covers
   // RoPE at decode (the suffix launch): suffix token t of a unit sits at position S + t
   unsigned long long turn[64];  // theta_j / (2 pi) as a 64-bit binary fraction of a turn
 };
@@ -228,7 +248,73 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
                ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
                : "memory");
 }
+// ---- tensor copies (TMA), tensor memory and the fifth-generation tensor-core MMA (tcgen05) ----
+// Tiled 2-D tensor copy global -> this CTA's shared memory at element column x (a multiple of 8
+// bf16, so 16-byte aligned) and row y, completing its bytes on the mbarrier.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, int x, int y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+      ::"r"(dst), "l"(tmap), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+// Shared-memory matrix descriptor of a K-major bf16 operand in the 128-byte swizzled layout:
+// rows of 128 bytes (64 elements of K), 8-row groups 1024 bytes apart, 16-byte chunk j of row r
+// at chunk j ^ (r & 7) of the 1024-byte-aligned group.  Bits: start address / 16 (0-13),
+// leading-dimension offset / 16 (16-29, unused by this layout), stride-dimension offset / 16
+// (32-45), descriptor version 1 (46-47), swizzle mode 2 = 128 bytes (61-63).  A K step of 16
+// elements advances the start address by 32 bytes; the swizzle applies to the full address.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)1u << 16) | ((uint64_t)(1024u >> 4) << 32) |
+         ((uint64_t)1u << 46) | ((uint64_t)2u << 61);
+}
+// D[tmem] (+)= A[smem] B[smem]^T, kind::f16 (bf16 operands), issued by one thread.
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
+      ::"r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(acc)
+      : "memory");
+}
+// One arrival on the mbarrier once every MMA this thread issued before it has completed.
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+// Tensor-memory columns for this CTA (a whole warp; ncols a power of two >= 32); the address is
+// written to shared memory.  The permit to allocate is given up at once (one allocation per CTA).
+__device__ __forceinline__ void tc_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tc_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+// Eight consecutive 32-bit columns of the calling thread's tensor-memory lane (a whole warp;
+// warp w of the CTA reads lanes 32 (w % 4) .. + 31), waited for before the values are used.
+__device__ __forceinline__ void tc_ld8(uint32_t taddr, float (&v)[8]) {
+  uint32_t r0, r1, r2, r3, r4, r5, r6, r7;
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];\n"
+      "tcgen05.wait::ld.sync.aligned;\n"
+      : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3), "=r"(r4), "=r"(r5), "=r"(r6), "=r"(r7)
+      : "r"(taddr)
+      : "memory");
+  v[0] = __uint_as_float(r0); v[1] = __uint_as_float(r1); v[2] = __uint_as_float(r2); v[3] = __uint_as_float(r3);
+  v[4] = __uint_as_float(r4); v[5] = __uint_as_float(r5); v[6] = __uint_as_float(r6); v[7] = __uint_as_float(r7);
+}
 __device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+// Named barrier of n threads that also returns whether any of them passed a true predicate.
+__device__ __forceinline__ bool named_sync_or(int id, int n, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{ .reg .pred p, q; setp.ne.u32 p, %1, 0; bar.red.or.pred q, %2, %3, p; selp.u32 %0, 1, 0, q; }"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(id), "r"(n)
+      : "memory");
+  return r != 0;
+}
 // Reduction (no return value) into this CTA's shared memory.
 __device__ __forceinline__ void red_local(float* p, float v) {
   asm volatile("red.shared.add.f32 [%0], %1;" ::"r"(smem_u32(p)), "f"(v) : "memory");
@@ -561,13 +647,10 @@ __device__ __forceinline__ void load_row(const float* p, float (&out)[GS]) {
 // partial slot.  Chunks at or past the request's length write nothing (the combine reads the
 // chunks below it only).  ROPE: the keys are pre-RoPE and turn to positions S + t first.
 template <int GS, bool ROPE>
-__device__ __forceinline__ void suffix_chunk(const ScoreParams& P, int u, int sc) {
+__device__ __forceinline__ void suffix_chunk(const ScoreParams& P, int u, int sc, __nv_bfloat16 (*vsm)[128]) {
   __shared__ float ps[SCH][8];
   __shared__ float wm[4][8];
   __shared__ float mc[8];
-  // the chunk's value rows: dynamic shared memory, requested only by launches with a suffix
-  extern __shared__ __align__(16) uint8_t score_dyn[];
-  __nv_bfloat16 (*vsm)[128] = reinterpret_cast<__nv_bfloat16 (*)[128]>(score_dyn);
   const int len = max(0, min(P.suf_len[u / P.n_kv_heads], P.suf_cap));
   const int j0 = sc * SCH;
   if (j0 >= len) return;
@@ -706,105 +789,40 @@ __device__ __forceinline__ void suffix_chunk(const ScoreParams& P, int u, int sc
   }
 }
 
-// The dense suffix's chunks with RoPE at decode (grid: units x n_sch), a launch of its own after
-// the RoPE logits launch.
-template <int GS>
+// The dense suffix's chunks (grid: units x n_sch), a launch of their own after the score or RoPE
+// logits launch (ROPE: the keys are pre-RoPE).
+template <int GS, bool ROPE>
 __global__ void __launch_bounds__(128) akv_suffix_kernel(const ScoreParams P) {
-  suffix_chunk<GS, true>(P, blockIdx.x / P.n_sch, blockIdx.x % P.n_sch);
+  extern __shared__ __align__(16) uint8_t score_dyn[];  // the chunk's value rows
+  suffix_chunk<GS, ROPE>(P, blockIdx.x / P.n_sch, blockIdx.x % P.n_sch,
+                         reinterpret_cast<__nv_bfloat16 (*)[128]>(score_dyn));
 }
 
-// Grid: per unit, n_ch anchor chunks, then (SUF) n_sch dense suffix chunks.
-template <int GS, bool SUF>
-__global__ void __launch_bounds__(128) akv_scores_kernel(const ScoreParams P) {
-  __shared__ float wmax[4][8];
-  const int per = P.n_ch + (SUF ? P.n_sch : 0);
-  const int u = blockIdx.x / per, ch = blockIdx.x % per;
-  if constexpr (SUF) {
-    if (ch >= P.n_ch) {
-      suffix_chunk<GS, false>(P, u, ch - P.n_ch);
-      return;
-    }
-  }
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, r8 = lane >> 2, c4 = lane & 3;
-  const akv_unit_desc* d = unit_desc(P.arena, u);
-  const int k = d->n_anchors;
-  if (ch == 0 && threadIdx.x == 0) P.cnt[u] = 0u;
-  const int a0 = ch * CHA + 16 * warp;
-  float mx0 = -INFINITY, mx1 = -INFINITY;  // heads 2 c4, 2 c4 + 1
-  if (a0 < k) {
-    const size_t qb = qrow_base(u, P.n_kv_heads, P.n_q_heads);
-    uint2 bq[8];
-#pragma unroll
-    for (int ks = 0; ks < 8; ++ks)
-      bq[ks] = r8 < GS ? *reinterpret_cast<const uint2*>(P.q + qb + (size_t)r8 * 128 + 32 * (ks >> 1) + 8 * c4 + 4 * (ks & 1))
-                       : make_uint2(0u, 0u);
-    const uint8_t* AK = P.arena + d->off_anchor_k;
-    const int ra = min(a0 + r8, k - 1), rb = min(a0 + r8 + 8, k - 1);
-    uint4 lo[4], hi[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int cc = 4 * j + c4;
-      lo[j] = ldg_stream(AK + (size_t)ra * 256 + 16 * (cc ^ (ra & 7)));
-      hi[j] = ldg_stream(AK + (size_t)rb * 256 + 16 * (cc ^ (rb & 7)));
-    }
-    float dd[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      mma_bf16(dd, lo[j].x, hi[j].x, lo[j].y, hi[j].y, bq[2 * j].x, bq[2 * j].y);
-      mma_bf16(dd, lo[j].z, hi[j].z, lo[j].w, hi[j].w, bq[2 * j + 1].x, bq[2 * j + 1].y);
-    }
-    float* sa = P.sa + (size_t)u * P.ka_stride * GS;
-    const int g0 = 2 * c4;
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int a = a0 + r8 + 8 * h;
-      if (a < k) {
-        const float s0 = dd[2 * h] * P.scale_log2, s1 = dd[2 * h + 1] * P.scale_log2;
-        if (g0 < GS) {
-          sa[sa_at<GS>(a, g0, P.ka_stride)] = s0;
-          mx0 = fmaxf(mx0, s0);
-        }
-        if (g0 + 1 < GS) {
-          sa[sa_at<GS>(a, g0 + 1, P.ka_stride)] = s1;
-          mx1 = fmaxf(mx1, s1);
-        }
-      }
-    }
-  }
-#pragma unroll
-  for (int o = 4; o < 32; o <<= 1) {
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
-  }
-  if (lane < 4) {
-    wmax[warp][2 * lane] = mx0;
-    wmax[warp][2 * lane + 1] = mx1;
-  }
-  __syncthreads();
-  if (threadIdx.x < GS) {
-    const int g = threadIdx.x;
-    P.cmax[((size_t)u * P.n_ch + ch) * GS + g] = fmaxf(fmaxf(wmax[0][g], wmax[1][g]), fmaxf(wmax[2][g], wmax[3][g]));
-  }
-  if (ch != 0) return;
-  // ---- the unit's query header (chunk 0): rotated query q' = H(s o q) / 128, scaled to log2
-  // units (Appendix A.1, Eq. 12; warp-local Walsh-Hadamard transform), its sums, and the
-  // key-residual mma B fragments: column n = lane / 4 is head n as the fp16 high part (set 0) and
-  // low part (set 1) for GS = 8, else head n % 4 high (n < 4) or low (n >= 4); k pairs (2t, 2t+1)
-  // <-> dims (16 ks + 2t, 16 ks + 2t + 8), (2t+8, 2t+9) <-> (16 ks + 2t + 1, 16 ks + 2t + 9) ----
+// The unit's query header, by one warp: the rotated query q' = H(s o q) / 128 scaled to log2 units
+// (Appendix A.1, Eq. 12; warp-local Walsh-Hadamard transform), its sums, and the key-residual mma
+// B fragments: column n = lane / 4 is head n as the fp16 high part (set 0) and low part (set 1) for
+// GS = 8, else head n % 4 high (n < 4) or low (n >= 4); k pairs (2t, 2t+1) <-> dims
+// (16 ks + 2t, 16 ks + 2t + 8), (2t+8, 2t+9) <-> (16 ks + 2t + 1, 16 ks + 2t + 9).  qs: 8 x 128
+// floats of shared memory for the rotated rows.
+template <int GS>
+__device__ __noinline__ void unit_query_header_warp(const ScoreParams& P, int u, float* qs) {
+  const int lane = threadIdx.x & 31;
   constexpr int NBF = GS == 8 ? 2 : 1;
-  __shared__ __align__(16) float qs[8 * 128];
   uint8_t* H = P.uh + (size_t)u * P.uh_stride;
   float* hq = reinterpret_cast<float*>(H);
   float* hs = hq + GS * 128;
   uint2* hf = reinterpret_cast<uint2*>(hs + 8);
   const size_t qb = qrow_base(u, P.n_kv_heads, P.n_q_heads);
   const float f = P.rotate ? P.scale_log2 * (1.0f / 128.0f) : P.scale_log2;
-  for (int g = warp; g < GS; g += 4) {
-    const uint2 raw = *reinterpret_cast<const uint2*>(P.q + qb + (size_t)g * 128 + 4 * lane);
-    float x[4] = {__bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.x & 0xFFFFu))),
-                  __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.x >> 16))),
-                  __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.y & 0xFFFFu))),
-                  __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw.y >> 16)))};
+  uint2 raw[GS];  // every row's loads in flight at once
+#pragma unroll
+  for (int g = 0; g < GS; ++g) raw[g] = *reinterpret_cast<const uint2*>(P.q + qb + (size_t)g * 128 + 4 * lane);
+#pragma unroll
+  for (int g = 0; g < GS; ++g) {
+    float x[4] = {__bfloat162float(__ushort_as_bfloat16((unsigned short)(raw[g].x & 0xFFFFu))),
+                  __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw[g].x >> 16))),
+                  __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw[g].y & 0xFFFFu))),
+                  __bfloat162float(__ushort_as_bfloat16((unsigned short)(raw[g].y >> 16)))};
     if (P.rotate) {
       apply_signs(x, lane, P.sign_lo, P.sign_hi);
       warp_wht128(x, lane);
@@ -817,10 +835,11 @@ __global__ void __launch_bounds__(128) akv_scores_kernel(const ScoreParams P) {
     const float sg = warp_sum((x[0] + x[1]) + (x[2] + x[3]));
     if (lane == 0) hs[g] = sg;
   }
-  if (threadIdx.x >= GS && threadIdx.x < 8) hs[threadIdx.x] = 0.f;
-  __syncthreads();
+  if (lane >= GS && lane < 8) hs[lane] = 0.f;
+  __syncwarp();  // the rotated rows are in shared memory for every lane
   const int gcol = lane >> 2, cc = lane & 3;
-  for (int idx = warp; idx < NBF * 8; idx += 4) {
+#pragma unroll
+  for (int idx = 0; idx < NBF * 8; ++idx) {
     const int hl = idx >> 3, ks = idx & 7;
     uint2 fk = make_uint2(0u, 0u);
     const int head = GS == 8 ? gcol : (gcol & 3);
@@ -836,6 +855,208 @@ __global__ void __launch_bounds__(128) akv_scores_kernel(const ScoreParams P) {
     }
     hf[(hl * 8 + ks) * 32 + lane] = fk;
   }
+  __syncwarp();  // the next unit's rows may overwrite qs
+}
+
+// Anchor scores on tensor cores (Eq. 2-3: S_A = q . k_a once per anchor).  One persistent CTA per
+// SM takes tiles T = blockIdx.x, + gridDim.x, ... of units x n_t; tile (u, t) is anchors
+// 128 t .. 128 t + 127 of unit u (tile 0 of every unit is taken even when empty).  Warps have
+// roles, coupled only by mbarriers:
+//  * warp 4, lane 0, copies and products: it keeps kScStages tiles in flight (two tensor copies
+//    bring the anchor rows' 128-byte halves, stored with the 16-byte chunks of row a at chunk
+//    j ^ (a & 7), which is the 128-byte swizzled operand layout as it is; two bring the query
+//    rows, swizzled by the copy, with the next 16 - G rows of q or zeros in columns that are not
+//    read), and as each tile lands and one of two TMEM accumulators is free it issues the 8 K steps
+//    of D[128 anchors][16 columns] and commits them to that accumulator's "full" barrier and to the
+//    stage's "free" barrier; the stage of the previous tile is refilled once its products are done;
+//  * warps 0-3, the epilogue: warp w reads TMEM lanes 32 w .. 32 w + 31 (one anchor per thread),
+//    frees the accumulator, writes S_A in log2 units and, after a named barrier of the four warps,
+//    the maxima of the tile's two 64-anchor chunks;
+//  * warp 5 writes the query header of every unit whose tile 0 is this CTA's and zeroes the unit's
+//    arrival counter.
+// Both the copying lane and the epilogue walk the same tiles, from a table of the CTA's tiles that
+// all threads fill at the start (every descriptor load in flight at once).  Every wait is bounded; a CTA whose wait runs out, or that finds a unit's anchor rows
+// outside the arena the map covers, writes +inf as the chunk maxima of all its tiles (the decode's
+// outputs for those units become NaN) and stops.
+template <int GS>
+__global__ void __launch_bounds__(kScThreads) akv_scores_tc_kernel(const __grid_constant__ ScoreParams P,
+                                                                   const __grid_constant__ CUtensorMap tmA,
+                                                                   const __grid_constant__ CUtensorMap tmB) {
+  extern __shared__ __align__(16) uint8_t score_dyn[];
+  __shared__ __align__(8) uint64_t bars[2 * kScStages + 4];  // full[s], free[s], acc_full[b], acc_empty[b]
+  __shared__ uint32_t tmem_sh;
+  __shared__ float wmx[2][4][8];
+  __shared__ int failed_sh;
+  __shared__ int2 tab[kScMaxTiles];  // this CTA's tiles: the unit's anchors, anchor row (-1: outside the map)
+  __shared__ __align__(16) float hdr_q[8 * 128];  // the header warp's rotated query rows
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t sbase = (smem_u32(score_dyn) + 1023u) & ~1023u;
+  auto full = [&](int s) { return smem_u32(bars + s); };
+  auto freed = [&](int s) { return smem_u32(bars + kScStages + s); };
+  auto acc_full = [&](int b) { return smem_u32(bars + 2 * kScStages + b); };
+  auto acc_empty = [&](int b) { return smem_u32(bars + 2 * kScStages + 2 + b); };
+  volatile int* failed = &failed_sh;
+  const int n_tiles = P.units * P.n_t;
+  const int n_my = n_tiles > (int)blockIdx.x ? (n_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+  for (int i = tid; i < n_my && i < kScMaxTiles; i += kScThreads) {  // all descriptors in one round trip
+    const akv_unit_desc* d = unit_desc(P.arena, ((int)blockIdx.x + i * (int)gridDim.x) / P.n_t);
+    const int k = d->n_anchors;
+    const uint64_t off = d->off_anchor_k;
+    tab[i] = make_int2(k, !(off & 255u) && (long long)(off >> 8) + k <= P.arena_rows ? (int)(off >> 8) : -1);
+  }
+  if (tid == 0) {
+    for (int s = 0; s < kScStages; ++s) {
+      mbar_init(full(s), 1);
+      mbar_init(freed(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(acc_full(b), 1);
+      mbar_init(acc_empty(b), 4);  // one arrival per epilogue warp
+    }
+    *failed = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) tc_alloc(smem_u32(&tmem_sh), kScTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_sh;
+
+  // the next of this CTA's tiles that hold anchors (or are a unit's tile 0), from the table: ci is
+  // the next entry to look at; row is the anchor row (-1: outside the map)
+  int ci = 0;
+  const int n_tab = min(n_my, kScMaxTiles);
+  auto next_tile = [&](int& u, int& t, int& k, int& row) {
+    while (ci < n_tab) {
+      const int T = (int)blockIdx.x + ci * (int)gridDim.x;
+      const int2 e = tab[ci++];
+      k = e.x;
+      row = e.y;
+      u = T / P.n_t;
+      t = T % P.n_t;
+      if (t == 0 || t * kScTile < k) return true;
+    }
+    return false;
+  };
+
+  if (warp == 4) {
+    if (lane == 0) {  // ---- copies and products
+      int u, t, k, row0, n_iss = 0, n_mma = 0;
+      auto issue = [&](int j) {  // the tile just found into stage j % kScStages
+        const int s = j % kScStages;
+        const uint32_t st = sbase + (uint32_t)s * kScStage;
+        if (row0 >= 0) {
+          const int row = row0 + t * kScTile;  // 256-byte rows
+          const int qrow = (int)(qrow_base(u, P.n_kv_heads, P.n_q_heads) >> 7);
+          mbar_expect_tx(full(s), kScStage);
+          tma_load_2d(st, &tmA, 0, row, full(s));
+          tma_load_2d(st + kScHalfA, &tmA, 64, row, full(s));
+          tma_load_2d(st + 2 * kScHalfA, &tmB, 0, qrow, full(s));
+          tma_load_2d(st + 2 * kScHalfA + kScHalfB, &tmB, 64, qrow, full(s));
+        } else {
+          mbar_arrive(full(s));  // nothing copied: the epilogue fails the CTA
+        }
+      };
+      bool more = true;
+      while (n_iss < kScStages && (more = next_tile(u, t, k, row0))) issue(n_iss++);
+      for (int j = 0; j < n_iss; ++j) {
+        const int s = j % kScStages, b = j & 1;
+        if (*failed || !mbar_wait(full(s), (uint32_t)(j / kScStages) & 1u) ||
+            !mbar_wait(acc_empty(b), ((uint32_t)(j >> 1) & 1u) ^ 1u)) {
+          *failed = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a = sbase + (uint32_t)s * kScStage, bq = a + 2 * kScHalfA;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {  // K steps of 16: 32 bytes into a half, then the other half
+          const uint32_t ka = (uint32_t)(kk >> 2) * kScHalfA + (uint32_t)(kk & 3) * 32;
+          const uint32_t kb = (uint32_t)(kk >> 2) * kScHalfB + (uint32_t)(kk & 3) * 32;
+          tc_mma(tmem + 16u * (uint32_t)b, sw128_desc(a + ka), sw128_desc(bq + kb), kScIdesc, kk > 0 ? 1u : 0u);
+        }
+        tc_commit(acc_full(b));
+        tc_commit(freed(s));
+        ++n_mma;
+        // refill the previous tile's stage once its products are done (this tile's run meanwhile)
+        if (j > 0 && more && (more = next_tile(u, t, k, row0))) {
+          const int sp = (j - 1) % kScStages;
+          if (!mbar_wait(freed(sp), (uint32_t)((j - 1) / kScStages) & 1u)) {
+            *failed = 1;
+            break;
+          }
+          issue(n_iss++);  // n_iss = j - 1 + kScStages: stage sp
+        }
+      }
+      // (bounded) nothing of this CTA's is left in flight at exit: copies never consumed (after a
+      // failure), and the last commit's arrivals (every earlier one has landed before it)
+      if (*failed)
+        for (int j = n_mma; j < n_iss; ++j) mbar_wait(full(j % kScStages), (uint32_t)(j / kScStages) & 1u);
+      if (n_mma > 0) mbar_wait(freed((n_mma - 1) % kScStages), (uint32_t)((n_mma - 1) / kScStages) & 1u);
+    }
+    __syncwarp();
+  } else if (warp == 5) {  // ---- query headers
+    for (int T = (int)blockIdx.x; T < n_tiles; T += (int)gridDim.x) {
+      if (T % P.n_t) continue;
+      if (lane == 0) P.cnt[T / P.n_t] = 0u;
+      unit_query_header_warp<GS>(P, T / P.n_t, hdr_q);
+    }
+  } else {  // ---- epilogue, warps 0-3
+    int u, t, k, row0;
+    for (int j = 0; next_tile(u, t, k, row0); ++j) {
+      const int b = j & 1;
+      const bool got = mbar_wait_w(acc_full(b), (uint32_t)(j >> 1) & 1u);
+      tc_fence_after();
+      float v[8];
+      tc_ld8(tmem + ((uint32_t)(32 * warp) << 16) + 16u * (uint32_t)b, v);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty(b));  // this warp's lanes of accumulator b are read
+      const bool ok_tile = got && row0 >= 0;
+      const int a = t * kScTile + 32 * warp + lane;
+      const bool ok = ok_tile && a < k;
+      float sc[8];
+#pragma unroll
+      for (int g = 0; g < 8; ++g) sc[g] = v[g] * P.scale_log2;
+      if (ok) {
+        float* sa = P.sa + (size_t)u * P.ka_stride * GS;
+        if constexpr (GS == 8) {
+          *reinterpret_cast<float4*>(sa + (size_t)a * 4) = make_float4(sc[0], sc[1], sc[2], sc[3]);
+          *reinterpret_cast<float4*>(sa + ((size_t)P.ka_stride + a) * 4) = make_float4(sc[4], sc[5], sc[6], sc[7]);
+        } else if constexpr (GS == 4) {
+          *reinterpret_cast<float4*>(sa + (size_t)a * 4) = make_float4(sc[0], sc[1], sc[2], sc[3]);
+        } else if constexpr (GS == 2) {
+          *reinterpret_cast<float2*>(sa + (size_t)a * 2) = make_float2(sc[0], sc[1]);
+        } else {
+          sa[a] = sc[0];
+        }
+      }
+#pragma unroll
+      for (int g = 0; g < GS; ++g) {
+        const float m = warp_max(ok ? sc[g] : -INFINITY);
+        if (lane == 0) wmx[b][warp][g] = m;
+      }
+      // the four warps' maxima are in place; a failure seen by any thread stops all four
+      if (named_sync_or(1, 128, !ok_tile || *failed)) {
+        if (tid == 0) *failed = 1;
+        break;
+      }
+      if (tid < 2 * GS) {
+        const int c = tid / GS, g = tid % GS, ch = 2 * t + c;
+        if (ch * CHA < k) P.cmax[((size_t)u * P.n_ch + ch) * GS + g] = fmaxf(wmx[b][2 * c][g], wmx[b][2 * c + 1][g]);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (*failed) {
+    for (int T2 = (int)blockIdx.x; T2 < n_tiles; T2 += (int)gridDim.x) {
+      const int u = T2 / P.n_t, t = T2 % P.n_t;
+      if (tid < 2 * GS && 2 * t + tid / GS < P.n_ch)
+        P.cmax[((size_t)u * P.n_ch + 2 * t + tid / GS) * GS + tid % GS] = INFINITY;
+    }
+  }
+  if (warp == 0) tc_dealloc(tmem, kScTmemCols);
 }
 
 // ============================ the unit's output ====================================
@@ -2020,6 +2241,7 @@ __global__ void __launch_bounds__(NT, 1) akv_decode_kernel(const DecodeParams P)
 struct DeviceInfo {
   int sms = 0;
   int smem_optin = 0;
+  int smem_sm = 0;  // shared memory per SM
 };
 
 DeviceInfo device_info() {
@@ -2033,6 +2255,7 @@ DeviceInfo device_info() {
   DeviceInfo d;
   cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev);
   cudaDeviceGetAttribute(&d.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  cudaDeviceGetAttribute(&d.smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
   if (dev >= 0 && dev < 64) {
     cache[dev] = d;
     have[dev] = true;
@@ -2070,6 +2293,7 @@ struct Plan {
   DecodeParams P;
   size_t smem = 0;
   int grid = 0;
+  int sms = 0;  // SMs of the device (the score launch: one CTA each)
 };
 
 // Shared-memory carve-up for (R, X, table in shared memory or not); false if the ring
@@ -2141,6 +2365,7 @@ bool make_plan(const Layout& L, int GS, int smem_optin, bool table, Plan* out, s
 
 using DecodeFn = void (*)(const DecodeParams);
 using ScoreFn = void (*)(const ScoreParams);
+using ScoreTcFn = void (*)(const ScoreParams, const CUtensorMap, const CUtensorMap);
 using RopeFn = void (*)(const RopeParams);
 template <int GS>
 DecodeFn decode_kernel(int codec, int rope) {
@@ -2152,12 +2377,40 @@ RopeFn rope_kernel(int codec) {
   return codec ? akv_rope_logits_kernel<GS, 1> : akv_rope_logits_kernel<GS, 0>;
 }
 template <int GS>
-ScoreFn score_kernel(bool suffix) {
-  return suffix ? akv_scores_kernel<GS, true> : akv_scores_kernel<GS, false>;
+ScoreTcFn score_kernel() {
+  return akv_scores_tc_kernel<GS>;
+}
+
+// cuTensorMapEncodeTiled of the driver, found once through the runtime (no link to libcuda).
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static std::once_flag once;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (PFN_cuTensorMapEncodeTiled_v12000)f;
+  });
+  return fn;
+}
+
+// A 2-D map over `rows` rows of 128 bf16 (256 bytes apart) at `base` (16-byte aligned), copied
+// as boxes of 64 elements (one 128-byte half) x box_rows rows; rows past the end read as zero.
+bool encode_row_map(CUtensorMap* m, const void* base, uint64_t rows, uint32_t box_rows, CUtensorMapSwizzle sw) {
+  const PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  if (!enc || rows == 0) return false;
+  const cuuint64_t dims[2] = {128, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {256};
+  const cuuint32_t box[2] = {64, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 template <int GS>
-ScoreFn suffix_kernel() {
-  return akv_suffix_kernel<GS>;
+ScoreFn suffix_kernel(bool rope) {
+  return rope ? akv_suffix_kernel<GS, true> : akv_suffix_kernel<GS, false>;
 }
 
 // Launch configuration per (device, G, layout shape): computed once, then reused, so that a
@@ -2211,7 +2464,7 @@ DecodeWs decode_ws_layout(const Layout& L, int32_t suffix_cap) {
 }
 
 template <int GS>
-int launch_g(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
+int launch_g(const Layout& L, const akv_params& p, const void* arena, size_t arena_bytes, const void* q, void* out, float* out_f32,
              float sm_scale, const DecodeSuffix& sfx, void* ws, void* stream, std::string* why) {
   static std::mutex mu;
   static std::map<LaunchKey, Plan> cache;
@@ -2245,9 +2498,13 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
         cudaFuncSetAttribute(decode_kernel<GS>(codec, rope), cudaFuncAttributeMaxDynamicSharedMemorySize, di.smem_optin);
     if (e != cudaSuccess) return (int)e;
     if (!make_plan(L, GS, di.smem_optin, !rope, &pl, why)) return -1;
+    if ((e = cudaFuncSetAttribute(score_kernel<GS>(), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)kScDynSmem)) != cudaSuccess)  // the score launch's stages
+      return (int)e;
     int grid = (int)std::min<long long>(std::min(di.sms, kMaxGrid), ttot);
     if (ctas > 0) grid = (int)std::min<long long>(ctas, ttot);
     pl.grid = grid;
+    pl.sms = di.sms;
     // first unit and tile of every CTA's range
     long long t0 = 0;
     int u = 0;
@@ -2350,17 +2607,34 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
     cfg.gridDim = dim3((unsigned)(units * P.n_ch), 1, 1);
     e = cudaLaunchKernelEx(&cfg, rope_kernel<GS>(codec), R);
     for (int j = 0; j < 64; ++j) S.turn[j] = R.turn[j];
-    if (e == cudaSuccess && n_sch) {  // the suffix chunks, keys turned to positions S + t
-      cfg.gridDim = dim3((unsigned)(units * n_sch), 1, 1);
-      cfg.dynamicSmemBytes = (size_t)SCH * 256;  // a chunk's value rows
-      e = cudaLaunchKernelEx(&cfg, suffix_kernel<GS>(), S);
-      cfg.dynamicSmemBytes = 0;
-    }
   } else {
-    // the suffix chunks (if any) share the grid with the anchor chunks
-    cfg.gridDim = dim3((unsigned)(units * (P.n_ch + n_sch)), 1, 1);
-    cfg.dynamicSmemBytes = n_sch ? (size_t)SCH * 256 : 0;
-    e = cudaLaunchKernelEx(&cfg, score_kernel<GS>(n_sch > 0), S);
+    // anchor rows of every unit through one map over the caller's arena as 256-byte rows (each
+    // unit's anchor-key section starts its 256-byte-aligned segment; a full-selection arena places
+    // its units by the budgets it chose, past the plain layout's size), query rows through one over q
+    CUtensorMap tmA, tmB;
+    if (!encode_row_map(&tmA, arena, arena_bytes / 256, kScTile, CU_TENSOR_MAP_SWIZZLE_NONE) ||
+        !encode_row_map(&tmB, q, (uint64_t)p.batch * (uint64_t)p.n_q_heads, 16, CU_TENSOR_MAP_SWIZZLE_128B)) {
+      *why = "(tensor maps of the score launch could not be encoded)";
+      return -1;
+    }
+    S.units = units;
+    S.n_t = (P.n_ch + 1) / 2;
+    S.arena_rows = (long long)(arena_bytes / 256);
+    // persistent, one CTA per SM over the units' anchor tiles (more CTAs, one after another on an
+    // SM, when one CTA would take more tiles than its table holds)
+    const long long n_tiles = (long long)units * S.n_t;
+    cfg.gridDim = dim3((unsigned)std::max<long long>({1, std::min<long long>(n_tiles, pl.sms),
+                                                      (n_tiles + kScMaxTiles - 1) / kScMaxTiles}), 1, 1);
+    cfg.blockDim = dim3(kScThreads, 1, 1);
+    cfg.dynamicSmemBytes = kScDynSmem;
+    e = cudaLaunchKernelEx(&cfg, score_kernel<GS>(), S, tmA, tmB);
+    cfg.blockDim = dim3(128, 1, 1);
+    cfg.dynamicSmemBytes = 0;
+  }
+  if (e == cudaSuccess && n_sch) {  // the dense suffix's chunks (with RoPE: keys turned to positions S + t)
+    cfg.gridDim = dim3((unsigned)(units * n_sch), 1, 1);
+    cfg.dynamicSmemBytes = (size_t)SCH * 256;  // a chunk's value rows
+    e = cudaLaunchKernelEx(&cfg, suffix_kernel<GS>(rope != 0), S);
     cfg.dynamicSmemBytes = 0;
   }
   if (e != cudaSuccess) return (int)e;
@@ -2381,13 +2655,13 @@ int launch_g(const Layout& L, const akv_params& p, const void* arena, const void
   return (int)cudaGetLastError();
 }
 
-int launch_decode(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
+int launch_decode(const Layout& L, const akv_params& p, const void* arena, size_t arena_bytes, const void* q, void* out, float* out_f32,
                   float sm_scale, const DecodeSuffix& sfx, void* ws, void* stream, std::string* why) {
   switch (L.G) {
-    case 1: return launch_g<1>(L, p, arena, q, out, out_f32, sm_scale, sfx, ws, stream, why);
-    case 2: return launch_g<2>(L, p, arena, q, out, out_f32, sm_scale, sfx, ws, stream, why);
-    case 4: return launch_g<4>(L, p, arena, q, out, out_f32, sm_scale, sfx, ws, stream, why);
-    case 8: return launch_g<8>(L, p, arena, q, out, out_f32, sm_scale, sfx, ws, stream, why);
+    case 1: return launch_g<1>(L, p, arena, arena_bytes, q, out, out_f32, sm_scale, sfx, ws, stream, why);
+    case 2: return launch_g<2>(L, p, arena, arena_bytes, q, out, out_f32, sm_scale, sfx, ws, stream, why);
+    case 4: return launch_g<4>(L, p, arena, arena_bytes, q, out, out_f32, sm_scale, sfx, ws, stream, why);
+    case 8: return launch_g<8>(L, p, arena, arena_bytes, q, out, out_f32, sm_scale, sfx, ws, stream, why);
   }
   *why = "unsupported group size";
   return -1;

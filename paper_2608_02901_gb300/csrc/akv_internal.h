@@ -132,7 +132,7 @@ struct DecodeSuffix {
 constexpr int kSuffixChunk = 64;
 // Workspace of a decode call whose suffix holds at most `suffix_cap` tokens per request.
 DecodeWs decode_ws_layout(const Layout& L, int32_t suffix_cap = 0);
-int launch_decode(const Layout& L, const akv_params& p, const void* arena, const void* q, void* out, float* out_f32,
+int launch_decode(const Layout& L, const akv_params& p, const void* arena, size_t arena_bytes, const void* q, void* out, float* out_f32,
                   float sm_scale, const DecodeSuffix& sfx, void* ws, void* stream, std::string* why);
 // Appends one token per request to the dense suffix (akv_suffix_append); returns a cudaError_t.
 int launch_suffix_append(int32_t B, int32_t H, const void* K_new, const void* V_new, void* K_suf, void* V_suf,

@@ -86,6 +86,9 @@ def test_suffix_logits_far_above_the_anchor_reference(dev):
 
 
 def test_suffix_lengths_above_capacity_are_taken_as_capacity(dev):
+    """Lengths past the capacity read as the capacity.  The decode launch's shared-memory float
+    reductions make its fp32 output depend on the order warps arrive in, at the last bit: the two
+    calls agree to 1e-6 (a length taken past 70 rows would move the output by far more)."""
     p = akv.Params(batch=2, n_kv_heads=1, n_q_heads=4, seed=13)
     lens = [2000, 900]
     units = seeded_units(p, lens, seed=5)
@@ -102,7 +105,7 @@ def test_suffix_lengths_above_capacity_are_taken_as_capacity(dev):
         akv.akv_decode_attn(p, lens, arena, qt, o16, out,
                             suffix=akv.Suffix(kt, vt, torch.tensor(ln, dtype=torch.int32, device=dev)))
         outs.append(out.cpu().numpy())
-    assert np.array_equal(outs[0], outs[1])
+    assert np.allclose(outs[0], outs[1], rtol=1e-6, atol=1e-7)
 
 
 def test_suffix_append_writes_rows_and_counts_them(dev):
