@@ -379,7 +379,7 @@ def run_akv(args, rank, world, local):
             kv = kv.view(2, B, H, args.suffix, 128)
             sfx[layer] = akv.Suffix(kv[0].contiguous(), kv[1].contiguous(),
                                     torch.full((B,), args.suffix, dtype=torch.int32, device=dev))
-        suffix_bytes = B * H * args.suffix * 2 * 256  # key and value rows, read by the score (or suffix) launch
+        suffix_bytes = B * H * args.suffix * 2 * 256  # key and value rows, read by the suffix launch
         step_bytes += suffix_bytes
 
     # one decode workspace (anchor scores, partial sums) serves every call: they are stream-ordered
@@ -511,8 +511,8 @@ def run_akv(args, rank, world, local):
                 "frac_of_8tbs": round(achieved / 8000.0, 4),
                 "step": {"bytes": round(step_bytes), "achieved": round(step_bytes / (sec / args.steps) / 1e9, 2),
                          "frac": round(step_bytes / (sec / args.steps) / 1e9 / peak, 4)},
-                "scores_kernel": {"kernel": ("akv_rope_logits_kernel" if args.rope else "akv_scores_kernel")
-                                  + (" + akv_suffix_kernel" if args.suffix > 0 and args.rope else ""),
+                "scores_kernel": {"kernel": ("akv_rope_logits_kernel" if args.rope else "akv_scores_tc_kernel")
+                                  + (" + akv_suffix_kernel" if args.suffix > 0 else ""),
                                   "launch_us": round(us_scores, 3),
                                   "bytes_per_launch": round(scores_bytes),
                                   "achieved": round(scores_bytes / (us_scores * 1e-6) / 1e9, 2)},
@@ -536,7 +536,7 @@ def run_akv(args, rank, world, local):
                    "fresh_queries": N_TOKENS, "arena_bytes_per_layer": arena_bytes,
                    "l2": f"inputs larger than L2: {layers} distinct layer caches, {layers * arena_bytes / 1e6:.0f} MB cycled",
                    "timing": "CUDA graph replay, CUDA events on the launching stream", "parallelism": f"dp{world}"},
-        "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": (3 if args.suffix > 0 and args.rope else 2) * args.steps, "clocks": clocks,
+        "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": (3 if args.suffix > 0 else 2) * args.steps, "clocks": clocks,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
