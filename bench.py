@@ -292,21 +292,37 @@ def kernel_traffic(workload: str):
 
 
 def build_layers(torch, akv, gen, p, lens, layers, source, dev, rank=0):
-    """Device arenas of `layers` distinct layer caches and the bytes one decode reads."""
+    """Device arenas of `layers` distinct layer caches, the bytes one decode reads, and (GPU-encoded
+    layers) the device time of the plain encoder per layer: CUDA events around each akv_encode call
+    after one untimed encode, the layer's K/V already on the device."""
     arena_bytes, ws_bytes = akv.akv_cache_size(p, lens)
     shapes = akv.akv_unit_shapes(p, lens)
     arenas = []
+    encode = None
     if source == "encoded":
         ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
         S = lens[0]
+        times = []
         for layer in range(layers):
             K, V = gen.clustered_batch_torch(p.batch, p.n_kv_heads, S, seed=rank_seed(1000 + layer, rank), device=dev)
             arena = torch.empty(arena_bytes, dtype=torch.uint8, device=dev)
+            if layer == 0:
+                akv.akv_encode(p, lens, K, V, arena, ws)  # untimed: first-call set-up
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
             akv.akv_encode(p, lens, K, V, arena, ws)
+            e1.record()
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1) * 1e3)
             arenas.append(arena)
             del K, V
         torch.cuda.synchronize()
         del ws
+        us = sum(times) / len(times)
+        tokens = p.batch * p.n_kv_heads * S
+        encode = {"kernel_set": "akv_encode (plain encoder)", "us_per_layer": round(us, 2), "tokens": tokens,
+                  "tokens_per_s": round(tokens / (us * 1e-6), 1),
+                  "input_GB_per_s": round(tokens * 512 / (us * 1e-6) / 1e9, 1), "layers_timed": len(times)}
     else:
         base = None
         for layer in range(layers):
@@ -322,7 +338,7 @@ def build_layers(torch, akv, gen, p, lens, layers, source, dev, rank=0):
             arenas.append(arena)
     # mean over the cycled layers of the exact bytes each decode reads
     step_bytes = sum(arena_read_bytes(torch, akv, p, lens, a) for a in arenas) / len(arenas)
-    return arenas, arena_bytes, step_bytes
+    return arenas, arena_bytes, step_bytes, encode
 
 
 def time_launches(torch, akv, step, n, stream, batch=32):
@@ -364,7 +380,7 @@ def run_akv(args, rank, world, local):
     p = workload_params(akv, args.workload, batch=B, n_kv_heads=H, n_q_heads=Hq, seed=rank_seed(11, rank),
                         rot_seed=0x5EED, lloyd=args.codec == "lloyd", rope=args.rope)
     layers = args.layers
-    arenas, arena_bytes, step_bytes = build_layers(torch, akv, gen, p, lens, layers, source, dev, rank)
+    arenas, arena_bytes, step_bytes, encode = build_layers(torch, akv, gen, p, lens, layers, source, dev, rank)
     n_tok = N_TOKENS
     qs = gen.queries_torch(n_tok * layers * B * Hq, seed=77 + rank, device=dev).view(n_tok, layers, B, Hq, 128)
     out = torch.empty((n_tok, layers, B, Hq, 128), dtype=torch.bfloat16, device=dev)
@@ -522,7 +538,7 @@ def run_akv(args, rank, world, local):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(torch, akv, p, lens, arenas[0])
+        cpu = cpu_baseline(torch, akv, p, lens, arenas[0], encoded=source == "encoded")
 
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": "GB/s", "us_per_step": round(us_step, 4),
@@ -538,6 +554,8 @@ def run_akv(args, rank, world, local):
                    "timing": "CUDA graph replay, CUDA events on the launching stream", "parallelism": f"dp{world}"},
         "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": (3 if args.suffix > 0 else 2) * args.steps, "clocks": clocks,
     }
+    if encode is not None:  # context: the compression pass of the layers this run decodes
+        line["encode"] = encode
     if rank == 0:
         print(json.dumps(line), flush=True)
 
@@ -547,10 +565,11 @@ def _oracle_units_from_arena(torch, arena):
     return oracle.unpack_arena(arena.cpu().numpy())
 
 
-def cpu_baseline(torch, akv, p, lens, arena, budget_s=16.0):
+def cpu_baseline(torch, akv, p, lens, arena, budget_s=16.0, encoded=False):
     """The fp64 oracle, as it stands, on the host cores, over the same layer cache the GPU reads:
     whole layer steps with OpenMP over the units (threads = min(cores, units)), then single units
-    on one core.  Bytes are the exact bytes of the units attended (the tile tables' sizes)."""
+    on one core.  Bytes are the exact bytes of the units attended (the tile tables' sizes).  For a
+    GPU-encoded workload also the oracle's encode of one unit of the same shape on one core."""
     import gen
     import oracle
     units = _oracle_units_from_arena(torch, arena)
@@ -577,12 +596,25 @@ def cpu_baseline(torch, akv, p, lens, arena, budget_s=16.0):
         if time.perf_counter() - t1 > budget_s / 2:
             break
     sec1 = time.perf_counter() - t1
-    return {"value": round(sum(ub) * done / sec / 1e9, 5), "unit": "GB/s", "cores": threads, "nproc": nproc,
+    enc = None
+    if encoded:  # the compression pass: one unit of the workload's shape, clustered K/V, one core
+        S = int(lens[0])
+        K, V = gen.clustered_batch(1, 1, [S], seed=1000)
+        t2 = time.perf_counter()
+        oracle.encode(K, V, [S], 1, p.anchor_frac, p.res_frac_k, p.res_frac_v, p.window, p.seed, p.rot_seed,
+                      rotate=p.rotate, lloyd=p.lloyd)
+        sec2 = time.perf_counter() - t2
+        enc = {"kind": "oracle encode", "cores": 1, "tokens": S, "seconds": round(sec2, 3),
+               "tokens_per_s": round(S / sec2, 1), "sample": f"one unit of {S} tokens"}
+    out = {"value": round(sum(ub) * done / sec / 1e9, 5), "unit": "GB/s", "cores": threads, "nproc": nproc,
             "kind": "oracle",
             "sample": f"{done} full layer steps of the workload's first layer cache ({n} units, OpenMP over units)",
             "seconds": round(sec, 2), "us_per_step": round(sec * 1e6 / done, 1),
             "single_core": {"value": round(b1 / sec1 / 1e9, 5), "unit": "GB/s", "cores": 1,
                             "sample": f"{one} single units of the same layer, one at a time", "seconds": round(sec1, 2)}}
+    if enc is not None:
+        out["encode"] = enc
+    return out
 
 
 def run_reference(args, rank, world, local):
