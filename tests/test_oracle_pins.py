@@ -541,6 +541,30 @@ def test_rope_attend_matches_dense_bruteforce(tiny, base):
     u.pos = np.arange(u.S, dtype=np.int32)
 
 
+@pytest.mark.parametrize("base", [10000.0, 500000.0])
+def test_rope_with_suffix_matches_dense_bruteforce(tiny, base):
+    """RoPE at decode with a dense suffix (Section 3.2; Appendix E.2): the compressed keys turned to
+    their stored positions and suffix token t turned to position S + t, after the request's S
+    compressed tokens, all in one softmax: equal to a dense softmax over the complex-rotated rows."""
+    _, _, u = tiny
+    n_suf = 37
+    ks, vs = _suffix_rows(n_suf, 930)
+    q = gen.queries(2, 83)
+    pos = np.random.default_rng(5).permutation(u.S).astype(np.int32)
+    u.pos = pos
+    try:
+        out = oracle.attend_suffix([u], q, 2, 1, 1.0, PAR["rot_seed"], ks[None], vs[None], [n_suf],
+                                   rope_theta=base)[0]
+    finally:
+        u.pos = np.arange(u.S, dtype=np.int32)
+    Kr = np.concatenate([_rope_complex(oracle.reconstruct(u, "k", PAR["rot_seed"]), pos, base),
+                         _rope_complex(gen.bf16_to_f64(ks), u.S + np.arange(n_suf), base)])
+    Vh = np.concatenate([oracle.reconstruct(u, "v", PAR["rot_seed"]), gen.bf16_to_f64(vs)])
+    for g in range(2):
+        y, _ = _softmax_attend(Kr, Vh, gen.bf16_to_f64(q[g]), 1.0)
+        assert np.allclose(out[g], y, rtol=0, atol=1e-10)
+
+
 def test_rope_at_position_zero_is_plain_attention(tiny):
     _, _, u = tiny
     q = gen.queries(4, 82)
